@@ -1,0 +1,261 @@
+/*
+ * CPU oracle for the LUT-network hot path of BitLogic (arXiv 2602.07400).
+ *
+ * TEST INFRASTRUCTURE ONLY.  Only the test-suite, the smoke check of the
+ * entry module and the CPU-baseline leg of the benchmark may load this
+ * library.  The product path (the CUDA library under the package) shares no
+ * code with it and never calls it.
+ *
+ * Every function is the plain definition written out as nested loops, in
+ * double precision, with no blocking, fusion or reordering.  The loops over
+ * independent outputs carry OpenMP pragmas; each output is still computed by
+ * exactly one thread, in the order written, so the result does not depend on
+ * the thread count.
+ *
+ * Layouts (shared with the CUDA path by convention only):
+ *   raw inputs       x[s*d + j]            uint8, sample-major
+ *   soft activations X[row*B + s]          feature-major, batch contiguous
+ *   connectivity     conn[j*k + i]         slot i of node j
+ *   table logits     theta[j*2^k + a]      fp32 (the model's parameters)
+ *   hard tables      table[j] bit a        entry a of node j
+ *   packed bits      xp[row*W + s/32] bit (s%32), W = ceil(N/32)
+ *
+ * Index convention (the paper leaves the LUT input bit order open, App. C.1
+ * "Bit-packed inference"): connectivity slot i is bit i of the table index a.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+int oracle_max_threads(void) {
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}
+
+void oracle_set_threads(int n) {
+#ifdef _OPENMP
+    if (n > 0) omp_set_num_threads(n);
+#else
+    (void)n;
+#endif
+}
+
+/* Linear thermometer thresholds: b equispaced levels at i/(b+1) of the value
+ * range (§3 "Encoders and heads"; App. A "Scope of the prior-method
+ * reproduction" places them at i/(b+1)).  On uint8 pixels the real threshold
+ * is 256*i/(b+1); a strict comparison p > 256*i/(b+1) equals p > floor(...).
+ * parity unpinned: the paper states no integer thresholds; the tests pin the
+ * three workload sets to this reading. */
+void oracle_linear_thresholds(int32_t b, int32_t* thr) {
+    for (int32_t i = 1; i <= b; ++i) thr[i - 1] = (int32_t)((256 * i) / (b + 1));
+}
+
+/* Thermometer encoder E: R^d -> {0,1}^{db} (§3 "Encoders and heads"):
+ * wire j*b + i is 1 when feature j exceeds threshold i (strict, as in the
+ * "(pixel > 0)" comparison of App. B "MNIST-specific encoder collapse"). */
+void oracle_encode_thermometer(const uint8_t* x, int64_t B, int32_t d,
+                               const uint8_t* thr, int32_t b, double* bits) {
+    for (int32_t j = 0; j < d; ++j)
+        for (int32_t i = 0; i < b; ++i)
+            for (int64_t s = 0; s < B; ++s)
+                bits[((int64_t)j * b + i) * B + s] = (x[s * d + j] > thr[i]) ? 1.0 : 0.0;
+}
+
+static double sigmoid(double z) { return 1.0 / (1.0 + exp(-z)); }
+
+/* Corner weight of table entry a for node inputs xs[0..k-1]:
+ * w_a = prod_i x_i^{a_i} (1 - x_i)^{1 - a_i} (the Kronecker-indicator basis of
+ * LightLUT, §2 "Gradient-based LUT methods"; 2^k parameters per node). */
+static double corner_weight(const double* xs, int32_t k, int64_t a) {
+    double wa = 1.0;
+    for (int32_t i = 0; i < k; ++i) wa *= ((a >> i) & 1) ? xs[i] : (1.0 - xs[i]);
+    return wa;
+}
+
+/* Soft LUT layer forward (one logic layer L_M(f_theta^(n)) of Eq. (1), §3):
+ * y_j(s) = sum_a sigmoid(theta_j[a]) * w_a(x_{M_j(0)}(s), ..., x_{M_j(k-1)}(s)). */
+void oracle_lut_forward(const double* X, int32_t w_in, int64_t B,
+                        const int32_t* conn, const float* theta, int32_t w, int32_t k,
+                        double* Y) {
+    const int64_t K = (int64_t)1 << k;
+    (void)w_in;
+#pragma omp parallel for schedule(dynamic, 16)
+    for (int32_t j = 0; j < w; ++j) {
+        double xs[8], t[64];
+        for (int64_t a = 0; a < K; ++a) t[a] = sigmoid((double)theta[(int64_t)j * K + a]);
+        for (int64_t s = 0; s < B; ++s) {
+            for (int32_t i = 0; i < k; ++i) xs[i] = X[(int64_t)conn[(int64_t)j * k + i] * B + s];
+            double y = 0.0;
+            for (int64_t a = 0; a < K; ++a) y += t[a] * corner_weight(xs, k, a);
+            Y[(int64_t)j * B + s] = y;
+        }
+    }
+}
+
+/* Group-sum head with temperature and cross-entropy (§3 "Encoders and
+ * heads": popcount GroupSum; §4 "Training": cross-entropy on the raw head
+ * logits, mean over the batch).  Class c owns the contiguous nodes
+ * [c*g, (c+1)*g), g = w/C, and logit[s][c] = (sum of its outputs)/tau.
+ * Gradients: dlogit = (softmax - onehot)/B, dY[j][s] = dlogit[s][c(j)]/tau.
+ * logits and dY may be NULL. */
+void oracle_head_loss(const double* Y, int32_t w, int64_t B, int32_t C, double tau,
+                      const int32_t* labels, double* logits, double* loss, double* dY) {
+    const int32_t g = w / C;
+    double* lg = (double*)malloc(sizeof(double) * (size_t)B * C);
+    double* per = (double*)malloc(sizeof(double) * (size_t)B);
+#pragma omp parallel for schedule(static)
+    for (int64_t s = 0; s < B; ++s) {
+        for (int32_t c = 0; c < C; ++c) {
+            double sum = 0.0;
+            for (int32_t j = c * g; j < (c + 1) * g; ++j) sum += Y[(int64_t)j * B + s];
+            lg[s * C + c] = sum / tau;
+        }
+        double m = lg[s * C];
+        for (int32_t c = 1; c < C; ++c) if (lg[s * C + c] > m) m = lg[s * C + c];
+        double z = 0.0;
+        for (int32_t c = 0; c < C; ++c) z += exp(lg[s * C + c] - m);
+        const double lse = m + log(z);
+        per[s] = lse - lg[s * C + labels[s]];
+        if (dY) {
+            for (int32_t c = 0; c < C; ++c) {
+                const double p = exp(lg[s * C + c] - lse);
+                const double dl = (p - (c == labels[s] ? 1.0 : 0.0)) / (double)B;
+                for (int32_t j = c * g; j < (c + 1) * g; ++j) dY[(int64_t)j * B + s] = dl / tau;
+            }
+        }
+    }
+    double tot = 0.0;
+    for (int64_t s = 0; s < B; ++s) tot += per[s];
+    if (loss) *loss = tot / (double)B;
+    if (logits) memcpy(logits, lg, sizeof(double) * (size_t)B * C);
+    free(lg);
+    free(per);
+}
+
+/* Soft LUT layer backward, by the chain rule on the forward definition:
+ *   dtheta_j[a] = t_a (1 - t_a) * sum_s dY[j][s] * w_a(x(s))
+ *   dy_j/dx_i   = sum_a t_a * (a_i ? +1 : -1) * prod_{m != i} (a_m ? x_m : 1 - x_m)
+ *   dX[M_j(i)][s] += dY[j][s] * dy_j/dx_i        (scatter-add in node order)
+ * dX (optional) is overwritten.  For each element of dX the additions happen
+ * in increasing (j, i) order. */
+void oracle_lut_backward(const double* X, int32_t w_in, int64_t B,
+                         const int32_t* conn, const float* theta, int32_t w, int32_t k,
+                         const double* dY, double* dtheta, double* dX) {
+    const int64_t K = (int64_t)1 << k;
+#pragma omp parallel for schedule(dynamic, 16)
+    for (int32_t j = 0; j < w; ++j) {
+        double xs[8];
+        for (int64_t a = 0; a < K; ++a) {
+            const double t = sigmoid((double)theta[(int64_t)j * K + a]);
+            double acc = 0.0;
+            for (int64_t s = 0; s < B; ++s) {
+                for (int32_t i = 0; i < k; ++i) xs[i] = X[(int64_t)conn[(int64_t)j * k + i] * B + s];
+                acc += dY[(int64_t)j * B + s] * corner_weight(xs, k, a);
+            }
+            dtheta[(int64_t)j * K + a] = t * (1.0 - t) * acc;
+        }
+    }
+    if (!dX) return;
+    memset(dX, 0, sizeof(double) * (size_t)w_in * (size_t)B);
+    double* tt = (double*)malloc(sizeof(double) * (size_t)w * (size_t)K);
+    for (int64_t q = 0; q < (int64_t)w * K; ++q) tt[q] = sigmoid((double)theta[q]);
+    /* samples are independent: one thread owns each sample column and walks
+     * the nodes in order, so the per-element addition order is (j, i) */
+#pragma omp parallel for schedule(static)
+    for (int64_t s = 0; s < B; ++s) {
+        double xs[8];
+        for (int32_t j = 0; j < w; ++j) {
+            for (int32_t i = 0; i < k; ++i) xs[i] = X[(int64_t)conn[(int64_t)j * k + i] * B + s];
+            const double g = dY[(int64_t)j * B + s];
+            for (int32_t i = 0; i < k; ++i) {
+                double der = 0.0;
+                for (int64_t a = 0; a < K; ++a) {
+                    double p = ((a >> i) & 1) ? 1.0 : -1.0;
+                    for (int32_t m = 0; m < k; ++m)
+                        if (m != i) p *= ((a >> m) & 1) ? xs[m] : (1.0 - xs[m]);
+                    der += tt[(int64_t)j * K + a] * p;
+                }
+                dX[(int64_t)conn[(int64_t)j * k + i] * B + s] += g * der;
+            }
+        }
+    }
+    free(tt);
+}
+
+/* Table discretization (§3 "Nodes are parameterizations": every surrogate
+ * discretizes to a 2^n-entry truth table; App. C.1 extracts it once per
+ * layer): entry a is 1 exactly when theta_j[a] > 0, i.e. sigmoid > 1/2. */
+void oracle_binarize_tables(const float* theta, int32_t w, int32_t k, uint64_t* table) {
+    const int64_t K = (int64_t)1 << k;
+    for (int32_t j = 0; j < w; ++j) {
+        uint64_t t = 0;
+        for (int64_t a = 0; a < K; ++a)
+            if (theta[(int64_t)j * K + a] > 0.0f) t |= (uint64_t)1 << a;
+        table[j] = t;
+    }
+}
+
+/* Thermometer encoding followed by packing 32 samples per uint32 along the
+ * batch (App. C.1 "Bit-packed inference" packs 64 per 64-bit word; this
+ * layout uses 32 per 32-bit word): sample s is bit s%32 of word s/32. */
+void oracle_pack_bits(const uint8_t* x, int64_t N, int32_t d,
+                      const uint8_t* thr, int32_t b, uint32_t* xp) {
+    const int64_t W = (N + 31) / 32;
+    memset(xp, 0, sizeof(uint32_t) * (size_t)d * (size_t)b * (size_t)W);
+    for (int64_t s = 0; s < N; ++s)
+        for (int32_t j = 0; j < d; ++j)
+            for (int32_t i = 0; i < b; ++i)
+                if (x[s * d + j] > thr[i])
+                    xp[((int64_t)j * b + i) * W + s / 32] |= (uint32_t)1 << (s % 32);
+}
+
+/* Hard LUT layer on packed bits (App. C.1): for each sample, the node's
+ * index a = sum_i bit(input M_j(i), s) << i selects table bit a.  Written
+ * per sample as a plain lookup on unpacked bits. */
+void oracle_hard_forward(const uint32_t* xp, int32_t w_in, int64_t N,
+                         const int32_t* conn, const uint64_t* table, int32_t w, int32_t k,
+                         uint32_t* yp) {
+    const int64_t W = (N + 31) / 32;
+    (void)w_in;
+    memset(yp, 0, sizeof(uint32_t) * (size_t)w * (size_t)W);
+#pragma omp parallel for schedule(static)
+    for (int32_t j = 0; j < w; ++j) {
+        for (int64_t s = 0; s < N; ++s) {
+            uint64_t a = 0;
+            for (int32_t i = 0; i < k; ++i) {
+                const uint32_t word = xp[(int64_t)conn[(int64_t)j * k + i] * W + s / 32];
+                a |= (uint64_t)((word >> (s % 32)) & 1u) << i;
+            }
+            if ((table[j] >> a) & 1u) yp[(int64_t)j * W + s / 32] |= (uint32_t)1 << (s % 32);
+        }
+    }
+}
+
+/* Popcount GroupSum head in hard mode (§3 "Encoders and heads"): the score
+ * of class c is the number of ones among its contiguous group of g = w/C
+ * nodes; the prediction is the first class with the largest score. */
+void oracle_popcount_head(const uint32_t* yp, int32_t w, int64_t N, int32_t C,
+                          int32_t* counts, int32_t* pred) {
+    const int64_t W = (N + 31) / 32;
+    const int32_t g = w / C;
+#pragma omp parallel for schedule(static)
+    for (int64_t s = 0; s < N; ++s) {
+        int32_t best = 0, bestc = 0;
+        for (int32_t c = 0; c < C; ++c) {
+            int32_t cnt = 0;
+            for (int32_t j = c * g; j < (c + 1) * g; ++j)
+                cnt += (int32_t)((yp[(int64_t)j * W + s / 32] >> (s % 32)) & 1u);
+            if (counts) counts[s * C + c] = cnt;
+            if (c == 0 || cnt > best) { best = cnt; bestc = c; }
+        }
+        if (pred) pred[s] = bestc;
+    }
+}
