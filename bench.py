@@ -1,0 +1,500 @@
+#!/usr/bin/env python3
+"""Throughput of the LUT-network hot path on GB300 (one JSON line on rank 0).
+
+A step is one pass of the whole hot path over one batch of synthetic input:
+the soft training step (thermometer encode, two LUT forwards, group-sum head
+with cross-entropy, two LUT backwards with the CSR input-gradient
+reduction) followed by the hard evaluation of the same batch (table
+binarization, encode + pack, hard layer 1, hard layer 2 with the fused
+popcount head and argmax).  ``value`` is the training throughput (samples
+per second through the fwd+bwd part); the hard part is reported in the
+``hard`` object.  L2 is flushed between steps (a 512 MB write outside the
+timed events), so every step starts cold.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload mnist]
+  python bench.py --impl reference ...   # the CPU oracle on the same workload
+
+Multi-GPU (torchrun, one process per GPU): every rank trains its own batch
+(weak scaling, no data-path collective); the job's time is the max over
+ranks and ``value`` sums the samples of all ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2602_07400_gb300 import synth  # noqa: E402
+
+METRIC = "LUT train samples/s (fwd+bwd) and hard bit-packed MSamples/s; % of roofline"
+FP32_LANES_PER_SM = 128
+SMI_FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=400)
+    p.add_argument("--warmup", type=int, default=20)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--workload", default="mnist", choices=sorted(synth.WORKLOADS))
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--profile", action="store_true",
+                   help="plain timed loop only (for ncu launch lists)")
+    return p.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            m = json.load(f)
+        return float(m["hbm_gbs"]), float(m.get("sm_max_mhz", 2070.0)), "measured"
+    return 6800.0, 2070.0, "fallback"
+
+
+# ------------------------------------------------------------- clocks --
+
+class ClockSampler:
+    def __init__(self, index: int, period_ms: int = 100):
+        self.index, self.period = index, period_ms
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.out = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={SMI_FIELDS}",
+                 "--format=csv,noheader,nounits", f"-lms", str(self.period)],
+                stdout=self.out, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        self.t0 = time.time()
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0,
+                    "note": "nvidia-smi unavailable"}
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.out.close()
+        sm, mx, pw, reasons = [], [], [], set()
+        names = ["active", "hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    mx.append(float(parts[2]))
+                    pw.append(float(parts[3]))
+                except ValueError:
+                    continue
+                for name, val in zip(names[1:], parts[5:9]):
+                    if val.lower().startswith("active"):
+                        reasons.add(name)
+        os.unlink(self.path)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None,
+                "power_w_max": max(pw) if pw else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------ work per call --
+
+def call_work(wl, B):
+    """Algorithmic work of each library call of one step on a batch of B:
+    (bytes, fp32 or logic ops).  Ops follow the lerp-tree counts: forward
+    2(2^k-1)+k per (node, sample); backward with input gradient
+    4(2^k-1)+2^k; backward without it 2(2^k-1)+2^k; hard layer 2^k-1 LOP3
+    per (node, 32-sample word)."""
+    K, k = wl.K, wl.k
+    w1, w2 = wl.widths
+    win, d, b, C = wl.w_in, wl.d, wl.b, wl.classes
+    W = (B + 31) // 32
+    f = 4
+    return {
+        "encode": (B * d + f * win * B, 0),
+        "forward1": (f * (win * B + w1 * B + w1 * K + w1 * k), (2 * (K - 1) + k) * w1 * B),
+        "forward2": (f * (w1 * B + w2 * B + w2 * K + w2 * k), (2 * (K - 1) + k) * w2 * B),
+        "head": (f * (2 * w2 * B + 3 * B * C), 0),
+        "backward2": (f * (w1 * B + w2 * B + w2 * k * B + 2 * w2 * K + w2 * k), (4 * (K - 1) + K) * w2 * B),
+        "csr2": (f * (w2 * k * B + w1 * B + w1 + w2 * k), 0),
+        "backward1": (f * (win * B + w1 * B + 2 * w1 * K + w1 * k), (2 * (K - 1) + K) * w1 * B),
+        "binarize": (f * (w1 * K + w2 * K) + 8 * (w1 + w2), 0),
+        "pack": (B * d + f * win * W, 0),
+        "hard1": (f * (win * W + w1 * W + w1 * k) + 8 * w1, (K - 1) * w1 * W),
+        "hard2": (f * (w1 * W + w2 * k + B * C * 2 + B) + 8 * w2, (K - 1) * w2 * W),
+    }
+
+
+KERNEL_OF_CALL = {
+    "encode": "encode_soft_kernel", "forward1": "lut_forward_kernel", "forward2": "lut_forward_kernel",
+    "head": "head_* (4 kernels)", "backward2": "lut_backward_kernel<k, dx>",
+    "csr2": "csr_reduce_kernel", "backward1": "lut_backward_kernel<k, no dx>",
+    "binarize": "binarize_kernel (x2)", "pack": "pack_bits_kernel", "hard1": "hard_layer_kernel",
+    "hard2": "hard_head_kernel + argmax_kernel",
+}
+
+
+# --------------------------------------------------------------- ours --
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def run_ours(args):
+    import paper_2602_07400_gb300 as bl
+    from paper_2602_07400_gb300.pipeline import HardInfer, Network, TrainStep
+
+    world, rank, local = dist_env()
+    torch.cuda.set_device(local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    bl.load()
+    wl = synth.WORKLOADS[args.workload]
+    hard_only = wl.name.startswith("hard_")
+    B = wl.batch
+    conn1, th1, conn2, th2 = synth.network(wl, seed=0)
+    net = Network(conn1, th1, conn2, th2, wl.w_in)
+    x_gen, lab_gen = synth.blob_batch(B, wl.d, wl.classes, wl.sigma, seed=1000 + rank,
+                                      device="cuda" if hard_only else "cpu")
+    st = None
+    if not hard_only:
+        st = TrainStep(net, B, wl.d, wl.thresholds, wl.classes, wl.tau)
+        st.load(x_gen.cuda(), lab_gen.cuda())
+    hi = HardInfer(net, B, wl.d, wl.thresholds, wl.classes)
+    if st is not None:
+        hi.x = st.x                      # the hard pass evaluates the same batch
+    else:
+        hi.x.copy_(x_gen)
+    del x_gen
+    flush = torch.empty(512 << 20, dtype=torch.uint8, device="cuda")
+    stream = torch.cuda.current_stream()
+
+    def step(mark):
+        if st is not None:
+            st.run(mark=mark)
+            mark("train_end")
+        hi.binarize(mark=mark)
+        hi.run(mark=mark)
+
+    for _ in range(args.warmup):
+        flush.fill_(1)
+        step(lambda n: None)
+    torch.cuda.synchronize()
+
+    K = args.steps
+    marks = []          # per step: list of (name, event)
+
+    def new_step_marks():
+        lst = []
+        marks.append(lst)
+
+        def mark(name):
+            ev = torch.cuda.Event(enable_timing=True)
+            ev.record(stream)
+            lst.append((name, ev))
+        return mark
+
+    clock = ClockSampler(local)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    clock.start()
+    wall0 = time.perf_counter()
+    for _ in range(K):
+        flush.fill_(1)
+        mark = new_step_marks()
+        mark("start")
+        step(mark)
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - wall0
+    if world > 1:
+        torch.distributed.barrier()
+    clocks = clock.stop()
+    assert bl.bitlogic_device_error() == 0
+
+    # per-call durations
+    calls = {}
+    train_ms, hard_ms = [], []
+    for lst in marks:
+        prev = lst[0][1]
+        t_train = 0.0
+        t_total = 0.0
+        for name, ev in lst[1:]:
+            dt = prev.elapsed_time(ev)
+            prev = ev
+            if name == "train_end":
+                t_train = t_total
+                continue
+            calls.setdefault(name, []).append(dt)
+            t_total += dt
+        train_ms.append(t_train)
+        hard_ms.append(t_total - t_train)
+    train_sum = float(sum(train_ms))
+    hard_sum = float(sum(hard_ms))
+    tot = torch.tensor([train_sum, hard_sum], dtype=torch.float64, device="cuda")
+    if world > 1:
+        torch.distributed.all_reduce(tot, op=torch.distributed.ReduceOp.MAX)
+    train_sum, hard_sum = float(tot[0]), float(tot[1])
+
+    launches = K * (hi.kernels_per_binarize + hi.kernels_per_run)
+    if st is not None:
+        launches += K * st.kernels_per_run
+
+    result = None
+    if rank == 0:
+        hbm, sm_max, peak_kind = peaks()
+        work = call_work(wl, B)
+        per_call_ms = {n: float(np.mean(v)) for n, v in calls.items()}
+        ms_step_train = train_sum / K
+        ms_step_hard = hard_sum / K
+        # roofline of the dominant single-kernel call
+        single = {n: t for n, t in per_call_ms.items() if n not in ("head", "binarize", "hard2")}
+        dom = max(single, key=single.get)
+        byts, ops = work[dom]
+        t_s = per_call_ms[dom] * 1e-3
+        fp32_peak = 152 * FP32_LANES_PER_SM * sm_max * 1e6
+        t_hbm, t_alu = byts / (hbm * 1e9), ops / fp32_peak
+        if t_alu >= t_hbm:
+            roof = {"bound": "alu", "achieved": ops / t_s / 1e12, "peak": fp32_peak / 1e12,
+                    "unit": "Tops/s (fp32 pipe lane-ops)"}
+        else:
+            roof = {"bound": "hbm", "achieved": byts / t_s / 1e9, "peak": hbm, "unit": "GB/s"}
+        roof["frac"] = roof["achieved"] / roof["peak"]
+        roof.update({"traffic": None, "kernel": KERNEL_OF_CALL[dom], "call": dom,
+                     "ms_per_launch": per_call_ms[dom], "algorithmic_bytes": byts,
+                     "algorithmic_ops": ops, "peak_source": f"{peak_kind} (HBM), "
+                     f"152 SMs x {FP32_LANES_PER_SM} fp32 lanes x {sm_max:.0f} MHz (alu)"})
+        calls_out = {}
+        for n, t in per_call_ms.items():
+            b_, o_ = work[n]
+            calls_out[n] = {"ms": round(t, 5), "GB/s": round(b_ / (t * 1e-3) / 1e9, 1),
+                            "Tops/s": round(o_ / (t * 1e-3) / 1e12, 2) if o_ else None}
+        value = world * B * K / (train_sum * 1e-3) if st is not None else world * B * K / (hard_sum * 1e-3)
+        result = {
+            "metric": METRIC,
+            "value": value,
+            "unit": "samples/s",
+            "n_gpus": world,
+            "steps": K,
+            "warmup": args.warmup,
+            "ms_per_step": ms_step_train if st is not None else ms_step_hard,
+            "higher_is_better": True,
+            "scaling": "weak",
+            "vs_baseline": None,
+            "dtype": "f32",
+            "data": "synthetic (seeded class-conditional Gaussian blobs, MNIST/CIFAR shapes; random-init tables)",
+            "config": {"workload": wl.name, "batch_per_gpu": B, "d": wl.d, "thresholds": list(wl.thresholds),
+                       "widths": list(wl.widths), "k": wl.k, "classes": wl.classes, "tau": wl.tau,
+                       "l2": "flushed between steps (512 MB write outside the timed events)",
+                       "parallelism": f"dp{world} (independent batches, no collective)"},
+            "hard": {"value": world * B * K / (hard_sum * 1e-3) / 1e6, "unit": "MSamples/s",
+                     "ms_per_batch": ms_step_hard, "batch": B,
+                     "includes": "binarize + encode/pack + 2 hard layers + popcount head + argmax"},
+            "ms_per_step_total": ms_step_train + ms_step_hard,
+            "calls": calls_out,
+            "roofline": roof,
+            "gpu_launches": launches,
+            "clocks": clocks,
+            "wall_s_timed_loop": wall,
+        }
+    if not args.profile and not args.no_e2e:
+        e2e = run_e2e(args, st, hi, wl, B)
+        if result is not None:
+            result["e2e"] = e2e["train"] if st is not None else e2e["hard"]
+            result["hard"]["e2e"] = e2e["hard"]
+    if world > 1:
+        torch.distributed.barrier()
+        torch.distributed.destroy_process_group()
+    return result
+
+
+def run_e2e(args, st, hi, wl, B):
+    """The same metric end to end: pinned host inputs copied in, the step
+    run through the public API, the step's result copied out, every step."""
+    world, rank, _ = dist_env()
+    x_host, lab_host = synth.blob_batch(B, wl.d, wl.classes, wl.sigma, seed=2000 + rank)
+    x_host = x_host.pin_memory()
+    lab_host = lab_host.pin_memory()
+    loss_host = torch.empty(1, dtype=torch.float32).pin_memory()
+    pred_host = torch.empty(B, dtype=torch.int32).pin_memory()
+    K = max(1, args.steps)
+    out = {}
+    if st is not None:
+        for _ in range(3):
+            st.load(x_host, lab_host, non_blocking=True)
+            st.run()
+            loss_host.copy_(st.loss, non_blocking=True)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(K):
+            st.load(x_host, lab_host, non_blocking=True)
+            st.run()
+            loss_host.copy_(st.loss, non_blocking=True)
+        e1.record()
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1)
+        t = torch.tensor([ms], dtype=torch.float64, device="cuda")
+        if world > 1:
+            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        out["train"] = {"value": world * B * K / (float(t[0]) * 1e-3), "unit": "samples/s",
+                        "h2d_bytes_per_step": x_host.numel() + 4 * lab_host.numel(),
+                        "d2h_bytes_per_step": 4}
+    for _ in range(3):
+        hi.x.copy_(x_host, non_blocking=True)
+        hi.binarize()
+        hi.run()
+        pred_host.copy_(hi.pred, non_blocking=True)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(K):
+        hi.x.copy_(x_host, non_blocking=True)
+        hi.binarize()
+        hi.run()
+        pred_host.copy_(hi.pred, non_blocking=True)
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    t = torch.tensor([ms], dtype=torch.float64, device="cuda")
+    if world > 1:
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    out["hard"] = {"value": world * B * K / (float(t[0]) * 1e-3) / 1e6, "unit": "MSamples/s",
+                   "h2d_bytes_per_step": x_host.numel(), "d2h_bytes_per_step": 4 * B}
+    return out
+
+
+# -------------------------------------------------- oracle (CPU) legs --
+
+def oracle_train_rate(wl, samples: int, seed: int = 0):
+    import oracle
+    conn1, th1, conn2, th2 = synth.network(wl, seed=0)
+    x, lab = synth.blob_batch(samples, wl.d, wl.classes, wl.sigma, seed=3000 + seed)
+    t0 = time.perf_counter()
+    oracle.train_step(x.numpy(), lab.numpy(), wl.thresholds, conn1, th1, conn2, th2,
+                      wl.classes, wl.tau)
+    return samples / (time.perf_counter() - t0)
+
+
+def oracle_hard_rate(wl, samples: int, seed: int = 0):
+    import oracle
+    conn1, th1, conn2, th2 = synth.network(wl, seed=0)
+    t1, t2 = oracle.binarize_tables(th1), oracle.binarize_tables(th2)
+    x, _ = synth.blob_batch(samples, wl.d, wl.classes, wl.sigma, seed=4000 + seed)
+    t0 = time.perf_counter()
+    oracle.hard_infer(x.numpy(), wl.thresholds, conn1, t1, conn2, t2, wl.classes)
+    return samples / (time.perf_counter() - t0)
+
+
+def calibrated(rate_fn, wl, budget_s: float, lo: int, hi: int):
+    r0 = rate_fn(wl, lo)
+    n = int(min(hi, max(lo, r0 * budget_s)))
+    n = max(lo, (n // lo) * lo)
+    return rate_fn(wl, n, seed=1), n
+
+
+def cpu_baseline(wl, budget_s=12.0):
+    import oracle
+    hard_only = wl.name.startswith("hard_")
+    cores = oracle.max_threads()
+    out = {}
+    if not hard_only:
+        r, n = calibrated(oracle_train_rate, wl, budget_s, 4, wl.batch)
+        out = {"value": r, "unit": "samples/s", "cores": cores, "kind": "oracle",
+               "sample": f"train step (fwd+bwd) on {n} of the {wl.batch} samples of a batch, "
+                         f"full network, fp64, OpenMP over independent outputs"}
+    rh, nh = calibrated(oracle_hard_rate, wl, budget_s / 2, 32, 1 << 16)
+    hard = {"value": rh / 1e6, "unit": "MSamples/s", "cores": cores, "kind": "oracle",
+            "sample": f"hard pass (encode+pack, 2 layers, popcount head) on {nh} samples"}
+    return out, hard
+
+
+def run_reference(args):
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return None
+    import oracle
+    wl = synth.WORKLOADS[args.workload]
+    hard_only = wl.name.startswith("hard_")
+    fn = oracle_hard_rate if hard_only else oracle_train_rate
+    lo = 32 if hard_only else 2
+    # size one step to about 1-2 s of oracle work
+    r0 = fn(wl, lo)
+    n = max(lo, int(r0 * 1.5) // lo * lo)
+    n = min(n, wl.batch)
+    for i in range(args.warmup):
+        fn(wl, lo, seed=100 + i)
+    tot_s, tot_n = 0.0, 0
+    for i in range(args.steps):
+        r = fn(wl, n, seed=i)
+        tot_s += n / r
+        tot_n += n
+    value = tot_n / tot_s
+    unit = "samples/s"
+    if hard_only:
+        value /= 1e6
+        unit = "MSamples/s"
+    cores = oracle.max_threads()
+    return {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": unit, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot_s / max(1, args.steps),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": {"workload": wl.name, "batch_per_gpu": wl.batch},
+        "cpu_baseline": {"value": value, "unit": unit, "cores": cores, "kind": "oracle",
+                         "sample": f"{n} samples of the workload per step (the plain C oracle, "
+                                   f"{'hard pass' if hard_only else 'train fwd+bwd'})"},
+        "e2e": {"value": value, "unit": unit, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        res = run_reference(args)
+        if res is not None:
+            print(json.dumps(res), flush=True)
+        return
+    res = run_ours(args)
+    if res is None:
+        return
+    if not args.profile and not args.no_cpu_baseline:
+        wl = synth.WORKLOADS[args.workload]
+        cb, cb_hard = cpu_baseline(wl)
+        if cb:
+            res["cpu_baseline"] = cb
+        res["hard"]["cpu_baseline"] = cb_hard
+    print(json.dumps(res), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,199 @@
+/*
+ * bitlogic.h -- C ABI of the GB300 (sm_103a) LUT-network hot path.
+ *
+ * The library implements the data-parallel hot path of BitLogic's
+ * gradient-based LUT networks (arXiv 2602.07400): the thermometer encoder,
+ * the soft forward/backward of a fixed-connectivity LUT layer, the group-sum
+ * head with temperature and cross-entropy, and the hard bit-packed
+ * evaluation mode with a popcount group-sum.  Every call is a hand-written
+ * CUDA kernel sequence enqueued on the caller's stream.
+ *
+ * Conventions shared by all calls
+ *   - Pointers marked "device" are caller-owned device memory; the library
+ *     never allocates, frees or synchronizes inside a compute call.  Arrays
+ *     marked "host" are read before the call returns.
+ *   - Every compute call enqueues its kernels on `stream` and returns a
+ *     status code (bitlogic_status_t).  Arguments are validated on the host
+ *     before any launch; a rejected call launches nothing.  No kernel traps
+ *     or asserts: a connectivity or CSR index that is out of range is read as
+ *     index 0 and recorded in a device-side flag that
+ *     bitlogic_device_error() reports.
+ *   - Layouts:
+ *       raw samples      x[s*d + j]             uint8, sample-major
+ *       soft activations X[row*B + s]           fp32, feature-major
+ *       connectivity     conn[j*k + i]          int32, slot i of node j
+ *       table logits     theta[j*2^k + a]       fp32
+ *       hard tables      table[j], bit a        uint64 = entry a of node j
+ *       packed bits      xp[row*W + s/32], bit s%32, W = ceil(N/32)
+ *     Slot i of a node is bit i of its table index a.
+ *   - Vectorised (16-byte) paths are taken when B % 4 == 0 and the arrays are
+ *     16-byte aligned; otherwise a scalar path runs.  Results are identical.
+ */
+#ifndef BITLOGIC_H
+#define BITLOGIC_H
+
+#include <stddef.h>
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    BITLOGIC_OK = 0,
+    BITLOGIC_ERR_NULL = -1,       /* a required pointer is NULL */
+    BITLOGIC_ERR_SHAPE = -2,      /* size <= 0, overflow, or w % C != 0 */
+    BITLOGIC_ERR_FANIN = -3,      /* k outside 1..6, or k > w_in */
+    BITLOGIC_ERR_ALIGN = -4,      /* workspace not 16-byte aligned */
+    BITLOGIC_ERR_WORKSPACE = -5,  /* workspace smaller than the query result */
+    BITLOGIC_ERR_CUDA = -6,       /* a CUDA launch or copy failed */
+    BITLOGIC_ERR_INDEX = -7,      /* index out of range (host-side check) */
+    BITLOGIC_ERR_DEVICE = -8,     /* device-side index check tripped */
+    BITLOGIC_ERR_THRESH = -9      /* thresholds: b outside 1..32 */
+} bitlogic_status_t;
+
+/* Thermometer encoder E: R^d -> {0,1}^{db} (paper §3, "Encoders and heads";
+ * linear thermometer with b thresholds, b+1 levels on b wires).
+ *   x        device uint8 [B][d]   raw samples
+ *   thr_host host uint8 [b]        thresholds, 1 <= b <= 32
+ *   bits     device fp32 [d*b][B]  bits[(j*b+i)*B + s] = (x[s][j] > thr[i])
+ * B == 0 is a no-op. */
+int bitlogic_encode_thermometer(const uint8_t* x, int64_t B, int32_t d,
+                                const uint8_t* thr_host, int32_t b,
+                                float* bits, cudaStream_t stream);
+
+/* Soft LUT layer forward: one logic layer L_M(f_theta^(n)) of the paper's
+ * Eq. (1) (§3), with the LightLUT node of §2 (Kronecker-indicator basis,
+ * 2^k parameters per node) read as
+ *   t = sigmoid(theta_j),  y_j(s) = sum_a t_a prod_i x_i^{a_i} (1-x_i)^{1-a_i},
+ * x_i = X[conn[j][i]][s].  Evaluated as a 2^k-1 step lerp tree.
+ *   X     device fp32 [w_in][B]     layer input
+ *   conn  device int32 [w][k]       fixed connectivity (§3 "Connectivity")
+ *   theta device fp32 [w][2^k]      table logits
+ *   Y     device fp32 [w][B]        output, overwritten
+ * 1 <= k <= 6, k <= w_in.  B == 0 is a no-op. */
+int bitlogic_lut_forward(const float* X, int32_t w_in, int64_t B,
+                         const int32_t* conn, const float* theta,
+                         int32_t w, int32_t k, float* Y, cudaStream_t stream);
+
+/* Bytes of workspace bitlogic_lut_backward needs (0 when want_dx == 0). */
+size_t bitlogic_lut_backward_workspace(int32_t w_in, int64_t B, int32_t w,
+                                       int32_t k, int32_t want_dx);
+
+/* Soft LUT layer backward (chain rule through the forward above):
+ *   dtheta[j][a] = t_a (1-t_a) sum_s dY[j][s] w_a(x(s))     (reduced over the
+ *                  batch inside the kernel, deterministic order)
+ *   dX[i][s]     = sum over edges (j, slot) with conn[j][slot] == i of
+ *                  dY[j][s] * dy_j/dx_slot(s)
+ * The input gradient uses the inverse-connectivity CSR map (off, edge) from
+ * bitlogic_build_csr(): per-edge terms are written to the workspace and
+ * summed per input in increasing edge order, so no atomics are used.
+ *   X, conn, theta  as in bitlogic_lut_forward
+ *   dY     device fp32 [w][B]
+ *   csr_off  device int32 [w_in+1], csr_edge device int32 [w*k]
+ *            (edge id = j*k + slot); required only when dX != NULL
+ *   dtheta device fp32 [w][2^k]   overwritten (not accumulated)
+ *   dX     device fp32 [w_in][B] or NULL (skips the input gradient)
+ *   workspace device, 16-byte aligned, >= bitlogic_lut_backward_workspace() */
+int bitlogic_lut_backward(const float* X, int32_t w_in, int64_t B,
+                          const int32_t* conn, const float* theta,
+                          int32_t w, int32_t k, const float* dY,
+                          const int32_t* csr_off, const int32_t* csr_edge,
+                          float* dtheta, float* dX,
+                          void* workspace, size_t ws_bytes, cudaStream_t stream);
+
+/* The two phases of bitlogic_lut_backward, for callers that time them
+ * separately or consume the per-edge terms themselves.
+ * bitlogic_lut_backward_edges: dtheta as above and, when edge_terms is not
+ *   NULL, edge_terms[(j*k + i)*B + s] = dY[j][s] * dy_j/dx_i(s)
+ *   (device fp32 [w*k][B], 16-byte aligned for the vector path).
+ * bitlogic_csr_reduce: dX[i][s] = sum of edge_terms[e][s] over the CSR edges e
+ *   of input i, in increasing e (n_edges = w*k). */
+int bitlogic_lut_backward_edges(const float* X, int32_t w_in, int64_t B,
+                                const int32_t* conn, const float* theta,
+                                int32_t w, int32_t k, const float* dY,
+                                float* dtheta, float* edge_terms, cudaStream_t stream);
+int bitlogic_csr_reduce(const float* edge_terms, int64_t B, const int32_t* csr_off,
+                        const int32_t* csr_edge, int32_t w_in, int32_t n_edges,
+                        float* dX, cudaStream_t stream);
+
+/* Bytes of workspace bitlogic_head_loss needs. */
+size_t bitlogic_head_loss_workspace(int64_t B, int32_t C);
+
+/* Group-sum head with temperature and softmax cross-entropy (§3 "Encoders
+ * and heads": popcount GroupSum; §4 "Training": cross-entropy on the raw
+ * head logits).  Class c owns the contiguous nodes [c*g, (c+1)*g), g = w/C:
+ *   logits[s][c] = (sum_{j in group c} Y[j][s]) / tau
+ *   loss         = mean_s ( logsumexp(logits[s]) - logits[s][labels[s]] )
+ *   dY[j][s]     = (softmax(logits[s])[c(j)] - [c(j) == labels[s]]) / (B tau)
+ *   Y      device fp32 [w][B];  labels device int32 [B], values in [0, C)
+ *   logits device fp32 [B][C] or NULL;  loss device fp32 [1]
+ *   dY     device fp32 [w][B] or NULL
+ *   workspace device, 16-byte aligned, >= bitlogic_head_loss_workspace()
+ * Requires B >= 1, C >= 1, w % C == 0, tau > 0. */
+int bitlogic_head_loss(const float* Y, int32_t w, int64_t B, int32_t C, float tau,
+                       const int32_t* labels, float* logits, float* loss, float* dY,
+                       void* workspace, size_t ws_bytes, cudaStream_t stream);
+
+/* Table discretization (§3: every surrogate discretizes to a 2^n-entry
+ * truth table; App. C.1 extracts it once per layer): bit a of table[j] is 1
+ * exactly when theta[j][a] > 0 (sigmoid > 1/2); bits >= 2^k are 0.
+ *   theta device fp32 [w][2^k];  table device uint64 [w] */
+int bitlogic_binarize_tables(const float* theta, int32_t w, int32_t k,
+                             uint64_t* table, cudaStream_t stream);
+
+/* Encoder fused with bit packing for the hard path (App. C.1 "Bit-packed
+ * inference": samples packed along the batch into words; here 32 samples
+ * per uint32): bit s%32 of xp[(j*b+i)*W + s/32] = (x[s][j] > thr[i]).
+ *   x device uint8 [N][d];  thr_host host uint8 [b], 1 <= b <= 32
+ *   xp device uint32 [d*b][W], W = ceil(N/32); tail bits (s >= N) are 0.
+ * N == 0 is a no-op. */
+int bitlogic_pack_bits(const uint8_t* x, int64_t N, int32_t d,
+                       const uint8_t* thr_host, int32_t b,
+                       uint32_t* xp, cudaStream_t stream);
+
+/* Hard LUT layer on packed bits (App. C.1: each layer's LUT evaluation
+ * becomes a bitwise operation on packed tensors): per node j and word,
+ * the k input words select table bits by a bit-sliced Shannon mux tree, so
+ * bit s of yp[j] = bit a_s of table[j] with a_s = sum_i bit_s(xp[conn[j][i]]) << i.
+ * With C > 0 the popcount GroupSum head is fused: counts[s][c] = number of
+ * ones among the nodes of group c (contiguous, g = w/C) for sample s, and
+ * pred[s] = the first class with the largest count.
+ *   xp    device uint32 [w_in][W];  conn device int32 [w][k]
+ *   table device uint64 [w]
+ *   yp    device uint32 [w][W], or NULL when C > 0 (then not written);
+ *         tail bits (s >= N) are written as 0
+ *   C     0 (no head) or the number of classes (w % C == 0)
+ *   counts device int32 [N][C] (required when C > 0); pred device int32 [N]
+ *         or NULL
+ * N == 0 is a no-op. */
+int bitlogic_hard_forward(const uint32_t* xp, int32_t w_in, int64_t N,
+                          const int32_t* conn, const uint64_t* table,
+                          int32_t w, int32_t k, uint32_t* yp,
+                          int32_t C, int32_t* counts, int32_t* pred,
+                          cudaStream_t stream);
+
+/* Inverse connectivity (host): for each input i, the edges e = j*k + slot
+ * with conn[j][slot] == i, in increasing e.  off_host [w_in+1],
+ * edge_host [w*k].  Returns BITLOGIC_ERR_INDEX when an index is outside
+ * [0, w_in).  Not part of the per-step path: built once per connectivity. */
+int bitlogic_build_csr(const int32_t* conn_host, int32_t w, int32_t k, int32_t w_in,
+                       int32_t* off_host, int32_t* edge_host);
+
+/* Synchronizes `stream`, then reports (and clears) the device-side index
+ * flag: BITLOGIC_OK, or BITLOGIC_ERR_DEVICE when a kernel met an index out of
+ * range since the last call, or BITLOGIC_ERR_CUDA. */
+int bitlogic_device_error(cudaStream_t stream);
+
+/* Static text for a status code. */
+const char* bitlogic_status_string(int code);
+
+/* ABI version (major*100 + minor). */
+int bitlogic_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BITLOGIC_H */

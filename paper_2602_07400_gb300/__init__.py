@@ -1,0 +1,286 @@
+"""Python binding of libbitlogic, the GB300 (sm_103a) LUT-network hot path.
+
+Each function has the name of the C entry point it calls (see
+``include/bitlogic.h``) and only marshals arguments: it checks dtypes,
+devices and shapes of torch tensors, passes their device pointers and the
+current CUDA stream, and raises ``BitLogicError`` on a non-zero status.  All
+arithmetic runs in the library's CUDA kernels; there is no other code path.
+If the library is missing or fails to load, every call raises.
+
+Layouts: raw samples ``x`` uint8 [B, d]; soft activations fp32
+[features, B] (batch contiguous); connectivity int32 [w, k]; table logits
+fp32 [w, 2^k]; hard tables int64 [w] holding uint64 bit patterns; packed
+bits int32 [rows, ceil(N/32)] holding uint32 words.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional, Tuple
+
+import numpy as np
+import torch
+
+from . import build as _build
+
+__all__ = [
+    "BitLogicError", "load", "bitlogic_encode_thermometer", "bitlogic_lut_forward",
+    "bitlogic_lut_backward_workspace", "bitlogic_lut_backward", "bitlogic_lut_backward_edges",
+    "bitlogic_csr_reduce", "bitlogic_head_loss_workspace",
+    "bitlogic_head_loss", "bitlogic_binarize_tables", "bitlogic_pack_bits",
+    "bitlogic_hard_forward", "bitlogic_build_csr", "bitlogic_device_error",
+    "bitlogic_status_string", "bitlogic_version", "LIB_PATH",
+]
+
+LIB_PATH = _build.LIB
+
+
+class BitLogicError(RuntimeError):
+    def __init__(self, fn: str, code: int, text: str):
+        super().__init__(f"{fn}: status {code} ({text})")
+        self.code = code
+
+
+_lib = None
+_P, _I32, _I64, _F32, _SZ = (ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64,
+                             ctypes.c_float, ctypes.c_size_t)
+_SIGS = {
+    "bitlogic_encode_thermometer": ([_P, _I64, _I32, _P, _I32, _P, _P], ctypes.c_int),
+    "bitlogic_lut_forward": ([_P, _I32, _I64, _P, _P, _I32, _I32, _P, _P], ctypes.c_int),
+    "bitlogic_lut_backward_workspace": ([_I32, _I64, _I32, _I32, _I32], _SZ),
+    "bitlogic_lut_backward": ([_P, _I32, _I64, _P, _P, _I32, _I32, _P, _P, _P, _P, _P,
+                               _P, _SZ, _P], ctypes.c_int),
+    "bitlogic_lut_backward_edges": ([_P, _I32, _I64, _P, _P, _I32, _I32, _P, _P, _P, _P],
+                                    ctypes.c_int),
+    "bitlogic_csr_reduce": ([_P, _I64, _P, _P, _I32, _I32, _P, _P], ctypes.c_int),
+    "bitlogic_head_loss_workspace": ([_I64, _I32], _SZ),
+    "bitlogic_head_loss": ([_P, _I32, _I64, _I32, _F32, _P, _P, _P, _P, _P, _SZ, _P],
+                           ctypes.c_int),
+    "bitlogic_binarize_tables": ([_P, _I32, _I32, _P, _P], ctypes.c_int),
+    "bitlogic_pack_bits": ([_P, _I64, _I32, _P, _I32, _P, _P], ctypes.c_int),
+    "bitlogic_hard_forward": ([_P, _I32, _I64, _P, _P, _I32, _I32, _P, _I32, _P, _P, _P],
+                              ctypes.c_int),
+    "bitlogic_build_csr": ([_P, _I32, _I32, _I32, _P, _P], ctypes.c_int),
+    "bitlogic_device_error": ([_P], ctypes.c_int),
+    "bitlogic_status_string": ([ctypes.c_int], ctypes.c_char_p),
+    "bitlogic_version": ([], ctypes.c_int),
+}
+
+
+def load(build_if_missing: bool = True):
+    """Load (building first if needed) the CUDA library; raises if absent."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH) or not _build.up_to_date():
+            if not build_if_missing:
+                raise RuntimeError(f"CUDA library {LIB_PATH} is missing")
+            _build.build()
+        lib = ctypes.CDLL(LIB_PATH)
+        for name, (args, res) in _SIGS.items():
+            fn = getattr(lib, name)
+            fn.argtypes = args
+            fn.restype = res
+        _lib = lib
+    return _lib
+
+
+def _check(fn: str, code: int):
+    if code != 0:
+        raise BitLogicError(fn, code, bitlogic_status_string(code))
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _need(t: torch.Tensor, name: str, dtype: torch.dtype, shape: Tuple[int, ...]):
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name}: expected {dtype}, got {t.dtype}")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be on a CUDA device")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name}: expected shape {tuple(shape)}, got {tuple(t.shape)}")
+
+
+def _thr_buf(thresholds) -> Tuple[ctypes.Array, int]:
+    vals = [int(v) for v in thresholds]
+    if any(v < 0 or v > 255 for v in vals):
+        raise ValueError("thresholds must be uint8 values")
+    return (ctypes.c_uint8 * max(1, len(vals)))(*vals), len(vals)
+
+
+def bitlogic_status_string(code: int) -> str:
+    return load().bitlogic_status_string(int(code)).decode()
+
+
+def bitlogic_version() -> int:
+    return load().bitlogic_version()
+
+
+def bitlogic_encode_thermometer(x: torch.Tensor, thresholds, bits: torch.Tensor, stream=None):
+    B, d = x.shape
+    buf, b = _thr_buf(thresholds)
+    _need(x, "x", torch.uint8, (B, d))
+    _need(bits, "bits", torch.float32, (d * b, B))
+    _check("bitlogic_encode_thermometer", load().bitlogic_encode_thermometer(
+        _ptr(x), B, d, buf, b, _ptr(bits), _stream(stream)))
+
+
+def bitlogic_lut_forward(X: torch.Tensor, conn: torch.Tensor, theta: torch.Tensor,
+                         Y: torch.Tensor, stream=None):
+    w_in, B = X.shape
+    w, k = conn.shape
+    _need(X, "X", torch.float32, (w_in, B))
+    _need(conn, "conn", torch.int32, (w, k))
+    _need(theta, "theta", torch.float32, (w, 1 << k))
+    _need(Y, "Y", torch.float32, (w, B))
+    _check("bitlogic_lut_forward", load().bitlogic_lut_forward(
+        _ptr(X), w_in, B, _ptr(conn), _ptr(theta), w, k, _ptr(Y), _stream(stream)))
+
+
+def bitlogic_lut_backward_workspace(w_in: int, B: int, w: int, k: int, want_dx: bool) -> int:
+    return int(load().bitlogic_lut_backward_workspace(w_in, B, w, k, int(bool(want_dx))))
+
+
+def bitlogic_lut_backward(X: torch.Tensor, conn: torch.Tensor, theta: torch.Tensor,
+                          dY: torch.Tensor, dtheta: torch.Tensor,
+                          dX: Optional[torch.Tensor] = None,
+                          csr_off: Optional[torch.Tensor] = None,
+                          csr_edge: Optional[torch.Tensor] = None,
+                          workspace: Optional[torch.Tensor] = None, stream=None):
+    w_in, B = X.shape
+    w, k = conn.shape
+    _need(X, "X", torch.float32, (w_in, B))
+    _need(conn, "conn", torch.int32, (w, k))
+    _need(theta, "theta", torch.float32, (w, 1 << k))
+    _need(dY, "dY", torch.float32, (w, B))
+    _need(dtheta, "dtheta", torch.float32, (w, 1 << k))
+    ws_bytes = 0
+    if dX is not None:
+        _need(dX, "dX", torch.float32, (w_in, B))
+        _need(csr_off, "csr_off", torch.int32, (w_in + 1,))
+        _need(csr_edge, "csr_edge", torch.int32, (w * k,))
+        if workspace is None or not workspace.is_cuda or workspace.dtype != torch.uint8:
+            raise ValueError("workspace: uint8 CUDA tensor required when dX is requested")
+        ws_bytes = workspace.numel()
+    _check("bitlogic_lut_backward", load().bitlogic_lut_backward(
+        _ptr(X), w_in, B, _ptr(conn), _ptr(theta), w, k, _ptr(dY), _ptr(csr_off),
+        _ptr(csr_edge), _ptr(dtheta), _ptr(dX), _ptr(workspace), ws_bytes, _stream(stream)))
+
+
+def bitlogic_lut_backward_edges(X: torch.Tensor, conn: torch.Tensor, theta: torch.Tensor,
+                                dY: torch.Tensor, dtheta: torch.Tensor,
+                                edge_terms: Optional[torch.Tensor] = None, stream=None):
+    w_in, B = X.shape
+    w, k = conn.shape
+    _need(X, "X", torch.float32, (w_in, B))
+    _need(conn, "conn", torch.int32, (w, k))
+    _need(theta, "theta", torch.float32, (w, 1 << k))
+    _need(dY, "dY", torch.float32, (w, B))
+    _need(dtheta, "dtheta", torch.float32, (w, 1 << k))
+    if edge_terms is not None:
+        _need(edge_terms, "edge_terms", torch.float32, (w * k, B))
+    _check("bitlogic_lut_backward_edges", load().bitlogic_lut_backward_edges(
+        _ptr(X), w_in, B, _ptr(conn), _ptr(theta), w, k, _ptr(dY), _ptr(dtheta),
+        _ptr(edge_terms), _stream(stream)))
+
+
+def bitlogic_csr_reduce(edge_terms: torch.Tensor, csr_off: torch.Tensor, csr_edge: torch.Tensor,
+                        dX: torch.Tensor, stream=None):
+    nE, B = edge_terms.shape
+    w_in = dX.shape[0]
+    _need(edge_terms, "edge_terms", torch.float32, (nE, B))
+    _need(csr_off, "csr_off", torch.int32, (w_in + 1,))
+    _need(csr_edge, "csr_edge", torch.int32, (nE,))
+    _need(dX, "dX", torch.float32, (w_in, B))
+    _check("bitlogic_csr_reduce", load().bitlogic_csr_reduce(
+        _ptr(edge_terms), B, _ptr(csr_off), _ptr(csr_edge), w_in, nE, _ptr(dX), _stream(stream)))
+
+
+def bitlogic_head_loss_workspace(B: int, C: int) -> int:
+    return int(load().bitlogic_head_loss_workspace(B, C))
+
+
+def bitlogic_head_loss(Y: torch.Tensor, labels: torch.Tensor, C: int, tau: float,
+                       loss: torch.Tensor, workspace: torch.Tensor,
+                       logits: Optional[torch.Tensor] = None,
+                       dY: Optional[torch.Tensor] = None, stream=None):
+    w, B = Y.shape
+    _need(Y, "Y", torch.float32, (w, B))
+    _need(labels, "labels", torch.int32, (B,))
+    _need(loss, "loss", torch.float32, (1,))
+    if logits is not None:
+        _need(logits, "logits", torch.float32, (B, C))
+    if dY is not None:
+        _need(dY, "dY", torch.float32, (w, B))
+    if workspace is None or not workspace.is_cuda or workspace.dtype != torch.uint8:
+        raise ValueError("workspace: uint8 CUDA tensor required")
+    _check("bitlogic_head_loss", load().bitlogic_head_loss(
+        _ptr(Y), w, B, C, float(tau), _ptr(labels), _ptr(logits), _ptr(loss), _ptr(dY),
+        _ptr(workspace), workspace.numel(), _stream(stream)))
+
+
+def bitlogic_binarize_tables(theta: torch.Tensor, table: torch.Tensor, stream=None):
+    w, K = theta.shape
+    k = K.bit_length() - 1
+    _need(theta, "theta", torch.float32, (w, K))
+    _need(table, "table", torch.int64, (w,))
+    _check("bitlogic_binarize_tables", load().bitlogic_binarize_tables(
+        _ptr(theta), w, k, _ptr(table), _stream(stream)))
+
+
+def bitlogic_pack_bits(x: torch.Tensor, thresholds, xp: torch.Tensor, stream=None):
+    N, d = x.shape
+    buf, b = _thr_buf(thresholds)
+    _need(x, "x", torch.uint8, (N, d))
+    _need(xp, "xp", torch.int32, (d * b, (N + 31) // 32))
+    _check("bitlogic_pack_bits", load().bitlogic_pack_bits(
+        _ptr(x), N, d, buf, b, _ptr(xp), _stream(stream)))
+
+
+def bitlogic_hard_forward(xp: torch.Tensor, N: int, conn: torch.Tensor, table: torch.Tensor,
+                          yp: Optional[torch.Tensor] = None, C: int = 0,
+                          counts: Optional[torch.Tensor] = None,
+                          pred: Optional[torch.Tensor] = None, stream=None):
+    w_in, W = xp.shape
+    w, k = conn.shape
+    if W != (N + 31) // 32:
+        raise ValueError("xp has the wrong number of words for N")
+    _need(xp, "xp", torch.int32, (w_in, W))
+    _need(conn, "conn", torch.int32, (w, k))
+    _need(table, "table", torch.int64, (w,))
+    if yp is not None:
+        _need(yp, "yp", torch.int32, (w, W))
+    if counts is not None:
+        _need(counts, "counts", torch.int32, (N, C))
+    if pred is not None:
+        _need(pred, "pred", torch.int32, (N,))
+    _check("bitlogic_hard_forward", load().bitlogic_hard_forward(
+        _ptr(xp), w_in, N, _ptr(conn), _ptr(table), w, k, _ptr(yp), C, _ptr(counts),
+        _ptr(pred), _stream(stream)))
+
+
+def bitlogic_build_csr(conn: np.ndarray, w_in: int) -> Tuple[np.ndarray, np.ndarray]:
+    """Host call: inverse connectivity of int32 conn [w, k] -> (off, edge)."""
+    conn = np.ascontiguousarray(conn, dtype=np.int32)
+    w, k = conn.shape
+    off = np.zeros(w_in + 1, np.int32)
+    edge = np.zeros(w * k, np.int32)
+    _check("bitlogic_build_csr", load().bitlogic_build_csr(
+        conn.ctypes.data_as(_P), w, k, w_in, off.ctypes.data_as(_P), edge.ctypes.data_as(_P)))
+    return off, edge
+
+
+def bitlogic_device_error(stream=None) -> int:
+    """Synchronizes the stream; returns 0 or the device index-flag status."""
+    return int(load().bitlogic_device_error(_stream(stream)))

@@ -1,0 +1,60 @@
+// Internal helpers shared by the CUDA translation units of libbitlogic.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "bitlogic.h"
+
+namespace bitlogic {
+
+// Device-side index flag.  `static` gives each translation unit its own
+// copy; every unit registers a reader with bitlogic_device_error().
+static __device__ unsigned int g_index_error;
+
+__device__ __forceinline__ void flag_index_error() { atomicOr(&g_index_error, 1u); }
+
+// Reads and clears this unit's flag (synchronizes the stream).
+static int read_and_clear_index_error(cudaStream_t stream) {
+    unsigned int v = 0, zero = 0;
+    if (cudaMemcpyFromSymbolAsync(&v, g_index_error, sizeof(v), 0,
+                                  cudaMemcpyDeviceToHost, stream) != cudaSuccess)
+        return BITLOGIC_ERR_CUDA;
+    if (cudaMemcpyToSymbolAsync(g_index_error, &zero, sizeof(zero), 0,
+                                cudaMemcpyHostToDevice, stream) != cudaSuccess)
+        return BITLOGIC_ERR_CUDA;
+    if (cudaStreamSynchronize(stream) != cudaSuccess) return BITLOGIC_ERR_CUDA;
+    return v ? BITLOGIC_ERR_DEVICE : BITLOGIC_OK;
+}
+
+inline int launch_status() {
+    return cudaGetLastError() == cudaSuccess ? BITLOGIC_OK : BITLOGIC_ERR_CUDA;
+}
+
+inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Thresholds travel by value in the kernel parameters: no constant-memory
+// state is shared between calls or streams.
+struct Thresholds {
+    int b;
+    uint8_t t[32];
+};
+
+inline int make_thresholds(const uint8_t* thr_host, int32_t b, Thresholds* out) {
+    if (!thr_host) return BITLOGIC_ERR_NULL;
+    if (b < 1 || b > 32) return BITLOGIC_ERR_THRESH;
+    out->b = b;
+    for (int i = 0; i < 32; ++i) out->t[i] = i < b ? thr_host[i] : 0;
+    return BITLOGIC_OK;
+}
+
+// Logistic function on the CUDA-core FP32 path: CUDA's expf and an
+// IEEE-rounded division (no fast-math).
+__device__ __forceinline__ float sigmoidf(float z) { return 1.0f / (1.0f + expf(-z)); }
+
+}  // namespace bitlogic
+
+#define BITLOGIC_ERROR_READER(name)                                            \
+    extern "C" int bitlogic_internal_index_error_##name(cudaStream_t s) {      \
+        return bitlogic::read_and_clear_index_error(s);                        \
+    }

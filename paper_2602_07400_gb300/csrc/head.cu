@@ -1,0 +1,174 @@
+// Group-sum head with temperature and softmax cross-entropy (paper §3
+// "Encoders and heads": popcount GroupSum; §4 "Training": cross-entropy on
+// the raw head logits, averaged over the batch).
+//
+//   logits[s][c] = (sum_{j in group c} Y[j][s]) / tau,  group c = [c*g, (c+1)*g)
+//   loss         = mean_s (logsumexp(logits[s]) - logits[s][label_s])
+//   dY[j][s]     = ((softmax(logits[s])[c(j)] - [c(j) == label_s]) / B) / tau
+//
+// Four short kernels: group sums (lanes over samples, warps over the rows of
+// a group), per-sample softmax (one warp per sample), the broadcast of
+// dlogit/tau over each group's rows, and a single-block batch mean.  Every
+// reduction runs in a fixed order.
+#include <cfloat>
+
+#include "common.cuh"
+
+namespace bitlogic {
+namespace {
+
+constexpr int kSumWarps = 8;
+
+__global__ void __launch_bounds__(kSumWarps * 32)
+head_group_sum_kernel(const float* __restrict__ Y, long long B, int C, int g, float tau,
+                      float* __restrict__ logits) {
+    __shared__ float part[kSumWarps][32];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int c = blockIdx.x;
+    const long long s = (long long)blockIdx.y * 32 + lane;
+    float acc = 0.f;
+    if (s < B) {
+        const long long j0 = (long long)c * g;
+        int r = warp;
+#pragma unroll 4
+        for (; r < g; r += kSumWarps) acc += __ldg(Y + (j0 + r) * B + s);
+    }
+    part[warp][lane] = acc;
+    __syncthreads();
+    if (warp == 0 && s < B) {
+        float t = 0.f;
+#pragma unroll
+        for (int q = 0; q < kSumWarps; ++q) t += part[q][lane];
+        logits[s * C + c] = t / tau;
+    }
+}
+
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+constexpr int kSoftWarps = 8;
+
+__global__ void __launch_bounds__(kSoftWarps * 32)
+head_softmax_kernel(const float* __restrict__ logits, long long B, int C,
+                    const int* __restrict__ labels, float* __restrict__ dlogit,
+                    float* __restrict__ per_sample) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const long long s = (long long)blockIdx.x * kSoftWarps + warp;
+    if (s >= B) return;
+    const float* l = logits + s * C;
+    float m = -FLT_MAX;
+    for (int c = lane; c < C; c += 32) m = fmaxf(m, l[c]);
+    m = warp_max(m);
+    float z = 0.f;
+    for (int c = lane; c < C; c += 32) z += expf(l[c] - m);
+    z = warp_sum(z);
+    const float lse = m + logf(z);
+    int lab = __ldg(labels + s);
+    if (lab < 0 || lab >= C) {
+        if (lane == 0) flag_index_error();
+        lab = 0;
+    }
+    if (lane == 0) per_sample[s] = lse - l[lab];
+    const float invB = 1.0f / (float)B;
+    for (int c = lane; c < C; c += 32) {
+        const float p = expf(l[c] - lse);
+        dlogit[s * C + c] = (p - (c == lab ? 1.0f : 0.0f)) * invB;
+    }
+}
+
+// dY[j][s] = dlogit[s][j / g] / tau: thread per sample, each block a run of
+// kRows rows, so stores along the batch are coalesced.
+constexpr int kDyThreads = 128;
+constexpr int kDyRows = 32;
+
+__global__ void __launch_bounds__(kDyThreads)
+head_dy_kernel(const float* __restrict__ dlogit, long long B, int C, int g, int w, float tau,
+               float* __restrict__ dY) {
+    const long long s = (long long)blockIdx.y * kDyThreads + threadIdx.x;
+    if (s >= B) return;
+    const int j0 = blockIdx.x * kDyRows;
+    const int j1 = min(w, j0 + kDyRows);
+    int c = j0 / g;
+    int cend = (c + 1) * g;
+    float v = __ldg(dlogit + s * C + c) / tau;
+    for (int j = j0; j < j1; ++j) {
+        if (j >= cend) {
+            ++c;
+            cend += g;
+            v = __ldg(dlogit + s * C + c) / tau;
+        }
+        dY[(long long)j * B + s] = v;
+    }
+}
+
+// loss = (sum_s per_sample[s]) / B in one block: strided per-thread sums in
+// index order, then a fixed shared-memory tree.
+__global__ void __launch_bounds__(256)
+head_mean_kernel(const float* __restrict__ per_sample, long long B, float* __restrict__ loss) {
+    __shared__ float red[256];
+    float acc = 0.f;
+    for (long long s = threadIdx.x; s < B; s += 256) acc += per_sample[s];
+    red[threadIdx.x] = acc;
+    __syncthreads();
+    for (int o = 128; o > 0; o >>= 1) {
+        if (threadIdx.x < o) red[threadIdx.x] += red[threadIdx.x + o];
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) loss[0] = red[0] / (float)B;
+}
+
+size_t align_up(size_t v) { return (v + 255) & ~(size_t)255; }
+
+}  // namespace
+}  // namespace bitlogic
+
+using namespace bitlogic;
+
+BITLOGIC_ERROR_READER(head)
+
+extern "C" size_t bitlogic_head_loss_workspace(int64_t B, int32_t C) {
+    if (B <= 0 || C <= 0) return 0;
+    const size_t bc = (size_t)B * (size_t)C * sizeof(float);
+    // dlogit [B][C], per-sample loss [B], logits [B][C] (used when the
+    // caller passes no logits buffer)
+    return align_up(bc) + align_up((size_t)B * sizeof(float)) + align_up(bc);
+}
+
+extern "C" int bitlogic_head_loss(const float* Y, int32_t w, int64_t B, int32_t C, float tau,
+                                  const int32_t* labels, float* logits, float* loss, float* dY,
+                                  void* workspace, size_t ws_bytes, cudaStream_t stream) {
+    if (!Y || !labels || !loss || !workspace) return BITLOGIC_ERR_NULL;
+    if (w <= 0 || B <= 0 || C <= 0 || w % C != 0 || !(tau > 0.f)) return BITLOGIC_ERR_SHAPE;
+    if (B > 0x7fffffffLL / (C > 0 ? C : 1)) return BITLOGIC_ERR_SHAPE;
+    if (!aligned16(workspace)) return BITLOGIC_ERR_ALIGN;
+    if (ws_bytes < bitlogic_head_loss_workspace(B, C)) return BITLOGIC_ERR_WORKSPACE;
+    const int g = w / C;
+    char* ws = static_cast<char*>(workspace);
+    const size_t bc = (size_t)B * (size_t)C * sizeof(float);
+    float* dlogit = reinterpret_cast<float*>(ws);
+    float* per = reinterpret_cast<float*>(ws + align_up(bc));
+    float* lg = logits ? logits : reinterpret_cast<float*>(ws + align_up(bc) + align_up((size_t)B * 4));
+
+    const long long sb = (B + 31) / 32;
+    if (sb > 65535) return BITLOGIC_ERR_SHAPE;
+    head_group_sum_kernel<<<dim3((unsigned)C, (unsigned)sb), kSumWarps * 32, 0, stream>>>(Y, B, C, g, tau, lg);
+    head_softmax_kernel<<<(unsigned)((B + kSoftWarps - 1) / kSoftWarps), kSoftWarps * 32, 0, stream>>>(
+        lg, B, C, labels, dlogit, per);
+    if (dY) {
+        const long long gy = (B + kDyThreads - 1) / kDyThreads;
+        if (gy > 65535) return BITLOGIC_ERR_SHAPE;
+        head_dy_kernel<<<dim3((unsigned)((w + kDyRows - 1) / kDyRows), (unsigned)gy), kDyThreads, 0, stream>>>(
+            dlogit, B, C, g, w, tau, dY);
+    }
+    head_mean_kernel<<<1, 256, 0, stream>>>(per, B, loss);
+    return launch_status();
+}

@@ -1,0 +1,159 @@
+"""The hot path as call sequences over device-resident buffers.
+
+``TrainStep`` runs one soft training step of the two-layer network of the
+paper's protocol (§4 "Architecture": encoder -> logic layer -> logic layer
+-> head): thermometer encode, two LUT forwards, group-sum head with
+cross-entropy, two LUT backwards.  ``HardInfer`` runs the hard bit-packed
+evaluation (App. C.1): binarize tables, encode + pack, hard layer 1, hard
+layer 2 with the fused popcount head and argmax.  Buffers are allocated once
+(torch provides the device memory); every step only enqueues library calls
+on the current stream, so a step can be replayed or captured in a CUDA graph.
+"""
+from __future__ import annotations
+
+from typing import Optional, Sequence
+
+import numpy as np
+import torch
+
+from . import (bitlogic_binarize_tables, bitlogic_build_csr, bitlogic_csr_reduce,
+               bitlogic_encode_thermometer, bitlogic_hard_forward, bitlogic_head_loss,
+               bitlogic_head_loss_workspace, bitlogic_lut_backward_edges, bitlogic_lut_forward,
+               bitlogic_pack_bits)
+
+
+def _nomark(name: str) -> None:
+    return None
+
+
+class Network:
+    """Connectivity, table logits and inverse connectivity of a two-layer
+    LUT network, resident on the device."""
+
+    def __init__(self, conn1: np.ndarray, theta1: np.ndarray, conn2: np.ndarray,
+                 theta2: np.ndarray, w_in: int, device="cuda"):
+        self.w_in = int(w_in)
+        self.w1, self.k1 = conn1.shape
+        self.w2, self.k2 = conn2.shape
+        dev = torch.device(device)
+        self.conn1 = torch.from_numpy(np.ascontiguousarray(conn1, np.int32)).to(dev)
+        self.conn2 = torch.from_numpy(np.ascontiguousarray(conn2, np.int32)).to(dev)
+        self.theta1 = torch.from_numpy(np.ascontiguousarray(theta1, np.float32)).to(dev)
+        self.theta2 = torch.from_numpy(np.ascontiguousarray(theta2, np.float32)).to(dev)
+        off1, edge1 = bitlogic_build_csr(conn1, self.w_in)
+        off2, edge2 = bitlogic_build_csr(conn2, self.w1)
+        self.off1, self.edge1 = torch.from_numpy(off1).to(dev), torch.from_numpy(edge1).to(dev)
+        self.off2, self.edge2 = torch.from_numpy(off2).to(dev), torch.from_numpy(edge2).to(dev)
+
+
+class TrainStep:
+    def __init__(self, net: Network, B: int, d: int, thresholds: Sequence[int], C: int,
+                 tau: float, want_dx1: bool = False, device="cuda"):
+        dev = torch.device(device)
+        self.net, self.B, self.d, self.C, self.tau = net, int(B), int(d), int(C), float(tau)
+        self.thr = [int(t) for t in thresholds]
+        assert d * len(self.thr) == net.w_in
+        f32 = dict(dtype=torch.float32, device=dev)
+        self.x = torch.zeros(B, d, dtype=torch.uint8, device=dev)
+        self.labels = torch.zeros(B, dtype=torch.int32, device=dev)
+        self.bits = torch.empty(net.w_in, B, **f32)
+        self.y1 = torch.empty(net.w1, B, **f32)
+        self.y2 = torch.empty(net.w2, B, **f32)
+        self.logits = torch.empty(B, C, **f32)
+        self.loss = torch.zeros(1, **f32)
+        self.dy2 = torch.empty(net.w2, B, **f32)
+        self.dy1 = torch.empty(net.w1, B, **f32)
+        self.dth1 = torch.empty_like(net.theta1)
+        self.dth2 = torch.empty_like(net.theta2)
+        self.dbits = torch.empty(net.w_in, B, **f32) if want_dx1 else None
+        # per-edge input-gradient terms of layer 2 (and of layer 1 when its
+        # input gradient is wanted), summed per input through the CSR map
+        self.edges2 = torch.empty(net.w2 * net.k2, B, **f32)
+        self.edges1 = torch.empty(net.w1 * net.k1, B, **f32) if want_dx1 else None
+        self.ws_head = torch.empty(bitlogic_head_loss_workspace(B, C), dtype=torch.uint8, device=dev)
+
+    def load(self, x: torch.Tensor, labels: torch.Tensor, non_blocking: bool = False):
+        self.x.copy_(x, non_blocking=non_blocking)
+        self.labels.copy_(labels, non_blocking=non_blocking)
+
+    def forward(self, stream=None, mark=_nomark):
+        n = self.net
+        bitlogic_encode_thermometer(self.x, self.thr, self.bits, stream)
+        mark("encode")
+        bitlogic_lut_forward(self.bits, n.conn1, n.theta1, self.y1, stream)
+        mark("forward1")
+        bitlogic_lut_forward(self.y1, n.conn2, n.theta2, self.y2, stream)
+        mark("forward2")
+        bitlogic_head_loss(self.y2, self.labels, self.C, self.tau, self.loss, self.ws_head,
+                           logits=self.logits, dY=self.dy2, stream=stream)
+        mark("head")
+
+    def backward(self, stream=None, mark=_nomark):
+        # each layer's backward is bitlogic_lut_backward split into its two
+        # phases (node kernel, then CSR reduction) so each can be timed
+        n = self.net
+        bitlogic_lut_backward_edges(self.y1, n.conn2, n.theta2, self.dy2, self.dth2,
+                                    self.edges2, stream)
+        mark("backward2")
+        bitlogic_csr_reduce(self.edges2, n.off2, n.edge2, self.dy1, stream)
+        mark("csr2")
+        bitlogic_lut_backward_edges(self.bits, n.conn1, n.theta1, self.dy1, self.dth1,
+                                    self.edges1, stream)
+        mark("backward1")
+        if self.dbits is not None:
+            bitlogic_csr_reduce(self.edges1, n.off1, n.edge1, self.dbits, stream)
+            mark("csr1")
+
+    def run(self, stream=None, mark=_nomark):
+        self.forward(stream, mark)
+        self.backward(stream, mark)
+
+    # kernels one run() launches (encode 1, forwards 2, head 4, backwards and
+    # CSR reductions 3 or 4)
+    @property
+    def kernels_per_run(self) -> int:
+        return 10 + (1 if self.dbits is not None else 0)
+
+
+class HardInfer:
+    def __init__(self, net: Network, N: int, d: int, thresholds: Sequence[int], C: int,
+                 keep_layer2: bool = False, device="cuda"):
+        dev = torch.device(device)
+        self.net, self.N, self.d, self.C = net, int(N), int(d), int(C)
+        self.thr = [int(t) for t in thresholds]
+        W = (N + 31) // 32
+        i32 = dict(dtype=torch.int32, device=dev)
+        self.x = torch.zeros(N, d, dtype=torch.uint8, device=dev)
+        self.table1 = torch.empty(net.w1, dtype=torch.int64, device=dev)
+        self.table2 = torch.empty(net.w2, dtype=torch.int64, device=dev)
+        self.xp = torch.empty(net.w_in, W, **i32)
+        self.yp1 = torch.empty(net.w1, W, **i32)
+        self.yp2 = torch.empty(net.w2, W, **i32) if keep_layer2 else None
+        self.counts = torch.empty(N, C, **i32)
+        self.pred = torch.empty(N, **i32)
+
+    def binarize(self, stream=None, mark=_nomark):
+        bitlogic_binarize_tables(self.net.theta1, self.table1, stream)
+        bitlogic_binarize_tables(self.net.theta2, self.table2, stream)
+        mark("binarize")
+
+    def run(self, stream=None, mark=_nomark):
+        n = self.net
+        bitlogic_pack_bits(self.x, self.thr, self.xp, stream)
+        mark("pack")
+        bitlogic_hard_forward(self.xp, self.N, n.conn1, self.table1, yp=self.yp1, stream=stream)
+        mark("hard1")
+        bitlogic_hard_forward(self.yp1, self.N, n.conn2, self.table2, yp=self.yp2, C=self.C,
+                              counts=self.counts, pred=self.pred, stream=stream)
+        mark("hard2")
+
+    # kernels: binarize 2; pack 1, layer 1, layer 2 with head, argmax
+    kernels_per_binarize = 2
+    kernels_per_run = 4
+
+
+def unpack_bits(words: torch.Tensor, N: int) -> np.ndarray:
+    """int32 words [rows, W] (uint32 bit patterns) -> uint8 bits [rows, N] on the host."""
+    w = words.detach().cpu().numpy().view(np.uint32)
+    bits = (w[:, :, None] >> np.arange(32, dtype=np.uint32)[None, None, :]) & 1
+    return bits.reshape(w.shape[0], -1)[:, :N].astype(np.uint8)

@@ -1,0 +1,119 @@
+"""The C ABI without a GPU: the library builds, loads, exports every symbol
+``include/bitlogic.h`` declares, and its host-only parts behave."""
+import ctypes
+import os
+import re
+import subprocess
+
+import numpy as np
+import pytest
+
+import paper_2602_07400_gb300 as bl
+from paper_2602_07400_gb300 import synth
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "bitlogic.h")
+
+
+def _declared():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(bitlogic_\w+)\s*\(", src)))
+
+
+def test_header_declares_the_boundary():
+    names = _declared()
+    for n in ["bitlogic_encode_thermometer", "bitlogic_lut_forward", "bitlogic_lut_backward",
+              "bitlogic_head_loss", "bitlogic_pack_bits", "bitlogic_hard_forward"]:
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol():
+    lib = bl.load()
+    for n in _declared():
+        assert hasattr(lib, n), n
+    out = subprocess.run(["nm", "-D", "--defined-only", bl.LIB_PATH], capture_output=True,
+                         text=True, check=True).stdout
+    exported = set(re.findall(r"\b(bitlogic_\w+)\b", out))
+    assert set(_declared()) <= exported
+
+
+def test_python_binding_names_match_header():
+    for n in _declared():
+        if n in ("bitlogic_internal_index_error",):
+            continue
+        assert hasattr(bl, n), n
+
+
+def test_status_strings_and_version():
+    assert bl.bitlogic_status_string(0) == "ok"
+    for c in range(-1, -10, -1):
+        assert bl.bitlogic_status_string(c) != "unknown status"
+    assert bl.bitlogic_version() >= 100
+
+
+def test_build_csr_matches_inverse_map():
+    w, k, w_in = 300, 6, 97
+    conn = synth.connectivity(w, k, w_in, seed=5)
+    off, edge = bl.bitlogic_build_csr(conn, w_in)
+    assert off[0] == 0 and off[-1] == w * k
+    flat = conn.reshape(-1)
+    for i in range(w_in):
+        es = edge[off[i]:off[i + 1]]
+        want = np.nonzero(flat == i)[0]
+        np.testing.assert_array_equal(es, want)        # increasing edge ids
+    # inputs never read get empty rows
+    conn2 = np.array([[0, 1], [1, 2]], np.int32)
+    off2, edge2 = bl.bitlogic_build_csr(conn2, 6)
+    assert off2.tolist() == [0, 1, 3, 4, 4, 4, 4]
+    assert edge2.tolist() == [0, 1, 2, 3]
+
+
+def test_build_csr_rejects_out_of_range():
+    conn = np.array([[0, 5]], np.int32)
+    with pytest.raises(bl.BitLogicError) as e:
+        bl.bitlogic_build_csr(conn, 5)
+    assert e.value.code == -7
+    with pytest.raises(bl.BitLogicError):
+        bl.bitlogic_build_csr(np.array([[0, -1]], np.int32), 5)
+
+
+def test_host_validation_returns_before_any_launch():
+    # every call below is rejected on the host, so no CUDA work is issued
+    lib = bl.load()
+    P = ctypes.c_void_p
+    fake = P(16)
+    thr = (ctypes.c_uint8 * 3)(64, 128, 192)
+    assert lib.bitlogic_lut_forward(None, 4, 8, fake, fake, 2, 2, fake, None) == -1
+    assert lib.bitlogic_lut_forward(fake, 4, 8, fake, fake, 2, 7, fake, None) == -3
+    assert lib.bitlogic_lut_forward(fake, 4, 8, fake, fake, 2, 0, fake, None) == -3
+    assert lib.bitlogic_lut_forward(fake, 2, 8, fake, fake, 2, 3, fake, None) == -3
+    assert lib.bitlogic_lut_forward(fake, 0, 8, fake, fake, 2, 2, fake, None) == -2
+    assert lib.bitlogic_lut_forward(fake, 4, -1, fake, fake, 2, 2, fake, None) == -2
+    # B == 0 is an accepted no-op
+    assert lib.bitlogic_lut_forward(fake, 4, 0, fake, fake, 2, 2, fake, None) == 0
+    # backward: dX requested without CSR / workspace, too-small / misaligned workspace
+    assert lib.bitlogic_lut_backward(fake, 4, 8, fake, fake, 2, 2, fake, None, None,
+                                     fake, fake, fake, 1 << 20, None) == -1
+    assert lib.bitlogic_lut_backward(fake, 4, 8, fake, fake, 2, 2, fake, fake, fake,
+                                     fake, fake, fake, 4, None) == -5
+    assert lib.bitlogic_lut_backward(fake, 4, 8, fake, fake, 2, 2, fake, fake, fake,
+                                     fake, fake, P(17), 1 << 20, None) == -4
+    # head: w % C != 0, tau <= 0
+    assert lib.bitlogic_head_loss(fake, 10, 8, 3, 1.0, fake, None, fake, None, fake, 1 << 20, None) == -2
+    assert lib.bitlogic_head_loss(fake, 9, 8, 3, 0.0, fake, None, fake, None, fake, 1 << 20, None) == -2
+    # thresholds: b out of range
+    assert lib.bitlogic_pack_bits(fake, 64, 4, thr, 0, fake, None) == -9
+    assert lib.bitlogic_pack_bits(fake, 64, 4, thr, 33, fake, None) == -9
+    assert lib.bitlogic_encode_thermometer(fake, 64, 4, None, 3, fake, None) == -1
+    # hard: headless call needs yp; head needs counts and w % C == 0
+    assert lib.bitlogic_hard_forward(fake, 8, 64, fake, fake, 4, 2, None, 0, None, None, None) == -1
+    assert lib.bitlogic_hard_forward(fake, 8, 64, fake, fake, 4, 2, None, 2, None, None, None) == -1
+    assert lib.bitlogic_hard_forward(fake, 8, 64, fake, fake, 4, 2, None, 3, fake, None, None) == -2
+    assert lib.bitlogic_binarize_tables(fake, 4, 7, fake, None) == -3
+
+
+def test_workspace_queries():
+    assert bl.bitlogic_lut_backward_workspace(100, 64, 10, 6, False) == 0
+    assert bl.bitlogic_lut_backward_workspace(100, 64, 10, 6, True) == 10 * 6 * 64 * 4
+    assert bl.bitlogic_head_loss_workspace(64, 10) >= 2 * 64 * 10 * 4 + 64 * 4

@@ -1,0 +1,318 @@
+"""GPU-vs-oracle parity of each C-ABI call on small, ragged and degenerate
+shapes (several tiles plus a tail), through the Python binding."""
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2602_07400_gb300 as bl
+from paper_2602_07400_gb300 import synth
+from parity_util import check_exact, check_fwd, check_grad
+
+pytestmark = pytest.mark.gpu
+
+oracle.set_threads(os.cpu_count() or 1)
+
+
+def dev(a, dtype=None):
+    t = torch.from_numpy(np.ascontiguousarray(a))
+    if dtype is not None:
+        t = t.to(dtype)
+    return t.cuda()
+
+
+def no_device_error():
+    assert bl.bitlogic_device_error() == 0
+
+
+# ---------------------------------------------------------------- encoder --
+
+@pytest.mark.parametrize("B,d,b", [(1, 5, 3), (37, 784, 3), (256, 70, 7), (1000, 33, 15), (65, 9, 32), (3, 1, 1)])
+def test_encode_thermometer(B, d, b):
+    rng = np.random.default_rng(B * 7 + d)
+    x = rng.integers(0, 256, size=(B, d), dtype=np.uint8)
+    thr = sorted(rng.choice(256, size=b, replace=False).tolist())
+    bits = torch.full((d * b, B), -1.0, device="cuda")
+    bl.bitlogic_encode_thermometer(dev(x), thr, bits)
+    check_exact(bits.cpu().numpy().astype(np.float64), oracle.encode_thermometer(x, thr), "bits")
+    no_device_error()
+
+
+# ----------------------------------------------------------- soft forward --
+
+SHAPES = [  # (k, w_in, w, B)
+    (1, 3, 5, 1), (2, 7, 9, 5), (3, 40, 33, 37), (4, 100, 65, 128), (5, 64, 130, 259),
+    (6, 300, 129, 256), (6, 6, 17, 100), (6, 1000, 64, 1027), (2, 2, 40, 64),
+]
+
+
+@pytest.mark.parametrize("k,w_in,w,B", SHAPES)
+@pytest.mark.parametrize("binary", [False, True])
+def test_lut_forward(k, w_in, w, B, binary):
+    X = (synth.binary_activations if binary else synth.uniform_activations)(w_in, B, seed=k + B)
+    conn = synth.connectivity(w, k, w_in, seed=w)
+    theta = synth.table_logits(w, 1 << k, seed=k)
+    Y = torch.full((w, B), np.nan, device="cuda")
+    bl.bitlogic_lut_forward(dev(X), dev(conn), dev(theta), Y)
+    check_fwd(Y, oracle.lut_forward(X.astype(np.float64), conn, theta), "Y")
+    no_device_error()
+
+
+def test_lut_forward_unaligned_scalar_path():
+    # a view that starts 4 bytes into an allocation takes the scalar path
+    k, w_in, w, B = 6, 50, 20, 64
+    X = synth.uniform_activations(w_in, B, seed=1)
+    conn = synth.connectivity(w, k, w_in, seed=2)
+    theta = synth.table_logits(w, 64, seed=3)
+    big = torch.zeros(w_in * B + 1, device="cuda")
+    big[1:] = dev(X).reshape(-1)
+    Xv = big[1:].view(w_in, B)
+    Y = torch.empty(w, B, device="cuda")
+    bl.bitlogic_lut_forward(Xv, dev(conn), dev(theta), Y)
+    check_fwd(Y, oracle.lut_forward(X.astype(np.float64), conn, theta), "Y")
+
+
+# ---------------------------------------------------------- soft backward --
+
+@pytest.mark.parametrize("k,w_in,w,B", SHAPES)
+def test_lut_backward(k, w_in, w, B):
+    X = synth.uniform_activations(w_in, B, seed=k * 3 + B)
+    conn = synth.connectivity(w, k, w_in, seed=w + 1)
+    theta = synth.table_logits(w, 1 << k, seed=k + 5)
+    dY = synth.uniform_gradients(w, B, seed=B, scale=1e-3)
+    off, edge = bl.bitlogic_build_csr(conn, w_in)
+    dth = torch.full((w, 1 << k), np.nan, device="cuda")
+    dX = torch.full((w_in, B), np.nan, device="cuda")
+    ws = torch.empty(bl.bitlogic_lut_backward_workspace(w_in, B, w, k, True), dtype=torch.uint8, device="cuda")
+    bl.bitlogic_lut_backward(dev(X), dev(conn), dev(theta), dev(dY), dth, dX=dX,
+                             csr_off=dev(off), csr_edge=dev(edge), workspace=ws)
+    wth, wdx = oracle.lut_backward(X.astype(np.float64), conn, theta, dY.astype(np.float64))
+    check_grad(dth, wth, "dtheta")
+    check_grad(dX, wdx, "dX")
+    # dX skipped: dtheta unchanged, nothing else written
+    dth2 = torch.full((w, 1 << k), np.nan, device="cuda")
+    bl.bitlogic_lut_backward(dev(X), dev(conn), dev(theta), dev(dY), dth2)
+    check_exact(dth2.cpu().numpy(), dth.cpu().numpy(), "dtheta without dX")
+    no_device_error()
+
+
+def test_backward_is_deterministic_and_handles_skewed_consumers():
+    # 3 inputs shared by 500 nodes (fan-in 2): every input has ~333 consumers
+    k, w_in, w, B = 2, 3, 500, 96
+    X = synth.uniform_activations(w_in, B, seed=1)
+    conn = synth.connectivity(w, k, w_in, seed=2)
+    theta = synth.table_logits(w, 4, seed=3)
+    dY = synth.uniform_gradients(w, B, seed=4, scale=1e-2)
+    off, edge = bl.bitlogic_build_csr(conn, w_in)
+    ws = torch.empty(bl.bitlogic_lut_backward_workspace(w_in, B, w, k, True), dtype=torch.uint8, device="cuda")
+    outs = []
+    for _ in range(2):
+        dth = torch.empty(w, 4, device="cuda")
+        dX = torch.empty(w_in, B, device="cuda")
+        bl.bitlogic_lut_backward(dev(X), dev(conn), dev(theta), dev(dY), dth, dX=dX,
+                                 csr_off=dev(off), csr_edge=dev(edge), workspace=ws)
+        outs.append((dth.cpu().numpy(), dX.cpu().numpy()))
+    check_exact(outs[0][0], outs[1][0], "dtheta run-to-run")
+    check_exact(outs[0][1], outs[1][1], "dX run-to-run")
+    wth, wdx = oracle.lut_backward(X.astype(np.float64), conn, theta, dY.astype(np.float64))
+    check_grad(outs[0][0], wth, "dtheta")
+    check_grad(outs[0][1], wdx, "dX")
+
+
+def test_backward_unused_inputs_get_zero():
+    k, w_in, w, B = 3, 50, 4, 40     # at most 12 of 50 inputs are read
+    X = synth.uniform_activations(w_in, B, seed=5)
+    conn = synth.connectivity(w, k, w_in, seed=6)
+    theta = synth.table_logits(w, 8, seed=7)
+    dY = synth.uniform_gradients(w, B, seed=8)
+    off, edge = bl.bitlogic_build_csr(conn, w_in)
+    dX = torch.full((w_in, B), np.nan, device="cuda")
+    ws = torch.empty(bl.bitlogic_lut_backward_workspace(w_in, B, w, k, True), dtype=torch.uint8, device="cuda")
+    bl.bitlogic_lut_backward(dev(X), dev(conn), dev(theta), dev(dY), torch.empty(w, 8, device="cuda"),
+                             dX=dX, csr_off=dev(off), csr_edge=dev(edge), workspace=ws)
+    unused = np.setdiff1d(np.arange(w_in), conn.reshape(-1))
+    assert unused.size > 0
+    assert torch.all(dX[torch.from_numpy(unused).cuda()] == 0)
+
+
+def test_empty_batch_is_a_noop():
+    k, w_in, w = 2, 5, 3
+    conn = dev(synth.connectivity(w, k, w_in, seed=1))
+    theta = dev(synth.table_logits(w, 4, seed=1))
+    X = torch.empty(w_in, 0, device="cuda")
+    Y = torch.empty(w, 0, device="cuda")
+    bl.bitlogic_lut_forward(X, conn, theta, Y)
+    dth = torch.full((w, 4), 7.0, device="cuda")
+    bl.bitlogic_lut_backward(X, conn, theta, torch.empty(w, 0, device="cuda"), dth)
+    assert torch.all(dth == 0)
+    xp = torch.empty(10, 0, dtype=torch.int32, device="cuda")
+    bl.bitlogic_pack_bits(torch.empty(0, 5, dtype=torch.uint8, device="cuda"), [1, 2], xp)
+
+
+# -------------------------------------------------------------------- head --
+
+@pytest.mark.parametrize("C,g,B,tau", [(10, 100, 256, 10.0), (3, 7, 37, 2.0), (100, 13, 259, 100.0),
+                                       (1, 40, 5, 1.0), (10, 800, 1, 20.0)])
+def test_head_loss(C, g, B, tau):
+    rng = np.random.default_rng(C + B)
+    Y = rng.random((C * g, B)).astype(np.float32)
+    labels = rng.integers(0, C, size=B).astype(np.int32)
+    loss = torch.zeros(1, device="cuda")
+    logits = torch.empty(B, C, device="cuda")
+    dY = torch.empty(C * g, B, device="cuda")
+    ws = torch.empty(bl.bitlogic_head_loss_workspace(B, C), dtype=torch.uint8, device="cuda")
+    bl.bitlogic_head_loss(dev(Y), dev(labels), C, tau, loss, ws, logits=logits, dY=dY)
+    wl, wloss, wdy = oracle.head_loss(Y.astype(np.float64), labels, C, tau)
+    check_fwd(logits, wl, "logits")
+    check_fwd(loss, np.array([wloss]), "loss")
+    check_grad(dY, wdy, "dY")
+    # optional outputs absent
+    loss2 = torch.zeros(1, device="cuda")
+    bl.bitlogic_head_loss(dev(Y), dev(labels), C, tau, loss2, ws)
+    check_exact(loss2.cpu().numpy(), loss.cpu().numpy(), "loss without optional outputs")
+    no_device_error()
+
+
+# -------------------------------------------------------------------- hard --
+
+def test_binarize_tables():
+    rng = np.random.default_rng(3)
+    for k in (1, 2, 5, 6):
+        theta = rng.standard_normal((77, 1 << k)).astype(np.float32)
+        theta[::5, 0] = 0.0
+        theta[1::7, -1] = -0.0
+        theta[2::9, 0] = np.float32(1e-45)
+        tab = torch.empty(77, dtype=torch.int64, device="cuda")
+        bl.bitlogic_binarize_tables(dev(theta), tab)
+        check_exact(tab.cpu().numpy().view(np.uint64), oracle.binarize_tables(theta), f"table k={k}")
+
+
+@pytest.mark.parametrize("N,d,b", [(1, 5, 3), (31, 8, 1), (32, 16, 7), (33, 9, 3), (1000, 784, 3),
+                                   (1025, 24, 15), (5000, 3, 32), (70000, 17, 2)])
+def test_pack_bits(N, d, b):
+    rng = np.random.default_rng(N + d)
+    x = rng.integers(0, 256, size=(N, d), dtype=np.uint8)
+    thr = sorted(rng.choice(256, size=b, replace=False).tolist())
+    xp = torch.full((d * b, (N + 31) // 32), -1, dtype=torch.int32, device="cuda")
+    bl.bitlogic_pack_bits(dev(x), thr, xp)
+    check_exact(xp.cpu().numpy().view(np.uint32), oracle.pack_bits(x, thr), "xp")
+
+
+HARD = [  # (k, w_in, w, N)
+    (1, 3, 5, 1), (2, 10, 9, 31), (3, 40, 33, 33), (4, 100, 65, 1000), (5, 64, 100, 1025),
+    (6, 300, 129, 4096), (6, 7, 20, 70001), (6, 2000, 256, 100000),
+]
+
+
+@pytest.mark.parametrize("k,w_in,w,N", HARD)
+def test_hard_forward(k, w_in, w, N):
+    W = (N + 31) // 32
+    xp = synth.random_words(w_in, W, seed=N)
+    if N % 32:
+        xp[:, -1] &= np.uint32((1 << (N % 32)) - 1)
+    conn = synth.connectivity(w, k, w_in, seed=k)
+    table = synth.random_tables(w, seed=w)
+    if k < 6:
+        table &= np.uint64((1 << (1 << k)) - 1)
+    yp = torch.full((w, W), -1, dtype=torch.int32, device="cuda")
+    bl.bitlogic_hard_forward(dev(xp.view(np.int32)), N, dev(conn), dev(table.view(np.int64)), yp=yp)
+    check_exact(yp.cpu().numpy().view(np.uint32), oracle.hard_forward(xp, N, conn, table), "yp")
+    no_device_error()
+
+
+@pytest.mark.parametrize("k,w_in,C,g,N", [(6, 200, 10, 100, 1024), (6, 300, 3, 7, 37), (4, 50, 10, 33, 5000),
+                                          (2, 9, 1, 13, 100), (6, 500, 10, 1500, 70001), (6, 64, 2, 9000, 999)])
+def test_hard_forward_popcount_head(k, w_in, C, g, N):
+    w = C * g
+    W = (N + 31) // 32
+    xp = synth.random_words(w_in, W, seed=N + 1)
+    if N % 32:
+        xp[:, -1] &= np.uint32((1 << (N % 32)) - 1)
+    conn = synth.connectivity(w, k, w_in, seed=k + 1)
+    table = synth.random_tables(w, seed=w + 1)
+    counts = torch.full((N, C), -1, dtype=torch.int32, device="cuda")
+    pred = torch.full((N,), -1, dtype=torch.int32, device="cuda")
+    yp = torch.full((w, W), -1, dtype=torch.int32, device="cuda")
+    bl.bitlogic_hard_forward(dev(xp.view(np.int32)), N, dev(conn), dev(table.view(np.int64)),
+                             yp=yp, C=C, counts=counts, pred=pred)
+    wyp = oracle.hard_forward(xp, N, conn, table)
+    wc, wp = oracle.popcount_head(wyp, N, C)
+    check_exact(yp.cpu().numpy().view(np.uint32), wyp, "yp")
+    check_exact(counts.cpu().numpy(), wc, "counts")
+    check_exact(pred.cpu().numpy(), wp, "pred")
+    # head without yp and pred
+    counts2 = torch.full((N, C), -1, dtype=torch.int32, device="cuda")
+    bl.bitlogic_hard_forward(dev(xp.view(np.int32)), N, dev(conn), dev(table.view(np.int64)),
+                             C=C, counts=counts2)
+    check_exact(counts2.cpu().numpy(), wc, "counts (no yp)")
+
+
+def test_hard_equals_soft_on_binarized_tables():
+    # the correctness anchor of App. C.1 on the GPU: the soft kernel on binary
+    # inputs with theta = +-800 (t exactly 0 or 1) equals the hard kernel
+    k, w_in, w, N = 6, 200, 96, 256
+    rng = np.random.default_rng(1)
+    Xb = rng.integers(0, 2, size=(w_in, N)).astype(np.float32)
+    conn = synth.connectivity(w, k, w_in, seed=1)
+    theta = synth.table_logits(w, 64, seed=2)
+    th_hard = np.where(theta > 0, 800.0, -800.0).astype(np.float32)
+    Y = torch.empty(w, N, device="cuda")
+    bl.bitlogic_lut_forward(dev(Xb), dev(conn), dev(th_hard), Y)
+    W = N // 32
+    xp = np.zeros((w_in, W), np.uint32)
+    for s in range(N):
+        xp[:, s // 32] |= Xb[:, s].astype(np.uint32) << np.uint32(s % 32)
+    tab = torch.empty(w, dtype=torch.int64, device="cuda")
+    bl.bitlogic_binarize_tables(dev(theta), tab)
+    yp = torch.empty(w, W, dtype=torch.int32, device="cuda")
+    bl.bitlogic_hard_forward(dev(xp.view(np.int32)), N, dev(conn), tab, yp=yp)
+    from paper_2602_07400_gb300.pipeline import unpack_bits
+    check_exact(Y.cpu().numpy(), unpack_bits(yp, N).astype(np.float32), "soft vs hard")
+
+
+# -------------------------------------------------------- error handling --
+
+def test_out_of_range_connectivity_is_flagged_not_faulted():
+    # an index past w_in reaches the kernel (bypassing the host CSR check):
+    # the kernel reads row 0 instead and raises the device flag
+    k, w_in, w, B = 2, 10, 4, 32
+    conn = synth.connectivity(w, k, w_in, seed=1)
+    bad = conn.copy()
+    bad[2, 1] = w_in + 5
+    theta = synth.table_logits(w, 4, seed=1)
+    X = synth.uniform_activations(w_in, B, seed=1)
+    assert bl.bitlogic_device_error() == 0
+    Y = torch.empty(w, B, device="cuda")
+    bl.bitlogic_lut_forward(dev(X), dev(bad), dev(theta), Y)
+    assert bl.bitlogic_device_error() == -8
+    assert bl.bitlogic_device_error() == 0          # the flag was cleared
+    clamped = bad.copy()
+    clamped[2, 1] = 0
+    check_fwd(Y, oracle.lut_forward(X.astype(np.float64), clamped, theta), "Y (clamped)")
+    yp = torch.empty(w, 1, dtype=torch.int32, device="cuda")
+    bl.bitlogic_hard_forward(torch.zeros(w_in, 1, dtype=torch.int32, device="cuda"), 32,
+                             dev(bad), torch.zeros(w, dtype=torch.int64, device="cuda"), yp=yp)
+    assert bl.bitlogic_device_error() == -8
+
+
+def test_bad_label_is_flagged():
+    C, g, B = 3, 4, 8
+    Y = torch.rand(C * g, B, device="cuda")
+    labels = torch.tensor([0, 1, 2, 3, 0, 1, 2, 0], dtype=torch.int32, device="cuda")
+    ws = torch.empty(bl.bitlogic_head_loss_workspace(B, C), dtype=torch.uint8, device="cuda")
+    bl.bitlogic_head_loss(Y, labels, C, 1.0, torch.zeros(1, device="cuda"), ws)
+    assert bl.bitlogic_device_error() == -8
+
+
+def test_binding_rejects_wrong_tensors():
+    X = torch.rand(10, 8, device="cuda")
+    conn = torch.zeros(4, 2, dtype=torch.int32, device="cuda")
+    theta = torch.zeros(4, 4, device="cuda")
+    with pytest.raises(TypeError):
+        bl.bitlogic_lut_forward(X.double(), conn, theta, torch.empty(4, 8, device="cuda"))
+    with pytest.raises(ValueError):
+        bl.bitlogic_lut_forward(X, conn, theta, torch.empty(4, 9, device="cuda"))
+    with pytest.raises(ValueError):
+        bl.bitlogic_lut_forward(X.cpu(), conn, theta, torch.empty(4, 8, device="cuda"))

@@ -1,0 +1,163 @@
+"""GPU-vs-oracle parity of whole steps at the workloads' sizes, in the launch
+configuration the benchmark times (``pipeline.TrainStep`` / ``HardInfer``).
+
+* tiny (256 x 784, 1000 x 1000, k=6): every output element, including the
+  input gradients of both layers.
+* mnist (1024 x 784, 8000 x 8000, k=6 and k=2): every output element.
+* cifar10 / cifar100 (64000- and 128000-wide layers): the forward, logits,
+  loss and head gradient over the full batch; table gradients of sampled
+  nodes of both layers and the layer-1 output gradient of sampled nodes, each
+  computed by the oracle on the sub-network that feeds them (every consumer
+  of a sampled node is included, so the sums are the full sums).
+* hard_cifar10 (2^22 samples): every sample runs on the GPU; sampled samples
+  (first and last included) are recomputed by the oracle from the raw
+  samples, bit-exact for the packed input, both layers, counts and argmax.
+"""
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2602_07400_gb300 import synth
+from paper_2602_07400_gb300.pipeline import HardInfer, Network, TrainStep, unpack_bits
+from parity_util import check_exact, check_fwd, check_grad
+
+pytestmark = pytest.mark.gpu
+
+oracle.set_threads(os.cpu_count() or 1)
+
+
+def _step(wl, want_dx1, seed=0, k=None):
+    if k is not None:
+        wl = synth.Workload(wl.name, wl.batch, wl.d, wl.classes, wl.sigma, wl.thresholds, wl.widths, k, wl.tau)
+    conn1, th1, conn2, th2 = synth.network(wl, seed)
+    x, labels = synth.blob_batch(wl.batch, wl.d, wl.classes, wl.sigma, seed=seed + 7)
+    net = Network(conn1, th1, conn2, th2, wl.w_in)
+    st = TrainStep(net, wl.batch, wl.d, wl.thresholds, wl.classes, wl.tau, want_dx1=want_dx1)
+    st.load(x.cuda(), labels.cuda())
+    st.run()
+    torch.cuda.synchronize()
+    return wl, st, x.numpy(), labels.numpy(), (conn1, th1, conn2, th2)
+
+
+def _full_compare(wl, st, x, labels, params, want_dx1):
+    conn1, th1, conn2, th2 = params
+    r = oracle.train_step(x, labels, wl.thresholds, conn1, th1, conn2, th2, wl.classes, wl.tau,
+                          want_dx1=want_dx1)
+    check_exact(st.bits.cpu().numpy().astype(np.float64), r["bits"], "bits")
+    check_fwd(st.y1, r["y1"], "y1")
+    check_fwd(st.y2, r["y2"], "y2")
+    check_fwd(st.logits, r["logits"], "logits")
+    check_fwd(st.loss, np.array([r["loss"]]), "loss")
+    check_grad(st.dy2, r["dy2"], "dy2")
+    check_grad(st.dth2, r["dth2"], "dtheta2")
+    check_grad(st.dy1, r["dy1"], "dy1")
+    check_grad(st.dth1, r["dth1"], "dtheta1")
+    if want_dx1:
+        check_grad(st.dbits, r["dbits"], "dbits")
+
+
+def test_tiny_step_all_outputs():
+    wl, st, x, labels, params = _step(synth.WORKLOADS["tiny"], want_dx1=True)
+    _full_compare(wl, st, x, labels, params, True)
+
+
+@pytest.mark.parametrize("k", [6, 2])
+def test_mnist_step_all_outputs(k):
+    wl, st, x, labels, params = _step(synth.WORKLOADS["mnist"], want_dx1=False, k=k)
+    _full_compare(wl, st, x, labels, params, False)
+
+
+def _sampled_compare(wl, st, x, labels, params, n_nodes=96, seed=0):
+    conn1, th1, conn2, th2 = params
+    bits = oracle.encode_thermometer(x, wl.thresholds)
+    check_exact(st.bits.cpu().numpy().astype(np.float64), bits, "bits")
+    y1 = oracle.lut_forward(bits, conn1, th1)
+    check_fwd(st.y1, y1, "y1")
+    y2 = oracle.lut_forward(y1, conn2, th2)
+    check_fwd(st.y2, y2, "y2")
+    logits, loss, dy2 = oracle.head_loss(y2, labels, wl.classes, wl.tau)
+    check_fwd(st.logits, logits, "logits")
+    check_fwd(st.loss, np.array([loss]), "loss")
+    check_grad(st.dy2, dy2, "dy2")
+    rng = np.random.default_rng(seed)
+    w1, w2 = wl.widths
+    # layer-2 table gradients of sampled nodes
+    n2 = np.unique(np.concatenate([[0, w2 - 1], rng.integers(0, w2, n_nodes)]))
+    dth2, _ = oracle.lut_backward(y1, conn2[n2], th2[n2], dy2[n2], want_dx=False)
+    check_grad(st.dth2[torch.from_numpy(n2).cuda()], dth2, "dtheta2[sampled]")
+    # layer-1 output gradient of sampled layer-1 nodes: all their consumers
+    n1 = np.unique(np.concatenate([[0, w1 - 1], rng.integers(0, w1, n_nodes)]))
+    cons = np.unique(np.nonzero(np.isin(conn2, n1))[0])
+    _, dx_sub = oracle.lut_backward(y1, conn2[cons], th2[cons], dy2[cons], want_dx=True)
+    dy1_s = dx_sub[n1]
+    check_grad(st.dy1[torch.from_numpy(n1).cuda()], dy1_s, "dy1[sampled]")
+    dth1, _ = oracle.lut_backward(bits, conn1[n1], th1[n1], dy1_s, want_dx=False)
+    check_grad(st.dth1[torch.from_numpy(n1).cuda()], dth1, "dtheta1[sampled]")
+
+
+@pytest.mark.slow
+def test_cifar10_step_sampled():
+    wl, st, x, labels, params = _step(synth.WORKLOADS["cifar10"], want_dx1=False)
+    _sampled_compare(wl, st, x, labels, params)
+
+
+@pytest.mark.slow
+def test_cifar100_step_sampled():
+    wl, st, x, labels, params = _step(synth.WORKLOADS["cifar100"], want_dx1=False)
+    _sampled_compare(wl, st, x, labels, params, n_nodes=64)
+
+
+def _hard_run(wl, N, seed=0, samples=1536):
+    conn1, th1, conn2, th2 = synth.network(wl, seed)
+    net = Network(conn1, th1, conn2, th2, wl.w_in)
+    hi = HardInfer(net, N, wl.d, wl.thresholds, wl.classes)
+    x, labels = synth.blob_batch(N, wl.d, wl.classes, wl.sigma, seed=seed + 11, device="cuda")
+    hi.x.copy_(x)
+    del x, labels
+    hi.binarize()
+    hi.run()
+    torch.cuda.synchronize()
+    S = synth.sample_positions(N, samples, seed=seed)
+    Sd = torch.from_numpy(S).cuda()
+    xs = hi.x.index_select(0, Sd).cpu().numpy()
+    t1 = oracle.binarize_tables(th1)
+    t2 = oracle.binarize_tables(th2)
+    check_exact(hi.table1.cpu().numpy().view(np.uint64), t1, "table1")
+    check_exact(hi.table2.cpu().numpy().view(np.uint64), t2, "table2")
+    r = oracle.hard_infer(xs, wl.thresholds, conn1, t1, conn2, t2, wl.classes)
+    n = len(S)
+
+    def cols(words):   # bits of the sampled samples, [rows, n]
+        wsel = words.index_select(1, (Sd // 32)).cpu().numpy().view(np.uint32)
+        return ((wsel >> (S % 32).astype(np.uint32)[None, :]) & 1).astype(np.uint8)
+
+    check_exact(cols(hi.xp), unpack_bits(torch.from_numpy(r["xp"].view(np.int32)), n), "xp[sampled]")
+    check_exact(cols(hi.yp1), unpack_bits(torch.from_numpy(r["yp1"].view(np.int32)), n), "yp1[sampled]")
+    check_exact(hi.counts.index_select(0, Sd).cpu().numpy(), r["counts"], "counts[sampled]")
+    check_exact(hi.pred.index_select(0, Sd).cpu().numpy(), r["pred"], "pred[sampled]")
+    # properties over every sample: counts of a sample sum to the number of
+    # ones among layer-2 outputs, each within [0, g]; pred is an argmax
+    g = wl.widths[1] // wl.classes
+    c = hi.counts
+    assert int(c.min()) >= 0 and int(c.max()) <= g
+    best = c.max(dim=1).values
+    assert torch.equal(c.gather(1, hi.pred.long()[:, None])[:, 0], best)
+    first = (c == best[:, None]).int().argmax(dim=1)
+    assert torch.equal(first.int(), hi.pred)
+
+
+@pytest.mark.slow
+def test_hard_cifar10_full_size_sampled():
+    wl = synth.WORKLOADS["hard_cifar10"]
+    _hard_run(wl, wl.batch)
+
+
+def test_hard_ragged_batch():
+    wl = synth.WORKLOADS["hard_cifar10"]
+    small = synth.Workload("hard_small", 0, wl.d, wl.classes, wl.sigma, wl.thresholds, (4000, 4000), 6, wl.tau)
+    _hard_run(small, 100003, samples=700)
+    _hard_run(small, 1024, samples=300)
+    _hard_run(small, 37, samples=37)
