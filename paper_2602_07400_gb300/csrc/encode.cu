@@ -122,9 +122,9 @@ extern "C" int bitlogic_encode_thermometer(const uint8_t* x, int64_t B, int32_t 
     Thresholds th;
     int st = make_thresholds(thr_host, b, &th);
     if (st) return st;
-    if (!x || !bits) return BITLOGIC_ERR_NULL;
     if (B < 0 || d <= 0) return BITLOGIC_ERR_SHAPE;
-    if (B == 0) return BITLOGIC_OK;
+    if (B == 0) return BITLOGIC_OK;   // an empty batch may come as NULL
+    if (!x || !bits) return BITLOGIC_ERR_NULL;
     const long long gy = (B + kEncTS - 1) / kEncTS;
     if (gy > 65535) return BITLOGIC_ERR_SHAPE;
     dim3 grid((unsigned)((d + kEncTF - 1) / kEncTF), (unsigned)gy);
@@ -138,9 +138,9 @@ extern "C" int bitlogic_pack_bits(const uint8_t* x, int64_t N, int32_t d,
     Thresholds th;
     int st = make_thresholds(thr_host, b, &th);
     if (st) return st;
-    if (!x || !xp) return BITLOGIC_ERR_NULL;
     if (N < 0 || d <= 0) return BITLOGIC_ERR_SHAPE;
-    if (N == 0) return BITLOGIC_OK;
+    if (N == 0) return BITLOGIC_OK;   // an empty batch may come as NULL
+    if (!x || !xp) return BITLOGIC_ERR_NULL;
     const long long W = (N + 31) / 32;
     const long long gy = (N + kPackTS - 1) / kPackTS;
     if (gy > 65535) return BITLOGIC_ERR_SHAPE;

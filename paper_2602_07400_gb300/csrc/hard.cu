@@ -280,15 +280,14 @@ extern "C" int bitlogic_hard_forward(const uint32_t* xp, int32_t w_in, int64_t N
                                      int32_t w, int32_t k, uint32_t* yp,
                                      int32_t C, int32_t* counts, int32_t* pred,
                                      cudaStream_t stream) {
-    if (!xp || !conn || !table) return BITLOGIC_ERR_NULL;
+    if (!conn || !table) return BITLOGIC_ERR_NULL;
     if (w_in <= 0 || w <= 0 || N < 0 || C < 0) return BITLOGIC_ERR_SHAPE;
     if (k < 1 || k > 6 || k > w_in) return BITLOGIC_ERR_FANIN;
+    if (C > 0 && w % C != 0) return BITLOGIC_ERR_SHAPE;
+    if (N == 0) return BITLOGIC_OK;   // an empty batch may come as NULL
+    if (!xp) return BITLOGIC_ERR_NULL;
     if (C == 0 && !yp) return BITLOGIC_ERR_NULL;
-    if (C > 0) {
-        if (!counts) return BITLOGIC_ERR_NULL;
-        if (w % C != 0) return BITLOGIC_ERR_SHAPE;
-    }
-    if (N == 0) return BITLOGIC_OK;
+    if (C > 0 && !counts) return BITLOGIC_ERR_NULL;
     if ((N + 31) / 32 > (1ll << 40)) return BITLOGIC_ERR_SHAPE;
     switch (k) {
         case 1: return launch_hard<1>(xp, w_in, N, conn, table, w, yp, C, counts, pred, stream);

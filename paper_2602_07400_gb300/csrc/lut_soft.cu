@@ -331,7 +331,8 @@ int launch_backward(const float* X, int w_in, long long B, const int* conn, cons
 
 int check_layer(const void* X, int32_t w_in, int64_t B, const void* conn, const void* theta,
                 int32_t w, int32_t k) {
-    if (!X || !conn || !theta) return BITLOGIC_ERR_NULL;
+    if (!conn || !theta) return BITLOGIC_ERR_NULL;
+    if (B > 0 && !X) return BITLOGIC_ERR_NULL;   // an empty batch may come as NULL
     if (w_in <= 0 || w <= 0 || B < 0) return BITLOGIC_ERR_SHAPE;
     if (k < 1 || k > 6 || k > w_in) return BITLOGIC_ERR_FANIN;
     if ((int64_t)w * k > 0x7fffffffLL) return BITLOGIC_ERR_SHAPE;
@@ -350,8 +351,8 @@ extern "C" int bitlogic_lut_forward(const float* X, int32_t w_in, int64_t B,
                                     int32_t w, int32_t k, float* Y, cudaStream_t stream) {
     int st = check_layer(X, w_in, B, conn, theta, w, k);
     if (st) return st;
-    if (!Y) return BITLOGIC_ERR_NULL;
     if (B == 0) return BITLOGIC_OK;
+    if (!Y) return BITLOGIC_ERR_NULL;
     const bool vec = (B % 4 == 0) && aligned16(X) && aligned16(Y);
     switch (k) {
         case 1: return launch_forward<1>(X, w_in, B, conn, theta, w, Y, vec, stream);
@@ -377,7 +378,7 @@ extern "C" int bitlogic_lut_backward_edges(const float* X, int32_t w_in, int64_t
                                            cudaStream_t stream) {
     int st = check_layer(X, w_in, B, conn, theta, w, k);
     if (st) return st;
-    if (!dY || !dtheta) return BITLOGIC_ERR_NULL;
+    if (!dtheta || (B > 0 && !dY)) return BITLOGIC_ERR_NULL;
     if (B == 0) {
         // empty batch: the batch sums are zero
         if (cudaMemsetAsync(dtheta, 0, sizeof(float) * (size_t)w * ((size_t)1 << k), stream) != cudaSuccess)
@@ -398,9 +399,9 @@ extern "C" int bitlogic_lut_backward_edges(const float* X, int32_t w_in, int64_t
 extern "C" int bitlogic_csr_reduce(const float* edge_terms, int64_t B, const int32_t* csr_off,
                                    const int32_t* csr_edge, int32_t w_in, int32_t n_edges,
                                    float* dX, cudaStream_t stream) {
-    if (!edge_terms || !csr_off || !csr_edge || !dX) return BITLOGIC_ERR_NULL;
     if (B < 0 || w_in <= 0 || n_edges < 0) return BITLOGIC_ERR_SHAPE;
     if (B == 0) return BITLOGIC_OK;
+    if (!edge_terms || !csr_off || !csr_edge || !dX) return BITLOGIC_ERR_NULL;
     const bool vec = (B % 4 == 0) && aligned16(edge_terms) && aligned16(dX);
     dim3 grid((unsigned)((w_in + kCsrWarps - 1) / kCsrWarps));
     if (vec)
@@ -418,8 +419,8 @@ extern "C" int bitlogic_lut_backward(const float* X, int32_t w_in, int64_t B,
                                      void* workspace, size_t ws_bytes, cudaStream_t stream) {
     int st = check_layer(X, w_in, B, conn, theta, w, k);
     if (st) return st;
-    if (!dY || !dtheta) return BITLOGIC_ERR_NULL;
-    const bool want_dx = dX != nullptr;
+    if (!dtheta || (B > 0 && !dY)) return BITLOGIC_ERR_NULL;
+    const bool want_dx = dX != nullptr && B > 0;
     if (want_dx) {
         if (!csr_off || !csr_edge) return BITLOGIC_ERR_NULL;
         if (!workspace) return BITLOGIC_ERR_NULL;
