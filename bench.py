@@ -123,6 +123,23 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
+# ------------------------------------------------- cross-rank helpers --
+
+def max_over_ranks(values, device):
+    """Element-wise max of per-rank timings (the job is as slow as its
+    slowest rank)."""
+    import torch.distributed as dist
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    if dist.is_available() and dist.is_initialized() and dist.get_world_size() > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(v) for v in t.tolist()]
+
+
+def job_rate(world: int, samples_per_rank_step: int, steps: int, max_ms: float) -> float:
+    """Whole-job samples/s: every rank's samples over the slowest rank's time."""
+    return world * samples_per_rank_step * steps / (max_ms * 1e-3)
+
+
 # ------------------------------------------------------ work per call --
 
 def call_work(wl, B):
@@ -259,12 +276,7 @@ def run_ours(args):
             t_total += dt
         train_ms.append(t_train)
         hard_ms.append(t_total - t_train)
-    train_sum = float(sum(train_ms))
-    hard_sum = float(sum(hard_ms))
-    tot = torch.tensor([train_sum, hard_sum], dtype=torch.float64, device="cuda")
-    if world > 1:
-        torch.distributed.all_reduce(tot, op=torch.distributed.ReduceOp.MAX)
-    train_sum, hard_sum = float(tot[0]), float(tot[1])
+    train_sum, hard_sum = max_over_ranks([sum(train_ms), sum(hard_ms)], "cuda")
 
     launches = K * (hi.kernels_per_binarize + hi.kernels_per_run)
     if st is not None:
@@ -299,7 +311,7 @@ def run_ours(args):
             b_, o_ = work[n]
             calls_out[n] = {"ms": round(t, 5), "GB/s": round(b_ / (t * 1e-3) / 1e9, 1),
                             "Tops/s": round(o_ / (t * 1e-3) / 1e12, 2) if o_ else None}
-        value = world * B * K / (train_sum * 1e-3) if st is not None else world * B * K / (hard_sum * 1e-3)
+        value = job_rate(world, B, K, train_sum if st is not None else hard_sum)
         result = {
             "metric": METRIC,
             "value": value,
@@ -317,7 +329,7 @@ def run_ours(args):
                        "widths": list(wl.widths), "k": wl.k, "classes": wl.classes, "tau": wl.tau,
                        "l2": "flushed between steps (512 MB write outside the timed events)",
                        "parallelism": f"dp{world} (independent batches, no collective)"},
-            "hard": {"value": world * B * K / (hard_sum * 1e-3) / 1e6, "unit": "MSamples/s",
+            "hard": {"value": job_rate(world, B, K, hard_sum) / 1e6, "unit": "MSamples/s",
                      "ms_per_batch": ms_step_hard, "batch": B,
                      "includes": "binarize + encode/pack + 2 hard layers + popcount head + argmax"},
             "ms_per_step_total": ms_step_train + ms_step_hard,
@@ -363,11 +375,8 @@ def run_e2e(args, st, hi, wl, B):
             loss_host.copy_(st.loss, non_blocking=True)
         e1.record()
         torch.cuda.synchronize()
-        ms = e0.elapsed_time(e1)
-        t = torch.tensor([ms], dtype=torch.float64, device="cuda")
-        if world > 1:
-            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        out["train"] = {"value": world * B * K / (float(t[0]) * 1e-3), "unit": "samples/s",
+        ms = max_over_ranks([e0.elapsed_time(e1)], "cuda")[0]
+        out["train"] = {"value": job_rate(world, B, K, ms), "unit": "samples/s",
                         "h2d_bytes_per_step": x_host.numel() + 4 * lab_host.numel(),
                         "d2h_bytes_per_step": 4}
     for _ in range(3):
@@ -385,11 +394,8 @@ def run_e2e(args, st, hi, wl, B):
         pred_host.copy_(hi.pred, non_blocking=True)
     e1.record()
     torch.cuda.synchronize()
-    ms = e0.elapsed_time(e1)
-    t = torch.tensor([ms], dtype=torch.float64, device="cuda")
-    if world > 1:
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-    out["hard"] = {"value": world * B * K / (float(t[0]) * 1e-3) / 1e6, "unit": "MSamples/s",
+    ms = max_over_ranks([e0.elapsed_time(e1)], "cuda")[0]
+    out["hard"] = {"value": job_rate(world, B, K, ms) / 1e6, "unit": "MSamples/s",
                    "h2d_bytes_per_step": x_host.numel(), "d2h_bytes_per_step": 4 * B}
     return out
 

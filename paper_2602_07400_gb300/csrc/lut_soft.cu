@@ -100,6 +100,20 @@ __device__ __forceinline__ void node_setup(const int* __restrict__ conn,
     __syncwarp();
 }
 
+// ---------------------------------------------------- async copy helpers --
+
+// Asynchronous 16-byte global -> shared copies (L2 only), grouped per stage.
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
+    const unsigned s = (unsigned)__cvta_generic_to_shared(smem);
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(s), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
+
+constexpr int kStageSamples = 128;   // samples per pipeline stage
+constexpr int kStages = 3;           // stages in flight per warp
+
 // ------------------------------------------------------------- forward --
 
 template <int k, bool VEC>
@@ -147,6 +161,72 @@ lut_forward_kernel(const float* __restrict__ X, int w_in, long long B,
             yr[s] = fwd_tree<k - 1, 0>(te, d, x);
         }
     }
+}
+
+// Forward with the k gathered input rows streamed through a ring of
+// shared-memory stages (cp.async).  Each lane copies, reads back and
+// evaluates its own 4 consecutive samples of a stage (16-byte chunks), so
+// the ring needs no warp synchronisation.  The block's y index selects a
+// batch slice (see forward_chunk).  Needs B % 4 == 0, chunk % 4 == 0 and
+// 16-byte aligned X and Y.
+template <int k>
+__global__ void __launch_bounds__(kFwdWarps * 32)
+lut_forward_staged_kernel(const float* __restrict__ X, int w_in, long long B,
+                          const int* __restrict__ conn, const float* __restrict__ theta, int w,
+                          float* __restrict__ Y, long long chunk) {
+    constexpr int H = 1 << (k - 1), CH = kStageSamples;
+    __shared__ __align__(16) float sRing[kFwdWarps][kStages * k * CH];
+    __shared__ float2 sPair[kFwdWarps][H];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int j = blockIdx.x * kFwdWarps + warp;
+    if (j >= w) return;
+    int rows[k];
+    float te[H], d[H], t0, t1;
+    node_setup<k>(conn, theta, j, w_in, lane, sPair[warp], rows, te, d, t0, t1);
+    float* ring = sRing[warp] + 4 * lane;       // this lane's column of every stage row
+    const long long s0 = (long long)blockIdx.y * chunk;
+    const long long s1 = min(B, s0 + chunk);
+    const float* src[k];
+#pragma unroll
+    for (int i = 0; i < k; ++i) src[i] = X + (long long)rows[i] * B + s0 + 4 * lane;
+    float* yr = Y + (long long)j * B + s0 + 4 * lane;
+    const int nst = (int)((s1 - s0 + CH - 1) / CH);
+    const long long lim = s1 - s0 - 4 * lane;   // this lane's chunks start below lim
+
+    int ib = 0;   // ring slot of the next stage to issue
+    auto issue = [&](int st) {
+        if (st < nst && (long long)st * CH < lim) {
+            float* buf = ring + ib * (k * CH);
+#pragma unroll
+            for (int r = 0; r < k; ++r) cp_async16(buf + r * CH, src[r] + (long long)st * CH);
+        }
+        cp_async_commit();
+        ib = (ib + 1 == kStages) ? 0 : ib + 1;
+    };
+#pragma unroll
+    for (int st = 0; st < kStages - 1; ++st) issue(st);
+    int rb = 0;   // ring slot of the stage being evaluated
+    for (int st = 0; st < nst; ++st) {
+        issue(st + kStages - 1);
+        cp_async_wait<kStages - 1>();
+        if ((long long)st * CH < lim) {
+            const float* buf = ring + rb * (k * CH);
+            float4 xv[k];
+#pragma unroll
+            for (int i = 0; i < k; ++i) xv[i] = *reinterpret_cast<const float4*>(buf + i * CH);
+            float o[4];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                float x[k];
+#pragma unroll
+                for (int i = 0; i < k; ++i) x[i] = comp(xv[i], c);
+                o[c] = fwd_tree<k - 1, 0>(te, d, x);
+            }
+            *reinterpret_cast<float4*>(yr + (long long)st * CH) = make_float4(o[0], o[1], o[2], o[3]);
+        }
+        rb = (rb + 1 == kStages) ? 0 : rb + 1;
+    }
+    cp_async_wait<0>();
 }
 
 // ------------------------------------------------------------ backward --
@@ -216,6 +296,164 @@ lut_backward_kernel(const float* __restrict__ X, int w_in, long long B,
             s1 += sRed[warp][r][2 * lane + 1];
         }
         float* out = dtheta + (long long)j * K + 2 * lane;
+        out[0] = t0 * (1.0f - t0) * s0;
+        out[1] = t1 * (1.0f - t1) * s1;
+    }
+}
+
+// ---------------------------------------- backward, shared-memory staged --
+
+template <int k>
+__host__ __device__ constexpr int staged_floats_per_warp() {
+    constexpr int rows = kStages * (k + 1) * kStageSamples;
+    constexpr int red = 32 * ((1 << (k - 1)) + 1);
+    return rows > red ? rows : red;
+}
+
+template <int k>
+constexpr size_t staged_smem_bytes() {
+    return (size_t)kBwdWarps * staged_floats_per_warp<k>() * sizeof(float) +
+           (size_t)kBwdWarps * (1 << (k - 1)) * sizeof(float2);
+}
+
+// Backward with two lanes per sample: lane h = lane & 1 owns the half of
+// the table whose top input x_{k-1} equals h, i.e. one of the two subtrees
+// under the root lerp.  Each lane runs the reverse tree of its subtree
+// (adjoint g * (h ? x_{k-1} : 1 - x_{k-1})), accumulates the leaf adjoints of
+// its half for dtheta, and the pair exchanges three values by shuffle: the
+// partial dx_i of the slots the partner stores, and the subtree value that
+// gives dx_{k-1} = g * (v_1 - v_0).  Lane h stores the slots i with
+// i % 2 == h.  Halving the per-thread table and accumulators doubles the
+// resident warps.  The k gathered rows and the dY row stream through a
+// kStages-deep cp.async ring as 16-byte chunks (each lane copies one chunk
+// per row; the pair partners read them after a warp sync).  Needs k >= 2,
+// B % 4 == 0 and 16-byte aligned X and dY.
+template <int k, bool WANT_DX>
+__global__ void __launch_bounds__(kBwdWarps * 32)
+lut_backward_staged_kernel(const float* __restrict__ X, int w_in, long long B,
+                           const int* __restrict__ conn, const float* __restrict__ theta, int w,
+                           const float* __restrict__ dY, float* __restrict__ dtheta,
+                           float* __restrict__ P) {
+    constexpr int K = 1 << k, H = K / 2, H2 = K / 4, R = k + 1, CH = kStageSamples;
+    constexpr int NQ = (k + 1) / 2;   // slots stored per lane (rounded up)
+    extern __shared__ __align__(16) float smem[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int h = lane & 1, pair = lane >> 1;
+    float* ring = smem + warp * staged_floats_per_warp<k>();
+    float2* sPair = reinterpret_cast<float2*>(smem + kBwdWarps * staged_floats_per_warp<k>()) + warp * H;
+    const int j = blockIdx.x * kBwdWarps + warp;
+    if (j >= w) return;
+
+    int rows[k];
+    bool bad = false;
+#pragma unroll
+    for (int i = 0; i < k; ++i) {
+        int c = __ldg(conn + (long long)j * k + i);
+        if ((unsigned)c >= (unsigned)w_in) { bad = true; c = 0; }
+        rows[i] = c;
+    }
+    if (bad && lane == 0) flag_index_error();
+    float t0 = 0.f, t1 = 0.f;
+    if (lane < H) {
+        t0 = sigmoidf(__ldg(theta + (long long)j * K + 2 * lane));
+        t1 = sigmoidf(__ldg(theta + (long long)j * K + 2 * lane + 1));
+        sPair[lane] = make_float2(t0, t1 - t0);
+    }
+    __syncwarp();
+    float te[H2], d[H2];
+#pragma unroll
+    for (int m = 0; m < H2; ++m) {
+        const float2 v = sPair[h * H2 + m];
+        te[m] = v.x;
+        d[m] = v.y;
+    }
+    __syncwarp();
+
+    const float* src[R];
+#pragma unroll
+    for (int i = 0; i < k; ++i) src[i] = X + (long long)rows[i] * B + 4 * lane;
+    src[k] = dY + (long long)j * B + 4 * lane;
+    float* pst[NQ];   // this lane's stored slots 2q + h, at its first sample
+#pragma unroll
+    for (int q = 0; q < NQ; ++q) pst[q] = P + ((long long)j * k + (2 * q + h < k ? 2 * q + h : 0)) * B + pair;
+    const int nst = (int)((B + CH - 1) / CH);
+
+    int ib = 0;
+    auto issue = [&](int st) {
+        if (st < nst && (long long)st * CH + 4 * lane < B) {
+            float* buf = ring + ib * (R * CH) + 4 * lane;
+#pragma unroll
+            for (int r = 0; r < R; ++r) cp_async16(buf + r * CH, src[r] + (long long)st * CH);
+        }
+        cp_async_commit();
+        ib = (ib + 1 == kStages) ? 0 : ib + 1;
+    };
+
+    float acc[H];
+#pragma unroll
+    for (int a = 0; a < H; ++a) acc[a] = 0.f;
+
+#pragma unroll
+    for (int st = 0; st < kStages - 1; ++st) issue(st);
+    int rb = 0;
+    for (int st = 0; st < nst; ++st) {
+        issue(st + kStages - 1);
+        cp_async_wait<kStages - 1>();
+        __syncwarp();
+        const float* buf = ring + rb * (R * CH) + pair;
+        const long long sbase = (long long)st * CH;
+#pragma unroll 2
+        for (int c = 0; c < CH / 16; ++c) {
+            const bool in = sbase + 16 * c + pair < B;
+            float x[k], omx[k], dx[k];
+#pragma unroll
+            for (int i = 0; i < k; ++i) {
+                x[i] = in ? buf[i * CH + 16 * c] : 0.f;
+                omx[i] = 1.0f - x[i];
+                dx[i] = 0.f;
+            }
+            const float g = in ? buf[k * CH + 16 * c] : 0.f;
+            const float adj = g * (h ? x[k - 1] : omx[k - 1]);
+            const float v = bwd_tree<k - 2, 0>(te, d, x, omx, adj, dx, acc);
+            if constexpr (WANT_DX) {
+#pragma unroll
+                for (int q = 0; q < NQ; ++q) {
+                    const int e = 2 * q, o = 2 * q + 1;   // lane 0 stores e, lane 1 stores o
+                    // what the partner needs from this lane
+                    float send;
+                    if (e == k - 1)      send = v;                    // lane 0 needs v_1
+                    else if (o == k - 1) send = h ? dx[e] : v;        // lane 1 needs v_0
+                    else if (o < k)      send = h ? dx[e] : dx[o];
+                    else                 send = dx[e];
+                    const float recv = __shfl_xor_sync(0xffffffffu, send, 1);
+                    float full;
+                    if (h == 0) full = (e == k - 1) ? g * (recv - v) : dx[e] + recv;
+                    else        full = (o == k - 1) ? g * (v - recv) : (o < k ? dx[o] + recv : 0.f);
+                    if (in && (h == 0 || o < k)) pst[q][sbase + 16 * c] = full;
+                }
+            }
+        }
+        __syncwarp();
+        rb = (rb + 1 == kStages) ? 0 : rb + 1;
+    }
+    cp_async_wait<0>();
+    __syncwarp();
+
+    // dtheta: entry a lives in half a / H at offset a % H of the lanes with
+    // that parity; sum those 16 lanes in lane order through the ring
+    float* red = ring;   // [32][H + 1]
+#pragma unroll
+    for (int a = 0; a < H; ++a) red[lane * (H + 1) + a] = acc[a];
+    __syncwarp();
+    if (lane < H) {
+        float s0 = 0.f, s1 = 0.f;
+        const int a0 = 2 * lane, hh = a0 / H, ao = a0 % H;
+#pragma unroll 4
+        for (int p = 0; p < 16; ++p) {
+            s0 += red[(2 * p + hh) * (H + 1) + ao];
+            s1 += red[(2 * p + hh) * (H + 1) + ao + 1];
+        }
+        float* out = dtheta + (long long)j * K + a0;
         out[0] = t0 * (1.0f - t0) * s0;
         out[1] = t1 * (1.0f - t1) * s1;
     }
@@ -311,9 +549,22 @@ int launch_forward(const float* X, int w_in, long long B, const int* conn, const
     if (ny > 65535) return BITLOGIC_ERR_SHAPE;
     dim3 grid((unsigned)((w + kFwdWarps - 1) / kFwdWarps), (unsigned)ny);
     if (vec)
-        lut_forward_kernel<k, true><<<grid, kFwdWarps * 32, 0, st>>>(X, w_in, B, conn, theta, w, Y, chunk);
+        lut_forward_staged_kernel<k><<<grid, kFwdWarps * 32, 0, st>>>(X, w_in, B, conn, theta, w, Y, chunk);
     else
         lut_forward_kernel<k, false><<<grid, kFwdWarps * 32, 0, st>>>(X, w_in, B, conn, theta, w, Y, chunk);
+    return launch_status();
+}
+
+template <int k, bool WANT_DX>
+int launch_staged(const float* X, int w_in, long long B, const int* conn, const float* theta,
+                  int w, const float* dY, float* dtheta, float* P, cudaStream_t st) {
+    constexpr size_t smem = staged_smem_bytes<k>();
+    auto kern = lut_backward_staged_kernel<k, WANT_DX>;
+    if (smem > 48 * 1024 &&
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+        return BITLOGIC_ERR_CUDA;
+    dim3 grid((unsigned)((w + kBwdWarps - 1) / kBwdWarps));
+    kern<<<grid, kBwdWarps * 32, smem, st>>>(X, w_in, B, conn, theta, w, dY, dtheta, P);
     return launch_status();
 }
 
@@ -321,6 +572,12 @@ template <int k>
 int launch_backward(const float* X, int w_in, long long B, const int* conn, const float* theta,
                     int w, const float* dY, float* dtheta, float* P, bool want_dx,
                     cudaStream_t st) {
+    if constexpr (k >= 2) {
+        const bool staged = (B % 4 == 0) && aligned16(X) && aligned16(dY);
+        if (staged)
+            return want_dx ? launch_staged<k, true>(X, w_in, B, conn, theta, w, dY, dtheta, P, st)
+                           : launch_staged<k, false>(X, w_in, B, conn, theta, w, dY, dtheta, P, st);
+    }
     dim3 grid((unsigned)((w + kBwdWarps - 1) / kBwdWarps));
     if (want_dx)
         lut_backward_kernel<k, true><<<grid, kBwdWarps * 32, 0, st>>>(X, w_in, B, conn, theta, w, dY, dtheta, P);
