@@ -56,6 +56,8 @@ def parse_args():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--profile", action="store_true",
                    help="plain timed loop only (for ncu launch lists)")
+    p.add_argument("--batch", type=int, default=0,
+                   help="override the workload's batch (smaller cases for ncu captures)")
     return p.parse_args()
 
 
@@ -157,10 +159,13 @@ def call_work(wl, B):
         "encode": (B * d + f * win * B, 0),
         "forward1": (f * (win * B + w1 * B + w1 * K + w1 * k), (2 * (K - 1) + k) * w1 * B),
         "forward2": (f * (w1 * B + w2 * B + w2 * K + w2 * k), (2 * (K - 1) + k) * w2 * B),
-        "head": (f * (2 * w2 * B + 3 * B * C), 0),
-        "backward2": (f * (w1 * B + w2 * B + w2 * k * B + 2 * w2 * K + w2 * k), (4 * (K - 1) + K) * w2 * B),
-        "csr2": (f * (w2 * k * B + w1 * B + w1 + w2 * k), 0),
-        "backward1": (f * (win * B + w1 * B + 2 * w1 * K + w1 * k), (2 * (K - 1) + K) * w1 * B),
+        "head": (f * (w2 * B + 4 * B * C), 0),
+        # layer 2: reads Y1 and the per-class gradient rows, writes dtheta and
+        # the per-edge input-gradient terms
+        "backward2": (f * (w1 * B + C * B + w2 * k * B + 2 * w2 * K + w2 * k), (4 * (K - 1) + K) * w2 * B),
+        # layer 1: reads the encoder bits and layer 2's per-edge terms (its
+        # output gradient, reduced through the CSR map in the kernel)
+        "backward1": (f * (win * B + w2 * k * B + 2 * w1 * K + w1 * k + w1 + w2 * k), (2 * (K - 1) + K) * w1 * B),
         "binarize": (f * (w1 * K + w2 * K) + 8 * (w1 + w2), 0),
         "pack": (B * d + f * win * W, 0),
         "hard1": (f * (win * W + w1 * W + w1 * k) + 8 * w1, (K - 1) * w1 * W),
@@ -169,9 +174,10 @@ def call_work(wl, B):
 
 
 KERNEL_OF_CALL = {
-    "encode": "encode_soft_kernel", "forward1": "lut_forward_kernel", "forward2": "lut_forward_kernel",
-    "head": "head_* (4 kernels)", "backward2": "lut_backward_kernel<k, dx>",
-    "csr2": "csr_reduce_kernel", "backward1": "lut_backward_kernel<k, no dx>",
+    "encode": "encode_soft_kernel", "forward1": "lut_forward_staged_kernel<k>",
+    "forward2": "lut_forward_staged_kernel<k>", "head": "head_* (3 kernels)",
+    "backward2": "lut_backward_node_kernel<k, dx, dY rows>",
+    "backward1": "lut_backward_node_kernel<k, no dx, CSR terms>",
     "binarize": "binarize_kernel (x2)", "pack": "pack_bits_kernel", "hard1": "hard_layer_kernel",
     "hard2": "hard_head_kernel + argmax_kernel",
 }
@@ -197,6 +203,9 @@ def run_ours(args):
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     bl.load()
     wl = synth.WORKLOADS[args.workload]
+    if args.batch:
+        wl = synth.Workload(wl.name, args.batch, wl.d, wl.classes, wl.sigma, wl.thresholds,
+                            wl.widths, wl.k, wl.tau)
     hard_only = wl.name.startswith("hard_")
     B = wl.batch
     conn1, th1, conn2, th2 = synth.network(wl, seed=0)

@@ -118,6 +118,28 @@ int bitlogic_csr_reduce(const float* edge_terms, int64_t B, const int32_t* csr_o
                         const int32_t* csr_edge, int32_t w_in, int32_t n_edges,
                         float* dX, cudaStream_t stream);
 
+/* General form of the layer backward, with the output gradient taken from
+ * one of two sources (exactly one of dY and up_terms is non-NULL):
+ *   dY rows:  node j reads row j / dy_group of dY ([w / dy_group][B]);
+ *             dy_group = 1 is an ordinary dY [w][B]; dy_group = w / C takes
+ *             the per-class gradient of bitlogic_head_loss_ex (the nodes of
+ *             a class share one gradient row), so the full dY is never stored.
+ *   up terms: dY[j][s] = sum over e in [up_off[j], up_off[j+1]) of
+ *             up_terms[up_edge[e]][s], in increasing e -- the input gradient
+ *             of the next layer (its per-edge terms and the CSR map of its
+ *             connectivity, up_edges = w_next * k_next), reduced on the fly;
+ *             the result equals bitlogic_csr_reduce of those terms bit for bit.
+ * dtheta, edge_terms as in bitlogic_lut_backward_edges (edge_terms may be
+ * NULL); dY_out (device fp32 [w][B] or NULL) receives the gradient used. */
+int bitlogic_lut_backward_ex(const float* X, int32_t w_in, int64_t B,
+                             const int32_t* conn, const float* theta,
+                             int32_t w, int32_t k,
+                             const float* dY, int32_t dy_group,
+                             const float* up_terms, const int32_t* up_off,
+                             const int32_t* up_edge, int32_t up_edges,
+                             float* dtheta, float* edge_terms, float* dY_out,
+                             cudaStream_t stream);
+
 /* Bytes of workspace bitlogic_head_loss needs. */
 size_t bitlogic_head_loss_workspace(int64_t B, int32_t C);
 
@@ -135,6 +157,15 @@ size_t bitlogic_head_loss_workspace(int64_t B, int32_t C);
 int bitlogic_head_loss(const float* Y, int32_t w, int64_t B, int32_t C, float tau,
                        const int32_t* labels, float* logits, float* loss, float* dY,
                        void* workspace, size_t ws_bytes, cudaStream_t stream);
+
+/* bitlogic_head_loss with one more optional output: dY_grouped, device fp32
+ * [C][B], row c = the gradient shared by every node of class c
+ * (dY_grouped[c][s] == dY[j][s] for every j in group c).  Either or both of
+ * dY and dY_grouped may be requested. */
+int bitlogic_head_loss_ex(const float* Y, int32_t w, int64_t B, int32_t C, float tau,
+                          const int32_t* labels, float* logits, float* loss, float* dY,
+                          float* dY_grouped, void* workspace, size_t ws_bytes,
+                          cudaStream_t stream);
 
 /* Table discretization (§3: every surrogate discretizes to a 2^n-entry
  * truth table; App. C.1 extracts it once per layer): bit a of table[j] is 1

@@ -26,7 +26,8 @@ from . import build as _build
 __all__ = [
     "BitLogicError", "load", "bitlogic_encode_thermometer", "bitlogic_lut_forward",
     "bitlogic_lut_backward_workspace", "bitlogic_lut_backward", "bitlogic_lut_backward_edges",
-    "bitlogic_csr_reduce", "bitlogic_head_loss_workspace",
+    "bitlogic_csr_reduce", "bitlogic_lut_backward_ex", "bitlogic_head_loss_ex",
+    "bitlogic_head_loss_workspace",
     "bitlogic_head_loss", "bitlogic_binarize_tables", "bitlogic_pack_bits",
     "bitlogic_hard_forward", "bitlogic_build_csr", "bitlogic_device_error",
     "bitlogic_status_string", "bitlogic_version", "LIB_PATH",
@@ -53,6 +54,10 @@ _SIGS = {
     "bitlogic_lut_backward_edges": ([_P, _I32, _I64, _P, _P, _I32, _I32, _P, _P, _P, _P],
                                     ctypes.c_int),
     "bitlogic_csr_reduce": ([_P, _I64, _P, _P, _I32, _I32, _P, _P], ctypes.c_int),
+    "bitlogic_lut_backward_ex": ([_P, _I32, _I64, _P, _P, _I32, _I32, _P, _I32, _P, _P, _P, _I32,
+                                  _P, _P, _P, _P], ctypes.c_int),
+    "bitlogic_head_loss_ex": ([_P, _I32, _I64, _I32, _F32, _P, _P, _P, _P, _P, _P, _SZ, _P],
+                              ctypes.c_int),
     "bitlogic_head_loss_workspace": ([_I64, _I32], _SZ),
     "bitlogic_head_loss": ([_P, _I32, _I64, _I32, _F32, _P, _P, _P, _P, _P, _SZ, _P],
                            ctypes.c_int),
@@ -205,6 +210,61 @@ def bitlogic_csr_reduce(edge_terms: torch.Tensor, csr_off: torch.Tensor, csr_edg
     _need(dX, "dX", torch.float32, (w_in, B))
     _check("bitlogic_csr_reduce", load().bitlogic_csr_reduce(
         _ptr(edge_terms), B, _ptr(csr_off), _ptr(csr_edge), w_in, nE, _ptr(dX), _stream(stream)))
+
+
+def bitlogic_lut_backward_ex(X: torch.Tensor, conn: torch.Tensor, theta: torch.Tensor,
+                             dtheta: torch.Tensor, dY: Optional[torch.Tensor] = None,
+                             dy_group: int = 1, up_terms: Optional[torch.Tensor] = None,
+                             up_off: Optional[torch.Tensor] = None,
+                             up_edge: Optional[torch.Tensor] = None,
+                             edge_terms: Optional[torch.Tensor] = None,
+                             dY_out: Optional[torch.Tensor] = None, stream=None):
+    w_in, B = X.shape
+    w, k = conn.shape
+    _need(X, "X", torch.float32, (w_in, B))
+    _need(conn, "conn", torch.int32, (w, k))
+    _need(theta, "theta", torch.float32, (w, 1 << k))
+    _need(dtheta, "dtheta", torch.float32, (w, 1 << k))
+    n_up = 0
+    if dY is not None:
+        if w % dy_group != 0:
+            raise ValueError("dy_group must divide w")
+        _need(dY, "dY", torch.float32, (w // dy_group, B))
+    if up_terms is not None:
+        n_up = up_terms.shape[0]
+        _need(up_terms, "up_terms", torch.float32, (n_up, B))
+        _need(up_off, "up_off", torch.int32, (w + 1,))
+        _need(up_edge, "up_edge", torch.int32, (n_up,))
+    if edge_terms is not None:
+        _need(edge_terms, "edge_terms", torch.float32, (w * k, B))
+    if dY_out is not None:
+        _need(dY_out, "dY_out", torch.float32, (w, B))
+    _check("bitlogic_lut_backward_ex", load().bitlogic_lut_backward_ex(
+        _ptr(X), w_in, B, _ptr(conn), _ptr(theta), w, k, _ptr(dY), int(dy_group),
+        _ptr(up_terms), _ptr(up_off), _ptr(up_edge), n_up, _ptr(dtheta), _ptr(edge_terms),
+        _ptr(dY_out), _stream(stream)))
+
+
+def bitlogic_head_loss_ex(Y: torch.Tensor, labels: torch.Tensor, C: int, tau: float,
+                          loss: torch.Tensor, workspace: torch.Tensor,
+                          logits: Optional[torch.Tensor] = None,
+                          dY: Optional[torch.Tensor] = None,
+                          dY_grouped: Optional[torch.Tensor] = None, stream=None):
+    w, B = Y.shape
+    _need(Y, "Y", torch.float32, (w, B))
+    _need(labels, "labels", torch.int32, (B,))
+    _need(loss, "loss", torch.float32, (1,))
+    if logits is not None:
+        _need(logits, "logits", torch.float32, (B, C))
+    if dY is not None:
+        _need(dY, "dY", torch.float32, (w, B))
+    if dY_grouped is not None:
+        _need(dY_grouped, "dY_grouped", torch.float32, (C, B))
+    if workspace is None or not workspace.is_cuda or workspace.dtype != torch.uint8:
+        raise ValueError("workspace: uint8 CUDA tensor required")
+    _check("bitlogic_head_loss_ex", load().bitlogic_head_loss_ex(
+        _ptr(Y), w, B, C, float(tau), _ptr(labels), _ptr(logits), _ptr(loss), _ptr(dY),
+        _ptr(dY_grouped), _ptr(workspace), workspace.numel(), _stream(stream)))
 
 
 def bitlogic_head_loss_workspace(B: int, C: int) -> int:

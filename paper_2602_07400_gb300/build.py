@@ -52,6 +52,8 @@ def build(force: bool = False, verbose: bool = False) -> str:
     nvcc = _nvcc()
     os.makedirs(BUILD, exist_ok=True)
     extra = ["-Xptxas", "-v"] if verbose else []
+    # optional extra nvcc flags (e.g. -D tuning constants) for experiments
+    extra += os.environ.get("BITLOGIC_NVCC_EXTRA", "").split()
 
     def compile_one(src: str):
         obj = os.path.join(BUILD, src.replace(".cu", ".o"))

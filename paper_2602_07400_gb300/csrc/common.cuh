@@ -40,6 +40,16 @@ struct Thresholds {
     uint8_t t[32];
 };
 
+// Threshold i of a by-value Thresholds with a compile-time unrolled select
+// (a runtime index into kernel parameters would copy them to local memory).
+__device__ __forceinline__ uint32_t threshold_at(const Thresholds& th, int i) {
+    uint32_t v = 0;
+#pragma unroll
+    for (int q = 0; q < 32; ++q)
+        if (q == i) v = th.t[q];
+    return v;
+}
+
 inline int make_thresholds(const uint8_t* thr_host, int32_t b, Thresholds* out) {
     if (!thr_host) return BITLOGIC_ERR_NULL;
     if (b < 1 || b > 32) return BITLOGIC_ERR_THRESH;

@@ -24,6 +24,8 @@ __global__ void __launch_bounds__(256)
 encode_soft_kernel(const uint8_t* __restrict__ x, long long B, int d, Thresholds th,
                    float* __restrict__ bits) {
     __shared__ uint8_t tile[kEncTF][kEncTS + 4];   // feature-major
+    __shared__ uint32_t sT[32];
+    if (threadIdx.x < th.b) sT[threadIdx.x] = threshold_at(th, threadIdx.x);
     const long long s0 = (long long)blockIdx.y * kEncTS;
     const int f0 = blockIdx.x * kEncTF;
     // load: thread t reads features f0 + (t % 32) of samples s0 + t/32 + 8q
@@ -45,66 +47,94 @@ encode_soft_kernel(const uint8_t* __restrict__ x, long long B, int d, Thresholds
     if (s >= B) return;
     for (int r = tr; r < rows; r += 4) {
         const int f = r / th.b, i = r - f * th.b;
-        bits[((long long)(f0 + f) * th.b + i) * B + s] = tile[f][tsl] > th.t[i] ? 1.0f : 0.0f;
+        bits[((long long)(f0 + f) * th.b + i) * B + s] = tile[f][tsl] > sT[i] ? 1.0f : 0.0f;
     }
 }
 
 // --------------------------------------------------------------- packed --
+//
+// One lane per output word (32 samples), so every store is a coalesced
+// 128-byte run of a wire row.  A block takes 1024 samples x 32 features: the
+// raw rows (32 contiguous bytes per sample) are scattered byte by byte into a
+// feature-major shared tile in which the 32 samples of word q sit in the
+// order u' = 4 (u % 8) + u / 8, so that 32-bit register r (r < 8) of the
+// lane holds samples r, r + 8, r + 16, r + 24.  For a threshold T every
+// register yields its four comparisons v > T as the high bits of its bytes
+// by byte-wise SWAR arithmetic (no carries cross a byte):
+//   T < 127:  v > T  <=>  v >= 128 or (v & 127) + (127 - T) >= 128
+//   T >= 127: v > T  <=>  v >= 128 and (v & 127) + (255 - T) >= 128
+// and shifting register r's high bits right by 7 - r puts sample
+// r + 8 j at bit r + 8 j of the word.
 
 constexpr int kPackWords = 32;             // words per tile (1024 samples)
 constexpr int kPackTS = kPackWords * 32;   // samples per tile
-constexpr int kPackTF = 8;                 // features per tile
-constexpr int kPackWarps = 8;
+constexpr int kPackTF = 32;                // features per tile
+constexpr int kPackWarps = 8;              // each warp: kPackTF / kPackWarps features
+
+__device__ __forceinline__ int pack_pos(int s) {   // tile position of sample s
+    const int u = s & 31;
+    return (s & ~31) | ((u & 7) << 2) | (u >> 3);
+}
 
 __global__ void __launch_bounds__(kPackWarps * 32)
 pack_bits_kernel(const uint8_t* __restrict__ x, long long N, int d, Thresholds th,
-                 uint32_t* __restrict__ xp, long long W, bool vec8) {
-    __shared__ __align__(16) uint8_t tile[kPackTS][kPackTF];   // sample-major, 8-byte rows
-    __shared__ uint32_t stage[kPackTF * 32][kPackWords];       // [wire in tile][word]
+                 uint32_t* __restrict__ xp, long long W, bool vec16) {
+    __shared__ __align__(16) uint8_t tile[kPackTF][kPackTS];   // feature-major, permuted samples
+    __shared__ uint32_t sC[32], sOr[32];   // per-threshold SWAR constants
+    if (threadIdx.x < th.b) {
+        const uint32_t T = threshold_at(th, threadIdx.x);
+        // T == 255: nothing exceeds it (C = 0, AND form: the sum never reaches 128)
+        sC[threadIdx.x] = (T < 127u ? 127u - T : 255u - T) * 0x01010101u;
+        sOr[threadIdx.x] = T < 127u ? 0x80808080u : 0u;
+    }
     const long long s0 = (long long)blockIdx.y * kPackTS;
     const int f0 = blockIdx.x * kPackTF;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nf = min(kPackTF, d - f0);
-    // load 1024 samples x 8 features
+    // fill: thread t takes samples t, t + 256, ...; 32 feature bytes each
     for (int sl = threadIdx.x; sl < kPackTS; sl += kPackWarps * 32) {
         const long long s = s0 + sl;
-        uint2 v = make_uint2(0u, 0u);
+        uint32_t v[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) v[q] = 0u;
         if (s < N) {
             const uint8_t* p = x + s * d + f0;
-            if (vec8 && nf == kPackTF) {
-                v = __ldg(reinterpret_cast<const uint2*>(p));
+            if (vec16 && nf == kPackTF) {
+                const uint4 a = __ldg(reinterpret_cast<const uint4*>(p));
+                const uint4 b = __ldg(reinterpret_cast<const uint4*>(p) + 1);
+                v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+                v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
             } else {
-                uint8_t b8[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-                for (int f = 0; f < nf; ++f) b8[f] = __ldg(p + f);
-                v.x = b8[0] | (b8[1] << 8) | (b8[2] << 16) | ((uint32_t)b8[3] << 24);
-                v.y = b8[4] | (b8[5] << 8) | (b8[6] << 16) | ((uint32_t)b8[7] << 24);
-            }
-        }
-        *reinterpret_cast<uint2*>(&tile[sl][0]) = v;
-    }
-    __syncthreads();
-    // each warp builds 4 words: lane = sample bit, one ballot per wire
 #pragma unroll
-    for (int u = 0; u < kPackWords / kPackWarps; ++u) {
-        const int q = warp * (kPackWords / kPackWarps) + u;
-        const uint2 v = *reinterpret_cast<const uint2*>(&tile[q * 32 + lane][0]);
-        for (int f = 0; f < nf; ++f) {
-            const uint32_t byte = ((f < 4 ? v.x : v.y) >> (8 * (f & 3))) & 0xffu;
-            for (int i = 0; i < th.b; ++i) {
-                const uint32_t word = __ballot_sync(0xffffffffu, byte > th.t[i]);
-                if (lane == 0) stage[f * th.b + i][q] = word;
+                for (int f = 0; f < kPackTF; ++f)
+                    if (f < nf) v[f >> 2] |= (uint32_t)__ldg(p + f) << (8 * (f & 3));
             }
         }
+        const int pos = pack_pos(sl);
+#pragma unroll
+        for (int f = 0; f < kPackTF; ++f) tile[f][pos] = (uint8_t)(v[f >> 2] >> (8 * (f & 3)));
     }
     __syncthreads();
-    // coalesced store: one 128-byte row segment per warp step
-    const long long q0 = (long long)blockIdx.y * kPackWords;
-    const int rows = nf * th.b;
-    for (int r = warp; r < rows; r += kPackWarps) {
-        const long long q = q0 + lane;
-        if (q < W) {
-            const int f = r / th.b, i = r - f * th.b;
-            xp[((long long)(f0 + f) * th.b + i) * W + q] = stage[r][lane];
+    const long long q = (long long)blockIdx.y * kPackWords + lane;   // this lane's word
+    if (q >= W) return;
+    for (int fl = warp; fl < nf; fl += kPackWarps) {
+        const uint4 a = *reinterpret_cast<const uint4*>(&tile[fl][32 * lane]);
+        const uint4 b = *reinterpret_cast<const uint4*>(&tile[fl][32 * lane + 16]);
+        const uint32_t r[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+        uint32_t lo7[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) lo7[i] = r[i] & 0x7f7f7f7fu;
+        uint32_t* out = xp + (long long)(f0 + fl) * th.b * W + q;
+        for (int i = 0; i < th.b; ++i) {
+            const uint32_t C = sC[i], orm = sOr[i];   // OR form below 127, AND form above
+            uint32_t word = 0u;
+#pragma unroll
+            for (int i8 = 0; i8 < 8; ++i8) {
+                const uint32_t sum = lo7[i8] + C;
+                const uint32_t hb = (r[i8] & sum) | ((r[i8] | sum) & orm);
+                word |= (hb >> (7 - i8)) & (0x01010101u << i8);
+            }
+            out[(long long)i * W] = word;
         }
     }
 }
@@ -144,8 +174,8 @@ extern "C" int bitlogic_pack_bits(const uint8_t* x, int64_t N, int32_t d,
     const long long W = (N + 31) / 32;
     const long long gy = (N + kPackTS - 1) / kPackTS;
     if (gy > 65535) return BITLOGIC_ERR_SHAPE;
-    const bool vec8 = (d % 8 == 0) && ((reinterpret_cast<uintptr_t>(x) & 7u) == 0);
+    const bool vec16 = (d % 16 == 0) && aligned16(x);
     dim3 grid((unsigned)((d + kPackTF - 1) / kPackTF), (unsigned)gy);
-    pack_bits_kernel<<<grid, kPackWarps * 32, 0, stream>>>(x, N, d, th, xp, W, vec8);
+    pack_bits_kernel<<<grid, kPackWarps * 32, 0, stream>>>(x, N, d, th, xp, W, vec16);
     return launch_status();
 }

@@ -60,7 +60,7 @@ constexpr int kSoftWarps = 8;
 __global__ void __launch_bounds__(kSoftWarps * 32)
 head_softmax_kernel(const float* __restrict__ logits, long long B, int C,
                     const int* __restrict__ labels, float* __restrict__ dlogit,
-                    float* __restrict__ per_sample) {
+                    float* __restrict__ per_sample, float tau, float* __restrict__ dYg) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const long long s = (long long)blockIdx.x * kSoftWarps + warp;
     if (s >= B) return;
@@ -81,7 +81,9 @@ head_softmax_kernel(const float* __restrict__ logits, long long B, int C,
     const float invB = 1.0f / (float)B;
     for (int c = lane; c < C; c += 32) {
         const float p = expf(l[c] - lse);
-        dlogit[s * C + c] = (p - (c == lab ? 1.0f : 0.0f)) * invB;
+        const float dl = (p - (c == lab ? 1.0f : 0.0f)) * invB;
+        dlogit[s * C + c] = dl;
+        if (dYg) dYg[(long long)c * B + s] = dl / tau;   // the gradient of every node of class c
     }
 }
 
@@ -143,14 +145,18 @@ extern "C" size_t bitlogic_head_loss_workspace(int64_t B, int32_t C) {
     return align_up(bc) + align_up((size_t)B * sizeof(float)) + align_up(bc);
 }
 
-extern "C" int bitlogic_head_loss(const float* Y, int32_t w, int64_t B, int32_t C, float tau,
-                                  const int32_t* labels, float* logits, float* loss, float* dY,
-                                  void* workspace, size_t ws_bytes, cudaStream_t stream) {
+extern "C" int bitlogic_head_loss_ex(const float* Y, int32_t w, int64_t B, int32_t C, float tau,
+                                     const int32_t* labels, float* logits, float* loss, float* dY,
+                                     float* dY_grouped, void* workspace, size_t ws_bytes,
+                                     cudaStream_t stream) {
     if (!Y || !labels || !loss || !workspace) return BITLOGIC_ERR_NULL;
     if (w <= 0 || B <= 0 || C <= 0 || w % C != 0 || !(tau > 0.f)) return BITLOGIC_ERR_SHAPE;
     if (B > 0x7fffffffLL / (C > 0 ? C : 1)) return BITLOGIC_ERR_SHAPE;
     if (!aligned16(workspace)) return BITLOGIC_ERR_ALIGN;
     if (ws_bytes < bitlogic_head_loss_workspace(B, C)) return BITLOGIC_ERR_WORKSPACE;
+    const long long sb = (B + 31) / 32;
+    const long long gy = (B + kDyThreads - 1) / kDyThreads;
+    if (sb > 65535 || gy > 65535) return BITLOGIC_ERR_SHAPE;
     const int g = w / C;
     char* ws = static_cast<char*>(workspace);
     const size_t bc = (size_t)B * (size_t)C * sizeof(float);
@@ -158,17 +164,19 @@ extern "C" int bitlogic_head_loss(const float* Y, int32_t w, int64_t B, int32_t 
     float* per = reinterpret_cast<float*>(ws + align_up(bc));
     float* lg = logits ? logits : reinterpret_cast<float*>(ws + align_up(bc) + align_up((size_t)B * 4));
 
-    const long long sb = (B + 31) / 32;
-    if (sb > 65535) return BITLOGIC_ERR_SHAPE;
     head_group_sum_kernel<<<dim3((unsigned)C, (unsigned)sb), kSumWarps * 32, 0, stream>>>(Y, B, C, g, tau, lg);
     head_softmax_kernel<<<(unsigned)((B + kSoftWarps - 1) / kSoftWarps), kSoftWarps * 32, 0, stream>>>(
-        lg, B, C, labels, dlogit, per);
-    if (dY) {
-        const long long gy = (B + kDyThreads - 1) / kDyThreads;
-        if (gy > 65535) return BITLOGIC_ERR_SHAPE;
+        lg, B, C, labels, dlogit, per, tau, dY_grouped);
+    if (dY)
         head_dy_kernel<<<dim3((unsigned)((w + kDyRows - 1) / kDyRows), (unsigned)gy), kDyThreads, 0, stream>>>(
             dlogit, B, C, g, w, tau, dY);
-    }
     head_mean_kernel<<<1, 256, 0, stream>>>(per, B, loss);
     return launch_status();
+}
+
+extern "C" int bitlogic_head_loss(const float* Y, int32_t w, int64_t B, int32_t C, float tau,
+                                  const int32_t* labels, float* logits, float* loss, float* dY,
+                                  void* workspace, size_t ws_bytes, cudaStream_t stream) {
+    return bitlogic_head_loss_ex(Y, w, B, C, tau, labels, logits, loss, dY, nullptr, workspace,
+                                 ws_bytes, stream);
 }

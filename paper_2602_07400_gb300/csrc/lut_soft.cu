@@ -12,16 +12,26 @@
 // down (two FMULs per lerp), each lerp adds adjoint * (hi - lo) into dx_l, and
 // at the leaves the adjoint is g * w_a, accumulated for dtheta.
 //
-// Work split: one warp per node, lanes over samples (batch-contiguous rows,
-// so every gathered row segment is a coalesced 128/512-byte access).  The
-// table lives in registers for the whole sweep of the node.
+// Data movement: activations are feature-major [rows][B], so the k rows a
+// node gathers are contiguous batch segments.  The vector paths stream them
+// through a ring of shared-memory stages filled by 16-byte cp.async copies,
+// which overlaps the gathers with the trees of earlier stages without
+// spending registers.
 #include "common.cuh"
 
 namespace bitlogic {
 namespace {
 
+#ifndef BITLOGIC_BWD_MIN_BLOCKS
+#define BITLOGIC_BWD_MIN_BLOCKS 4
+#endif
 constexpr int kFwdWarps = 4;
-constexpr int kBwdWarps = 4;
+constexpr int kBwdWarps = 4;   // warps per block in the staged backward
+#ifndef BITLOGIC_BWD_WARPS_PER_NODE
+#define BITLOGIC_BWD_WARPS_PER_NODE 2
+#endif
+constexpr int kWarpsPerNode = BITLOGIC_BWD_WARPS_PER_NODE;   // 1, 2 or 4
+constexpr int kNodesPerBlock = kBwdWarps / kWarpsPerNode;
 constexpr int kCsrWarps = 8;
 
 // ---------------------------------------------------------------- trees --
@@ -38,13 +48,17 @@ __device__ __forceinline__ float fwd_tree(const float (&te)[H], const float (&d)
     }
 }
 
-// Returns the subtree value; `adj` is the adjoint of this subtree's output.
+// Reverse tree of the subtree at level L, index M; `adj` is the adjoint of
+// its output.  Returns the subtree value, adds adjoint * (hi - lo) into
+// dx[l] for each lerp at level l (the lerp with M == 0 is the first to touch
+// dx[l] and initialises it), and the leaf adjoints into acc.
 template <int L, int M, int H, int K, int k>
 __device__ __forceinline__ float bwd_tree(const float (&te)[H], const float (&d)[H],
                                           const float (&x)[k], const float (&omx)[k],
                                           float adj, float (&dx)[k], float (&acc)[K]) {
     if constexpr (L == 0) {
-        dx[0] = fmaf(adj, d[M], dx[0]);
+        if constexpr (M == 0) dx[0] = adj * d[M];
+        else dx[0] = fmaf(adj, d[M], dx[0]);
         acc[2 * M] = fmaf(adj, omx[0], acc[2 * M]);
         acc[2 * M + 1] = fmaf(adj, x[0], acc[2 * M + 1]);
         return fmaf(x[0], d[M], te[M]);
@@ -52,8 +66,90 @@ __device__ __forceinline__ float bwd_tree(const float (&te)[H], const float (&d)
         const float lo = bwd_tree<L - 1, 2 * M>(te, d, x, omx, adj * omx[L], dx, acc);
         const float hi = bwd_tree<L - 1, 2 * M + 1>(te, d, x, omx, adj * x[L], dx, acc);
         const float diff = hi - lo;
-        dx[L] = fmaf(adj, diff, dx[L]);
+        if constexpr (M == 0) dx[L] = adj * diff;
+        else dx[L] = fmaf(adj, diff, dx[L]);
         return fmaf(x[L], diff, lo);
+    }
+}
+
+// ------------------------------------------- subtable polynomial forms --
+//
+// A subtable of 2^L consecutive table entries over x_0..x_{L-1} is the
+// multilinear polynomial sum_S c_S prod_{i in S} x_i whose coefficients are
+// the subset differences (Moebius transform) of its entries.  Evaluated by
+// Horner steps it costs 2^L - 1 FFMA, against 2^L - 1 lerps (about twice the
+// instructions) for the same subtable as a lerp tree.  The upper levels stay
+// lerps.  |c_S| <= 2^(L-1), so rounding stays at a few ulp of 1.
+
+// In-place subset-difference transform of 2^L values.
+template <int L>
+__device__ __forceinline__ void moebius(float (&c)[1 << L]) {
+#pragma unroll
+    for (int b = 0; b < L; ++b)
+#pragma unroll
+        for (int a = 0; a < (1 << L); ++a)
+            if (a & (1 << b)) c[a] -= c[a ^ (1 << b)];
+}
+
+// Horner value of the subtable whose coefficients start at cf[O].
+template <int L, int O, int N, int k>
+__device__ __forceinline__ float poly(const float (&cf)[N], const float (&x)[k]) {
+    if constexpr (L == 1) {
+        return fmaf(cf[O + 1], x[0], cf[O]);
+    } else {
+        const float lo = poly<L - 1, O>(cf, x);
+        const float hi = poly<L - 1, O + (1 << (L - 1))>(cf, x);
+        return fmaf(x[L - 1], hi, lo);
+    }
+}
+
+// Forward tree with Moebius subtables of 2^L entries at the bottom: value of
+// the subtree at level LV (levels below L are inside the subtables).
+template <int LV, int M, int L, int N, int k>
+__device__ __forceinline__ float fwd_tree_poly(const float (&cf)[N], const float (&x)[k]) {
+    if constexpr (LV == L - 1) {
+        return poly<L, M * (1 << L)>(cf, x);
+    } else {
+        const float lo = fwd_tree_poly<LV - 1, 2 * M, L>(cf, x);
+        const float hi = fwd_tree_poly<LV - 1, 2 * M + 1, L>(cf, x);
+        return fmaf(x[LV], hi - lo, lo);
+    }
+}
+
+__host__ __device__ constexpr int fwd_poly_levels(int k) { return k < 3 ? k : 3; }
+
+// Reverse tree whose leaves are 4-entry subtables in Moebius form over
+// (x_0, x_1): quad m has coefficients cq[4m .. 4m+3] = (c0, c1, c2, c3),
+// value v = (c0 + c1 x0) + x1 (c2 + c3 x0), dv/dx0 = c1 + c3 x1,
+// dv/dx1 = c2 + c3 x0, and entry a of the quad has corner weight W[a]
+// (W = ((1-x0)(1-x1), x0(1-x1), (1-x0)x1, x0 x1), shared by all quads), so
+// its leaf adjoint is adj * W[a].  Above the quads the lerps of bwd_tree.
+template <int LV, int M, int N, int NA, int k>
+__device__ __forceinline__ float bwd_tree_quad(const float (&cq)[N], const float (&x)[k],
+                                               const float (&omx)[k], const float (&W)[4],
+                                               float adj, float (&dx)[k], float (&acc)[NA]) {
+    if constexpr (LV == 1) {
+        const float c0 = cq[4 * M], c1 = cq[4 * M + 1], c2 = cq[4 * M + 2], c3 = cq[4 * M + 3];
+        const float in0 = fmaf(c1, x[0], c0);
+        const float in1 = fmaf(c3, x[0], c2);
+        const float dv0 = fmaf(c3, x[1], c1);
+        if constexpr (M == 0) {
+            dx[0] = adj * dv0;
+            dx[1] = adj * in1;
+        } else {
+            dx[0] = fmaf(adj, dv0, dx[0]);
+            dx[1] = fmaf(adj, in1, dx[1]);
+        }
+#pragma unroll
+        for (int a = 0; a < 4; ++a) acc[4 * M + a] = fmaf(adj, W[a], acc[4 * M + a]);
+        return fmaf(x[1], in1, in0);
+    } else {
+        const float lo = bwd_tree_quad<LV - 1, 2 * M>(cq, x, omx, W, adj * omx[LV], dx, acc);
+        const float hi = bwd_tree_quad<LV - 1, 2 * M + 1>(cq, x, omx, W, adj * x[LV], dx, acc);
+        const float diff = hi - lo;
+        if constexpr (M == 0) dx[LV] = adj * diff;
+        else dx[LV] = fmaf(adj, diff, dx[LV]);
+        return fmaf(x[LV], diff, lo);
     }
 }
 
@@ -63,6 +159,24 @@ __device__ __forceinline__ float comp(const float4& v, int c) {
 
 __device__ __forceinline__ float4 ldg4(const float* p) {
     return __ldg(reinterpret_cast<const float4*>(p));
+}
+
+__device__ __forceinline__ float4 add4(float4 a, const float4& b) {
+    a.x += b.x; a.y += b.y; a.z += b.z; a.w += b.w;
+    return a;
+}
+
+template <int k>
+__device__ __forceinline__ void load_rows(const int* __restrict__ conn, int j, int w_in, int lane,
+                                          int (&rows)[k]) {
+    bool bad = false;
+#pragma unroll
+    for (int i = 0; i < k; ++i) {
+        int c = __ldg(conn + (long long)j * k + i);
+        if ((unsigned)c >= (unsigned)w_in) { bad = true; c = 0; }
+        rows[i] = c;
+    }
+    if (bad && lane == 0) flag_index_error();
 }
 
 // Per-warp node set-up: connectivity rows (range-checked), sigmoid of the
@@ -76,14 +190,7 @@ __device__ __forceinline__ void node_setup(const int* __restrict__ conn,
                                            float (&te)[1 << (k - 1)], float (&d)[1 << (k - 1)],
                                            float& t0, float& t1) {
     constexpr int K = 1 << k, H = K / 2;
-    bool bad = false;
-#pragma unroll
-    for (int i = 0; i < k; ++i) {
-        int c = __ldg(conn + (long long)j * k + i);
-        if ((unsigned)c >= (unsigned)w_in) { bad = true; c = 0; }
-        rows[i] = c;
-    }
-    if (bad && lane == 0) flag_index_error();
+    load_rows<k>(conn, j, w_in, lane, rows);
     t0 = t1 = 0.f;
     if (lane < H) {
         t0 = sigmoidf(__ldg(theta + (long long)j * K + 2 * lane));
@@ -111,12 +218,20 @@ __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commi
 template <int N>
 __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
 
-constexpr int kStageSamples = 128;   // samples per pipeline stage
-constexpr int kStages = 3;           // stages in flight per warp
+#ifndef BITLOGIC_STAGE_SAMPLES
+#define BITLOGIC_STAGE_SAMPLES 128
+#endif
+#ifndef BITLOGIC_STAGES
+#define BITLOGIC_STAGES 3
+#endif
+constexpr int kStageSamples = BITLOGIC_STAGE_SAMPLES;   // samples per pipeline stage
+constexpr int kStages = BITLOGIC_STAGES;                // stages in flight per warp
 
 // ------------------------------------------------------------- forward --
 
-template <int k, bool VEC>
+// Scalar forward (any B, any alignment): one warp per (node, batch slice),
+// one sample per lane.
+template <int k>
 __global__ void __launch_bounds__(kFwdWarps * 32)
 lut_forward_kernel(const float* __restrict__ X, int w_in, long long B,
                    const int* __restrict__ conn, const float* __restrict__ theta, int w,
@@ -129,60 +244,53 @@ lut_forward_kernel(const float* __restrict__ X, int w_in, long long B,
     int rows[k];
     float te[H], d[H], t0, t1;
     node_setup<k>(conn, theta, j, w_in, lane, sPair[warp], rows, te, d, t0, t1);
-
     const long long s0 = (long long)blockIdx.y * chunk;
     const long long s1 = min(B, s0 + chunk);
     const float* xr[k];
 #pragma unroll
     for (int i = 0; i < k; ++i) xr[i] = X + (long long)rows[i] * B;
     float* yr = Y + (long long)j * B;
-
-    if constexpr (VEC) {
-        // B % 4 == 0 and chunk % 4 == 0: every float4 is in range
-        for (long long s = s0 + 4 * lane; s < s1; s += 128) {
-            float4 xv[k];
+    for (long long s = s0 + lane; s < s1; s += 32) {
+        float x[k];
 #pragma unroll
-            for (int i = 0; i < k; ++i) xv[i] = ldg4(xr[i] + s);
-            float o[4];
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                float x[k];
-#pragma unroll
-                for (int i = 0; i < k; ++i) x[i] = comp(xv[i], c);
-                o[c] = fwd_tree<k - 1, 0>(te, d, x);
-            }
-            *reinterpret_cast<float4*>(yr + s) = make_float4(o[0], o[1], o[2], o[3]);
-        }
-    } else {
-        for (long long s = s0 + lane; s < s1; s += 32) {
-            float x[k];
-#pragma unroll
-            for (int i = 0; i < k; ++i) x[i] = __ldg(xr[i] + s);
-            yr[s] = fwd_tree<k - 1, 0>(te, d, x);
-        }
+        for (int i = 0; i < k; ++i) x[i] = __ldg(xr[i] + s);
+        yr[s] = fwd_tree<k - 1, 0>(te, d, x);
     }
 }
 
-// Forward with the k gathered input rows streamed through a ring of
-// shared-memory stages (cp.async).  Each lane copies, reads back and
-// evaluates its own 4 consecutive samples of a stage (16-byte chunks), so
-// the ring needs no warp synchronisation.  The block's y index selects a
-// batch slice (see forward_chunk).  Needs B % 4 == 0, chunk % 4 == 0 and
-// 16-byte aligned X and Y.
+// Staged forward: one warp per (node, batch slice).  Each lane copies, reads
+// back and evaluates its own 4 consecutive samples of a stage (16-byte
+// chunks), so the ring needs no warp synchronisation.  Needs B % 4 == 0,
+// chunk % 4 == 0 and 16-byte aligned X and Y.
 template <int k>
 __global__ void __launch_bounds__(kFwdWarps * 32)
 lut_forward_staged_kernel(const float* __restrict__ X, int w_in, long long B,
                           const int* __restrict__ conn, const float* __restrict__ theta, int w,
                           float* __restrict__ Y, long long chunk) {
-    constexpr int H = 1 << (k - 1), CH = kStageSamples;
+    constexpr int K = 1 << k, CH = kStageSamples, L = fwd_poly_levels(k), S = 1 << L;
     __shared__ __align__(16) float sRing[kFwdWarps][kStages * k * CH];
-    __shared__ float2 sPair[kFwdWarps][H];
+    __shared__ __align__(16) float sCoef[kFwdWarps][K];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int j = blockIdx.x * kFwdWarps + warp;
     if (j >= w) return;
     int rows[k];
-    float te[H], d[H], t0, t1;
-    node_setup<k>(conn, theta, j, w_in, lane, sPair[warp], rows, te, d, t0, t1);
+    load_rows<k>(conn, j, w_in, lane, rows);
+    // lane l < K / S: sigmoid of subtable l's entries, then its coefficients
+    if (lane < K / S) {
+        float c[S];
+#pragma unroll
+        for (int a = 0; a < S; ++a) c[a] = sigmoidf(__ldg(theta + (long long)j * K + lane * S + a));
+        moebius<L>(c);
+#pragma unroll
+        for (int a = 0; a < S; ++a) sCoef[warp][lane * S + a] = c[a];
+    }
+    __syncwarp();
+    float cf[K];
+#pragma unroll
+    for (int a = 0; a < K; a += 4) {
+        const float4 v = *reinterpret_cast<const float4*>(&sCoef[warp][a]);
+        cf[a] = v.x; cf[a + 1] = v.y; cf[a + 2] = v.z; cf[a + 3] = v.w;
+    }
     float* ring = sRing[warp] + 4 * lane;       // this lane's column of every stage row
     const long long s0 = (long long)blockIdx.y * chunk;
     const long long s1 = min(B, s0 + chunk);
@@ -220,7 +328,7 @@ lut_forward_staged_kernel(const float* __restrict__ X, int w_in, long long B,
                 float x[k];
 #pragma unroll
                 for (int i = 0; i < k; ++i) x[i] = comp(xv[i], c);
-                o[c] = fwd_tree<k - 1, 0>(te, d, x);
+                o[c] = fwd_tree_poly<k - 1, 0, L>(cf, x);
             }
             *reinterpret_cast<float4*>(yr + (long long)st * CH) = make_float4(o[0], o[1], o[2], o[3]);
         }
@@ -231,36 +339,77 @@ lut_forward_staged_kernel(const float* __restrict__ X, int w_in, long long B,
 
 // ------------------------------------------------------------ backward --
 
-template <int k, bool WANT_DX>
-__global__ void __launch_bounds__(kBwdWarps * 32)
+// Where a node's output gradient dY[j][.] comes from.
+//   rows:  dY + (j / group) * B   (group = 1: one row per node; group = g:
+//          the head's per-class gradient, shared by the g nodes of a class)
+//   terms: sum over e in [off[j], off[j+1]) of terms[edge[e]][.] in
+//          increasing e -- the next layer's input gradient, reduced on the
+//          fly from its per-edge terms instead of being materialised
+struct GradSource {
+    const float* dY;
+    int group;
+    const float* terms;
+    const int* off;
+    const int* edge;
+    int n_edges;
+};
+
+// CSR range of node j in the upstream terms (range-checked).
+__device__ __forceinline__ void term_range(const GradSource& gs, int j, int lane, int& e0, int& e1) {
+    e0 = __ldg(gs.off + j);
+    e1 = __ldg(gs.off + j + 1);
+    if (e0 < 0 || e1 < e0 || e1 > gs.n_edges) {
+        if (lane == 0) flag_index_error();
+        e0 = e1 = 0;
+    }
+}
+
+// Scalar backward (any B, any alignment, any k): one warp per node, one
+// sample per lane, next sample's gathers issued before this sample's tree.
+template <int k, bool WANT_DX, bool TERMS>
+__global__ void __launch_bounds__(kFwdWarps * 32)
 lut_backward_kernel(const float* __restrict__ X, int w_in, long long B,
                     const int* __restrict__ conn, const float* __restrict__ theta, int w,
-                    const float* __restrict__ dY, float* __restrict__ dtheta,
-                    float* __restrict__ P) {
+                    GradSource gs, float* __restrict__ dtheta, float* __restrict__ P,
+                    float* __restrict__ dY_out) {
     constexpr int K = 1 << k, H = K / 2;
-    __shared__ float2 sPair[kBwdWarps][H];
-    __shared__ float sRed[kBwdWarps][32][K + 1];
+    __shared__ float2 sPair[kFwdWarps][H];
+    __shared__ float sRed[kFwdWarps][32][K + 1];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int j = blockIdx.x * kBwdWarps + warp;
+    const int j = blockIdx.x * kFwdWarps + warp;
     if (j >= w) return;
     int rows[k];
     float te[H], d[H], t0, t1;
     node_setup<k>(conn, theta, j, w_in, lane, sPair[warp], rows, te, d, t0, t1);
+    int e0 = 0, e1 = 0;
+    if constexpr (TERMS) term_range(gs, j, lane, e0, e1);
+    const float* gr = TERMS ? nullptr : gs.dY + (long long)(j / gs.group) * B;
+    float* pr = P + (long long)j * k * B;
 
-    const float* gr = dY + (long long)j * B;
-    float* pr = P + (long long)j * k * B;   // rows j*k + i of the per-edge terms
+    auto grad = [&](long long s) {
+        if constexpr (TERMS) {
+            float g = 0.f;
+            for (int e = e0; e < e1; ++e) {
+                const int id = __ldg(gs.edge + e);
+                if ((unsigned)id < (unsigned)gs.n_edges) g += __ldg(gs.terms + (long long)id * B + s);
+                else if (lane == 0) flag_index_error();
+            }
+            return g;
+        } else {
+            return __ldg(gr + s);
+        }
+    };
 
     float acc[K];
 #pragma unroll
     for (int a = 0; a < K; ++a) acc[a] = 0.f;
-
-    // one sample per lane per step (coalesced 128-byte rows), with the next
-    // step's gathers issued before this step's tree
     float xn[k], gn = 0.f;
+#pragma unroll
+    for (int i = 0; i < k; ++i) xn[i] = 0.f;
     if (lane < B) {
 #pragma unroll
         for (int i = 0; i < k; ++i) xn[i] = __ldg(X + (long long)rows[i] * B + lane);
-        gn = __ldg(gr + lane);
+        gn = grad(lane);
     }
     for (long long s = lane; s < B; s += 32) {
         float x[k], omx[k], dx[k];
@@ -269,22 +418,19 @@ lut_backward_kernel(const float* __restrict__ X, int w_in, long long B,
         for (int i = 0; i < k; ++i) {
             x[i] = xn[i];
             omx[i] = 1.0f - x[i];
-            dx[i] = 0.f;
         }
         if (s + 32 < B) {
 #pragma unroll
             for (int i = 0; i < k; ++i) xn[i] = __ldg(X + (long long)rows[i] * B + s + 32);
-            gn = __ldg(gr + s + 32);
+            gn = grad(s + 32);
         }
+        if (dY_out) dY_out[(long long)j * B + s] = g;
         bwd_tree<k - 1, 0>(te, d, x, omx, g, dx, acc);
         if constexpr (WANT_DX) {
 #pragma unroll
             for (int i = 0; i < k; ++i) pr[(long long)i * B + s] = dx[i];
         }
     }
-
-    // dtheta: sum the per-lane partials over the 32 lanes in lane order
-    // (transpose through shared memory), then scale by t (1 - t).
 #pragma unroll
     for (int a = 0; a < K; ++a) sRed[warp][lane][a] = acc[a];
     __syncwarp();
@@ -301,92 +447,186 @@ lut_backward_kernel(const float* __restrict__ X, int w_in, long long B,
     }
 }
 
-// ---------------------------------------- backward, shared-memory staged --
+// ---------------------------------------- backward, one block per node --
 
-template <int k>
-__host__ __device__ constexpr int staged_floats_per_warp() {
-    constexpr int rows = kStages * (k + 1) * kStageSamples;
+constexpr int kGatherStages = 4;   // stages whose upstream rows are gathered together
+
+// Per-warp shared memory of the staged backward: the cp.async ring (k input
+// rows, plus the gradient row for a dY source) and, for a CSR-terms source,
+// the summed gradient of kGatherStages stages; reused for the dtheta
+// transpose at the end.
+template <int k, bool TERMS>
+__host__ __device__ constexpr int ring_floats() {
+    return kStages * (TERMS ? k : k + 1) * kStageSamples;
+}
+template <int k, bool TERMS>
+__host__ __device__ constexpr int node_floats_per_warp() {
+    constexpr int rows = ring_floats<k, TERMS>() + (TERMS ? kGatherStages * kStageSamples : 0);
     constexpr int red = 32 * ((1 << (k - 1)) + 1);
     return rows > red ? rows : red;
 }
 
-template <int k>
-constexpr size_t staged_smem_bytes() {
-    return (size_t)kBwdWarps * staged_floats_per_warp<k>() * sizeof(float) +
-           (size_t)kBwdWarps * (1 << (k - 1)) * sizeof(float2);
+template <int k, bool TERMS>
+constexpr size_t node_smem_bytes() {
+    return (size_t)kBwdWarps * node_floats_per_warp<k, TERMS>() * sizeof(float) +
+           (size_t)kNodesPerBlock * (1 << k) * sizeof(float);
 }
 
-// Backward with two lanes per sample: lane h = lane & 1 owns the half of
-// the table whose top input x_{k-1} equals h, i.e. one of the two subtrees
-// under the root lerp.  Each lane runs the reverse tree of its subtree
-// (adjoint g * (h ? x_{k-1} : 1 - x_{k-1})), accumulates the leaf adjoints of
-// its half for dtheta, and the pair exchanges three values by shuffle: the
-// partial dx_i of the slots the partner stores, and the subtree value that
-// gives dx_{k-1} = g * (v_1 - v_0).  Lane h stores the slots i with
+// Staged backward.  A block holds kNodesPerBlock nodes with kWarpsPerNode
+// warps each; each warp of a node takes a contiguous range of its 128-sample
+// stages.
+//
+// Within a warp every sample is split over two lanes: lane h = lane & 1 owns
+// the half of the table whose top input x_{k-1} equals h, i.e. one of the two
+// subtrees under the root lerp.  Each lane runs the reverse tree of its
+// subtree (adjoint g * (h ? x_{k-1} : 1 - x_{k-1})) and accumulates the leaf
+// adjoints of its half for dtheta; the pair exchanges one value per stored
+// slot by shuffle (the partner's partial dx_i, or the subtree value that
+// gives dx_{k-1} = g * (v_1 - v_0)).  Lane h stores the slots i with
 // i % 2 == h.  Halving the per-thread table and accumulators doubles the
-// resident warps.  The k gathered rows and the dY row stream through a
-// kStages-deep cp.async ring as 16-byte chunks (each lane copies one chunk
-// per row; the pair partners read them after a warp sync).  Needs k >= 2,
-// B % 4 == 0 and 16-byte aligned X and dY.
-template <int k, bool WANT_DX>
-__global__ void __launch_bounds__(kBwdWarps * 32)
-lut_backward_staged_kernel(const float* __restrict__ X, int w_in, long long B,
-                           const int* __restrict__ conn, const float* __restrict__ theta, int w,
-                           const float* __restrict__ dY, float* __restrict__ dtheta,
-                           float* __restrict__ P) {
+// resident warps.
+//
+// The k gathered rows (and, for a dY source, the node's gradient row) stream
+// through a kStages-deep cp.async ring.  For a CSR-terms source the node's
+// edge ids are read once into lanes; every kGatherStages stages the warp
+// sums the upstream rows in increasing edge order, 2 KB contiguous per row
+// (random rows in DRAM want long contiguous reads), into a shared buffer the
+// stages then read.  dtheta: each lane's partials, then the lanes of each
+// parity, then the node's warps, in a fixed order.  Needs k >= 2,
+// B % 4 == 0 and 16-byte aligned X and sources.
+template <int k, bool WANT_DX, bool TERMS>
+__global__ void __launch_bounds__(kBwdWarps * 32, BITLOGIC_BWD_MIN_BLOCKS)
+lut_backward_node_kernel(const float* __restrict__ X, int w_in, long long B,
+                         const int* __restrict__ conn, const float* __restrict__ theta, int w,
+                         GradSource gs, float* __restrict__ dtheta, float* __restrict__ P,
+                         float* __restrict__ dY_out) {
     constexpr int K = 1 << k, H = K / 2, H2 = K / 4, R = k + 1, CH = kStageSamples;
     constexpr int NQ = (k + 1) / 2;   // slots stored per lane (rounded up)
     extern __shared__ __align__(16) float smem[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int h = lane & 1, pair = lane >> 1;
-    float* ring = smem + warp * staged_floats_per_warp<k>();
-    float2* sPair = reinterpret_cast<float2*>(smem + kBwdWarps * staged_floats_per_warp<k>()) + warp * H;
-    const int j = blockIdx.x * kBwdWarps + warp;
-    if (j >= w) return;
+    const int nb = warp / kWarpsPerNode, sub = warp % kWarpsPerNode;   // node in block, warp in node
+    constexpr int FPW = node_floats_per_warp<k, TERMS>();
+    float* ring = smem + warp * FPW;
+    float* gbuf = ring + ring_floats<k, TERMS>();   // summed upstream gradient (terms source)
+    float* sT = smem + kBwdWarps * FPW + nb * K;   // sigmoid of the node's logits
+    const int j = blockIdx.x * kNodesPerBlock + nb;
+    const bool live = j < w;   // a dead warp still reaches the block barriers
 
     int rows[k];
-    bool bad = false;
 #pragma unroll
-    for (int i = 0; i < k; ++i) {
-        int c = __ldg(conn + (long long)j * k + i);
-        if ((unsigned)c >= (unsigned)w_in) { bad = true; c = 0; }
-        rows[i] = c;
-    }
-    if (bad && lane == 0) flag_index_error();
+    for (int i = 0; i < k; ++i) rows[i] = 0;
     float t0 = 0.f, t1 = 0.f;
-    if (lane < H) {
-        t0 = sigmoidf(__ldg(theta + (long long)j * K + 2 * lane));
-        t1 = sigmoidf(__ldg(theta + (long long)j * K + 2 * lane + 1));
-        sPair[lane] = make_float2(t0, t1 - t0);
+    if (live) {
+        load_rows<k>(conn, j, w_in, lane, rows);
+        if (sub == 0 && lane < H) {
+            t0 = sigmoidf(__ldg(theta + (long long)j * K + 2 * lane));
+            t1 = sigmoidf(__ldg(theta + (long long)j * K + 2 * lane + 1));
+            *reinterpret_cast<float2*>(sT + 2 * lane) = make_float2(t0, t1);
+        }
     }
-    __syncwarp();
-    float te[H2], d[H2];
+    __syncthreads();
+    // this lane's half of the table: entries h*H .. h*H + H - 1, as 4-entry
+    // Moebius quads (k >= 3) or as level-0 lerp constants (k == 2)
+    constexpr bool QUADS = k >= 3;
+    float cq[QUADS ? H : 1];
+    float te[QUADS ? 1 : H2], d[QUADS ? 1 : H2];
+    if constexpr (QUADS) {
 #pragma unroll
-    for (int m = 0; m < H2; ++m) {
-        const float2 v = sPair[h * H2 + m];
-        te[m] = v.x;
-        d[m] = v.y;
+        for (int m = 0; m < H / 4; ++m) {
+            const float4 t = live ? *reinterpret_cast<const float4*>(sT + h * H + 4 * m)
+                                  : make_float4(0.f, 0.f, 0.f, 0.f);
+            const float c1 = t.y - t.x;
+            cq[4 * m] = t.x;
+            cq[4 * m + 1] = c1;
+            cq[4 * m + 2] = t.z - t.x;
+            cq[4 * m + 3] = (t.w - t.z) - c1;
+        }
+    } else {
+#pragma unroll
+        for (int m = 0; m < H2; ++m) {
+            const float2 t = live ? *reinterpret_cast<const float2*>(sT + h * H + 2 * m) : make_float2(0.f, 0.f);
+            te[m] = t.x;
+            d[m] = t.y - t.x;
+        }
     }
-    __syncwarp();
+    // upstream edges of node j: ids held one per lane (the first 32)
+    int e0 = 0, deg = 0, my_id = 0;
+    if constexpr (TERMS) {
+        if (live) {
+            int e1;
+            term_range(gs, j, lane, e0, e1);
+            deg = e1 - e0;
+            if (lane < deg) {
+                my_id = __ldg(gs.edge + e0 + lane);
+                if ((unsigned)my_id >= (unsigned)gs.n_edges) {
+                    flag_index_error();
+                    my_id = -1;   // read as a zero row
+                }
+            }
+        }
+    }
 
+    const int jj = live ? j : 0;
     const float* src[R];
 #pragma unroll
     for (int i = 0; i < k; ++i) src[i] = X + (long long)rows[i] * B + 4 * lane;
-    src[k] = dY + (long long)j * B + 4 * lane;
+    src[k] = TERMS ? nullptr : gs.dY + (long long)(jj / gs.group) * B + 4 * lane;
     float* pst[NQ];   // this lane's stored slots 2q + h, at its first sample
 #pragma unroll
-    for (int q = 0; q < NQ; ++q) pst[q] = P + ((long long)j * k + (2 * q + h < k ? 2 * q + h : 0)) * B + pair;
+    for (int q = 0; q < NQ; ++q) pst[q] = P + ((long long)jj * k + (2 * q + h < k ? 2 * q + h : 0)) * B + pair;
     const int nst = (int)((B + CH - 1) / CH);
+    const int per = (nst + kWarpsPerNode - 1) / kWarpsPerNode;
+    const int first = sub * per;
+    const int mine = !live ? 0 : max(0, min(nst, first + per) - first);
+    auto stage_base = [&](int i) { return (long long)(first + i) * CH; };
+    constexpr int RR = TERMS ? k : R;   // rows per ring stage
 
     int ib = 0;
-    auto issue = [&](int st) {
-        if (st < nst && (long long)st * CH + 4 * lane < B) {
-            float* buf = ring + ib * (R * CH) + 4 * lane;
+    auto issue = [&](int i) {   // i-th stage of this warp
+        if (i < mine) {
+            const long long sb = stage_base(i);
+            if (sb + 4 * lane < B) {
+                float* buf = ring + ib * (RR * CH) + 4 * lane;
 #pragma unroll
-            for (int r = 0; r < R; ++r) cp_async16(buf + r * CH, src[r] + (long long)st * CH);
+                for (int r = 0; r < RR; ++r) cp_async16(buf + r * CH, src[r] + sb);
+            }
         }
         cp_async_commit();
         ib = (ib + 1 == kStages) ? 0 : ib + 1;
+    };
+
+    // gradient of stages i .. i + kGatherStages - 1 from the upstream terms:
+    // lane covers samples 4 lane + 128 u (u < kGatherStages), so one row is
+    // read as kGatherStages x 512 contiguous bytes; rows in edge order, from 0
+    auto gather = [&](int i) {
+        if constexpr (TERMS) {
+            float4 g[kGatherStages];
+#pragma unroll
+            for (int u = 0; u < kGatherStages; ++u) g[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+            const long long s0 = stage_base(i) + 4 * lane;
+            const int nu = min(kGatherStages, mine - i);
+#pragma unroll 2
+            for (int q = 0; q < deg; ++q) {
+                const int id = q < 32 ? __shfl_sync(0xffffffffu, my_id, q) : __ldg(gs.edge + e0 + q);
+                if (id >= 0 && (unsigned)id < (unsigned)gs.n_edges) {
+                    const float* row = gs.terms + (long long)id * B + s0;
+#pragma unroll
+                    for (int u = 0; u < kGatherStages; ++u)
+                        if (u < nu && s0 + u * CH < B) g[u] = add4(g[u], ldg4(row + u * CH));
+                } else if (q >= 32 && lane == 0) {
+                    flag_index_error();
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < kGatherStages; ++u) {
+                const long long s = s0 + u * CH;
+                if (u < nu && s < B) {
+                    *reinterpret_cast<float4*>(gbuf + u * CH + 4 * lane) = g[u];
+                    if (dY_out) *reinterpret_cast<float4*>(dY_out + (long long)jj * B + s) = g[u];
+                }
+            }
+        }
     };
 
     float acc[H];
@@ -394,42 +634,59 @@ lut_backward_staged_kernel(const float* __restrict__ X, int w_in, long long B,
     for (int a = 0; a < H; ++a) acc[a] = 0.f;
 
 #pragma unroll
-    for (int st = 0; st < kStages - 1; ++st) issue(st);
+    for (int i = 0; i < kStages - 1; ++i) issue(i);
     int rb = 0;
-    for (int st = 0; st < nst; ++st) {
-        issue(st + kStages - 1);
+    for (int i = 0; i < mine; ++i) {
+        issue(i + kStages - 1);
+        const long long sbase = stage_base(i);
+        float* buf = ring + rb * (RR * CH);
+        if constexpr (TERMS) {
+            if (i % kGatherStages == 0) {
+                __syncwarp();   // previous readers of gbuf are done
+                gather(i);
+            }
+        } else {
+            const long long s4 = sbase + 4 * lane;   // this lane's 16-byte chunk
+            if (dY_out && s4 < B)
+                *reinterpret_cast<float4*>(dY_out + (long long)jj * B + s4) = ldg4(src[k] + sbase);
+        }
         cp_async_wait<kStages - 1>();
         __syncwarp();
-        const float* buf = ring + rb * (R * CH) + pair;
-        const long long sbase = (long long)st * CH;
+        const bool full = sbase + CH <= B;
+        const float* rbuf = buf + pair;
+        const float* gsrc = TERMS ? gbuf + (i % kGatherStages) * CH + pair : rbuf + k * CH;
 #pragma unroll 2
         for (int c = 0; c < CH / 16; ++c) {
-            const bool in = sbase + 16 * c + pair < B;
+            const bool in = full || sbase + 16 * c + pair < B;
             float x[k], omx[k], dx[k];
 #pragma unroll
-            for (int i = 0; i < k; ++i) {
-                x[i] = in ? buf[i * CH + 16 * c] : 0.f;
-                omx[i] = 1.0f - x[i];
-                dx[i] = 0.f;
+            for (int q = 0; q < k; ++q) {
+                x[q] = in ? rbuf[q * CH + 16 * c] : 0.f;
+                omx[q] = 1.0f - x[q];
             }
-            const float g = in ? buf[k * CH + 16 * c] : 0.f;
+            const float g = in ? gsrc[16 * c] : 0.f;
             const float adj = g * (h ? x[k - 1] : omx[k - 1]);
-            const float v = bwd_tree<k - 2, 0>(te, d, x, omx, adj, dx, acc);
+            float v;
+            if constexpr (QUADS) {
+                const float W[4] = {omx[0] * omx[1], x[0] * omx[1], omx[0] * x[1], x[0] * x[1]};
+                v = bwd_tree_quad<k - 2, 0>(cq, x, omx, W, adj, dx, acc);
+            } else {
+                v = bwd_tree<k - 2, 0>(te, d, x, omx, adj, dx, acc);
+            }
             if constexpr (WANT_DX) {
 #pragma unroll
                 for (int q = 0; q < NQ; ++q) {
-                    const int e = 2 * q, o = 2 * q + 1;   // lane 0 stores e, lane 1 stores o
-                    // what the partner needs from this lane
+                    const int ev = 2 * q, od = 2 * q + 1;   // lane 0 stores ev, lane 1 stores od
                     float send;
-                    if (e == k - 1)      send = v;                    // lane 0 needs v_1
-                    else if (o == k - 1) send = h ? dx[e] : v;        // lane 1 needs v_0
-                    else if (o < k)      send = h ? dx[e] : dx[o];
-                    else                 send = dx[e];
+                    if (ev == k - 1)      send = v;                      // lane 0 needs v_1
+                    else if (od == k - 1) send = h ? dx[ev] : v;         // lane 1 needs v_0
+                    else if (od < k)      send = h ? dx[ev] : dx[od];
+                    else                  send = dx[ev];
                     const float recv = __shfl_xor_sync(0xffffffffu, send, 1);
-                    float full;
-                    if (h == 0) full = (e == k - 1) ? g * (recv - v) : dx[e] + recv;
-                    else        full = (o == k - 1) ? g * (v - recv) : (o < k ? dx[o] + recv : 0.f);
-                    if (in && (h == 0 || o < k)) pst[q][sbase + 16 * c] = full;
+                    float full_dx;
+                    if (h == 0) full_dx = (ev == k - 1) ? g * (recv - v) : dx[ev] + recv;
+                    else        full_dx = (od == k - 1) ? g * (v - recv) : (od < k ? dx[od] + recv : 0.f);
+                    if (in && (h == 0 || od < k)) pst[q][sbase + 16 * c] = full_dx;
                 }
             }
         }
@@ -440,18 +697,22 @@ lut_backward_staged_kernel(const float* __restrict__ X, int w_in, long long B,
     __syncwarp();
 
     // dtheta: entry a lives in half a / H at offset a % H of the lanes with
-    // that parity; sum those 16 lanes in lane order through the ring
-    float* red = ring;   // [32][H + 1]
+    // that parity; sum those 16 lanes, then the node's warps, in a fixed order
+    float* red = ring;   // [32][H + 1] per warp
 #pragma unroll
     for (int a = 0; a < H; ++a) red[lane * (H + 1) + a] = acc[a];
-    __syncwarp();
-    if (lane < H) {
+    __syncthreads();
+    if (live && sub == 0 && lane < H) {
         float s0 = 0.f, s1 = 0.f;
         const int a0 = 2 * lane, hh = a0 / H, ao = a0 % H;
+#pragma unroll
+        for (int q = 0; q < kWarpsPerNode; ++q) {
+            const float* rq = smem + (warp + q) * FPW;
 #pragma unroll 4
-        for (int p = 0; p < 16; ++p) {
-            s0 += red[(2 * p + hh) * (H + 1) + ao];
-            s1 += red[(2 * p + hh) * (H + 1) + ao + 1];
+            for (int p = 0; p < 16; ++p) {
+                s0 += rq[(2 * p + hh) * (H + 1) + ao];
+                s1 += rq[(2 * p + hh) * (H + 1) + ao + 1];
+            }
         }
         float* out = dtheta + (long long)j * K + a0;
         out[0] = t0 * (1.0f - t0) * s0;
@@ -460,7 +721,10 @@ lut_backward_staged_kernel(const float* __restrict__ X, int w_in, long long B,
 }
 
 // dX[i][s] = sum over the CSR edges of input i (increasing edge id) of
-// P[edge][s].  One warp per input row, lanes over samples.
+// P[edge][s].  One warp per input row, lanes over samples.  The row's edge
+// ids are read once (one per lane) so the loads issue back to back, and each
+// pass reads 2 KB contiguous from every edge row (4 x 16 bytes per lane):
+// the rows are random in DRAM and short reads waste its bandwidth.
 template <bool VEC>
 __global__ void __launch_bounds__(kCsrWarps * 32)
 csr_reduce_kernel(const float* __restrict__ P, long long B, const int* __restrict__ off,
@@ -473,54 +737,61 @@ csr_reduce_kernel(const float* __restrict__ P, long long B, const int* __restric
         if (lane == 0) flag_index_error();
         e0 = e1 = 0;
     }
+    const int deg = e1 - e0;
+    int my_id = -1;   // ids of the first 32 edges, -1 when out of range
+    if (lane < deg) {
+        my_id = __ldg(edge + e0 + lane);
+        if ((unsigned)my_id >= (unsigned)nE) {
+            flag_index_error();
+            my_id = -1;
+        }
+    }
+    auto edge_id = [&](int q) {
+        if (q < 32) return __shfl_sync(0xffffffffu, my_id, q);
+        const int id = __ldg(edge + e0 + q);
+        if ((unsigned)id >= (unsigned)nE) {
+            if (lane == 0) flag_index_error();
+            return -1;
+        }
+        return id;
+    };
     float* out = dX + (long long)i * B;
     if constexpr (VEC) {
         for (long long base = 0; base < B; base += 512) {
             float4 acc[4];
 #pragma unroll
-            for (int q = 0; q < 4; ++q) acc[q] = make_float4(0.f, 0.f, 0.f, 0.f);
-            for (int e = e0; e < e1; ++e) {
-                int eid = __ldg(edge + e);
-                if ((unsigned)eid >= (unsigned)nE) {
-                    if (lane == 0) flag_index_error();
-                    continue;
-                }
-                const float* pr = P + (long long)eid * B;
+            for (int u = 0; u < 4; ++u) acc[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 2
+            for (int q = 0; q < deg; ++q) {
+                const int id = edge_id(q);
+                if (id < 0) continue;
+                const float* pr = P + (long long)id * B + base + 4 * lane;
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const long long s = base + 128 * q + 4 * lane;
-                    if (s < B) {
-                        const float4 v = ldg4(pr + s);
-                        acc[q].x += v.x; acc[q].y += v.y; acc[q].z += v.z; acc[q].w += v.w;
-                    }
-                }
+                for (int u = 0; u < 4; ++u)
+                    if (base + 128 * u + 4 * lane < B) acc[u] = add4(acc[u], ldg4(pr + 128 * u));
             }
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const long long s = base + 128 * q + 4 * lane;
-                if (s < B) *reinterpret_cast<float4*>(out + s) = acc[q];
+            for (int u = 0; u < 4; ++u) {
+                const long long s = base + 128 * u + 4 * lane;
+                if (s < B) *reinterpret_cast<float4*>(out + s) = acc[u];
             }
         }
     } else {
         for (long long base = 0; base < B; base += 128) {
             float acc[4] = {0.f, 0.f, 0.f, 0.f};
-            for (int e = e0; e < e1; ++e) {
-                int eid = __ldg(edge + e);
-                if ((unsigned)eid >= (unsigned)nE) {
-                    if (lane == 0) flag_index_error();
-                    continue;
-                }
-                const float* pr = P + (long long)eid * B;
+#pragma unroll 2
+            for (int q = 0; q < deg; ++q) {
+                const int id = edge_id(q);
+                if (id < 0) continue;
+                const float* pr = P + (long long)id * B + base + lane;
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const long long s = base + 32 * q + lane;
-                    if (s < B) acc[q] += __ldg(pr + s);
-                }
+                for (int u = 0; u < 4; ++u)
+                    if (base + 32 * u + lane < B) acc[u] += __ldg(pr + 32 * u);
             }
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const long long s = base + 32 * q + lane;
-                if (s < B) out[s] = acc[q];
+            for (int u = 0; u < 4; ++u) {
+                const long long s = base + 32 * u + lane;
+                if (s < B) out[s] = acc[u];
             }
         }
     }
@@ -528,22 +799,26 @@ csr_reduce_kernel(const float* __restrict__ P, long long B, const int* __restric
 
 // ----------------------------------------------------------- launchers --
 
-// Samples per forward block: the whole batch when the layer input fits in
-// a fraction of L2, else a batch slice so that the gathered working set of
-// the blocks resident at one time stays in L2.
-long long forward_chunk(int w_in, long long B) {
+// Samples per forward work item (node x batch slice): small enough that the
+// gathered working set of the resident items stays in L2 and that the launch
+// has ~6 waves of items, but at least 512 samples so the per-item set-up
+// stays small.
+long long forward_chunk(int w_in, int w, long long B) {
     const long long l2_budget = 48ll << 20;
-    if ((long long)w_in * B * 4 <= l2_budget) return B;
-    long long c = l2_budget / ((long long)w_in * 4);
+    long long c = B;
+    if ((long long)w_in * B * 4 > l2_budget) c = l2_budget / ((long long)w_in * 4);
+    const long long items_wanted = 6ll * 152 * 16;
+    const long long by_waves = (long long)w * B / items_wanted;
+    if (by_waves < c) c = by_waves;
     c = (c / 128) * 128;
-    if (c < 256) c = 256;
+    if (c < 512) c = 512;
     return c < B ? c : B;
 }
 
 template <int k>
 int launch_forward(const float* X, int w_in, long long B, const int* conn, const float* theta,
                    int w, float* Y, bool vec, cudaStream_t st) {
-    long long chunk = forward_chunk(w_in, B);
+    long long chunk = forward_chunk(w_in, w, B);
     if (vec) chunk = (chunk + 3) / 4 * 4;
     const long long ny = (B + chunk - 1) / chunk;
     if (ny > 65535) return BITLOGIC_ERR_SHAPE;
@@ -551,39 +826,45 @@ int launch_forward(const float* X, int w_in, long long B, const int* conn, const
     if (vec)
         lut_forward_staged_kernel<k><<<grid, kFwdWarps * 32, 0, st>>>(X, w_in, B, conn, theta, w, Y, chunk);
     else
-        lut_forward_kernel<k, false><<<grid, kFwdWarps * 32, 0, st>>>(X, w_in, B, conn, theta, w, Y, chunk);
+        lut_forward_kernel<k><<<grid, kFwdWarps * 32, 0, st>>>(X, w_in, B, conn, theta, w, Y, chunk);
     return launch_status();
 }
 
-template <int k, bool WANT_DX>
-int launch_staged(const float* X, int w_in, long long B, const int* conn, const float* theta,
-                  int w, const float* dY, float* dtheta, float* P, cudaStream_t st) {
-    constexpr size_t smem = staged_smem_bytes<k>();
-    auto kern = lut_backward_staged_kernel<k, WANT_DX>;
-    if (smem > 48 * 1024 &&
-        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
-        return BITLOGIC_ERR_CUDA;
-    dim3 grid((unsigned)((w + kBwdWarps - 1) / kBwdWarps));
-    kern<<<grid, kBwdWarps * 32, smem, st>>>(X, w_in, B, conn, theta, w, dY, dtheta, P);
+template <int k, bool WANT_DX, bool TERMS>
+int launch_backward_impl(const float* X, int w_in, long long B, const int* conn, const float* theta,
+                         int w, const GradSource& gs, float* dtheta, float* P, float* dY_out,
+                         bool staged, cudaStream_t st) {
+    if constexpr (k >= 2) {
+        if (staged) {
+            constexpr size_t smem = node_smem_bytes<k, TERMS>();
+            auto kern = lut_backward_node_kernel<k, WANT_DX, TERMS>;
+            if (smem > 48 * 1024 &&
+                cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+                return BITLOGIC_ERR_CUDA;
+            kern<<<(unsigned)((w + kNodesPerBlock - 1) / kNodesPerBlock), kBwdWarps * 32, smem, st>>>(
+                X, w_in, B, conn, theta, w, gs, dtheta, P, dY_out);
+            return launch_status();
+        }
+    }
+    dim3 grid((unsigned)((w + kFwdWarps - 1) / kFwdWarps));
+    lut_backward_kernel<k, WANT_DX, TERMS><<<grid, kFwdWarps * 32, 0, st>>>(X, w_in, B, conn, theta, w, gs,
+                                                                            dtheta, P, dY_out);
     return launch_status();
 }
 
 template <int k>
 int launch_backward(const float* X, int w_in, long long B, const int* conn, const float* theta,
-                    int w, const float* dY, float* dtheta, float* P, bool want_dx,
+                    int w, const GradSource& gs, float* dtheta, float* P, float* dY_out,
                     cudaStream_t st) {
-    if constexpr (k >= 2) {
-        const bool staged = (B % 4 == 0) && aligned16(X) && aligned16(dY);
-        if (staged)
-            return want_dx ? launch_staged<k, true>(X, w_in, B, conn, theta, w, dY, dtheta, P, st)
-                           : launch_staged<k, false>(X, w_in, B, conn, theta, w, dY, dtheta, P, st);
+    const bool terms = gs.terms != nullptr;
+    const bool staged = (B % 4 == 0) && aligned16(X) && aligned16(terms ? gs.terms : gs.dY) &&
+                        (!dY_out || aligned16(dY_out)) && (!P || aligned16(P));
+    if (P) {
+        return terms ? launch_backward_impl<k, true, true>(X, w_in, B, conn, theta, w, gs, dtheta, P, dY_out, staged, st)
+                     : launch_backward_impl<k, true, false>(X, w_in, B, conn, theta, w, gs, dtheta, P, dY_out, staged, st);
     }
-    dim3 grid((unsigned)((w + kBwdWarps - 1) / kBwdWarps));
-    if (want_dx)
-        lut_backward_kernel<k, true><<<grid, kBwdWarps * 32, 0, st>>>(X, w_in, B, conn, theta, w, dY, dtheta, P);
-    else
-        lut_backward_kernel<k, false><<<grid, kBwdWarps * 32, 0, st>>>(X, w_in, B, conn, theta, w, dY, dtheta, P);
-    return launch_status();
+    return terms ? launch_backward_impl<k, false, true>(X, w_in, B, conn, theta, w, gs, dtheta, P, dY_out, staged, st)
+                 : launch_backward_impl<k, false, false>(X, w_in, B, conn, theta, w, gs, dtheta, P, dY_out, staged, st);
 }
 
 int check_layer(const void* X, int32_t w_in, int64_t B, const void* conn, const void* theta,
@@ -628,29 +909,50 @@ extern "C" size_t bitlogic_lut_backward_workspace(int32_t w_in, int64_t B, int32
     return (size_t)w * (size_t)k * (size_t)B * sizeof(float);
 }
 
-extern "C" int bitlogic_lut_backward_edges(const float* X, int32_t w_in, int64_t B,
-                                           const int32_t* conn, const float* theta,
-                                           int32_t w, int32_t k, const float* dY,
-                                           float* dtheta, float* edge_terms,
-                                           cudaStream_t stream) {
+extern "C" int bitlogic_lut_backward_ex(const float* X, int32_t w_in, int64_t B,
+                                        const int32_t* conn, const float* theta,
+                                        int32_t w, int32_t k,
+                                        const float* dY, int32_t dy_group,
+                                        const float* up_terms, const int32_t* up_off,
+                                        const int32_t* up_edge, int32_t up_edges,
+                                        float* dtheta, float* edge_terms, float* dY_out,
+                                        cudaStream_t stream) {
     int st = check_layer(X, w_in, B, conn, theta, w, k);
     if (st) return st;
-    if (!dtheta || (B > 0 && !dY)) return BITLOGIC_ERR_NULL;
+    if (!dtheta) return BITLOGIC_ERR_NULL;
+    const bool terms = up_terms != nullptr;
+    if (B > 0 && terms == (dY != nullptr)) return BITLOGIC_ERR_NULL;   // exactly one source
+    if (terms) {
+        if (!up_off || !up_edge) return BITLOGIC_ERR_NULL;
+        if (up_edges < 0) return BITLOGIC_ERR_SHAPE;
+    } else if (dy_group < 1 || dy_group > w) {
+        return BITLOGIC_ERR_SHAPE;
+    }
     if (B == 0) {
         // empty batch: the batch sums are zero
         if (cudaMemsetAsync(dtheta, 0, sizeof(float) * (size_t)w * ((size_t)1 << k), stream) != cudaSuccess)
             return BITLOGIC_ERR_CUDA;
         return BITLOGIC_OK;
     }
-    const bool want = edge_terms != nullptr;
+    GradSource gs{dY, dy_group, up_terms, up_off, up_edge, up_edges};
     switch (k) {
-        case 1: return launch_backward<1>(X, w_in, B, conn, theta, w, dY, dtheta, edge_terms, want, stream);
-        case 2: return launch_backward<2>(X, w_in, B, conn, theta, w, dY, dtheta, edge_terms, want, stream);
-        case 3: return launch_backward<3>(X, w_in, B, conn, theta, w, dY, dtheta, edge_terms, want, stream);
-        case 4: return launch_backward<4>(X, w_in, B, conn, theta, w, dY, dtheta, edge_terms, want, stream);
-        case 5: return launch_backward<5>(X, w_in, B, conn, theta, w, dY, dtheta, edge_terms, want, stream);
-        default: return launch_backward<6>(X, w_in, B, conn, theta, w, dY, dtheta, edge_terms, want, stream);
+        case 1: return launch_backward<1>(X, w_in, B, conn, theta, w, gs, dtheta, edge_terms, dY_out, stream);
+        case 2: return launch_backward<2>(X, w_in, B, conn, theta, w, gs, dtheta, edge_terms, dY_out, stream);
+        case 3: return launch_backward<3>(X, w_in, B, conn, theta, w, gs, dtheta, edge_terms, dY_out, stream);
+        case 4: return launch_backward<4>(X, w_in, B, conn, theta, w, gs, dtheta, edge_terms, dY_out, stream);
+        case 5: return launch_backward<5>(X, w_in, B, conn, theta, w, gs, dtheta, edge_terms, dY_out, stream);
+        default: return launch_backward<6>(X, w_in, B, conn, theta, w, gs, dtheta, edge_terms, dY_out, stream);
     }
+}
+
+extern "C" int bitlogic_lut_backward_edges(const float* X, int32_t w_in, int64_t B,
+                                           const int32_t* conn, const float* theta,
+                                           int32_t w, int32_t k, const float* dY,
+                                           float* dtheta, float* edge_terms,
+                                           cudaStream_t stream) {
+    if (B > 0 && !dY) return BITLOGIC_ERR_NULL;
+    return bitlogic_lut_backward_ex(X, w_in, B, conn, theta, w, k, dY, 1,
+                                    nullptr, nullptr, nullptr, 0, dtheta, edge_terms, nullptr, stream);
 }
 
 extern "C" int bitlogic_csr_reduce(const float* edge_terms, int64_t B, const int32_t* csr_off,

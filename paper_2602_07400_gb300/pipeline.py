@@ -17,8 +17,8 @@ import numpy as np
 import torch
 
 from . import (bitlogic_binarize_tables, bitlogic_build_csr, bitlogic_csr_reduce,
-               bitlogic_encode_thermometer, bitlogic_hard_forward, bitlogic_head_loss,
-               bitlogic_head_loss_workspace, bitlogic_lut_backward_edges, bitlogic_lut_forward,
+               bitlogic_encode_thermometer, bitlogic_hard_forward, bitlogic_head_loss_ex,
+               bitlogic_head_loss_workspace, bitlogic_lut_backward_ex, bitlogic_lut_forward,
                bitlogic_pack_bits)
 
 
@@ -47,12 +47,20 @@ class Network:
 
 
 class TrainStep:
+    """One soft training step.  The backward is fused across the call
+    boundaries the ABI offers: the head emits one gradient row per class
+    (``dyg``) that the layer-2 backward reads for every node of the class, and
+    the layer-1 backward reduces layer 2's per-edge input-gradient terms on
+    the fly through the CSR map, so neither dY2 nor dY1 is stored (set
+    ``keep_dy1`` to also write dY1, e.g. to check it)."""
+
     def __init__(self, net: Network, B: int, d: int, thresholds: Sequence[int], C: int,
-                 tau: float, want_dx1: bool = False, device="cuda"):
+                 tau: float, want_dx1: bool = False, keep_dy1: bool = False, device="cuda"):
         dev = torch.device(device)
         self.net, self.B, self.d, self.C, self.tau = net, int(B), int(d), int(C), float(tau)
         self.thr = [int(t) for t in thresholds]
         assert d * len(self.thr) == net.w_in
+        assert net.w2 % C == 0
         f32 = dict(dtype=torch.float32, device=dev)
         self.x = torch.zeros(B, d, dtype=torch.uint8, device=dev)
         self.labels = torch.zeros(B, dtype=torch.int32, device=dev)
@@ -61,13 +69,13 @@ class TrainStep:
         self.y2 = torch.empty(net.w2, B, **f32)
         self.logits = torch.empty(B, C, **f32)
         self.loss = torch.zeros(1, **f32)
-        self.dy2 = torch.empty(net.w2, B, **f32)
-        self.dy1 = torch.empty(net.w1, B, **f32)
+        self.dyg = torch.empty(C, B, **f32)          # gradient row shared by each class's nodes
+        self.dy1 = torch.empty(net.w1, B, **f32) if keep_dy1 else None
         self.dth1 = torch.empty_like(net.theta1)
         self.dth2 = torch.empty_like(net.theta2)
         self.dbits = torch.empty(net.w_in, B, **f32) if want_dx1 else None
         # per-edge input-gradient terms of layer 2 (and of layer 1 when its
-        # input gradient is wanted), summed per input through the CSR map
+        # input gradient is wanted)
         self.edges2 = torch.empty(net.w2 * net.k2, B, **f32)
         self.edges1 = torch.empty(net.w1 * net.k1, B, **f32) if want_dx1 else None
         self.ws_head = torch.empty(bitlogic_head_loss_workspace(B, C), dtype=torch.uint8, device=dev)
@@ -84,21 +92,18 @@ class TrainStep:
         mark("forward1")
         bitlogic_lut_forward(self.y1, n.conn2, n.theta2, self.y2, stream)
         mark("forward2")
-        bitlogic_head_loss(self.y2, self.labels, self.C, self.tau, self.loss, self.ws_head,
-                           logits=self.logits, dY=self.dy2, stream=stream)
+        bitlogic_head_loss_ex(self.y2, self.labels, self.C, self.tau, self.loss, self.ws_head,
+                              logits=self.logits, dY_grouped=self.dyg, stream=stream)
         mark("head")
 
     def backward(self, stream=None, mark=_nomark):
-        # each layer's backward is bitlogic_lut_backward split into its two
-        # phases (node kernel, then CSR reduction) so each can be timed
         n = self.net
-        bitlogic_lut_backward_edges(self.y1, n.conn2, n.theta2, self.dy2, self.dth2,
-                                    self.edges2, stream)
+        bitlogic_lut_backward_ex(self.y1, n.conn2, n.theta2, self.dth2, dY=self.dyg,
+                                 dy_group=n.w2 // self.C, edge_terms=self.edges2, stream=stream)
         mark("backward2")
-        bitlogic_csr_reduce(self.edges2, n.off2, n.edge2, self.dy1, stream)
-        mark("csr2")
-        bitlogic_lut_backward_edges(self.bits, n.conn1, n.theta1, self.dy1, self.dth1,
-                                    self.edges1, stream)
+        bitlogic_lut_backward_ex(self.bits, n.conn1, n.theta1, self.dth1, up_terms=self.edges2,
+                                 up_off=n.off2, up_edge=n.edge2, edge_terms=self.edges1,
+                                 dY_out=self.dy1, stream=stream)
         mark("backward1")
         if self.dbits is not None:
             bitlogic_csr_reduce(self.edges1, n.off1, n.edge1, self.dbits, stream)
@@ -108,11 +113,11 @@ class TrainStep:
         self.forward(stream, mark)
         self.backward(stream, mark)
 
-    # kernels one run() launches (encode 1, forwards 2, head 4, backwards and
-    # CSR reductions 3 or 4)
+    # kernels one run() launches: encode 1, forwards 2, head 3, backwards 2
+    # (+ the layer-1 CSR reduction when the input gradient is wanted)
     @property
     def kernels_per_run(self) -> int:
-        return 10 + (1 if self.dbits is not None else 0)
+        return 8 + (1 if self.dbits is not None else 0)
 
 
 class HardInfer:

@@ -98,6 +98,69 @@ def test_lut_backward(k, w_in, w, B):
     no_device_error()
 
 
+@pytest.mark.parametrize("k,w_in,w,B,group", [(6, 300, 120, 256, 12), (6, 64, 40, 1024, 40), (3, 50, 30, 37, 5),
+                                               (2, 9, 20, 100, 1), (1, 4, 6, 8, 3)])
+def test_backward_grouped_dy(k, w_in, w, B, group):
+    # dY given as one row per group of `group` consecutive nodes
+    X = synth.uniform_activations(w_in, B, seed=k + B)
+    conn = synth.connectivity(w, k, w_in, seed=w)
+    theta = synth.table_logits(w, 1 << k, seed=k)
+    rows = synth.uniform_gradients(w // group, B, seed=group, scale=1e-3)
+    dY = np.repeat(rows, group, axis=0)
+    dth = torch.empty(w, 1 << k, device="cuda")
+    P = torch.empty(w * k, B, device="cuda")
+    out = torch.empty(w, B, device="cuda")
+    bl.bitlogic_lut_backward_ex(dev(X), dev(conn), dev(theta), dth, dY=dev(rows), dy_group=group,
+                                edge_terms=P, dY_out=out)
+    check_exact(out.cpu().numpy(), dY, "dY_out")
+    off, edge = bl.bitlogic_build_csr(conn, w_in)
+    dX = torch.empty(w_in, B, device="cuda")
+    bl.bitlogic_csr_reduce(P, dev(off), dev(edge), dX)
+    wth, wdx = oracle.lut_backward(X.astype(np.float64), conn, theta, dY.astype(np.float64))
+    check_grad(dth, wth, "dtheta")
+    check_grad(dX, wdx, "dX")
+    # same as the ungrouped call on the expanded dY, bit for bit
+    dth2 = torch.empty(w, 1 << k, device="cuda")
+    P2 = torch.empty(w * k, B, device="cuda")
+    bl.bitlogic_lut_backward_edges(dev(X), dev(conn), dev(theta), dev(dY), dth2, P2)
+    check_exact(dth2.cpu().numpy(), dth.cpu().numpy(), "dtheta grouped vs full")
+    check_exact(P2.cpu().numpy(), P.cpu().numpy(), "edge terms grouped vs full")
+
+
+@pytest.mark.parametrize("k,w_in,w,B", [(6, 200, 150, 256), (6, 1000, 300, 1024), (4, 40, 64, 36),
+                                        (2, 12, 30, 7), (1, 5, 8, 64)])
+def test_backward_from_upstream_terms(k, w_in, w, B):
+    # layer A (this call) gets its output gradient as the CSR sum of layer
+    # B's per-edge terms; equals csr_reduce + backward_edges bit for bit
+    kb, wb = 3, 2 * w
+    X = synth.uniform_activations(w_in, B, seed=B)
+    conn = synth.connectivity(w, k, w_in, seed=1)
+    theta = synth.table_logits(w, 1 << k, seed=2)
+    conn_b = synth.connectivity(wb, kb, w, seed=3)       # layer B reads layer A's outputs
+    off_b, edge_b = bl.bitlogic_build_csr(conn_b, w)
+    terms = synth.uniform_gradients(wb * kb, B, seed=4, scale=1e-3)
+    dth = torch.empty(w, 1 << k, device="cuda")
+    out = torch.empty(w, B, device="cuda")
+    P = torch.empty(w * k, B, device="cuda")
+    bl.bitlogic_lut_backward_ex(dev(X), dev(conn), dev(theta), dth, up_terms=dev(terms),
+                                up_off=dev(off_b), up_edge=dev(edge_b), edge_terms=P, dY_out=out)
+    dY_ref = torch.empty(w, B, device="cuda")
+    bl.bitlogic_csr_reduce(dev(terms), dev(off_b), dev(edge_b), dY_ref)
+    check_exact(out.cpu().numpy(), dY_ref.cpu().numpy(), "dY from terms vs csr_reduce")
+    dth_ref = torch.empty(w, 1 << k, device="cuda")
+    P_ref = torch.empty(w * k, B, device="cuda")
+    bl.bitlogic_lut_backward_edges(dev(X), dev(conn), dev(theta), dY_ref, dth_ref, P_ref)
+    check_exact(dth.cpu().numpy(), dth_ref.cpu().numpy(), "dtheta fused vs unfused")
+    check_exact(P.cpu().numpy(), P_ref.cpu().numpy(), "edge terms fused vs unfused")
+    # and against the oracle on the dense dY of the upstream terms
+    dY = np.zeros((w, B))
+    for e in range(wb * kb):
+        dY[conn_b.reshape(-1)[e]] += terms[e].astype(np.float64)
+    wth, _ = oracle.lut_backward(X.astype(np.float64), conn, theta, dY, want_dx=False)
+    check_grad(dth, wth, "dtheta")
+    no_device_error()
+
+
 def test_backward_is_deterministic_and_handles_skewed_consumers():
     # 3 inputs shared by 500 nodes (fan-in 2): every input has ~333 consumers
     k, w_in, w, B = 2, 3, 500, 96
@@ -173,6 +236,21 @@ def test_head_loss(C, g, B, tau):
     bl.bitlogic_head_loss(dev(Y), dev(labels), C, tau, loss2, ws)
     check_exact(loss2.cpu().numpy(), loss.cpu().numpy(), "loss without optional outputs")
     no_device_error()
+
+
+def test_head_grouped_gradient_rows():
+    C, g, B = 10, 80, 259
+    rng = np.random.default_rng(3)
+    Y = rng.random((C * g, B)).astype(np.float32)
+    labels = rng.integers(0, C, size=B).astype(np.int32)
+    ws = torch.empty(bl.bitlogic_head_loss_workspace(B, C), dtype=torch.uint8, device="cuda")
+    dY = torch.empty(C * g, B, device="cuda")
+    dYg = torch.empty(C, B, device="cuda")
+    loss = torch.zeros(1, device="cuda")
+    bl.bitlogic_head_loss_ex(dev(Y), dev(labels), C, 7.0, loss, ws, dY=dY, dY_grouped=dYg)
+    full = dY.cpu().numpy().reshape(C, g, B)
+    for c in range(C):
+        check_exact(full[c], np.repeat(dYg[c:c + 1].cpu().numpy(), g, axis=0), f"class {c}")
 
 
 # -------------------------------------------------------------------- hard --

@@ -29,17 +29,26 @@ pytestmark = pytest.mark.gpu
 oracle.set_threads(os.cpu_count() or 1)
 
 
-def _step(wl, want_dx1, seed=0, k=None):
+def _step(wl, want_dx1, seed=0, k=None, keep_dy1=True):
     if k is not None:
         wl = synth.Workload(wl.name, wl.batch, wl.d, wl.classes, wl.sigma, wl.thresholds, wl.widths, k, wl.tau)
     conn1, th1, conn2, th2 = synth.network(wl, seed)
     x, labels = synth.blob_batch(wl.batch, wl.d, wl.classes, wl.sigma, seed=seed + 7)
     net = Network(conn1, th1, conn2, th2, wl.w_in)
-    st = TrainStep(net, wl.batch, wl.d, wl.thresholds, wl.classes, wl.tau, want_dx1=want_dx1)
+    st = TrainStep(net, wl.batch, wl.d, wl.thresholds, wl.classes, wl.tau, want_dx1=want_dx1,
+                   keep_dy1=keep_dy1)
     st.load(x.cuda(), labels.cuda())
     st.run()
     torch.cuda.synchronize()
     return wl, st, x.numpy(), labels.numpy(), (conn1, th1, conn2, th2)
+
+
+def _check_grouped(st, dy2, wl):
+    # the head's gradient rows: every node of a class shares its row
+    g = wl.widths[1] // wl.classes
+    rows = dy2.reshape(wl.classes, g, -1)
+    assert np.all(rows == rows[:, :1, :])
+    check_grad(st.dyg, rows[:, 0, :], "dY2 (per-class rows)")
 
 
 def _full_compare(wl, st, x, labels, params, want_dx1):
@@ -51,7 +60,7 @@ def _full_compare(wl, st, x, labels, params, want_dx1):
     check_fwd(st.y2, r["y2"], "y2")
     check_fwd(st.logits, r["logits"], "logits")
     check_fwd(st.loss, np.array([r["loss"]]), "loss")
-    check_grad(st.dy2, r["dy2"], "dy2")
+    _check_grouped(st, r["dy2"], wl)
     check_grad(st.dth2, r["dth2"], "dtheta2")
     check_grad(st.dy1, r["dy1"], "dy1")
     check_grad(st.dth1, r["dth1"], "dtheta1")
@@ -70,6 +79,15 @@ def test_mnist_step_all_outputs(k):
     _full_compare(wl, st, x, labels, params, False)
 
 
+def test_mnist_bench_configuration_matches():
+    # the benchmark runs without storing dY1; its outputs equal the checked
+    # configuration's bit for bit
+    _, a, *_ = _step(synth.WORKLOADS["mnist"], want_dx1=False, keep_dy1=True)
+    _, b, *_ = _step(synth.WORKLOADS["mnist"], want_dx1=False, keep_dy1=False)
+    for name in ("y2", "logits", "loss", "dyg", "dth2", "dth1"):
+        check_exact(getattr(b, name).cpu().numpy(), getattr(a, name).cpu().numpy(), name)
+
+
 def _sampled_compare(wl, st, x, labels, params, n_nodes=96, seed=0):
     conn1, th1, conn2, th2 = params
     bits = oracle.encode_thermometer(x, wl.thresholds)
@@ -81,7 +99,7 @@ def _sampled_compare(wl, st, x, labels, params, n_nodes=96, seed=0):
     logits, loss, dy2 = oracle.head_loss(y2, labels, wl.classes, wl.tau)
     check_fwd(st.logits, logits, "logits")
     check_fwd(st.loss, np.array([loss]), "loss")
-    check_grad(st.dy2, dy2, "dy2")
+    _check_grouped(st, dy2, wl)
     rng = np.random.default_rng(seed)
     w1, w2 = wl.widths
     # layer-2 table gradients of sampled nodes
