@@ -50,7 +50,8 @@ typedef enum {
     BITLOGIC_ERR_CUDA = -6,       /* a CUDA launch or copy failed */
     BITLOGIC_ERR_INDEX = -7,      /* index out of range (host-side check) */
     BITLOGIC_ERR_DEVICE = -8,     /* device-side index check tripped */
-    BITLOGIC_ERR_THRESH = -9      /* thresholds: b outside 1..32 */
+    BITLOGIC_ERR_THRESH = -9,     /* thresholds: b outside 1..32 */
+    BITLOGIC_ERR_TOO_LARGE = -10  /* sizes beyond bitlogic_head_loss_noalloc's fixed scratch */
 } bitlogic_status_t;
 
 /* Thermometer encoder E: R^d -> {0,1}^{db} (paper §3, "Encoders and heads";
@@ -166,6 +167,26 @@ int bitlogic_head_loss_ex(const float* Y, int32_t w, int64_t B, int32_t C, float
                           const int32_t* labels, float* logits, float* loss, float* dY,
                           float* dY_grouped, void* workspace, size_t ws_bytes,
                           cudaStream_t stream);
+
+/* bitlogic_head_loss without a workspace argument, for callers that cannot
+ * allocate device memory: code hosted inside another runtime that owns the
+ * device allocator, or loops with a fixed memory budget where cudaMalloc /
+ * cudaFree (which may synchronize the device or fail) are not allowed.  The
+ * paper has no counterpart; this is a convenience of the library.
+ *   Same arguments and results as bitlogic_head_loss; the caller still
+ *   passes every input and output.
+ *   Scratch: a fixed 8 MiB device array inside the library, reserved on
+ *   every GPU that loads it until the process exits.  The call requires
+ *   bitlogic_head_loss_workspace(B, C) <= 8 MiB (about B * C <= 1M) and
+ *   returns BITLOGIC_ERR_TOO_LARGE otherwise, launching nothing.
+ *   The first call on a device looks up the array's device address (a
+ *   runtime query, not an allocation); make that first call before any
+ *   stream capture.  All calls share the array: calls that overlap on the
+ *   GPU (on different streams, or from different threads) race.  The array
+ *   keeps the last call's contents; nothing in it needs to start at zero. */
+int bitlogic_head_loss_noalloc(const float* Y, int32_t w, int64_t B, int32_t C, float tau,
+                               const int32_t* labels, float* logits, float* loss, float* dY,
+                               cudaStream_t stream);
 
 /* Table discretization (§3: every surrogate discretizes to a 2^n-entry
  * truth table; App. C.1 extracts it once per layer): bit a of table[j] is 1

@@ -27,7 +27,7 @@ __all__ = [
     "BitLogicError", "load", "bitlogic_encode_thermometer", "bitlogic_lut_forward",
     "bitlogic_lut_backward_workspace", "bitlogic_lut_backward", "bitlogic_lut_backward_edges",
     "bitlogic_csr_reduce", "bitlogic_lut_backward_ex", "bitlogic_head_loss_ex",
-    "bitlogic_head_loss_workspace",
+    "bitlogic_head_loss_workspace", "bitlogic_head_loss_noalloc",
     "bitlogic_head_loss", "bitlogic_binarize_tables", "bitlogic_pack_bits",
     "bitlogic_hard_forward", "bitlogic_build_csr", "bitlogic_device_error",
     "bitlogic_status_string", "bitlogic_version", "LIB_PATH",
@@ -59,6 +59,7 @@ _SIGS = {
     "bitlogic_head_loss_ex": ([_P, _I32, _I64, _I32, _F32, _P, _P, _P, _P, _P, _P, _SZ, _P],
                               ctypes.c_int),
     "bitlogic_head_loss_workspace": ([_I64, _I32], _SZ),
+    "bitlogic_head_loss_noalloc": ([_P, _I32, _I64, _I32, _F32, _P, _P, _P, _P, _P], ctypes.c_int),
     "bitlogic_head_loss": ([_P, _I32, _I64, _I32, _F32, _P, _P, _P, _P, _P, _SZ, _P],
                            ctypes.c_int),
     "bitlogic_binarize_tables": ([_P, _I32, _I32, _P, _P], ctypes.c_int),
@@ -288,6 +289,24 @@ def bitlogic_head_loss(Y: torch.Tensor, labels: torch.Tensor, C: int, tau: float
     _check("bitlogic_head_loss", load().bitlogic_head_loss(
         _ptr(Y), w, B, C, float(tau), _ptr(labels), _ptr(logits), _ptr(loss), _ptr(dY),
         _ptr(workspace), workspace.numel(), _stream(stream)))
+
+
+def bitlogic_head_loss_noalloc(Y: torch.Tensor, labels: torch.Tensor, C: int, tau: float,
+                               loss: torch.Tensor, logits: Optional[torch.Tensor] = None,
+                               dY: Optional[torch.Tensor] = None, stream=None):
+    """bitlogic_head_loss with the library's fixed scratch instead of a
+    caller workspace (for callers that cannot allocate device memory)."""
+    w, B = Y.shape
+    _need(Y, "Y", torch.float32, (w, B))
+    _need(labels, "labels", torch.int32, (B,))
+    _need(loss, "loss", torch.float32, (1,))
+    if logits is not None:
+        _need(logits, "logits", torch.float32, (B, C))
+    if dY is not None:
+        _need(dY, "dY", torch.float32, (w, B))
+    _check("bitlogic_head_loss_noalloc", load().bitlogic_head_loss_noalloc(
+        _ptr(Y), w, B, C, float(tau), _ptr(labels), _ptr(logits), _ptr(loss), _ptr(dY),
+        _stream(stream)))
 
 
 def bitlogic_binarize_tables(theta: torch.Tensor, table: torch.Tensor, stream=None):

@@ -21,6 +21,7 @@ extern "C" const char* bitlogic_status_string(int code) {
         case BITLOGIC_ERR_INDEX: return "index out of range";
         case BITLOGIC_ERR_DEVICE: return "a kernel met an out-of-range index (read as 0)";
         case BITLOGIC_ERR_THRESH: return "number of thresholds must be 1..32";
+        case BITLOGIC_ERR_TOO_LARGE: return "sizes exceed the fixed scratch of the allocation-free entry point";
         default: return "unknown status";
     }
 }

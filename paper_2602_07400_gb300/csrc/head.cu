@@ -11,6 +11,7 @@
 // dlogit/tau over each group's rows, and a single-block batch mean.  Every
 // reduction runs in a fixed order.
 #include <cfloat>
+#include <mutex>
 
 #include "common.cuh"
 
@@ -179,4 +180,52 @@ extern "C" int bitlogic_head_loss(const float* Y, int32_t w, int64_t B, int32_t 
                                   void* workspace, size_t ws_bytes, cudaStream_t stream) {
     return bitlogic_head_loss_ex(Y, w, B, C, tau, labels, logits, loss, dY, nullptr, workspace,
                                  ws_bytes, stream);
+}
+
+// ------------------------------------- allocation-free variant of the head --
+//
+// For callers that cannot allocate device memory themselves (see the header):
+// the head's workspace lives in a fixed file-scope device array instead of a
+// caller buffer.  Every GPU that loads the library reserves the array until
+// the process exits; all calls share it.
+
+namespace {
+
+constexpr size_t kNoAllocScratchBytes = (size_t)8 << 20;   // 8 MiB
+static __device__ __align__(256) unsigned char g_head_scratch[kNoAllocScratchBytes];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_scratch_mutex;
+void* g_scratch_addr[kMaxDevices] = {};
+
+// Device address of the scratch array on the current device.  The host-side
+// name g_head_scratch is only a stand-in, so the address is looked up once per
+// device (with that device current) and cached.
+int noalloc_scratch(void** out) {
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return BITLOGIC_ERR_CUDA;
+    std::lock_guard<std::mutex> lock(g_scratch_mutex);
+    if (!g_scratch_addr[dev]) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_head_scratch) != cudaSuccess || !p) return BITLOGIC_ERR_CUDA;
+        g_scratch_addr[dev] = p;
+    }
+    *out = g_scratch_addr[dev];
+    return BITLOGIC_OK;
+}
+
+}  // namespace
+
+extern "C" int bitlogic_head_loss_noalloc(const float* Y, int32_t w, int64_t B, int32_t C, float tau,
+                                          const int32_t* labels, float* logits, float* loss,
+                                          float* dY, cudaStream_t stream) {
+    if (B <= 0 || C <= 0 || B > 0x7fffffffLL / C) return BITLOGIC_ERR_SHAPE;
+    if (bitlogic_head_loss_workspace(B, C) > kNoAllocScratchBytes) return BITLOGIC_ERR_TOO_LARGE;
+    void* ws = nullptr;
+    const int st = noalloc_scratch(&ws);
+    if (st) return st;
+    // every byte of the workspace that the kernels read is written first in
+    // the same call, so nothing has to be cleared between calls
+    return bitlogic_head_loss_ex(Y, w, B, C, tau, labels, logits, loss, dY, nullptr, ws,
+                                 kNoAllocScratchBytes, stream);
 }
