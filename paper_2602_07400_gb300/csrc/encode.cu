@@ -54,27 +54,30 @@ encode_soft_kernel(const uint8_t* __restrict__ x, long long B, int d, Thresholds
 // --------------------------------------------------------------- packed --
 //
 // One lane per output word (32 samples), so every store is a coalesced
-// 128-byte run of a wire row.  A block takes 1024 samples x 32 features: the
-// raw rows (32 contiguous bytes per sample) are scattered byte by byte into a
-// feature-major shared tile in which the 32 samples of word q sit in the
-// order u' = 4 (u % 8) + u / 8, so that 32-bit register r (r < 8) of the
-// lane holds samples r, r + 8, r + 16, r + 24.  For a threshold T every
-// register yields its four comparisons v > T as the high bits of its bytes
-// by byte-wise SWAR arithmetic (no carries cross a byte):
+// 128-byte run of a wire row.  A block takes 1024 samples x 32 features and
+// stages them in a feature-major shared tile in which the 32 samples of word
+// q sit in the order u' = 4 (u % 8) + u / 8, so that 32-bit register r
+// (r < 8) of the lane holds samples r, r + 8, r + 16, r + 24.
+//
+// Fill: thread 8q + r loads the 32 feature bytes of samples 32q + r + 8j
+// (j < 4) and transposes each 4 x 4 byte block (4 samples x 4 features) with
+// two rounds of byte permutes, so that every shared store is one 32-bit
+// word: features f of samples r, r + 8, r + 16, r + 24 at tile[f][32q + 4r].
+//
+// Compare: for a threshold T every register yields its four comparisons
+// v > T as the high bits of its bytes by byte-wise SWAR arithmetic (no carry
+// crosses a byte):
 //   T < 127:  v > T  <=>  v >= 128 or (v & 127) + (127 - T) >= 128
 //   T >= 127: v > T  <=>  v >= 128 and (v & 127) + (255 - T) >= 128
-// and shifting register r's high bits right by 7 - r puts sample
-// r + 8 j at bit r + 8 j of the word.
+// and register r's high bits, moved right by 7 - r, put sample r + 8j at bit
+// r + 8j of the word.  The move is a multiply-high by 2^(25 + r), which runs
+// on the FMA pipe and leaves the logic pipe to the comparisons.
 
 constexpr int kPackWords = 32;             // words per tile (1024 samples)
 constexpr int kPackTS = kPackWords * 32;   // samples per tile
 constexpr int kPackTF = 32;                // features per tile
 constexpr int kPackWarps = 8;              // each warp: kPackTF / kPackWarps features
-
-__device__ __forceinline__ int pack_pos(int s) {   // tile position of sample s
-    const int u = s & 31;
-    return (s & ~31) | ((u & 7) << 2) | (u >> 3);
-}
+static_assert(kPackWarps * 32 == kPackWords * 8, "fill: 8 threads per word");
 
 __global__ void __launch_bounds__(kPackWarps * 32)
 pack_bits_kernel(const uint8_t* __restrict__ x, long long N, int d, Thresholds th,
@@ -91,28 +94,42 @@ pack_bits_kernel(const uint8_t* __restrict__ x, long long N, int d, Thresholds t
     const int f0 = blockIdx.x * kPackTF;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nf = min(kPackTF, d - f0);
-    // fill: thread t takes samples t, t + 256, ...; 32 feature bytes each
-    for (int sl = threadIdx.x; sl < kPackTS; sl += kPackWarps * 32) {
-        const long long s = s0 + sl;
-        uint32_t v[8];
+    {
+        const int wq = threadIdx.x >> 3, r = threadIdx.x & 7;
+        uint32_t v[4][8];   // [sample j][feature quad]
 #pragma unroll
-        for (int q = 0; q < 8; ++q) v[q] = 0u;
-        if (s < N) {
-            const uint8_t* p = x + s * d + f0;
-            if (vec16 && nf == kPackTF) {
-                const uint4 a = __ldg(reinterpret_cast<const uint4*>(p));
-                const uint4 b = __ldg(reinterpret_cast<const uint4*>(p) + 1);
-                v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
-                v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
-            } else {
+        for (int j = 0; j < 4; ++j) {
+            const long long s = s0 + 32 * wq + r + 8 * j;
 #pragma unroll
-                for (int f = 0; f < kPackTF; ++f)
-                    if (f < nf) v[f >> 2] |= (uint32_t)__ldg(p + f) << (8 * (f & 3));
+            for (int f4 = 0; f4 < 8; ++f4) v[j][f4] = 0u;
+            if (s < N) {
+                const uint8_t* p = x + s * d + f0;
+                if (vec16 && nf == kPackTF) {
+                    const uint4 a = __ldg(reinterpret_cast<const uint4*>(p));
+                    const uint4 b = __ldg(reinterpret_cast<const uint4*>(p) + 1);
+                    v[j][0] = a.x; v[j][1] = a.y; v[j][2] = a.z; v[j][3] = a.w;
+                    v[j][4] = b.x; v[j][5] = b.y; v[j][6] = b.z; v[j][7] = b.w;
+                } else {
+#pragma unroll
+                    for (int f = 0; f < kPackTF; ++f)
+                        if (f < nf) v[j][f >> 2] |= (uint32_t)__ldg(p + f) << (8 * (f & 3));
+                }
             }
         }
-        const int pos = pack_pos(sl);
+        uint32_t* dst = reinterpret_cast<uint32_t*>(&tile[0][32 * wq + 4 * r]);
+        constexpr int kRow = kPackTS / 4;   // words per tile row
 #pragma unroll
-        for (int f = 0; f < kPackTF; ++f) tile[f][pos] = (uint8_t)(v[f >> 2] >> (8 * (f & 3)));
+        for (int f4 = 0; f4 < 8; ++f4) {
+            // bytes (s0 f0, s1 f0, s0 f1, s1 f1) and (s0 f2, s1 f2, s0 f3, s1 f3), likewise s2/s3
+            const uint32_t a0 = __byte_perm(v[0][f4], v[1][f4], 0x5140);
+            const uint32_t a1 = __byte_perm(v[0][f4], v[1][f4], 0x7362);
+            const uint32_t b0 = __byte_perm(v[2][f4], v[3][f4], 0x5140);
+            const uint32_t b1 = __byte_perm(v[2][f4], v[3][f4], 0x7362);
+            dst[(4 * f4 + 0) * kRow] = __byte_perm(a0, b0, 0x5410);
+            dst[(4 * f4 + 1) * kRow] = __byte_perm(a0, b0, 0x7632);
+            dst[(4 * f4 + 2) * kRow] = __byte_perm(a1, b1, 0x5410);
+            dst[(4 * f4 + 3) * kRow] = __byte_perm(a1, b1, 0x7632);
+        }
     }
     __syncthreads();
     const long long q = (long long)blockIdx.y * kPackWords + lane;   // this lane's word
@@ -131,8 +148,8 @@ pack_bits_kernel(const uint8_t* __restrict__ x, long long N, int d, Thresholds t
 #pragma unroll
             for (int i8 = 0; i8 < 8; ++i8) {
                 const uint32_t sum = lo7[i8] + C;
-                const uint32_t hb = (r[i8] & sum) | ((r[i8] | sum) & orm);
-                word |= (hb >> (7 - i8)) & (0x01010101u << i8);
+                const uint32_t hb = ((r[i8] & sum) | ((r[i8] | sum) & orm)) & 0x80808080u;
+                word += i8 < 7 ? __umulhi(hb, 1u << ((25 + i8) & 31)) : hb;   // disjoint bits
             }
             out[(long long)i * W] = word;
         }

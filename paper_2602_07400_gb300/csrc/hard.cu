@@ -157,6 +157,115 @@ hard_layer_kernel(const uint32_t* __restrict__ xp, int w_in, long long W,
     }
 }
 
+// ------------------------------------------- staged layer (vector path) --
+//
+// The vector paths (W % 4 == 0, 16-byte aligned rows) stream the gathered
+// input words through a per-warp ring of shared-memory stages filled by
+// 16-byte cp.async copies; a stage holds the k input rows of one node over
+// 128 words.  Lane l copies, and later reads, only words 4l .. 4l + 3 of each
+// row, so the ring is lane-private: a lane waits for its own copies
+// (cp.async.wait_group) and no warp synchronisation guards the ring.  The
+// ring runs across node boundaries, so the copies of the next node are in
+// flight while the current node is evaluated, and the connectivity row and
+// table of the next node are loaded one node ahead.
+
+constexpr int kRing = 4;          // stages per warp ring
+constexpr int kStageWords = 128;  // words per stage (4 per lane)
+
+template <int k>
+__device__ __forceinline__ void issue_rows(uint4* slot, const uint32_t* __restrict__ xp, long long W,
+                                           const int (&rows)[k], long long wq) {
+#pragma unroll
+    for (int i = 0; i < k; ++i) cp_async16(slot + i * 32, xp + (long long)rows[i] * W + wq);
+}
+
+template <int k>
+__device__ __forceinline__ void read_stage(const uint4* slot, uint32_t (&x)[4][k]) {
+#pragma unroll
+    for (int i = 0; i < k; ++i) {
+        const uint4 v = slot[i * 32];
+        x[0][i] = v.x; x[1][i] = v.y; x[2][i] = v.z; x[3][i] = v.w;
+    }
+}
+
+template <int k>
+__host__ __device__ constexpr int ring_bytes_per_warp(int stages) { return stages * k * 32 * 16; }
+
+// Warp w of block b evaluates nodes jfirst, jfirst + jstride, ... (jfirst =
+// 8b + w, jstride = 8 * gridDim.x) over the block's word chunk
+// (blockIdx.y), stage by stage.
+template <int k>
+__global__ void __launch_bounds__(kHardWarps * 32, 2)
+hard_layer_staged_kernel(const uint32_t* __restrict__ xp, int w_in, long long W,
+                         const int* __restrict__ conn, const uint64_t* __restrict__ table, int w,
+                         uint32_t* __restrict__ yp, long long wchunk, uint32_t tail_mask) {
+    constexpr int H = 1 << (k - 1);
+    constexpr int kSlot = k * 32;   // uint4 per stage
+    extern __shared__ uint4 ring_smem[];
+    __shared__ __align__(16) int2 sPQ[kHardWarps][H < 2 ? 2 : H];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    uint4* ring = ring_smem + (size_t)warp * (kRing * kSlot) + lane;
+    const long long q0 = (long long)blockIdx.y * wchunk;
+    const long long q1 = min(W, q0 + wchunk);
+    const int nst = (int)((q1 - q0 + kStageWords - 1) / kStageWords);
+    const int jstride = gridDim.x * kHardWarps;
+    const int jfirst = blockIdx.x * kHardWarps + warp;
+
+    // issue stream: (node ji, stage si), kRing - 1 stages ahead of the compute stream
+    int ji = jfirst, si = 0, slot_i = 0;
+    int rows[k], rows_next[k];
+#pragma unroll
+    for (int i = 0; i < k; ++i) rows[i] = rows_next[i] = 0;
+    if (ji < w) node_rows<k>(conn, ji, w_in, lane, rows);
+    if (ji + jstride < w) node_rows<k>(conn, ji + jstride, w_in, lane, rows_next);
+    auto issue = [&]() {
+        if (ji < w) {
+            const long long wq = q0 + (long long)si * kStageWords + 4 * lane;
+            if (wq < q1) issue_rows<k>(ring + slot_i * kSlot, xp, W, rows, wq);
+            if (++si == nst) {
+                si = 0;
+                ji += jstride;
+#pragma unroll
+                for (int i = 0; i < k; ++i) rows[i] = rows_next[i];
+                if (ji + jstride < w) node_rows<k>(conn, ji + jstride, w_in, lane, rows_next);
+            }
+        }
+        cp_async_commit();
+        slot_i = slot_i + 1 == kRing ? 0 : slot_i + 1;
+    };
+#pragma unroll 1
+    for (int s = 0; s < kRing - 1; ++s) issue();
+
+    int p[H], q[H];
+    int sc = 0, slot_c = 0;
+    uint64_t tab = jfirst < w ? __ldg(table + jfirst) : 0ull;
+#pragma unroll 1
+    for (int jc = jfirst; jc < w;) {
+        if (sc == 0) {
+            node_pairs<k>(tab, lane, sPQ[warp], p, q);
+            if (jc + jstride < w) tab = __ldg(table + jc + jstride);
+        }
+        issue();
+        cp_async_wait<kRing - 1>();
+        const long long wq = q0 + (long long)sc * kStageWords + 4 * lane;
+        if (wq < q1) {
+            uint32_t x[4][k];
+            read_stage<k>(ring + slot_c * kSlot, x);
+            uint32_t y[4];
+#pragma unroll
+            for (int r = 0; r < 4; ++r) y[r] = mux_tree<k - 1, 0>(p, q, x[r]);
+            if (wq + 4 == W) y[3] &= tail_mask;   // W % 4 == 0: word W - 1 is y[3]
+            store_words<4>(yp + (long long)jc * W + wq, y);
+        }
+        slot_c = slot_c + 1 == kRing ? 0 : slot_c + 1;
+        if (++sc == nst) {
+            sc = 0;
+            jc += jstride;
+        }
+    }
+    cp_async_wait<0>();
+}
+
 // ------------------------------------------------- layer + popcount head --
 
 // Carry-save adder on bit-sliced words: (a + b + c) = 2*carry + sum.
@@ -169,10 +278,10 @@ __device__ __forceinline__ void csa(uint32_t& carry, uint32_t& sum, uint32_t a, 
 
 constexpr int kHeadWarps = 8;
 constexpr int kBigPlanes = 10;   // weight-8 planes: up to 8 * 1023 + 7 nodes per warp
-constexpr int kHeadR = 2;        // words per lane in the head kernel
 
-// grid.x: groups of 32 * kHeadR words, grid.y: class c x split.  Lane l
-// covers words kHeadR * l .. kHeadR * l + kHeadR - 1 of the group.  Warp r of
+// Scalar path (any W and alignment).  grid.x: groups of 32 * R words,
+// grid.y: class c x split.  Lane l covers words R * l .. R * l + R - 1 of
+// the group.  Warp r of
 // a block takes nodes n0 + r, n0 + r + 8, ... of its slice and feeds their
 // output words, eight nodes at a time, through a Harley-Seal carry-save tree
 // into per-lane bit-sliced counters.  At the end every lane turns its
@@ -274,6 +383,169 @@ hard_head_kernel(const uint32_t* __restrict__ xp, int w_in, long long W, long lo
     }
 }
 
+// ------------------------------------------- staged head (vector path) --
+//
+// grid.x: class c x split (fast), grid.y: groups of 128 words, so that the
+// blocks in flight share a few word groups and the gathered slice of the
+// layer input (w_in rows x 128 words) stays in L2.  Warp r of a block takes
+// nodes n0 + r, n0 + r + kHSWarps, ... of its slice; one ring stage holds one
+// node's k rows over the block's 128 words (4 words per lane).  The node
+// outputs feed, four nodes at a time, a carry-save tree into per-lane
+// bit-sliced counters (ones, twos, then kHeadNB ripple planes of weight 4,
+// 8, ...).  At the end the warps' counters are added bit-sliced in shared
+// memory, each lane turns one bit column into a per-sample count, and one
+// integer atomicAdd per (sample, class) publishes the block's total (exact
+// and order-independent).
+
+constexpr int kHSWarps = 6;     // warps per block of the staged head
+constexpr int kHeadNB = 5;      // weight-4 planes: up to 4 * 31 + 3 = 127 nodes per warp
+constexpr int kHeadPlanes = 2 + kHeadNB;
+constexpr int kSumPlanes = kHeadPlanes + 3;   // sum of kHSWarps <= 8 warps' counts
+constexpr int kMaxNodesPerWarp = 4 * ((1 << kHeadNB) - 1) + 3;
+static_assert(kHSWarps <= 8, "kSumPlanes assumes at most 8 warps");
+
+template <int k>
+__host__ __device__ constexpr int head_smem_bytes() {
+    const int ring = kHSWarps * ring_bytes_per_warp<k>(kRing);
+    const int flush = (kHSWarps * kHeadPlanes + kSumPlanes) * kStageWords * 4;
+    return ring > flush ? ring : flush;
+}
+
+template <int k>
+__global__ void __launch_bounds__(kHSWarps * 32, 2)
+hard_head_staged_kernel(const uint32_t* __restrict__ xp, int w_in, long long W, long long N,
+                        const int* __restrict__ conn, const uint64_t* __restrict__ table,
+                        int C, int g, int splits, int per_split, uint32_t* __restrict__ yp,
+                        int* __restrict__ counts, uint32_t tail_mask) {
+    constexpr int H = 1 << (k - 1);
+    constexpr int kSlot = k * 32;   // uint4 per stage
+    extern __shared__ uint4 ring_smem[];
+    __shared__ __align__(16) int2 sPQ[kHSWarps][H < 2 ? 2 : H];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int c = blockIdx.x / splits, sp = blockIdx.x - c * splits;
+    const int n0 = c * g + sp * per_split;
+    const int n1 = min(c * g + g, n0 + per_split);
+    const long long wq = (long long)blockIdx.y * kStageWords + 4 * lane;   // this lane's 4 words
+    const bool active = wq < W;   // W % 4 == 0: all four words are in range
+    uint4* ring = ring_smem + (size_t)warp * (kRing * kSlot) + lane;
+    const int jfirst = n0 + warp;
+
+    // issue stream: node ji, kRing - 1 nodes ahead of the compute stream
+    int ji = jfirst, slot_i = 0;
+    int rows[k], rows_next[k];
+#pragma unroll
+    for (int i = 0; i < k; ++i) rows[i] = rows_next[i] = 0;
+    if (ji < n1) node_rows<k>(conn, ji, w_in, lane, rows);
+    if (ji + kHSWarps < n1) node_rows<k>(conn, ji + kHSWarps, w_in, lane, rows_next);
+    auto issue = [&]() {
+        if (ji < n1) {
+            if (active) issue_rows<k>(ring + slot_i * kSlot, xp, W, rows, wq);
+            ji += kHSWarps;
+#pragma unroll
+            for (int i = 0; i < k; ++i) rows[i] = rows_next[i];
+            if (ji + kHSWarps < n1) node_rows<k>(conn, ji + kHSWarps, w_in, lane, rows_next);
+        }
+        cp_async_commit();
+        slot_i = slot_i + 1 == kRing ? 0 : slot_i + 1;
+    };
+#pragma unroll 1
+    for (int s = 0; s < kRing - 1; ++s) issue();
+
+    uint32_t ones[4], twos[4], big[kHeadNB][4];
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+        ones[r] = twos[r] = 0;
+#pragma unroll
+        for (int b = 0; b < kHeadNB; ++b) big[b][r] = 0;
+    }
+    int p[H], q[H];
+    int slot_c = 0;
+    uint64_t tab = jfirst < n1 ? __ldg(table + jfirst) : 0ull;
+    // one node: its four output words (0 past the slice or the words)
+    auto node = [&](int j, uint32_t (&y)[4]) {
+#pragma unroll
+        for (int r = 0; r < 4; ++r) y[r] = 0;
+        if (j >= n1) return;
+        node_pairs<k>(tab, lane, sPQ[warp], p, q);
+        if (j + kHSWarps < n1) tab = __ldg(table + j + kHSWarps);
+        issue();
+        cp_async_wait<kRing - 1>();
+        if (active) {
+            uint32_t x[4][k];
+            read_stage<k>(ring + slot_c * kSlot, x);
+#pragma unroll
+            for (int r = 0; r < 4; ++r) y[r] = mux_tree<k - 1, 0>(p, q, x[r]);
+            if (wq + 4 == W) y[3] &= tail_mask;
+            if (yp) store_words<4>(yp + (long long)j * W + wq, y);
+        }
+        slot_c = slot_c + 1 == kRing ? 0 : slot_c + 1;
+    };
+#pragma unroll 1
+    for (int j = jfirst; j < n1; j += 4 * kHSWarps) {
+        uint32_t ya[4], yb[4], t1[4];
+        node(j, ya);
+        node(j + kHSWarps, yb);
+#pragma unroll
+        for (int r = 0; r < 4; ++r) csa(t1[r], ones[r], ones[r], ya[r], yb[r]);
+        node(j + 2 * kHSWarps, ya);
+        node(j + 3 * kHSWarps, yb);
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+            uint32_t t2, e;
+            csa(t2, ones[r], ones[r], ya[r], yb[r]);
+            csa(e, twos[r], twos[r], t1[r], t2);
+#pragma unroll
+            for (int b = 0; b < kHeadNB; ++b) {   // ripple-add the weight-4 word
+                const uint32_t cy = big[b][r] & e;
+                big[b][r] ^= e;
+                e = cy;
+            }
+        }
+    }
+    cp_async_wait<0>();
+    __syncthreads();   // every warp is done with its ring: reuse it for the flush
+
+    // planes [warp][plane][word], then the block sum [plane][word]
+    uint32_t* pl = reinterpret_cast<uint32_t*>(ring_smem);
+    uint32_t* sum = pl + kHSWarps * kHeadPlanes * kStageWords;
+    {
+        uint4* mine = reinterpret_cast<uint4*>(pl + warp * kHeadPlanes * kStageWords) + lane;
+        mine[0] = make_uint4(ones[0], ones[1], ones[2], ones[3]);
+        mine[kStageWords / 4] = make_uint4(twos[0], twos[1], twos[2], twos[3]);
+#pragma unroll
+        for (int b = 0; b < kHeadNB; ++b)
+            mine[(2 + b) * (kStageWords / 4)] = make_uint4(big[b][0], big[b][1], big[b][2], big[b][3]);
+    }
+    __syncthreads();
+    if (threadIdx.x < kStageWords) {
+        const int wd = threadIdx.x;
+        uint32_t a[kSumPlanes];
+#pragma unroll
+        for (int pp = 0; pp < kSumPlanes; ++pp) a[pp] = pp < kHeadPlanes ? pl[pp * kStageWords + wd] : 0u;
+#pragma unroll
+        for (int wr = 1; wr < kHSWarps; ++wr) {   // bit-sliced ripple-carry add of warp wr
+            uint32_t cy = 0;
+#pragma unroll
+            for (int pp = 0; pp < kSumPlanes; ++pp) {
+                const uint32_t b = pp < kHeadPlanes ? pl[(wr * kHeadPlanes + pp) * kStageWords + wd] : 0u;
+                const uint32_t ao = a[pp], u = ao ^ b;
+                a[pp] = u ^ cy;
+                cy = (ao & b) | (u & cy);
+            }
+        }
+#pragma unroll
+        for (int pp = 0; pp < kSumPlanes; ++pp) sum[pp * kStageWords + wd] = a[pp];
+    }
+    __syncthreads();
+    for (int wd = warp; wd < kStageWords; wd += kHSWarps) {
+        int cnt = 0;
+#pragma unroll
+        for (int pp = 0; pp < kSumPlanes; ++pp) cnt |= (int)((sum[pp * kStageWords + wd] >> lane) & 1u) << pp;
+        const long long s = ((long long)blockIdx.y * kStageWords + wd) * 32 + lane;
+        if (cnt && s < N) atomicAdd(counts + s * C + c, cnt);
+    }
+}
+
 __global__ void __launch_bounds__(256)
 argmax_kernel(const int* __restrict__ counts, long long N, int C, int* __restrict__ pred) {
     const long long s = (long long)blockIdx.x * 256 + threadIdx.x;
@@ -298,48 +570,83 @@ long long hard_word_chunk(int w_in, long long W) {
     return c < W ? c : W;
 }
 
+int sm_count() {
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+        return 152;
+    return n;
+}
+
+template <typename F>
+int set_dynamic_smem(F* kernel, int bytes) {
+    if (bytes <= 48 * 1024) return BITLOGIC_OK;
+    return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) == cudaSuccess
+               ? BITLOGIC_OK : BITLOGIC_ERR_CUDA;
+}
+
 template <int k>
 int launch_hard(const uint32_t* xp, int w_in, long long N, const int* conn, const uint64_t* table,
                 int w, uint32_t* yp, int C, int* counts, int* pred, cudaStream_t st) {
     const long long W = (N + 31) / 32;
     const uint32_t tail_mask = (N % 32) ? ((1u << (N % 32)) - 1u) : 0xffffffffu;
+    const bool vec4 = (W % 4 == 0) && aligned16(xp) && (!yp || aligned16(yp));
     if (C == 0) {
-        const bool vec = (W % 4 == 0) && aligned16(xp) && aligned16(yp);
         const long long chunk = hard_word_chunk(w_in, W);
         const long long ny = (W + chunk - 1) / chunk;
         if (ny > 65535) return BITLOGIC_ERR_SHAPE;
-        dim3 grid((unsigned)((w + kHardWarps - 1) / kHardWarps), (unsigned)ny);
-        if (vec)
-            hard_layer_kernel<k, 4><<<grid, kHardWarps * 32, 0, st>>>(xp, w_in, W, conn, table, w, yp, chunk, tail_mask);
-        else
-            hard_layer_kernel<k, 1><<<grid, kHardWarps * 32, 0, st>>>(xp, w_in, W, conn, table, w, yp, chunk, tail_mask);
+        if (vec4) {
+            // nodes per warp: enough blocks for about four waves of two per SM
+            const long long groups = (w + kHardWarps - 1) / kHardWarps;
+            long long npw = groups * ny / (8ll * sm_count());
+            npw = npw < 1 ? 1 : (npw > 8 ? 8 : npw);
+            const long long gx = (w + kHardWarps * npw - 1) / (kHardWarps * npw);
+            const int smem = kHardWarps * ring_bytes_per_warp<k>(kRing);
+            if (set_dynamic_smem(hard_layer_staged_kernel<k>, smem)) return BITLOGIC_ERR_CUDA;
+            hard_layer_staged_kernel<k><<<dim3((unsigned)gx, (unsigned)ny), kHardWarps * 32, smem, st>>>(
+                xp, w_in, W, conn, table, w, yp, chunk, tail_mask);
+        } else {
+            dim3 grid((unsigned)((w + kHardWarps - 1) / kHardWarps), (unsigned)ny);
+            hard_layer_kernel<k, 1><<<grid, kHardWarps * 32, 0, st>>>(xp, w_in, W, conn, table, w, yp, chunk,
+                                                                     tail_mask);
+        }
         return launch_status();
     }
     const int g = w / C;
-    const bool vec = (W % kHeadR == 0) && ((reinterpret_cast<uintptr_t>(xp) & 7u) == 0) &&
-                     (!yp || (reinterpret_cast<uintptr_t>(yp) & 7u) == 0);
-    const int R = vec ? kHeadR : 1;
-    const long long wg = (W + 32 * R - 1) / (32 * R);
-    // split a class over several blocks when there are few word groups, so
-    // that at least ~4 blocks per SM are in flight
-    int splits = 1;
-    while (wg * C * splits < 608 && g / (splits * 2) >= 64) splits *= 2;
-    int per_split = (g + splits - 1) / splits;
-    // each warp's slice must fit the counters
-    while ((per_split + kHeadWarps - 1) / kHeadWarps > 8 * ((1 << kBigPlanes) - 1)) {
-        splits *= 2;
-        per_split = (g + splits - 1) / splits;
-    }
-    if ((long long)C * splits > 65535) return BITLOGIC_ERR_SHAPE;
     if (cudaMemsetAsync(counts, 0, sizeof(int) * (size_t)N * (size_t)C, st) != cudaSuccess)
         return BITLOGIC_ERR_CUDA;
-    dim3 grid((unsigned)wg, (unsigned)(C * splits));
-    if (vec)
-        hard_head_kernel<k, kHeadR><<<grid, kHeadWarps * 32, 0, st>>>(xp, w_in, W, N, conn, table, C, g, splits,
-                                                                      per_split, yp, counts, tail_mask);
-    else
+    if (vec4) {
+        const long long wg = W / kStageWords + (W % kStageWords ? 1 : 0);
+        // split a class over several blocks until a word group has about one
+        // block per SM (the blocks in flight then share one or two word
+        // groups), keeping at least 8 nodes per warp
+        int splits = 1;
+        while (C * splits < sm_count() && g / (splits * 2) >= 8 * kHSWarps) splits *= 2;
+        int per_split = (g + splits - 1) / splits;
+        while ((per_split + kHSWarps - 1) / kHSWarps > kMaxNodesPerWarp) {   // counter capacity
+            splits *= 2;
+            per_split = (g + splits - 1) / splits;
+        }
+        if ((long long)C * splits > 0x7fffffffll || wg > 65535) return BITLOGIC_ERR_SHAPE;
+        const int smem = head_smem_bytes<k>();
+        if (set_dynamic_smem(hard_head_staged_kernel<k>, smem)) return BITLOGIC_ERR_CUDA;
+        hard_head_staged_kernel<k><<<dim3((unsigned)(C * splits), (unsigned)wg), kHSWarps * 32, smem, st>>>(
+            xp, w_in, W, N, conn, table, C, g, splits, per_split, yp, counts, tail_mask);
+    } else {
+        const long long wg = (W + 31) / 32;
+        int splits = 1;
+        while (wg * C * splits < 608 && g / (splits * 2) >= 64) splits *= 2;
+        int per_split = (g + splits - 1) / splits;
+        // each warp's slice must fit the counters
+        while ((per_split + kHeadWarps - 1) / kHeadWarps > 8 * ((1 << kBigPlanes) - 1)) {
+            splits *= 2;
+            per_split = (g + splits - 1) / splits;
+        }
+        if ((long long)C * splits > 65535) return BITLOGIC_ERR_SHAPE;
+        dim3 grid((unsigned)wg, (unsigned)(C * splits));
         hard_head_kernel<k, 1><<<grid, kHeadWarps * 32, 0, st>>>(xp, w_in, W, N, conn, table, C, g, splits,
-                                                                 per_split, yp, counts, tail_mask);
+                                                                per_split, yp, counts, tail_mask);
+    }
     if (pred) argmax_kernel<<<(unsigned)((N + 255) / 256), 256, 0, st>>>(counts, N, C, pred);
     return launch_status();
 }

@@ -207,17 +207,6 @@ __device__ __forceinline__ void node_setup(const int* __restrict__ conn,
     __syncwarp();
 }
 
-// ---------------------------------------------------- async copy helpers --
-
-// Asynchronous 16-byte global -> shared copies (L2 only), grouped per stage.
-__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
-    const unsigned s = (unsigned)__cvta_generic_to_shared(smem);
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(s), "l"(gmem) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
-
 #ifndef BITLOGIC_STAGE_SAMPLES
 #define BITLOGIC_STAGE_SAMPLES 128
 #endif

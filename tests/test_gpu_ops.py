@@ -281,6 +281,7 @@ def test_pack_bits(N, d, b):
 HARD = [  # (k, w_in, w, N)
     (1, 3, 5, 1), (2, 10, 9, 31), (3, 40, 33, 33), (4, 100, 65, 1000), (5, 64, 100, 1025),
     (6, 300, 129, 4096), (6, 7, 20, 70001), (6, 2000, 256, 100000),
+    (6, 16384, 300, 32891),   # staged path over two word chunks (768 + 260 words)
 ]
 
 
