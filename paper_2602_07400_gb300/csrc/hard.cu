@@ -51,12 +51,35 @@ __device__ __forceinline__ uint32_t mux_tree(const int (&p)[H], const int (&q)[H
     }
 }
 
+// The tree for four words at once with the level-0 pairs read from shared
+// memory (broadcast loads) instead of registers: depth first, so at most one
+// partial result per level and word is live.
+template <int L, int M, int k>
+__device__ __forceinline__ void mux_tree4_smem(const int2* __restrict__ sPQ, const uint32_t (&x)[4][k],
+                                               uint32_t (&out)[4]) {
+    if constexpr (L == 0) {
+        const int2 v = sPQ[M];
+#pragma unroll
+        for (int r = 0; r < 4; ++r) out[r] = (uint32_t)((int)x[r][0] * v.x + v.y);
+    } else {
+        uint32_t lo[4], hi[4];
+        mux_tree4_smem<L - 1, 2 * M, k>(sPQ, x, lo);
+        mux_tree4_smem<L - 1, 2 * M + 1, k>(sPQ, x, hi);
+#pragma unroll
+        for (int r = 0; r < 4; ++r) out[r] = (x[r][L] & hi[r]) | (~x[r][L] & lo[r]);
+    }
+}
+
 // Per-warp node set-up: lane m derives (p, q) of pair m from the table, the
-// warp shares them through shared memory.
+// warp shares them through shared memory (sPQ: 2 * 2^(k-1) ints per warp).
+#ifndef BITLOGIC_PQ_LAYOUT
+#define BITLOGIC_PQ_LAYOUT 0
+#endif
 template <int k>
 __device__ __forceinline__ void node_pairs(uint64_t T, int lane, int2* sPQ,
                                            int (&p)[1 << (k - 1)], int (&q)[1 << (k - 1)]) {
     constexpr int H = 1 << (k - 1);
+#if BITLOGIC_PQ_LAYOUT == 0
     if (lane < H) {
         const int t0 = (int)((T >> (2 * lane)) & 1u), t1 = (int)((T >> (2 * lane + 1)) & 1u);
         sPQ[lane] = make_int2(t1 - t0, -t0);
@@ -71,6 +94,57 @@ __device__ __forceinline__ void node_pairs(uint64_t T, int lane, int2* sPQ,
             const int2 v = sPQ[m];
             p[m] = v.x; q[m] = v.y;
         }
+    }
+#elif BITLOGIC_PQ_LAYOUT == 1
+    if (lane < H) {
+        const int t0 = (int)((T >> (2 * lane)) & 1u), t1 = (int)((T >> (2 * lane + 1)) & 1u);
+        sPQ[lane] = make_int2(t1 - t0, -t0);
+    }
+    __syncwarp();
+#pragma unroll
+    for (int m = 0; m < H; ++m) {
+        const int2 v = sPQ[m];
+        p[m] = v.x; q[m] = v.y;
+    }
+#else
+    int* sP = reinterpret_cast<int*>(sPQ);
+    int* sQ = sP + H;
+    if (lane < H) {
+        const int t0 = (int)((T >> (2 * lane)) & 1u), t1 = (int)((T >> (2 * lane + 1)) & 1u);
+        sP[lane] = t1 - t0;
+        sQ[lane] = -t0;
+    }
+    __syncwarp();
+#if BITLOGIC_PQ_LAYOUT == 2
+    if constexpr (H >= 4) {
+#pragma unroll
+        for (int m = 0; m < H; m += 4) {
+            const int4 a = *reinterpret_cast<const int4*>(sP + m);
+            const int4 b = *reinterpret_cast<const int4*>(sQ + m);
+            p[m] = a.x; p[m + 1] = a.y; p[m + 2] = a.z; p[m + 3] = a.w;
+            q[m] = b.x; q[m + 1] = b.y; q[m + 2] = b.z; q[m + 3] = b.w;
+        }
+    } else
+#endif
+    {
+#pragma unroll
+        for (int m = 0; m < H; ++m) {
+            p[m] = sP[m];
+            q[m] = sQ[m];
+        }
+    }
+#endif
+    __syncwarp();
+}
+
+// Pair set-up when the tree reads the pairs from shared memory: lane m
+// writes pair m; the warp synchronises before the tree reads them.
+template <int k>
+__device__ __forceinline__ void node_pairs_smem(uint64_t T, int lane, int2* sPQ) {
+    constexpr int H = 1 << (k - 1);
+    if (lane < H) {
+        const int t0 = (int)((T >> (2 * lane)) & 1u), t1 = (int)((T >> (2 * lane + 1)) & 1u);
+        sPQ[lane] = make_int2(t1 - t0, -t0);
     }
     __syncwarp();
 }
@@ -169,15 +243,7 @@ hard_layer_kernel(const uint32_t* __restrict__ xp, int w_in, long long W,
 // flight while the current node is evaluated, and the connectivity row and
 // table of the next node are loaded one node ahead.
 
-constexpr int kRing = 4;          // stages per warp ring
 constexpr int kStageWords = 128;  // words per stage (4 per lane)
-
-template <int k>
-__device__ __forceinline__ void issue_rows(uint4* slot, const uint32_t* __restrict__ xp, long long W,
-                                           const int (&rows)[k], long long wq) {
-#pragma unroll
-    for (int i = 0; i < k; ++i) cp_async16(slot + i * 32, xp + (long long)rows[i] * W + wq);
-}
 
 template <int k>
 __device__ __forceinline__ void read_stage(const uint4* slot, uint32_t (&x)[4][k]) {
@@ -191,79 +257,135 @@ __device__ __forceinline__ void read_stage(const uint4* slot, uint32_t (&x)[4][k
 template <int k>
 __host__ __device__ constexpr int ring_bytes_per_warp(int stages) { return stages * k * 32 * 16; }
 
-// Warp w of block b evaluates nodes jfirst, jfirst + jstride, ... (jfirst =
-// 8b + w, jstride = 8 * gridDim.x) over the block's word chunk
-// (blockIdx.y), stage by stage.
+// A node's k input rows as 32-bit offsets, in 16-byte units from the start
+// of the packed input, of the lane's first words: (row * W + wl) / 4.  The
+// launchers use the staged kernels only when w_in * W / 4 < 2^32.
 template <int k>
-__global__ void __launch_bounds__(kHardWarps * 32, 2)
-hard_layer_staged_kernel(const uint32_t* __restrict__ xp, int w_in, long long W,
-                         const int* __restrict__ conn, const uint64_t* __restrict__ table, int w,
-                         uint32_t* __restrict__ yp, long long wchunk, uint32_t tail_mask) {
+__device__ __forceinline__ void node_offsets(const int* __restrict__ conn, int j, int w_in, int lane,
+                                             uint32_t W4, uint32_t wl4, uint32_t (&off)[k]) {
+    int rows[k];
+    node_rows<k>(conn, j, w_in, lane, rows);
+#pragma unroll
+    for (int i = 0; i < k; ++i) off[i] = (uint32_t)rows[i] * W4 + wl4;
+}
+
+// Copies of one stage (the lane's 16 bytes of each of the k rows, `s16`
+// 16-byte units past the node's offsets) into a ring slot.
+template <int k>
+__device__ __forceinline__ void issue_stage(uint4* slot, const uint4* __restrict__ xp4,
+                                            const uint32_t (&off)[k], uint32_t s16) {
+#pragma unroll
+    for (int i = 0; i < k; ++i) cp_async16(slot + i * 32, xp4 + (off[i] + s16));
+}
+
+// Three stages per node and warp ring, three blocks per SM: the level-0
+// pairs are read from shared memory (80 registers per thread), so 24 warps
+// per SM hide the latency of the half-rate logic pipe.
+#ifndef BITLOGIC_HARD_NS
+#define BITLOGIC_HARD_NS 3
+#endif
+#ifndef BITLOGIC_HARD_MINB
+#define BITLOGIC_HARD_MINB 3
+#endif
+constexpr int kLayerNS = BITLOGIC_HARD_NS;       // stages per node = ring slots per warp
+constexpr int kLayerMinBlocks = BITLOGIC_HARD_MINB;
+
+// Warp w of block b evaluates nodes j = 8b + w, j + jstride, ... (jstride =
+// 8 * gridDim.x) over the block's chunk of NS * 128 words (blockIdx.y).  A
+// node is exactly NS stages and the warp's ring has NS slots, so stage s of
+// every node lives in slot s and all slot offsets are compile-time
+// constants: while stage s of node j is evaluated, the copies of stage
+// s + NS - 1 (the last stage of node j, or stage s - 1 of the warp's next
+// node) are in flight.  FULL: the chunk lies inside the words and holds no
+// partial tail word, so no lane checks.
+template <int k, int NS, bool FULL>
+__device__ __forceinline__ void layer_staged_body(const uint4* __restrict__ xp4, int w_in, long long W,
+                                                  const int* __restrict__ conn,
+                                                  const uint64_t* __restrict__ table, int w,
+                                                  uint32_t* __restrict__ yp, uint32_t tail_mask,
+                                                  uint4* ring_smem, int2* sPQ) {
     constexpr int H = 1 << (k - 1);
     constexpr int kSlot = k * 32;   // uint4 per stage
-    extern __shared__ uint4 ring_smem[];
-    __shared__ __align__(16) int2 sPQ[kHardWarps][H < 2 ? 2 : H];
+    static_assert(NS >= 2, "at least one stage in flight");
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    uint4* ring = ring_smem + (size_t)warp * (kRing * kSlot) + lane;
-    const long long q0 = (long long)blockIdx.y * wchunk;
-    const long long q1 = min(W, q0 + wchunk);
-    const int nst = (int)((q1 - q0 + kStageWords - 1) / kStageWords);
+    uint4* ring = ring_smem + (size_t)warp * (NS * kSlot) + lane;
+    const long long wl = (long long)blockIdx.y * (NS * kStageWords) + 4 * lane;   // stage 0 words
+    const uint32_t W4 = (uint32_t)(W >> 2), wl4 = (uint32_t)(wl >> 2);
     const int jstride = gridDim.x * kHardWarps;
-    const int jfirst = blockIdx.x * kHardWarps + warp;
+    int j = blockIdx.x * kHardWarps + warp;
 
-    // issue stream: (node ji, stage si), kRing - 1 stages ahead of the compute stream
-    int ji = jfirst, si = 0, slot_i = 0;
-    int rows[k], rows_next[k];
+    uint32_t oc[k], on[k];   // row offsets of node j and of node j + jstride
 #pragma unroll
-    for (int i = 0; i < k; ++i) rows[i] = rows_next[i] = 0;
-    if (ji < w) node_rows<k>(conn, ji, w_in, lane, rows);
-    if (ji + jstride < w) node_rows<k>(conn, ji + jstride, w_in, lane, rows_next);
-    auto issue = [&]() {
-        if (ji < w) {
-            const long long wq = q0 + (long long)si * kStageWords + 4 * lane;
-            if (wq < q1) issue_rows<k>(ring + slot_i * kSlot, xp, W, rows, wq);
-            if (++si == nst) {
-                si = 0;
-                ji += jstride;
+    for (int i = 0; i < k; ++i) oc[i] = on[i] = 0;
+    if (j < w) node_offsets<k>(conn, j, w_in, lane, W4, wl4, oc);
+    if (j + jstride < w) node_offsets<k>(conn, j + jstride, w_in, lane, W4, wl4, on);
+    // stage s of a node into slot s (W % 4 == 0: a lane's four words are all
+    // in range or all out); one commit group per stage
+    auto issue = [&](const uint32_t (&off)[k], int node, int s) {
+        bool ok = node < w;
+        if constexpr (!FULL) ok = ok && wl + s * kStageWords < W;
+        if (ok) issue_stage<k>(ring + s * kSlot, xp4, off, (uint32_t)(s * kStageWords / 4));
+        cp_async_commit();
+    };
 #pragma unroll
-                for (int i = 0; i < k; ++i) rows[i] = rows_next[i];
-                if (ji + jstride < w) node_rows<k>(conn, ji + jstride, w_in, lane, rows_next);
+    for (int s = 0; s < NS - 1; ++s) issue(oc, j, s);
+    uint64_t tab = j < w ? __ldg(table + j) : 0ull;
+#pragma unroll 1
+    for (; j < w; j += jstride) {
+        node_pairs_smem<k>(tab, lane, sPQ);
+        const int jn = j + jstride;
+        if (jn < w) tab = __ldg(table + jn);
+        uint32_t* out = yp + (long long)j * W + wl;
+#pragma unroll
+        for (int s = 0; s < NS; ++s) {
+            if (s == 0) {
+                issue(oc, j, NS - 1);
+                if (jn + jstride < w) node_offsets<k>(conn, jn + jstride, w_in, lane, W4, wl4, oc);
+            } else {
+                issue(on, jn, s - 1);
+            }
+            cp_async_wait<NS - 1>();
+            bool ok = true;
+            if constexpr (!FULL) ok = wl + s * kStageWords < W;
+            if (ok) {
+                uint32_t x[4][k];
+                read_stage<k>(ring + s * kSlot, x);
+                uint32_t y[4];
+                mux_tree4_smem<k - 1, 0, k>(sPQ, x, y);
+                if constexpr (!FULL) {
+                    if (wl + s * kStageWords + 4 == W) y[3] &= tail_mask;   // word W - 1 is y[3]
+                }
+                store_words<4>(out + s * kStageWords, y);
             }
         }
-        cp_async_commit();
-        slot_i = slot_i + 1 == kRing ? 0 : slot_i + 1;
-    };
-#pragma unroll 1
-    for (int s = 0; s < kRing - 1; ++s) issue();
-
-    int p[H], q[H];
-    int sc = 0, slot_c = 0;
-    uint64_t tab = jfirst < w ? __ldg(table + jfirst) : 0ull;
-#pragma unroll 1
-    for (int jc = jfirst; jc < w;) {
-        if (sc == 0) {
-            node_pairs<k>(tab, lane, sPQ[warp], p, q);
-            if (jc + jstride < w) tab = __ldg(table + jc + jstride);
-        }
-        issue();
-        cp_async_wait<kRing - 1>();
-        const long long wq = q0 + (long long)sc * kStageWords + 4 * lane;
-        if (wq < q1) {
-            uint32_t x[4][k];
-            read_stage<k>(ring + slot_c * kSlot, x);
-            uint32_t y[4];
+        __syncwarp();   // the pairs are read before the next node rewrites them
 #pragma unroll
-            for (int r = 0; r < 4; ++r) y[r] = mux_tree<k - 1, 0>(p, q, x[r]);
-            if (wq + 4 == W) y[3] &= tail_mask;   // W % 4 == 0: word W - 1 is y[3]
-            store_words<4>(yp + (long long)jc * W + wq, y);
-        }
-        slot_c = slot_c + 1 == kRing ? 0 : slot_c + 1;
-        if (++sc == nst) {
-            sc = 0;
-            jc += jstride;
+        for (int i = 0; i < k; ++i) {
+            const uint32_t t = oc[i];
+            oc[i] = on[i];
+            on[i] = t;
         }
     }
     cp_async_wait<0>();
+}
+
+template <int k>
+__global__ void __launch_bounds__(kHardWarps * 32, kLayerMinBlocks)
+hard_layer_staged_kernel(const uint4* __restrict__ xp4, int w_in, long long W,
+                         const int* __restrict__ conn, const uint64_t* __restrict__ table, int w,
+                         uint32_t* __restrict__ yp, uint32_t tail_mask) {
+    constexpr int H = 1 << (k - 1);
+    extern __shared__ uint4 ring_smem[];
+    __shared__ __align__(16) int2 sPQ[kHardWarps][H < 2 ? 2 : H];
+    const long long end = (long long)(blockIdx.y + 1) * (kLayerNS * kStageWords);
+    const bool full = end < W || (end == W && tail_mask == 0xffffffffu);
+    int2* mine = sPQ[threadIdx.x >> 5];
+    if (full)
+        layer_staged_body<k, kLayerNS, true>(xp4, w_in, W, conn, table, w, yp, tail_mask,
+                                              ring_smem, mine);
+    else
+        layer_staged_body<k, kLayerNS, false>(xp4, w_in, W, conn, table, w, yp, tail_mask,
+                                                         ring_smem, mine);
 }
 
 // ------------------------------------------------- layer + popcount head --
@@ -389,7 +511,9 @@ hard_head_kernel(const uint32_t* __restrict__ xp, int w_in, long long W, long lo
 // blocks in flight share a few word groups and the gathered slice of the
 // layer input (w_in rows x 128 words) stays in L2.  Warp r of a block takes
 // nodes n0 + r, n0 + r + kHSWarps, ... of its slice; one ring stage holds one
-// node's k rows over the block's 128 words (4 words per lane).  The node
+// node's k rows over the block's 128 words (4 words per lane), and the
+// node's level-0 pairs are read from shared memory (broadcast loads), which
+// keeps the kernel at 128 registers and 16 warps per SM.  The node
 // outputs feed, four nodes at a time, a carry-save tree into per-lane
 // bit-sliced counters (ones, twos, then kHeadNB ripple planes of weight 4,
 // 8, ...).  At the end the warps' counters are added bit-sliced in shared
@@ -397,7 +521,15 @@ hard_head_kernel(const uint32_t* __restrict__ xp, int w_in, long long W, long lo
 // integer atomicAdd per (sample, class) publishes the block's total (exact
 // and order-independent).
 
-constexpr int kHSWarps = 6;     // warps per block of the staged head
+#ifndef BITLOGIC_HEAD_WARPS
+#define BITLOGIC_HEAD_WARPS 8
+#endif
+#ifndef BITLOGIC_HEAD_MINB
+#define BITLOGIC_HEAD_MINB 2
+#endif
+constexpr int kHeadMinBlocks = BITLOGIC_HEAD_MINB;
+constexpr int kHeadRing = 4;      // node stages per warp ring
+constexpr int kHSWarps = BITLOGIC_HEAD_WARPS;     // warps per block of the staged head
 constexpr int kHeadNB = 5;      // weight-4 planes: up to 4 * 31 + 3 = 127 nodes per warp
 constexpr int kHeadPlanes = 2 + kHeadNB;
 constexpr int kSumPlanes = kHeadPlanes + 3;   // sum of kHSWarps <= 8 warps' counts
@@ -406,51 +538,51 @@ static_assert(kHSWarps <= 8, "kSumPlanes assumes at most 8 warps");
 
 template <int k>
 __host__ __device__ constexpr int head_smem_bytes() {
-    const int ring = kHSWarps * ring_bytes_per_warp<k>(kRing);
+    const int ring = kHSWarps * ring_bytes_per_warp<k>(kHeadRing);
     const int flush = (kHSWarps * kHeadPlanes + kSumPlanes) * kStageWords * 4;
     return ring > flush ? ring : flush;
 }
 
-template <int k>
-__global__ void __launch_bounds__(kHSWarps * 32, 2)
-hard_head_staged_kernel(const uint32_t* __restrict__ xp, int w_in, long long W, long long N,
-                        const int* __restrict__ conn, const uint64_t* __restrict__ table,
-                        int C, int g, int splits, int per_split, uint32_t* __restrict__ yp,
-                        int* __restrict__ counts, uint32_t tail_mask) {
+template <int k, bool FULL>
+__device__ __forceinline__ void head_staged_body(const uint4* __restrict__ xp4, int w_in, long long W,
+                                                 long long N, const int* __restrict__ conn,
+                                                 const uint64_t* __restrict__ table, int C, int g,
+                                                 int splits, int per_split, uint32_t* __restrict__ yp,
+                                                 int* __restrict__ counts, uint32_t tail_mask,
+                                                 uint4* ring_smem, int2* sPQ) {
     constexpr int H = 1 << (k - 1);
     constexpr int kSlot = k * 32;   // uint4 per stage
-    extern __shared__ uint4 ring_smem[];
-    __shared__ __align__(16) int2 sPQ[kHSWarps][H < 2 ? 2 : H];
+    static_assert(kHeadRing == 4, "a loop iteration is kHeadRing node steps");
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int c = blockIdx.x / splits, sp = blockIdx.x - c * splits;
     const int n0 = c * g + sp * per_split;
     const int n1 = min(c * g + g, n0 + per_split);
     const long long wq = (long long)blockIdx.y * kStageWords + 4 * lane;   // this lane's 4 words
-    const bool active = wq < W;   // W % 4 == 0: all four words are in range
-    uint4* ring = ring_smem + (size_t)warp * (kRing * kSlot) + lane;
+    const bool active = FULL || wq < W;   // W % 4 == 0: all four words are in range
+    const uint32_t W4 = (uint32_t)(W >> 2), wq4 = (uint32_t)(wq >> 2);
+    uint4* ring = ring_smem + (size_t)warp * (kHeadRing * kSlot) + lane;
     const int jfirst = n0 + warp;
 
-    // issue stream: node ji, kRing - 1 nodes ahead of the compute stream
-    int ji = jfirst, slot_i = 0;
-    int rows[k], rows_next[k];
+    // issue stream: node ji, kHeadRing - 1 nodes ahead of the compute stream
+    int ji = jfirst;
+    uint32_t oi[k], on[k];   // row offsets of node ji and of the warp's node after it
 #pragma unroll
-    for (int i = 0; i < k; ++i) rows[i] = rows_next[i] = 0;
-    if (ji < n1) node_rows<k>(conn, ji, w_in, lane, rows);
-    if (ji + kHSWarps < n1) node_rows<k>(conn, ji + kHSWarps, w_in, lane, rows_next);
-    auto issue = [&]() {
+    for (int i = 0; i < k; ++i) oi[i] = on[i] = 0;
+    if (ji < n1) node_offsets<k>(conn, ji, w_in, lane, W4, wq4, oi);
+    if (ji + kHSWarps < n1) node_offsets<k>(conn, ji + kHSWarps, w_in, lane, W4, wq4, on);
+    auto issue = [&](int slot) {
         if (ji < n1) {
-            if (active) issue_rows<k>(ring + slot_i * kSlot, xp, W, rows, wq);
+            if (active) issue_stage<k>(ring + slot * kSlot, xp4, oi, 0u);
             ji += kHSWarps;
 #pragma unroll
-            for (int i = 0; i < k; ++i) rows[i] = rows_next[i];
-            if (ji + kHSWarps < n1) node_rows<k>(conn, ji + kHSWarps, w_in, lane, rows_next);
+            for (int i = 0; i < k; ++i) oi[i] = on[i];
+            if (ji + kHSWarps < n1) node_offsets<k>(conn, ji + kHSWarps, w_in, lane, W4, wq4, on);
         }
         cp_async_commit();
-        slot_i = slot_i + 1 == kRing ? 0 : slot_i + 1;
     };
-#pragma unroll 1
-    for (int s = 0; s < kRing - 1; ++s) issue();
-
+    issue(0);
+    issue(1);
+    issue(2);
     uint32_t ones[4], twos[4], big[kHeadNB][4];
 #pragma unroll
     for (int r = 0; r < 4; ++r) {
@@ -458,37 +590,37 @@ hard_head_staged_kernel(const uint32_t* __restrict__ xp, int w_in, long long W, 
 #pragma unroll
         for (int b = 0; b < kHeadNB; ++b) big[b][r] = 0;
     }
-    int p[H], q[H];
-    int slot_c = 0;
     uint64_t tab = jfirst < n1 ? __ldg(table + jfirst) : 0ull;
-    // one node: its four output words (0 past the slice or the words)
-    auto node = [&](int j, uint32_t (&y)[4]) {
+    // node step u of a loop iteration (node jj): the loop body has kHeadRing
+    // steps, so step u reads slot u and refills slot u + 3 (mod kHeadRing).
+    // Returns the node's four output words (0 past the slice or the words).
+    auto node = [&](int jj, int u, uint32_t (&y)[4]) {
+        __syncwarp();   // the previous node's pairs are read
+        node_pairs_smem<k>(tab, lane, sPQ);   // table 0 past the slice: harmless
+        tab = jj + kHSWarps < n1 ? __ldg(table + jj + kHSWarps) : 0ull;
+        issue((u + kHeadRing - 1) % kHeadRing);
+        cp_async_wait<kHeadRing - 1>();
 #pragma unroll
         for (int r = 0; r < 4; ++r) y[r] = 0;
-        if (j >= n1) return;
-        node_pairs<k>(tab, lane, sPQ[warp], p, q);
-        if (j + kHSWarps < n1) tab = __ldg(table + j + kHSWarps);
-        issue();
-        cp_async_wait<kRing - 1>();
-        if (active) {
+        if (jj < n1 && active) {
             uint32_t x[4][k];
-            read_stage<k>(ring + slot_c * kSlot, x);
-#pragma unroll
-            for (int r = 0; r < 4; ++r) y[r] = mux_tree<k - 1, 0>(p, q, x[r]);
-            if (wq + 4 == W) y[3] &= tail_mask;
-            if (yp) store_words<4>(yp + (long long)j * W + wq, y);
+            read_stage<k>(ring + u * kSlot, x);
+            mux_tree4_smem<k - 1, 0, k>(sPQ, x, y);
+            if constexpr (!FULL) {
+                if (wq + 4 == W) y[3] &= tail_mask;
+            }
+            if (yp) store_words<4>(yp + (long long)jj * W + wq, y);
         }
-        slot_c = slot_c + 1 == kRing ? 0 : slot_c + 1;
     };
 #pragma unroll 1
     for (int j = jfirst; j < n1; j += 4 * kHSWarps) {
         uint32_t ya[4], yb[4], t1[4];
-        node(j, ya);
-        node(j + kHSWarps, yb);
+        node(j, 0, ya);
+        node(j + kHSWarps, 1, yb);
 #pragma unroll
         for (int r = 0; r < 4; ++r) csa(t1[r], ones[r], ones[r], ya[r], yb[r]);
-        node(j + 2 * kHSWarps, ya);
-        node(j + 3 * kHSWarps, yb);
+        node(j + 2 * kHSWarps, 2, ya);
+        node(j + 3 * kHSWarps, 3, yb);
 #pragma unroll
         for (int r = 0; r < 4; ++r) {
             uint32_t t2, e;
@@ -546,6 +678,27 @@ hard_head_staged_kernel(const uint32_t* __restrict__ xp, int w_in, long long W, 
     }
 }
 
+
+template <int k>
+__global__ void __launch_bounds__(kHSWarps * 32, kHeadMinBlocks)
+hard_head_staged_kernel(const uint4* __restrict__ xp4, int w_in, long long W, long long N,
+                        const int* __restrict__ conn, const uint64_t* __restrict__ table,
+                        int C, int g, int splits, int per_split, uint32_t* __restrict__ yp,
+                        int* __restrict__ counts, uint32_t tail_mask) {
+    constexpr int H = 1 << (k - 1);
+    extern __shared__ uint4 ring_smem[];
+    __shared__ __align__(16) int2 sPQ[kHSWarps][H < 2 ? 2 : H];
+    const long long end = (long long)(blockIdx.y + 1) * kStageWords;
+    const bool full = end < W || (end == W && tail_mask == 0xffffffffu);
+    int2* mine = sPQ[threadIdx.x >> 5];
+    if (full)
+        head_staged_body<k, true>(xp4, w_in, W, N, conn, table, C, g, splits, per_split, yp, counts,
+                                  tail_mask, ring_smem, mine);
+    else
+        head_staged_body<k, false>(xp4, w_in, W, N, conn, table, C, g, splits, per_split, yp, counts,
+                                   tail_mask, ring_smem, mine);
+}
+
 __global__ void __launch_bounds__(256)
 argmax_kernel(const int* __restrict__ counts, long long N, int C, int* __restrict__ pred) {
     const long long s = (long long)blockIdx.x * 256 + threadIdx.x;
@@ -578,9 +731,11 @@ int sm_count() {
     return n;
 }
 
+// Opt in to more than the default 48 KB of shared memory per block when the
+// dynamic part plus the kernel's static part (a few KB) may exceed it.
 template <typename F>
 int set_dynamic_smem(F* kernel, int bytes) {
-    if (bytes <= 48 * 1024) return BITLOGIC_OK;
+    if (bytes <= 40 * 1024) return BITLOGIC_OK;
     return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) == cudaSuccess
                ? BITLOGIC_OK : BITLOGIC_ERR_CUDA;
 }
@@ -590,22 +745,27 @@ int launch_hard(const uint32_t* xp, int w_in, long long N, const int* conn, cons
                 int w, uint32_t* yp, int C, int* counts, int* pred, cudaStream_t st) {
     const long long W = (N + 31) / 32;
     const uint32_t tail_mask = (N % 32) ? ((1u << (N % 32)) - 1u) : 0xffffffffu;
-    const bool vec4 = (W % 4 == 0) && aligned16(xp) && (!yp || aligned16(yp));
+    // staged kernels: 16-byte rows and 32-bit row offsets in 16-byte units
+    const bool vec4 = (W % 4 == 0) && aligned16(xp) && (!yp || aligned16(yp)) &&
+                      (unsigned long long)w_in * (unsigned long long)(W / 4) < (1ull << 32);
     if (C == 0) {
-        const long long chunk = hard_word_chunk(w_in, W);
-        const long long ny = (W + chunk - 1) / chunk;
-        if (ny > 65535) return BITLOGIC_ERR_SHAPE;
         if (vec4) {
-            // nodes per warp: enough blocks for about four waves of two per SM
+            // chunks of kLayerNS stages; nodes per warp: enough blocks for
+            // about four waves of two per SM
+            const long long gy = (W + kLayerNS * kStageWords - 1) / (kLayerNS * kStageWords);
+            if (gy > 65535) return BITLOGIC_ERR_SHAPE;
             const long long groups = (w + kHardWarps - 1) / kHardWarps;
-            long long npw = groups * ny / (8ll * sm_count());
+            long long npw = groups * gy / (8ll * sm_count());
             npw = npw < 1 ? 1 : (npw > 8 ? 8 : npw);
             const long long gx = (w + kHardWarps * npw - 1) / (kHardWarps * npw);
-            const int smem = kHardWarps * ring_bytes_per_warp<k>(kRing);
+            const int smem = kHardWarps * ring_bytes_per_warp<k>(kLayerNS);
             if (set_dynamic_smem(hard_layer_staged_kernel<k>, smem)) return BITLOGIC_ERR_CUDA;
-            hard_layer_staged_kernel<k><<<dim3((unsigned)gx, (unsigned)ny), kHardWarps * 32, smem, st>>>(
-                xp, w_in, W, conn, table, w, yp, chunk, tail_mask);
+            hard_layer_staged_kernel<k><<<dim3((unsigned)gx, (unsigned)gy), kHardWarps * 32, smem, st>>>(
+                reinterpret_cast<const uint4*>(xp), w_in, W, conn, table, w, yp, tail_mask);
         } else {
+            const long long chunk = hard_word_chunk(w_in, W);
+            const long long ny = (W + chunk - 1) / chunk;
+            if (ny > 65535) return BITLOGIC_ERR_SHAPE;
             dim3 grid((unsigned)((w + kHardWarps - 1) / kHardWarps), (unsigned)ny);
             hard_layer_kernel<k, 1><<<grid, kHardWarps * 32, 0, st>>>(xp, w_in, W, conn, table, w, yp, chunk,
                                                                      tail_mask);
@@ -631,7 +791,8 @@ int launch_hard(const uint32_t* xp, int w_in, long long N, const int* conn, cons
         const int smem = head_smem_bytes<k>();
         if (set_dynamic_smem(hard_head_staged_kernel<k>, smem)) return BITLOGIC_ERR_CUDA;
         hard_head_staged_kernel<k><<<dim3((unsigned)(C * splits), (unsigned)wg), kHSWarps * 32, smem, st>>>(
-            xp, w_in, W, N, conn, table, C, g, splits, per_split, yp, counts, tail_mask);
+            reinterpret_cast<const uint4*>(xp), w_in, W, N, conn, table, C, g, splits, per_split, yp, counts,
+            tail_mask);
     } else {
         const long long wg = (W + 31) / 32;
         int splits = 1;
