@@ -536,11 +536,21 @@ constexpr int kSumPlanes = kHeadPlanes + 3;   // sum of kHSWarps <= 8 warps' cou
 constexpr int kMaxNodesPerWarp = 4 * ((1 << kHeadNB) - 1) + 3;
 static_assert(kHSWarps <= 8, "kSumPlanes assumes at most 8 warps");
 
+// The block's node slice (connectivity rows, checked once, and tables) is
+// staged in shared memory behind the ring: at most kHeadSliceNodes nodes.
+// Two blocks per SM of 8 warps: 2 x (113664 + 2048 static + 1024) <= 228 KB.
+constexpr int kHeadSliceNodes = 60 * kHSWarps;
+
 template <int k>
-__host__ __device__ constexpr int head_smem_bytes() {
+__host__ __device__ constexpr int head_ring_bytes() {
     const int ring = kHSWarps * ring_bytes_per_warp<k>(kHeadRing);
     const int flush = (kHSWarps * kHeadPlanes + kSumPlanes) * kStageWords * 4;
     return ring > flush ? ring : flush;
+}
+
+template <int k>
+__host__ __device__ constexpr int head_smem_bytes() {
+    return head_ring_bytes<k>() + kHeadSliceNodes * (k * 4 + 8);
 }
 
 template <int k, bool FULL>
@@ -549,8 +559,8 @@ __device__ __forceinline__ void head_staged_body(const uint4* __restrict__ xp4, 
                                                  const uint64_t* __restrict__ table, int C, int g,
                                                  int splits, int per_split, uint32_t* __restrict__ yp,
                                                  int* __restrict__ counts, uint32_t tail_mask,
-                                                 uint4* ring_smem, int2* sPQ) {
-    constexpr int H = 1 << (k - 1);
+                                                 uint4* ring_smem, int2* sPQ, const int* sConn,
+                                                 const uint64_t* sTab) {
     constexpr int kSlot = k * 32;   // uint4 per stage
     static_assert(kHeadRing == 4, "a loop iteration is kHeadRing node steps");
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -563,20 +573,19 @@ __device__ __forceinline__ void head_staged_body(const uint4* __restrict__ xp4, 
     uint4* ring = ring_smem + (size_t)warp * (kHeadRing * kSlot) + lane;
     const int jfirst = n0 + warp;
 
-    // issue stream: node ji, kHeadRing - 1 nodes ahead of the compute stream
+    // issue stream: node ji, kHeadRing - 1 nodes ahead of the compute stream;
+    // its rows come from the staged slice (broadcast loads)
     int ji = jfirst;
-    uint32_t oi[k], on[k];   // row offsets of node ji and of the warp's node after it
-#pragma unroll
-    for (int i = 0; i < k; ++i) oi[i] = on[i] = 0;
-    if (ji < n1) node_offsets<k>(conn, ji, w_in, lane, W4, wq4, oi);
-    if (ji + kHSWarps < n1) node_offsets<k>(conn, ji + kHSWarps, w_in, lane, W4, wq4, on);
     auto issue = [&](int slot) {
         if (ji < n1) {
-            if (active) issue_stage<k>(ring + slot * kSlot, xp4, oi, 0u);
-            ji += kHSWarps;
+            if (active) {
+                const int* rr = sConn + (ji - n0) * k;
+                uint32_t off[k];
 #pragma unroll
-            for (int i = 0; i < k; ++i) oi[i] = on[i];
-            if (ji + kHSWarps < n1) node_offsets<k>(conn, ji + kHSWarps, w_in, lane, W4, wq4, on);
+                for (int i = 0; i < k; ++i) off[i] = (uint32_t)rr[i] * W4 + wq4;
+                issue_stage<k>(ring + slot * kSlot, xp4, off, 0u);
+            }
+            ji += kHSWarps;
         }
         cp_async_commit();
     };
@@ -590,14 +599,12 @@ __device__ __forceinline__ void head_staged_body(const uint4* __restrict__ xp4, 
 #pragma unroll
         for (int b = 0; b < kHeadNB; ++b) big[b][r] = 0;
     }
-    uint64_t tab = jfirst < n1 ? __ldg(table + jfirst) : 0ull;
     // node step u of a loop iteration (node jj): the loop body has kHeadRing
     // steps, so step u reads slot u and refills slot u + 3 (mod kHeadRing).
     // Returns the node's four output words (0 past the slice or the words).
     auto node = [&](int jj, int u, uint32_t (&y)[4]) {
         __syncwarp();   // the previous node's pairs are read
-        node_pairs_smem<k>(tab, lane, sPQ);   // table 0 past the slice: harmless
-        tab = jj + kHSWarps < n1 ? __ldg(table + jj + kHSWarps) : 0ull;
+        node_pairs_smem<k>(jj < n1 ? sTab[jj - n0] : 0ull, lane, sPQ);   // 0 past the slice: harmless
         issue((u + kHeadRing - 1) % kHeadRing);
         cp_async_wait<kHeadRing - 1>();
 #pragma unroll
@@ -688,15 +695,34 @@ hard_head_staged_kernel(const uint4* __restrict__ xp4, int w_in, long long W, lo
     constexpr int H = 1 << (k - 1);
     extern __shared__ uint4 ring_smem[];
     __shared__ __align__(16) int2 sPQ[kHSWarps][H < 2 ? 2 : H];
+    int* sConn = reinterpret_cast<int*>(reinterpret_cast<unsigned char*>(ring_smem) + head_ring_bytes<k>());
+    uint64_t* sTab = reinterpret_cast<uint64_t*>(sConn + kHeadSliceNodes * k);
+    {   // stage the slice: out-of-range rows read row 0 and raise the flag
+        const int c = blockIdx.x / splits, sp = blockIdx.x - c * splits;
+        const int n0 = c * g + sp * per_split;
+        const int cnt = max(0, min(c * g + g, n0 + per_split) - n0);
+        bool bad = false;
+        for (int t = threadIdx.x; t < cnt * k; t += kHSWarps * 32) {
+            int v = __ldg(conn + (long long)n0 * k + t);
+            if ((unsigned)v >= (unsigned)w_in) {
+                bad = true;
+                v = 0;
+            }
+            sConn[t] = v;
+        }
+        for (int t = threadIdx.x; t < cnt; t += kHSWarps * 32) sTab[t] = __ldg(table + n0 + t);
+        if (bad) flag_index_error();
+        __syncthreads();
+    }
     const long long end = (long long)(blockIdx.y + 1) * kStageWords;
     const bool full = end < W || (end == W && tail_mask == 0xffffffffu);
     int2* mine = sPQ[threadIdx.x >> 5];
     if (full)
         head_staged_body<k, true>(xp4, w_in, W, N, conn, table, C, g, splits, per_split, yp, counts,
-                                  tail_mask, ring_smem, mine);
+                                  tail_mask, ring_smem, mine, sConn, sTab);
     else
         head_staged_body<k, false>(xp4, w_in, W, N, conn, table, C, g, splits, per_split, yp, counts,
-                                   tail_mask, ring_smem, mine);
+                                   tail_mask, ring_smem, mine, sConn, sTab);
 }
 
 __global__ void __launch_bounds__(256)
@@ -783,7 +809,8 @@ int launch_hard(const uint32_t* xp, int w_in, long long N, const int* conn, cons
         int splits = 1;
         while (C * splits < sm_count() && g / (splits * 2) >= 8 * kHSWarps) splits *= 2;
         int per_split = (g + splits - 1) / splits;
-        while ((per_split + kHSWarps - 1) / kHSWarps > kMaxNodesPerWarp) {   // counter capacity
+        // counter capacity and the staged slice
+        while ((per_split + kHSWarps - 1) / kHSWarps > kMaxNodesPerWarp || per_split > kHeadSliceNodes) {
             splits *= 2;
             per_split = (g + splits - 1) / splits;
         }
