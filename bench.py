@@ -144,7 +144,7 @@ def job_rate(world: int, samples_per_rank_step: int, steps: int, max_ms: float) 
 
 # ------------------------------------------------------ work per call --
 
-def call_work(wl, B):
+def call_work(wl, B, fuse_dy1=False):
     """Algorithmic work of each library call of one step on a batch of B:
     (bytes, fp32 or logic ops).  Ops follow the lerp-tree counts: forward
     2(2^k-1)+k per (node, sample); backward with input gradient
@@ -163,9 +163,13 @@ def call_work(wl, B):
         # layer 2: reads Y1 and the per-class gradient rows, writes dtheta and
         # the per-edge input-gradient terms
         "backward2": (f * (w1 * B + C * B + w2 * k * B + 2 * w2 * K + w2 * k), (4 * (K - 1) + K) * w2 * B),
-        # layer 1: reads the encoder bits and layer 2's per-edge terms (its
-        # output gradient, reduced through the CSR map in the kernel)
-        "backward1": (f * (win * B + w2 * k * B + 2 * w1 * K + w1 * k + w1 + w2 * k), (2 * (K - 1) + K) * w1 * B),
+        # layer 1 (fused form): reads the encoder bits and layer 2's per-edge
+        # terms (its output gradient, reduced through the CSR map in the
+        # kernel); unfused form: the CSR reduction of those terms into dY1
+        # ("csr2"), then the dtheta-only backward reading dY1
+        "backward1": (f * (win * B + w2 * k * B + 2 * w1 * K + w1 * k + w1 + w2 * k), (2 * (K - 1) + K) * w1 * B)
+        if fuse_dy1 else (f * (win * B + w1 * B + 2 * w1 * K + w1 * k), (2 * (K - 1) + K) * w1 * B),
+        "csr2": (f * (w2 * k * B + w1 * B + w1 + 1 + w2 * k), 0),
         "binarize": (f * (w1 * K + w2 * K) + 8 * (w1 + w2), 0),
         "pack": (B * d + f * win * W, 0),
         "hard1": (f * (win * W + w1 * W + w1 * k) + 8 * w1, (K - 1) * w1 * W),
@@ -177,9 +181,9 @@ KERNEL_OF_CALL = {
     "encode": "encode_soft_kernel", "forward1": "lut_forward_staged_kernel<k>",
     "forward2": "lut_forward_staged_kernel<k>", "head": "head_* (3 kernels)",
     "backward2": "lut_backward_node_kernel<k, dx, dY rows>",
-    "backward1": "lut_backward_node_kernel<k, no dx, CSR terms>",
-    "binarize": "binarize_kernel (x2)", "pack": "pack_bits_kernel", "hard1": "hard_layer_kernel",
-    "hard2": "hard_head_kernel + argmax_kernel",
+    "backward1": "lut_backward_theta_kernel<k>", "csr2": "csr_reduce_kernel",
+    "binarize": "binarize_kernel (x2)", "pack": "pack_bits_kernel", "hard1": "hard_layer_staged_kernel<k>",
+    "hard2": "hard_head_staged_kernel<k> + argmax_kernel",
 }
 
 
@@ -294,7 +298,7 @@ def run_ours(args):
     result = None
     if rank == 0:
         hbm, sm_max, peak_kind = peaks()
-        work = call_work(wl, B)
+        work = call_work(wl, B, fuse_dy1=st.fuse_dy1 if st is not None else False)
         per_call_ms = {n: float(np.mean(v)) for n, v in calls.items()}
         ms_step_train = train_sum / K
         ms_step_hard = hard_sum / K

@@ -109,8 +109,11 @@ int bitlogic_lut_backward(const float* X, int32_t w_in, int64_t B,
  * bitlogic_lut_backward_edges: dtheta as above and, when edge_terms is not
  *   NULL, edge_terms[(j*k + i)*B + s] = dY[j][s] * dy_j/dx_i(s)
  *   (device fp32 [w*k][B], 16-byte aligned for the vector path).
- * bitlogic_csr_reduce: dX[i][s] = sum of edge_terms[e][s] over the CSR edges e
- *   of input i, in increasing e (n_edges = w*k). */
+ * bitlogic_csr_reduce: dX[i][s] = sum of edge_terms[csr_edge[p]][s] over the
+ *   CSR positions p of input i, in increasing p (n_edges = w*k).  csr_edge
+ *   may be NULL when the term rows are already stored in CSR order (row p,
+ *   see edge_pos of bitlogic_lut_backward_ex): the sum then reads each
+ *   input's rows as one contiguous block. */
 int bitlogic_lut_backward_edges(const float* X, int32_t w_in, int64_t B,
                                 const int32_t* conn, const float* theta,
                                 int32_t w, int32_t k, const float* dY,
@@ -125,21 +128,27 @@ int bitlogic_csr_reduce(const float* edge_terms, int64_t B, const int32_t* csr_o
  *             dy_group = 1 is an ordinary dY [w][B]; dy_group = w / C takes
  *             the per-class gradient of bitlogic_head_loss_ex (the nodes of
  *             a class share one gradient row), so the full dY is never stored.
- *   up terms: dY[j][s] = sum over e in [up_off[j], up_off[j+1]) of
- *             up_terms[up_edge[e]][s], in increasing e -- the input gradient
+ *   up terms: dY[j][s] = sum over p in [up_off[j], up_off[j+1]) of
+ *             up_terms[up_edge[p]][s], in increasing p -- the input gradient
  *             of the next layer (its per-edge terms and the CSR map of its
  *             connectivity, up_edges = w_next * k_next), reduced on the fly;
  *             the result equals bitlogic_csr_reduce of those terms bit for bit.
+ *             up_edge may be NULL when the terms are stored in CSR order.
  * dtheta, edge_terms as in bitlogic_lut_backward_edges (edge_terms may be
- * NULL); dY_out (device fp32 [w][B] or NULL) receives the gradient used. */
+ * NULL).  edge_pos (device int32 [w*k] or NULL): when given, the term of
+ * edge e = j*k + i is stored at row edge_pos[e] instead of row e; with the
+ * positions of bitlogic_csr_positions the rows come out in CSR order, so
+ * their consumer reads each input's rows contiguously (a position outside
+ * [0, w*k) raises the device flag and stores at row e).  dY_out (device fp32
+ * [w][B] or NULL) receives the gradient used. */
 int bitlogic_lut_backward_ex(const float* X, int32_t w_in, int64_t B,
                              const int32_t* conn, const float* theta,
                              int32_t w, int32_t k,
                              const float* dY, int32_t dy_group,
                              const float* up_terms, const int32_t* up_off,
                              const int32_t* up_edge, int32_t up_edges,
-                             float* dtheta, float* edge_terms, float* dY_out,
-                             cudaStream_t stream);
+                             float* dtheta, float* edge_terms, const int32_t* edge_pos,
+                             float* dY_out, cudaStream_t stream);
 
 /* Bytes of workspace bitlogic_head_loss needs. */
 size_t bitlogic_head_loss_workspace(int64_t B, int32_t C);
@@ -232,6 +241,11 @@ int bitlogic_hard_forward(const uint32_t* xp, int32_t w_in, int64_t N,
  * [0, w_in).  Not part of the per-step path: built once per connectivity. */
 int bitlogic_build_csr(const int32_t* conn_host, int32_t w, int32_t k, int32_t w_in,
                        int32_t* off_host, int32_t* edge_host);
+
+/* Host: the CSR position of every edge, the inverse permutation of
+ * edge_host: pos_host[edge_host[p]] = p for p < n_edges.  Returns
+ * BITLOGIC_ERR_INDEX unless edge_host is a permutation of [0, n_edges). */
+int bitlogic_csr_positions(const int32_t* edge_host, int32_t n_edges, int32_t* pos_host);
 
 /* Synchronizes `stream`, then reports (and clears) the device-side index
  * flag: BITLOGIC_OK, or BITLOGIC_ERR_DEVICE when a kernel met an index out of

@@ -29,7 +29,7 @@ __all__ = [
     "bitlogic_csr_reduce", "bitlogic_lut_backward_ex", "bitlogic_head_loss_ex",
     "bitlogic_head_loss_workspace", "bitlogic_head_loss_noalloc",
     "bitlogic_head_loss", "bitlogic_binarize_tables", "bitlogic_pack_bits",
-    "bitlogic_hard_forward", "bitlogic_build_csr", "bitlogic_device_error",
+    "bitlogic_hard_forward", "bitlogic_build_csr", "bitlogic_csr_positions", "bitlogic_device_error",
     "bitlogic_status_string", "bitlogic_version", "LIB_PATH",
 ]
 
@@ -55,7 +55,7 @@ _SIGS = {
                                     ctypes.c_int),
     "bitlogic_csr_reduce": ([_P, _I64, _P, _P, _I32, _I32, _P, _P], ctypes.c_int),
     "bitlogic_lut_backward_ex": ([_P, _I32, _I64, _P, _P, _I32, _I32, _P, _I32, _P, _P, _P, _I32,
-                                  _P, _P, _P, _P], ctypes.c_int),
+                                  _P, _P, _P, _P, _P], ctypes.c_int),
     "bitlogic_head_loss_ex": ([_P, _I32, _I64, _I32, _F32, _P, _P, _P, _P, _P, _P, _SZ, _P],
                               ctypes.c_int),
     "bitlogic_head_loss_workspace": ([_I64, _I32], _SZ),
@@ -67,6 +67,7 @@ _SIGS = {
     "bitlogic_hard_forward": ([_P, _I32, _I64, _P, _P, _I32, _I32, _P, _I32, _P, _P, _P],
                               ctypes.c_int),
     "bitlogic_build_csr": ([_P, _I32, _I32, _I32, _P, _P], ctypes.c_int),
+    "bitlogic_csr_positions": ([_P, _I32, _P], ctypes.c_int),
     "bitlogic_device_error": ([_P], ctypes.c_int),
     "bitlogic_status_string": ([ctypes.c_int], ctypes.c_char_p),
     "bitlogic_version": ([], ctypes.c_int),
@@ -201,13 +202,15 @@ def bitlogic_lut_backward_edges(X: torch.Tensor, conn: torch.Tensor, theta: torc
         _ptr(edge_terms), _stream(stream)))
 
 
-def bitlogic_csr_reduce(edge_terms: torch.Tensor, csr_off: torch.Tensor, csr_edge: torch.Tensor,
-                        dX: torch.Tensor, stream=None):
+def bitlogic_csr_reduce(edge_terms: torch.Tensor, csr_off: torch.Tensor,
+                        csr_edge: Optional[torch.Tensor], dX: torch.Tensor, stream=None):
+    """csr_edge None: the term rows are stored in CSR order."""
     nE, B = edge_terms.shape
     w_in = dX.shape[0]
     _need(edge_terms, "edge_terms", torch.float32, (nE, B))
     _need(csr_off, "csr_off", torch.int32, (w_in + 1,))
-    _need(csr_edge, "csr_edge", torch.int32, (nE,))
+    if csr_edge is not None:
+        _need(csr_edge, "csr_edge", torch.int32, (nE,))
     _need(dX, "dX", torch.float32, (w_in, B))
     _check("bitlogic_csr_reduce", load().bitlogic_csr_reduce(
         _ptr(edge_terms), B, _ptr(csr_off), _ptr(csr_edge), w_in, nE, _ptr(dX), _stream(stream)))
@@ -219,7 +222,10 @@ def bitlogic_lut_backward_ex(X: torch.Tensor, conn: torch.Tensor, theta: torch.T
                              up_off: Optional[torch.Tensor] = None,
                              up_edge: Optional[torch.Tensor] = None,
                              edge_terms: Optional[torch.Tensor] = None,
+                             edge_pos: Optional[torch.Tensor] = None,
                              dY_out: Optional[torch.Tensor] = None, stream=None):
+    """up_edge None with up_terms: the upstream term rows are in CSR order.
+    edge_pos: store the term of edge e at row edge_pos[e] of edge_terms."""
     w_in, B = X.shape
     w, k = conn.shape
     _need(X, "X", torch.float32, (w_in, B))
@@ -235,15 +241,18 @@ def bitlogic_lut_backward_ex(X: torch.Tensor, conn: torch.Tensor, theta: torch.T
         n_up = up_terms.shape[0]
         _need(up_terms, "up_terms", torch.float32, (n_up, B))
         _need(up_off, "up_off", torch.int32, (w + 1,))
-        _need(up_edge, "up_edge", torch.int32, (n_up,))
+        if up_edge is not None:
+            _need(up_edge, "up_edge", torch.int32, (n_up,))
     if edge_terms is not None:
         _need(edge_terms, "edge_terms", torch.float32, (w * k, B))
+    if edge_pos is not None:
+        _need(edge_pos, "edge_pos", torch.int32, (w * k,))
     if dY_out is not None:
         _need(dY_out, "dY_out", torch.float32, (w, B))
     _check("bitlogic_lut_backward_ex", load().bitlogic_lut_backward_ex(
         _ptr(X), w_in, B, _ptr(conn), _ptr(theta), w, k, _ptr(dY), int(dy_group),
         _ptr(up_terms), _ptr(up_off), _ptr(up_edge), n_up, _ptr(dtheta), _ptr(edge_terms),
-        _ptr(dY_out), _stream(stream)))
+        _ptr(edge_pos), _ptr(dY_out), _stream(stream)))
 
 
 def bitlogic_head_loss_ex(Y: torch.Tensor, labels: torch.Tensor, C: int, tau: float,
@@ -358,6 +367,15 @@ def bitlogic_build_csr(conn: np.ndarray, w_in: int) -> Tuple[np.ndarray, np.ndar
     _check("bitlogic_build_csr", load().bitlogic_build_csr(
         conn.ctypes.data_as(_P), w, k, w_in, off.ctypes.data_as(_P), edge.ctypes.data_as(_P)))
     return off, edge
+
+
+def bitlogic_csr_positions(csr_edge: np.ndarray) -> np.ndarray:
+    """Host call: pos[csr_edge[p]] = p (the CSR position of every edge)."""
+    edge = np.ascontiguousarray(csr_edge, dtype=np.int32)
+    pos = np.zeros(edge.shape[0], np.int32)
+    _check("bitlogic_csr_positions", load().bitlogic_csr_positions(
+        edge.ctypes.data_as(_P), edge.shape[0], pos.ctypes.data_as(_P)))
+    return pos
 
 
 def bitlogic_device_error(stream=None) -> int:

@@ -47,6 +47,18 @@ extern "C" int bitlogic_build_csr(const int32_t* conn_host, int32_t w, int32_t k
     return BITLOGIC_OK;
 }
 
+extern "C" int bitlogic_csr_positions(const int32_t* edge_host, int32_t n_edges, int32_t* pos_host) {
+    if (!edge_host || !pos_host) return BITLOGIC_ERR_NULL;
+    if (n_edges < 0) return BITLOGIC_ERR_SHAPE;
+    for (int32_t e = 0; e < n_edges; ++e) pos_host[e] = -1;
+    for (int32_t p = 0; p < n_edges; ++p) {
+        const int32_t e = edge_host[p];
+        if (e < 0 || e >= n_edges || pos_host[e] != -1) return BITLOGIC_ERR_INDEX;
+        pos_host[e] = p;
+    }
+    return BITLOGIC_OK;
+}
+
 extern "C" int bitlogic_device_error(cudaStream_t stream) {
     int worst = BITLOGIC_OK;
     const int r[4] = {bitlogic_internal_index_error_lut_soft(stream),

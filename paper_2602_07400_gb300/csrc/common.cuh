@@ -62,15 +62,11 @@ inline int make_thresholds(const uint8_t* thr_host, int32_t b, Thresholds* out) 
 // IEEE-rounded division (no fast-math).
 __device__ __forceinline__ float sigmoidf(float z) { return 1.0f / (1.0f + expf(-z)); }
 
-// Asynchronous global -> shared copies (cp.async; the 16-byte form bypasses
-// L1), grouped per pipeline stage.
+// Asynchronous 16-byte global -> shared copies (cp.async, bypassing L1),
+// grouped per pipeline stage.
 __device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
     const unsigned s = (unsigned)__cvta_generic_to_shared(smem);
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(s), "l"(gmem) : "memory");
-}
-__device__ __forceinline__ void cp_async8(void* smem, const void* gmem) {
-    const unsigned s = (unsigned)__cvta_generic_to_shared(smem);
-    asm volatile("cp.async.ca.shared.global [%0], [%1], 8;\n" ::"r"(s), "l"(gmem) : "memory");
 }
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
 template <int N>

@@ -44,6 +44,42 @@ head_group_sum_kernel(const float* __restrict__ Y, long long B, int C, int g, fl
     }
 }
 
+// Vector form (B % 4 == 0, 16-byte aligned Y): one block of 32 warps per
+// (class, 128 samples), lane = 4 consecutive samples, warp r sums rows r,
+// r + 32, ... of the group with 16-byte loads (enough loads in flight for
+// HBM), then thread t adds the 32 warps' partial sums of sample t in order.
+constexpr int kSumVecWarps = 32;
+
+__global__ void __launch_bounds__(kSumVecWarps * 32)
+head_group_sum_vec_kernel(const float* __restrict__ Y, long long B, int C, int g, float tau,
+                          float* __restrict__ logits) {
+    __shared__ __align__(16) float part[kSumVecWarps][128];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int c = blockIdx.x;
+    const long long s4 = (long long)blockIdx.y * 128 + 4 * lane;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (s4 < B) {   // B % 4 == 0: all four samples are in range
+        const float* base = Y + (long long)c * g * B + s4;
+#pragma unroll 4
+        for (int r = warp; r < g; r += kSumVecWarps) {
+            const float4 v = __ldg(reinterpret_cast<const float4*>(base + (long long)r * B));
+            acc.x += v.x;
+            acc.y += v.y;
+            acc.z += v.z;
+            acc.w += v.w;
+        }
+    }
+    *reinterpret_cast<float4*>(&part[warp][4 * lane]) = acc;
+    __syncthreads();
+    if (threadIdx.x < 128) {
+        const long long s = (long long)blockIdx.y * 128 + threadIdx.x;
+        float t = 0.f;
+#pragma unroll 8
+        for (int q = 0; q < kSumVecWarps; ++q) t += part[q][threadIdx.x];
+        if (s < B) logits[s * C + c] = t / tau;
+    }
+}
+
 __device__ __forceinline__ float warp_max(float v) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
@@ -165,7 +201,11 @@ extern "C" int bitlogic_head_loss_ex(const float* Y, int32_t w, int64_t B, int32
     float* per = reinterpret_cast<float*>(ws + align_up(bc));
     float* lg = logits ? logits : reinterpret_cast<float*>(ws + align_up(bc) + align_up((size_t)B * 4));
 
-    head_group_sum_kernel<<<dim3((unsigned)C, (unsigned)sb), kSumWarps * 32, 0, stream>>>(Y, B, C, g, tau, lg);
+    if (B % 4 == 0 && aligned16(Y))
+        head_group_sum_vec_kernel<<<dim3((unsigned)C, (unsigned)((B + 127) / 128)), kSumVecWarps * 32, 0, stream>>>(
+            Y, B, C, g, tau, lg);
+    else
+        head_group_sum_kernel<<<dim3((unsigned)C, (unsigned)sb), kSumWarps * 32, 0, stream>>>(Y, B, C, g, tau, lg);
     head_softmax_kernel<<<(unsigned)((B + kSoftWarps - 1) / kSoftWarps), kSoftWarps * 32, 0, stream>>>(
         lg, B, C, labels, dlogit, per, tau, dY_grouped);
     if (dY)

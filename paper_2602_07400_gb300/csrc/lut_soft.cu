@@ -32,8 +32,6 @@ constexpr int kBwdWarps = 4;   // warps per block in the staged backward
 #endif
 constexpr int kWarpsPerNode = BITLOGIC_BWD_WARPS_PER_NODE;   // 1, 2 or 4
 constexpr int kNodesPerBlock = kBwdWarps / kWarpsPerNode;
-constexpr int kCsrWarps = 8;
-
 // ---------------------------------------------------------------- trees --
 
 template <int L, int M, int H, int k>
@@ -333,7 +331,8 @@ lut_forward_staged_kernel(const float* __restrict__ X, int w_in, long long B,
 //          the head's per-class gradient, shared by the g nodes of a class)
 //   terms: sum over e in [off[j], off[j+1]) of terms[edge[e]][.] in
 //          increasing e -- the next layer's input gradient, reduced on the
-//          fly from its per-edge terms instead of being materialised
+//          fly from its per-edge terms instead of being materialised.  With
+//          edge == nullptr the term rows are stored in CSR order (row e).
 struct GradSource {
     const float* dY;
     int group;
@@ -342,6 +341,22 @@ struct GradSource {
     const int* edge;
     int n_edges;
 };
+
+// Term row of CSR position e (edge == nullptr: rows in CSR order).
+__device__ __forceinline__ int term_row(const GradSource& gs, int e) {
+    return gs.edge ? __ldg(gs.edge + e) : e;
+}
+
+// Row of edge e's term in the per-edge buffer: e itself, or pos[e] when the
+// caller asks for CSR order (an out-of-range position raises the flag and
+// falls back to row e, so every store stays inside the buffer).
+__device__ __forceinline__ long long edge_row(const int* __restrict__ pos, long long e, long long n) {
+    if (!pos) return e;
+    const int r = __ldg(pos + e);
+    if (r >= 0 && (long long)r < n) return r;
+    flag_index_error();
+    return e;
+}
 
 // CSR range of node j in the upstream terms (range-checked).
 __device__ __forceinline__ void term_range(const GradSource& gs, int j, int lane, int& e0, int& e1) {
@@ -360,7 +375,7 @@ __global__ void __launch_bounds__(kFwdWarps * 32)
 lut_backward_kernel(const float* __restrict__ X, int w_in, long long B,
                     const int* __restrict__ conn, const float* __restrict__ theta, int w,
                     GradSource gs, float* __restrict__ dtheta, float* __restrict__ P,
-                    float* __restrict__ dY_out) {
+                    const int* __restrict__ epos, float* __restrict__ dY_out) {
     constexpr int K = 1 << k, H = K / 2;
     __shared__ float2 sPair[kFwdWarps][H];
     __shared__ float sRed[kFwdWarps][32][K + 1];
@@ -373,13 +388,17 @@ lut_backward_kernel(const float* __restrict__ X, int w_in, long long B,
     int e0 = 0, e1 = 0;
     if constexpr (TERMS) term_range(gs, j, lane, e0, e1);
     const float* gr = TERMS ? nullptr : gs.dY + (long long)(j / gs.group) * B;
-    float* pr = P + (long long)j * k * B;
+    float* pr[WANT_DX ? k : 1];
+    if constexpr (WANT_DX) {
+#pragma unroll
+        for (int i = 0; i < k; ++i) pr[i] = P + edge_row(epos, (long long)j * k + i, (long long)w * k) * B;
+    }
 
     auto grad = [&](long long s) {
         if constexpr (TERMS) {
             float g = 0.f;
             for (int e = e0; e < e1; ++e) {
-                const int id = __ldg(gs.edge + e);
+                const int id = term_row(gs, e);
                 if ((unsigned)id < (unsigned)gs.n_edges) g += __ldg(gs.terms + (long long)id * B + s);
                 else if (lane == 0) flag_index_error();
             }
@@ -417,7 +436,7 @@ lut_backward_kernel(const float* __restrict__ X, int w_in, long long B,
         bwd_tree<k - 1, 0>(te, d, x, omx, g, dx, acc);
         if constexpr (WANT_DX) {
 #pragma unroll
-            for (int i = 0; i < k; ++i) pr[(long long)i * B + s] = dx[i];
+            for (int i = 0; i < k; ++i) pr[i][s] = dx[i];
         }
     }
 #pragma unroll
@@ -488,7 +507,7 @@ __global__ void __launch_bounds__(kBwdWarps * 32, BITLOGIC_BWD_MIN_BLOCKS)
 lut_backward_node_kernel(const float* __restrict__ X, int w_in, long long B,
                          const int* __restrict__ conn, const float* __restrict__ theta, int w,
                          GradSource gs, float* __restrict__ dtheta, float* __restrict__ P,
-                         float* __restrict__ dY_out) {
+                         const int* __restrict__ epos, float* __restrict__ dY_out) {
     constexpr int K = 1 << k, H = K / 2, H2 = K / 4, R = k + 1, CH = kStageSamples;
     constexpr int NQ = (k + 1) / 2;   // slots stored per lane (rounded up)
     extern __shared__ __align__(16) float smem[];
@@ -547,7 +566,7 @@ lut_backward_node_kernel(const float* __restrict__ X, int w_in, long long B,
             term_range(gs, j, lane, e0, e1);
             deg = e1 - e0;
             if (lane < deg) {
-                my_id = __ldg(gs.edge + e0 + lane);
+                my_id = term_row(gs, e0 + lane);
                 if ((unsigned)my_id >= (unsigned)gs.n_edges) {
                     flag_index_error();
                     my_id = -1;   // read as a zero row
@@ -563,7 +582,13 @@ lut_backward_node_kernel(const float* __restrict__ X, int w_in, long long B,
     src[k] = TERMS ? nullptr : gs.dY + (long long)(jj / gs.group) * B + 4 * lane;
     float* pst[NQ];   // this lane's stored slots 2q + h, at its first sample
 #pragma unroll
-    for (int q = 0; q < NQ; ++q) pst[q] = P + ((long long)jj * k + (2 * q + h < k ? 2 * q + h : 0)) * B + pair;
+    for (int q = 0; q < NQ; ++q) {
+        pst[q] = nullptr;
+        if constexpr (WANT_DX) {
+            const long long e = (long long)jj * k + (2 * q + h < k ? 2 * q + h : 0);
+            pst[q] = P + (live ? edge_row(epos, e, (long long)w * k) : e) * B + pair;
+        }
+    }
     const int nst = (int)((B + CH - 1) / CH);
     const int per = (nst + kWarpsPerNode - 1) / kWarpsPerNode;
     const int first = sub * per;
@@ -597,7 +622,7 @@ lut_backward_node_kernel(const float* __restrict__ X, int w_in, long long B,
             const int nu = min(kGatherStages, mine - i);
 #pragma unroll 2
             for (int q = 0; q < deg; ++q) {
-                const int id = q < 32 ? __shfl_sync(0xffffffffu, my_id, q) : __ldg(gs.edge + e0 + q);
+                const int id = q < 32 ? __shfl_sync(0xffffffffu, my_id, q) : term_row(gs, e0 + q);
                 if (id >= 0 && (unsigned)id < (unsigned)gs.n_edges) {
                     const float* row = gs.terms + (long long)id * B + s0;
 #pragma unroll
@@ -709,80 +734,231 @@ lut_backward_node_kernel(const float* __restrict__ X, int w_in, long long B,
     }
 }
 
-// dX[i][s] = sum over the CSR edges of input i (increasing edge id) of
-// P[edge][s].  One warp per input row, lanes over samples.  The row's edge
-// ids are read once (one per lane) so the loads issue back to back, and each
-// pass reads 2 KB contiguous from every edge row (4 x 16 bytes per lane):
-// the rows are random in DRAM and short reads waste its bandwidth.
+// ------------------------------------- dtheta only, one lane per sample --
+//
+// Without an input gradient the backward needs no table values:
+// dtheta_a = t_a (1 - t_a) sum_s g_s w_a(x_s), w_a the corner weight of
+// entry a.  With the slots split into a low half (0 .. kl-1, kl = k/2) and a
+// high half, w_a = u(a_lo) v(a_hi): per sample the lane builds U = g times
+// the corner weights of the low half and V = the corner weights of the high
+// half by doubling products, then adds the outer product U V^T into its 2^k
+// accumulators (k = 6: 6 FADD + 14 + 12 FMUL + 64 FFMA = 96 FP32 operations
+// per sample, against 190 for the separate corner-weight tree).
+//
+// Persistent warps: warp g of the grid takes nodes g, g + G, ... (G warps in
+// the grid, sized to one wave) over the whole batch, 4 consecutive samples
+// per lane in each 128-sample stage.  Its k input rows and gradient row
+// stream through a lane-private cp.async ring (a lane reads only the 16
+// bytes per row it copied) that runs across node boundaries, so the next
+// node's first stages load while the current node finishes.  A node's
+// dtheta is reduced inside the warp by a fixed butterfly of shuffles, with
+// no block barrier.  Needs B % 4 == 0 and 16-byte aligned X, dY and dY_out.
+
+constexpr int kThetaWarps = 4;
+
+template <int k>
+__host__ __device__ constexpr int theta_floats_per_warp() {
+    return kStages * (k + 1) * kStageSamples;
+}
+
+// Reduce-scatter of N values per lane over the lane offsets O, O/2, ..., 1:
+// at each step a lane keeps half of its values (the upper half when lane bit
+// O is set), adds its partner's copy of that half and hands over the other
+// half; once one value is left the remaining steps add it across lanes.
+// Afterwards, for N0 = 2^k >= 32 values, lane l holds the sums of entries
+// l N0/32 .. l N0/32 + N0/32 - 1; for N0 < 32, of entry l >> (5 - k).  The
+// order of every addition is fixed.
+template <int N, int O, int M>
+__device__ __forceinline__ void warp_reduce_scatter(float (&v)[M], int lane) {
+    if constexpr (O > 0) {
+        if constexpr (N > 1) {
+            const bool up = (lane & O) != 0;
+#pragma unroll
+            for (int i = 0; i < N / 2; ++i) {
+                const float send = up ? v[i] : v[i + N / 2];
+                const float keep = up ? v[i + N / 2] : v[i];
+                v[i] = keep + __shfl_xor_sync(0xffffffffu, send, O);
+            }
+            warp_reduce_scatter<N / 2, O / 2>(v, lane);
+        } else {
+            v[0] += __shfl_xor_sync(0xffffffffu, v[0], O);
+            warp_reduce_scatter<1, O / 2>(v, lane);
+        }
+    }
+}
+
+template <int k>
+__global__ void __launch_bounds__(kThetaWarps * 32, BITLOGIC_BWD_MIN_BLOCKS)
+lut_backward_theta_kernel(const float* __restrict__ X, int w_in, long long B,
+                          const int* __restrict__ conn, const float* __restrict__ theta, int w,
+                          const float* __restrict__ dY, int group, float* __restrict__ dtheta,
+                          float* __restrict__ dY_out) {
+    constexpr int K = 1 << k, KL = k / 2, NU = 1 << KL, NV = 1 << (k - KL), R = k + 1;
+    constexpr int CH = kStageSamples;
+    extern __shared__ __align__(16) float smem[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    float* ring = smem + warp * theta_floats_per_warp<k>();
+    const int G = gridDim.x * kThetaWarps;
+    const int jfirst = blockIdx.x * kThetaWarps + warp;
+    const int nst = (int)((B + CH - 1) / CH);
+
+    // issue stream: stage si of node ji, kStages - 1 stages ahead of the
+    // compute stream; rows of the warp's node after ji are loaded ahead
+    int ji = jfirst, si = 0, ib = 0;
+    int ri[k], rn[k];
+#pragma unroll
+    for (int i = 0; i < k; ++i) ri[i] = rn[i] = 0;
+    if (ji < w) load_rows<k>(conn, ji, w_in, lane, ri);
+    if (ji + G < w) load_rows<k>(conn, ji + G, w_in, lane, rn);
+    auto issue = [&]() {
+        if (ji < w) {
+            const long long s4 = (long long)si * CH + 4 * lane;
+            if (s4 < B) {
+                float* buf = ring + ib * (R * CH) + 4 * lane;
+#pragma unroll
+                for (int r = 0; r < k; ++r) cp_async16(buf + r * CH, X + (long long)ri[r] * B + s4);
+                cp_async16(buf + k * CH, dY + (long long)(ji / group) * B + s4);
+            }
+            if (++si == nst) {
+                si = 0;
+                ji += G;
+#pragma unroll
+                for (int i = 0; i < k; ++i) ri[i] = rn[i];
+                if (ji + G < w) load_rows<k>(conn, ji + G, w_in, lane, rn);
+            }
+        }
+        cp_async_commit();
+        ib = (ib + 1 == kStages) ? 0 : ib + 1;
+    };
+#pragma unroll 1
+    for (int i = 0; i < kStages - 1; ++i) issue();
+
+    int rb = 0;
+#pragma unroll 1
+    for (int j = jfirst; j < w; j += G) {
+        float acc[K];
+#pragma unroll
+        for (int a = 0; a < K; ++a) acc[a] = 0.f;
+#pragma unroll 1
+        for (int sc = 0; sc < nst; ++sc) {
+            issue();
+            cp_async_wait<kStages - 1>();
+            const long long s4 = (long long)sc * CH + 4 * lane;   // this lane's 4 samples
+            if (s4 < B) {   // B % 4 == 0: all four samples are in range
+                const float* buf = ring + rb * (R * CH) + 4 * lane;
+                float4 xv[k];
+#pragma unroll
+                for (int q = 0; q < k; ++q) xv[q] = *reinterpret_cast<const float4*>(buf + q * CH);
+                const float4 gv = *reinterpret_cast<const float4*>(buf + k * CH);
+                if (dY_out) *reinterpret_cast<float4*>(dY_out + (long long)j * B + s4) = gv;
+#pragma unroll
+                for (int r = 0; r < 4; ++r) {
+                    float x[k], omx[k];
+#pragma unroll
+                    for (int q = 0; q < k; ++q) {
+                        x[q] = comp(xv[q], r);
+                        omx[q] = 1.0f - x[q];
+                    }
+                    float U[NU], V[NV];
+                    U[0] = comp(gv, r);
+#pragma unroll
+                    for (int q = 0; q < KL; ++q) {   // slot q doubles U: index bit q
+#pragma unroll
+                        for (int m = 0; m < (1 << q); ++m) {
+                            U[m + (1 << q)] = U[m] * x[q];
+                            U[m] = U[m] * omx[q];
+                        }
+                    }
+                    V[0] = omx[KL];
+                    V[1] = x[KL];
+#pragma unroll
+                    for (int q = KL + 1; q < k; ++q) {   // slot q doubles V: index bit q - KL
+#pragma unroll
+                        for (int m = 0; m < (1 << (q - KL)); ++m) {
+                            V[m + (1 << (q - KL))] = V[m] * x[q];
+                            V[m] = V[m] * omx[q];
+                        }
+                    }
+#pragma unroll
+                    for (int b = 0; b < NV; ++b)
+#pragma unroll
+                        for (int a = 0; a < NU; ++a) acc[a + b * NU] = fmaf(U[a], V[b], acc[a + b * NU]);
+                }
+            }
+            rb = (rb + 1 == kStages) ? 0 : rb + 1;
+        }
+        // the node's dtheta: butterfly over the lanes, then t (1 - t)
+        warp_reduce_scatter<K, 16>(acc, lane);
+        constexpr int NF = K >= 32 ? K / 32 : 1;   // entries per lane
+        constexpr int SH = K >= 32 ? 0 : 5 - k;    // lanes sharing an entry (K < 32)
+        if ((lane & ((1 << SH) - 1)) == 0) {
+#pragma unroll
+            for (int i = 0; i < NF; ++i) {
+                const int a = K >= 32 ? lane * NF + i : lane >> SH;
+                const float t = sigmoidf(__ldg(theta + (long long)j * K + a));
+                dtheta[(long long)j * K + a] = t * (1.0f - t) * acc[i];
+            }
+        }
+    }
+    cp_async_wait<0>();
+}
+
+// dX[i][s] = sum over the CSR positions p of input i (increasing p) of
+// P[edge[p]][s].  One block per input row i (and batch slice); warp r of the
+// block owns 128 samples (vector path: 4 per lane) or 32 (scalar path) and
+// issues the loads of all of the row's terms back to back, so each warp has
+// deg x 512 bytes in flight.  The row's ids are read once, one per lane.
+constexpr int kCsrWarps = 8;
+
 template <bool VEC>
 __global__ void __launch_bounds__(kCsrWarps * 32)
 csr_reduce_kernel(const float* __restrict__ P, long long B, const int* __restrict__ off,
                   const int* __restrict__ edge, int w_in, int nE, float* __restrict__ dX) {
+    constexpr int SPW = VEC ? 128 : 32;   // samples per warp
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int i = blockIdx.x * kCsrWarps + warp;
-    if (i >= w_in) return;
+    const int i = blockIdx.x;
     int e0 = __ldg(off + i), e1 = __ldg(off + i + 1);
     if (e0 < 0 || e1 < e0 || e1 > nE) {
-        if (lane == 0) flag_index_error();
+        if (threadIdx.x == 0) flag_index_error();
         e0 = e1 = 0;
     }
     const int deg = e1 - e0;
-    int my_id = -1;   // ids of the first 32 edges, -1 when out of range
+    int my_id = -1;   // ids of the first 32 positions, -1 when out of range
     if (lane < deg) {
-        my_id = __ldg(edge + e0 + lane);
+        my_id = edge ? __ldg(edge + e0 + lane) : e0 + lane;
         if ((unsigned)my_id >= (unsigned)nE) {
-            flag_index_error();
+            if (warp == 0) flag_index_error();
             my_id = -1;
         }
     }
-    auto edge_id = [&](int q) {
+    auto edge_id = [&](int q) {   // warp-uniform call
         if (q < 32) return __shfl_sync(0xffffffffu, my_id, q);
-        const int id = __ldg(edge + e0 + q);
+        const int id = edge ? __ldg(edge + e0 + q) : e0 + q;
         if ((unsigned)id >= (unsigned)nE) {
-            if (lane == 0) flag_index_error();
+            if (lane == 0 && warp == 0) flag_index_error();
             return -1;
         }
         return id;
     };
-    float* out = dX + (long long)i * B;
+    const long long s = ((long long)blockIdx.y * kCsrWarps + warp) * SPW + (VEC ? 4 : 1) * lane;
+    const bool in = s < B;   // vector path: B % 4 == 0, all four samples in range
+    float* out = dX + (long long)i * B + s;
     if constexpr (VEC) {
-        for (long long base = 0; base < B; base += 512) {
-            float4 acc[4];
-#pragma unroll
-            for (int u = 0; u < 4; ++u) acc[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 2
-            for (int q = 0; q < deg; ++q) {
-                const int id = edge_id(q);
-                if (id < 0) continue;
-                const float* pr = P + (long long)id * B + base + 4 * lane;
-#pragma unroll
-                for (int u = 0; u < 4; ++u)
-                    if (base + 128 * u + 4 * lane < B) acc[u] = add4(acc[u], ldg4(pr + 128 * u));
-            }
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const long long s = base + 128 * u + 4 * lane;
-                if (s < B) *reinterpret_cast<float4*>(out + s) = acc[u];
-            }
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 8
+        for (int q = 0; q < deg; ++q) {
+            const int id = edge_id(q);
+            if (in && id >= 0) acc = add4(acc, ldg4(P + (long long)id * B + s));
         }
+        if (in) *reinterpret_cast<float4*>(out) = acc;
     } else {
-        for (long long base = 0; base < B; base += 128) {
-            float acc[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll 2
-            for (int q = 0; q < deg; ++q) {
-                const int id = edge_id(q);
-                if (id < 0) continue;
-                const float* pr = P + (long long)id * B + base + lane;
-#pragma unroll
-                for (int u = 0; u < 4; ++u)
-                    if (base + 32 * u + lane < B) acc[u] += __ldg(pr + 32 * u);
-            }
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const long long s = base + 32 * u + lane;
-                if (s < B) out[s] = acc[u];
-            }
+        float acc = 0.f;
+#pragma unroll 8
+        for (int q = 0; q < deg; ++q) {
+            const int id = edge_id(q);
+            if (in && id >= 0) acc += __ldg(P + (long long)id * B + s);
         }
+        if (in) *out = acc;
     }
 }
 
@@ -804,6 +980,14 @@ long long forward_chunk(int w_in, int w, long long B) {
     return c < B ? c : B;
 }
 
+int sm_count() {
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+        return 152;
+    return n;
+}
+
 template <int k>
 int launch_forward(const float* X, int w_in, long long B, const int* conn, const float* theta,
                    int w, float* Y, bool vec, cudaStream_t st) {
@@ -821,8 +1005,8 @@ int launch_forward(const float* X, int w_in, long long B, const int* conn, const
 
 template <int k, bool WANT_DX, bool TERMS>
 int launch_backward_impl(const float* X, int w_in, long long B, const int* conn, const float* theta,
-                         int w, const GradSource& gs, float* dtheta, float* P, float* dY_out,
-                         bool staged, cudaStream_t st) {
+                         int w, const GradSource& gs, float* dtheta, float* P, const int* epos,
+                         float* dY_out, bool staged, cudaStream_t st) {
     if constexpr (k >= 2) {
         if (staged) {
             constexpr size_t smem = node_smem_bytes<k, TERMS>();
@@ -831,29 +1015,47 @@ int launch_backward_impl(const float* X, int w_in, long long B, const int* conn,
                 cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
                 return BITLOGIC_ERR_CUDA;
             kern<<<(unsigned)((w + kNodesPerBlock - 1) / kNodesPerBlock), kBwdWarps * 32, smem, st>>>(
-                X, w_in, B, conn, theta, w, gs, dtheta, P, dY_out);
+                X, w_in, B, conn, theta, w, gs, dtheta, P, epos, dY_out);
             return launch_status();
         }
     }
     dim3 grid((unsigned)((w + kFwdWarps - 1) / kFwdWarps));
     lut_backward_kernel<k, WANT_DX, TERMS><<<grid, kFwdWarps * 32, 0, st>>>(X, w_in, B, conn, theta, w, gs,
-                                                                            dtheta, P, dY_out);
+                                                                            dtheta, P, epos, dY_out);
     return launch_status();
 }
 
 template <int k>
 int launch_backward(const float* X, int w_in, long long B, const int* conn, const float* theta,
-                    int w, const GradSource& gs, float* dtheta, float* P, float* dY_out,
-                    cudaStream_t st) {
+                    int w, const GradSource& gs, float* dtheta, float* P, const int* epos,
+                    float* dY_out, cudaStream_t st) {
     const bool terms = gs.terms != nullptr;
     const bool staged = (B % 4 == 0) && aligned16(X) && aligned16(terms ? gs.terms : gs.dY) &&
                         (!dY_out || aligned16(dY_out)) && (!P || aligned16(P));
-    if (P) {
-        return terms ? launch_backward_impl<k, true, true>(X, w_in, B, conn, theta, w, gs, dtheta, P, dY_out, staged, st)
-                     : launch_backward_impl<k, true, false>(X, w_in, B, conn, theta, w, gs, dtheta, P, dY_out, staged, st);
+    if (staged && !P && !terms) {   // dtheta only, from dY rows
+        constexpr size_t smem = (size_t)kThetaWarps * theta_floats_per_warp<k>() * sizeof(float);
+        auto kern = lut_backward_theta_kernel<k>;
+        if (smem > 40 * 1024 &&
+            cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+            return BITLOGIC_ERR_CUDA;
+        // one wave of persistent warps filling every SM alike (nodes dealt
+        // round-robin, so warps differ by at most one node)
+        const long long resident = (long long)sm_count() * BITLOGIC_BWD_MIN_BLOCKS * kThetaWarps;
+        const long long warps = w < resident ? w : resident;
+        kern<<<(unsigned)((warps + kThetaWarps - 1) / kThetaWarps), kThetaWarps * 32, smem, st>>>(
+            X, w_in, B, conn, theta, w, gs.dY, gs.group, dtheta, dY_out);
+        return launch_status();
     }
-    return terms ? launch_backward_impl<k, false, true>(X, w_in, B, conn, theta, w, gs, dtheta, P, dY_out, staged, st)
-                 : launch_backward_impl<k, false, false>(X, w_in, B, conn, theta, w, gs, dtheta, P, dY_out, staged, st);
+    if (P) {
+        return terms ? launch_backward_impl<k, true, true>(X, w_in, B, conn, theta, w, gs, dtheta, P, epos, dY_out,
+                                                           staged, st)
+                     : launch_backward_impl<k, true, false>(X, w_in, B, conn, theta, w, gs, dtheta, P, epos, dY_out,
+                                                            staged, st);
+    }
+    return terms ? launch_backward_impl<k, false, true>(X, w_in, B, conn, theta, w, gs, dtheta, P, epos, dY_out,
+                                                        staged, st)
+                 : launch_backward_impl<k, false, false>(X, w_in, B, conn, theta, w, gs, dtheta, P, epos, dY_out,
+                                                         staged, st);
 }
 
 int check_layer(const void* X, int32_t w_in, int64_t B, const void* conn, const void* theta,
@@ -904,15 +1106,15 @@ extern "C" int bitlogic_lut_backward_ex(const float* X, int32_t w_in, int64_t B,
                                         const float* dY, int32_t dy_group,
                                         const float* up_terms, const int32_t* up_off,
                                         const int32_t* up_edge, int32_t up_edges,
-                                        float* dtheta, float* edge_terms, float* dY_out,
-                                        cudaStream_t stream) {
+                                        float* dtheta, float* edge_terms, const int32_t* edge_pos,
+                                        float* dY_out, cudaStream_t stream) {
     int st = check_layer(X, w_in, B, conn, theta, w, k);
     if (st) return st;
     if (!dtheta) return BITLOGIC_ERR_NULL;
     const bool terms = up_terms != nullptr;
     if (B > 0 && terms == (dY != nullptr)) return BITLOGIC_ERR_NULL;   // exactly one source
     if (terms) {
-        if (!up_off || !up_edge) return BITLOGIC_ERR_NULL;
+        if (!up_off) return BITLOGIC_ERR_NULL;   // up_edge NULL: terms in CSR order
         if (up_edges < 0) return BITLOGIC_ERR_SHAPE;
     } else if (dy_group < 1 || dy_group > w) {
         return BITLOGIC_ERR_SHAPE;
@@ -925,12 +1127,12 @@ extern "C" int bitlogic_lut_backward_ex(const float* X, int32_t w_in, int64_t B,
     }
     GradSource gs{dY, dy_group, up_terms, up_off, up_edge, up_edges};
     switch (k) {
-        case 1: return launch_backward<1>(X, w_in, B, conn, theta, w, gs, dtheta, edge_terms, dY_out, stream);
-        case 2: return launch_backward<2>(X, w_in, B, conn, theta, w, gs, dtheta, edge_terms, dY_out, stream);
-        case 3: return launch_backward<3>(X, w_in, B, conn, theta, w, gs, dtheta, edge_terms, dY_out, stream);
-        case 4: return launch_backward<4>(X, w_in, B, conn, theta, w, gs, dtheta, edge_terms, dY_out, stream);
-        case 5: return launch_backward<5>(X, w_in, B, conn, theta, w, gs, dtheta, edge_terms, dY_out, stream);
-        default: return launch_backward<6>(X, w_in, B, conn, theta, w, gs, dtheta, edge_terms, dY_out, stream);
+        case 1: return launch_backward<1>(X, w_in, B, conn, theta, w, gs, dtheta, edge_terms, edge_pos, dY_out, stream);
+        case 2: return launch_backward<2>(X, w_in, B, conn, theta, w, gs, dtheta, edge_terms, edge_pos, dY_out, stream);
+        case 3: return launch_backward<3>(X, w_in, B, conn, theta, w, gs, dtheta, edge_terms, edge_pos, dY_out, stream);
+        case 4: return launch_backward<4>(X, w_in, B, conn, theta, w, gs, dtheta, edge_terms, edge_pos, dY_out, stream);
+        case 5: return launch_backward<5>(X, w_in, B, conn, theta, w, gs, dtheta, edge_terms, edge_pos, dY_out, stream);
+        default: return launch_backward<6>(X, w_in, B, conn, theta, w, gs, dtheta, edge_terms, edge_pos, dY_out, stream);
     }
 }
 
@@ -941,7 +1143,7 @@ extern "C" int bitlogic_lut_backward_edges(const float* X, int32_t w_in, int64_t
                                            cudaStream_t stream) {
     if (B > 0 && !dY) return BITLOGIC_ERR_NULL;
     return bitlogic_lut_backward_ex(X, w_in, B, conn, theta, w, k, dY, 1,
-                                    nullptr, nullptr, nullptr, 0, dtheta, edge_terms, nullptr, stream);
+                                    nullptr, nullptr, nullptr, 0, dtheta, edge_terms, nullptr, nullptr, stream);
 }
 
 extern "C" int bitlogic_csr_reduce(const float* edge_terms, int64_t B, const int32_t* csr_off,
@@ -949,9 +1151,12 @@ extern "C" int bitlogic_csr_reduce(const float* edge_terms, int64_t B, const int
                                    float* dX, cudaStream_t stream) {
     if (B < 0 || w_in <= 0 || n_edges < 0) return BITLOGIC_ERR_SHAPE;
     if (B == 0) return BITLOGIC_OK;
-    if (!edge_terms || !csr_off || !csr_edge || !dX) return BITLOGIC_ERR_NULL;
+    if (!edge_terms || !csr_off || !dX) return BITLOGIC_ERR_NULL;   // csr_edge NULL: terms in CSR order
     const bool vec = (B % 4 == 0) && aligned16(edge_terms) && aligned16(dX);
-    dim3 grid((unsigned)((w_in + kCsrWarps - 1) / kCsrWarps));
+    const long long per_block = (long long)kCsrWarps * (vec ? 128 : 32);
+    const long long gy = (B + per_block - 1) / per_block;
+    if (gy > 65535) return BITLOGIC_ERR_SHAPE;
+    dim3 grid((unsigned)w_in, (unsigned)gy);
     if (vec)
         csr_reduce_kernel<true><<<grid, kCsrWarps * 32, 0, stream>>>(edge_terms, B, csr_off, csr_edge, w_in, n_edges, dX);
     else

@@ -16,7 +16,7 @@ from typing import Optional, Sequence
 import numpy as np
 import torch
 
-from . import (bitlogic_binarize_tables, bitlogic_build_csr, bitlogic_csr_reduce,
+from . import (bitlogic_binarize_tables, bitlogic_build_csr, bitlogic_csr_positions, bitlogic_csr_reduce,
                bitlogic_encode_thermometer, bitlogic_hard_forward, bitlogic_head_loss_ex,
                bitlogic_head_loss_workspace, bitlogic_lut_backward_ex, bitlogic_lut_forward,
                bitlogic_pack_bits)
@@ -44,6 +44,10 @@ class Network:
         off2, edge2 = bitlogic_build_csr(conn2, self.w1)
         self.off1, self.edge1 = torch.from_numpy(off1).to(dev), torch.from_numpy(edge1).to(dev)
         self.off2, self.edge2 = torch.from_numpy(off2).to(dev), torch.from_numpy(edge2).to(dev)
+        # CSR position of every edge: the per-edge gradient terms are stored
+        # in CSR order, so each input's terms are one contiguous block
+        self.pos1 = torch.from_numpy(bitlogic_csr_positions(edge1)).to(dev)
+        self.pos2 = torch.from_numpy(bitlogic_csr_positions(edge2)).to(dev)
 
 
 class TrainStep:
@@ -55,7 +59,8 @@ class TrainStep:
     ``keep_dy1`` to also write dY1, e.g. to check it)."""
 
     def __init__(self, net: Network, B: int, d: int, thresholds: Sequence[int], C: int,
-                 tau: float, want_dx1: bool = False, keep_dy1: bool = False, device="cuda"):
+                 tau: float, want_dx1: bool = False, keep_dy1: bool = False,
+                 fuse_dy1: bool = False, device="cuda"):
         dev = torch.device(device)
         self.net, self.B, self.d, self.C, self.tau = net, int(B), int(d), int(C), float(tau)
         self.thr = [int(t) for t in thresholds]
@@ -70,7 +75,11 @@ class TrainStep:
         self.logits = torch.empty(B, C, **f32)
         self.loss = torch.zeros(1, **f32)
         self.dyg = torch.empty(C, B, **f32)          # gradient row shared by each class's nodes
-        self.dy1 = torch.empty(net.w1, B, **f32) if keep_dy1 else None
+        # layer 1's output gradient: summed from layer 2's terms inside the
+        # layer-1 backward (fuse_dy1), or by a CSR reduction into dy1 that the
+        # dtheta-only kernel then reads
+        self.fuse_dy1 = bool(fuse_dy1)
+        self.dy1 = torch.empty(net.w1, B, **f32) if (keep_dy1 or not fuse_dy1) else None
         self.dth1 = torch.empty_like(net.theta1)
         self.dth2 = torch.empty_like(net.theta2)
         self.dbits = torch.empty(net.w_in, B, **f32) if want_dx1 else None
@@ -101,12 +110,19 @@ class TrainStep:
         bitlogic_lut_backward_ex(self.y1, n.conn2, n.theta2, self.dth2, dY=self.dyg,
                                  dy_group=n.w2 // self.C, edge_terms=self.edges2, stream=stream)
         mark("backward2")
-        bitlogic_lut_backward_ex(self.bits, n.conn1, n.theta1, self.dth1, up_terms=self.edges2,
-                                 up_off=n.off2, up_edge=n.edge2, edge_terms=self.edges1,
-                                 dY_out=self.dy1, stream=stream)
+        pos1 = n.pos1 if self.edges1 is not None else None
+        if self.fuse_dy1:
+            bitlogic_lut_backward_ex(self.bits, n.conn1, n.theta1, self.dth1, up_terms=self.edges2,
+                                     up_off=n.off2, up_edge=n.edge2, edge_terms=self.edges1,
+                                     edge_pos=pos1, dY_out=self.dy1, stream=stream)
+        else:
+            bitlogic_csr_reduce(self.edges2, n.off2, n.edge2, self.dy1, stream)
+            mark("csr2")
+            bitlogic_lut_backward_ex(self.bits, n.conn1, n.theta1, self.dth1, dY=self.dy1,
+                                     edge_terms=self.edges1, edge_pos=pos1, stream=stream)
         mark("backward1")
         if self.dbits is not None:
-            bitlogic_csr_reduce(self.edges1, n.off1, n.edge1, self.dbits, stream)
+            bitlogic_csr_reduce(self.edges1, n.off1, None, self.dbits, stream)
             mark("csr1")
 
     def run(self, stream=None, mark=_nomark):
@@ -114,10 +130,11 @@ class TrainStep:
         self.backward(stream, mark)
 
     # kernels one run() launches: encode 1, forwards 2, head 3, backwards 2
-    # (+ the layer-1 CSR reduction when the input gradient is wanted)
+    # (+ the CSR reduction of layer 2's terms unless fused, + the layer-1 CSR
+    # reduction when the input gradient is wanted)
     @property
     def kernels_per_run(self) -> int:
-        return 8 + (1 if self.dbits is not None else 0)
+        return 8 + (0 if self.fuse_dy1 else 1) + (1 if self.dbits is not None else 0)
 
 
 class HardInfer:

@@ -69,6 +69,21 @@ def test_build_csr_matches_inverse_map():
     assert edge2.tolist() == [0, 1, 2, 3]
 
 
+def test_csr_positions_invert_the_edge_map():
+    conn = synth.connectivity(200, 6, 97, seed=7)
+    off, edge = bl.bitlogic_build_csr(conn, 97)
+    pos = bl.bitlogic_csr_positions(edge)
+    np.testing.assert_array_equal(pos[edge], np.arange(edge.size))
+    np.testing.assert_array_equal(edge[pos], np.arange(edge.size))
+    # each input's edges occupy its CSR range
+    flat = conn.reshape(-1)
+    assert np.all(pos >= off[flat]) and np.all(pos < off[flat + 1])
+    for bad in ([0, 0, 1], [0, 3, 1], [-1, 0, 1]):
+        with pytest.raises(bl.BitLogicError) as e:
+            bl.bitlogic_csr_positions(np.array(bad, np.int32))
+        assert e.value.code == -7
+
+
 def test_build_csr_rejects_out_of_range():
     conn = np.array([[0, 5]], np.int32)
     with pytest.raises(bl.BitLogicError) as e:

@@ -91,10 +91,14 @@ def test_lut_backward(k, w_in, w, B):
     wth, wdx = oracle.lut_backward(X.astype(np.float64), conn, theta, dY.astype(np.float64))
     check_grad(dth, wth, "dtheta")
     check_grad(dX, wdx, "dX")
-    # dX skipped: dtheta unchanged, nothing else written
+    # dX skipped: the dtheta-only kernel (another summation order), within
+    # the tolerance of the oracle and deterministic from run to run
     dth2 = torch.full((w, 1 << k), np.nan, device="cuda")
     bl.bitlogic_lut_backward(dev(X), dev(conn), dev(theta), dev(dY), dth2)
-    check_exact(dth2.cpu().numpy(), dth.cpu().numpy(), "dtheta without dX")
+    check_grad(dth2, wth, "dtheta without dX")
+    dth3 = torch.full((w, 1 << k), np.nan, device="cuda")
+    bl.bitlogic_lut_backward(dev(X), dev(conn), dev(theta), dev(dY), dth3)
+    check_exact(dth3.cpu().numpy(), dth2.cpu().numpy(), "dtheta without dX, second run")
     no_device_error()
 
 
@@ -158,6 +162,34 @@ def test_backward_from_upstream_terms(k, w_in, w, B):
         dY[conn_b.reshape(-1)[e]] += terms[e].astype(np.float64)
     wth, _ = oracle.lut_backward(X.astype(np.float64), conn, theta, dY, want_dx=False)
     check_grad(dth, wth, "dtheta")
+    # without this layer's own terms: the dtheta-only kernel reads the
+    # upstream rows through its ring (another summation order for dtheta)
+    dth_t = torch.full((w, 1 << k), np.nan, device="cuda")
+    out_t = torch.full((w, B), np.nan, device="cuda")
+    bl.bitlogic_lut_backward_ex(dev(X), dev(conn), dev(theta), dth_t, up_terms=dev(terms),
+                                up_off=dev(off_b), up_edge=dev(edge_b), dY_out=out_t)
+    check_exact(out_t.cpu().numpy(), out.cpu().numpy(), "dY from terms (dtheta-only kernel)")
+    check_grad(dth_t, wth, "dtheta (dtheta-only kernel)")
+    # the same with every per-edge buffer in CSR order: upstream rows
+    # permuted to CSR positions (no edge map), this layer's terms stored at
+    # its own CSR positions; all results identical bit for bit
+    off_a, edge_a = bl.bitlogic_build_csr(conn, w_in)
+    pos_a = bl.bitlogic_csr_positions(edge_a)
+    dth_c = torch.empty(w, 1 << k, device="cuda")
+    out_c = torch.empty(w, B, device="cuda")
+    P_c = torch.full((w * k, B), np.nan, device="cuda")
+    bl.bitlogic_lut_backward_ex(dev(X), dev(conn), dev(theta), dth_c, up_terms=dev(terms[edge_b]),
+                                up_off=dev(off_b), up_edge=None, edge_terms=P_c, edge_pos=dev(pos_a),
+                                dY_out=out_c)
+    check_exact(out_c.cpu().numpy(), out.cpu().numpy(), "dY from CSR-ordered terms")
+    check_exact(dth_c.cpu().numpy(), dth.cpu().numpy(), "dtheta from CSR-ordered terms")
+    check_exact(P_c.cpu().numpy(), P.cpu().numpy()[edge_a], "edge terms stored in CSR order")
+    dX = torch.empty(w_in, B, device="cuda")
+    dX_c = torch.empty(w_in, B, device="cuda")
+    bl.bitlogic_csr_reduce(P, dev(off_a), dev(edge_a), dX)
+    bl.bitlogic_csr_reduce(P_c, dev(off_a), None, dX_c)
+    check_exact(dX_c.cpu().numpy(), dX.cpu().numpy(), "csr_reduce of CSR-ordered terms")
+    no_device_error()
     no_device_error()
 
 

@@ -29,14 +29,14 @@ pytestmark = pytest.mark.gpu
 oracle.set_threads(os.cpu_count() or 1)
 
 
-def _step(wl, want_dx1, seed=0, k=None, keep_dy1=True):
+def _step(wl, want_dx1, seed=0, k=None, keep_dy1=True, fuse_dy1=False):
     if k is not None:
         wl = synth.Workload(wl.name, wl.batch, wl.d, wl.classes, wl.sigma, wl.thresholds, wl.widths, k, wl.tau)
     conn1, th1, conn2, th2 = synth.network(wl, seed)
     x, labels = synth.blob_batch(wl.batch, wl.d, wl.classes, wl.sigma, seed=seed + 7)
     net = Network(conn1, th1, conn2, th2, wl.w_in)
     st = TrainStep(net, wl.batch, wl.d, wl.thresholds, wl.classes, wl.tau, want_dx1=want_dx1,
-                   keep_dy1=keep_dy1)
+                   keep_dy1=keep_dy1, fuse_dy1=fuse_dy1)
     st.load(x.cuda(), labels.cuda())
     st.run()
     torch.cuda.synchronize()
@@ -76,6 +76,14 @@ def test_tiny_step_all_outputs():
 @pytest.mark.parametrize("k", [6, 2])
 def test_mnist_step_all_outputs(k):
     wl, st, x, labels, params = _step(synth.WORKLOADS["mnist"], want_dx1=False, k=k)
+    _full_compare(wl, st, x, labels, params, False)
+
+
+def test_mnist_step_fused_layer1_gradient():
+    # layer 1's output gradient summed inside its backward from layer 2's
+    # CSR-ordered terms, instead of a CSR reduction followed by the
+    # dtheta-only kernel
+    wl, st, x, labels, params = _step(synth.WORKLOADS["mnist"], want_dx1=False, fuse_dy1=True)
     _full_compare(wl, st, x, labels, params, False)
 
 
