@@ -502,7 +502,7 @@ constexpr size_t node_smem_bytes() {
 // stages then read.  dtheta: each lane's partials, then the lanes of each
 // parity, then the node's warps, in a fixed order.  Needs k >= 2,
 // B % 4 == 0 and 16-byte aligned X and sources.
-template <int k, bool WANT_DX, bool TERMS>
+template <int k, bool WANT_DX, bool TERMS, bool POS>
 __global__ void __launch_bounds__(kBwdWarps * 32, BITLOGIC_BWD_MIN_BLOCKS)
 lut_backward_node_kernel(const float* __restrict__ X, int w_in, long long B,
                          const int* __restrict__ conn, const float* __restrict__ theta, int w,
@@ -583,11 +583,9 @@ lut_backward_node_kernel(const float* __restrict__ X, int w_in, long long B,
     float* pst[NQ];   // this lane's stored slots 2q + h, at its first sample
 #pragma unroll
     for (int q = 0; q < NQ; ++q) {
-        pst[q] = nullptr;
-        if constexpr (WANT_DX) {
-            const long long e = (long long)jj * k + (2 * q + h < k ? 2 * q + h : 0);
-            pst[q] = P + (live ? edge_row(epos, e, (long long)w * k) : e) * B + pair;
-        }
+        const long long e = (long long)jj * k + (2 * q + h < k ? 2 * q + h : 0);
+        if constexpr (POS) pst[q] = P + (live ? edge_row(epos, e, (long long)w * k) : e) * B + pair;
+        else pst[q] = P + e * B + pair;
     }
     const int nst = (int)((B + CH - 1) / CH);
     const int per = (nst + kWarpsPerNode - 1) / kWarpsPerNode;
@@ -1010,7 +1008,10 @@ int launch_backward_impl(const float* X, int w_in, long long B, const int* conn,
     if constexpr (k >= 2) {
         if (staged) {
             constexpr size_t smem = node_smem_bytes<k, TERMS>();
-            auto kern = lut_backward_node_kernel<k, WANT_DX, TERMS>;
+            // term rows at caller-given positions: a separate instantiation,
+            // so the common form compiles without the position lookups
+            auto kern = (WANT_DX && epos) ? lut_backward_node_kernel<k, WANT_DX, TERMS, WANT_DX>
+                                          : lut_backward_node_kernel<k, WANT_DX, TERMS, false>;
             if (smem > 48 * 1024 &&
                 cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
                 return BITLOGIC_ERR_CUDA;

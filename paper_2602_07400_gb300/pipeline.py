@@ -60,7 +60,7 @@ class TrainStep:
 
     def __init__(self, net: Network, B: int, d: int, thresholds: Sequence[int], C: int,
                  tau: float, want_dx1: bool = False, keep_dy1: bool = False,
-                 fuse_dy1: bool = False, device="cuda"):
+                 fuse_dy1: bool = False, csr_order: bool = False, device="cuda"):
         dev = torch.device(device)
         self.net, self.B, self.d, self.C, self.tau = net, int(B), int(d), int(C), float(tau)
         self.thr = [int(t) for t in thresholds]
@@ -79,6 +79,9 @@ class TrainStep:
         # layer-1 backward (fuse_dy1), or by a CSR reduction into dy1 that the
         # dtheta-only kernel then reads
         self.fuse_dy1 = bool(fuse_dy1)
+        # per-edge terms stored in CSR order (each input's terms contiguous,
+        # read without the edge map) instead of edge order
+        self.csr_order = bool(csr_order)
         self.dy1 = torch.empty(net.w1, B, **f32) if (keep_dy1 or not fuse_dy1) else None
         self.dth1 = torch.empty_like(net.theta1)
         self.dth2 = torch.empty_like(net.theta2)
@@ -107,22 +110,25 @@ class TrainStep:
 
     def backward(self, stream=None, mark=_nomark):
         n = self.net
+        co = self.csr_order
         bitlogic_lut_backward_ex(self.y1, n.conn2, n.theta2, self.dth2, dY=self.dyg,
-                                 dy_group=n.w2 // self.C, edge_terms=self.edges2, stream=stream)
+                                 dy_group=n.w2 // self.C, edge_terms=self.edges2,
+                                 edge_pos=n.pos2 if co else None, stream=stream)
         mark("backward2")
-        pos1 = n.pos1 if self.edges1 is not None else None
+        pos1 = n.pos1 if (co and self.edges1 is not None) else None
+        edge2 = None if co else n.edge2
         if self.fuse_dy1:
             bitlogic_lut_backward_ex(self.bits, n.conn1, n.theta1, self.dth1, up_terms=self.edges2,
-                                     up_off=n.off2, up_edge=n.edge2, edge_terms=self.edges1,
+                                     up_off=n.off2, up_edge=edge2, edge_terms=self.edges1,
                                      edge_pos=pos1, dY_out=self.dy1, stream=stream)
         else:
-            bitlogic_csr_reduce(self.edges2, n.off2, n.edge2, self.dy1, stream)
+            bitlogic_csr_reduce(self.edges2, n.off2, edge2, self.dy1, stream)
             mark("csr2")
             bitlogic_lut_backward_ex(self.bits, n.conn1, n.theta1, self.dth1, dY=self.dy1,
                                      edge_terms=self.edges1, edge_pos=pos1, stream=stream)
         mark("backward1")
         if self.dbits is not None:
-            bitlogic_csr_reduce(self.edges1, n.off1, None, self.dbits, stream)
+            bitlogic_csr_reduce(self.edges1, n.off1, None if co else n.edge1, self.dbits, stream)
             mark("csr1")
 
     def run(self, stream=None, mark=_nomark):
