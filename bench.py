@@ -21,6 +21,7 @@ ranks and ``value`` sums the samples of all ranks.
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import os
 import statistics
@@ -177,6 +178,38 @@ def call_work(wl, B, fuse_dy1=False):
     }
 
 
+# DRAM traffic per launch of the roofline kernel, dram__bytes_read.sum +
+# dram__bytes_write.sum from one ncu capture, keyed by workload
+# and call.  Valid only for the kernel source it was taken on: the source
+# file's SHA-256 is recorded, and any later change reports null.
+TRAFFIC = {
+    ("mnist", "backward2"): {
+        "bytes": 58.816768e6 + 146.201856e6, "source": "lut_soft.cu",
+        "sha256": "5489bab3e02c6c3da48b76c7b638cf0db63090fb20e5b3bb43ab35490eb3f674",
+        "note": "ncu capture of this workload"},
+    ("hard_cifar10", "hard1"): {
+        "bytes": 16 * (1.218435e9 + 2.055860e9), "source": "hard.cu",
+        "sha256": "10ccb1e76ad68c073d03604ace6aede6b750faa1a4edd52a47d3c55b57b91c61",
+        "note": "ncu capture at 2^18 samples, scaled x16 to 2^22 by the words processed"},
+}
+
+
+def kernel_traffic(workload: str, call: str):
+    """(bytes per launch, note) when the capture matches the current source, else (None, why)."""
+    t = TRAFFIC.get((workload, call))
+    if t is None:
+        return None, "no capture for this workload"
+    path = os.path.join(ROOT, "paper_2602_07400_gb300", "csrc", t["source"])
+    try:
+        with open(path, "rb") as f:
+            digest = hashlib.sha256(f.read()).hexdigest()
+    except OSError:
+        return None, "kernel source not found"
+    if digest != t["sha256"]:
+        return None, f"{t['source']} changed since the capture"
+    return t["bytes"], t["note"]
+
+
 KERNEL_OF_CALL = {
     "encode": "encode_soft_kernel", "forward1": "lut_forward_staged_kernel<k>",
     "forward2": "lut_forward_staged_kernel<k>", "head": "head_* (3 kernels)",
@@ -315,7 +348,8 @@ def run_ours(args):
         else:
             roof = {"bound": "hbm", "achieved": byts / t_s / 1e9, "peak": hbm, "unit": "GB/s"}
         roof["frac"] = roof["achieved"] / roof["peak"]
-        roof.update({"traffic": None, "kernel": KERNEL_OF_CALL[dom], "call": dom,
+        traffic, traffic_note = kernel_traffic(wl.name, dom)
+        roof.update({"traffic": traffic, "traffic_source": traffic_note, "kernel": KERNEL_OF_CALL[dom], "call": dom,
                      "ms_per_launch": per_call_ms[dom], "algorithmic_bytes": byts,
                      "algorithmic_ops": ops, "peak_source": f"{peak_kind} (HBM), "
                      f"152 SMs x {FP32_LANES_PER_SM} fp32 lanes x {sm_max:.0f} MHz (alu)"})
