@@ -143,13 +143,20 @@ pack_bits_kernel(const uint8_t* __restrict__ x, long long N, int d, Thresholds t
         for (int i = 0; i < 8; ++i) lo7[i] = r[i] & 0x7f7f7f7fu;
         uint32_t* out = xp + (long long)(f0 + fl) * th.b * W + q;
         for (int i = 0; i < th.b; ++i) {
-            const uint32_t C = sC[i], orm = sOr[i];   // OR form below 127, AND form above
+            const uint32_t C = sC[i];
             uint32_t word = 0u;
+            if (sOr[i]) {   // T < 127: OR form (warp-uniform branch)
 #pragma unroll
-            for (int i8 = 0; i8 < 8; ++i8) {
-                const uint32_t sum = lo7[i8] + C;
-                const uint32_t hb = ((r[i8] & sum) | ((r[i8] | sum) & orm)) & 0x80808080u;
-                word += i8 < 7 ? __umulhi(hb, 1u << ((25 + i8) & 31)) : hb;   // disjoint bits
+                for (int i8 = 0; i8 < 8; ++i8) {
+                    const uint32_t hb = (r[i8] | (lo7[i8] + C)) & 0x80808080u;
+                    word += i8 < 7 ? __umulhi(hb, 1u << ((25 + i8) & 31)) : hb;   // disjoint bits
+                }
+            } else {        // T >= 127: AND form
+#pragma unroll
+                for (int i8 = 0; i8 < 8; ++i8) {
+                    const uint32_t hb = (r[i8] & (lo7[i8] + C)) & 0x80808080u;
+                    word += i8 < 7 ? __umulhi(hb, 1u << ((25 + i8) & 31)) : hb;
+                }
             }
             out[(long long)i * W] = word;
         }
