@@ -17,6 +17,8 @@
 // through a ring of shared-memory stages filled by 16-byte cp.async copies,
 // which overlaps the gathers with the trees of earlier stages without
 // spending registers.
+#include <type_traits>
+
 #include "common.cuh"
 
 namespace bitlogic {
@@ -667,9 +669,12 @@ lut_backward_node_kernel(const float* __restrict__ X, int w_in, long long B,
         const bool full = sbase + CH <= B;
         const float* rbuf = buf + pair;
         const float* gsrc = TERMS ? gbuf + (i % kGatherStages) * CH + pair : rbuf + k * CH;
+        // full stages (all but a ragged last one) compile without range checks
+        auto stage = [&](auto full_stage) {
+        constexpr bool kFull = decltype(full_stage)::value;
 #pragma unroll 2
         for (int c = 0; c < CH / 16; ++c) {
-            const bool in = full || sbase + 16 * c + pair < B;
+            const bool in = kFull || sbase + 16 * c + pair < B;
             float x[k], omx[k], dx[k];
 #pragma unroll
             for (int q = 0; q < k; ++q) {
@@ -702,6 +707,9 @@ lut_backward_node_kernel(const float* __restrict__ X, int w_in, long long B,
                 }
             }
         }
+        };
+        if (full) stage(std::true_type{});
+        else stage(std::false_type{});
         __syncwarp();
         rb = (rb + 1 == kStages) ? 0 : rb + 1;
     }
