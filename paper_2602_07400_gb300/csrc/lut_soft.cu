@@ -949,20 +949,35 @@ csr_reduce_kernel(const float* __restrict__ P, long long B, const int* __restric
     const long long s = ((long long)blockIdx.y * kCsrWarps + warp) * SPW + (VEC ? 4 : 1) * lane;
     const bool in = s < B;   // vector path: B % 4 == 0, all four samples in range
     float* out = dX + (long long)i * B + s;
+    // loads of up to kCsrBatch rows are issued before the first add; the
+    // adds keep increasing position order
+    constexpr int kCsrBatch = 8;
     if constexpr (VEC) {
         float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 8
-        for (int q = 0; q < deg; ++q) {
-            const int id = edge_id(q);
-            if (in && id >= 0) acc = add4(acc, ldg4(P + (long long)id * B + s));
+        for (int q0 = 0; q0 < deg; q0 += kCsrBatch) {
+            float4 v[kCsrBatch];
+#pragma unroll
+            for (int u = 0; u < kCsrBatch; ++u) {
+                const int id = q0 + u < deg ? edge_id(q0 + u) : -1;   // warp-uniform condition
+                v[u] = (in && id >= 0) ? ldg4(P + (long long)id * B + s) : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+#pragma unroll
+            for (int u = 0; u < kCsrBatch; ++u)
+                if (q0 + u < deg) acc = add4(acc, v[u]);
         }
         if (in) *reinterpret_cast<float4*>(out) = acc;
     } else {
         float acc = 0.f;
-#pragma unroll 8
-        for (int q = 0; q < deg; ++q) {
-            const int id = edge_id(q);
-            if (in && id >= 0) acc += __ldg(P + (long long)id * B + s);
+        for (int q0 = 0; q0 < deg; q0 += kCsrBatch) {
+            float v[kCsrBatch];
+#pragma unroll
+            for (int u = 0; u < kCsrBatch; ++u) {
+                const int id = q0 + u < deg ? edge_id(q0 + u) : -1;
+                v[u] = (in && id >= 0) ? __ldg(P + (long long)id * B + s) : 0.f;
+            }
+#pragma unroll
+            for (int u = 0; u < kCsrBatch; ++u)
+                if (q0 + u < deg) acc += v[u];
         }
         if (in) *out = acc;
     }

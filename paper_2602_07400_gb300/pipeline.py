@@ -60,7 +60,7 @@ class TrainStep:
 
     def __init__(self, net: Network, B: int, d: int, thresholds: Sequence[int], C: int,
                  tau: float, want_dx1: bool = False, keep_dy1: bool = False,
-                 fuse_dy1: bool = False, csr_order: bool = False, device="cuda"):
+                 fuse_dy1: bool = False, csr_order: bool = True, device="cuda"):
         dev = torch.device(device)
         self.net, self.B, self.d, self.C, self.tau = net, int(B), int(d), int(C), float(tau)
         self.thr = [int(t) for t in thresholds]

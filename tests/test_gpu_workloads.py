@@ -29,14 +29,14 @@ pytestmark = pytest.mark.gpu
 oracle.set_threads(os.cpu_count() or 1)
 
 
-def _step(wl, want_dx1, seed=0, k=None, keep_dy1=True, fuse_dy1=False):
+def _step(wl, want_dx1, seed=0, k=None, keep_dy1=True, fuse_dy1=False, csr_order=True):
     if k is not None:
         wl = synth.Workload(wl.name, wl.batch, wl.d, wl.classes, wl.sigma, wl.thresholds, wl.widths, k, wl.tau)
     conn1, th1, conn2, th2 = synth.network(wl, seed)
     x, labels = synth.blob_batch(wl.batch, wl.d, wl.classes, wl.sigma, seed=seed + 7)
     net = Network(conn1, th1, conn2, th2, wl.w_in)
     st = TrainStep(net, wl.batch, wl.d, wl.thresholds, wl.classes, wl.tau, want_dx1=want_dx1,
-                   keep_dy1=keep_dy1, fuse_dy1=fuse_dy1)
+                   keep_dy1=keep_dy1, fuse_dy1=fuse_dy1, csr_order=csr_order)
     st.load(x.cuda(), labels.cuda())
     st.run()
     torch.cuda.synchronize()
@@ -85,6 +85,17 @@ def test_mnist_step_fused_layer1_gradient():
     # dtheta-only kernel
     wl, st, x, labels, params = _step(synth.WORKLOADS["mnist"], want_dx1=False, fuse_dy1=True)
     _full_compare(wl, st, x, labels, params, False)
+
+
+def test_mnist_step_edge_ordered_terms():
+    # layer 2's per-edge terms in edge order, read through the CSR edge map
+    wl, st, x, labels, params = _step(synth.WORKLOADS["mnist"], want_dx1=False, csr_order=False)
+    _full_compare(wl, st, x, labels, params, False)
+
+
+def test_tiny_step_edge_ordered_terms():
+    wl, st, x, labels, params = _step(synth.WORKLOADS["tiny"], want_dx1=True, csr_order=False)
+    _full_compare(wl, st, x, labels, params, True)
 
 
 def test_mnist_bench_configuration_matches():
