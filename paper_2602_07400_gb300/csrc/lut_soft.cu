@@ -264,11 +264,15 @@ lut_forward_staged_kernel(const float* __restrict__ X, int w_in, long long B,
     if (j >= w) return;
     int rows[k];
     load_rows<k>(conn, j, w_in, lane, rows);
-    // lane l < K / S: sigmoid of subtable l's entries, then its coefficients
+    // sigmoid of the table spread over the lanes (entries l, l + 32), then
+    // lane l < K / S turns subtable l into its Moebius coefficients
+#pragma unroll
+    for (int a = lane; a < K; a += 32) sCoef[warp][a] = sigmoidf(__ldg(theta + (long long)j * K + a));
+    __syncwarp();
     if (lane < K / S) {
         float c[S];
 #pragma unroll
-        for (int a = 0; a < S; ++a) c[a] = sigmoidf(__ldg(theta + (long long)j * K + lane * S + a));
+        for (int a = 0; a < S; ++a) c[a] = sCoef[warp][lane * S + a];
         moebius<L>(c);
 #pragma unroll
         for (int a = 0; a < S; ++a) sCoef[warp][lane * S + a] = c[a];
@@ -672,8 +676,7 @@ lut_backward_node_kernel(const float* __restrict__ X, int w_in, long long B,
         // full stages (all but a ragged last one) compile without range checks
         auto stage = [&](auto full_stage) {
         constexpr bool kFull = decltype(full_stage)::value;
-#pragma unroll 2
-        for (int c = 0; c < CH / 16; ++c) {
+        auto sample = [&](int c) {
             const bool in = kFull || sbase + 16 * c + pair < B;
             float x[k], omx[k], dx[k];
 #pragma unroll
@@ -706,6 +709,13 @@ lut_backward_node_kernel(const float* __restrict__ X, int w_in, long long B,
                     if (in && (h == 0 || od < k)) pst[q][sbase + 16 * c] = full_dx;
                 }
             }
+        };
+        if constexpr (kFull) {
+#pragma unroll 4
+            for (int c = 0; c < CH / 16; ++c) sample(c);
+        } else {
+#pragma unroll 2
+            for (int c = 0; c < CH / 16; ++c) sample(c);
         }
         };
         if (full) stage(std::true_type{});
