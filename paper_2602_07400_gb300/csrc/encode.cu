@@ -51,6 +51,55 @@ encode_soft_kernel(const uint8_t* __restrict__ x, long long B, int d, Thresholds
     }
 }
 
+// Vector form (B % 4 == 0, 16-byte aligned output): tiles of 32 features x
+// 128 samples; each thread loads 16 feature bytes of one sample (one 16-byte
+// load when d % 16 == 0 and x is aligned), the tile is transposed through
+// shared memory, and each thread writes 4 consecutive samples of a wire row
+// as one float4 (512 contiguous bytes per warp).
+constexpr int kEncVS = 128;   // samples per tile (vector form)
+
+__global__ void __launch_bounds__(256)
+encode_soft_vec_kernel(const uint8_t* __restrict__ x, long long B, int d, Thresholds th,
+                       float* __restrict__ bits, bool vec16) {
+    __shared__ __align__(16) uint8_t tile[kEncTF][kEncVS];   // feature-major
+    __shared__ uint32_t sT[32];
+    if (threadIdx.x < th.b) sT[threadIdx.x] = threshold_at(th, threadIdx.x);
+    const long long s0 = (long long)blockIdx.y * kEncVS;
+    const int f0 = blockIdx.x * kEncTF;
+    const int nf = min(kEncTF, d - f0);
+    {   // thread t: sample t / 2, features 16 (t % 2) .. 16 (t % 2) + 15
+        const int sl = threadIdx.x >> 1, half = threadIdx.x & 1;
+        const long long s = s0 + sl;
+        uint32_t v[4] = {0u, 0u, 0u, 0u};
+        if (s < B) {
+            const uint8_t* p = x + s * d + f0 + 16 * half;
+            if (vec16 && nf == kEncTF) {
+                const uint4 a = __ldg(reinterpret_cast<const uint4*>(p));
+                v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+            } else {
+#pragma unroll
+                for (int f = 0; f < 16; ++f)
+                    if (16 * half + f < nf) v[f >> 2] |= (uint32_t)__ldg(p + f) << (8 * (f & 3));
+            }
+        }
+#pragma unroll
+        for (int f = 0; f < 16; ++f) tile[16 * half + f][sl] = (uint8_t)(v[f >> 2] >> (8 * (f & 3)));
+    }
+    __syncthreads();
+    const int u = threadIdx.x & 31, rg = threadIdx.x >> 5;   // 8 rows per pass
+    const long long s = s0 + 4 * u;
+    if (s >= B) return;   // B % 4 == 0: the thread's four samples are in range
+    const int rows = nf * th.b;
+    for (int r = rg; r < rows; r += 8) {
+        const int f = r / th.b, i = r - f * th.b;
+        const uint32_t q = *reinterpret_cast<const uint32_t*>(&tile[f][4 * u]);
+        const uint32_t T = sT[i];
+        const float4 o = make_float4((q & 0xffu) > T ? 1.0f : 0.0f, ((q >> 8) & 0xffu) > T ? 1.0f : 0.0f,
+                                     ((q >> 16) & 0xffu) > T ? 1.0f : 0.0f, (q >> 24) > T ? 1.0f : 0.0f);
+        *reinterpret_cast<float4*>(bits + ((long long)(f0 + f) * th.b + i) * B + s) = o;
+    }
+}
+
 // --------------------------------------------------------------- packed --
 //
 // One lane per output word (32 samples), so every store is a coalesced
@@ -179,6 +228,14 @@ extern "C" int bitlogic_encode_thermometer(const uint8_t* x, int64_t B, int32_t 
     if (B < 0 || d <= 0) return BITLOGIC_ERR_SHAPE;
     if (B == 0) return BITLOGIC_OK;   // an empty batch may come as NULL
     if (!x || !bits) return BITLOGIC_ERR_NULL;
+    if (B % 4 == 0 && aligned16(bits)) {
+        const long long gy = (B + kEncVS - 1) / kEncVS;
+        if (gy > 65535) return BITLOGIC_ERR_SHAPE;
+        const bool vec16 = (d % 16 == 0) && aligned16(x);
+        dim3 grid((unsigned)((d + kEncTF - 1) / kEncTF), (unsigned)gy);
+        encode_soft_vec_kernel<<<grid, 256, 0, stream>>>(x, B, d, th, bits, vec16);
+        return launch_status();
+    }
     const long long gy = (B + kEncTS - 1) / kEncTS;
     if (gy > 65535) return BITLOGIC_ERR_SHAPE;
     dim3 grid((unsigned)((d + kEncTF - 1) / kEncTF), (unsigned)gy);

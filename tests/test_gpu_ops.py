@@ -29,7 +29,8 @@ def no_device_error():
 
 # ---------------------------------------------------------------- encoder --
 
-@pytest.mark.parametrize("B,d,b", [(1, 5, 3), (37, 784, 3), (256, 70, 7), (1000, 33, 15), (65, 9, 32), (3, 1, 1)])
+@pytest.mark.parametrize("B,d,b", [(1, 5, 3), (37, 784, 3), (256, 70, 7), (1000, 33, 15), (65, 9, 32), (3, 1, 1),
+                                   (1024, 784, 3), (132, 3072, 7)])
 def test_encode_thermometer(B, d, b):
     rng = np.random.default_rng(B * 7 + d)
     x = rng.integers(0, 256, size=(B, d), dtype=np.uint8)
