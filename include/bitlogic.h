@@ -186,7 +186,7 @@ int bitlogic_head_loss_ex(const float* Y, int32_t w, int64_t B, int32_t C, float
  *   passes every input and output.
  *   Scratch: a fixed 8 MiB device array inside the library, reserved on
  *   every GPU that loads it until the process exits.  The call requires
- *   bitlogic_head_loss_workspace(B, C) <= 8 MiB (about B * C <= 1M) and
+ *   bitlogic_head_loss_workspace(B, C) <= 8 MiB (about B * C <= 340K) and
  *   returns BITLOGIC_ERR_TOO_LARGE otherwise, launching nothing.
  *   The first call on a device looks up the array's device address (a
  *   runtime query, not an allocation); make that first call before any

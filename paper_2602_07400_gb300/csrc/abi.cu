@@ -1,8 +1,28 @@
 // Host-side parts of the C ABI that launch no kernels: status strings, the
 // inverse-connectivity (CSR) builder, and the device-side index flag reader.
+#include <atomic>
 #include <vector>
 
 #include "common.cuh"
+
+namespace bitlogic {
+
+int sm_count() {
+    constexpr int kMaxDevices = 64;
+    static std::atomic<int> cache[kMaxDevices];   // 0: not queried yet
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 152;
+    if (dev < kMaxDevices) {
+        const int c = cache[dev].load(std::memory_order_relaxed);
+        if (c > 0) return c;
+    }
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 152;
+    if (dev < kMaxDevices) cache[dev].store(n, std::memory_order_relaxed);
+    return n;
+}
+
+}  // namespace bitlogic
 
 extern "C" int bitlogic_internal_index_error_lut_soft(cudaStream_t);
 extern "C" int bitlogic_internal_index_error_head(cudaStream_t);

@@ -33,6 +33,10 @@ inline int launch_status() {
 
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+// Number of SMs of the current device (queried once per device, then
+// cached; 152 if the query fails).  Defined in abi.cu.
+int sm_count();
+
 // Thresholds travel by value in the kernel parameters: no constant-memory
 // state is shared between calls or streams.
 struct Thresholds {

@@ -749,14 +749,6 @@ long long hard_word_chunk(int w_in, long long W) {
     return c < W ? c : W;
 }
 
-int sm_count() {
-    int dev = 0, n = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
-        return 152;
-    return n;
-}
-
 // Opt in to more than the default 48 KB of shared memory per block when the
 // dynamic part plus the kernel's static part (a few KB) may exceed it.
 template <typename F>

@@ -45,23 +45,28 @@ head_group_sum_kernel(const float* __restrict__ Y, long long B, int C, int g, fl
 }
 
 // Vector form (B % 4 == 0, 16-byte aligned Y): one block of 32 warps per
-// (class, 128 samples), lane = 4 consecutive samples, warp r sums rows r,
-// r + 32, ... of the group with 16-byte loads (enough loads in flight for
-// HBM), then thread t adds the 32 warps' partial sums of sample t in order.
+// (class, row split, 128 samples), lane = 4 consecutive samples, warp r sums
+// rows r, r + 32, ... of the split with 16-byte loads, then thread t adds the
+// 32 warps' partial sums of sample t in order.  With one split the block
+// writes the logits; with several (so that enough blocks pull from HBM) it
+// writes the split's sum, and the softmax kernel adds the splits in order.
 constexpr int kSumVecWarps = 32;
+constexpr int kMaxRowSplits = 4;
 
 __global__ void __launch_bounds__(kSumVecWarps * 32)
 head_group_sum_vec_kernel(const float* __restrict__ Y, long long B, int C, int g, float tau,
-                          float* __restrict__ logits) {
+                          float* __restrict__ logits, float* __restrict__ split_sums, int splits,
+                          int rows_per_split) {
     __shared__ __align__(16) float part[kSumVecWarps][128];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int c = blockIdx.x;
+    const int c = blockIdx.x / splits, rs = blockIdx.x - c * splits;
+    const int r0 = rs * rows_per_split, r1 = min(g, r0 + rows_per_split);
     const long long s4 = (long long)blockIdx.y * 128 + 4 * lane;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
     if (s4 < B) {   // B % 4 == 0: all four samples are in range
         const float* base = Y + (long long)c * g * B + s4;
 #pragma unroll 4
-        for (int r = warp; r < g; r += kSumVecWarps) {
+        for (int r = r0 + warp; r < r1; r += kSumVecWarps) {
             const float4 v = __ldg(reinterpret_cast<const float4*>(base + (long long)r * B));
             acc.x += v.x;
             acc.y += v.y;
@@ -76,7 +81,10 @@ head_group_sum_vec_kernel(const float* __restrict__ Y, long long B, int C, int g
         float t = 0.f;
 #pragma unroll 8
         for (int q = 0; q < kSumVecWarps; ++q) t += part[q][threadIdx.x];
-        if (s < B) logits[s * C + c] = t / tau;
+        if (s < B) {
+            if (splits == 1) logits[s * C + c] = t / tau;
+            else split_sums[((long long)rs * B + s) * C + c] = t;
+        }
     }
 }
 
@@ -95,12 +103,21 @@ __device__ __forceinline__ float warp_sum(float v) {
 constexpr int kSoftWarps = 8;
 
 __global__ void __launch_bounds__(kSoftWarps * 32)
-head_softmax_kernel(const float* __restrict__ logits, long long B, int C,
+head_softmax_kernel(float* __restrict__ logits, long long B, int C,
                     const int* __restrict__ labels, float* __restrict__ dlogit,
-                    float* __restrict__ per_sample, float tau, float* __restrict__ dYg) {
+                    float* __restrict__ per_sample, float tau, float* __restrict__ dYg,
+                    const float* __restrict__ split_sums, int splits) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const long long s = (long long)blockIdx.x * kSoftWarps + warp;
     if (s >= B) return;
+    if (split_sums) {   // logits from the row splits' sums, added in split order
+        for (int c = lane; c < C; c += 32) {
+            float t = 0.f;
+            for (int rs = 0; rs < splits; ++rs) t += __ldg(split_sums + ((long long)rs * B + s) * C + c);
+            logits[s * C + c] = t / tau;
+        }
+        __syncwarp();
+    }
     const float* l = logits + s * C;
     float m = -FLT_MAX;
     for (int c = lane; c < C; c += 32) m = fmaxf(m, l[c]);
@@ -178,8 +195,8 @@ extern "C" size_t bitlogic_head_loss_workspace(int64_t B, int32_t C) {
     if (B <= 0 || C <= 0) return 0;
     const size_t bc = (size_t)B * (size_t)C * sizeof(float);
     // dlogit [B][C], per-sample loss [B], logits [B][C] (used when the
-    // caller passes no logits buffer)
-    return align_up(bc) + align_up((size_t)B * sizeof(float)) + align_up(bc);
+    // caller passes no logits buffer), the row splits' sums [splits][B][C]
+    return align_up(bc) + align_up((size_t)B * sizeof(float)) + align_up(bc) + align_up(kMaxRowSplits * bc);
 }
 
 extern "C" int bitlogic_head_loss_ex(const float* Y, int32_t w, int64_t B, int32_t C, float tau,
@@ -200,14 +217,25 @@ extern "C" int bitlogic_head_loss_ex(const float* Y, int32_t w, int64_t B, int32
     float* dlogit = reinterpret_cast<float*>(ws);
     float* per = reinterpret_cast<float*>(ws + align_up(bc));
     float* lg = logits ? logits : reinterpret_cast<float*>(ws + align_up(bc) + align_up((size_t)B * 4));
+    float* split_sums = reinterpret_cast<float*>(ws + align_up(bc) + align_up((size_t)B * 4) + align_up(bc));
+    int splits = 1;
 
-    if (B % 4 == 0 && aligned16(Y))
-        head_group_sum_vec_kernel<<<dim3((unsigned)C, (unsigned)((B + 127) / 128)), kSumVecWarps * 32, 0, stream>>>(
-            Y, B, C, g, tau, lg);
-    else
+    if (B % 4 == 0 && aligned16(Y)) {
+        // split the rows of a class until about two blocks per SM pull from
+        // HBM, keeping at least 16 rows per warp
+        const long long nsb = (B + 127) / 128;
+        const int sms = sm_count();
+        while (splits < kMaxRowSplits && (long long)C * splits * nsb < 2ll * sms &&
+               g / (2 * splits) >= 16 * kSumVecWarps)
+            splits *= 2;
+        const int rows_per_split = (g + splits - 1) / splits;
+        if ((long long)C * splits > 0x7fffffffll || nsb > 65535) return BITLOGIC_ERR_SHAPE;
+        head_group_sum_vec_kernel<<<dim3((unsigned)(C * splits), (unsigned)nsb), kSumVecWarps * 32, 0, stream>>>(
+            Y, B, C, g, tau, lg, split_sums, splits, rows_per_split);
+    } else
         head_group_sum_kernel<<<dim3((unsigned)C, (unsigned)sb), kSumWarps * 32, 0, stream>>>(Y, B, C, g, tau, lg);
     head_softmax_kernel<<<(unsigned)((B + kSoftWarps - 1) / kSoftWarps), kSoftWarps * 32, 0, stream>>>(
-        lg, B, C, labels, dlogit, per, tau, dY_grouped);
+        lg, B, C, labels, dlogit, per, tau, dY_grouped, splits > 1 ? split_sums : nullptr, splits);
     if (dY)
         head_dy_kernel<<<dim3((unsigned)((w + kDyRows - 1) / kDyRows), (unsigned)gy), kDyThreads, 0, stream>>>(
             dlogit, B, C, g, w, tau, dY);

@@ -1011,14 +1011,6 @@ long long forward_chunk(int w_in, int w, long long B) {
     return c < B ? c : B;
 }
 
-int sm_count() {
-    int dev = 0, n = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
-        return 152;
-    return n;
-}
-
 template <int k>
 int launch_forward(const float* X, int w_in, long long B, const int* conn, const float* theta,
                    int w, float* Y, bool vec, cudaStream_t st) {

@@ -250,7 +250,8 @@ def test_empty_batch_is_a_noop():
 # -------------------------------------------------------------------- head --
 
 @pytest.mark.parametrize("C,g,B,tau", [(10, 100, 256, 10.0), (3, 7, 37, 2.0), (100, 13, 259, 100.0),
-                                       (1, 40, 5, 1.0), (10, 800, 1, 20.0)])
+                                       (1, 40, 5, 1.0), (10, 800, 1, 20.0),
+                                       (3, 1025, 256, 5.0), (10, 6400, 256, 50.0)])   # rows split over blocks
 def test_head_loss(C, g, B, tau):
     rng = np.random.default_rng(C + B)
     Y = rng.random((C * g, B)).astype(np.float32)
