@@ -184,12 +184,12 @@ def call_work(wl, B, fuse_dy1=False):
 # file's SHA-256 is recorded, and any later change reports null.
 TRAFFIC = {
     ("mnist", "backward2"): {
-        "bytes": 58.816768e6 + 146.201856e6, "source": "lut_soft.cu",
-        "sha256": "5489bab3e02c6c3da48b76c7b638cf0db63090fb20e5b3bb43ab35490eb3f674",
+        "bytes": 59.695872e6 + 147.913472e6, "source": "lut_soft.cu",
+        "sha256": "ce01d9d3fec57eea20ef26863dbf4290149384de3fe362e07bac6528dab3bf5d",
         "note": "ncu capture of this workload"},
     ("hard_cifar10", "hard1"): {
-        "bytes": 16 * (1.218435e9 + 2.055860e9), "source": "hard.cu",
-        "sha256": "10ccb1e76ad68c073d03604ace6aede6b750faa1a4edd52a47d3c55b57b91c61",
+        "bytes": 16 * (1.216602e9 + 2.055721e9), "source": "hard.cu",
+        "sha256": "2c4964460f09f019f90be5400f2f43dfa68a16578b033e57d48da1afaa926821",
         "note": "ncu capture at 2^18 samples, scaled x16 to 2^22 by the words processed"},
 }
 
