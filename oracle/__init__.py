@@ -57,6 +57,7 @@ def _load():
                 "oracle_pack_bits": ([P, i64, i32, P, i32, P], None),
                 "oracle_hard_forward": ([P, i32, i64, P, P, i32, i32, P], None),
                 "oracle_popcount_head": ([P, i32, i64, i32, P, P], None),
+                "oracle_adamw_step": ([P, P, P, P, i64, i64, dbl, dbl, dbl, dbl, dbl], None),
             }
             for name, (args, res) in sig.items():
                 fn = getattr(lib, name)
@@ -178,6 +179,19 @@ def popcount_head(yp: np.ndarray, N: int, C: int):
     pred = np.empty(N, np.int32)
     _load().oracle_popcount_head(_p(yp), w, N, C, _p(counts), _p(pred))
     return counts, pred
+
+
+def adamw_step(theta: np.ndarray, m: np.ndarray, v: np.ndarray, g: np.ndarray, t: int,
+               lr: float = 0.01, beta1: float = 0.9, beta2: float = 0.999, eps: float = 1e-8,
+               wd: float = 0.0):
+    """One AdamW step (§4 "Training"); returns new (theta, m, v) in float64."""
+    th = _c(theta, np.float64).copy()
+    mm = _c(m, np.float64).copy()
+    vv = _c(v, np.float64).copy()
+    gg = _c(g, np.float64)
+    _load().oracle_adamw_step(_p(th), _p(mm), _p(vv), _p(gg), th.size, int(t), float(lr),
+                              float(beta1), float(beta2), float(eps), float(wd))
+    return th, mm, vv
 
 
 # ---- composites used by the parity tests and the CPU baseline ------------

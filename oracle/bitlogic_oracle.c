@@ -259,3 +259,25 @@ void oracle_popcount_head(const uint32_t* yp, int32_t w, int64_t N, int32_t C,
         if (pred) pred[s] = bestc;
     }
 }
+
+/* One AdamW step (§4 "Training": AdamW with beta1 0.9, beta2 0.999,
+ * eps 1e-8, constant learning rate 0.01, weight decay 0), with decoupled
+ * weight decay, for step number t >= 1 and every parameter i:
+ *   m_i     = beta1 m_i + (1 - beta1) g_i
+ *   v_i     = beta2 v_i + (1 - beta2) g_i^2
+ *   theta_i = theta_i - lr ( (m_i / (1 - beta1^t)) / (sqrt(v_i / (1 - beta2^t)) + eps)
+ *                             + wd theta_i )                                       */
+void oracle_adamw_step(double* theta, double* m, double* v, const double* g, int64_t n,
+                       int64_t t, double lr, double beta1, double beta2, double eps,
+                       double wd) {
+    const double bc1 = 1.0 - pow(beta1, (double)t);
+    const double bc2 = 1.0 - pow(beta2, (double)t);
+#pragma omp parallel for schedule(static)
+    for (int64_t i = 0; i < n; ++i) {
+        m[i] = beta1 * m[i] + (1.0 - beta1) * g[i];
+        v[i] = beta2 * v[i] + (1.0 - beta2) * g[i] * g[i];
+        const double mhat = m[i] / bc1;
+        const double vhat = v[i] / bc2;
+        theta[i] = theta[i] - lr * (mhat / (sqrt(vhat) + eps) + wd * theta[i]);
+    }
+}

@@ -388,3 +388,43 @@ def test_blob_batch_shapes():
     assert lab.dtype == torch.int32 and int(lab.min()) >= 0 and int(lab.max()) < 4
     x2, lab2 = synth.blob_batch(300, 17, 4, 40.0, seed=1)
     assert torch.equal(x, x2) and torch.equal(lab, lab2)
+
+
+# ------------------------------------------------------------------ AdamW --
+
+def test_adamw_matches_torch_optimizer():
+    # the oracle's AdamW (§4 "Training") equals torch.optim.AdamW in float64
+    # over several steps, with and without decoupled weight decay
+    import torch
+    rng = np.random.default_rng(11)
+    for wd in (0.0, 0.05):
+        theta0 = rng.standard_normal(300)
+        p = torch.nn.Parameter(torch.tensor(theta0, dtype=torch.float64))
+        opt = torch.optim.AdamW([p], lr=0.01, betas=(0.9, 0.999), eps=1e-8, weight_decay=wd)
+        th, m, v = theta0.copy(), np.zeros(300), np.zeros(300)
+        for t in range(1, 6):
+            g = rng.standard_normal(300) * 10.0 ** rng.integers(-6, 1, size=300)
+            p.grad = torch.tensor(g, dtype=torch.float64)
+            opt.step()
+            th, m, v = oracle.adamw_step(th, m, v, g, t, lr=0.01, wd=wd)
+            st = opt.state[p]
+            np.testing.assert_allclose(th, p.detach().numpy(), rtol=1e-12, atol=1e-15)
+            np.testing.assert_allclose(m, st["exp_avg"].numpy(), rtol=1e-12, atol=0)
+            np.testing.assert_allclose(v, st["exp_avg_sq"].numpy(), rtol=1e-12, atol=0)
+
+
+def test_adamw_first_step_closed_form():
+    # step 1 from zero moments: m = (1-b1) g, v = (1-b2) g^2, the bias
+    # corrections cancel them, so theta moves by lr * g / (|g| + eps)
+    rng = np.random.default_rng(12)
+    theta0 = rng.standard_normal(50)
+    g = rng.standard_normal(50) * 1e-3
+    g[0] = 0.0
+    th, m, v = oracle.adamw_step(theta0, np.zeros(50), np.zeros(50), g, 1, lr=0.01)
+    np.testing.assert_allclose(m, 0.1 * g, rtol=1e-14, atol=0)      # (1 - 0.9) rounds in binary
+    np.testing.assert_allclose(v, 0.001 * g * g, rtol=1e-14, atol=0)
+    np.testing.assert_allclose(th, theta0 - 0.01 * g / (np.abs(g) + 1e-8), rtol=1e-12, atol=1e-15)
+    assert th[0] == theta0[0]
+    # zero gradient: only the decoupled decay moves theta
+    th2, _, _ = oracle.adamw_step(theta0, np.zeros(50), np.zeros(50), np.zeros(50), 3, lr=0.01, wd=0.1)
+    np.testing.assert_allclose(th2, theta0 * (1 - 0.01 * 0.1), rtol=1e-15, atol=0)
