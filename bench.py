@@ -386,6 +386,16 @@ def run_ours(args):
             "clocks": clocks,
             "wall_s_timed_loop": wall,
         }
+    if st is not None and not args.profile:
+        # the AdamW update of both layers' logits (not part of `value`, which
+        # is the fwd+bwd step): timed on its own from the last gradients
+        upd = time_update(st, max(3, min(args.steps, 50)))
+        if result is not None:
+            n_par = int(st.net.theta1.numel() + st.net.theta2.numel())
+            result["optimizer"] = {"ms_per_update": upd, "kernel": "adamw_vec_kernel (x2)",
+                                   "algorithmic_bytes": 28 * n_par,
+                                   "GB/s": 28 * n_par / (upd * 1e-3) / 1e9,
+                                   "settings": "AdamW beta (0.9, 0.999), eps 1e-8, lr 0.01, wd 0"}
     if not args.profile and not args.no_e2e:
         e2e = run_e2e(args, st, hi, wl, B)
         if result is not None:
@@ -395,6 +405,20 @@ def run_ours(args):
         torch.distributed.barrier()
         torch.distributed.destroy_process_group()
     return result
+
+
+def time_update(st, iters: int) -> float:
+    """Mean ms of one AdamW update of both layers (CUDA events on the launching stream)."""
+    for _ in range(3):
+        st.update()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(iters):
+        st.update()
+    e1.record()
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / iters
 
 
 def run_e2e(args, st, hi, wl, B):

@@ -51,7 +51,8 @@ typedef enum {
     BITLOGIC_ERR_INDEX = -7,      /* index out of range (host-side check) */
     BITLOGIC_ERR_DEVICE = -8,     /* device-side index check tripped */
     BITLOGIC_ERR_THRESH = -9,     /* thresholds: b outside 1..32 */
-    BITLOGIC_ERR_TOO_LARGE = -10  /* sizes beyond bitlogic_head_loss_noalloc's fixed scratch */
+    BITLOGIC_ERR_TOO_LARGE = -10, /* sizes beyond bitlogic_head_loss_noalloc's fixed scratch */
+    BITLOGIC_ERR_HYPER = -11      /* optimizer hyperparameter out of range */
 } bitlogic_status_t;
 
 /* Thermometer encoder E: R^d -> {0,1}^{db} (paper §3, "Encoders and heads";
@@ -196,6 +197,21 @@ int bitlogic_head_loss_ex(const float* Y, int32_t w, int64_t B, int32_t C, float
 int bitlogic_head_loss_noalloc(const float* Y, int32_t w, int64_t B, int32_t C, float tau,
                                const int32_t* labels, float* logits, float* loss, float* dY,
                                cudaStream_t stream);
+
+/* One AdamW step on the table logits (§4 "Training": AdamW with beta1 0.9,
+ * beta2 0.999, eps 1e-8, constant learning rate 0.01, weight decay 0),
+ * weight decay decoupled, step number `step` >= 1, for every parameter i:
+ *   m_i     = beta1 m_i + (1 - beta1) g_i
+ *   v_i     = beta2 v_i + (1 - beta2) g_i^2
+ *   theta_i = theta_i - lr ( (m_i / (1 - beta1^step))
+ *                            / (sqrt(v_i / (1 - beta2^step)) + eps) + wd theta_i )
+ *   theta, m, v  device fp32 [n], updated in place (m, v start at zero)
+ *   grad         device fp32 [n] (e.g. the dtheta of bitlogic_lut_backward)
+ * Returns BITLOGIC_ERR_HYPER unless 0 <= beta1, beta2 < 1, eps > 0, lr >= 0
+ * and wd >= 0. */
+int bitlogic_adamw_update(float* theta, float* m, float* v, const float* grad, int64_t n,
+                          int64_t step, float lr, float beta1, float beta2, float eps,
+                          float weight_decay, cudaStream_t stream);
 
 /* Table discretization (§3: every surrogate discretizes to a 2^n-entry
  * truth table; App. C.1 extracts it once per layer): bit a of table[j] is 1

@@ -30,6 +30,7 @@ __all__ = [
     "bitlogic_head_loss_workspace", "bitlogic_head_loss_noalloc",
     "bitlogic_head_loss", "bitlogic_binarize_tables", "bitlogic_pack_bits",
     "bitlogic_hard_forward", "bitlogic_build_csr", "bitlogic_csr_positions", "bitlogic_device_error",
+    "bitlogic_adamw_update",
     "bitlogic_status_string", "bitlogic_version", "LIB_PATH",
 ]
 
@@ -68,6 +69,7 @@ _SIGS = {
                               ctypes.c_int),
     "bitlogic_build_csr": ([_P, _I32, _I32, _I32, _P, _P], ctypes.c_int),
     "bitlogic_csr_positions": ([_P, _I32, _P], ctypes.c_int),
+    "bitlogic_adamw_update": ([_P, _P, _P, _P, _I64, _I64, _F32, _F32, _F32, _F32, _F32, _P], ctypes.c_int),
     "bitlogic_device_error": ([_P], ctypes.c_int),
     "bitlogic_status_string": ([ctypes.c_int], ctypes.c_char_p),
     "bitlogic_version": ([], ctypes.c_int),
@@ -367,6 +369,18 @@ def bitlogic_build_csr(conn: np.ndarray, w_in: int) -> Tuple[np.ndarray, np.ndar
     _check("bitlogic_build_csr", load().bitlogic_build_csr(
         conn.ctypes.data_as(_P), w, k, w_in, off.ctypes.data_as(_P), edge.ctypes.data_as(_P)))
     return off, edge
+
+
+def bitlogic_adamw_update(theta: torch.Tensor, m: torch.Tensor, v: torch.Tensor, grad: torch.Tensor,
+                          step: int, lr: float = 0.01, betas=(0.9, 0.999), eps: float = 1e-8,
+                          weight_decay: float = 0.0, stream=None):
+    """One AdamW step in place on theta, m, v (same shape, fp32, device)."""
+    shape = tuple(theta.shape)
+    for t, name in ((theta, "theta"), (m, "m"), (v, "v"), (grad, "grad")):
+        _need(t, name, torch.float32, shape)
+    _check("bitlogic_adamw_update", load().bitlogic_adamw_update(
+        _ptr(theta), _ptr(m), _ptr(v), _ptr(grad), theta.numel(), int(step), float(lr),
+        float(betas[0]), float(betas[1]), float(eps), float(weight_decay), _stream(stream)))
 
 
 def bitlogic_csr_positions(csr_edge: np.ndarray) -> np.ndarray:

@@ -28,6 +28,7 @@ extern "C" int bitlogic_internal_index_error_lut_soft(cudaStream_t);
 extern "C" int bitlogic_internal_index_error_head(cudaStream_t);
 extern "C" int bitlogic_internal_index_error_encode(cudaStream_t);
 extern "C" int bitlogic_internal_index_error_hard(cudaStream_t);
+extern "C" int bitlogic_internal_index_error_optim(cudaStream_t);
 
 extern "C" const char* bitlogic_status_string(int code) {
     switch (code) {
@@ -42,6 +43,7 @@ extern "C" const char* bitlogic_status_string(int code) {
         case BITLOGIC_ERR_DEVICE: return "a kernel met an out-of-range index (read as 0)";
         case BITLOGIC_ERR_THRESH: return "number of thresholds must be 1..32";
         case BITLOGIC_ERR_TOO_LARGE: return "sizes exceed the fixed scratch of the allocation-free entry point";
+        case BITLOGIC_ERR_HYPER: return "optimizer hyperparameter out of range";
         default: return "unknown status";
     }
 }
@@ -81,10 +83,11 @@ extern "C" int bitlogic_csr_positions(const int32_t* edge_host, int32_t n_edges,
 
 extern "C" int bitlogic_device_error(cudaStream_t stream) {
     int worst = BITLOGIC_OK;
-    const int r[4] = {bitlogic_internal_index_error_lut_soft(stream),
+    const int r[5] = {bitlogic_internal_index_error_lut_soft(stream),
                       bitlogic_internal_index_error_head(stream),
                       bitlogic_internal_index_error_encode(stream),
-                      bitlogic_internal_index_error_hard(stream)};
+                      bitlogic_internal_index_error_hard(stream),
+                      bitlogic_internal_index_error_optim(stream)};
     for (int v : r) {
         if (v == BITLOGIC_ERR_CUDA) return v;
         if (v != BITLOGIC_OK) worst = v;

@@ -16,7 +16,8 @@ from typing import Optional, Sequence
 import numpy as np
 import torch
 
-from . import (bitlogic_binarize_tables, bitlogic_build_csr, bitlogic_csr_positions, bitlogic_csr_reduce,
+from . import (bitlogic_adamw_update, bitlogic_binarize_tables, bitlogic_build_csr, bitlogic_csr_positions,
+               bitlogic_csr_reduce,
                bitlogic_encode_thermometer, bitlogic_hard_forward, bitlogic_head_loss_ex,
                bitlogic_head_loss_workspace, bitlogic_lut_backward_ex, bitlogic_lut_forward,
                bitlogic_pack_bits)
@@ -134,6 +135,23 @@ class TrainStep:
     def run(self, stream=None, mark=_nomark):
         self.forward(stream, mark)
         self.backward(stream, mark)
+
+    def update(self, lr: float = 0.01, betas=(0.9, 0.999), eps: float = 1e-8,
+               weight_decay: float = 0.0, stream=None, mark=_nomark):
+        """AdamW step on both layers' table logits from the last backward
+        (§4 "Training": the paper's settings are the defaults); the moment
+        buffers start at zero on the first call."""
+        n = self.net
+        if not hasattr(self, "opt_m1"):
+            self.opt_m1, self.opt_v1 = torch.zeros_like(n.theta1), torch.zeros_like(n.theta1)
+            self.opt_m2, self.opt_v2 = torch.zeros_like(n.theta2), torch.zeros_like(n.theta2)
+            self.opt_step = 0
+        self.opt_step += 1
+        bitlogic_adamw_update(n.theta1, self.opt_m1, self.opt_v1, self.dth1, self.opt_step, lr, betas, eps,
+                              weight_decay, stream)
+        bitlogic_adamw_update(n.theta2, self.opt_m2, self.opt_v2, self.dth2, self.opt_step, lr, betas, eps,
+                              weight_decay, stream)
+        mark("update")
 
     # kernels one run() launches: encode 1, forwards 2, head 3, backwards 2
     # (+ the CSR reduction of layer 2's terms unless fused, + the layer-1 CSR

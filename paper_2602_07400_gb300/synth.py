@@ -84,13 +84,15 @@ def class_means(C: int, d: int, seed: int) -> torch.Tensor:
 
 def blob_batch(n: int, d: int, C: int, sigma: float, seed: int,
                device: str | torch.device = "cpu",
-               chunk: int = 1 << 16) -> Tuple[torch.Tensor, torch.Tensor]:
+               chunk: int = 1 << 16, means_seed: int | None = None) -> Tuple[torch.Tensor, torch.Tensor]:
     """Return ``(x, labels)``: ``x`` uint8 [n, d] (sample-major, as a raw
-    image batch is stored) and ``labels`` int32 [n].  Data drawn on a CUDA
+    image batch is stored) and ``labels`` int32 [n].  The class means come
+    from ``means_seed`` (default: ``seed``); keep it fixed across batches to
+    draw several batches of one synthetic dataset.  Data drawn on a CUDA
     device differ from data drawn on the CPU for the same seed; every
     comparison uses one draw, copied where needed."""
     device = torch.device(device)
-    mu = class_means(C, d, seed).to(device)
+    mu = class_means(C, d, seed if means_seed is None else means_seed).to(device)
     g = torch.Generator(device="cpu").manual_seed(seed + 1)
     labels = torch.randint(0, C, (n,), generator=g, dtype=torch.int64)
     labels_dev = labels.to(device)

@@ -47,7 +47,7 @@ def test_python_binding_names_match_header():
 
 def test_status_strings_and_version():
     assert bl.bitlogic_status_string(0) == "ok"
-    for c in range(-1, -10, -1):
+    for c in range(-1, -12, -1):
         assert bl.bitlogic_status_string(c) != "unknown status"
     assert bl.bitlogic_version() >= 100
 
@@ -126,6 +126,15 @@ def test_host_validation_returns_before_any_launch():
     assert lib.bitlogic_hard_forward(fake, 8, 64, fake, fake, 4, 2, None, 2, None, None, None) == -1
     assert lib.bitlogic_hard_forward(fake, 8, 64, fake, fake, 4, 2, None, 3, fake, None, None) == -2
     assert lib.bitlogic_binarize_tables(fake, 4, 7, fake, None) == -3
+    # AdamW: step >= 1, betas in [0, 1), eps > 0, n >= 0; n == 0 is a no-op
+    F = ctypes.c_float
+    adamw = lib.bitlogic_adamw_update
+    assert adamw(fake, fake, fake, fake, 8, 0, F(0.01), F(0.9), F(0.999), F(1e-8), F(0.0), None) == -11
+    assert adamw(fake, fake, fake, fake, 8, 1, F(0.01), F(1.0), F(0.999), F(1e-8), F(0.0), None) == -11
+    assert adamw(fake, fake, fake, fake, 8, 1, F(0.01), F(0.9), F(0.999), F(0.0), F(0.0), None) == -11
+    assert adamw(fake, fake, fake, fake, -1, 1, F(0.01), F(0.9), F(0.999), F(1e-8), F(0.0), None) == -2
+    assert adamw(None, None, None, None, 0, 1, F(0.01), F(0.9), F(0.999), F(1e-8), F(0.0), None) == 0
+    assert adamw(None, fake, fake, fake, 8, 1, F(0.01), F(0.9), F(0.999), F(1e-8), F(0.0), None) == -1
 
 
 def test_workspace_queries():

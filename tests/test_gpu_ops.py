@@ -429,3 +429,37 @@ def test_binding_rejects_wrong_tensors():
         bl.bitlogic_lut_forward(X, conn, theta, torch.empty(4, 9, device="cuda"))
     with pytest.raises(ValueError):
         bl.bitlogic_lut_forward(X.cpu(), conn, theta, torch.empty(4, 8, device="cuda"))
+
+
+# ------------------------------------------------------------------ AdamW --
+
+@pytest.mark.parametrize("n,wd", [(4096, 0.0), (1000003, 0.0), (64000 * 64, 0.1), (7, 0.05)])
+def test_adamw_update(n, wd):
+    # two steps in a row (steps 1 and 2, the state carried on the device),
+    # each against the oracle from the same inputs; the error scale of each
+    # moment update is the size of its two terms
+    rng = np.random.default_rng(n)
+    theta = rng.standard_normal(n).astype(np.float32)
+    m = np.zeros(n, np.float32)
+    v = np.zeros(n, np.float32)
+    th_d, m_d, v_d = dev(theta), dev(m), dev(v)
+    for step in (1, 2):
+        g = (rng.standard_normal(n) * 10.0 ** rng.integers(-7, -1, size=n)).astype(np.float32)
+        g[::97] = 0.0
+        bl.bitlogic_adamw_update(th_d, m_d, v_d, dev(g), step, lr=0.01, weight_decay=wd)
+        # the oracle gets the hyperparameters as the kernel receives them (fp32)
+        f = lambda a: float(np.float32(a))
+        th_o, m_o, v_o = oracle.adamw_step(theta, m, v, g, step, lr=f(0.01), beta1=f(0.9), beta2=f(0.999),
+                                           eps=f(1e-8), wd=f(wd))
+        got_th, got_m, got_v = (t.cpu().numpy().astype(np.float64) for t in (th_d, m_d, v_d))
+        scale_m = 0.9 * np.abs(m) + 0.1 * np.abs(g.astype(np.float64))
+        scale_v = 0.999 * np.abs(v) + 0.001 * g.astype(np.float64) ** 2
+        # theta: the step is at most a few learning rates, so its terms are
+        # |theta| and 4 lr (a result near 0 comes from cancellation)
+        scale_th = np.abs(theta.astype(np.float64)) + 4 * 0.01
+        assert np.all(np.abs(got_m - m_o) <= 1e-6 * scale_m + 1e-30), "m"
+        assert np.all(np.abs(got_v - v_o) <= 1e-6 * scale_v + 1e-30), "v"
+        err = np.abs(got_th - th_o)
+        assert np.all(err <= 1e-6 * scale_th), f"theta: {err.max()}"
+        theta, m, v = got_th.astype(np.float32), got_m.astype(np.float32), got_v.astype(np.float32)
+    no_device_error()

@@ -198,3 +198,44 @@ def test_hard_ragged_batch():
     _hard_run(small, 100003, samples=700)
     _hard_run(small, 1024, samples=300)
     _hard_run(small, 37, samples=37)
+
+
+def test_tiny_training_steps_match_oracle_and_lower_the_loss():
+    # forward + backward + AdamW (§4 settings), repeated: the first two
+    # updates of both layers' logits match the oracle's trajectory, and over
+    # 30 steps on fresh batches of one dataset the loss falls
+    wl = synth.WORKLOADS["tiny"]
+    conn1, th1, conn2, th2 = synth.network(wl, 0)
+    net = Network(conn1, th1, conn2, th2, wl.w_in)
+    st = TrainStep(net, wl.batch, wl.d, wl.thresholds, wl.classes, wl.tau)
+    o_th1, o_th2 = th1.astype(np.float64), th2.astype(np.float64)
+    o_m = [np.zeros_like(o_th1), np.zeros_like(o_th2)]
+    o_v = [np.zeros_like(o_th1), np.zeros_like(o_th2)]
+    losses, accs = [], []
+    for step in range(1, 31):
+        x, labels = synth.blob_batch(wl.batch, wl.d, wl.classes, wl.sigma, seed=100 + step, means_seed=7)
+        st.load(x.cuda(), labels.cuda())
+        st.run()
+        st.update()
+        losses.append(float(st.loss.item()))
+        accs.append(float((st.logits.argmax(1).cpu() == labels.long()).float().mean()))
+        if step <= 2:
+            # the oracle's step from the GPU's current logits, so each update
+            # is checked on its own
+            r = oracle.train_step(x.numpy(), labels.numpy(), wl.thresholds, conn1, o_th1.astype(np.float32),
+                                  conn2, o_th2.astype(np.float32), wl.classes, wl.tau)
+            o_th1, o_m[0], o_v[0] = oracle.adamw_step(o_th1, o_m[0], o_v[0], r["dth1"], step)
+            o_th2, o_m[1], o_v[1] = oracle.adamw_step(o_th2, o_m[1], o_v[1], r["dth2"], step)
+            # the step follows gradients held to 1e-4 relative: bound the
+            # logits by 1e-5 relative plus 1e-3 of the learning rate
+            for got, want, name in ((net.theta1, o_th1, "theta1"), (net.theta2, o_th2, "theta2")):
+                err = np.abs(got.cpu().numpy().astype(np.float64) - want)
+                assert np.all(err <= 1e-5 * np.abs(want) + 1e-3 * 0.01), f"{name} after step {step}: {err.max()}"
+            o_th1 = net.theta1.cpu().numpy().astype(np.float64)
+            o_th2 = net.theta2.cpu().numpy().astype(np.float64)
+            o_m = [st.opt_m1.cpu().numpy().astype(np.float64), st.opt_m2.cpu().numpy().astype(np.float64)]
+            o_v = [st.opt_v1.cpu().numpy().astype(np.float64), st.opt_v2.cpu().numpy().astype(np.float64)]
+    # batches of one synthetic dataset (fixed class means): the loss falls and
+    # the training accuracy climbs from chance
+    assert np.mean(losses[-5:]) < 0.95 * np.mean(losses[:3]), losses
+    assert accs[-1] >= 0.9, accs
