@@ -50,9 +50,9 @@ def _load():
                 "oracle_set_threads": ([ctypes.c_int], None),
                 "oracle_linear_thresholds": ([i32, P], None),
                 "oracle_encode_thermometer": ([P, i64, i32, P, i32, P], None),
-                "oracle_lut_forward": ([P, i32, i64, P, P, i32, i32, P], None),
+                "oracle_lut_forward": ([P, i32, i64, P, P, i32, i32, i32, P], None),
                 "oracle_head_loss": ([P, i32, i64, i32, dbl, P, P, P, P], None),
-                "oracle_lut_backward": ([P, i32, i64, P, P, i32, i32, P, P, P], None),
+                "oracle_lut_backward": ([P, i32, i64, P, P, i32, i32, i32, P, P, P], None),
                 "oracle_binarize_tables": ([P, i32, i32, P], None),
                 "oracle_pack_bits": ([P, i64, i32, P, i32, P], None),
                 "oracle_hard_forward": ([P, i32, i64, P, P, i32, i32, P], None),
@@ -99,8 +99,19 @@ def encode_thermometer(x: np.ndarray, thr) -> np.ndarray:
     return bits
 
 
-def lut_forward(X: np.ndarray, conn: np.ndarray, theta: np.ndarray) -> np.ndarray:
-    """X float64 [w_in, B], conn int32 [w, k], theta float32 [w, 2^k] -> Y float64 [w, B]."""
+NODES = {"soft": 0, "st": 1}
+
+
+def _node(node: str) -> int:
+    if node not in NODES:
+        raise ValueError(f"node must be one of {sorted(NODES)}")
+    return NODES[node]
+
+
+def lut_forward(X: np.ndarray, conn: np.ndarray, theta: np.ndarray, node: str = "soft") -> np.ndarray:
+    """X float64 [w_in, B], conn int32 [w, k], theta float32 [w, 2^k] -> Y float64 [w, B].
+    node "soft": tables sigmoid(theta); "st": hard samples [theta > 0]
+    (LightLUT straight-through)."""
     X = _c(X, np.float64)
     conn = _c(conn, np.int32)
     theta = _c(theta, np.float32)
@@ -108,7 +119,7 @@ def lut_forward(X: np.ndarray, conn: np.ndarray, theta: np.ndarray) -> np.ndarra
     w, k = conn.shape
     assert theta.shape == (w, 1 << k)
     Y = np.empty((w, B), np.float64)
-    _load().oracle_lut_forward(_p(X), w_in, B, _p(conn), _p(theta), w, k, _p(Y))
+    _load().oracle_lut_forward(_p(X), w_in, B, _p(conn), _p(theta), w, k, _node(node), _p(Y))
     return Y
 
 
@@ -125,8 +136,9 @@ def head_loss(Y: np.ndarray, labels: np.ndarray, C: int, tau: float):
 
 
 def lut_backward(X: np.ndarray, conn: np.ndarray, theta: np.ndarray, dY: np.ndarray,
-                 want_dx: bool = True):
-    """-> (dtheta float64 [w, 2^k], dX float64 [w_in, B] or None)."""
+                 want_dx: bool = True, node: str = "soft"):
+    """-> (dtheta float64 [w, 2^k], dX float64 [w_in, B] or None).  node as
+    in ``lut_forward``; for "st" dtheta is the straight-through estimate."""
     X = _c(X, np.float64)
     conn = _c(conn, np.int32)
     theta = _c(theta, np.float32)
@@ -135,7 +147,7 @@ def lut_backward(X: np.ndarray, conn: np.ndarray, theta: np.ndarray, dY: np.ndar
     w, k = conn.shape
     dtheta = np.empty((w, 1 << k), np.float64)
     dX = np.empty((w_in, B), np.float64) if want_dx else None
-    _load().oracle_lut_backward(_p(X), w_in, B, _p(conn), _p(theta), w, k, _p(dY),
+    _load().oracle_lut_backward(_p(X), w_in, B, _p(conn), _p(theta), w, k, _node(node), _p(dY),
                                 _p(dtheta), _p(dX))
     return dtheta, dX
 
@@ -197,14 +209,15 @@ def adamw_step(theta: np.ndarray, m: np.ndarray, v: np.ndarray, g: np.ndarray, t
 # ---- composites used by the parity tests and the CPU baseline ------------
 
 def train_step(x: np.ndarray, labels: np.ndarray, thr, conn1, th1, conn2, th2,
-               C: int, tau: float, want_dx1: bool = False):
-    """Encoder -> two LUT layers -> group-sum head + CE -> both backwards."""
+               C: int, tau: float, want_dx1: bool = False, node: str = "soft"):
+    """Encoder -> two LUT layers -> group-sum head + CE -> both backwards
+    (both layers of the node form ``node``)."""
     bits = encode_thermometer(x, thr)
-    y1 = lut_forward(bits, conn1, th1)
-    y2 = lut_forward(y1, conn2, th2)
+    y1 = lut_forward(bits, conn1, th1, node)
+    y2 = lut_forward(y1, conn2, th2, node)
     logits, loss, dy2 = head_loss(y2, labels, C, tau)
-    dth2, dy1 = lut_backward(y1, conn2, th2, dy2, want_dx=True)
-    dth1, dbits = lut_backward(bits, conn1, th1, dy1, want_dx=want_dx1)
+    dth2, dy1 = lut_backward(y1, conn2, th2, dy2, want_dx=True, node=node)
+    dth1, dbits = lut_backward(bits, conn1, th1, dy1, want_dx=want_dx1, node=node)
     return dict(bits=bits, y1=y1, y2=y2, logits=logits, loss=loss, dy2=dy2,
                 dth2=dth2, dy1=dy1, dth1=dth1, dbits=dbits)
 

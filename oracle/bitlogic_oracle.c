@@ -80,17 +80,29 @@ static double corner_weight(const double* xs, int32_t k, int64_t a) {
     return wa;
 }
 
-/* Soft LUT layer forward (one logic layer L_M(f_theta^(n)) of Eq. (1), §3):
- * y_j(s) = sum_a sigmoid(theta_j[a]) * w_a(x_{M_j(0)}(s), ..., x_{M_j(k-1)}(s)). */
+/* Value of table entry theta for the two LightLUT node forms of the node
+ * sweep (§2 "Gradient-based LUT methods", §4 "Node parameterization"):
+ * node 0 (soft) uses t = sigmoid(theta); node 1 (straight-through hard) uses
+ * the hard sample t = [theta > 0] -- the value the entry discretizes to --
+ * while the gradient still reaches theta through the sigmoid (see the
+ * backward).  theta = 0 samples 0, as in the table discretization below. */
+static double table_value(float theta, int32_t node) {
+    if (node == 1) return theta > 0.0f ? 1.0 : 0.0;
+    return sigmoid((double)theta);
+}
+
+/* LUT layer forward (one logic layer L_M(f_theta^(n)) of Eq. (1), §3):
+ * y_j(s) = sum_a t(theta_j[a]) * w_a(x_{M_j(0)}(s), ..., x_{M_j(k-1)}(s)),
+ * t the node form's table value (table_value). */
 void oracle_lut_forward(const double* X, int32_t w_in, int64_t B,
                         const int32_t* conn, const float* theta, int32_t w, int32_t k,
-                        double* Y) {
+                        int32_t node, double* Y) {
     const int64_t K = (int64_t)1 << k;
     (void)w_in;
 #pragma omp parallel for schedule(dynamic, 16)
     for (int32_t j = 0; j < w; ++j) {
         double xs[8], t[64];
-        for (int64_t a = 0; a < K; ++a) t[a] = sigmoid((double)theta[(int64_t)j * K + a]);
+        for (int64_t a = 0; a < K; ++a) t[a] = table_value(theta[(int64_t)j * K + a], node);
         for (int64_t s = 0; s < B; ++s) {
             for (int32_t i = 0; i < k; ++i) xs[i] = X[(int64_t)conn[(int64_t)j * k + i] * B + s];
             double y = 0.0;
@@ -140,15 +152,20 @@ void oracle_head_loss(const double* Y, int32_t w, int64_t B, int32_t C, double t
     free(per);
 }
 
-/* Soft LUT layer backward, by the chain rule on the forward definition:
- *   dtheta_j[a] = t_a (1 - t_a) * sum_s dY[j][s] * w_a(x(s))
+/* LUT layer backward, by the chain rule on the forward definition, with
+ * sg_a = sigmoid(theta_j[a]) and t_a the node form's table value:
+ *   dtheta_j[a] = sg_a (1 - sg_a) * sum_s dY[j][s] * w_a(x(s))
  *   dy_j/dx_i   = sum_a t_a * (a_i ? +1 : -1) * prod_{m != i} (a_m ? x_m : 1 - x_m)
  *   dX[M_j(i)][s] += dY[j][s] * dy_j/dx_i        (scatter-add in node order)
+ * For the soft node t_a = sg_a and this is the exact gradient.  For the
+ * straight-through node the forward used t_a = [theta > 0]; the estimator
+ * passes dL/dt_a = sum_s dY w_a to theta as if t_a were sigmoid(theta), and
+ * the input gradient is the exact one of the hard-table forward.
  * dX (optional) is overwritten.  For each element of dX the additions happen
  * in increasing (j, i) order. */
 void oracle_lut_backward(const double* X, int32_t w_in, int64_t B,
                          const int32_t* conn, const float* theta, int32_t w, int32_t k,
-                         const double* dY, double* dtheta, double* dX) {
+                         int32_t node, const double* dY, double* dtheta, double* dX) {
     const int64_t K = (int64_t)1 << k;
 #pragma omp parallel for schedule(dynamic, 16)
     for (int32_t j = 0; j < w; ++j) {
@@ -166,7 +183,7 @@ void oracle_lut_backward(const double* X, int32_t w_in, int64_t B,
     if (!dX) return;
     memset(dX, 0, sizeof(double) * (size_t)w_in * (size_t)B);
     double* tt = (double*)malloc(sizeof(double) * (size_t)w * (size_t)K);
-    for (int64_t q = 0; q < (int64_t)w * K; ++q) tt[q] = sigmoid((double)theta[q]);
+    for (int64_t q = 0; q < (int64_t)w * K; ++q) tt[q] = table_value(theta[q], node);
     /* samples are independent: one thread owns each sample column and walks
      * the nodes in order, so the per-element addition order is (j, i) */
 #pragma omp parallel for schedule(static)

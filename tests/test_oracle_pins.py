@@ -151,7 +151,7 @@ def test_partition_of_unity():
 
 # ---------------------------------------------------------------- backward --
 
-@pytest.mark.parametrize("k", [1, 2, 3, 6])
+@pytest.mark.parametrize("k", [1, 2, 3, 4, 6])
 def test_finite_differences(k):
     rng = np.random.default_rng(100 + k)
     w_in, w, B = max(k + 2, 8), 5, 4
@@ -210,6 +210,105 @@ def test_dx_scatter_is_sum_over_consumers():
     _, dB = oracle.lut_backward(X, conn[1:], theta[1:], dY[1:])
     np.testing.assert_allclose(dX, dA + dB, rtol=1e-13, atol=1e-15)
     assert np.all(dX[3:] == 0.0)
+
+
+# ------------------------------------------ straight-through hard node --
+#
+# LightLUT's hard form (§2 "Gradient-based LUT methods", §4 "Node
+# parameterization"): the forward samples each table entry as [theta > 0];
+# the straight-through estimator sends the table gradient to theta through
+# the sigmoid.
+
+def _shannon_forward_torch(X, conn, t):
+    """y_j = the node's table folded one input at a time (slot i = bit i of
+    the entry index): a different formulation from the oracle's sum of
+    corner weights."""
+    w, k = conn.shape
+    xs = X[torch.as_tensor(conn, dtype=torch.long)]      # [w, k, B]
+    B = X.shape[1]
+    T = t.reshape((w,) + (2,) * k).unsqueeze(1).expand((w, B) + (2,) * k)
+    for i in range(k):   # the last axis is the lowest remaining index bit
+        xi = xs[:, i, :].reshape((w, B) + (1,) * (k - 1 - i))
+        T = T[..., 0] * (1 - xi) + T[..., 1] * xi
+    return T
+
+
+@pytest.mark.parametrize("k", [1, 2, 4, 6])
+def test_st_backward_matches_torch_straight_through(k):
+    # torch autograd through t = sigmoid(theta) + ([theta > 0] - sigmoid(theta)).detach()
+    rng = np.random.default_rng(500 + k)
+    w_in, w, B = max(k + 3, 9), 7, 5
+    X = rng.random((w_in, B))
+    conn = synth.connectivity(w, k, w_in, seed=k + 50)
+    theta = synth.table_logits(w, 1 << k, seed=k + 51)
+    theta[0, 0] = 0.0                        # a tie samples 0
+    dY = rng.standard_normal((w, B))
+    Xt = torch.tensor(X, dtype=torch.float64, requires_grad=True)
+    tht = torch.tensor(theta.astype(np.float64), requires_grad=True)
+    sg = torch.sigmoid(tht)
+    t = sg + ((tht > 0).to(torch.float64) - sg).detach()
+    Y = _shannon_forward_torch(Xt, conn, t)
+    (Y * torch.tensor(dY)).sum().backward()
+    np.testing.assert_allclose(oracle.lut_forward(X, conn, theta, "st"), Y.detach().numpy(),
+                               rtol=1e-13, atol=1e-15)
+    dth, dX = oracle.lut_backward(X, conn, theta, dY, node="st")
+    np.testing.assert_allclose(dth, tht.grad.numpy(), rtol=1e-12, atol=1e-15)
+    np.testing.assert_allclose(dX, Xt.grad.numpy(), rtol=1e-12, atol=1e-14)
+
+
+@pytest.mark.parametrize("k", [2, 4, 6])
+def test_st_forward_is_the_saturated_soft_forward(k):
+    # tables at theta = +-800 have sigmoid exactly 1 / 0 in double, so the
+    # soft forward on them is the hard-sampled forward, on any inputs
+    rng = np.random.default_rng(600 + k)
+    w_in, w, B = 40, 17, 9
+    X = rng.random((w_in, B))
+    conn = synth.connectivity(w, k, w_in, seed=k + 60)
+    theta = synth.table_logits(w, 1 << k, seed=k + 61)
+    sat = np.where(theta > 0, 800.0, -800.0).astype(np.float32)
+    np.testing.assert_array_equal(oracle.lut_forward(X, conn, theta, "st"),
+                                  oracle.lut_forward(X, conn, sat, "soft"))
+    # the input gradient is the soft one of the saturated tables; dtheta keeps
+    # the sigmoid slope of the real logits
+    dY = rng.standard_normal((w, B))
+    dth, dX = oracle.lut_backward(X, conn, theta, dY, node="st")
+    _, dXs = oracle.lut_backward(X, conn, sat, dY, node="soft")
+    np.testing.assert_allclose(dX, dXs, rtol=1e-13, atol=1e-15)
+    dths, _ = oracle.lut_backward(X, conn, theta, dY, want_dx=False, node="soft")
+    np.testing.assert_array_equal(dth, dths)
+
+
+@pytest.mark.parametrize("k", [2, 4, 6])
+def test_st_binary_inputs_give_the_hard_lookup(k):
+    # on binary inputs the straight-through forward is the deployed network:
+    # the bit-packed lookup of the discretized tables (App. C.1)
+    rng = np.random.default_rng(700 + k)
+    w_in, w, N = 45, 29, 70
+    Xb = rng.integers(0, 2, size=(w_in, N)).astype(np.float64)
+    conn = synth.connectivity(w, k, w_in, seed=k + 70)
+    theta = synth.table_logits(w, 1 << k, seed=k + 71)
+    y = oracle.lut_forward(Xb, conn, theta, "st")
+    W = (N + 31) // 32
+    xp = np.zeros((w_in, W), np.uint32)
+    for s in range(N):
+        xp[:, s // 32] |= (Xb[:, s].astype(np.uint32) << np.uint32(s % 32))
+    yp = oracle.hard_forward(xp, N, conn, oracle.binarize_tables(theta))
+    np.testing.assert_array_equal(_unpack(yp, N), y)
+
+
+def test_st_k1_closed_form():
+    # k = 1, theta = (0, 2): y = [0 > 0] (1 - x) + [2 > 0] x = x;
+    # dtheta = (s'(0) sum g (1 - x), s'(2) sum g x), s' = s (1 - s); dx = g (1 - 0)
+    X = np.array([[0.25, 0.5, 1.0]])
+    conn = np.array([[0]], np.int32)
+    theta = np.array([[0.0, 2.0]], np.float32)
+    g = np.array([[1.0, -2.0, 0.5]])
+    np.testing.assert_array_equal(oracle.lut_forward(X, conn, theta, "st"), X)
+    dth, dX = oracle.lut_backward(X, conn, theta, g, node="st")
+    s2 = 1.0 / (1.0 + math.exp(-2.0))
+    want = [0.25 * float(np.sum(g * (1 - X))), s2 * (1 - s2) * float(np.sum(g * X))]
+    np.testing.assert_allclose(dth[0], want, rtol=1e-14)
+    np.testing.assert_allclose(dX, g, rtol=1e-14)
 
 
 # -------------------------------------------------------------------- head --
