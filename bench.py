@@ -41,6 +41,14 @@ from paper_2602_07400_gb300 import synth  # noqa: E402
 
 METRIC = "LUT train samples/s (fwd+bwd) and hard bit-packed MSamples/s; % of roofline"
 FP32_LANES_PER_SM = 128
+# the paper's own figures for a workload of the same shape, on its hardware
+# (context only, not a target: another machine and its own timing protocol)
+PAPER_CONTEXT = {
+    "hard_mnist_w4000": "paper, hardware evaluation table: RTX 3090 bit-packed forward of the w=4000 MNIST "
+                        "network, batch 1024: 8.66 MSamples/s (RTX 2080 Ti 6.98)",
+    "hard_mnist_w4000_4m": "paper, hardware evaluation table: RTX 3090 bit-packed forward of the w=4000 MNIST "
+                           "network, batch 1024: 8.66 MSamples/s; FPGA max-throughput mode ~126 MSamples/s",
+}
 SMI_FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
@@ -53,6 +61,8 @@ def parse_args():
     p.add_argument("--warmup", type=int, default=20)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default="mnist", choices=sorted(synth.WORKLOADS))
+    p.add_argument("--node", default="soft", choices=["soft", "st"],
+                   help="LightLUT node form of the training step: soft, or straight-through hard")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--profile", action="store_true",
@@ -251,7 +261,7 @@ def run_ours(args):
                                       device="cuda" if hard_only else "cpu")
     st = None
     if not hard_only:
-        st = TrainStep(net, B, wl.d, wl.thresholds, wl.classes, wl.tau)
+        st = TrainStep(net, B, wl.d, wl.thresholds, wl.classes, wl.tau, node=args.node)
         st.load(x_gen.cuda(), lab_gen.cuda())
     hi = HardInfer(net, B, wl.d, wl.thresholds, wl.classes)
     if st is not None:
@@ -374,12 +384,14 @@ def run_ours(args):
             "data": "synthetic (seeded class-conditional Gaussian blobs, MNIST/CIFAR shapes; random-init tables)",
             "config": {"workload": wl.name, "batch_per_gpu": B, "d": wl.d, "thresholds": list(wl.thresholds),
                        "widths": list(wl.widths), "k": wl.k, "classes": wl.classes, "tau": wl.tau,
+                       "node": "LightLUT " + ("soft" if args.node == "soft" else "straight-through hard"),
                        "l2": "flushed between steps (512 MB write outside the timed events)",
                        "parallelism": f"dp{world} (independent batches, no collective)"},
             "hard": {"value": job_rate(world, B, K, hard_sum) / 1e6, "unit": "MSamples/s",
                      "ms_per_batch": ms_step_hard, "batch": B,
                      "includes": "binarize + encode/pack + 2 hard layers + popcount head + argmax"},
             "ms_per_step_total": ms_step_train + ms_step_hard,
+            **({"context": PAPER_CONTEXT[wl.name]} if wl.name in PAPER_CONTEXT else {}),
             "calls": calls_out,
             "roofline": roof,
             "gpu_launches": launches,
@@ -473,13 +485,13 @@ def run_e2e(args, st, hi, wl, B):
 
 # -------------------------------------------------- oracle (CPU) legs --
 
-def oracle_train_rate(wl, samples: int, seed: int = 0):
+def oracle_train_rate(wl, samples: int, seed: int = 0, node: str = "soft"):
     import oracle
     conn1, th1, conn2, th2 = synth.network(wl, seed=0)
     x, lab = synth.blob_batch(samples, wl.d, wl.classes, wl.sigma, seed=3000 + seed)
     t0 = time.perf_counter()
     oracle.train_step(x.numpy(), lab.numpy(), wl.thresholds, conn1, th1, conn2, th2,
-                      wl.classes, wl.tau)
+                      wl.classes, wl.tau, node=node)
     return samples / (time.perf_counter() - t0)
 
 
@@ -500,13 +512,13 @@ def calibrated(rate_fn, wl, budget_s: float, lo: int, hi: int):
     return rate_fn(wl, n, seed=1), n
 
 
-def cpu_baseline(wl, budget_s=12.0):
+def cpu_baseline(wl, budget_s=12.0, node="soft"):
     import oracle
     hard_only = wl.name.startswith("hard_")
     cores = oracle.max_threads()
     out = {}
     if not hard_only:
-        r, n = calibrated(oracle_train_rate, wl, budget_s, 4, wl.batch)
+        r, n = calibrated(lambda w_, n_, seed=0: oracle_train_rate(w_, n_, seed, node), wl, budget_s, 4, wl.batch)
         out = {"value": r, "unit": "samples/s", "cores": cores, "kind": "oracle",
                "sample": f"train step (fwd+bwd) on {n} of the {wl.batch} samples of a batch, "
                          f"full network, fp64, OpenMP over independent outputs"}
@@ -523,7 +535,7 @@ def run_reference(args):
     import oracle
     wl = synth.WORKLOADS[args.workload]
     hard_only = wl.name.startswith("hard_")
-    fn = oracle_hard_rate if hard_only else oracle_train_rate
+    fn = oracle_hard_rate if hard_only else (lambda w_, n_, seed=0: oracle_train_rate(w_, n_, seed, args.node))
     lo = 32 if hard_only else 2
     # size one step to about 1-2 s of oracle work
     r0 = fn(wl, lo)
@@ -566,7 +578,7 @@ def main():
         return
     if not args.profile and not args.no_cpu_baseline:
         wl = synth.WORKLOADS[args.workload]
-        cb, cb_hard = cpu_baseline(wl)
+        cb, cb_hard = cpu_baseline(wl, node=args.node)
         if cb:
             res["cpu_baseline"] = cb
         res["hard"]["cpu_baseline"] = cb_hard

@@ -52,8 +52,23 @@ typedef enum {
     BITLOGIC_ERR_DEVICE = -8,     /* device-side index check tripped */
     BITLOGIC_ERR_THRESH = -9,     /* thresholds: b outside 1..32 */
     BITLOGIC_ERR_TOO_LARGE = -10, /* sizes beyond bitlogic_head_loss_noalloc's fixed scratch */
-    BITLOGIC_ERR_HYPER = -11      /* optimizer hyperparameter out of range */
+    BITLOGIC_ERR_HYPER = -11,     /* optimizer hyperparameter out of range */
+    BITLOGIC_ERR_NODE = -12       /* unknown node form */
 } bitlogic_status_t;
+
+/* Node forms of the LightLUT parameterization (§2 "Gradient-based LUT
+ * methods"; the node sweep of §4 lists both):
+ *   BITLOGIC_NODE_SOFT  table entry t_a = sigmoid(theta_a) in the forward.
+ *   BITLOGIC_NODE_ST    straight-through hard sampling: the forward uses the
+ *                       discretized entry t_a = [theta_a > 0] (the value
+ *                       bitlogic_binarize_tables deploys; theta = 0 gives 0),
+ *                       the input gradient is that of the hard-table forward,
+ *                       and the table gradient reaches theta through the
+ *                       sigmoid slope as if t_a were sigmoid(theta_a). */
+typedef enum {
+    BITLOGIC_NODE_SOFT = 0,
+    BITLOGIC_NODE_ST = 1
+} bitlogic_node_t;
 
 /* Thermometer encoder E: R^d -> {0,1}^{db} (paper §3, "Encoders and heads";
  * linear thermometer with b thresholds, b+1 levels on b wires).
@@ -78,6 +93,15 @@ int bitlogic_encode_thermometer(const uint8_t* x, int64_t B, int32_t d,
 int bitlogic_lut_forward(const float* X, int32_t w_in, int64_t B,
                          const int32_t* conn, const float* theta,
                          int32_t w, int32_t k, float* Y, cudaStream_t stream);
+
+/* bitlogic_lut_forward for either node form: node is a bitlogic_node_t
+ * (BITLOGIC_ERR_NODE otherwise); BITLOGIC_NODE_SOFT is bitlogic_lut_forward.
+ * With BITLOGIC_NODE_ST and binary inputs every output is 0 or 1: the
+ * deployed network's value, as bitlogic_hard_forward computes it. */
+int bitlogic_lut_forward_node(const float* X, int32_t w_in, int64_t B,
+                              const int32_t* conn, const float* theta,
+                              int32_t w, int32_t k, int32_t node, float* Y,
+                              cudaStream_t stream);
 
 /* Bytes of workspace bitlogic_lut_backward needs (0 when want_dx == 0). */
 size_t bitlogic_lut_backward_workspace(int32_t w_in, int64_t B, int32_t w,
@@ -150,6 +174,20 @@ int bitlogic_lut_backward_ex(const float* X, int32_t w_in, int64_t B,
                              const int32_t* up_edge, int32_t up_edges,
                              float* dtheta, float* edge_terms, const int32_t* edge_pos,
                              float* dY_out, cudaStream_t stream);
+
+/* bitlogic_lut_backward_ex for either node form (node as in
+ * bitlogic_lut_forward_node).  For BITLOGIC_NODE_ST:
+ *   dtheta[j][a] = s_a (1 - s_a) sum_s dY[j][s] w_a(x(s)),  s_a = sigmoid(theta)
+ *   (the straight-through estimate: the same expression as the soft node),
+ *   and the edge terms use the hard entries [theta > 0]. */
+int bitlogic_lut_backward_node(const float* X, int32_t w_in, int64_t B,
+                               const int32_t* conn, const float* theta,
+                               int32_t w, int32_t k, int32_t node,
+                               const float* dY, int32_t dy_group,
+                               const float* up_terms, const int32_t* up_off,
+                               const int32_t* up_edge, int32_t up_edges,
+                               float* dtheta, float* edge_terms, const int32_t* edge_pos,
+                               float* dY_out, cudaStream_t stream);
 
 /* Bytes of workspace bitlogic_head_loss needs. */
 size_t bitlogic_head_loss_workspace(int64_t B, int32_t C);

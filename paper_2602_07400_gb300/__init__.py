@@ -30,11 +30,23 @@ __all__ = [
     "bitlogic_head_loss_workspace", "bitlogic_head_loss_noalloc",
     "bitlogic_head_loss", "bitlogic_binarize_tables", "bitlogic_pack_bits",
     "bitlogic_hard_forward", "bitlogic_build_csr", "bitlogic_csr_positions", "bitlogic_device_error",
-    "bitlogic_adamw_update",
+    "bitlogic_adamw_update", "bitlogic_lut_forward_node", "bitlogic_lut_backward_node", "NODE_FORMS",
     "bitlogic_status_string", "bitlogic_version", "LIB_PATH",
 ]
 
 LIB_PATH = _build.LIB
+
+# node forms (bitlogic_node_t): the soft LightLUT node and its
+# straight-through hard form
+NODE_FORMS = {"soft": 0, "st": 1}
+
+
+def _node_code(node) -> int:
+    if isinstance(node, str):
+        if node not in NODE_FORMS:
+            raise ValueError(f"node must be one of {sorted(NODE_FORMS)}")
+        return NODE_FORMS[node]
+    return int(node)
 
 
 class BitLogicError(RuntimeError):
@@ -49,6 +61,7 @@ _P, _I32, _I64, _F32, _SZ = (ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64,
 _SIGS = {
     "bitlogic_encode_thermometer": ([_P, _I64, _I32, _P, _I32, _P, _P], ctypes.c_int),
     "bitlogic_lut_forward": ([_P, _I32, _I64, _P, _P, _I32, _I32, _P, _P], ctypes.c_int),
+    "bitlogic_lut_forward_node": ([_P, _I32, _I64, _P, _P, _I32, _I32, _I32, _P, _P], ctypes.c_int),
     "bitlogic_lut_backward_workspace": ([_I32, _I64, _I32, _I32, _I32], _SZ),
     "bitlogic_lut_backward": ([_P, _I32, _I64, _P, _P, _I32, _I32, _P, _P, _P, _P, _P,
                                _P, _SZ, _P], ctypes.c_int),
@@ -57,6 +70,8 @@ _SIGS = {
     "bitlogic_csr_reduce": ([_P, _I64, _P, _P, _I32, _I32, _P, _P], ctypes.c_int),
     "bitlogic_lut_backward_ex": ([_P, _I32, _I64, _P, _P, _I32, _I32, _P, _I32, _P, _P, _P, _I32,
                                   _P, _P, _P, _P, _P], ctypes.c_int),
+    "bitlogic_lut_backward_node": ([_P, _I32, _I64, _P, _P, _I32, _I32, _I32, _P, _I32, _P, _P, _P, _I32,
+                                    _P, _P, _P, _P, _P], ctypes.c_int),
     "bitlogic_head_loss_ex": ([_P, _I32, _I64, _I32, _F32, _P, _P, _P, _P, _P, _P, _SZ, _P],
                               ctypes.c_int),
     "bitlogic_head_loss_workspace": ([_I64, _I32], _SZ),
@@ -157,6 +172,20 @@ def bitlogic_lut_forward(X: torch.Tensor, conn: torch.Tensor, theta: torch.Tenso
         _ptr(X), w_in, B, _ptr(conn), _ptr(theta), w, k, _ptr(Y), _stream(stream)))
 
 
+def bitlogic_lut_forward_node(X: torch.Tensor, conn: torch.Tensor, theta: torch.Tensor,
+                              Y: torch.Tensor, node="soft", stream=None):
+    """node "soft" or "st" (or the bitlogic_node_t value)."""
+    code = _node_code(node)
+    w_in, B = X.shape
+    w, k = conn.shape
+    _need(X, "X", torch.float32, (w_in, B))
+    _need(conn, "conn", torch.int32, (w, k))
+    _need(theta, "theta", torch.float32, (w, 1 << k))
+    _need(Y, "Y", torch.float32, (w, B))
+    _check("bitlogic_lut_forward_node", load().bitlogic_lut_forward_node(
+        _ptr(X), w_in, B, _ptr(conn), _ptr(theta), w, k, code, _ptr(Y), _stream(stream)))
+
+
 def bitlogic_lut_backward_workspace(w_in: int, B: int, w: int, k: int, want_dx: bool) -> int:
     return int(load().bitlogic_lut_backward_workspace(w_in, B, w, k, int(bool(want_dx))))
 
@@ -228,6 +257,25 @@ def bitlogic_lut_backward_ex(X: torch.Tensor, conn: torch.Tensor, theta: torch.T
                              dY_out: Optional[torch.Tensor] = None, stream=None):
     """up_edge None with up_terms: the upstream term rows are in CSR order.
     edge_pos: store the term of edge e at row edge_pos[e] of edge_terms."""
+    _backward_general("bitlogic_lut_backward_ex", None, X, conn, theta, dtheta, dY, dy_group, up_terms,
+                      up_off, up_edge, edge_terms, edge_pos, dY_out, stream)
+
+
+def bitlogic_lut_backward_node(X: torch.Tensor, conn: torch.Tensor, theta: torch.Tensor,
+                               dtheta: torch.Tensor, node="soft", dY: Optional[torch.Tensor] = None,
+                               dy_group: int = 1, up_terms: Optional[torch.Tensor] = None,
+                               up_off: Optional[torch.Tensor] = None,
+                               up_edge: Optional[torch.Tensor] = None,
+                               edge_terms: Optional[torch.Tensor] = None,
+                               edge_pos: Optional[torch.Tensor] = None,
+                               dY_out: Optional[torch.Tensor] = None, stream=None):
+    """bitlogic_lut_backward_ex for the node form ``node`` ("soft" or "st")."""
+    _backward_general("bitlogic_lut_backward_node", _node_code(node), X, conn, theta, dtheta, dY, dy_group,
+                      up_terms, up_off, up_edge, edge_terms, edge_pos, dY_out, stream)
+
+
+def _backward_general(fn, node, X, conn, theta, dtheta, dY, dy_group, up_terms, up_off, up_edge,
+                      edge_terms, edge_pos, dY_out, stream):
     w_in, B = X.shape
     w, k = conn.shape
     _need(X, "X", torch.float32, (w_in, B))
@@ -251,10 +299,11 @@ def bitlogic_lut_backward_ex(X: torch.Tensor, conn: torch.Tensor, theta: torch.T
         _need(edge_pos, "edge_pos", torch.int32, (w * k,))
     if dY_out is not None:
         _need(dY_out, "dY_out", torch.float32, (w, B))
-    _check("bitlogic_lut_backward_ex", load().bitlogic_lut_backward_ex(
-        _ptr(X), w_in, B, _ptr(conn), _ptr(theta), w, k, _ptr(dY), int(dy_group),
-        _ptr(up_terms), _ptr(up_off), _ptr(up_edge), n_up, _ptr(dtheta), _ptr(edge_terms),
-        _ptr(edge_pos), _ptr(dY_out), _stream(stream)))
+    rest = (_ptr(dY), int(dy_group), _ptr(up_terms), _ptr(up_off), _ptr(up_edge), n_up, _ptr(dtheta),
+            _ptr(edge_terms), _ptr(edge_pos), _ptr(dY_out), _stream(stream))
+    head = (_ptr(X), w_in, B, _ptr(conn), _ptr(theta), w, k)
+    args = head + rest if node is None else head + (node,) + rest
+    _check(fn, getattr(load(), fn)(*args))
 
 
 def bitlogic_head_loss_ex(Y: torch.Tensor, labels: torch.Tensor, C: int, tau: float,

@@ -44,6 +44,7 @@ extern "C" const char* bitlogic_status_string(int code) {
         case BITLOGIC_ERR_THRESH: return "number of thresholds must be 1..32";
         case BITLOGIC_ERR_TOO_LARGE: return "sizes exceed the fixed scratch of the allocation-free entry point";
         case BITLOGIC_ERR_HYPER: return "optimizer hyperparameter out of range";
+        case BITLOGIC_ERR_NODE: return "unknown node form";
         default: return "unknown status";
     }
 }

@@ -2,7 +2,10 @@
 //
 // Node (LightLUT, §2 of the paper: Kronecker-indicator basis, 2^k logits per
 // node), read as t = sigmoid(theta), y = sum_a t_a prod_i x_i^{a_i}(1-x_i)^{1-a_i}
-// with connectivity slot i = bit i of the table index a.
+// with connectivity slot i = bit i of the table index a.  The straight-through
+// hard form of the same node (§4 node sweep) takes t_a = [theta_a > 0] in the
+// forward and in the input gradient, and the sigmoid slope for dtheta; only
+// the per-node table set-up differs between the two forms.
 //
 // Evaluation: the multilinear form is a complete binary lerp tree over the
 // k inputs (level l interpolates with x_l), 2^k - 1 lerps per (node, sample).
@@ -179,23 +182,33 @@ __device__ __forceinline__ void load_rows(const int* __restrict__ conn, int j, i
     if (bad && lane == 0) flag_index_error();
 }
 
-// Per-warp node set-up: connectivity rows (range-checked), sigmoid of the
-// table logits, level-0 constants broadcast to every lane through shared
-// memory.  Lane l (l < 2^(k-1)) keeps t[2l] and t[2l+1] for the dtheta
-// epilogue.
+// Table entry of a node form (bitlogic_node_t): the sigmoid sg of the logit
+// th for the soft LightLUT node, the hard sample [th > 0] for the
+// straight-through node (whose theta gradient still takes the slope of sg).
+__device__ __forceinline__ float table_value(float th, float sg, int node) {
+    return node == BITLOGIC_NODE_ST ? (th > 0.f ? 1.f : 0.f) : sg;
+}
+
+// Per-warp node set-up: connectivity rows (range-checked), table entries of
+// the node form, level-0 constants broadcast to every lane through shared
+// memory.  Lane l (l < 2^(k-1)) keeps the sigmoids of entries 2l and 2l+1
+// for the dtheta epilogue.
 template <int k>
 __device__ __forceinline__ void node_setup(const int* __restrict__ conn,
                                            const float* __restrict__ theta, int j, int w_in,
-                                           int lane, float2* sPair, int (&rows)[k],
+                                           int node, int lane, float2* sPair, int (&rows)[k],
                                            float (&te)[1 << (k - 1)], float (&d)[1 << (k - 1)],
                                            float& t0, float& t1) {
     constexpr int K = 1 << k, H = K / 2;
     load_rows<k>(conn, j, w_in, lane, rows);
     t0 = t1 = 0.f;
     if (lane < H) {
-        t0 = sigmoidf(__ldg(theta + (long long)j * K + 2 * lane));
-        t1 = sigmoidf(__ldg(theta + (long long)j * K + 2 * lane + 1));
-        sPair[lane] = make_float2(t0, t1 - t0);
+        const float th0 = __ldg(theta + (long long)j * K + 2 * lane);
+        const float th1 = __ldg(theta + (long long)j * K + 2 * lane + 1);
+        t0 = sigmoidf(th0);
+        t1 = sigmoidf(th1);
+        const float v0 = table_value(th0, t0, node), v1 = table_value(th1, t1, node);
+        sPair[lane] = make_float2(v0, v1 - v0);
     }
     __syncwarp();
 #pragma unroll
@@ -224,7 +237,7 @@ template <int k>
 __global__ void __launch_bounds__(kFwdWarps * 32)
 lut_forward_kernel(const float* __restrict__ X, int w_in, long long B,
                    const int* __restrict__ conn, const float* __restrict__ theta, int w,
-                   float* __restrict__ Y, long long chunk) {
+                   int node, float* __restrict__ Y, long long chunk) {
     constexpr int H = 1 << (k - 1);
     __shared__ float2 sPair[kFwdWarps][H];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -232,7 +245,7 @@ lut_forward_kernel(const float* __restrict__ X, int w_in, long long B,
     if (j >= w) return;
     int rows[k];
     float te[H], d[H], t0, t1;
-    node_setup<k>(conn, theta, j, w_in, lane, sPair[warp], rows, te, d, t0, t1);
+    node_setup<k>(conn, theta, j, w_in, node, lane, sPair[warp], rows, te, d, t0, t1);
     const long long s0 = (long long)blockIdx.y * chunk;
     const long long s1 = min(B, s0 + chunk);
     const float* xr[k];
@@ -255,7 +268,7 @@ template <int k>
 __global__ void __launch_bounds__(kFwdWarps * 32)
 lut_forward_staged_kernel(const float* __restrict__ X, int w_in, long long B,
                           const int* __restrict__ conn, const float* __restrict__ theta, int w,
-                          float* __restrict__ Y, long long chunk) {
+                          int node, float* __restrict__ Y, long long chunk) {
     constexpr int K = 1 << k, CH = kStageSamples, L = fwd_poly_levels(k), S = 1 << L;
     __shared__ __align__(16) float sRing[kFwdWarps][kStages * k * CH];
     __shared__ __align__(16) float sCoef[kFwdWarps][K];
@@ -264,10 +277,13 @@ lut_forward_staged_kernel(const float* __restrict__ X, int w_in, long long B,
     if (j >= w) return;
     int rows[k];
     load_rows<k>(conn, j, w_in, lane, rows);
-    // sigmoid of the table spread over the lanes (entries l, l + 32), then
-    // lane l < K / S turns subtable l into its Moebius coefficients
+    // table entries spread over the lanes (entries l, l + 32), then lane
+    // l < K / S turns subtable l into its Moebius coefficients
 #pragma unroll
-    for (int a = lane; a < K; a += 32) sCoef[warp][a] = sigmoidf(__ldg(theta + (long long)j * K + a));
+    for (int a = lane; a < K; a += 32) {
+        const float th = __ldg(theta + (long long)j * K + a);
+        sCoef[warp][a] = table_value(th, sigmoidf(th), node);
+    }
     __syncwarp();
     if (lane < K / S) {
         float c[S];
@@ -379,7 +395,7 @@ __device__ __forceinline__ void term_range(const GradSource& gs, int j, int lane
 template <int k, bool WANT_DX, bool TERMS>
 __global__ void __launch_bounds__(kFwdWarps * 32)
 lut_backward_kernel(const float* __restrict__ X, int w_in, long long B,
-                    const int* __restrict__ conn, const float* __restrict__ theta, int w,
+                    const int* __restrict__ conn, const float* __restrict__ theta, int w, int node,
                     GradSource gs, float* __restrict__ dtheta, float* __restrict__ P,
                     const int* __restrict__ epos, float* __restrict__ dY_out) {
     constexpr int K = 1 << k, H = K / 2;
@@ -390,7 +406,7 @@ lut_backward_kernel(const float* __restrict__ X, int w_in, long long B,
     if (j >= w) return;
     int rows[k];
     float te[H], d[H], t0, t1;
-    node_setup<k>(conn, theta, j, w_in, lane, sPair[warp], rows, te, d, t0, t1);
+    node_setup<k>(conn, theta, j, w_in, node, lane, sPair[warp], rows, te, d, t0, t1);
     int e0 = 0, e1 = 0;
     if constexpr (TERMS) term_range(gs, j, lane, e0, e1);
     const float* gr = TERMS ? nullptr : gs.dY + (long long)(j / gs.group) * B;
@@ -512,7 +528,7 @@ template <int k, bool WANT_DX, bool TERMS, bool POS>
 __global__ void __launch_bounds__(kBwdWarps * 32, BITLOGIC_BWD_MIN_BLOCKS)
 lut_backward_node_kernel(const float* __restrict__ X, int w_in, long long B,
                          const int* __restrict__ conn, const float* __restrict__ theta, int w,
-                         GradSource gs, float* __restrict__ dtheta, float* __restrict__ P,
+                         int node, GradSource gs, float* __restrict__ dtheta, float* __restrict__ P,
                          const int* __restrict__ epos, float* __restrict__ dY_out) {
     constexpr int K = 1 << k, H = K / 2, H2 = K / 4, R = k + 1, CH = kStageSamples;
     constexpr int NQ = (k + 1) / 2;   // slots stored per lane (rounded up)
@@ -523,7 +539,7 @@ lut_backward_node_kernel(const float* __restrict__ X, int w_in, long long B,
     constexpr int FPW = node_floats_per_warp<k, TERMS>();
     float* ring = smem + warp * FPW;
     float* gbuf = ring + ring_floats<k, TERMS>();   // summed upstream gradient (terms source)
-    float* sT = smem + kBwdWarps * FPW + nb * K;   // sigmoid of the node's logits
+    float* sT = smem + kBwdWarps * FPW + nb * K;   // the node's table entries
     const int j = blockIdx.x * kNodesPerBlock + nb;
     const bool live = j < w;   // a dead warp still reaches the block barriers
 
@@ -533,10 +549,13 @@ lut_backward_node_kernel(const float* __restrict__ X, int w_in, long long B,
     float t0 = 0.f, t1 = 0.f;
     if (live) {
         load_rows<k>(conn, j, w_in, lane, rows);
-        if (sub == 0 && lane < H) {
-            t0 = sigmoidf(__ldg(theta + (long long)j * K + 2 * lane));
-            t1 = sigmoidf(__ldg(theta + (long long)j * K + 2 * lane + 1));
-            *reinterpret_cast<float2*>(sT + 2 * lane) = make_float2(t0, t1);
+        if (sub == 0 && lane < H) {   // t0, t1: sigmoids, for the dtheta epilogue
+            const float th0 = __ldg(theta + (long long)j * K + 2 * lane);
+            const float th1 = __ldg(theta + (long long)j * K + 2 * lane + 1);
+            t0 = sigmoidf(th0);
+            t1 = sigmoidf(th1);
+            *reinterpret_cast<float2*>(sT + 2 * lane) =
+                make_float2(table_value(th0, t0, node), table_value(th1, t1, node));
         }
     }
     __syncthreads();
@@ -1013,22 +1032,22 @@ long long forward_chunk(int w_in, int w, long long B) {
 
 template <int k>
 int launch_forward(const float* X, int w_in, long long B, const int* conn, const float* theta,
-                   int w, float* Y, bool vec, cudaStream_t st) {
+                   int w, int node, float* Y, bool vec, cudaStream_t st) {
     long long chunk = forward_chunk(w_in, w, B);
     if (vec) chunk = (chunk + 3) / 4 * 4;
     const long long ny = (B + chunk - 1) / chunk;
     if (ny > 65535) return BITLOGIC_ERR_SHAPE;
     dim3 grid((unsigned)((w + kFwdWarps - 1) / kFwdWarps), (unsigned)ny);
     if (vec)
-        lut_forward_staged_kernel<k><<<grid, kFwdWarps * 32, 0, st>>>(X, w_in, B, conn, theta, w, Y, chunk);
+        lut_forward_staged_kernel<k><<<grid, kFwdWarps * 32, 0, st>>>(X, w_in, B, conn, theta, w, node, Y, chunk);
     else
-        lut_forward_kernel<k><<<grid, kFwdWarps * 32, 0, st>>>(X, w_in, B, conn, theta, w, Y, chunk);
+        lut_forward_kernel<k><<<grid, kFwdWarps * 32, 0, st>>>(X, w_in, B, conn, theta, w, node, Y, chunk);
     return launch_status();
 }
 
 template <int k, bool WANT_DX, bool TERMS>
 int launch_backward_impl(const float* X, int w_in, long long B, const int* conn, const float* theta,
-                         int w, const GradSource& gs, float* dtheta, float* P, const int* epos,
+                         int w, int node, const GradSource& gs, float* dtheta, float* P, const int* epos,
                          float* dY_out, bool staged, cudaStream_t st) {
     if constexpr (k >= 2) {
         if (staged) {
@@ -1041,24 +1060,26 @@ int launch_backward_impl(const float* X, int w_in, long long B, const int* conn,
                 cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
                 return BITLOGIC_ERR_CUDA;
             kern<<<(unsigned)((w + kNodesPerBlock - 1) / kNodesPerBlock), kBwdWarps * 32, smem, st>>>(
-                X, w_in, B, conn, theta, w, gs, dtheta, P, epos, dY_out);
+                X, w_in, B, conn, theta, w, node, gs, dtheta, P, epos, dY_out);
             return launch_status();
         }
     }
     dim3 grid((unsigned)((w + kFwdWarps - 1) / kFwdWarps));
-    lut_backward_kernel<k, WANT_DX, TERMS><<<grid, kFwdWarps * 32, 0, st>>>(X, w_in, B, conn, theta, w, gs,
-                                                                            dtheta, P, epos, dY_out);
+    lut_backward_kernel<k, WANT_DX, TERMS><<<grid, kFwdWarps * 32, 0, st>>>(X, w_in, B, conn, theta, w, node,
+                                                                            gs, dtheta, P, epos, dY_out);
     return launch_status();
 }
 
 template <int k>
 int launch_backward(const float* X, int w_in, long long B, const int* conn, const float* theta,
-                    int w, const GradSource& gs, float* dtheta, float* P, const int* epos,
+                    int w, int node, const GradSource& gs, float* dtheta, float* P, const int* epos,
                     float* dY_out, cudaStream_t st) {
     const bool terms = gs.terms != nullptr;
     const bool staged = (B % 4 == 0) && aligned16(X) && aligned16(terms ? gs.terms : gs.dY) &&
                         (!dY_out || aligned16(dY_out)) && (!P || aligned16(P));
-    if (staged && !P && !terms) {   // dtheta only, from dY rows
+    // dtheta only, from dY rows: the table entries are not needed, so both
+    // node forms run the same kernel
+    if (staged && !P && !terms) {
         constexpr size_t smem = (size_t)kThetaWarps * theta_floats_per_warp<k>() * sizeof(float);
         auto kern = lut_backward_theta_kernel<k>;
         if (smem > 40 * 1024 &&
@@ -1073,14 +1094,14 @@ int launch_backward(const float* X, int w_in, long long B, const int* conn, cons
         return launch_status();
     }
     if (P) {
-        return terms ? launch_backward_impl<k, true, true>(X, w_in, B, conn, theta, w, gs, dtheta, P, epos, dY_out,
+        return terms ? launch_backward_impl<k, true, true>(X, w_in, B, conn, theta, w, node, gs, dtheta, P, epos, dY_out,
                                                            staged, st)
-                     : launch_backward_impl<k, true, false>(X, w_in, B, conn, theta, w, gs, dtheta, P, epos, dY_out,
+                     : launch_backward_impl<k, true, false>(X, w_in, B, conn, theta, w, node, gs, dtheta, P, epos, dY_out,
                                                             staged, st);
     }
-    return terms ? launch_backward_impl<k, false, true>(X, w_in, B, conn, theta, w, gs, dtheta, P, epos, dY_out,
+    return terms ? launch_backward_impl<k, false, true>(X, w_in, B, conn, theta, w, node, gs, dtheta, P, epos, dY_out,
                                                         staged, st)
-                 : launch_backward_impl<k, false, false>(X, w_in, B, conn, theta, w, gs, dtheta, P, epos, dY_out,
+                 : launch_backward_impl<k, false, false>(X, w_in, B, conn, theta, w, node, gs, dtheta, P, epos, dY_out,
                                                          staged, st);
 }
 
@@ -1101,22 +1122,30 @@ using namespace bitlogic;
 
 BITLOGIC_ERROR_READER(lut_soft)
 
-extern "C" int bitlogic_lut_forward(const float* X, int32_t w_in, int64_t B,
-                                    const int32_t* conn, const float* theta,
-                                    int32_t w, int32_t k, float* Y, cudaStream_t stream) {
+extern "C" int bitlogic_lut_forward_node(const float* X, int32_t w_in, int64_t B,
+                                         const int32_t* conn, const float* theta,
+                                         int32_t w, int32_t k, int32_t node, float* Y,
+                                         cudaStream_t stream) {
     int st = check_layer(X, w_in, B, conn, theta, w, k);
     if (st) return st;
+    if (node != BITLOGIC_NODE_SOFT && node != BITLOGIC_NODE_ST) return BITLOGIC_ERR_NODE;
     if (B == 0) return BITLOGIC_OK;
     if (!Y) return BITLOGIC_ERR_NULL;
     const bool vec = (B % 4 == 0) && aligned16(X) && aligned16(Y);
     switch (k) {
-        case 1: return launch_forward<1>(X, w_in, B, conn, theta, w, Y, vec, stream);
-        case 2: return launch_forward<2>(X, w_in, B, conn, theta, w, Y, vec, stream);
-        case 3: return launch_forward<3>(X, w_in, B, conn, theta, w, Y, vec, stream);
-        case 4: return launch_forward<4>(X, w_in, B, conn, theta, w, Y, vec, stream);
-        case 5: return launch_forward<5>(X, w_in, B, conn, theta, w, Y, vec, stream);
-        default: return launch_forward<6>(X, w_in, B, conn, theta, w, Y, vec, stream);
+        case 1: return launch_forward<1>(X, w_in, B, conn, theta, w, node, Y, vec, stream);
+        case 2: return launch_forward<2>(X, w_in, B, conn, theta, w, node, Y, vec, stream);
+        case 3: return launch_forward<3>(X, w_in, B, conn, theta, w, node, Y, vec, stream);
+        case 4: return launch_forward<4>(X, w_in, B, conn, theta, w, node, Y, vec, stream);
+        case 5: return launch_forward<5>(X, w_in, B, conn, theta, w, node, Y, vec, stream);
+        default: return launch_forward<6>(X, w_in, B, conn, theta, w, node, Y, vec, stream);
     }
+}
+
+extern "C" int bitlogic_lut_forward(const float* X, int32_t w_in, int64_t B,
+                                    const int32_t* conn, const float* theta,
+                                    int32_t w, int32_t k, float* Y, cudaStream_t stream) {
+    return bitlogic_lut_forward_node(X, w_in, B, conn, theta, w, k, BITLOGIC_NODE_SOFT, Y, stream);
 }
 
 extern "C" size_t bitlogic_lut_backward_workspace(int32_t w_in, int64_t B, int32_t w,
@@ -1126,16 +1155,17 @@ extern "C" size_t bitlogic_lut_backward_workspace(int32_t w_in, int64_t B, int32
     return (size_t)w * (size_t)k * (size_t)B * sizeof(float);
 }
 
-extern "C" int bitlogic_lut_backward_ex(const float* X, int32_t w_in, int64_t B,
-                                        const int32_t* conn, const float* theta,
-                                        int32_t w, int32_t k,
-                                        const float* dY, int32_t dy_group,
-                                        const float* up_terms, const int32_t* up_off,
-                                        const int32_t* up_edge, int32_t up_edges,
-                                        float* dtheta, float* edge_terms, const int32_t* edge_pos,
-                                        float* dY_out, cudaStream_t stream) {
+extern "C" int bitlogic_lut_backward_node(const float* X, int32_t w_in, int64_t B,
+                                          const int32_t* conn, const float* theta,
+                                          int32_t w, int32_t k, int32_t node,
+                                          const float* dY, int32_t dy_group,
+                                          const float* up_terms, const int32_t* up_off,
+                                          const int32_t* up_edge, int32_t up_edges,
+                                          float* dtheta, float* edge_terms, const int32_t* edge_pos,
+                                          float* dY_out, cudaStream_t stream) {
     int st = check_layer(X, w_in, B, conn, theta, w, k);
     if (st) return st;
+    if (node != BITLOGIC_NODE_SOFT && node != BITLOGIC_NODE_ST) return BITLOGIC_ERR_NODE;
     if (!dtheta) return BITLOGIC_ERR_NULL;
     const bool terms = up_terms != nullptr;
     if (B > 0 && terms == (dY != nullptr)) return BITLOGIC_ERR_NULL;   // exactly one source
@@ -1153,13 +1183,26 @@ extern "C" int bitlogic_lut_backward_ex(const float* X, int32_t w_in, int64_t B,
     }
     GradSource gs{dY, dy_group, up_terms, up_off, up_edge, up_edges};
     switch (k) {
-        case 1: return launch_backward<1>(X, w_in, B, conn, theta, w, gs, dtheta, edge_terms, edge_pos, dY_out, stream);
-        case 2: return launch_backward<2>(X, w_in, B, conn, theta, w, gs, dtheta, edge_terms, edge_pos, dY_out, stream);
-        case 3: return launch_backward<3>(X, w_in, B, conn, theta, w, gs, dtheta, edge_terms, edge_pos, dY_out, stream);
-        case 4: return launch_backward<4>(X, w_in, B, conn, theta, w, gs, dtheta, edge_terms, edge_pos, dY_out, stream);
-        case 5: return launch_backward<5>(X, w_in, B, conn, theta, w, gs, dtheta, edge_terms, edge_pos, dY_out, stream);
-        default: return launch_backward<6>(X, w_in, B, conn, theta, w, gs, dtheta, edge_terms, edge_pos, dY_out, stream);
+        case 1: return launch_backward<1>(X, w_in, B, conn, theta, w, node, gs, dtheta, edge_terms, edge_pos, dY_out, stream);
+        case 2: return launch_backward<2>(X, w_in, B, conn, theta, w, node, gs, dtheta, edge_terms, edge_pos, dY_out, stream);
+        case 3: return launch_backward<3>(X, w_in, B, conn, theta, w, node, gs, dtheta, edge_terms, edge_pos, dY_out, stream);
+        case 4: return launch_backward<4>(X, w_in, B, conn, theta, w, node, gs, dtheta, edge_terms, edge_pos, dY_out, stream);
+        case 5: return launch_backward<5>(X, w_in, B, conn, theta, w, node, gs, dtheta, edge_terms, edge_pos, dY_out, stream);
+        default: return launch_backward<6>(X, w_in, B, conn, theta, w, node, gs, dtheta, edge_terms, edge_pos, dY_out, stream);
     }
+}
+
+extern "C" int bitlogic_lut_backward_ex(const float* X, int32_t w_in, int64_t B,
+                                        const int32_t* conn, const float* theta,
+                                        int32_t w, int32_t k,
+                                        const float* dY, int32_t dy_group,
+                                        const float* up_terms, const int32_t* up_off,
+                                        const int32_t* up_edge, int32_t up_edges,
+                                        float* dtheta, float* edge_terms, const int32_t* edge_pos,
+                                        float* dY_out, cudaStream_t stream) {
+    return bitlogic_lut_backward_node(X, w_in, B, conn, theta, w, k, BITLOGIC_NODE_SOFT, dY, dy_group,
+                                      up_terms, up_off, up_edge, up_edges, dtheta, edge_terms, edge_pos,
+                                      dY_out, stream);
 }
 
 extern "C" int bitlogic_lut_backward_edges(const float* X, int32_t w_in, int64_t B,

@@ -16,10 +16,10 @@ from typing import Optional, Sequence
 import numpy as np
 import torch
 
-from . import (bitlogic_adamw_update, bitlogic_binarize_tables, bitlogic_build_csr, bitlogic_csr_positions,
-               bitlogic_csr_reduce,
+from . import (NODE_FORMS, bitlogic_adamw_update, bitlogic_binarize_tables, bitlogic_build_csr,
+               bitlogic_csr_positions, bitlogic_csr_reduce,
                bitlogic_encode_thermometer, bitlogic_hard_forward, bitlogic_head_loss_ex,
-               bitlogic_head_loss_workspace, bitlogic_lut_backward_ex, bitlogic_lut_forward,
+               bitlogic_head_loss_workspace, bitlogic_lut_backward_node, bitlogic_lut_forward_node,
                bitlogic_pack_bits)
 
 
@@ -57,12 +57,17 @@ class TrainStep:
     (``dyg``) that the layer-2 backward reads for every node of the class, and
     the layer-1 backward reduces layer 2's per-edge input-gradient terms on
     the fly through the CSR map, so neither dY2 nor dY1 is stored (set
-    ``keep_dy1`` to also write dY1, e.g. to check it)."""
+    ``keep_dy1`` to also write dY1, e.g. to check it).  ``node`` picks the
+    LightLUT form of both layers: "soft", or "st" (hard table samples in the
+    forward, straight-through gradient to the logits)."""
 
     def __init__(self, net: Network, B: int, d: int, thresholds: Sequence[int], C: int,
                  tau: float, want_dx1: bool = False, keep_dy1: bool = False,
-                 fuse_dy1: bool = False, csr_order: bool = True, device="cuda"):
+                 fuse_dy1: bool = False, csr_order: bool = True, node: str = "soft", device="cuda"):
         dev = torch.device(device)
+        if node not in NODE_FORMS:
+            raise ValueError(f"node must be one of {sorted(NODE_FORMS)}")
+        self.node = node
         self.net, self.B, self.d, self.C, self.tau = net, int(B), int(d), int(C), float(tau)
         self.thr = [int(t) for t in thresholds]
         assert d * len(self.thr) == net.w_in
@@ -101,9 +106,9 @@ class TrainStep:
         n = self.net
         bitlogic_encode_thermometer(self.x, self.thr, self.bits, stream)
         mark("encode")
-        bitlogic_lut_forward(self.bits, n.conn1, n.theta1, self.y1, stream)
+        bitlogic_lut_forward_node(self.bits, n.conn1, n.theta1, self.y1, self.node, stream)
         mark("forward1")
-        bitlogic_lut_forward(self.y1, n.conn2, n.theta2, self.y2, stream)
+        bitlogic_lut_forward_node(self.y1, n.conn2, n.theta2, self.y2, self.node, stream)
         mark("forward2")
         bitlogic_head_loss_ex(self.y2, self.labels, self.C, self.tau, self.loss, self.ws_head,
                               logits=self.logits, dY_grouped=self.dyg, stream=stream)
@@ -112,21 +117,22 @@ class TrainStep:
     def backward(self, stream=None, mark=_nomark):
         n = self.net
         co = self.csr_order
-        bitlogic_lut_backward_ex(self.y1, n.conn2, n.theta2, self.dth2, dY=self.dyg,
-                                 dy_group=n.w2 // self.C, edge_terms=self.edges2,
-                                 edge_pos=n.pos2 if co else None, stream=stream)
+        nd = self.node
+        bitlogic_lut_backward_node(self.y1, n.conn2, n.theta2, self.dth2, nd, dY=self.dyg,
+                                   dy_group=n.w2 // self.C, edge_terms=self.edges2,
+                                   edge_pos=n.pos2 if co else None, stream=stream)
         mark("backward2")
         pos1 = n.pos1 if (co and self.edges1 is not None) else None
         edge2 = None if co else n.edge2
         if self.fuse_dy1:
-            bitlogic_lut_backward_ex(self.bits, n.conn1, n.theta1, self.dth1, up_terms=self.edges2,
-                                     up_off=n.off2, up_edge=edge2, edge_terms=self.edges1,
-                                     edge_pos=pos1, dY_out=self.dy1, stream=stream)
+            bitlogic_lut_backward_node(self.bits, n.conn1, n.theta1, self.dth1, nd, up_terms=self.edges2,
+                                       up_off=n.off2, up_edge=edge2, edge_terms=self.edges1,
+                                       edge_pos=pos1, dY_out=self.dy1, stream=stream)
         else:
             bitlogic_csr_reduce(self.edges2, n.off2, edge2, self.dy1, stream)
             mark("csr2")
-            bitlogic_lut_backward_ex(self.bits, n.conn1, n.theta1, self.dth1, dY=self.dy1,
-                                     edge_terms=self.edges1, edge_pos=pos1, stream=stream)
+            bitlogic_lut_backward_node(self.bits, n.conn1, n.theta1, self.dth1, nd, dY=self.dy1,
+                                       edge_terms=self.edges1, edge_pos=pos1, stream=stream)
         mark("backward1")
         if self.dbits is not None:
             bitlogic_csr_reduce(self.edges1, n.off1, None if co else n.edge1, self.dbits, stream)

@@ -68,12 +68,22 @@ WORKLOADS = {
     # MNIST-shaped training throughput, 8000 x 8000, k=6 (and k=2)
     "mnist": Workload("mnist", 1024, 784, 10, 40.0, (64, 128, 192), (8000, 8000), 6, 20.0),
     "mnist_k2": Workload("mnist_k2", 1024, 784, 10, 40.0, (64, 128, 192), (8000, 8000), 2, 20.0),
+    # fan-in 4, the rank the paper pins for its method comparisons (App. C.2)
+    "mnist_k4": Workload("mnist_k4", 1024, 784, 10, 40.0, (64, 128, 192), (8000, 8000), 4, 20.0),
     # CIFAR-10-shaped: 3072 features, 7 thresholds -> 21504 bits, 64000 x 64000
     "cifar10": Workload("cifar10", 1024, 3072, 10, 50.0, _even(32, 7), (64000, 64000), 6, 50.0),
     # CIFAR-100-shaped wide: 15 thresholds -> 46080 bits, 128000 x 128000
     "cifar100": Workload("cifar100", 2048, 3072, 100, 50.0, _even(16, 15), (128000, 128000), 6, 100.0),
     # hard bit-packed inference on the CIFAR-10-shaped network, 2^22 samples
     "hard_cifar10": Workload("hard_cifar10", 1 << 22, 3072, 10, 50.0, _even(32, 7), (64000, 64000), 6, 50.0),
+    # the shape of the paper's deployed MNIST network (§5 hardware
+    # evaluation: w = 4000 per layer, n = 4, b = 4 thresholds -> 3136 bits,
+    # popcount head 10 x 400) at its GPU batch of 1024 and at 2^22 samples;
+    # equispaced thresholds stand in for the fitted quantile ones (the
+    # throughput does not depend on the threshold values)
+    "hard_mnist_w4000": Workload("hard_mnist_w4000", 1024, 784, 10, 40.0, _even(51, 4), (4000, 4000), 4, 40.0),
+    "hard_mnist_w4000_4m": Workload("hard_mnist_w4000_4m", 1 << 22, 784, 10, 40.0, _even(51, 4), (4000, 4000),
+                                    4, 40.0),
 }
 
 

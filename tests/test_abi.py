@@ -47,7 +47,7 @@ def test_python_binding_names_match_header():
 
 def test_status_strings_and_version():
     assert bl.bitlogic_status_string(0) == "ok"
-    for c in range(-1, -12, -1):
+    for c in range(-1, -13, -1):
         assert bl.bitlogic_status_string(c) != "unknown status"
     assert bl.bitlogic_version() >= 100
 
@@ -135,6 +135,15 @@ def test_host_validation_returns_before_any_launch():
     assert adamw(fake, fake, fake, fake, -1, 1, F(0.01), F(0.9), F(0.999), F(1e-8), F(0.0), None) == -2
     assert adamw(None, None, None, None, 0, 1, F(0.01), F(0.9), F(0.999), F(1e-8), F(0.0), None) == 0
     assert adamw(None, fake, fake, fake, 8, 1, F(0.01), F(0.9), F(0.999), F(1e-8), F(0.0), None) == -1
+    # node form: only soft (0) and straight-through (1)
+    fwd_node, bwd_node = lib.bitlogic_lut_forward_node, lib.bitlogic_lut_backward_node
+    assert fwd_node(fake, 8, 64, fake, fake, 4, 2, 2, fake, None) == -12
+    assert fwd_node(fake, 8, 64, fake, fake, 4, 2, -1, fake, None) == -12
+    assert fwd_node(fake, 8, 64, fake, fake, 4, 7, 1, fake, None) == -3
+    assert bwd_node(fake, 8, 64, fake, fake, 4, 2, 2, fake, 1, None, None, None, 0, fake, None, None,
+                    None, None) == -12
+    with pytest.raises(ValueError):
+        bl.bitlogic_lut_forward_node(None, None, None, None, node="hard")
 
 
 def test_workspace_queries():

@@ -103,6 +103,58 @@ def test_lut_backward(k, w_in, w, B):
     no_device_error()
 
 
+# ------------------------------------------ straight-through hard node --
+#
+# Forward and input gradient with the hard entries [theta > 0], dtheta with
+# the sigmoid slope (LightLUT's straight-through form, §4 node sweep).
+
+ST_ATOL = 1e-6   # fp32 evaluation of 0/1 tables on fractional inputs: absolute bound
+
+
+@pytest.mark.parametrize("k,w_in,w,B", SHAPES)
+@pytest.mark.parametrize("binary", [False, True])
+def test_lut_forward_st(k, w_in, w, B, binary):
+    X = (synth.binary_activations if binary else synth.uniform_activations)(w_in, B, seed=k + 2 * B)
+    conn = synth.connectivity(w, k, w_in, seed=w + 3)
+    theta = synth.table_logits(w, 1 << k, seed=k + 9)
+    theta[0, :] = 0.0                    # ties sample 0
+    Y = torch.full((w, B), np.nan, device="cuda")
+    bl.bitlogic_lut_forward_node(dev(X), dev(conn), dev(theta), Y, node="st")
+    want = oracle.lut_forward(X.astype(np.float64), conn, theta, "st")
+    if binary:   # integer arithmetic in fp32: the deployed table entries exactly
+        check_exact(Y.cpu().numpy().astype(np.float64), want, "Y")
+    else:
+        check_fwd(Y, want, "Y", atol=ST_ATOL)
+    no_device_error()
+
+
+@pytest.mark.parametrize("k,w_in,w,B", SHAPES)
+@pytest.mark.parametrize("binary", [False, True])
+def test_lut_backward_st(k, w_in, w, B, binary):
+    X = (synth.binary_activations if binary else synth.uniform_activations)(w_in, B, seed=k * 5 + B)
+    conn = synth.connectivity(w, k, w_in, seed=w + 4)
+    theta = synth.table_logits(w, 1 << k, seed=k + 11)
+    dY = synth.uniform_gradients(w, B, seed=B + 1, scale=1e-3)
+    off, edge = bl.bitlogic_build_csr(conn, w_in)
+    dth = torch.full((w, 1 << k), np.nan, device="cuda")
+    P = torch.full((w * k, B), np.nan, device="cuda")
+    bl.bitlogic_lut_backward_node(dev(X), dev(conn), dev(theta), dth, node="st", dY=dev(dY), edge_terms=P)
+    dX = torch.full((w_in, B), np.nan, device="cuda")
+    bl.bitlogic_csr_reduce(P, dev(off), dev(edge), dX)
+    wth, wdx = oracle.lut_backward(X.astype(np.float64), conn, theta, dY.astype(np.float64), node="st")
+    check_grad(dth, wth, "dtheta")
+    check_grad(dX, wdx, "dX")
+    # the soft node on the same inputs gives the same dtheta (the estimator
+    # keeps the sigmoid slope) but another dX
+    wth_s, _ = oracle.lut_backward(X.astype(np.float64), conn, theta, dY.astype(np.float64), want_dx=False)
+    np.testing.assert_allclose(wth, wth_s, rtol=1e-12, atol=0)
+    # without dX: the dtheta-only kernel serves both forms
+    dth2 = torch.full((w, 1 << k), np.nan, device="cuda")
+    bl.bitlogic_lut_backward_node(dev(X), dev(conn), dev(theta), dth2, node="st", dY=dev(dY))
+    check_grad(dth2, wth, "dtheta without dX")
+    no_device_error()
+
+
 @pytest.mark.parametrize("k,w_in,w,B,group", [(6, 300, 120, 256, 12), (6, 64, 40, 1024, 40), (3, 50, 30, 37, 5),
                                                (2, 9, 20, 100, 1), (1, 4, 6, 8, 3)])
 def test_backward_grouped_dy(k, w_in, w, B, group):

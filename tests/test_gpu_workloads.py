@@ -29,14 +29,14 @@ pytestmark = pytest.mark.gpu
 oracle.set_threads(os.cpu_count() or 1)
 
 
-def _step(wl, want_dx1, seed=0, k=None, keep_dy1=True, fuse_dy1=False, csr_order=True):
+def _step(wl, want_dx1, seed=0, k=None, keep_dy1=True, fuse_dy1=False, csr_order=True, node="soft"):
     if k is not None:
         wl = synth.Workload(wl.name, wl.batch, wl.d, wl.classes, wl.sigma, wl.thresholds, wl.widths, k, wl.tau)
     conn1, th1, conn2, th2 = synth.network(wl, seed)
     x, labels = synth.blob_batch(wl.batch, wl.d, wl.classes, wl.sigma, seed=seed + 7)
     net = Network(conn1, th1, conn2, th2, wl.w_in)
     st = TrainStep(net, wl.batch, wl.d, wl.thresholds, wl.classes, wl.tau, want_dx1=want_dx1,
-                   keep_dy1=keep_dy1, fuse_dy1=fuse_dy1, csr_order=csr_order)
+                   keep_dy1=keep_dy1, fuse_dy1=fuse_dy1, csr_order=csr_order, node=node)
     st.load(x.cuda(), labels.cuda())
     st.run()
     torch.cuda.synchronize()
@@ -51,11 +51,14 @@ def _check_grouped(st, dy2, wl):
     check_grad(st.dyg, rows[:, 0, :], "dY2 (per-class rows)")
 
 
-def _full_compare(wl, st, x, labels, params, want_dx1):
+def _full_compare(wl, st, x, labels, params, want_dx1, node="soft"):
     conn1, th1, conn2, th2 = params
     r = oracle.train_step(x, labels, wl.thresholds, conn1, th1, conn2, th2, wl.classes, wl.tau,
-                          want_dx1=want_dx1)
+                          want_dx1=want_dx1, node=node)
     check_exact(st.bits.cpu().numpy().astype(np.float64), r["bits"], "bits")
+    if node == "st":   # hard tables on binary inputs: every activation is a table entry
+        check_exact(st.y1.cpu().numpy().astype(np.float64), r["y1"], "y1")
+        check_exact(st.y2.cpu().numpy().astype(np.float64), r["y2"], "y2")
     check_fwd(st.y1, r["y1"], "y1")
     check_fwd(st.y2, r["y2"], "y2")
     check_fwd(st.logits, r["logits"], "logits")
@@ -73,10 +76,34 @@ def test_tiny_step_all_outputs():
     _full_compare(wl, st, x, labels, params, True)
 
 
-@pytest.mark.parametrize("k", [6, 2])
-def test_mnist_step_all_outputs(k):
-    wl, st, x, labels, params = _step(synth.WORKLOADS["mnist"], want_dx1=False, k=k)
-    _full_compare(wl, st, x, labels, params, False)
+@pytest.mark.parametrize("k,node", [(6, "soft"), (2, "soft"), (4, "soft"), (4, "st")])
+def test_mnist_step_all_outputs(k, node):
+    # k = 4 is the fan-in the paper pins for its comparisons (App. C.2)
+    wl, st, x, labels, params = _step(synth.WORKLOADS["mnist"], want_dx1=False, k=k, node=node)
+    _full_compare(wl, st, x, labels, params, False, node=node)
+
+
+def test_tiny_step_st_all_outputs():
+    # LightLUT straight-through: hard table samples forward, sigmoid-slope
+    # dtheta, input gradients of the hard-table forward (both layers)
+    wl, st, x, labels, params = _step(synth.WORKLOADS["tiny"], want_dx1=True, node="st")
+    _full_compare(wl, st, x, labels, params, True, node="st")
+
+
+@pytest.mark.parametrize("k", [6, 4])
+def test_st_forward_is_the_deployed_network(k):
+    # the straight-through forward of a batch equals the bit-packed hard
+    # path on the discretized tables (App. C.1): layer-2 outputs bit for bit,
+    # and head logits = popcounts / tau
+    wl, st, x, labels, params = _step(synth.WORKLOADS["tiny"], want_dx1=False, k=k, node="st")
+    hi = HardInfer(st.net, wl.batch, wl.d, wl.thresholds, wl.classes, keep_layer2=True)
+    hi.x = st.x
+    hi.binarize()
+    hi.run()
+    torch.cuda.synchronize()
+    check_exact(st.y2.cpu().numpy().astype(np.uint8), unpack_bits(hi.yp2, wl.batch), "y2 vs hard layer 2")
+    counts = hi.counts.cpu().numpy().astype(np.float64)
+    check_fwd(st.logits, counts / wl.tau, "logits vs popcounts / tau")
 
 
 def test_mnist_step_fused_layer1_gradient():
@@ -239,3 +266,24 @@ def test_tiny_training_steps_match_oracle_and_lower_the_loss():
     # the training accuracy climbs from chance
     assert np.mean(losses[-5:]) < 0.95 * np.mean(losses[:3]), losses
     assert accs[-1] >= 0.9, accs
+
+
+def test_tiny_straight_through_training_lowers_the_loss():
+    # the straight-through hard node trained with AdamW: its forward is the
+    # deployed network at every step, and its loss still falls (30 steps)
+    wl = synth.WORKLOADS["tiny"]
+    conn1, th1, conn2, th2 = synth.network(wl, 0)
+    net = Network(conn1, th1, conn2, th2, wl.w_in)
+    st = TrainStep(net, wl.batch, wl.d, wl.thresholds, wl.classes, wl.tau, node="st")
+    losses, accs = [], []
+    for step in range(1, 31):
+        x, labels = synth.blob_batch(wl.batch, wl.d, wl.classes, wl.sigma, seed=100 + step, means_seed=7)
+        st.load(x.cuda(), labels.cuda())
+        st.run()
+        st.update()
+        losses.append(float(st.loss.item()))
+        accs.append(float((st.logits.argmax(1).cpu() == labels.long()).float().mean()))
+        y2 = st.y2.cpu().numpy()
+        assert np.all((y2 == 0.0) | (y2 == 1.0))
+    assert np.mean(losses[-5:]) < 0.75 * np.mean(losses[:3]), losses
+    assert accs[-1] >= 0.75, accs
