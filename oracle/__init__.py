@@ -50,6 +50,7 @@ def _load():
                 "oracle_set_threads": ([ctypes.c_int], None),
                 "oracle_linear_thresholds": ([i32, P], None),
                 "oracle_encode_thermometer": ([P, i64, i32, P, i32, P], None),
+                "oracle_quantile_thresholds": ([P, i64, i32, P], None),
                 "oracle_lut_forward": ([P, i32, i64, P, P, i32, i32, i32, P], None),
                 "oracle_head_loss": ([P, i32, i64, i32, dbl, P, P, P, P], None),
                 "oracle_lut_backward": ([P, i32, i64, P, P, i32, i32, i32, P, P, P], None),
@@ -97,6 +98,17 @@ def encode_thermometer(x: np.ndarray, thr) -> np.ndarray:
     bits = np.empty((d * thr.size, B), np.float64)
     _load().oracle_encode_thermometer(_p(x), B, d, _p(thr), thr.size, _p(bits))
     return bits
+
+
+def quantile_thresholds(x: np.ndarray, b: int) -> np.ndarray:
+    """Quantile thermometer thresholds (uint8 [b]) fitted on the flattened
+    pixels of ``x`` (any shape, uint8, at least one value)."""
+    x = _c(np.asarray(x).reshape(-1), np.uint8)
+    if x.size == 0:
+        raise ValueError("no pixels to fit")
+    thr = np.empty(b, np.uint8)
+    _load().oracle_quantile_thresholds(_p(x), x.size, int(b), _p(thr))
+    return thr
 
 
 NODES = {"soft": 0, "st": 1}

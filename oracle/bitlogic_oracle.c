@@ -69,6 +69,32 @@ void oracle_encode_thermometer(const uint8_t* x, int64_t B, int32_t d,
                 bits[((int64_t)j * b + i) * B + s] = (x[s * d + j] > thr[i]) ? 1.0 : 0.0;
 }
 
+static int cmp_u8(const void* a, const void* b) {
+    return (int)*(const uint8_t*)a - (int)*(const uint8_t*)b;
+}
+
+/* Distributive (quantile) thermometer fit (§3 "Encoders and heads"; App. A
+ * "Initialization": fit once from the empirical pixel quantiles of the
+ * training split; App. B "MNIST-specific encoder collapse": quantiles of the
+ * globally flattened pixel distribution).  Reading: threshold i (1..b) is
+ * the quantile at level i/(b+1) with linear interpolation between order
+ * statistics, h = (n-1) i/(b+1), q = v[floor h] + (h - floor h)(v[floor h + 1]
+ * - v[floor h]) over the sorted pixels v; on integer pixels the encoder's
+ * strict compare pixel > q equals pixel > floor(q), so the stored threshold
+ * is floor(q), here in exact integer arithmetic.  n >= 1. */
+void oracle_quantile_thresholds(const uint8_t* x, int64_t n, int32_t b, uint8_t* thr) {
+    uint8_t* v = (uint8_t*)malloc((size_t)n);
+    memcpy(v, x, (size_t)n);
+    qsort(v, (size_t)n, 1, cmp_u8);
+    for (int32_t i = 1; i <= b; ++i) {
+        const int64_t num = (n - 1) * (int64_t)i;      /* h = num / (b + 1) */
+        const int64_t lo = num / (b + 1), rem = num % (b + 1);
+        const int64_t step = lo + 1 < n ? (int64_t)v[lo + 1] - (int64_t)v[lo] : 0;
+        thr[i - 1] = (uint8_t)((int64_t)v[lo] + (rem * step) / (b + 1));
+    }
+    free(v);
+}
+
 static double sigmoid(double z) { return 1.0 / (1.0 + exp(-z)); }
 
 /* Corner weight of table entry a for node inputs xs[0..k-1]:

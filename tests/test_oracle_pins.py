@@ -65,6 +65,60 @@ def test_encoder_unary_code_and_layout():
     assert bits[j, i, s] == float(x[s, j] > thr[i])
 
 
+# ------------------------------------------------ quantile thermometer fit --
+#
+# Distributive thermometer (§3, App. A, App. B): thresholds at the empirical
+# quantiles i/(b+1) of the flattened training pixels.
+
+def _np_quantile_thresholds(x, b):
+    # numpy's linear-interpolation quantile on the pixel scale, then the
+    # floor that the strict integer compare implies; the true fractional
+    # part is 0 or at least 1/(b+1), so a 1e-9 nudge only absorbs rounding
+    q = np.quantile(np.asarray(x, np.float64).reshape(-1), [i / (b + 1) for i in range(1, b + 1)],
+                    method="linear")
+    return np.floor(q + 1e-9).astype(np.int64), q
+
+
+@pytest.mark.parametrize("n,b,seed", [(1, 3, 0), (2, 4, 1), (3, 7, 2), (7, 15, 3), (1000, 4, 4),
+                                      (4097, 8, 5), (100003, 32, 6), (256, 1, 7)])
+def test_quantile_fit_matches_numpy(n, b, seed):
+    rng = np.random.default_rng(seed)
+    x = rng.integers(0, 256, size=n, dtype=np.uint8)
+    got = oracle.quantile_thresholds(x, b)
+    want, q = _np_quantile_thresholds(x, b)
+    np.testing.assert_array_equal(got.astype(np.int64), want)
+    # the stored integer threshold encodes exactly as the real quantile
+    v = np.arange(256)[:, None]
+    np.testing.assert_array_equal(v > got[None, :].astype(np.int64), v > q[None, :] + 1e-9)
+
+
+def test_quantile_fit_collapses_on_a_point_mass_at_zero():
+    # the MNIST observation of App. B: with a point mass at zero between the
+    # 7/9 and 8/9 quantiles, b = 4 gives four zero thresholds (every wire is
+    # pixel > 0) and b = 8 seven zeros and a last threshold above zero
+    rng = np.random.default_rng(11)
+    n = 200000
+    x = np.where(rng.random(n) < 0.83, 0, rng.integers(1, 256, size=n)).astype(np.uint8)
+    assert list(oracle.quantile_thresholds(x, 4)) == [0, 0, 0, 0]
+    t8 = oracle.quantile_thresholds(x, 8)
+    assert list(t8[:7]) == [0] * 7 and t8[7] > 0
+    # the collapsed encoder emits b identical wires per feature
+    bits = oracle.encode_thermometer(x[:64].reshape(8, 8), oracle.quantile_thresholds(x, 4))
+    w = bits.reshape(8, 4, 8)
+    assert np.all(w == w[:, :1, :])
+
+
+def test_quantile_fit_on_a_flat_histogram_is_near_linear():
+    # every value equally often: the quantile at level p is 255 p up to the
+    # one-step interpolation between neighbouring values
+    x = np.repeat(np.arange(256, dtype=np.uint8), 50)
+    for b in (3, 7, 15):
+        t = oracle.quantile_thresholds(x, b).astype(np.float64)
+        assert np.all(np.abs(t - 255.0 * np.arange(1, b + 1) / (b + 1)) <= 1.0)
+    # a constant image: every threshold is that constant
+    assert list(oracle.quantile_thresholds(np.full(99, 37, np.uint8), 5)) == [37] * 5
+
+
 # ----------------------------------------------------------- soft forward --
 
 def test_soft_node_golden_k2():
