@@ -9,7 +9,9 @@ binarization, encode + pack, hard layer 1, hard layer 2 with the fused
 popcount head and argmax).  ``value`` is the training throughput (samples
 per second through the fwd+bwd part); the hard part is reported in the
 ``hard`` object.  L2 is flushed between steps (a 512 MB write outside the
-timed events), so every step starts cold.
+timed events), so every step starts cold.  The timed loop replays the step as
+CUDA graphs captured once (no host work between launches); the per-call
+split comes from eager steps with an event after every call.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload mnist]
   python bench.py --impl reference ...   # the CPU oracle on the same workload
@@ -65,6 +67,8 @@ def parse_args():
                    help="LightLUT node form of the training step: soft, or straight-through hard")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-graph", action="store_true",
+                   help="time eager launches instead of CUDA-graph replays of the step")
     p.add_argument("--profile", action="store_true",
                    help="plain timed loop only (for ncu launch lists)")
     p.add_argument("--batch", type=int, default=0,
@@ -285,17 +289,52 @@ def run_ours(args):
     torch.cuda.synchronize()
 
     K = args.steps
-    marks = []          # per step: list of (name, event)
+    use_graph = not (args.no_graph or args.profile)
 
-    def new_step_marks():
-        lst = []
-        marks.append(lst)
+    def eager_steps(n):
+        """n eager steps with a CUDA event after every library call:
+        per-call durations and per-step (train, hard) sums."""
+        marks = []
+        for _ in range(n):
+            flush.fill_(1)
+            lst = []
+            marks.append(lst)
 
-        def mark(name):
-            ev = torch.cuda.Event(enable_timing=True)
-            ev.record(stream)
-            lst.append((name, ev))
-        return mark
+            def mark(name, lst=lst):
+                ev = torch.cuda.Event(enable_timing=True)
+                ev.record(stream)
+                lst.append((name, ev))
+            mark("start")
+            step(mark)
+        torch.cuda.synchronize()
+        calls, train_ms, hard_ms = {}, [], []
+        for lst in marks:
+            prev = lst[0][1]
+            t_train = 0.0
+            t_total = 0.0
+            for name, ev in lst[1:]:
+                dt = prev.elapsed_time(ev)
+                prev = ev
+                if name == "train_end":
+                    t_train = t_total
+                    continue
+                calls.setdefault(name, []).append(dt)
+                t_total += dt
+            train_ms.append(t_train)
+            hard_ms.append(t_total - t_train)
+        return calls, train_ms, hard_ms
+
+    if use_graph:
+        # the step as two CUDA graphs (training fwd+bwd; hard pass with its
+        # binarization), replayed in the timed loop
+        g_train = st.capture() if st is not None else None
+        g_hard = hi.capture(binarize=True)
+        for _ in range(3):
+            flush.fill_(1)
+            if g_train is not None:
+                g_train.replay()
+            g_hard.replay()
+        torch.cuda.synchronize()
 
     clock = ClockSampler(local)
     if world > 1:
@@ -303,36 +342,35 @@ def run_ours(args):
     torch.cuda.synchronize()
     clock.start()
     wall0 = time.perf_counter()
-    for _ in range(K):
-        flush.fill_(1)
-        mark = new_step_marks()
-        mark("start")
-        step(mark)
-    torch.cuda.synchronize()
+    if use_graph:
+        evs = []
+        for _ in range(K):
+            flush.fill_(1)
+            e = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+            e[0].record(stream)
+            if g_train is not None:
+                g_train.replay()
+            e[1].record(stream)
+            g_hard.replay()
+            e[2].record(stream)
+            evs.append(e)
+        torch.cuda.synchronize()
+        train_ms = [e[0].elapsed_time(e[1]) for e in evs]
+        hard_ms = [e[1].elapsed_time(e[2]) for e in evs]
+    else:
+        calls, train_ms, hard_ms = eager_steps(K)
     wall = time.perf_counter() - wall0
     if world > 1:
         torch.distributed.barrier()
     clocks = clock.stop()
     assert bl.bitlogic_device_error() == 0
-
-    # per-call durations
-    calls = {}
-    train_ms, hard_ms = [], []
-    for lst in marks:
-        prev = lst[0][1]
-        t_train = 0.0
-        t_total = 0.0
-        for name, ev in lst[1:]:
-            dt = prev.elapsed_time(ev)
-            prev = ev
-            if name == "train_end":
-                t_train = t_total
-                continue
-            calls.setdefault(name, []).append(dt)
-            t_total += dt
-        train_ms.append(t_train)
-        hard_ms.append(t_total - t_train)
     train_sum, hard_sum = max_over_ranks([sum(train_ms), sum(hard_ms)], "cuda")
+    eager_ms = None
+    if use_graph:
+        # per-call split (and the roofline kernel's duration) from eager steps
+        # with an event after every call, outside the timed loop
+        calls, tr_e, hd_e = eager_steps(max(3, min(K, 100)))
+        eager_ms = {"train": float(np.mean(tr_e)), "hard": float(np.mean(hd_e))}
 
     launches = K * (hi.kernels_per_binarize + hi.kernels_per_run)
     if st is not None:
@@ -391,6 +429,10 @@ def run_ours(args):
                      "ms_per_batch": ms_step_hard, "batch": B,
                      "includes": "binarize + encode/pack + 2 hard layers + popcount head + argmax"},
             "ms_per_step_total": ms_step_train + ms_step_hard,
+            "timing": ("CUDA-graph replays of the step (training fwd+bwd graph, hard-pass graph), CUDA events "
+                       "around each replay; per-call split from eager steps with an event after every call"
+                       if use_graph else "eager launches, CUDA events after every library call"),
+            **({"eager_ms_per_step": eager_ms} if eager_ms else {}),
             **({"context": PAPER_CONTEXT[wl.name]} if wl.name in PAPER_CONTEXT else {}),
             "calls": calls_out,
             "roofline": roof,
@@ -408,8 +450,10 @@ def run_ours(args):
                                    "algorithmic_bytes": 28 * n_par,
                                    "GB/s": 28 * n_par / (upd * 1e-3) / 1e9,
                                    "settings": "AdamW beta (0.9, 0.999), eps 1e-8, lr 0.01, wd 0"}
+    if not args.profile and rank == 0:
+        result["fit"] = time_quantile_fit(wl, flush)
     if not args.profile and not args.no_e2e:
-        e2e = run_e2e(args, st, hi, wl, B)
+        e2e = run_e2e(args, st, hi, wl, B, g_train if use_graph else None, g_hard if use_graph else None)
         if result is not None:
             result["e2e"] = e2e["train"] if st is not None else e2e["hard"]
             result["hard"]["e2e"] = e2e["hard"]
@@ -417,6 +461,37 @@ def run_ours(args):
         torch.distributed.barrier()
         torch.distributed.destroy_process_group()
     return result
+
+
+# training split sizes of the datasets the workloads stand in for
+SPLIT_SAMPLES = {784: 60000, 3072: 50000}
+
+
+def time_quantile_fit(wl, flush, iters: int = 20):
+    """The quantile thermometer fit's device pass (the pixel histogram) over a
+    training split of the workload's shape, L2 flushed before every call."""
+    import paper_2602_07400_gb300 as bl
+    n_samples = SPLIT_SAMPLES.get(wl.d, 50000)
+    x, _ = synth.blob_batch(n_samples, wl.d, wl.classes, wl.sigma, seed=5000, device="cuda")
+    hist = torch.zeros(256, dtype=torch.int64, device="cuda")
+    for _ in range(3):
+        bl.bitlogic_pixel_histogram(x, hist)
+    ms = []
+    for _ in range(iters):
+        flush.fill_(2)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        bl.bitlogic_pixel_histogram(x, hist)
+        e1.record()
+        ms.append((e0, e1))
+    torch.cuda.synchronize()
+    t = float(np.mean([a.elapsed_time(b) for a, b in ms]))
+    hbm, _, _ = peaks()
+    gbs = x.numel() / (t * 1e-3) / 1e9
+    thr = bl.bitlogic_quantile_thresholds(hist, wl.b)
+    return {"kernel": "pixel_histogram_kernel", "split": f"{n_samples} x {wl.d} uint8 (a training split of the "
+            f"workload's shape)", "ms": t, "GB/s": gbs, "frac_hbm": gbs / hbm,
+            "thresholds_b": [int(v) for v in thr]}
 
 
 def time_update(st, iters: int) -> float:
@@ -433,9 +508,18 @@ def time_update(st, iters: int) -> float:
     return e0.elapsed_time(e1) / iters
 
 
-def run_e2e(args, st, hi, wl, B):
+def run_e2e(args, st, hi, wl, B, g_train=None, g_hard=None):
     """The same metric end to end: pinned host inputs copied in, the step
-    run through the public API, the step's result copied out, every step."""
+    run through the public API (the captured graphs when given), the step's
+    result copied out, every step."""
+    train_run = g_train.replay if g_train is not None else st.run if st is not None else None
+
+    def hard_run():
+        if g_hard is not None:
+            g_hard.replay()
+        else:
+            hi.binarize()
+            hi.run()
     world, rank, _ = dist_env()
     x_host, lab_host = synth.blob_batch(B, wl.d, wl.classes, wl.sigma, seed=2000 + rank)
     x_host = x_host.pin_memory()
@@ -447,14 +531,14 @@ def run_e2e(args, st, hi, wl, B):
     if st is not None:
         for _ in range(3):
             st.load(x_host, lab_host, non_blocking=True)
-            st.run()
+            train_run()
             loss_host.copy_(st.loss, non_blocking=True)
         torch.cuda.synchronize()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record()
         for _ in range(K):
             st.load(x_host, lab_host, non_blocking=True)
-            st.run()
+            train_run()
             loss_host.copy_(st.loss, non_blocking=True)
         e1.record()
         torch.cuda.synchronize()
@@ -464,16 +548,14 @@ def run_e2e(args, st, hi, wl, B):
                         "d2h_bytes_per_step": 4}
     for _ in range(3):
         hi.x.copy_(x_host, non_blocking=True)
-        hi.binarize()
-        hi.run()
+        hard_run()
         pred_host.copy_(hi.pred, non_blocking=True)
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record()
     for _ in range(K):
         hi.x.copy_(x_host, non_blocking=True)
-        hi.binarize()
-        hi.run()
+        hard_run()
         pred_host.copy_(hi.pred, non_blocking=True)
     e1.record()
     torch.cuda.synchronize()

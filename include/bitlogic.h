@@ -80,6 +80,30 @@ int bitlogic_encode_thermometer(const uint8_t* x, int64_t B, int32_t d,
                                 const uint8_t* thr_host, int32_t b,
                                 float* bits, cudaStream_t stream);
 
+/* Distributive (quantile) thermometer fit (§3 "Encoders and heads"; App. A
+ * "Initialization": thresholds fit once from the empirical pixel quantiles
+ * of the training split, over the globally flattened pixels, App. B).  Two
+ * steps, so that a training split larger than device memory can be streamed
+ * through in pieces and the library never synchronizes:
+ *   bitlogic_pixel_histogram   device: hist[v] += number of bytes of x equal
+ *                              to v (x device uint8 [n], any alignment; hist
+ *                              device uint64 [256], zeroed by the caller
+ *                              before the first piece).  n == 0 is a no-op.
+ *   bitlogic_quantile_thresholds  host: from the finished histogram (copied
+ *                              to the host, hist_host uint64 [256]), threshold
+ *                              i = 1..b is the quantile at level i/(b+1) with
+ *                              linear interpolation between order statistics,
+ *                              floored to the integer that the encoder's
+ *                              strict compare needs (pixel > floor(q) equals
+ *                              pixel > q on integer pixels); exact integer
+ *                              arithmetic.  thr_host uint8 [b], ascending and
+ *                              possibly repeated (a point mass collapses
+ *                              neighbouring thresholds).  1 <= b <= 32
+ *                              (BITLOGIC_ERR_THRESH); an empty histogram gives
+ *                              BITLOGIC_ERR_SHAPE. */
+int bitlogic_pixel_histogram(const uint8_t* x, int64_t n, uint64_t* hist, cudaStream_t stream);
+int bitlogic_quantile_thresholds(const uint64_t* hist_host, int32_t b, uint8_t* thr_host);
+
 /* Soft LUT layer forward: one logic layer L_M(f_theta^(n)) of the paper's
  * Eq. (1) (§3), with the LightLUT node of §2 (Kronecker-indicator basis,
  * 2^k parameters per node) read as

@@ -30,7 +30,7 @@ __all__ = [
     "bitlogic_head_loss_workspace", "bitlogic_head_loss_noalloc",
     "bitlogic_head_loss", "bitlogic_binarize_tables", "bitlogic_pack_bits",
     "bitlogic_hard_forward", "bitlogic_build_csr", "bitlogic_csr_positions", "bitlogic_device_error",
-    "bitlogic_adamw_update", "bitlogic_lut_forward_node", "bitlogic_lut_backward_node", "NODE_FORMS",
+    "bitlogic_adamw_update", "bitlogic_pixel_histogram", "bitlogic_quantile_thresholds", "bitlogic_lut_forward_node", "bitlogic_lut_backward_node", "NODE_FORMS",
     "bitlogic_status_string", "bitlogic_version", "LIB_PATH",
 ]
 
@@ -61,6 +61,8 @@ _P, _I32, _I64, _F32, _SZ = (ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64,
 _SIGS = {
     "bitlogic_encode_thermometer": ([_P, _I64, _I32, _P, _I32, _P, _P], ctypes.c_int),
     "bitlogic_lut_forward": ([_P, _I32, _I64, _P, _P, _I32, _I32, _P, _P], ctypes.c_int),
+    "bitlogic_pixel_histogram": ([_P, _I64, _P, _P], ctypes.c_int),
+    "bitlogic_quantile_thresholds": ([_P, _I32, _P], ctypes.c_int),
     "bitlogic_lut_forward_node": ([_P, _I32, _I64, _P, _P, _I32, _I32, _I32, _P, _P], ctypes.c_int),
     "bitlogic_lut_backward_workspace": ([_I32, _I64, _I32, _I32, _I32], _SZ),
     "bitlogic_lut_backward": ([_P, _I32, _I64, _P, _P, _I32, _I32, _P, _P, _P, _P, _P,
@@ -158,6 +160,30 @@ def bitlogic_encode_thermometer(x: torch.Tensor, thresholds, bits: torch.Tensor,
     _need(bits, "bits", torch.float32, (d * b, B))
     _check("bitlogic_encode_thermometer", load().bitlogic_encode_thermometer(
         _ptr(x), B, d, buf, b, _ptr(bits), _stream(stream)))
+
+
+def bitlogic_pixel_histogram(x: torch.Tensor, hist: torch.Tensor, stream=None):
+    """hist (int64 [256] on the device, holding uint64 counts) += the value
+    counts of the bytes of x (uint8, any shape, contiguous)."""
+    if not isinstance(x, torch.Tensor) or x.dtype != torch.uint8 or not x.is_cuda or not x.is_contiguous():
+        raise TypeError("x must be a contiguous uint8 CUDA tensor")
+    _need(hist, "hist", torch.int64, (256,))
+    _check("bitlogic_pixel_histogram", load().bitlogic_pixel_histogram(
+        _ptr(x), x.numel(), _ptr(hist), _stream(stream)))
+
+
+def bitlogic_quantile_thresholds(hist, b: int) -> np.ndarray:
+    """Quantile thermometer thresholds (uint8 [b]) from a finished
+    histogram (256 counts, host array or tensor)."""
+    if isinstance(hist, torch.Tensor):
+        hist = hist.detach().cpu().numpy()
+    h = np.ascontiguousarray(np.asarray(hist).astype(np.uint64))
+    if h.shape != (256,):
+        raise ValueError("hist must hold 256 counts")
+    thr = np.empty(max(1, int(b)), np.uint8)
+    _check("bitlogic_quantile_thresholds", load().bitlogic_quantile_thresholds(
+        h.ctypes.data_as(ctypes.c_void_p), int(b), thr.ctypes.data_as(ctypes.c_void_p)))
+    return thr[:b]
 
 
 def bitlogic_lut_forward(X: torch.Tensor, conn: torch.Tensor, theta: torch.Tensor,

@@ -7,7 +7,8 @@ cross-entropy, two LUT backwards.  ``HardInfer`` runs the hard bit-packed
 evaluation (App. C.1): binarize tables, encode + pack, hard layer 1, hard
 layer 2 with the fused popcount head and argmax.  Buffers are allocated once
 (torch provides the device memory); every step only enqueues library calls
-on the current stream, so a step can be replayed or captured in a CUDA graph.
+on the current stream, so a step can be captured once as a CUDA graph and
+replayed (``capture``), which removes the host work between the launches.
 """
 from __future__ import annotations
 
@@ -17,7 +18,7 @@ import numpy as np
 import torch
 
 from . import (NODE_FORMS, bitlogic_adamw_update, bitlogic_binarize_tables, bitlogic_build_csr,
-               bitlogic_csr_positions, bitlogic_csr_reduce,
+               bitlogic_csr_positions, bitlogic_csr_reduce, bitlogic_pixel_histogram, bitlogic_quantile_thresholds,
                bitlogic_encode_thermometer, bitlogic_hard_forward, bitlogic_head_loss_ex,
                bitlogic_head_loss_workspace, bitlogic_lut_backward_node, bitlogic_lut_forward_node,
                bitlogic_pack_bits)
@@ -25,6 +26,36 @@ from . import (NODE_FORMS, bitlogic_adamw_update, bitlogic_binarize_tables, bitl
 
 def _nomark(name: str) -> None:
     return None
+
+
+def fit_quantile_thresholds(batches, b: int, stream=None) -> list:
+    """Quantile thermometer thresholds fitted on the pixels of every batch
+    (uint8 CUDA tensors, e.g. the training split in pieces): one device
+    histogram over all of them, read back once."""
+    hist = None
+    for x in batches:
+        if hist is None:
+            hist = torch.zeros(256, dtype=torch.int64, device=x.device)
+        bitlogic_pixel_histogram(x, hist, stream)
+    if hist is None:
+        raise ValueError("no batches to fit")
+    return [int(t) for t in bitlogic_quantile_thresholds(hist, b)]
+
+
+def capture_graph(fn) -> torch.cuda.CUDAGraph:
+    """Record ``fn()`` (library calls on the current stream) as a CUDA graph:
+    one warm-up call on a side stream first (lazy set-up such as kernel
+    attributes happens outside the capture), then the captured call.  Replay
+    with ``graph.replay()``; the graph stays bound to the buffers ``fn`` used."""
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        fn()
+    torch.cuda.current_stream().wait_stream(side)
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        fn()
+    return graph
 
 
 class Network:
@@ -142,6 +173,11 @@ class TrainStep:
         self.forward(stream, mark)
         self.backward(stream, mark)
 
+    def capture(self) -> torch.cuda.CUDAGraph:
+        """One run() (forward + backward) as a CUDA graph: a replay launches
+        the same kernels with no host work between them."""
+        return capture_graph(self.run)
+
     def update(self, lr: float = 0.01, betas=(0.9, 0.999), eps: float = 1e-8,
                weight_decay: float = 0.0, stream=None, mark=_nomark):
         """AdamW step on both layers' table logits from the last backward
@@ -198,6 +234,15 @@ class HardInfer:
         bitlogic_hard_forward(self.yp1, self.N, n.conn2, self.table2, yp=self.yp2, C=self.C,
                               counts=self.counts, pred=self.pred, stream=stream)
         mark("hard2")
+
+    def capture(self, binarize: bool = True) -> torch.cuda.CUDAGraph:
+        """One hard pass (with the table binarization when ``binarize``) as a
+        CUDA graph."""
+        def one():
+            if binarize:
+                self.binarize()
+            self.run()
+        return capture_graph(one)
 
     # kernels: binarize 2; pack 1, layer 1, layer 2 with head, argmax
     kernels_per_binarize = 2

@@ -135,6 +135,11 @@ def test_host_validation_returns_before_any_launch():
     assert adamw(fake, fake, fake, fake, -1, 1, F(0.01), F(0.9), F(0.999), F(1e-8), F(0.0), None) == -2
     assert adamw(None, None, None, None, 0, 1, F(0.01), F(0.9), F(0.999), F(1e-8), F(0.0), None) == 0
     assert adamw(None, fake, fake, fake, 8, 1, F(0.01), F(0.9), F(0.999), F(1e-8), F(0.0), None) == -1
+    # pixel histogram: negative size, NULL with bytes to count; n == 0 is a no-op
+    assert lib.bitlogic_pixel_histogram(fake, -1, fake, None) == -2
+    assert lib.bitlogic_pixel_histogram(None, 5, fake, None) == -1
+    assert lib.bitlogic_pixel_histogram(fake, 5, None, None) == -1
+    assert lib.bitlogic_pixel_histogram(None, 0, None, None) == 0
     # node form: only soft (0) and straight-through (1)
     fwd_node, bwd_node = lib.bitlogic_lut_forward_node, lib.bitlogic_lut_backward_node
     assert fwd_node(fake, 8, 64, fake, fake, 4, 2, 2, fake, None) == -12
@@ -144,6 +149,27 @@ def test_host_validation_returns_before_any_launch():
                     None, None) == -12
     with pytest.raises(ValueError):
         bl.bitlogic_lut_forward_node(None, None, None, None, node="hard")
+
+
+@pytest.mark.parametrize("n,b,seed", [(1, 1, 0), (5, 4, 1), (1000, 8, 2), (65537, 32, 3), (300, 15, 4)])
+def test_quantile_thresholds_from_a_histogram_match_the_oracle(n, b, seed):
+    # host-only step of the quantile fit: thresholds from 256 counts
+    import oracle
+    rng = np.random.default_rng(seed)
+    x = rng.integers(0, 256, size=n, dtype=np.uint8)
+    if seed % 2:
+        x[rng.random(n) < 0.8] = 0               # a point mass, as in digit images
+    hist = np.bincount(x, minlength=256).astype(np.uint64)
+    np.testing.assert_array_equal(bl.bitlogic_quantile_thresholds(hist, b), oracle.quantile_thresholds(x, b))
+
+
+def test_quantile_thresholds_rejects_bad_input():
+    with pytest.raises(bl.BitLogicError):
+        bl.bitlogic_quantile_thresholds(np.zeros(256, np.uint64), 4)    # empty
+    with pytest.raises(bl.BitLogicError):
+        bl.bitlogic_quantile_thresholds(np.ones(256, np.uint64), 33)    # b > 32
+    with pytest.raises(bl.BitLogicError):
+        bl.bitlogic_quantile_thresholds(np.ones(256, np.uint64), 0)
 
 
 def test_workspace_queries():

@@ -41,6 +41,50 @@ def test_encode_thermometer(B, d, b):
     no_device_error()
 
 
+# ------------------------------------------------ quantile thermometer fit --
+
+@pytest.mark.parametrize("n,offset,skew", [(1, 0, False), (15, 3, False), (16, 0, True), (17, 1, True),
+                                           (4095, 7, False), (100003, 0, True), ((1 << 22) + 5, 9, True)])
+def test_pixel_histogram_and_quantile_fit(n, offset, skew):
+    rng = np.random.default_rng(n + offset)
+    x = rng.integers(0, 256, size=n, dtype=np.uint8)
+    if skew:   # a point mass at zero, as in digit images
+        x[rng.random(n) < 0.85] = 0
+    buf = torch.zeros(n + offset, dtype=torch.uint8, device="cuda")
+    buf[offset:] = dev(x)
+    view = buf[offset:]                        # offset bytes into the allocation
+    hist = torch.zeros(256, dtype=torch.int64, device="cuda")
+    bl.bitlogic_pixel_histogram(view, hist)
+    want = np.bincount(x, minlength=256)
+    check_exact(hist.cpu().numpy(), want, "histogram")
+    bl.bitlogic_pixel_histogram(view, hist)   # counts accumulate
+    check_exact(hist.cpu().numpy(), 2 * want, "histogram, two passes")
+    for b in (1, 4, 8, 15, 32):
+        got = bl.bitlogic_quantile_thresholds(hist, b)
+        check_exact(got, oracle.quantile_thresholds(np.concatenate([x, x]), b), f"thresholds b={b}")
+
+
+def test_quantile_fit_then_encode_mnist_shaped():
+    # fit on several batches of the MNIST-shaped blobs, then encode with the
+    # fitted thresholds (repeated ones included) through both encoders
+    from paper_2602_07400_gb300.pipeline import fit_quantile_thresholds
+    wl = synth.WORKLOADS["mnist"]
+    xs = [synth.blob_batch(2048, wl.d, wl.classes, wl.sigma, seed=50 + i, means_seed=3)[0] for i in range(3)]
+    for x in xs[:2]:
+        x[:, : wl.d // 2] = 0                  # a third of all pixels black: the lowest thresholds repeat
+    thr = fit_quantile_thresholds([x.cuda() for x in xs], 8)
+    allx = np.concatenate([x.numpy() for x in xs])
+    assert thr == [int(t) for t in oracle.quantile_thresholds(allx, 8)]
+    assert thr[0] == thr[1] == 0
+    x = xs[0][:300].numpy()
+    bits = torch.empty(wl.d * 8, 300, device="cuda")
+    bl.bitlogic_encode_thermometer(dev(x), thr, bits)
+    check_exact(bits.cpu().numpy().astype(np.float64), oracle.encode_thermometer(x, thr), "bits")
+    xp = torch.empty(wl.d * 8, (300 + 31) // 32, dtype=torch.int32, device="cuda")
+    bl.bitlogic_pack_bits(dev(x), thr, xp)
+    check_exact(xp.cpu().numpy().view(np.uint32), oracle.pack_bits(x, thr), "packed bits")
+
+
 # ----------------------------------------------------------- soft forward --
 
 SHAPES = [  # (k, w_in, w, B)

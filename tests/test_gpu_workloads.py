@@ -134,6 +134,41 @@ def test_mnist_bench_configuration_matches():
         check_exact(getattr(b, name).cpu().numpy(), getattr(a, name).cpu().numpy(), name)
 
 
+def test_graph_replay_matches_eager_launches():
+    # the step captured once as CUDA graphs and replayed on new inputs gives
+    # the eager launches' results bit for bit (training step and hard pass)
+    wl = synth.WORKLOADS["tiny"]
+    conn1, th1, conn2, th2 = synth.network(wl, 0)
+    net = Network(conn1, th1, conn2, th2, wl.w_in)
+    st = TrainStep(net, wl.batch, wl.d, wl.thresholds, wl.classes, wl.tau, want_dx1=True)
+    hi = HardInfer(net, wl.batch, wl.d, wl.thresholds, wl.classes)
+    hi.x = st.x
+    x, labels = synth.blob_batch(wl.batch, wl.d, wl.classes, wl.sigma, seed=21)
+    st.load(x.cuda(), labels.cuda())
+    g_train, g_hard = st.capture(), hi.capture(binarize=True)
+    x2, labels2 = synth.blob_batch(wl.batch, wl.d, wl.classes, wl.sigma, seed=22)
+    st.load(x2.cuda(), labels2.cuda())
+    g_train.replay()
+    g_hard.replay()
+    torch.cuda.synchronize()
+    names = ("y1", "y2", "logits", "loss", "dyg", "dth1", "dth2", "dbits")
+    got = {n: getattr(st, n).clone() for n in names}
+    got_pred, got_counts = hi.pred.clone(), hi.counts.clone()
+    st.run()
+    hi.binarize()
+    hi.run()
+    torch.cuda.synchronize()
+    for n in names:
+        check_exact(got[n].cpu().numpy(), getattr(st, n).cpu().numpy(), n)
+    check_exact(got_pred.cpu().numpy(), hi.pred.cpu().numpy(), "pred")
+    check_exact(got_counts.cpu().numpy(), hi.counts.cpu().numpy(), "counts")
+    # and the replayed step is the oracle's step on the new batch
+    r = oracle.train_step(x2.numpy(), labels2.numpy(), wl.thresholds, conn1, th1, conn2, th2, wl.classes,
+                          wl.tau, want_dx1=True)
+    check_fwd(got["loss"], np.array([r["loss"]]), "loss")
+    check_grad(got["dth1"], r["dth1"], "dtheta1")
+
+
 def _sampled_compare(wl, st, x, labels, params, n_nodes=96, seed=0):
     conn1, th1, conn2, th2 = params
     bits = oracle.encode_thermometer(x, wl.thresholds)
