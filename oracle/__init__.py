@@ -51,6 +51,9 @@ def _load():
                 "oracle_linear_thresholds": ([i32, P], None),
                 "oracle_encode_thermometer": ([P, i64, i32, P, i32, P], None),
                 "oracle_quantile_thresholds": ([P, i64, i32, P], None),
+                "oracle_route_forward": ([P, i32, i64, P, P, i64, i32, P, P], None),
+                "oracle_route_backward": ([P, i32, i64, P, P, i64, i32, P, P, P], None),
+                "oracle_route_snap": ([P, P, i64, i32, P], None),
                 "oracle_lut_forward": ([P, i32, i64, P, P, i32, i32, i32, P], None),
                 "oracle_head_loss": ([P, i32, i64, i32, dbl, P, P, P, P], None),
                 "oracle_lut_backward": ([P, i32, i64, P, P, i32, i32, i32, P, P, P], None),
@@ -164,6 +167,45 @@ def lut_backward(X: np.ndarray, conn: np.ndarray, theta: np.ndarray, dY: np.ndar
     return dtheta, dX
 
 
+def route_forward(X: np.ndarray, cand: np.ndarray, r: np.ndarray):
+    """Learnable routing forward.  X float64 [w_in, B]; cand int32 [slots, Kc];
+    r float32 [slots, Kc] -> (Xr float64 [slots, B], prob float64 [slots, Kc])."""
+    X = _c(X, np.float64)
+    cand = _c(cand, np.int32)
+    r = _c(r, np.float32)
+    w_in, B = X.shape
+    n, Kc = cand.shape
+    assert r.shape == (n, Kc) and Kc <= 64
+    Xr = np.empty((n, B), np.float64)
+    prob = np.empty((n, Kc), np.float64)
+    _load().oracle_route_forward(_p(X), w_in, B, _p(cand), _p(r), n, Kc, _p(Xr), _p(prob))
+    return Xr, prob
+
+
+def route_backward(X: np.ndarray, cand: np.ndarray, r: np.ndarray, G: np.ndarray, want_dx: bool = True):
+    """-> (dr float64 [slots, Kc], dX float64 [w_in, B] or None)."""
+    X = _c(X, np.float64)
+    cand = _c(cand, np.int32)
+    r = _c(r, np.float32)
+    G = _c(G, np.float64)
+    w_in, B = X.shape
+    n, Kc = cand.shape
+    dr = np.empty((n, Kc), np.float64)
+    dX = np.empty((w_in, B), np.float64) if want_dx else None
+    _load().oracle_route_backward(_p(X), w_in, B, _p(cand), _p(r), n, Kc, _p(G), _p(dr), _p(dX))
+    return dr, dX
+
+
+def route_snap(cand: np.ndarray, r: np.ndarray) -> np.ndarray:
+    """int32 [slots]: each slot's most likely candidate (first on ties)."""
+    cand = _c(cand, np.int32)
+    r = _c(r, np.float32)
+    n, Kc = cand.shape
+    conn = np.empty(n, np.int32)
+    _load().oracle_route_snap(_p(cand), _p(r), n, Kc, _p(conn))
+    return conn
+
+
 def binarize_tables(theta: np.ndarray) -> np.ndarray:
     theta = _c(theta, np.float32)
     w, K = theta.shape
@@ -232,6 +274,29 @@ def train_step(x: np.ndarray, labels: np.ndarray, thr, conn1, th1, conn2, th2,
     dth1, dbits = lut_backward(bits, conn1, th1, dy1, want_dx=want_dx1, node=node)
     return dict(bits=bits, y1=y1, y2=y2, logits=logits, loss=loss, dy2=dy2,
                 dth2=dth2, dy1=dy1, dth1=dth1, dbits=dbits)
+
+
+def routed_train_step(x: np.ndarray, labels: np.ndarray, thr, cand1, r1, th1, cand2, r2, th2,
+                      C: int, tau: float, node: str = "soft"):
+    """Encoder -> two routed LUT layers (routing, then the node over the
+    slot inputs) -> group-sum head + CE -> both backwards, through the
+    routing as well."""
+    w1, k1 = th1.shape[0], int(np.log2(th1.shape[1]))
+    w2, k2 = th2.shape[0], int(np.log2(th2.shape[1]))
+    id1 = np.arange(w1 * k1, dtype=np.int32).reshape(w1, k1)
+    id2 = np.arange(w2 * k2, dtype=np.int32).reshape(w2, k2)
+    bits = encode_thermometer(x, thr)
+    xr1, p1 = route_forward(bits, cand1, r1)
+    y1 = lut_forward(xr1, id1, th1, node)
+    xr2, p2 = route_forward(y1, cand2, r2)
+    y2 = lut_forward(xr2, id2, th2, node)
+    logits, loss, dy2 = head_loss(y2, labels, C, tau)
+    dth2, dxr2 = lut_backward(xr2, id2, th2, dy2, want_dx=True, node=node)
+    dr2, dy1 = route_backward(y1, cand2, r2, dxr2, want_dx=True)
+    dth1, dxr1 = lut_backward(xr1, id1, th1, dy1, want_dx=True, node=node)
+    dr1, _ = route_backward(bits, cand1, r1, dxr1, want_dx=False)
+    return dict(bits=bits, xr1=xr1, y1=y1, xr2=xr2, y2=y2, logits=logits, loss=loss, dy2=dy2,
+                dth2=dth2, dxr2=dxr2, dr2=dr2, dy1=dy1, dth1=dth1, dxr1=dxr1, dr1=dr1, p1=p1, p2=p2)
 
 
 def hard_infer(x: np.ndarray, thr, conn1, table1, conn2, table2, C: int):

@@ -233,6 +233,80 @@ void oracle_lut_backward(const double* X, int32_t w_in, int64_t B,
     free(tt);
 }
 
+/* Learnable routing (§3 "Connectivity is the main per-layer design choice":
+ * a per-slot candidate pool, a selection that is differentiable in training
+ * and snapped to a sparse mapping at discretization; App. A
+ * "Initialization": pools drawn uniformly, routing logits zero so the
+ * expected selection is uniform).  Slot e (e = j*k + i, n_slots = w*k) has
+ * candidates cand[e*Kc + m] and logits r[e*Kc + m], m < Kc; its input is the
+ * expected selection
+ *   p_e = softmax(r_e),  Xr[e][s] = sum_m p_e[m] X[cand[e][m]][s].
+ * prob (optional) receives p. */
+void oracle_route_forward(const double* X, int32_t w_in, int64_t B, const int32_t* cand,
+                          const float* r, int64_t n_slots, int32_t Kc, double* Xr, double* prob) {
+    (void)w_in;
+#pragma omp parallel for schedule(dynamic, 64)
+    for (int64_t e = 0; e < n_slots; ++e) {
+        double p[64], mx = -INFINITY, z = 0.0;
+        for (int32_t m = 0; m < Kc; ++m) if ((double)r[e * Kc + m] > mx) mx = (double)r[e * Kc + m];
+        for (int32_t m = 0; m < Kc; ++m) z += exp((double)r[e * Kc + m] - mx);
+        for (int32_t m = 0; m < Kc; ++m) p[m] = exp((double)r[e * Kc + m] - mx) / z;
+        if (prob) for (int32_t m = 0; m < Kc; ++m) prob[e * Kc + m] = p[m];
+        for (int64_t s = 0; s < B; ++s) {
+            double v = 0.0;
+            for (int32_t m = 0; m < Kc; ++m) v += p[m] * X[(int64_t)cand[e * Kc + m] * B + s];
+            Xr[e * B + s] = v;
+        }
+    }
+}
+
+/* Routing backward by the chain rule, G[e][s] = dL/dXr[e][s]:
+ *   dr[e][m]  = sum_s G[e][s] sum_m' (dp[m']/dr[m]) X[cand[e][m']][s],
+ *               dp[m']/dr[m] = p[m'] ([m' == m] - p[m])
+ *   dX[c][s] += p[m] G[e][s] for every (e, m) with cand[e][m] == c,
+ *               added in increasing (e, m) order (dX optional, overwritten). */
+void oracle_route_backward(const double* X, int32_t w_in, int64_t B, const int32_t* cand,
+                           const float* r, int64_t n_slots, int32_t Kc, const double* G,
+                           double* dr, double* dX) {
+    double* prob = (double*)malloc(sizeof(double) * (size_t)n_slots * (size_t)Kc);
+    double* Xr = (double*)malloc(sizeof(double) * (size_t)n_slots * (size_t)B);
+    oracle_route_forward(X, w_in, B, cand, r, n_slots, Kc, Xr, prob);
+    free(Xr);
+#pragma omp parallel for schedule(dynamic, 64)
+    for (int64_t e = 0; e < n_slots; ++e) {
+        const double* p = prob + e * Kc;
+        for (int32_t m = 0; m < Kc; ++m) {
+            double acc = 0.0;
+            for (int64_t s = 0; s < B; ++s) {
+                double dxr = 0.0;   /* dXr[e][s] / dr[m] */
+                for (int32_t q = 0; q < Kc; ++q)
+                    dxr += p[q] * ((q == m ? 1.0 : 0.0) - p[m]) * X[(int64_t)cand[e * Kc + q] * B + s];
+                acc += G[e * B + s] * dxr;
+            }
+            dr[e * Kc + m] = acc;
+        }
+    }
+    if (dX) {
+        memset(dX, 0, sizeof(double) * (size_t)w_in * (size_t)B);
+#pragma omp parallel for schedule(static)
+        for (int64_t s = 0; s < B; ++s)
+            for (int64_t e = 0; e < n_slots; ++e)
+                for (int32_t m = 0; m < Kc; ++m)
+                    dX[(int64_t)cand[e * Kc + m] * B + s] += prob[e * Kc + m] * G[e * B + s];
+    }
+    free(prob);
+}
+
+/* Discretization of learnable routing: each slot keeps its most likely
+ * candidate (the first one on ties). */
+void oracle_route_snap(const int32_t* cand, const float* r, int64_t n_slots, int32_t Kc, int32_t* conn) {
+    for (int64_t e = 0; e < n_slots; ++e) {
+        int32_t best = 0;
+        for (int32_t m = 1; m < Kc; ++m) if (r[e * Kc + m] > r[e * Kc + best]) best = m;
+        conn[e] = cand[e * Kc + best];
+    }
+}
+
 /* Table discretization (§3 "Nodes are parameterizations": every surrogate
  * discretizes to a 2^n-entry truth table; App. C.1 extracts it once per
  * layer): entry a is 1 exactly when theta_j[a] > 0, i.e. sigmoid > 1/2. */

@@ -133,6 +133,12 @@ def connectivity(w: int, k: int, w_in: int, seed: int) -> np.ndarray:
     return conn.astype(np.int32)
 
 
+def candidate_pools(slots: int, Kc: int, w_in: int, seed: int) -> np.ndarray:
+    """int32 [slots, Kc]: a uniformly drawn pool of Kc distinct inputs per
+    node slot (learnable routing's candidate-pool mask, App. A)."""
+    return connectivity(slots, Kc, w_in, seed)
+
+
 def table_logits(w: int, K: int, seed: int, scale: float = 1.0) -> np.ndarray:
     """float32 [w, K] ~ N(0, scale^2)."""
     rng = np.random.default_rng(seed)

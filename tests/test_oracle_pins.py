@@ -365,6 +365,97 @@ def test_st_k1_closed_form():
     np.testing.assert_allclose(dX, g, rtol=1e-14)
 
 
+# ------------------------------------------------------ learnable routing --
+#
+# Per-slot candidate pools with softmax routing logits (§3 "Connectivity",
+# App. A "Initialization"); the slot input is the expected selection.
+
+def test_route_zero_logits_average_the_pool():
+    # logits initialised to zero: the uniform expected selection
+    rng = np.random.default_rng(1)
+    X = rng.random((30, 7))
+    cand = synth.candidate_pools(12, 8, 30, seed=2)
+    Xr, p = oracle.route_forward(X, cand, np.zeros((12, 8), np.float32))
+    np.testing.assert_allclose(p, 1.0 / 8, rtol=1e-15)
+    np.testing.assert_allclose(Xr, X[cand].mean(axis=1), rtol=1e-14)
+
+
+def test_route_saturated_logits_select_one_candidate():
+    rng = np.random.default_rng(3)
+    X = rng.random((40, 9))
+    cand = synth.candidate_pools(10, 16, 40, seed=4)
+    r = np.zeros((10, 16), np.float32)
+    pick = rng.integers(0, 16, size=10)
+    r[np.arange(10), pick] = 60.0
+    Xr, _ = oracle.route_forward(X, cand, r)
+    np.testing.assert_allclose(Xr, X[cand[np.arange(10), pick]], rtol=0, atol=1e-24)
+    np.testing.assert_array_equal(oracle.route_snap(cand, r), cand[np.arange(10), pick])
+
+
+def test_route_snap_takes_the_first_maximum():
+    cand = np.array([[5, 6, 7, 8], [1, 2, 3, 4]], np.int32)
+    r = np.array([[0.5, 2.0, 2.0, -1.0], [-3.0, -3.0, -3.0, -3.0]], np.float32)
+    np.testing.assert_array_equal(oracle.route_snap(cand, r), [6, 1])
+
+
+@pytest.mark.parametrize("k,Kc", [(2, 4), (4, 16), (6, 8)])
+def test_routed_layer_matches_torch_autograd(k, Kc):
+    # routing then a soft node over the slot inputs, against torch autograd
+    # through torch.softmax, an index gather and the Shannon-expansion node
+    rng = np.random.default_rng(800 + k)
+    w_in, w, B = 50, 6, 5
+    X = rng.random((w_in, B))
+    cand = synth.candidate_pools(w * k, Kc, w_in, seed=k)
+    r = synth.table_logits(w * k, Kc, seed=k + 1)
+    theta = synth.table_logits(w, 1 << k, seed=k + 2)
+    dY = rng.standard_normal((w, B))
+    ident = np.arange(w * k, dtype=np.int32).reshape(w, k)
+    Xr, _ = oracle.route_forward(X, cand, r)
+    dth, G = oracle.lut_backward(Xr, ident, theta, dY)
+    dr, dX = oracle.route_backward(X, cand, r, G)
+    Xt = torch.tensor(X, requires_grad=True)
+    rt = torch.tensor(r.astype(np.float64), requires_grad=True)
+    tht = torch.tensor(theta.astype(np.float64), requires_grad=True)
+    P = torch.softmax(rt, dim=1)
+    Xrt = (P[:, :, None] * Xt[torch.as_tensor(cand, dtype=torch.long)]).sum(dim=1)
+    Y = _shannon_forward_torch(Xrt, ident, torch.sigmoid(tht))
+    (Y * torch.tensor(dY)).sum().backward()
+    np.testing.assert_allclose(Xr, Xrt.detach().numpy(), rtol=1e-13, atol=1e-15)
+    np.testing.assert_allclose(dth, tht.grad.numpy(), rtol=1e-11, atol=1e-15)
+    np.testing.assert_allclose(dr, rt.grad.numpy(), rtol=1e-10, atol=1e-14)
+    np.testing.assert_allclose(dX, Xt.grad.numpy(), rtol=1e-11, atol=1e-14)
+
+
+def test_route_finite_differences_and_gradient_mass():
+    rng = np.random.default_rng(21)
+    w_in, n, Kc, B = 20, 9, 6, 4
+    X = rng.random((w_in, B))
+    cand = synth.candidate_pools(n, Kc, w_in, seed=5)
+    r = synth.table_logits(n, Kc, seed=6)
+    G = rng.standard_normal((n, B))
+
+    def L(Xv, rv):
+        return float(np.sum(G * oracle.route_forward(Xv, cand, rv)[0]))
+
+    dr, dX = oracle.route_backward(X, cand, r, G)
+    for (e, m) in [(0, 0), (4, 5), (n - 1, 2)]:
+        rp, rm = r.copy(), r.copy()
+        rp[e, m] = np.float32(r[e, m] + np.float32(1e-2))
+        rm[e, m] = np.float32(r[e, m] - np.float32(1e-2))
+        fd = (L(X, rp) - L(X, rm)) / (float(rp[e, m]) - float(rm[e, m]))
+        assert dr[e, m] == pytest.approx(fd, rel=2e-5, abs=1e-9)
+    h = 1e-3
+    for (c, s) in [(cand[0, 0], 0), (cand[3, 2], 3), (w_in - 1, 1)]:
+        Xp, Xm = X.copy(), X.copy()
+        Xp[c, s] += h
+        Xm[c, s] -= h
+        assert dX[c, s] == pytest.approx((L(Xp, r) - L(Xm, r)) / (2 * h), rel=1e-9, abs=1e-12)
+    # the probabilities of a slot sum to one: the input gradient carries the
+    # slot gradients' total, and the logit gradients of a slot sum to zero
+    np.testing.assert_allclose(dX.sum(axis=0), G.sum(axis=0), rtol=1e-12)
+    np.testing.assert_allclose(dr.sum(axis=1), 0.0, atol=1e-13)
+
+
 # -------------------------------------------------------------------- head --
 
 def test_head_matches_torch_autograd():
