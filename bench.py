@@ -159,6 +159,36 @@ def job_rate(world: int, samples_per_rank_step: int, steps: int, max_ms: float) 
 
 # ------------------------------------------------------ work per call --
 
+def call_work_routed(wl, B):
+    """Work of the calls of a routed training step: the routing calls count
+    their HBM bytes (each slot's Kc candidate rows are gathered from the
+    layer input, which stays in L2, so the gathered bytes are not HBM
+    traffic) and one FMA per (candidate, sample); the LUT calls read the
+    slot rows through the identity connectivity."""
+    K, k, Kc = wl.K, wl.k, wl.Kc
+    w1, w2 = wl.widths
+    win, d, C = wl.w_in, wl.d, wl.classes
+    s1, s2 = w1 * k, w2 * k
+    f = 4
+    return {
+        "encode": (B * d + f * win * B, 0),
+        "route1": (f * (win * B + s1 * B + 2 * s1 * Kc), Kc * s1 * B),
+        "forward1": (f * (s1 * B + w1 * B + w1 * K + w1 * k), (2 * (K - 1) + k) * w1 * B),
+        "route2": (f * (w1 * B + s2 * B + 2 * s2 * Kc), Kc * s2 * B),
+        "forward2": (f * (s2 * B + w2 * B + w2 * K + w2 * k), (2 * (K - 1) + k) * w2 * B),
+        "head": (f * (w2 * B + 4 * B * C), 0),
+        "backward2": (f * (s2 * B + C * B + s2 * B + 2 * w2 * K + w2 * k), (4 * (K - 1) + K) * w2 * B),
+        "route_bwd2": (f * (w1 * B + 2 * s2 * B + w1 * B + 3 * s2 * Kc), 2 * Kc * s2 * B),
+        "backward1": (f * (s1 * B + w1 * B + s1 * B + 2 * w1 * K + w1 * k), (4 * (K - 1) + K) * w1 * B),
+        "route_bwd1": (f * (win * B + s1 * B + 2 * s1 * Kc), Kc * s1 * B),
+        "binarize": (f * (w1 * K + w2 * K) + 8 * (w1 + w2), 0),
+        "pack": (B * d + f * win * ((B + 31) // 32), 0),
+        "hard1": (f * (win * ((B + 31) // 32) + w1 * ((B + 31) // 32) + w1 * k) + 8 * w1,
+                  (K - 1) * w1 * ((B + 31) // 32)),
+        "hard2": (f * (w1 * ((B + 31) // 32) + w2 * k + B * C * 2 + B) + 8 * w2, (K - 1) * w2 * ((B + 31) // 32)),
+    }
+
+
 def call_work(wl, B, fuse_dy1=False):
     """Algorithmic work of each library call of one step on a batch of B:
     (bytes, fp32 or logic ops).  Ops follow the lerp-tree counts: forward
@@ -231,6 +261,8 @@ KERNEL_OF_CALL = {
     "backward1": "lut_backward_theta_kernel<k>", "csr2": "csr_reduce_kernel",
     "binarize": "binarize_kernel (x2)", "pack": "pack_bits_kernel", "hard1": "hard_layer_staged_kernel<k>",
     "hard2": "hard_head_staged_kernel<k> + argmax_kernel",
+    "route1": "route_forward_vec_kernel<KC>", "route2": "route_forward_vec_kernel<KC>",
+    "route_bwd2": "route_dr_kernel + route_dx_kernel", "route_bwd1": "route_dr_kernel<KC>",
 }
 
 
@@ -245,7 +277,7 @@ def dist_env():
 
 def run_ours(args):
     import paper_2602_07400_gb300 as bl
-    from paper_2602_07400_gb300.pipeline import HardInfer, Network, TrainStep
+    from paper_2602_07400_gb300.pipeline import HardInfer, Network, RoutedNetwork, RoutedTrainStep, TrainStep
 
     world, rank, local = dist_env()
     torch.cuda.set_device(local)
@@ -259,13 +291,20 @@ def run_ours(args):
                             wl.widths, wl.k, wl.tau)
     hard_only = wl.name.startswith("hard_")
     B = wl.batch
-    conn1, th1, conn2, th2 = synth.network(wl, seed=0)
-    net = Network(conn1, th1, conn2, th2, wl.w_in)
+    if wl.Kc:
+        rnet = RoutedNetwork(*synth.routed_network(wl, seed=0), wl.w_in)
+        net = rnet.snap()                # the hard pass evaluates the discretized network
+    else:
+        conn1, th1, conn2, th2 = synth.network(wl, seed=0)
+        net = Network(conn1, th1, conn2, th2, wl.w_in)
     x_gen, lab_gen = synth.blob_batch(B, wl.d, wl.classes, wl.sigma, seed=1000 + rank,
                                       device="cuda" if hard_only else "cpu")
     st = None
     if not hard_only:
-        st = TrainStep(net, B, wl.d, wl.thresholds, wl.classes, wl.tau, node=args.node)
+        if wl.Kc:
+            st = RoutedTrainStep(rnet, B, wl.d, wl.thresholds, wl.classes, wl.tau, node=args.node)
+        else:
+            st = TrainStep(net, B, wl.d, wl.thresholds, wl.classes, wl.tau, node=args.node)
         st.load(x_gen.cuda(), lab_gen.cuda())
     hi = HardInfer(net, B, wl.d, wl.thresholds, wl.classes)
     if st is not None:
@@ -379,12 +418,12 @@ def run_ours(args):
     result = None
     if rank == 0:
         hbm, sm_max, peak_kind = peaks()
-        work = call_work(wl, B, fuse_dy1=st.fuse_dy1 if st is not None else False)
+        work = call_work_routed(wl, B) if wl.Kc else call_work(wl, B, fuse_dy1=st.fuse_dy1 if st is not None else False)
         per_call_ms = {n: float(np.mean(v)) for n, v in calls.items()}
         ms_step_train = train_sum / K
         ms_step_hard = hard_sum / K
         # roofline of the dominant single-kernel call
-        single = {n: t for n, t in per_call_ms.items() if n not in ("head", "binarize", "hard2")}
+        single = {n: t for n, t in per_call_ms.items() if n not in ("head", "binarize", "hard2", "route_bwd2")}
         dom = max(single, key=single.get)
         byts, ops = work[dom]
         t_s = per_call_ms[dom] * 1e-3
@@ -422,6 +461,7 @@ def run_ours(args):
             "data": "synthetic (seeded class-conditional Gaussian blobs, MNIST/CIFAR shapes; random-init tables)",
             "config": {"workload": wl.name, "batch_per_gpu": B, "d": wl.d, "thresholds": list(wl.thresholds),
                        "widths": list(wl.widths), "k": wl.k, "classes": wl.classes, "tau": wl.tau,
+                       "routing": f"learnable, {wl.Kc} candidates per slot" if wl.Kc else "fixed (random-unique)",
                        "node": "LightLUT " + ("soft" if args.node == "soft" else "straight-through hard"),
                        "l2": "flushed between steps (512 MB write outside the timed events)",
                        "parallelism": f"dp{world} (independent batches, no collective)"},
@@ -446,7 +486,10 @@ def run_ours(args):
         upd = time_update(st, max(3, min(args.steps, 50)))
         if result is not None:
             n_par = int(st.net.theta1.numel() + st.net.theta2.numel())
-            result["optimizer"] = {"ms_per_update": upd, "kernel": "adamw_vec_kernel (x2)",
+            if wl.Kc:
+                n_par += int(st.net.r1.numel() + st.net.r2.numel())
+            result["optimizer"] = {"ms_per_update": upd,
+                                   "kernel": f"adamw_vec_kernel (x{4 if wl.Kc else 2})",
                                    "algorithmic_bytes": 28 * n_par,
                                    "GB/s": 28 * n_par / (upd * 1e-3) / 1e9,
                                    "settings": "AdamW beta (0.9, 0.999), eps 1e-8, lr 0.01, wd 0"}
@@ -569,8 +612,13 @@ def run_e2e(args, st, hi, wl, B, g_train=None, g_hard=None):
 
 def oracle_train_rate(wl, samples: int, seed: int = 0, node: str = "soft"):
     import oracle
-    conn1, th1, conn2, th2 = synth.network(wl, seed=0)
     x, lab = synth.blob_batch(samples, wl.d, wl.classes, wl.sigma, seed=3000 + seed)
+    if wl.Kc:
+        params = synth.routed_network(wl, seed=0)
+        t0 = time.perf_counter()
+        oracle.routed_train_step(x.numpy(), lab.numpy(), wl.thresholds, *params, wl.classes, wl.tau, node=node)
+        return samples / (time.perf_counter() - t0)
+    conn1, th1, conn2, th2 = synth.network(wl, seed=0)
     t0 = time.perf_counter()
     oracle.train_step(x.numpy(), lab.numpy(), wl.thresholds, conn1, th1, conn2, th2,
                       wl.classes, wl.tau, node=node)

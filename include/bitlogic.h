@@ -213,6 +213,40 @@ int bitlogic_lut_backward_node(const float* X, int32_t w_in, int64_t B,
                                float* dtheta, float* edge_terms, const int32_t* edge_pos,
                                float* dY_out, cudaStream_t stream);
 
+/* Learnable routing (§3 "Connectivity is the main per-layer design choice":
+ * a per-slot candidate pool whose selection is differentiable in training
+ * and snapped to a sparse mapping at discretization; App. A
+ * "Initialization": pools drawn uniformly, logits zero).  Slot e = j*k + i of
+ * a layer of w nodes (slots = w*k) has candidates cand[e][m] and logits
+ * r[e][m], m < Kc, 1 <= Kc <= 32:
+ *   p_e = softmax(r_e),   Xr[e][s] = sum_m p_e[m] X[cand[e][m]][s].
+ * The rows Xr [slots][B] are the layer's slot inputs: the LUT calls read
+ * them through the identity connectivity conn[j][i] = j*k + i, and the LUT
+ * backward's per-edge terms over them are G = dL/dXr.
+ *   X     device fp32 [w_in][B];   cand device int32 [slots][Kc] in [0, w_in)
+ *   r     device fp32 [slots][Kc]
+ *   Xr    device fp32 [slots][B], overwritten (may be NULL when B == 0)
+ *   prob  device fp32 [slots][Kc] or NULL: receives p
+ * bitlogic_route_backward, with G device fp32 [slots][B]:
+ *   dr[e][m] = p_e[m] (A_m - sum_m' p_e[m'] A_m'),  A_m = sum_s G[e][s] X[cand[e][m]][s]
+ *   (device fp32 [slots][Kc], overwritten; batch sums in a fixed order), and
+ *   when dX is not NULL
+ *   dX[c][s] = sum of prob[id] G[id / Kc][s] over the CSR positions of input
+ *   c in increasing order (csr_off/csr_edge from bitlogic_build_csr over cand
+ *   as a [slots][Kc] connectivity, so id = e*Kc + m; prob as written by
+ *   bitlogic_route_forward), device fp32 [w_in][B], overwritten.
+ * bitlogic_route_snap: conn[e] = cand[e][argmax_m r[e][m]] (first maximum),
+ *   device int32 [slots]: the fixed connectivity of the discretized layer.
+ * A candidate index outside [0, w_in) is read as 0 and raises the device flag. */
+int bitlogic_route_forward(const float* X, int32_t w_in, int64_t B, const int32_t* cand, const float* r,
+                           int32_t slots, int32_t Kc, float* Xr, float* prob, cudaStream_t stream);
+int bitlogic_route_backward(const float* X, int32_t w_in, int64_t B, const int32_t* cand, const float* r,
+                            int32_t slots, int32_t Kc, const float* G, float* dr, const float* prob,
+                            const int32_t* csr_off, const int32_t* csr_edge, float* dX,
+                            cudaStream_t stream);
+int bitlogic_route_snap(const int32_t* cand, const float* r, int32_t slots, int32_t Kc, int32_t* conn,
+                        cudaStream_t stream);
+
 /* Bytes of workspace bitlogic_head_loss needs. */
 size_t bitlogic_head_loss_workspace(int64_t B, int32_t C);
 

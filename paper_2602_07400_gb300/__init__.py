@@ -30,7 +30,8 @@ __all__ = [
     "bitlogic_head_loss_workspace", "bitlogic_head_loss_noalloc",
     "bitlogic_head_loss", "bitlogic_binarize_tables", "bitlogic_pack_bits",
     "bitlogic_hard_forward", "bitlogic_build_csr", "bitlogic_csr_positions", "bitlogic_device_error",
-    "bitlogic_adamw_update", "bitlogic_pixel_histogram", "bitlogic_quantile_thresholds", "bitlogic_lut_forward_node", "bitlogic_lut_backward_node", "NODE_FORMS",
+    "bitlogic_adamw_update", "bitlogic_route_forward", "bitlogic_route_backward", "bitlogic_route_snap",
+    "bitlogic_pixel_histogram", "bitlogic_quantile_thresholds", "bitlogic_lut_forward_node", "bitlogic_lut_backward_node", "NODE_FORMS",
     "bitlogic_status_string", "bitlogic_version", "LIB_PATH",
 ]
 
@@ -62,6 +63,9 @@ _SIGS = {
     "bitlogic_encode_thermometer": ([_P, _I64, _I32, _P, _I32, _P, _P], ctypes.c_int),
     "bitlogic_lut_forward": ([_P, _I32, _I64, _P, _P, _I32, _I32, _P, _P], ctypes.c_int),
     "bitlogic_pixel_histogram": ([_P, _I64, _P, _P], ctypes.c_int),
+    "bitlogic_route_forward": ([_P, _I32, _I64, _P, _P, _I32, _I32, _P, _P, _P], ctypes.c_int),
+    "bitlogic_route_backward": ([_P, _I32, _I64, _P, _P, _I32, _I32, _P, _P, _P, _P, _P, _P, _P], ctypes.c_int),
+    "bitlogic_route_snap": ([_P, _P, _I32, _I32, _P, _P], ctypes.c_int),
     "bitlogic_quantile_thresholds": ([_P, _I32, _P], ctypes.c_int),
     "bitlogic_lut_forward_node": ([_P, _I32, _I64, _P, _P, _I32, _I32, _I32, _P, _P], ctypes.c_int),
     "bitlogic_lut_backward_workspace": ([_I32, _I64, _I32, _I32, _I32], _SZ),
@@ -160,6 +164,55 @@ def bitlogic_encode_thermometer(x: torch.Tensor, thresholds, bits: torch.Tensor,
     _need(bits, "bits", torch.float32, (d * b, B))
     _check("bitlogic_encode_thermometer", load().bitlogic_encode_thermometer(
         _ptr(x), B, d, buf, b, _ptr(bits), _stream(stream)))
+
+
+def bitlogic_route_forward(X: torch.Tensor, cand: torch.Tensor, r: torch.Tensor, Xr: torch.Tensor,
+                           prob: Optional[torch.Tensor] = None, stream=None):
+    """Slot inputs of learnable routing: cand int32 [slots, Kc], r fp32
+    [slots, Kc] -> Xr fp32 [slots, B] (and the probabilities into prob)."""
+    w_in, B = X.shape
+    slots, Kc = cand.shape
+    _need(X, "X", torch.float32, (w_in, B))
+    _need(cand, "cand", torch.int32, (slots, Kc))
+    _need(r, "r", torch.float32, (slots, Kc))
+    _need(Xr, "Xr", torch.float32, (slots, B))
+    if prob is not None:
+        _need(prob, "prob", torch.float32, (slots, Kc))
+    _check("bitlogic_route_forward", load().bitlogic_route_forward(
+        _ptr(X), w_in, B, _ptr(cand), _ptr(r), slots, Kc, _ptr(Xr), _ptr(prob), _stream(stream)))
+
+
+def bitlogic_route_backward(X: torch.Tensor, cand: torch.Tensor, r: torch.Tensor, G: torch.Tensor,
+                            dr: torch.Tensor, prob: Optional[torch.Tensor] = None,
+                            csr_off: Optional[torch.Tensor] = None, csr_edge: Optional[torch.Tensor] = None,
+                            dX: Optional[torch.Tensor] = None, stream=None):
+    """dr from the slot-input gradient G; dX (with prob and the candidate
+    CSR map) when given."""
+    w_in, B = X.shape
+    slots, Kc = cand.shape
+    _need(X, "X", torch.float32, (w_in, B))
+    _need(cand, "cand", torch.int32, (slots, Kc))
+    _need(r, "r", torch.float32, (slots, Kc))
+    _need(G, "G", torch.float32, (slots, B))
+    _need(dr, "dr", torch.float32, (slots, Kc))
+    if dX is not None:
+        _need(dX, "dX", torch.float32, (w_in, B))
+        _need(prob, "prob", torch.float32, (slots, Kc))
+        _need(csr_off, "csr_off", torch.int32, (w_in + 1,))
+        _need(csr_edge, "csr_edge", torch.int32, (slots * Kc,))
+    _check("bitlogic_route_backward", load().bitlogic_route_backward(
+        _ptr(X), w_in, B, _ptr(cand), _ptr(r), slots, Kc, _ptr(G), _ptr(dr), _ptr(prob), _ptr(csr_off),
+        _ptr(csr_edge), _ptr(dX), _stream(stream)))
+
+
+def bitlogic_route_snap(cand: torch.Tensor, r: torch.Tensor, conn: torch.Tensor, stream=None):
+    """conn int32 [slots]: each slot's most likely candidate (first on ties)."""
+    slots, Kc = cand.shape
+    _need(cand, "cand", torch.int32, (slots, Kc))
+    _need(r, "r", torch.float32, (slots, Kc))
+    _need(conn, "conn", torch.int32, (slots,))
+    _check("bitlogic_route_snap", load().bitlogic_route_snap(
+        _ptr(cand), _ptr(r), slots, Kc, _ptr(conn), _stream(stream)))
 
 
 def bitlogic_pixel_histogram(x: torch.Tensor, hist: torch.Tensor, stream=None):

@@ -21,7 +21,7 @@ from . import (NODE_FORMS, bitlogic_adamw_update, bitlogic_binarize_tables, bitl
                bitlogic_csr_positions, bitlogic_csr_reduce, bitlogic_pixel_histogram, bitlogic_quantile_thresholds,
                bitlogic_encode_thermometer, bitlogic_hard_forward, bitlogic_head_loss_ex,
                bitlogic_head_loss_workspace, bitlogic_lut_backward_node, bitlogic_lut_forward_node,
-               bitlogic_pack_bits)
+               bitlogic_pack_bits, bitlogic_route_backward, bitlogic_route_forward, bitlogic_route_snap)
 
 
 def _nomark(name: str) -> None:
@@ -201,6 +201,136 @@ class TrainStep:
     @property
     def kernels_per_run(self) -> int:
         return 8 + (0 if self.fuse_dy1 else 1) + (1 if self.dbits is not None else 0)
+
+
+class RoutedNetwork:
+    """A two-layer LUT network with learnable routing (§3 "Connectivity"):
+    per node slot a candidate pool (int32 [w*k, Kc]) and routing logits
+    (fp32 [w*k, Kc], zero at initialisation), plus the table logits.  The
+    nodes read their slot inputs through the identity connectivity."""
+
+    def __init__(self, cand1: np.ndarray, r1: np.ndarray, theta1: np.ndarray, cand2: np.ndarray,
+                 r2: np.ndarray, theta2: np.ndarray, w_in: int, device="cuda"):
+        dev = torch.device(device)
+        self.w_in = int(w_in)
+        self.w1, K1 = theta1.shape
+        self.w2, K2 = theta2.shape
+        self.k1, self.k2 = K1.bit_length() - 1, K2.bit_length() - 1
+        self.Kc = cand1.shape[1]
+        assert cand1.shape == (self.w1 * self.k1, self.Kc) and cand2.shape == (self.w2 * self.k2, self.Kc)
+        t = lambda a, dt: torch.from_numpy(np.ascontiguousarray(a, dt)).to(dev)
+        self.cand1, self.cand2 = t(cand1, np.int32), t(cand2, np.int32)
+        self.r1, self.r2 = t(r1, np.float32), t(r2, np.float32)
+        self.theta1, self.theta2 = t(theta1, np.float32), t(theta2, np.float32)
+        self.ident1 = torch.arange(self.w1 * self.k1, dtype=torch.int32, device=dev).view(self.w1, self.k1)
+        self.ident2 = torch.arange(self.w2 * self.k2, dtype=torch.int32, device=dev).view(self.w2, self.k2)
+        # candidate CSR of layer 2 (its input gradient feeds layer 1)
+        off2, edge2 = bitlogic_build_csr(np.ascontiguousarray(cand2, np.int32), self.w1)
+        self.coff2, self.cedge2 = t(off2, np.int32), t(edge2, np.int32)
+
+    def snap(self) -> "Network":
+        """The discretized network: each slot keeps its most likely candidate."""
+        conns = []
+        for cand, r, w, k in ((self.cand1, self.r1, self.w1, self.k1), (self.cand2, self.r2, self.w2, self.k2)):
+            conn = torch.empty(w * k, dtype=torch.int32, device=cand.device)
+            bitlogic_route_snap(cand, r, conn)
+            conns.append(conn.view(w, k).cpu().numpy())
+        return Network(conns[0], self.theta1.cpu().numpy(), conns[1], self.theta2.cpu().numpy(), self.w_in,
+                       device=self.cand1.device)
+
+
+class RoutedTrainStep:
+    """One training step of a RoutedNetwork: encode, per layer the routing
+    (slot inputs as the expected selection) and the LUT nodes over them,
+    head, and the backward through nodes and routing (gradients of the
+    table and routing logits)."""
+
+    def __init__(self, net: RoutedNetwork, B: int, d: int, thresholds: Sequence[int], C: int, tau: float,
+                 node: str = "soft", device="cuda"):
+        dev = torch.device(device)
+        if node not in NODE_FORMS:
+            raise ValueError(f"node must be one of {sorted(NODE_FORMS)}")
+        self.net, self.B, self.d, self.C, self.tau, self.node = net, int(B), int(d), int(C), float(tau), node
+        self.thr = [int(t) for t in thresholds]
+        assert d * len(self.thr) == net.w_in and net.w2 % C == 0
+        f32 = dict(dtype=torch.float32, device=dev)
+        s1, s2 = net.w1 * net.k1, net.w2 * net.k2
+        self.x = torch.zeros(B, d, dtype=torch.uint8, device=dev)
+        self.labels = torch.zeros(B, dtype=torch.int32, device=dev)
+        self.bits = torch.empty(net.w_in, B, **f32)
+        self.xr1, self.xr2 = torch.empty(s1, B, **f32), torch.empty(s2, B, **f32)
+        self.p1, self.p2 = torch.empty(s1, net.Kc, **f32), torch.empty(s2, net.Kc, **f32)
+        self.y1 = torch.empty(net.w1, B, **f32)
+        self.y2 = torch.empty(net.w2, B, **f32)
+        self.logits = torch.empty(B, C, **f32)
+        self.loss = torch.zeros(1, **f32)
+        self.dyg = torch.empty(C, B, **f32)
+        self.g1, self.g2 = torch.empty(s1, B, **f32), torch.empty(s2, B, **f32)   # dL/dXr
+        self.dy1 = torch.empty(net.w1, B, **f32)
+        self.dth1, self.dth2 = torch.empty_like(net.theta1), torch.empty_like(net.theta2)
+        self.dr1, self.dr2 = torch.empty_like(net.r1), torch.empty_like(net.r2)
+        self.ws_head = torch.empty(bitlogic_head_loss_workspace(B, C), dtype=torch.uint8, device=dev)
+
+    def load(self, x: torch.Tensor, labels: torch.Tensor, non_blocking: bool = False):
+        self.x.copy_(x, non_blocking=non_blocking)
+        self.labels.copy_(labels, non_blocking=non_blocking)
+
+    def forward(self, stream=None, mark=_nomark):
+        n = self.net
+        bitlogic_encode_thermometer(self.x, self.thr, self.bits, stream)
+        mark("encode")
+        bitlogic_route_forward(self.bits, n.cand1, n.r1, self.xr1, self.p1, stream)
+        mark("route1")
+        bitlogic_lut_forward_node(self.xr1, n.ident1, n.theta1, self.y1, self.node, stream)
+        mark("forward1")
+        bitlogic_route_forward(self.y1, n.cand2, n.r2, self.xr2, self.p2, stream)
+        mark("route2")
+        bitlogic_lut_forward_node(self.xr2, n.ident2, n.theta2, self.y2, self.node, stream)
+        mark("forward2")
+        bitlogic_head_loss_ex(self.y2, self.labels, self.C, self.tau, self.loss, self.ws_head,
+                              logits=self.logits, dY_grouped=self.dyg, stream=stream)
+        mark("head")
+
+    def backward(self, stream=None, mark=_nomark):
+        n = self.net
+        # layer 2: node gradients per slot (identity connectivity: the edge
+        # terms are dL/dXr2), then the routing: dr2 and dY1
+        bitlogic_lut_backward_node(self.xr2, n.ident2, n.theta2, self.dth2, self.node, dY=self.dyg,
+                                   dy_group=n.w2 // self.C, edge_terms=self.g2, stream=stream)
+        mark("backward2")
+        bitlogic_route_backward(self.y1, n.cand2, n.r2, self.g2, self.dr2, self.p2, n.coff2, n.cedge2,
+                                self.dy1, stream)
+        mark("route_bwd2")
+        bitlogic_lut_backward_node(self.xr1, n.ident1, n.theta1, self.dth1, self.node, dY=self.dy1,
+                                   edge_terms=self.g1, stream=stream)
+        mark("backward1")
+        bitlogic_route_backward(self.bits, n.cand1, n.r1, self.g1, self.dr1, stream=stream)
+        mark("route_bwd1")
+
+    def run(self, stream=None, mark=_nomark):
+        self.forward(stream, mark)
+        self.backward(stream, mark)
+
+    def capture(self) -> torch.cuda.CUDAGraph:
+        return capture_graph(self.run)
+
+    def update(self, lr: float = 0.01, betas=(0.9, 0.999), eps: float = 1e-8, weight_decay: float = 0.0,
+               stream=None, mark=_nomark):
+        """AdamW (§4 settings) on the table and routing logits of both layers."""
+        n = self.net
+        params = ((n.theta1, self.dth1), (n.theta2, self.dth2), (n.r1, self.dr1), (n.r2, self.dr2))
+        if not hasattr(self, "opt_state"):
+            self.opt_state = [(torch.zeros_like(p), torch.zeros_like(p)) for p, _ in params]
+            self.opt_step = 0
+        self.opt_step += 1
+        for (p, g), (m, v) in zip(params, self.opt_state):
+            bitlogic_adamw_update(p, m, v, g, self.opt_step, lr, betas, eps, weight_decay, stream)
+        mark("update")
+
+    # encode 1, routing forwards 2, LUT forwards 2, head 3, LUT backwards 2,
+    # routing dr 2, routing dX 1
+    kernels_per_run = 13
+    fuse_dy1 = False
 
 
 class HardInfer:

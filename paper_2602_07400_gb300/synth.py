@@ -42,6 +42,7 @@ class Workload:
     widths: Tuple[int, int]    # nodes of layer 1 and layer 2
     k: int                     # fan-in of every node
     tau: float                 # group-sum temperature
+    Kc: int = 0                # learnable routing: candidates per slot (0: fixed connectivity)
 
     @property
     def b(self) -> int:
@@ -70,6 +71,10 @@ WORKLOADS = {
     "mnist_k2": Workload("mnist_k2", 1024, 784, 10, 40.0, (64, 128, 192), (8000, 8000), 2, 20.0),
     # fan-in 4, the rank the paper pins for its method comparisons (App. C.2)
     "mnist_k4": Workload("mnist_k4", 1024, 784, 10, 40.0, (64, 128, 192), (8000, 8000), 4, 20.0),
+    # learnable routing with 16 candidates per slot in both layers, the
+    # connectivity of the paper's best-of-space configuration (App. C.2), k=4
+    "mnist_k4_routed16": Workload("mnist_k4_routed16", 1024, 784, 10, 40.0, (64, 128, 192), (8000, 8000), 4,
+                                  20.0, Kc=16),
     # CIFAR-10-shaped: 3072 features, 7 thresholds -> 21504 bits, 64000 x 64000
     "cifar10": Workload("cifar10", 1024, 3072, 10, 50.0, _even(32, 7), (64000, 64000), 6, 50.0),
     # CIFAR-100-shaped wide: 15 thresholds -> 46080 bits, 128000 x 128000
@@ -171,6 +176,19 @@ def random_tables(w: int, seed: int) -> np.ndarray:
     rng = np.random.default_rng(seed)
     return rng.integers(0, 1 << 63, size=(w,), dtype=np.uint64) * np.uint64(2) + \
         rng.integers(0, 2, size=(w,), dtype=np.uint64)
+
+
+def routed_network(wl: Workload, seed: int = 0):
+    """Candidate pools (layer 1 seed ``seed``, layer 2 ``seed + 1``), zero
+    routing logits (App. A) and table logits of the routed network of ``wl``."""
+    w1, w2 = wl.widths
+    cand1 = candidate_pools(w1 * wl.k, wl.Kc, wl.w_in, seed)
+    cand2 = candidate_pools(w2 * wl.k, wl.Kc, w1, seed + 1)
+    r1 = np.zeros((w1 * wl.k, wl.Kc), np.float32)
+    r2 = np.zeros((w2 * wl.k, wl.Kc), np.float32)
+    th1 = table_logits(w1, wl.K, seed + 100)
+    th2 = table_logits(w2, wl.K, seed + 101)
+    return cand1, r1, th1, cand2, r2, th2
 
 
 def network(wl: Workload, seed: int = 0):

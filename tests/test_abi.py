@@ -140,6 +140,20 @@ def test_host_validation_returns_before_any_launch():
     assert lib.bitlogic_pixel_histogram(None, 5, fake, None) == -1
     assert lib.bitlogic_pixel_histogram(fake, 5, None, None) == -1
     assert lib.bitlogic_pixel_histogram(None, 0, None, None) == 0
+    # routing: candidates per slot 1..32 and <= w_in, slots > 0, pointers
+    rf, rb, rs = lib.bitlogic_route_forward, lib.bitlogic_route_backward, lib.bitlogic_route_snap
+    assert rf(fake, 64, 8, fake, fake, 10, 33, fake, None, None) == -3
+    assert rf(fake, 64, 8, fake, fake, 10, 0, fake, None, None) == -3
+    assert rf(fake, 4, 8, fake, fake, 10, 5, fake, None, None) == -3
+    assert rf(fake, 64, 8, fake, fake, 0, 4, fake, None, None) == -2
+    assert rf(fake, 64, 8, None, fake, 10, 4, fake, None, None) == -1
+    assert rf(fake, 64, 8, fake, fake, 10, 4, None, None, None) == -1
+    assert rf(fake, 64, 0, fake, fake, 10, 4, None, None, None) == 0
+    assert rb(fake, 64, 8, fake, fake, 10, 4, fake, None, None, None, None, None, None) == -1
+    assert rb(fake, 64, 8, fake, fake, 10, 4, fake, fake, None, fake, fake, fake, None) == -1
+    assert rs(fake, fake, 10, 0, fake, None) == -3
+    assert rs(fake, fake, 0, 4, fake, None) == -2
+    assert rs(None, fake, 10, 4, fake, None) == -1
     # node form: only soft (0) and straight-through (1)
     fwd_node, bwd_node = lib.bitlogic_lut_forward_node, lib.bitlogic_lut_backward_node
     assert fwd_node(fake, 8, 64, fake, fake, 4, 2, 2, fake, None) == -12

@@ -199,6 +199,67 @@ def test_lut_backward_st(k, w_in, w, B, binary):
     no_device_error()
 
 
+# ------------------------------------------------------ learnable routing --
+
+ROUTE = [  # (slots, Kc, w_in, B)
+    (1, 1, 1, 1), (5, 3, 7, 37), (24, 4, 50, 128), (64, 8, 300, 259), (96, 16, 1000, 1024),
+    (40, 32, 64, 100), (33, 16, 2352, 1027), (7, 5, 9, 4),
+]
+
+
+@pytest.mark.parametrize("slots,Kc,w_in,B", ROUTE)
+def test_route_forward_backward(slots, Kc, w_in, B):
+    rng = np.random.default_rng(slots * 31 + Kc)
+    X = synth.uniform_activations(w_in, B, seed=slots + B)
+    cand = synth.candidate_pools(slots, Kc, w_in, seed=Kc + 3)
+    r = synth.table_logits(slots, Kc, seed=slots + 4)
+    G = synth.uniform_gradients(slots, B, seed=B + 5, scale=1e-3)
+    Xr = torch.full((slots, B), np.nan, device="cuda")
+    prob = torch.full((slots, Kc), np.nan, device="cuda")
+    bl.bitlogic_route_forward(dev(X), dev(cand), dev(r), Xr, prob)
+    wXr, wp = oracle.route_forward(X.astype(np.float64), cand, r)
+    check_fwd(Xr, wXr, "Xr")
+    check_fwd(prob, wp, "prob")
+    off, edge = bl.bitlogic_build_csr(cand, w_in)
+    dr = torch.full((slots, Kc), np.nan, device="cuda")
+    dX = torch.full((w_in, B), np.nan, device="cuda")
+    bl.bitlogic_route_backward(dev(X), dev(cand), dev(r), dev(G), dr, prob, dev(off), dev(edge), dX)
+    wdr, wdX = oracle.route_backward(X.astype(np.float64), cand, r, G.astype(np.float64))
+    check_grad(dr, wdr, "dr")
+    check_grad(dX, wdX, "dX")
+    dr2 = torch.full((slots, Kc), np.nan, device="cuda")
+    bl.bitlogic_route_backward(dev(X), dev(cand), dev(r), dev(G), dr2)   # dr only
+    check_exact(dr2.cpu().numpy(), dr.cpu().numpy(), "dr without dX")
+    conn = torch.full((slots,), -1, dtype=torch.int32, device="cuda")
+    bl.bitlogic_route_snap(dev(cand), dev(r), conn)
+    check_exact(conn.cpu().numpy(), oracle.route_snap(cand, r), "snap")
+    no_device_error()
+
+
+def test_route_unaligned_and_tied_logits():
+    # a view 4 bytes into an allocation takes the scalar paths; tied logits
+    # snap to the first candidate
+    slots, Kc, w_in, B = 12, 8, 40, 64
+    X = synth.uniform_activations(w_in, B, seed=1)
+    cand = synth.candidate_pools(slots, Kc, w_in, seed=2)
+    r = np.zeros((slots, Kc), np.float32)
+    r[:, 3] = 1.0
+    r[:, 6] = 1.0
+    big = torch.zeros(w_in * B + 1, device="cuda")
+    big[1:] = dev(X).reshape(-1)
+    Xv = big[1:].view(w_in, B)
+    Xr = torch.empty(slots, B, device="cuda")
+    bl.bitlogic_route_forward(Xv, dev(cand), dev(r), Xr)
+    check_fwd(Xr, oracle.route_forward(X.astype(np.float64), cand, r)[0], "Xr (scalar path)")
+    G = synth.uniform_gradients(slots, B, seed=3, scale=1e-3)
+    dr = torch.empty(slots, Kc, device="cuda")
+    bl.bitlogic_route_backward(Xv, dev(cand), dev(r), dev(G), dr)
+    check_grad(dr, oracle.route_backward(X.astype(np.float64), cand, r, G.astype(np.float64), False)[0], "dr")
+    conn = torch.empty(slots, dtype=torch.int32, device="cuda")
+    bl.bitlogic_route_snap(dev(cand), dev(r), conn)
+    check_exact(conn.cpu().numpy(), cand[:, 3], "snap to the first maximum")
+
+
 @pytest.mark.parametrize("k,w_in,w,B,group", [(6, 300, 120, 256, 12), (6, 64, 40, 1024, 40), (3, 50, 30, 37, 5),
                                                (2, 9, 20, 100, 1), (1, 4, 6, 8, 3)])
 def test_backward_grouped_dy(k, w_in, w, B, group):

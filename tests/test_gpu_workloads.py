@@ -169,6 +169,91 @@ def test_graph_replay_matches_eager_launches():
     check_grad(got["dth1"], r["dth1"], "dtheta1")
 
 
+def _routed(wl, Kc, seed=0, node="soft"):
+    from paper_2602_07400_gb300.pipeline import RoutedNetwork, RoutedTrainStep
+    w1, w2 = wl.widths
+    cand1 = synth.candidate_pools(w1 * wl.k, Kc, wl.w_in, seed)
+    cand2 = synth.candidate_pools(w2 * wl.k, Kc, w1, seed + 1)
+    r1 = synth.table_logits(w1 * wl.k, Kc, seed + 2, scale=0.5)
+    r2 = synth.table_logits(w2 * wl.k, Kc, seed + 3, scale=0.5)
+    th1 = synth.table_logits(w1, wl.K, seed + 100)
+    th2 = synth.table_logits(w2, wl.K, seed + 101)
+    net = RoutedNetwork(cand1, r1, th1, cand2, r2, th2, wl.w_in)
+    st = RoutedTrainStep(net, wl.batch, wl.d, wl.thresholds, wl.classes, wl.tau, node=node)
+    return net, st, (cand1, r1, th1, cand2, r2, th2)
+
+
+@pytest.mark.parametrize("k,Kc,node", [(6, 8, "soft"), (4, 16, "soft"), (4, 16, "st")])
+def test_tiny_routed_step_all_outputs(k, Kc, node):
+    # learnable routing (candidate pools, softmax expected selection) in both
+    # layers: every output and gradient, routing logits included
+    wl = synth.WORKLOADS["tiny"]
+    wl = synth.Workload(wl.name, wl.batch, wl.d, wl.classes, wl.sigma, wl.thresholds, wl.widths, k, wl.tau)
+    net, st, (cand1, r1, th1, cand2, r2, th2) = _routed(wl, Kc)
+    st.node = node
+    x, labels = synth.blob_batch(wl.batch, wl.d, wl.classes, wl.sigma, seed=31)
+    st.load(x.cuda(), labels.cuda())
+    st.run()
+    torch.cuda.synchronize()
+    r = oracle.routed_train_step(x.numpy(), labels.numpy(), wl.thresholds, cand1, r1, th1, cand2, r2, th2,
+                                 wl.classes, wl.tau, node=node)
+    check_exact(st.bits.cpu().numpy().astype(np.float64), r["bits"], "bits")
+    for name in ("xr1", "y1", "xr2", "y2", "logits"):
+        check_fwd(getattr(st, name), r[name], name, atol=1e-6 if node == "st" else 0.0)
+    check_fwd(st.loss, np.array([r["loss"]]), "loss")
+    for name in ("dth2", "dr2", "dy1", "dth1", "dr1"):
+        check_grad(getattr(st, name), r[name], name)
+    check_grad(st.g2, r["dxr2"], "dXr2")
+    assert bl_device_ok()
+
+
+def bl_device_ok():
+    import paper_2602_07400_gb300 as bl
+    return bl.bitlogic_device_error() == 0
+
+
+def test_routed_training_learns_and_snaps_to_a_deployable_network():
+    # AdamW on table and routing logits (routing logits start at zero, App. A);
+    # the loss falls, and the snapped network's hard pass is the oracle's
+    from paper_2602_07400_gb300.pipeline import RoutedNetwork, RoutedTrainStep
+    wl = synth.WORKLOADS["tiny"]
+    wl = synth.Workload(wl.name, wl.batch, wl.d, wl.classes, wl.sigma, wl.thresholds, wl.widths, 4, wl.tau)
+    Kc = 8
+    w1, w2 = wl.widths
+    cand1 = synth.candidate_pools(w1 * 4, Kc, wl.w_in, 0)
+    cand2 = synth.candidate_pools(w2 * 4, Kc, w1, 1)
+    zeros1 = np.zeros((w1 * 4, Kc), np.float32)
+    zeros2 = np.zeros((w2 * 4, Kc), np.float32)
+    net = RoutedNetwork(cand1, zeros1, synth.table_logits(w1, 16, 100), cand2, zeros2,
+                        synth.table_logits(w2, 16, 101), wl.w_in)
+    st = RoutedTrainStep(net, wl.batch, wl.d, wl.thresholds, wl.classes, wl.tau)
+    losses = []
+    for step in range(1, 61):
+        x, labels = synth.blob_batch(wl.batch, wl.d, wl.classes, wl.sigma, seed=200 + step, means_seed=7)
+        st.load(x.cuda(), labels.cuda())
+        st.run()
+        st.update()
+        losses.append(float(st.loss.item()))
+    # uniform routing averages the pools at first, so the loss starts flat
+    # and falls slowly at the paper's learning rate
+    assert np.mean(losses[-5:]) < 0.97 * np.mean(losses[:3]), losses
+    assert float(net.r1.abs().max()) > 0.0   # the routing logits moved
+    fixed = net.snap()
+    hi = HardInfer(fixed, 300, wl.d, wl.thresholds, wl.classes)
+    x, _ = synth.blob_batch(300, wl.d, wl.classes, wl.sigma, seed=99)
+    hi.x.copy_(x.cuda())
+    hi.binarize()
+    hi.run()
+    torch.cuda.synchronize()
+    conn1 = oracle.route_snap(cand1, net.r1.cpu().numpy()).reshape(w1, 4)
+    conn2 = oracle.route_snap(cand2, net.r2.cpu().numpy()).reshape(w2, 4)
+    t1 = oracle.binarize_tables(net.theta1.cpu().numpy())
+    t2 = oracle.binarize_tables(net.theta2.cpu().numpy())
+    ro = oracle.hard_infer(x.numpy(), wl.thresholds, conn1, t1, conn2, t2, wl.classes)
+    check_exact(hi.counts.cpu().numpy(), ro["counts"], "counts of the snapped network")
+    check_exact(hi.pred.cpu().numpy(), ro["pred"], "pred of the snapped network")
+
+
 def _sampled_compare(wl, st, x, labels, params, n_nodes=96, seed=0):
     conn1, th1, conn2, th2 = params
     bits = oracle.encode_thermometer(x, wl.thresholds)
