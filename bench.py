@@ -228,8 +228,8 @@ def call_work(wl, B, fuse_dy1=False):
 # file's SHA-256 is recorded, and any later change reports null.
 TRAFFIC = {
     ("mnist", "backward2"): {
-        "bytes": 59.695872e6 + 147.913472e6, "source": "lut_soft.cu",
-        "sha256": "ce01d9d3fec57eea20ef26863dbf4290149384de3fe362e07bac6528dab3bf5d",
+        "bytes": 59.724032e6 + 147.739392e6, "source": "lut_soft.cu",
+        "sha256": "26c8964377cea4e35c20a6db76fc85ec085463013f798c56481836d387617598",
         "note": "ncu capture of this workload"},
     ("hard_cifar10", "hard1"): {
         "bytes": 16 * (1.216602e9 + 2.055721e9), "source": "hard.cu",
