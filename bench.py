@@ -493,6 +493,26 @@ def run_ours(args):
                                    "algorithmic_bytes": 28 * n_par,
                                    "GB/s": 28 * n_par / (upd * 1e-3) / 1e9,
                                    "settings": "AdamW beta (0.9, 0.999), eps 1e-8, lr 0.01, wd 0"}
+    if st is not None and world > 1 and not args.profile:
+        # the data-parallel exchange of a training step (all-reduce of the
+        # gradients before the update), timed on its own: the fwd+bwd step
+        # above has no collective
+        from paper_2602_07400_gb300.pipeline import allreduce_gradients
+        grads = st.gradients()
+        for _ in range(3):
+            allreduce_gradients(grads)
+        torch.cuda.synchronize()
+        torch.distributed.barrier()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(20):
+            allreduce_gradients(grads)
+        e1.record()
+        torch.cuda.synchronize()
+        ms_x = max_over_ranks([e0.elapsed_time(e1) / 20], "cuda")[0]
+        if result is not None:
+            result["dp_exchange"] = {"ms": ms_x, "collective": "NCCL all-reduce (sum) of the gradients, then / N",
+                                     "bytes_per_rank": int(sum(g.numel() * 4 for g in grads))}
     if not args.profile and rank == 0:
         result["fit"] = time_quantile_fit(wl, flush)
     if not args.profile and not args.no_e2e:

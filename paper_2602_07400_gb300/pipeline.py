@@ -58,6 +58,22 @@ def capture_graph(fn) -> torch.cuda.CUDAGraph:
     return graph
 
 
+def allreduce_gradients(grads, group=None) -> None:
+    """Data-parallel exchange of a training step (§8 of the build plan: the
+    batch is sharded over ranks, every rank holds the whole network): sum
+    the ranks' gradients and divide by the number of ranks, in place, one
+    all-reduce per tensor in list order.  Each rank's loss is the mean over
+    its own batch, so with equal batches the result is the gradient of the
+    mean loss over all ranks' samples; every rank then applies the same
+    update."""
+    import torch.distributed as dist
+    world = dist.get_world_size(group)
+    for g in grads:
+        dist.all_reduce(g, op=dist.ReduceOp.SUM, group=group)
+        if world > 1:
+            g.div_(world)
+
+
 class Network:
     """Connectivity, table logits and inverse connectivity of a two-layer
     LUT network, resident on the device."""
@@ -177,6 +193,10 @@ class TrainStep:
         """One run() (forward + backward) as a CUDA graph: a replay launches
         the same kernels with no host work between them."""
         return capture_graph(self.run)
+
+    def gradients(self):
+        """The tensors a data-parallel step exchanges before the update."""
+        return [self.dth1, self.dth2]
 
     def update(self, lr: float = 0.01, betas=(0.9, 0.999), eps: float = 1e-8,
                weight_decay: float = 0.0, stream=None, mark=_nomark):
@@ -313,6 +333,9 @@ class RoutedTrainStep:
 
     def capture(self) -> torch.cuda.CUDAGraph:
         return capture_graph(self.run)
+
+    def gradients(self):
+        return [self.dth1, self.dth2, self.dr1, self.dr2]
 
     def update(self, lr: float = 0.01, betas=(0.9, 0.999), eps: float = 1e-8, weight_decay: float = 0.0,
                stream=None, mark=_nomark):

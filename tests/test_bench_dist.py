@@ -1,6 +1,7 @@
-"""The benchmark's multi-rank arithmetic on CPU with the gloo backend
-(world size 2): the job time is the slowest rank's, the job throughput
-counts every rank's samples."""
+"""The benchmark's multi-rank arithmetic and the data-parallel gradient
+exchange on CPU with the gloo backend (world size 2): the job time is the
+slowest rank's, the job throughput counts every rank's samples, and the
+all-reduced half-batch gradients equal the full batch's."""
 import os
 import socket
 
@@ -45,3 +46,46 @@ def test_single_process_is_identity():
     import bench
     assert bench.max_over_ranks([3.0, 4.0], "cpu") == [3.0, 4.0]
     assert bench.job_rate(1, 1024, 10, 5.0) == pytest.approx(1024 * 10 / 5e-3)
+
+
+def _dp_worker(rank, world, port, out):
+    import numpy as np
+    import oracle
+    from paper_2602_07400_gb300 import synth
+    from paper_2602_07400_gb300.pipeline import allreduce_gradients
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        wl = synth.Workload("dp", 64, 48, 4, 40.0, (64, 128, 192), (40, 40), 4, 5.0)
+        conn1, th1, conn2, th2 = synth.network(wl, 0)
+        x, labels = synth.blob_batch(wl.batch, wl.d, wl.classes, wl.sigma, seed=5)
+        half = wl.batch // world
+        sl = slice(rank * half, (rank + 1) * half)   # this rank's shard of the batch
+        r = oracle.train_step(x.numpy()[sl], labels.numpy()[sl], wl.thresholds, conn1, th1, conn2, th2,
+                              wl.classes, wl.tau)
+        grads = [torch.from_numpy(r["dth1"].copy()), torch.from_numpy(r["dth2"].copy())]
+        allreduce_gradients(grads)
+        out[rank] = [g.numpy() for g in grads]
+    finally:
+        dist.destroy_process_group()
+
+
+def test_data_parallel_gradient_exchange_gloo():
+    # two ranks, each with half the batch: after the exchange both hold the
+    # gradient of the full batch's mean loss
+    import numpy as np
+    import oracle
+    from paper_2602_07400_gb300 import synth
+    world = 2
+    port = _free_port()
+    mgr = mp.get_context("spawn").Manager()
+    out = mgr.dict()
+    mp.start_processes(_dp_worker, args=(world, port, out), nprocs=world, join=True, start_method="spawn")
+    wl = synth.Workload("dp", 64, 48, 4, 40.0, (64, 128, 192), (40, 40), 4, 5.0)
+    conn1, th1, conn2, th2 = synth.network(wl, 0)
+    x, labels = synth.blob_batch(wl.batch, wl.d, wl.classes, wl.sigma, seed=5)
+    full = oracle.train_step(x.numpy(), labels.numpy(), wl.thresholds, conn1, th1, conn2, th2, wl.classes, wl.tau)
+    for rank in range(world):
+        np.testing.assert_allclose(out[rank][0], full["dth1"], rtol=1e-10, atol=1e-15)
+        np.testing.assert_allclose(out[rank][1], full["dth2"], rtol=1e-10, atol=1e-15)
+    np.testing.assert_array_equal(out[0][0], out[1][0])
