@@ -516,7 +516,7 @@ def run_ours(args):
     if not args.profile and rank == 0:
         result["fit"] = time_quantile_fit(wl, flush)
     if not args.profile and not args.no_e2e:
-        e2e = run_e2e(args, st, hi, wl, B, g_train if use_graph else None, g_hard if use_graph else None)
+        e2e = run_e2e(args, st, hi, wl, B, use_graph)
         if result is not None:
             result["e2e"] = e2e["train"] if st is not None else e2e["hard"]
             result["hard"]["e2e"] = e2e["hard"]
@@ -571,18 +571,13 @@ def time_update(st, iters: int) -> float:
     return e0.elapsed_time(e1) / iters
 
 
-def run_e2e(args, st, hi, wl, B, g_train=None, g_hard=None):
-    """The same metric end to end: pinned host inputs copied in, the step
-    run through the public API (the captured graphs when given), the step's
-    result copied out, every step."""
-    train_run = g_train.replay if g_train is not None else st.run if st is not None else None
-
-    def hard_run():
-        if g_hard is not None:
-            g_hard.replay()
-        else:
-            hi.binarize()
-            hi.run()
+def run_e2e(args, st, hi, wl, B, use_graph=True):
+    """The same metric end to end through the public API: every step copies
+    its batch from pinned host memory and its result (loss, or predictions)
+    back.  With graphs, ``pipeline.Prefetcher`` overlaps the copy of the
+    next batch with the current step (two input buffers, a copy stream);
+    without, the copy, the step and the read-back run in sequence."""
+    from paper_2602_07400_gb300.pipeline import Prefetcher
     world, rank, _ = dist_env()
     x_host, lab_host = synth.blob_batch(B, wl.d, wl.classes, wl.sigma, seed=2000 + rank)
     x_host = x_host.pin_memory()
@@ -591,40 +586,55 @@ def run_e2e(args, st, hi, wl, B, g_train=None, g_hard=None):
     pred_host = torch.empty(B, dtype=torch.int32).pin_memory()
     K = max(1, args.steps)
     out = {}
-    if st is not None:
+
+    def timed(pf, host, res, eager):
+        if pf is None:
+            for _ in range(3):
+                eager()
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            for _ in range(K):
+                eager()
+            e1.record()
+            torch.cuda.synchronize()
+            return max_over_ranks([e0.elapsed_time(e1)], "cuda")[0]
         for _ in range(3):
-            st.load(x_host, lab_host, non_blocking=True)
-            train_run()
-            loss_host.copy_(st.loss, non_blocking=True)
+            pf.prefetch(host)
+            pf.run(res)
         torch.cuda.synchronize()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record()
-        for _ in range(K):
-            st.load(x_host, lab_host, non_blocking=True)
-            train_run()
-            loss_host.copy_(st.loss, non_blocking=True)
+        pf.start()
+        pf.prefetch(host)
+        for i in range(K):
+            if i + 1 < K:
+                pf.prefetch(host)   # batch i + 1 streams in while step i runs
+            pf.run(res)
         e1.record()
         torch.cuda.synchronize()
-        ms = max_over_ranks([e0.elapsed_time(e1)], "cuda")[0]
+        return max_over_ranks([e0.elapsed_time(e1)], "cuda")[0]
+
+    if st is not None:
+        def eager_train():
+            st.load(x_host, lab_host, non_blocking=True)
+            st.run()
+            loss_host.copy_(st.loss, non_blocking=True)
+        pf = Prefetcher(st, ("x", "labels"), "loss") if use_graph else None
+        ms = timed(pf, {"x": x_host, "labels": lab_host}, loss_host, eager_train)
         out["train"] = {"value": job_rate(world, B, K, ms), "unit": "samples/s",
                         "h2d_bytes_per_step": x_host.numel() + 4 * lab_host.numel(),
-                        "d2h_bytes_per_step": 4}
-    for _ in range(3):
+                        "d2h_bytes_per_step": 4, "overlap": bool(use_graph)}
+
+    def eager_hard():
         hi.x.copy_(x_host, non_blocking=True)
-        hard_run()
+        hi.binarize()
+        hi.run()
         pred_host.copy_(hi.pred, non_blocking=True)
-    torch.cuda.synchronize()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record()
-    for _ in range(K):
-        hi.x.copy_(x_host, non_blocking=True)
-        hard_run()
-        pred_host.copy_(hi.pred, non_blocking=True)
-    e1.record()
-    torch.cuda.synchronize()
-    ms = max_over_ranks([e0.elapsed_time(e1)], "cuda")[0]
+    pf = Prefetcher(hi, ("x",), "pred", capture=lambda: hi.capture(binarize=True)) if use_graph else None
+    ms = timed(pf, {"x": x_host}, pred_host, eager_hard)
     out["hard"] = {"value": job_rate(world, B, K, ms) / 1e6, "unit": "MSamples/s",
-                   "h2d_bytes_per_step": x_host.numel(), "d2h_bytes_per_step": 4 * B}
+                   "h2d_bytes_per_step": x_host.numel(), "d2h_bytes_per_step": 4 * B, "overlap": bool(use_graph)}
     return out
 
 

@@ -74,6 +74,52 @@ def allreduce_gradients(grads, group=None) -> None:
             g.div_(world)
 
 
+class Prefetcher:
+    """Runs a step object (TrainStep, RoutedTrainStep or HardInfer) over
+    host batches with the host-to-device copy of the next batch overlapping
+    the current step: two device input buffers, each with its own captured
+    graph of the step, and a copy stream.  ``prefetch`` enqueues a batch's
+    copy; ``run`` replays the step on the oldest fetched batch and copies its
+    result (the attribute ``out``) into a host tensor, all asynchronously."""
+
+    def __init__(self, step, names=("x", "labels"), out="loss", capture=None):
+        self.step, self.names, self.out = step, tuple(names), out
+        self.bufs = [{n: torch.empty_like(getattr(step, n)) for n in self.names} for _ in range(2)]
+        self.graphs = []
+        for b in range(2):
+            for n in self.names:
+                setattr(step, n, self.bufs[b][n])
+            self.graphs.append(capture() if capture is not None else step.capture())
+        self.copy_stream = torch.cuda.Stream()
+        self.copied = [torch.cuda.Event() for _ in range(2)]
+        self.consumed = [torch.cuda.Event() for _ in range(2)]
+        self.n_fetched = 0
+        self.n_run = 0
+
+    def start(self):
+        """Order the copy stream after the work already on the current stream."""
+        self.copy_stream.wait_stream(torch.cuda.current_stream())
+
+    def prefetch(self, host: dict):
+        b = self.n_fetched % 2
+        cs = self.copy_stream
+        cs.wait_event(self.consumed[b])   # the step that last read buffer b is done
+        with torch.cuda.stream(cs):
+            for n in self.names:
+                self.bufs[b][n].copy_(host[n], non_blocking=True)
+        self.copied[b].record(cs)
+        self.n_fetched += 1
+
+    def run(self, out_host: torch.Tensor):
+        b = self.n_run % 2
+        cur = torch.cuda.current_stream()
+        cur.wait_event(self.copied[b])
+        self.graphs[b].replay()
+        out_host.copy_(getattr(self.step, self.out), non_blocking=True)
+        self.consumed[b].record(cur)
+        self.n_run += 1
+
+
 class Network:
     """Connectivity, table logits and inverse connectivity of a two-layer
     LUT network, resident on the device."""

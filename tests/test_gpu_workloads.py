@@ -169,6 +169,46 @@ def test_graph_replay_matches_eager_launches():
     check_grad(got["dth1"], r["dth1"], "dtheta1")
 
 
+def test_prefetcher_overlapped_steps_match_eager_steps():
+    # batches streamed through the two-buffer prefetcher (copy of batch i+1
+    # during step i) give every step's loss and predictions bit for bit
+    from paper_2602_07400_gb300.pipeline import Prefetcher
+    wl = synth.WORKLOADS["tiny"]
+    conn1, th1, conn2, th2 = synth.network(wl, 0)
+    net = Network(conn1, th1, conn2, th2, wl.w_in)
+    st = TrainStep(net, wl.batch, wl.d, wl.thresholds, wl.classes, wl.tau)
+    hi = HardInfer(net, wl.batch, wl.d, wl.thresholds, wl.classes)
+    batches = [synth.blob_batch(wl.batch, wl.d, wl.classes, wl.sigma, seed=60 + i) for i in range(5)]
+    want_loss, want_pred = [], []
+    for x, labels in batches:
+        st.load(x.cuda(), labels.cuda())
+        st.run()
+        hi.x.copy_(x.cuda())
+        hi.binarize()
+        hi.run()
+        want_loss.append(float(st.loss.item()))
+        want_pred.append(hi.pred.cpu().numpy().copy())
+    hosts = [({"x": x.pin_memory(), "labels": l.pin_memory()}) for x, l in batches]
+    pf = Prefetcher(st, ("x", "labels"), "loss")
+    ph = Prefetcher(hi, ("x",), "pred", capture=lambda: hi.capture(binarize=True))
+    loss_out = [torch.empty(1).pin_memory() for _ in batches]
+    pred_out = [torch.empty(wl.batch, dtype=torch.int32).pin_memory() for _ in batches]
+    pf.start()
+    ph.start()
+    pf.prefetch(hosts[0])
+    ph.prefetch({"x": hosts[0]["x"]})
+    for i in range(len(batches)):
+        if i + 1 < len(batches):
+            pf.prefetch(hosts[i + 1])
+            ph.prefetch({"x": hosts[i + 1]["x"]})
+        pf.run(loss_out[i])
+        ph.run(pred_out[i])
+    torch.cuda.synchronize()
+    for i in range(len(batches)):
+        assert float(loss_out[i][0]) == want_loss[i], i
+        np.testing.assert_array_equal(pred_out[i].numpy(), want_pred[i])
+
+
 def _routed(wl, Kc, seed=0, node="soft"):
     from paper_2602_07400_gb300.pipeline import RoutedNetwork, RoutedTrainStep
     w1, w2 = wl.widths
