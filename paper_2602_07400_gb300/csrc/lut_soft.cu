@@ -33,10 +33,11 @@ namespace {
 constexpr int kFwdWarps = 4;
 constexpr int kBwdWarps = 4;   // warps per block in the staged backward
 #ifndef BITLOGIC_BWD_WARPS_PER_NODE
-#define BITLOGIC_BWD_WARPS_PER_NODE 2
+#define BITLOGIC_BWD_WARPS_PER_NODE 1
 #endif
 constexpr int kWarpsPerNode = BITLOGIC_BWD_WARPS_PER_NODE;   // 1, 2 or 4
 constexpr int kNodesPerBlock = kBwdWarps / kWarpsPerNode;
+static_assert(kWarpsPerNode == 1 || kWarpsPerNode == 2 || kWarpsPerNode == 4, "1, 2 or 4 warps per node");
 // ---------------------------------------------------------------- trees --
 
 template <int L, int M, int H, int k>
@@ -220,14 +221,16 @@ __device__ __forceinline__ void node_setup(const int* __restrict__ conn,
     __syncwarp();
 }
 
-#ifndef BITLOGIC_STAGE_SAMPLES
-#define BITLOGIC_STAGE_SAMPLES 128
-#endif
 #ifndef BITLOGIC_STAGES
 #define BITLOGIC_STAGES 3
 #endif
-constexpr int kStageSamples = BITLOGIC_STAGE_SAMPLES;   // samples per pipeline stage
+// samples per pipeline stage: every lane copies and reads one 16-byte chunk
+// (4 consecutive samples) of each row, so a stage is exactly 32 x 4 samples;
+// the lane offsets of all staged kernels rely on it
+constexpr int kStageSamples = 128;
 constexpr int kStages = BITLOGIC_STAGES;                // stages in flight per warp
+static_assert(kStageSamples == 32 * 4, "a stage is one 16-byte chunk per lane");
+static_assert(kStages >= 2 && kStages <= 8, "the rings hold 2 to 8 stages");
 
 // ------------------------------------------------------------- forward --
 

@@ -84,7 +84,9 @@ class Prefetcher:
 
     def __init__(self, step, names=("x", "labels"), out="loss", capture=None):
         self.step, self.names, self.out = step, tuple(names), out
-        self.bufs = [{n: torch.empty_like(getattr(step, n)) for n in self.names} for _ in range(2)]
+        # the buffers start as copies of the step's current inputs, so the
+        # warm-up run of each capture reads valid data (labels in range)
+        self.bufs = [{n: getattr(step, n).clone() for n in self.names} for _ in range(2)]
         self.graphs = []
         for b in range(2):
             for n in self.names:

@@ -207,6 +207,7 @@ def test_prefetcher_overlapped_steps_match_eager_steps():
     for i in range(len(batches)):
         assert float(loss_out[i][0]) == want_loss[i], i
         np.testing.assert_array_equal(pred_out[i].numpy(), want_pred[i])
+    assert bl_device_ok()   # no run (the captures' warm-ups included) met a bad index or label
 
 
 def _routed(wl, Kc, seed=0, node="soft"):
