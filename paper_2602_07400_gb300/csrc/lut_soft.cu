@@ -28,16 +28,24 @@ namespace bitlogic {
 namespace {
 
 #ifndef BITLOGIC_BWD_MIN_BLOCKS
-#define BITLOGIC_BWD_MIN_BLOCKS 4
+#define BITLOGIC_BWD_MIN_BLOCKS 4   // dtheta-only kernel: blocks per SM
+#endif
+#ifndef BITLOGIC_NODE_MIN_BLOCKS
+#define BITLOGIC_NODE_MIN_BLOCKS 3  // backward with input gradient: blocks per SM
 #endif
 constexpr int kFwdWarps = 4;
-constexpr int kBwdWarps = 4;   // warps per block in the staged backward
+#ifndef BITLOGIC_BWD_WARPS
+#define BITLOGIC_BWD_WARPS 4
+#endif
+constexpr int kBwdWarps = BITLOGIC_BWD_WARPS;   // warps per block in the staged backward
 #ifndef BITLOGIC_BWD_WARPS_PER_NODE
 #define BITLOGIC_BWD_WARPS_PER_NODE 1
 #endif
 constexpr int kWarpsPerNode = BITLOGIC_BWD_WARPS_PER_NODE;   // 1, 2 or 4
 constexpr int kNodesPerBlock = kBwdWarps / kWarpsPerNode;
 static_assert(kWarpsPerNode == 1 || kWarpsPerNode == 2 || kWarpsPerNode == 4, "1, 2 or 4 warps per node");
+static_assert(kBwdWarps >= kWarpsPerNode && kBwdWarps % kWarpsPerNode == 0 && kBwdWarps <= 16,
+              "whole nodes per block");
 // ---------------------------------------------------------------- trees --
 
 template <int L, int M, int H, int k>
@@ -528,7 +536,7 @@ constexpr size_t node_smem_bytes() {
 // parity, then the node's warps, in a fixed order.  Needs k >= 2,
 // B % 4 == 0 and 16-byte aligned X and sources.
 template <int k, bool WANT_DX, bool TERMS, bool POS>
-__global__ void __launch_bounds__(kBwdWarps * 32, BITLOGIC_BWD_MIN_BLOCKS)
+__global__ void __launch_bounds__(kBwdWarps * 32, BITLOGIC_NODE_MIN_BLOCKS)
 lut_backward_node_kernel(const float* __restrict__ X, int w_in, long long B,
                          const int* __restrict__ conn, const float* __restrict__ theta, int w,
                          int node, GradSource gs, float* __restrict__ dtheta, float* __restrict__ P,
