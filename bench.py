@@ -228,8 +228,8 @@ def call_work(wl, B, fuse_dy1=False):
 # file's SHA-256 is recorded, and any later change reports null.
 TRAFFIC = {
     ("mnist", "backward2"): {
-        "bytes": 59.724032e6 + 147.739392e6, "source": "lut_soft.cu",
-        "sha256": "26c8964377cea4e35c20a6db76fc85ec085463013f798c56481836d387617598",
+        "bytes": 58.960640e6 + 147.236608e6, "source": "lut_soft.cu",
+        "sha256": "2c9c5b523d6f03a4bd686783b702c5c09dd7a536bdd7776bfc030e0138f65040",
         "note": "ncu capture of this workload"},
     ("hard_cifar10", "hard1"): {
         "bytes": 16 * (1.216602e9 + 2.055721e9), "source": "hard.cu",
