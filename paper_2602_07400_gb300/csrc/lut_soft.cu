@@ -33,7 +33,18 @@ namespace {
 #ifndef BITLOGIC_NODE_MIN_BLOCKS
 #define BITLOGIC_NODE_MIN_BLOCKS 3  // backward with input gradient: blocks per SM
 #endif
-constexpr int kFwdWarps = 4;
+#ifndef BITLOGIC_FWD_WARPS
+#define BITLOGIC_FWD_WARPS 1
+#endif
+#ifndef BITLOGIC_FWD_MIN_CHUNK
+#define BITLOGIC_FWD_MIN_CHUNK 1024
+#endif
+#ifndef BITLOGIC_FWD_WAVES
+#define BITLOGIC_FWD_WAVES 2
+#endif
+constexpr int kFwdWarps = BITLOGIC_FWD_WARPS;
+static_assert(kFwdWarps >= 1 && kFwdWarps <= 16, "forward warps per block");
+static_assert(BITLOGIC_FWD_MIN_CHUNK % 128 == 0 && BITLOGIC_FWD_MIN_CHUNK >= 128, "whole stages per chunk");
 #ifndef BITLOGIC_BWD_WARPS
 #define BITLOGIC_BWD_WARPS 4
 #endif
@@ -1030,14 +1041,15 @@ csr_reduce_kernel(const float* __restrict__ P, long long B, const int* __restric
 // has ~6 waves of items, but at least 512 samples so the per-item set-up
 // stays small.
 long long forward_chunk(int w_in, int w, long long B) {
-    const long long l2_budget = 48ll << 20;
-    long long c = B;
-    if ((long long)w_in * B * 4 > l2_budget) c = l2_budget / ((long long)w_in * 4);
-    const long long items_wanted = 6ll * 152 * 16;
-    const long long by_waves = (long long)w * B / items_wanted;
-    if (by_waves < c) c = by_waves;
+    // a warp keeps a node over the whole batch (the per-node set-up, the
+    // sigmoids and Moebius coefficients, is paid once) unless that leaves
+    // fewer than about BITLOGIC_FWD_WAVES waves of warps; the slices keep at
+    // least BITLOGIC_FWD_MIN_CHUNK samples
+    (void)w_in;
+    const long long items_wanted = (long long)BITLOGIC_FWD_WAVES * sm_count() * 16;
+    long long c = (long long)w * B / items_wanted;
     c = (c / 128) * 128;
-    if (c < 512) c = 512;
+    if (c < BITLOGIC_FWD_MIN_CHUNK) c = BITLOGIC_FWD_MIN_CHUNK;
     return c < B ? c : B;
 }
 
