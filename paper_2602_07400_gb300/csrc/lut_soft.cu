@@ -28,7 +28,7 @@ namespace bitlogic {
 namespace {
 
 #ifndef BITLOGIC_BWD_MIN_BLOCKS
-#define BITLOGIC_BWD_MIN_BLOCKS 4   // dtheta-only kernel: blocks per SM
+#define BITLOGIC_BWD_MIN_BLOCKS 3   // dtheta-only kernel: blocks per SM
 #endif
 #ifndef BITLOGIC_NODE_MIN_BLOCKS
 #define BITLOGIC_NODE_MIN_BLOCKS 3  // backward with input gradient: blocks per SM
