@@ -228,8 +228,8 @@ def call_work(wl, B, fuse_dy1=False):
 # file's SHA-256 is recorded, and any later change reports null.
 TRAFFIC = {
     ("mnist", "backward2"): {
-        "bytes": 58.960640e6 + 147.236608e6, "source": "lut_soft.cu",
-        "sha256": "2c9c5b523d6f03a4bd686783b702c5c09dd7a536bdd7776bfc030e0138f65040",
+        "bytes": 59.129856e6 + 147.198464e6, "source": "lut_soft.cu",
+        "sha256": "91e3bbe1bd6693797fcc9c4448a3b4b31c195c9493e7c2853613653632db2089",
         "note": "ncu capture of this workload"},
     ("hard_cifar10", "hard1"): {
         "bytes": 16 * (1.216602e9 + 2.055721e9), "source": "hard.cu",
