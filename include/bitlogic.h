@@ -2,11 +2,13 @@
  * bitlogic.h -- C ABI of the GB300 (sm_103a) LUT-network hot path.
  *
  * The library implements the data-parallel hot path of BitLogic's
- * gradient-based LUT networks (arXiv 2602.07400): the thermometer encoder,
- * the soft forward/backward of a fixed-connectivity LUT layer, the group-sum
- * head with temperature and cross-entropy, and the hard bit-packed
- * evaluation mode with a popcount group-sum.  Every call is a hand-written
- * CUDA kernel sequence enqueued on the caller's stream.
+ * gradient-based LUT networks (arXiv 2602.07400): the thermometer encoder
+ * (with the quantile fit of its thresholds), the soft forward/backward of a
+ * LUT layer (LightLUT soft or straight-through hard node; fixed connectivity
+ * or learnable routing over candidate pools), the group-sum head with
+ * temperature and cross-entropy, the AdamW update of the logits, and the
+ * hard bit-packed evaluation mode with a popcount group-sum.  Every call is
+ * a hand-written CUDA kernel sequence enqueued on the caller's stream.
  *
  * Conventions shared by all calls
  *   - Pointers marked "device" are caller-owned device memory; the library
@@ -27,7 +29,10 @@
  *       packed bits      xp[row*W + s/32], bit s%32, W = ceil(N/32)
  *     Slot i of a node is bit i of its table index a.
  *   - Vectorised (16-byte) paths are taken when B % 4 == 0 and the arrays are
- *     16-byte aligned; otherwise a scalar path runs.  Results are identical.
+ *     16-byte aligned; otherwise a scalar path runs.  Integer, byte and bit
+ *     results are identical on both; floating-point results agree within
+ *     rounding (the soft forward evaluates its table in another order on the
+ *     vector path), and each path is deterministic from run to run.
  */
 #ifndef BITLOGIC_H
 #define BITLOGIC_H
