@@ -31,7 +31,7 @@ namespace {
 #define BITLOGIC_BWD_MIN_BLOCKS 3   // dtheta-only kernel: blocks per SM
 #endif
 #ifndef BITLOGIC_NODE_MIN_BLOCKS
-#define BITLOGIC_NODE_MIN_BLOCKS 3  // backward with input gradient: blocks per SM
+#define BITLOGIC_NODE_MIN_BLOCKS 12  // backward with input gradient: blocks per SM
 #endif
 #ifndef BITLOGIC_FWD_WARPS
 #define BITLOGIC_FWD_WARPS 1
@@ -46,7 +46,7 @@ constexpr int kFwdWarps = BITLOGIC_FWD_WARPS;
 static_assert(kFwdWarps >= 1 && kFwdWarps <= 16, "forward warps per block");
 static_assert(BITLOGIC_FWD_MIN_CHUNK % 128 == 0 && BITLOGIC_FWD_MIN_CHUNK >= 128, "whole stages per chunk");
 #ifndef BITLOGIC_BWD_WARPS
-#define BITLOGIC_BWD_WARPS 4
+#define BITLOGIC_BWD_WARPS 1
 #endif
 constexpr int kBwdWarps = BITLOGIC_BWD_WARPS;   // warps per block in the staged backward
 #ifndef BITLOGIC_BWD_WARPS_PER_NODE
