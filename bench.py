@@ -228,8 +228,8 @@ def call_work(wl, B, fuse_dy1=False):
 # file's SHA-256 is recorded, and any later change reports null.
 TRAFFIC = {
     ("mnist", "backward2"): {
-        "bytes": 59.129856e6 + 147.198464e6, "source": "lut_soft.cu",
-        "sha256": "91e3bbe1bd6693797fcc9c4448a3b4b31c195c9493e7c2853613653632db2089",
+        "bytes": 59.670016e6 + 147.641856e6, "source": "lut_soft.cu",
+        "sha256": "7a19ec4e05385f0d6a2daa82f5d764d2eec33d190fdbd4d2686e2535434dacc6",
         "note": "ncu capture of this workload"},
     ("hard_cifar10", "hard1"): {
         "bytes": 16 * (1.216602e9 + 2.055721e9), "source": "hard.cu",

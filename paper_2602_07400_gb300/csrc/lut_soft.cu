@@ -28,7 +28,7 @@ namespace bitlogic {
 namespace {
 
 #ifndef BITLOGIC_BWD_MIN_BLOCKS
-#define BITLOGIC_BWD_MIN_BLOCKS 3   // dtheta-only kernel: blocks per SM
+#define BITLOGIC_BWD_MIN_BLOCKS 16  // dtheta-only kernel: blocks per SM
 #endif
 #ifndef BITLOGIC_NODE_MIN_BLOCKS
 #define BITLOGIC_NODE_MIN_BLOCKS 12  // backward with input gradient: blocks per SM
@@ -811,7 +811,11 @@ lut_backward_node_kernel(const float* __restrict__ X, int w_in, long long B,
 // dtheta is reduced inside the warp by a fixed butterfly of shuffles, with
 // no block barrier.  Needs B % 4 == 0 and 16-byte aligned X, dY and dY_out.
 
-constexpr int kThetaWarps = 4;
+#ifndef BITLOGIC_THETA_WARPS
+#define BITLOGIC_THETA_WARPS 1
+#endif
+constexpr int kThetaWarps = BITLOGIC_THETA_WARPS;   // warps per block of the dtheta-only kernel
+static_assert(kThetaWarps >= 1 && kThetaWarps <= 16, "dtheta-only warps per block");
 
 template <int k>
 __host__ __device__ constexpr int theta_floats_per_warp() {
