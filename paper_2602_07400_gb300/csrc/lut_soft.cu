@@ -525,7 +525,8 @@ constexpr size_t node_smem_bytes() {
 }
 
 // Staged backward.  A block holds kNodesPerBlock nodes with kWarpsPerNode
-// warps each; each warp of a node takes a contiguous range of its 128-sample
+// warps each (by default one warp per node and per block, over the whole
+// batch); each warp of a node takes a contiguous range of its 128-sample
 // stages.
 //
 // Within a warp every sample is split over two lanes: lane h = lane & 1 owns
@@ -1040,15 +1041,12 @@ csr_reduce_kernel(const float* __restrict__ P, long long B, const int* __restric
 
 // ----------------------------------------------------------- launchers --
 
-// Samples per forward work item (node x batch slice): small enough that the
-// gathered working set of the resident items stays in L2 and that the launch
-// has ~6 waves of items, but at least 512 samples so the per-item set-up
-// stays small.
+// Samples per forward work item (node x batch slice): a warp keeps a node
+// over the whole batch (the per-node set-up, the sigmoids and Moebius
+// coefficients, is paid once) unless that leaves fewer than about
+// BITLOGIC_FWD_WAVES waves of warps; the slices keep at least
+// BITLOGIC_FWD_MIN_CHUNK samples.
 long long forward_chunk(int w_in, int w, long long B) {
-    // a warp keeps a node over the whole batch (the per-node set-up, the
-    // sigmoids and Moebius coefficients, is paid once) unless that leaves
-    // fewer than about BITLOGIC_FWD_WAVES waves of warps; the slices keep at
-    // least BITLOGIC_FWD_MIN_CHUNK samples
     (void)w_in;
     const long long items_wanted = (long long)BITLOGIC_FWD_WAVES * sm_count() * 16;
     long long c = (long long)w * B / items_wanted;
