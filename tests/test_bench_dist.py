@@ -89,3 +89,17 @@ def test_data_parallel_gradient_exchange_gloo():
         np.testing.assert_allclose(out[rank][0], full["dth1"], rtol=1e-10, atol=1e-15)
         np.testing.assert_allclose(out[rank][1], full["dth2"], rtol=1e-10, atol=1e-15)
     np.testing.assert_array_equal(out[0][0], out[1][0])
+
+
+def test_traffic_record_digest_ignores_comments(tmp_path):
+    # a capture stays valid across comment edits of its kernel source and
+    # turns null once the code changes
+    import bench
+    a = tmp_path / "a.cu"
+    a.write_text("// note\nint f(int x) { return x + 1; } /* block\ncomment */\n")
+    b = tmp_path / "b.cu"
+    b.write_text("int f(int x)   { return x + 1; }  // another note\n")
+    c = tmp_path / "c.cu"
+    c.write_text("int f(int x) { return x + 2; }\n")
+    assert bench.code_digest(str(a)) == bench.code_digest(str(b))
+    assert bench.code_digest(str(a)) != bench.code_digest(str(c))
