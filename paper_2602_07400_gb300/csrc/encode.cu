@@ -103,35 +103,45 @@ encode_soft_vec_kernel(const uint8_t* __restrict__ x, long long B, int d, Thresh
 // --------------------------------------------------------------- packed --
 //
 // One lane per output word (32 samples), so every store is a coalesced
-// 128-byte run of a wire row.  A block takes 1024 samples x 32 features and
-// stages them in a feature-major shared tile in which the 32 samples of word
-// q sit in the order u' = 4 (u % 8) + u / 8, so that 32-bit register r
-// (r < 8) of the lane holds samples r, r + 8, r + 16, r + 24.
+// 128-byte run of a wire row.  A block takes 1024 samples x 32 features.
+// Sample group (q, r) of word q holds samples 32q + r + 8j (j < 4): a 32-bit
+// register of one feature over those four samples is one byte per sample.
 //
-// Fill: thread 8q + r loads the 32 feature bytes of samples 32q + r + 8j
-// (j < 4) and transposes each 4 x 4 byte block (4 samples x 4 features) with
-// two rounds of byte permutes, so that every shared store is one 32-bit
-// word: features f of samples r, r + 8, r + 16, r + 24 at tile[f][32q + 4r].
+// Fill: thread 8q + r loads the 32 feature bytes of the four samples of group
+// (q, r) and transposes each 4 x 4 byte block (4 samples x 4 features) with
+// two rounds of byte permutes into four words, one per feature.  The shared
+// tile is [feature quad][sample group][feature in quad]: the four words of a
+// block are one 16-byte cell, written with one 16-byte store (8 per thread).
+// Cells are XOR-swizzled within each word's 8 groups (cell r ^ (q & 7)), so
+// the 8 lanes of a 16-byte access phase always hit 8 different bank groups,
+// both in the fill (lanes = the 8 groups of one word) and in the compare
+// (lanes = 8 words, one group each).
 //
-// Compare: for a threshold T every register yields its four comparisons
-// v > T as the high bits of its bytes by byte-wise SWAR arithmetic (no carry
-// crosses a byte):
+// Compare: warp w takes feature quad w; lane q reads the 8 cells of its word
+// (8 sixteen-byte loads: four features x 32 samples), and for a threshold T
+// every register yields its four comparisons v > T as the high bits of its
+// bytes by byte-wise SWAR arithmetic (no carry crosses a byte):
 //   T < 127:  v > T  <=>  v >= 128 or (v & 127) + (127 - T) >= 128
 //   T >= 127: v > T  <=>  v >= 128 and (v & 127) + (255 - T) >= 128
 // and register r's high bits, moved right by 7 - r, put sample r + 8j at bit
 // r + 8j of the word.  The move is a multiply-high by 2^(25 + r), which runs
-// on the FMA pipe and leaves the logic pipe to the comparisons.
+// on the FMA pipe and leaves the logic pipe to the comparisons.  Per 128
+// input bytes: 8 global loads, 8 shared stores, 8 shared loads.
 
 constexpr int kPackWords = 32;             // words per tile (1024 samples)
 constexpr int kPackTS = kPackWords * 32;   // samples per tile
 constexpr int kPackTF = 32;                // features per tile
-constexpr int kPackWarps = 8;              // each warp: kPackTF / kPackWarps features
+constexpr int kPackQuads = kPackTF / 4;    // feature quads per tile
+constexpr int kPackWarps = 8;              // warp w: feature quad w
 static_assert(kPackWarps * 32 == kPackWords * 8, "fill: 8 threads per word");
+static_assert(kPackWarps == kPackQuads, "compare: one feature quad per warp");
+
+__device__ __forceinline__ int pack_cell(int q, int r) { return 8 * q + (r ^ (q & 7)); }
 
 __global__ void __launch_bounds__(kPackWarps * 32)
 pack_bits_kernel(const uint8_t* __restrict__ x, long long N, int d, Thresholds th,
                  uint32_t* __restrict__ xp, long long W, bool vec16) {
-    __shared__ __align__(16) uint8_t tile[kPackTF][kPackTS];   // feature-major, permuted samples
+    __shared__ __align__(16) uint4 tile[kPackQuads][kPackWords * 8];   // [quad][swizzled group]
     __shared__ uint32_t sC[32], sOr[32];   // per-threshold SWAR constants
     if (threadIdx.x < th.b) {
         const uint32_t T = threshold_at(th, threadIdx.x);
@@ -165,8 +175,7 @@ pack_bits_kernel(const uint8_t* __restrict__ x, long long N, int d, Thresholds t
                 }
             }
         }
-        uint32_t* dst = reinterpret_cast<uint32_t*>(&tile[0][32 * wq + 4 * r]);
-        constexpr int kRow = kPackTS / 4;   // words per tile row
+        const int cell = pack_cell(wq, r);
 #pragma unroll
         for (int f4 = 0; f4 < 8; ++f4) {
             // bytes (s0 f0, s1 f0, s0 f1, s1 f1) and (s0 f2, s1 f2, s0 f3, s1 f3), likewise s2/s3
@@ -174,36 +183,41 @@ pack_bits_kernel(const uint8_t* __restrict__ x, long long N, int d, Thresholds t
             const uint32_t a1 = __byte_perm(v[0][f4], v[1][f4], 0x7362);
             const uint32_t b0 = __byte_perm(v[2][f4], v[3][f4], 0x5140);
             const uint32_t b1 = __byte_perm(v[2][f4], v[3][f4], 0x7362);
-            dst[(4 * f4 + 0) * kRow] = __byte_perm(a0, b0, 0x5410);
-            dst[(4 * f4 + 1) * kRow] = __byte_perm(a0, b0, 0x7632);
-            dst[(4 * f4 + 2) * kRow] = __byte_perm(a1, b1, 0x5410);
-            dst[(4 * f4 + 3) * kRow] = __byte_perm(a1, b1, 0x7632);
+            tile[f4][cell] = make_uint4(__byte_perm(a0, b0, 0x5410), __byte_perm(a0, b0, 0x7632),
+                                        __byte_perm(a1, b1, 0x5410), __byte_perm(a1, b1, 0x7632));
         }
     }
     __syncthreads();
     const long long q = (long long)blockIdx.y * kPackWords + lane;   // this lane's word
     if (q >= W) return;
-    for (int fl = warp; fl < nf; fl += kPackWarps) {
-        const uint4 a = *reinterpret_cast<const uint4*>(&tile[fl][32 * lane]);
-        const uint4 b = *reinterpret_cast<const uint4*>(&tile[fl][32 * lane + 16]);
-        const uint32_t r[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+    const int fq = warp;   // this warp's feature quad: features 4 fq .. 4 fq + 3
+    if (4 * fq >= nf) return;
+    uint32_t reg[4][8];    // [feature in quad][sample group r]
+#pragma unroll
+    for (int r = 0; r < 8; ++r) {
+        const uint4 c = tile[fq][pack_cell(lane, r)];
+        reg[0][r] = c.x; reg[1][r] = c.y; reg[2][r] = c.z; reg[3][r] = c.w;
+    }
+#pragma unroll
+    for (int fi = 0; fi < 4; ++fi) {
+        if (4 * fq + fi >= nf) break;
         uint32_t lo7[8];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) lo7[i] = r[i] & 0x7f7f7f7fu;
-        uint32_t* out = xp + (long long)(f0 + fl) * th.b * W + q;
+        for (int i = 0; i < 8; ++i) lo7[i] = reg[fi][i] & 0x7f7f7f7fu;
+        uint32_t* out = xp + (long long)(f0 + 4 * fq + fi) * th.b * W + q;
         for (int i = 0; i < th.b; ++i) {
             const uint32_t C = sC[i];
             uint32_t word = 0u;
             if (sOr[i]) {   // T < 127: OR form (warp-uniform branch)
 #pragma unroll
                 for (int i8 = 0; i8 < 8; ++i8) {
-                    const uint32_t hb = (r[i8] | (lo7[i8] + C)) & 0x80808080u;
+                    const uint32_t hb = (reg[fi][i8] | (lo7[i8] + C)) & 0x80808080u;
                     word += i8 < 7 ? __umulhi(hb, 1u << ((25 + i8) & 31)) : hb;   // disjoint bits
                 }
             } else {        // T >= 127: AND form
 #pragma unroll
                 for (int i8 = 0; i8 < 8; ++i8) {
-                    const uint32_t hb = (r[i8] & (lo7[i8] + C)) & 0x80808080u;
+                    const uint32_t hb = (reg[fi][i8] & (lo7[i8] + C)) & 0x80808080u;
                     word += i8 < 7 ? __umulhi(hb, 1u << ((25 + i8) & 31)) : hb;
                 }
             }
