@@ -402,6 +402,24 @@ def test_empty_batch_is_a_noop():
     assert torch.all(dth == 0)
     xp = torch.empty(10, 0, dtype=torch.int32, device="cuda")
     bl.bitlogic_pack_bits(torch.empty(0, 5, dtype=torch.uint8, device="cuda"), [1, 2], xp)
+    # straight-through node, routing: an empty batch leaves the batch sums at
+    # zero, and the routing forward still gives the slot probabilities
+    dth = torch.full((w, 4), 7.0, device="cuda")
+    bl.bitlogic_lut_backward_node(X, conn, theta, dth, node="st", dY=torch.empty(w, 0, device="cuda"))
+    assert torch.all(dth == 0)
+    slots, Kc = 6, 3
+    cand = synth.candidate_pools(slots, Kc, w_in, seed=2)
+    r = synth.table_logits(slots, Kc, seed=3)
+    prob = torch.full((slots, Kc), np.nan, device="cuda")
+    bl.bitlogic_route_forward(X, dev(cand), dev(r), torch.empty(slots, 0, device="cuda"), prob)
+    check_fwd(prob, oracle.route_forward(np.zeros((w_in, 1)), cand, r)[1], "prob of an empty batch")
+    dr = torch.full((slots, Kc), 7.0, device="cuda")
+    bl.bitlogic_route_backward(X, dev(cand), dev(r), torch.empty(slots, 0, device="cuda"), dr)
+    assert torch.all(dr == 0)
+    hist = torch.zeros(256, dtype=torch.int64, device="cuda")
+    bl.bitlogic_pixel_histogram(torch.empty(0, dtype=torch.uint8, device="cuda"), hist)
+    assert int(hist.sum()) == 0
+    no_device_error()
 
 
 # -------------------------------------------------------------------- head --
