@@ -652,15 +652,25 @@ def run_e2e(args, st, hi, wl, B, use_graph=True):
 
 # -------------------------------------------------- oracle (CPU) legs --
 
+_NETWORKS = {}
+
+
+def _network(wl):
+    """The workload's network (drawn once per process)."""
+    if wl.name not in _NETWORKS:
+        _NETWORKS[wl.name] = synth.routed_network(wl, seed=0) if wl.Kc else synth.network(wl, seed=0)
+    return _NETWORKS[wl.name]
+
+
 def oracle_train_rate(wl, samples: int, seed: int = 0, node: str = "soft"):
     import oracle
     x, lab = synth.blob_batch(samples, wl.d, wl.classes, wl.sigma, seed=3000 + seed)
     if wl.Kc:
-        params = synth.routed_network(wl, seed=0)
+        params = _network(wl)
         t0 = time.perf_counter()
         oracle.routed_train_step(x.numpy(), lab.numpy(), wl.thresholds, *params, wl.classes, wl.tau, node=node)
         return samples / (time.perf_counter() - t0)
-    conn1, th1, conn2, th2 = synth.network(wl, seed=0)
+    conn1, th1, conn2, th2 = _network(wl)
     t0 = time.perf_counter()
     oracle.train_step(x.numpy(), lab.numpy(), wl.thresholds, conn1, th1, conn2, th2,
                       wl.classes, wl.tau, node=node)
@@ -669,7 +679,7 @@ def oracle_train_rate(wl, samples: int, seed: int = 0, node: str = "soft"):
 
 def oracle_hard_rate(wl, samples: int, seed: int = 0):
     import oracle
-    conn1, th1, conn2, th2 = synth.network(wl, seed=0)
+    conn1, th1, conn2, th2 = synth.network(wl, seed=0) if wl.Kc else _network(wl)
     t1, t2 = oracle.binarize_tables(th1), oracle.binarize_tables(th2)
     x, _ = synth.blob_batch(samples, wl.d, wl.classes, wl.sigma, seed=4000 + seed)
     t0 = time.perf_counter()
@@ -709,9 +719,12 @@ def run_reference(args):
     hard_only = wl.name.startswith("hard_")
     fn = oracle_hard_rate if hard_only else (lambda w_, n_, seed=0: oracle_train_rate(w_, n_, seed, args.node))
     lo = 32 if hard_only else 2
-    # size one step to about 1-2 s of oracle work
-    r0 = fn(wl, lo)
-    n = max(lo, int(r0 * 1.5) // lo * lo)
+    # size one step so that the whole run (warm-up and timed steps) takes
+    # about two minutes of oracle work, at most 1.5 s per step; the rate is
+    # calibrated on a sample large enough to amortise the per-call set-up
+    per_step_s = min(1.5, 120.0 / max(1, args.steps + args.warmup))
+    r0 = fn(wl, min(wl.batch, 4096 if hard_only else 64))
+    n = max(lo, int(r0 * per_step_s) // lo * lo)
     n = min(n, wl.batch)
     for i in range(args.warmup):
         fn(wl, lo, seed=100 + i)
