@@ -52,8 +52,9 @@ void oracle_set_threads(int n) {
  * range (§3 "Encoders and heads"; App. A "Scope of the prior-method
  * reproduction" places them at i/(b+1)).  On uint8 pixels the real threshold
  * is 256*i/(b+1); a strict comparison p > 256*i/(b+1) equals p > floor(...).
- * parity unpinned: the paper states no integer thresholds; the tests pin the
- * three workload sets to this reading. */
+ * The paper states no integer thresholds; the tests pin this reading to the
+ * threshold sets the workloads state ({64, 128, 192} for b = 3, multiples of
+ * 32 for b = 7, of 16 for b = 15). */
 void oracle_linear_thresholds(int32_t b, int32_t* thr) {
     for (int32_t i = 1; i <= b; ++i) thr[i - 1] = (int32_t)((256 * i) / (b + 1));
 }
