@@ -172,8 +172,9 @@ def call_work_routed(wl, B):
     s1, s2 = w1 * k, w2 * k
     f = 4
     return {
-        "encode": (B * d + f * win * B, 0),
-        "route1": (f * (win * B + s1 * B + 2 * s1 * Kc), Kc * s1 * B),
+        # the encoder's wires are bytes in the routed step (layer 1 gathers them)
+        "encode": (B * d + win * B, 0),
+        "route1": (win * B + f * (s1 * B + 2 * s1 * Kc), Kc * s1 * B),
         "forward1": (f * (s1 * B + w1 * B + w1 * K + w1 * k), (2 * (K - 1) + k) * w1 * B),
         "route2": (f * (w1 * B + s2 * B + 2 * s2 * Kc), Kc * s2 * B),
         "forward2": (f * (s2 * B + w2 * B + w2 * K + w2 * k), (2 * (K - 1) + k) * w2 * B),
@@ -181,7 +182,7 @@ def call_work_routed(wl, B):
         "backward2": (f * (s2 * B + C * B + s2 * B + 2 * w2 * K + w2 * k), (4 * (K - 1) + K) * w2 * B),
         "route_bwd2": (f * (w1 * B + 2 * s2 * B + w1 * B + 3 * s2 * Kc), 2 * Kc * s2 * B),
         "backward1": (f * (s1 * B + w1 * B + s1 * B + 2 * w1 * K + w1 * k), (4 * (K - 1) + K) * w1 * B),
-        "route_bwd1": (f * (win * B + s1 * B + 2 * s1 * Kc), Kc * s1 * B),
+        "route_bwd1": (win * B + f * (s1 * B + 2 * s1 * Kc), Kc * s1 * B),
         "binarize": (f * (w1 * K + w2 * K) + 8 * (w1 + w2), 0),
         "pack": (B * d + f * win * ((B + 31) // 32), 0),
         "hard1": (f * (win * ((B + 31) // 32) + w1 * ((B + 31) // 32) + w1 * k) + 8 * w1,
@@ -274,7 +275,7 @@ KERNEL_OF_CALL = {
     "binarize": "binarize_kernel (x2)", "pack": "pack_bits_kernel", "hard1": "hard_layer_staged_kernel<k>",
     "hard2": "hard_head_staged_kernel<k> + argmax_kernel",
     "route1": "route_forward_vec_kernel<KC>", "route2": "route_forward_vec_kernel<KC>",
-    "route_bwd2": "route_dr_kernel + route_dx_kernel", "route_bwd1": "route_dr_kernel<KC>",
+    "route_bwd2": "route_dr_kernel + route_dx_kernel", "route_bwd1": "route_dr_kernel<KC> (byte rows)",
 }
 
 

@@ -85,6 +85,13 @@ int bitlogic_encode_thermometer(const uint8_t* x, int64_t B, int32_t d,
                                 const uint8_t* thr_host, int32_t b,
                                 float* bits, cudaStream_t stream);
 
+/* The same wires as bytes (0 or 1): bits device uint8 [d*b][B], for
+ * consumers that gather the encoder rows and want a quarter of the bytes
+ * (bitlogic_route_forward_u8). */
+int bitlogic_encode_thermometer_u8(const uint8_t* x, int64_t B, int32_t d,
+                                   const uint8_t* thr_host, int32_t b,
+                                   uint8_t* bits, cudaStream_t stream);
+
 /* Distributive (quantile) thermometer fit (§3 "Encoders and heads"; App. A
  * "Initialization": thresholds fit once from the empirical pixel quantiles
  * of the training split, over the globally flattened pixels, App. B).  Two
@@ -251,6 +258,15 @@ int bitlogic_route_backward(const float* X, int32_t w_in, int64_t B, const int32
                             cudaStream_t stream);
 int bitlogic_route_snap(const int32_t* cand, const float* r, int32_t slots, int32_t Kc, int32_t* conn,
                         cudaStream_t stream);
+
+/* Routing over a layer input held as bytes (X device uint8 [w_in][B], the
+ * values as numbers, e.g. the 0/1 wires of bitlogic_encode_thermometer_u8):
+ * the same Xr, prob and dr as the fp32 calls on the same values (bit for
+ * bit); no input gradient (a byte input is not trained). */
+int bitlogic_route_forward_u8(const uint8_t* X, int32_t w_in, int64_t B, const int32_t* cand, const float* r,
+                              int32_t slots, int32_t Kc, float* Xr, float* prob, cudaStream_t stream);
+int bitlogic_route_backward_u8(const uint8_t* X, int32_t w_in, int64_t B, const int32_t* cand, const float* r,
+                               int32_t slots, int32_t Kc, const float* G, float* dr, cudaStream_t stream);
 
 /* Bytes of workspace bitlogic_head_loss needs. */
 size_t bitlogic_head_loss_workspace(int64_t B, int32_t C);

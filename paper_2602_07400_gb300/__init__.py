@@ -31,6 +31,7 @@ __all__ = [
     "bitlogic_head_loss", "bitlogic_binarize_tables", "bitlogic_pack_bits",
     "bitlogic_hard_forward", "bitlogic_build_csr", "bitlogic_csr_positions", "bitlogic_device_error",
     "bitlogic_adamw_update", "bitlogic_route_forward", "bitlogic_route_backward", "bitlogic_route_snap",
+    "bitlogic_route_forward_u8", "bitlogic_route_backward_u8", "bitlogic_encode_thermometer_u8",
     "bitlogic_pixel_histogram", "bitlogic_quantile_thresholds", "bitlogic_lut_forward_node", "bitlogic_lut_backward_node", "NODE_FORMS",
     "bitlogic_status_string", "bitlogic_version", "LIB_PATH",
 ]
@@ -66,6 +67,9 @@ _SIGS = {
     "bitlogic_route_forward": ([_P, _I32, _I64, _P, _P, _I32, _I32, _P, _P, _P], ctypes.c_int),
     "bitlogic_route_backward": ([_P, _I32, _I64, _P, _P, _I32, _I32, _P, _P, _P, _P, _P, _P, _P], ctypes.c_int),
     "bitlogic_route_snap": ([_P, _P, _I32, _I32, _P, _P], ctypes.c_int),
+    "bitlogic_route_forward_u8": ([_P, _I32, _I64, _P, _P, _I32, _I32, _P, _P, _P], ctypes.c_int),
+    "bitlogic_route_backward_u8": ([_P, _I32, _I64, _P, _P, _I32, _I32, _P, _P, _P], ctypes.c_int),
+    "bitlogic_encode_thermometer_u8": ([_P, _I64, _I32, _P, _I32, _P, _P], ctypes.c_int),
     "bitlogic_quantile_thresholds": ([_P, _I32, _P], ctypes.c_int),
     "bitlogic_lut_forward_node": ([_P, _I32, _I64, _P, _P, _I32, _I32, _I32, _P, _P], ctypes.c_int),
     "bitlogic_lut_backward_workspace": ([_I32, _I64, _I32, _I32, _I32], _SZ),
@@ -166,19 +170,52 @@ def bitlogic_encode_thermometer(x: torch.Tensor, thresholds, bits: torch.Tensor,
         _ptr(x), B, d, buf, b, _ptr(bits), _stream(stream)))
 
 
+def bitlogic_encode_thermometer_u8(x: torch.Tensor, thresholds, bits: torch.Tensor, stream=None):
+    B, d = x.shape
+    buf, b = _thr_buf(thresholds)
+    _need(x, "x", torch.uint8, (B, d))
+    _need(bits, "bits", torch.uint8, (d * b, B))
+    _check("bitlogic_encode_thermometer_u8", load().bitlogic_encode_thermometer_u8(
+        _ptr(x), B, d, buf, b, _ptr(bits), _stream(stream)))
+
+
+def bitlogic_route_forward_u8(X: torch.Tensor, cand: torch.Tensor, r: torch.Tensor, Xr: torch.Tensor,
+                              prob: Optional[torch.Tensor] = None, stream=None):
+    """bitlogic_route_forward over a uint8 layer input [w_in, B]."""
+    _route_forward("bitlogic_route_forward_u8", torch.uint8, X, cand, r, Xr, prob, stream)
+
+
+def bitlogic_route_backward_u8(X: torch.Tensor, cand: torch.Tensor, r: torch.Tensor, G: torch.Tensor,
+                               dr: torch.Tensor, stream=None):
+    """dr of a routing over a uint8 layer input (no input gradient)."""
+    w_in, B = X.shape
+    slots, Kc = cand.shape
+    _need(X, "X", torch.uint8, (w_in, B))
+    _need(cand, "cand", torch.int32, (slots, Kc))
+    _need(r, "r", torch.float32, (slots, Kc))
+    _need(G, "G", torch.float32, (slots, B))
+    _need(dr, "dr", torch.float32, (slots, Kc))
+    _check("bitlogic_route_backward_u8", load().bitlogic_route_backward_u8(
+        _ptr(X), w_in, B, _ptr(cand), _ptr(r), slots, Kc, _ptr(G), _ptr(dr), _stream(stream)))
+
+
 def bitlogic_route_forward(X: torch.Tensor, cand: torch.Tensor, r: torch.Tensor, Xr: torch.Tensor,
                            prob: Optional[torch.Tensor] = None, stream=None):
     """Slot inputs of learnable routing: cand int32 [slots, Kc], r fp32
     [slots, Kc] -> Xr fp32 [slots, B] (and the probabilities into prob)."""
+    _route_forward("bitlogic_route_forward", torch.float32, X, cand, r, Xr, prob, stream)
+
+
+def _route_forward(fn, dtype, X, cand, r, Xr, prob, stream):
     w_in, B = X.shape
     slots, Kc = cand.shape
-    _need(X, "X", torch.float32, (w_in, B))
+    _need(X, "X", dtype, (w_in, B))
     _need(cand, "cand", torch.int32, (slots, Kc))
     _need(r, "r", torch.float32, (slots, Kc))
     _need(Xr, "Xr", torch.float32, (slots, B))
     if prob is not None:
         _need(prob, "prob", torch.float32, (slots, Kc))
-    _check("bitlogic_route_forward", load().bitlogic_route_forward(
+    _check(fn, getattr(load(), fn)(
         _ptr(X), w_in, B, _ptr(cand), _ptr(r), slots, Kc, _ptr(Xr), _ptr(prob), _stream(stream)))
 
 

@@ -20,9 +20,21 @@ namespace {
 constexpr int kEncTS = 64;   // samples per tile
 constexpr int kEncTF = 32;   // features per tile
 
+// Output wires as fp32 (the soft layers' input) or as bytes (byte-row
+// consumers such as the routing gathers).
+__device__ __forceinline__ void put_bit(float* p, bool v) { *p = v ? 1.0f : 0.0f; }
+__device__ __forceinline__ void put_bit(uint8_t* p, bool v) { *p = v ? 1u : 0u; }
+__device__ __forceinline__ void put_bits4(float* p, bool a, bool b, bool c, bool d) {
+    *reinterpret_cast<float4*>(p) = make_float4(a ? 1.0f : 0.0f, b ? 1.0f : 0.0f, c ? 1.0f : 0.0f, d ? 1.0f : 0.0f);
+}
+__device__ __forceinline__ void put_bits4(uint8_t* p, bool a, bool b, bool c, bool d) {
+    *reinterpret_cast<uint32_t*>(p) = (uint32_t)a | ((uint32_t)b << 8) | ((uint32_t)c << 16) | ((uint32_t)d << 24);
+}
+
+template <typename OutT>
 __global__ void __launch_bounds__(256)
 encode_soft_kernel(const uint8_t* __restrict__ x, long long B, int d, Thresholds th,
-                   float* __restrict__ bits) {
+                   OutT* __restrict__ bits) {
     __shared__ uint8_t tile[kEncTF][kEncTS + 4];   // feature-major
     __shared__ uint32_t sT[32];
     if (threadIdx.x < th.b) sT[threadIdx.x] = threshold_at(th, threadIdx.x);
@@ -47,7 +59,7 @@ encode_soft_kernel(const uint8_t* __restrict__ x, long long B, int d, Thresholds
     if (s >= B) return;
     for (int r = tr; r < rows; r += 4) {
         const int f = r / th.b, i = r - f * th.b;
-        bits[((long long)(f0 + f) * th.b + i) * B + s] = tile[f][tsl] > sT[i] ? 1.0f : 0.0f;
+        put_bit(bits + ((long long)(f0 + f) * th.b + i) * B + s, tile[f][tsl] > sT[i]);
     }
 }
 
@@ -58,9 +70,10 @@ encode_soft_kernel(const uint8_t* __restrict__ x, long long B, int d, Thresholds
 // as one float4 (512 contiguous bytes per warp).
 constexpr int kEncVS = 128;   // samples per tile (vector form)
 
+template <typename OutT>
 __global__ void __launch_bounds__(256)
 encode_soft_vec_kernel(const uint8_t* __restrict__ x, long long B, int d, Thresholds th,
-                       float* __restrict__ bits, bool vec16) {
+                       OutT* __restrict__ bits, bool vec16) {
     __shared__ __align__(16) uint8_t tile[kEncTF][kEncVS];   // feature-major
     __shared__ uint32_t sT[32];
     if (threadIdx.x < th.b) sT[threadIdx.x] = threshold_at(th, threadIdx.x);
@@ -94,9 +107,8 @@ encode_soft_vec_kernel(const uint8_t* __restrict__ x, long long B, int d, Thresh
         const int f = r / th.b, i = r - f * th.b;
         const uint32_t q = *reinterpret_cast<const uint32_t*>(&tile[f][4 * u]);
         const uint32_t T = sT[i];
-        const float4 o = make_float4((q & 0xffu) > T ? 1.0f : 0.0f, ((q >> 8) & 0xffu) > T ? 1.0f : 0.0f,
-                                     ((q >> 16) & 0xffu) > T ? 1.0f : 0.0f, (q >> 24) > T ? 1.0f : 0.0f);
-        *reinterpret_cast<float4*>(bits + ((long long)(f0 + f) * th.b + i) * B + s) = o;
+        put_bits4(bits + ((long long)(f0 + f) * th.b + i) * B + s, (q & 0xffu) > T, ((q >> 8) & 0xffu) > T,
+                  ((q >> 16) & 0xffu) > T, (q >> 24) > T);
     }
 }
 
@@ -233,9 +245,10 @@ using namespace bitlogic;
 
 BITLOGIC_ERROR_READER(encode)
 
-extern "C" int bitlogic_encode_thermometer(const uint8_t* x, int64_t B, int32_t d,
-                                           const uint8_t* thr_host, int32_t b,
-                                           float* bits, cudaStream_t stream) {
+namespace {
+template <typename OutT>
+int encode_impl(const uint8_t* x, int64_t B, int32_t d, const uint8_t* thr_host, int32_t b, OutT* bits,
+                cudaStream_t stream) {
     Thresholds th;
     int st = make_thresholds(thr_host, b, &th);
     if (st) return st;
@@ -247,14 +260,27 @@ extern "C" int bitlogic_encode_thermometer(const uint8_t* x, int64_t B, int32_t 
         if (gy > 65535) return BITLOGIC_ERR_SHAPE;
         const bool vec16 = (d % 16 == 0) && aligned16(x);
         dim3 grid((unsigned)((d + kEncTF - 1) / kEncTF), (unsigned)gy);
-        encode_soft_vec_kernel<<<grid, 256, 0, stream>>>(x, B, d, th, bits, vec16);
+        encode_soft_vec_kernel<OutT><<<grid, 256, 0, stream>>>(x, B, d, th, bits, vec16);
         return launch_status();
     }
     const long long gy = (B + kEncTS - 1) / kEncTS;
     if (gy > 65535) return BITLOGIC_ERR_SHAPE;
     dim3 grid((unsigned)((d + kEncTF - 1) / kEncTF), (unsigned)gy);
-    encode_soft_kernel<<<grid, 256, 0, stream>>>(x, B, d, th, bits);
+    encode_soft_kernel<OutT><<<grid, 256, 0, stream>>>(x, B, d, th, bits);
     return launch_status();
+}
+}  // namespace
+
+extern "C" int bitlogic_encode_thermometer(const uint8_t* x, int64_t B, int32_t d,
+                                           const uint8_t* thr_host, int32_t b,
+                                           float* bits, cudaStream_t stream) {
+    return encode_impl(x, B, d, thr_host, b, bits, stream);
+}
+
+extern "C" int bitlogic_encode_thermometer_u8(const uint8_t* x, int64_t B, int32_t d,
+                                              const uint8_t* thr_host, int32_t b,
+                                              uint8_t* bits, cudaStream_t stream) {
+    return encode_impl(x, B, d, thr_host, b, bits, stream);
 }
 
 extern "C" int bitlogic_pack_bits(const uint8_t* x, int64_t N, int32_t d,

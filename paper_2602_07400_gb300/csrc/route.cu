@@ -15,11 +15,17 @@
 //   dX[c][s] = sum over candidate edges (e, m) with cand[e][m] == c, in
 //              increasing e*Kc + m, of p_e[m] G[e][s]   (CSR, no atomics).
 //
+// Layer inputs are fp32 rows or byte rows (the encoder's 0/1 wires); the
+// forward reads byte rows 16 samples per lane and load (the dr kernel keeps
+// 4: at 16 it needs twice the registers and measured slower).
+//
 // Kernels: the slot's softmax is computed by its warp (candidate m on lane
 // m, Kc <= 32) and held in registers; the gathers stream KC 16-byte loads per
 // lane and step (KC = Kc rounded up to a power of two, the padding having
 // weight 0 on the slot's first candidate).  The pools of a layer read a few
 // thousand distinct rows, which stay in L2.
+#include <type_traits>
+
 #include "common.cuh"
 
 namespace bitlogic {
@@ -28,6 +34,17 @@ namespace {
 constexpr int kRouteWarps = 8;
 
 __device__ __forceinline__ float4 ldg4r(const float* p) { return __ldg(reinterpret_cast<const float4*>(p)); }
+
+// Layer inputs come as fp32 rows or as byte rows (the encoder's 0/1 wires,
+// a quarter of the bytes to gather): one value and four consecutive values
+// of a row, as floats.
+__device__ __forceinline__ float in_value(const float* p) { return __ldg(p); }
+__device__ __forceinline__ float in_value(const uint8_t* p) { return (float)__ldg(p); }
+__device__ __forceinline__ float4 in_quad(const float* p) { return ldg4r(p); }
+__device__ __forceinline__ float4 in_quad(const uint8_t* p) {
+    const uint32_t w = __ldg(reinterpret_cast<const uint32_t*>(p));
+    return make_float4((float)(w & 0xffu), (float)((w >> 8) & 0xffu), (float)((w >> 16) & 0xffu), (float)(w >> 24));
+}
 
 // Softmax of the slot's logits on lanes m < Kc (other lanes 0), the lane's
 // candidate row (range-checked; a bad index is read as row 0 and flagged).
@@ -55,9 +72,9 @@ __device__ __forceinline__ void slot_softmax(const int* __restrict__ cand, const
 
 // Forward, vector path (B % 4 == 0, 16-byte aligned X and Xr): one warp per
 // (slot, batch chunk), 4 consecutive samples per lane and step.
-template <int KC>
+template <int KC, typename T>
 __global__ void __launch_bounds__(kRouteWarps * 32)
-route_forward_vec_kernel(const float* __restrict__ X, int w_in, long long B, const int* __restrict__ cand,
+route_forward_vec_kernel(const T* __restrict__ X, int w_in, long long B, const int* __restrict__ cand,
                          const float* __restrict__ r, long long slots, int Kc, float* __restrict__ Xr,
                          float* __restrict__ prob, long long chunk) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -68,7 +85,7 @@ route_forward_vec_kernel(const float* __restrict__ X, int w_in, long long B, con
     slot_softmax(cand, r, e, Kc, w_in, lane, p, c);
     if (prob && blockIdx.y == 0 && lane < Kc) prob[e * Kc + lane] = p;
     float pm[KC];
-    const float* row[KC];
+    const T* row[KC];
     const int c0 = __shfl_sync(0xffffffffu, c, 0);
 #pragma unroll
     for (int m = 0; m < KC; ++m) {
@@ -87,7 +104,7 @@ route_forward_vec_kernel(const float* __restrict__ X, int w_in, long long B, con
         for (int m0 = 0; m0 < KC; m0 += G) {
             float4 v[G];
 #pragma unroll
-            for (int u = 0; u < G; ++u) v[u] = ldg4r(row[m0 + u] + s);
+            for (int u = 0; u < G; ++u) v[u] = in_quad(row[m0 + u] + s);
 #pragma unroll
             for (int u = 0; u < G; ++u) {
                 const float q = pm[m0 + u];
@@ -101,9 +118,63 @@ route_forward_vec_kernel(const float* __restrict__ X, int w_in, long long B, con
     }
 }
 
-// Forward, scalar path (any B and alignment): one sample per lane and step.
+// Forward over byte rows, 16 consecutive samples per lane and step (one
+// 16-byte load per candidate row: a quarter of the load instructions of the
+// 4-sample form).  Needs B % 16 == 0 and 16-byte aligned X and Xr.
+template <int KC>
 __global__ void __launch_bounds__(kRouteWarps * 32)
-route_forward_kernel(const float* __restrict__ X, int w_in, long long B, const int* __restrict__ cand,
+route_forward_bytes16_kernel(const uint8_t* __restrict__ X, int w_in, long long B, const int* __restrict__ cand,
+                             const float* __restrict__ r, long long slots, int Kc, float* __restrict__ Xr,
+                             float* __restrict__ prob, long long chunk) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const long long e = (long long)blockIdx.x * kRouteWarps + warp;
+    if (e >= slots) return;
+    float p;
+    int c;
+    slot_softmax(cand, r, e, Kc, w_in, lane, p, c);
+    if (prob && blockIdx.y == 0 && lane < Kc) prob[e * Kc + lane] = p;
+    float pm[KC];
+    const uint8_t* row[KC];
+    const int c0 = __shfl_sync(0xffffffffu, c, 0);
+#pragma unroll
+    for (int m = 0; m < KC; ++m) {
+        pm[m] = __shfl_sync(0xffffffffu, p, m & 31);
+        const int cm = __shfl_sync(0xffffffffu, c, m & 31);
+        row[m] = X + (long long)(m < Kc ? cm : c0) * B;
+        if (m >= Kc) pm[m] = 0.f;
+    }
+    const long long s0 = (long long)blockIdx.y * chunk;
+    const long long s1 = min(B, s0 + chunk);
+    float* out = Xr + e * B;
+    for (long long s = s0 + 16 * lane; s < s1; s += 512) {
+        float acc[16];
+#pragma unroll
+        for (int t = 0; t < 16; ++t) acc[t] = 0.f;
+        constexpr int G = KC < 4 ? KC : 4;   // loads issued together
+#pragma unroll
+        for (int m0 = 0; m0 < KC; m0 += G) {
+            uint4 v[G];
+#pragma unroll
+            for (int u = 0; u < G; ++u) v[u] = __ldg(reinterpret_cast<const uint4*>(row[m0 + u] + s));
+#pragma unroll
+            for (int u = 0; u < G; ++u) {
+                const float q = pm[m0 + u];
+                const uint32_t w[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+#pragma unroll
+                for (int t = 0; t < 16; ++t)
+                    acc[t] = fmaf(q, (float)((w[t >> 2] >> (8 * (t & 3))) & 0xffu), acc[t]);
+            }
+        }
+#pragma unroll
+        for (int t = 0; t < 16; t += 4)
+            *reinterpret_cast<float4*>(out + s + t) = make_float4(acc[t], acc[t + 1], acc[t + 2], acc[t + 3]);
+    }
+}
+
+// Forward, scalar path (any B and alignment): one sample per lane and step.
+template <typename T>
+__global__ void __launch_bounds__(kRouteWarps * 32)
+route_forward_kernel(const T* __restrict__ X, int w_in, long long B, const int* __restrict__ cand,
                      const float* __restrict__ r, long long slots, int Kc, float* __restrict__ Xr,
                      float* __restrict__ prob, long long chunk) {
     __shared__ float sp[kRouteWarps][32];
@@ -122,19 +193,19 @@ route_forward_kernel(const float* __restrict__ X, int w_in, long long B, const i
     const long long s1 = min(B, s0 + chunk);
     for (long long s = s0 + lane; s < s1; s += 32) {
         float acc = 0.f;
-        for (int m = 0; m < Kc; ++m) acc = fmaf(sp[warp][m], __ldg(X + (long long)sc[warp][m] * B + s), acc);
+        for (int m = 0; m < Kc; ++m) acc = fmaf(sp[warp][m], in_value(X + (long long)sc[warp][m] * B + s), acc);
         Xr[e * B + s] = acc;
     }
 }
 
 // dr: one warp per slot over the whole batch.  Each lane accumulates its
 // samples' A_m (m < KC), then the warp sums every A_m with a fixed butterfly.
-// The vector path holds the candidate rows as 32-bit offsets in 16-byte
-// units (needs w_in B / 4 < 2^32) and is held to 64 registers (four blocks
+// The vector path holds the candidate rows as 32-bit offsets in units of 4
+// samples (needs w_in B / 4 < 2^32) and is held to 64 registers (four blocks
 // per SM; two for 32 candidates), so that more warps keep gathers in flight.
-template <int KC, bool VEC>
+template <int KC, bool VEC, typename T>
 __global__ void __launch_bounds__(kRouteWarps * 32, VEC ? (KC <= 16 ? 4 : 2) : 1)
-route_dr_kernel(const float* __restrict__ X, int w_in, long long B, const int* __restrict__ cand,
+route_dr_kernel(const T* __restrict__ X, int w_in, long long B, const int* __restrict__ cand,
                 const float* __restrict__ r, long long slots, int Kc, const float* __restrict__ G,
                 float* __restrict__ dr) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -149,7 +220,6 @@ route_dr_kernel(const float* __restrict__ X, int w_in, long long B, const int* _
     for (int m = 0; m < KC; ++m) A[m] = 0.f;
     const float* g = G + e * B;
     if constexpr (VEC) {
-        const float4* X4 = reinterpret_cast<const float4*>(X);
         const unsigned B4 = (unsigned)(B / 4);
         unsigned row[KC];
 #pragma unroll
@@ -165,7 +235,7 @@ route_dr_kernel(const float* __restrict__ X, int w_in, long long B, const int* _
             for (int m0 = 0; m0 < KC; m0 += GR) {
                 float4 v[GR];
 #pragma unroll
-                for (int u = 0; u < GR; ++u) v[u] = __ldg(X4 + row[m0 + u] + s4);
+                for (int u = 0; u < GR; ++u) v[u] = in_quad(X + 4 * (size_t)(row[m0 + u] + s4));
 #pragma unroll
                 for (int u = 0; u < GR; ++u) {
                     float a = A[m0 + u];
@@ -178,7 +248,7 @@ route_dr_kernel(const float* __restrict__ X, int w_in, long long B, const int* _
             }
         }
     } else {
-        const float* row[KC];
+        const T* row[KC];
 #pragma unroll
         for (int m = 0; m < KC; ++m) {
             const int cm = __shfl_sync(0xffffffffu, c, m & 31);
@@ -187,7 +257,7 @@ route_dr_kernel(const float* __restrict__ X, int w_in, long long B, const int* _
         for (long long s = lane; s < B; s += 32) {
             const float gv = __ldg(g + s);
 #pragma unroll
-            for (int m = 0; m < KC; ++m) A[m] = fmaf(gv, __ldg(row[m] + s), A[m]);
+            for (int m = 0; m < KC; ++m) A[m] = fmaf(gv, in_value(row[m] + s), A[m]);
         }
     }
 #pragma unroll
@@ -322,8 +392,8 @@ int check_route(const void* X, int32_t w_in, int64_t B, const void* cand, const 
     return BITLOGIC_OK;
 }
 
-template <int KC>
-int launch_route_forward(const float* X, int w_in, long long B, const int* cand, const float* r, long long slots,
+template <int KC, typename T>
+int launch_route_forward(const T* X, int w_in, long long B, const int* cand, const float* r, long long slots,
                          int Kc, float* Xr, float* prob, bool vec, cudaStream_t st) {
     // batch chunks of 1024 samples (8 steps per warp)
     const long long chunk = 1024;
@@ -331,22 +401,74 @@ int launch_route_forward(const float* X, int w_in, long long B, const int* cand,
     if (gy > 65535) return BITLOGIC_ERR_SHAPE;
     dim3 grid((unsigned)((slots + kRouteWarps - 1) / kRouteWarps), (unsigned)gy);
     if (vec)
-        route_forward_vec_kernel<KC><<<grid, kRouteWarps * 32, 0, st>>>(X, w_in, B, cand, r, slots, Kc, Xr, prob,
-                                                                        chunk);
+        route_forward_vec_kernel<KC, T><<<grid, kRouteWarps * 32, 0, st>>>(X, w_in, B, cand, r, slots, Kc, Xr,
+                                                                           prob, chunk);
     else
-        route_forward_kernel<<<grid, kRouteWarps * 32, 0, st>>>(X, w_in, B, cand, r, slots, Kc, Xr, prob, chunk);
+        route_forward_kernel<T><<<grid, kRouteWarps * 32, 0, st>>>(X, w_in, B, cand, r, slots, Kc, Xr, prob, chunk);
     return launch_status();
 }
 
-template <int KC>
-int launch_route_dr(const float* X, int w_in, long long B, const int* cand, const float* r, long long slots, int Kc,
+template <int KC, typename T>
+int launch_route_dr(const T* X, int w_in, long long B, const int* cand, const float* r, long long slots, int Kc,
                     const float* G, float* dr, bool vec, cudaStream_t st) {
     const unsigned blocks = (unsigned)((slots + kRouteWarps - 1) / kRouteWarps);
     if (vec)
-        route_dr_kernel<KC, true><<<blocks, kRouteWarps * 32, 0, st>>>(X, w_in, B, cand, r, slots, Kc, G, dr);
+        route_dr_kernel<KC, true, T><<<blocks, kRouteWarps * 32, 0, st>>>(X, w_in, B, cand, r, slots, Kc, G, dr);
     else
-        route_dr_kernel<KC, false><<<blocks, kRouteWarps * 32, 0, st>>>(X, w_in, B, cand, r, slots, Kc, G, dr);
+        route_dr_kernel<KC, false, T><<<blocks, kRouteWarps * 32, 0, st>>>(X, w_in, B, cand, r, slots, Kc, G, dr);
     return launch_status();
+}
+
+// Entry-point bodies shared by the fp32 and byte-row inputs.
+template <int KC>
+int launch_route_forward_bytes16(const uint8_t* X, int w_in, long long B, const int* cand, const float* r,
+                                 long long slots, int Kc, float* Xr, float* prob, cudaStream_t st) {
+    const long long chunk = 1024;
+    const long long gy = (B + chunk - 1) / chunk;
+    if (gy > 65535) return BITLOGIC_ERR_SHAPE;
+    dim3 grid((unsigned)((slots + kRouteWarps - 1) / kRouteWarps), (unsigned)gy);
+    route_forward_bytes16_kernel<KC><<<grid, kRouteWarps * 32, 0, st>>>(X, w_in, B, cand, r, slots, Kc, Xr, prob,
+                                                                        chunk);
+    return launch_status();
+}
+
+template <typename T>
+int route_forward_impl(const T* X, int32_t w_in, int64_t B, const int32_t* cand, const float* r, int32_t slots,
+                       int32_t Kc, float* Xr, float* prob, cudaStream_t stream) {
+    int st = check_route(X, w_in, B, cand, r, slots, Kc);
+    if (st) return st;
+    if (B == 0 && !prob) return BITLOGIC_OK;
+    if (B > 0 && !Xr) return BITLOGIC_ERR_NULL;
+    const bool vec = (B % 4 == 0) && aligned16(X) && aligned16(Xr);
+    if constexpr (std::is_same<T, uint8_t>::value) {
+        if (B > 0 && B % 16 == 0 && vec) {   // byte rows: 16 samples per lane and load
+            if (Kc <= 4) return launch_route_forward_bytes16<4>(X, w_in, B, cand, r, slots, Kc, Xr, prob, stream);
+            if (Kc <= 8) return launch_route_forward_bytes16<8>(X, w_in, B, cand, r, slots, Kc, Xr, prob, stream);
+            if (Kc <= 16)
+                return launch_route_forward_bytes16<16>(X, w_in, B, cand, r, slots, Kc, Xr, prob, stream);
+            return launch_route_forward_bytes16<32>(X, w_in, B, cand, r, slots, Kc, Xr, prob, stream);
+        }
+    }
+    if (B == 0) {   // probabilities only
+        route_forward_kernel<T><<<(unsigned)((slots + kRouteWarps - 1) / kRouteWarps), kRouteWarps * 32, 0,
+                                  stream>>>(X, w_in, 0, cand, r, slots, Kc, Xr, prob, 1);
+        return launch_status();
+    }
+    if (Kc <= 4) return launch_route_forward<4, T>(X, w_in, B, cand, r, slots, Kc, Xr, prob, vec, stream);
+    if (Kc <= 8) return launch_route_forward<8, T>(X, w_in, B, cand, r, slots, Kc, Xr, prob, vec, stream);
+    if (Kc <= 16) return launch_route_forward<16, T>(X, w_in, B, cand, r, slots, Kc, Xr, prob, vec, stream);
+    return launch_route_forward<32, T>(X, w_in, B, cand, r, slots, Kc, Xr, prob, vec, stream);
+}
+
+template <typename T>
+int route_dr_impl(const T* X, int32_t w_in, int64_t B, const int32_t* cand, const float* r, int32_t slots,
+                  int32_t Kc, const float* G, float* dr, cudaStream_t stream) {
+    const bool vec = (B % 4 == 0) && aligned16(X) && aligned16(G) &&
+                     (unsigned long long)w_in * (unsigned long long)(B / 4) < (1ull << 32);
+    if (Kc <= 4) return launch_route_dr<4, T>(X, w_in, B, cand, r, slots, Kc, G, dr, vec, stream);
+    if (Kc <= 8) return launch_route_dr<8, T>(X, w_in, B, cand, r, slots, Kc, G, dr, vec, stream);
+    if (Kc <= 16) return launch_route_dr<16, T>(X, w_in, B, cand, r, slots, Kc, G, dr, vec, stream);
+    return launch_route_dr<32, T>(X, w_in, B, cand, r, slots, Kc, G, dr, vec, stream);
 }
 
 }  // namespace
@@ -358,20 +480,13 @@ BITLOGIC_ERROR_READER(route)
 
 extern "C" int bitlogic_route_forward(const float* X, int32_t w_in, int64_t B, const int32_t* cand, const float* r,
                                       int32_t slots, int32_t Kc, float* Xr, float* prob, cudaStream_t stream) {
-    int st = check_route(X, w_in, B, cand, r, slots, Kc);
-    if (st) return st;
-    if (B == 0 && !prob) return BITLOGIC_OK;
-    if (B > 0 && !Xr) return BITLOGIC_ERR_NULL;
-    const bool vec = (B % 4 == 0) && aligned16(X) && aligned16(Xr);
-    if (B == 0) {   // probabilities only
-        route_forward_kernel<<<(unsigned)((slots + kRouteWarps - 1) / kRouteWarps), kRouteWarps * 32, 0, stream>>>(
-            X, w_in, 0, cand, r, slots, Kc, Xr, prob, 1);
-        return launch_status();
-    }
-    if (Kc <= 4) return launch_route_forward<4>(X, w_in, B, cand, r, slots, Kc, Xr, prob, vec, stream);
-    if (Kc <= 8) return launch_route_forward<8>(X, w_in, B, cand, r, slots, Kc, Xr, prob, vec, stream);
-    if (Kc <= 16) return launch_route_forward<16>(X, w_in, B, cand, r, slots, Kc, Xr, prob, vec, stream);
-    return launch_route_forward<32>(X, w_in, B, cand, r, slots, Kc, Xr, prob, vec, stream);
+    return route_forward_impl(X, w_in, B, cand, r, slots, Kc, Xr, prob, stream);
+}
+
+extern "C" int bitlogic_route_forward_u8(const uint8_t* X, int32_t w_in, int64_t B, const int32_t* cand,
+                                         const float* r, int32_t slots, int32_t Kc, float* Xr, float* prob,
+                                         cudaStream_t stream) {
+    return route_forward_impl(X, w_in, B, cand, r, slots, Kc, Xr, prob, stream);
 }
 
 extern "C" int bitlogic_route_backward(const float* X, int32_t w_in, int64_t B, const int32_t* cand, const float* r,
@@ -388,15 +503,10 @@ extern "C" int bitlogic_route_backward(const float* X, int32_t w_in, int64_t B, 
             return BITLOGIC_ERR_CUDA;
         return BITLOGIC_OK;
     }
-    const bool vec = (B % 4 == 0) && aligned16(X) && aligned16(G) &&
-                     (unsigned long long)w_in * (unsigned long long)(B / 4) < (1ull << 32);
-    if (Kc <= 4) st = launch_route_dr<4>(X, w_in, B, cand, r, slots, Kc, G, dr, vec, stream);
-    else if (Kc <= 8) st = launch_route_dr<8>(X, w_in, B, cand, r, slots, Kc, G, dr, vec, stream);
-    else if (Kc <= 16) st = launch_route_dr<16>(X, w_in, B, cand, r, slots, Kc, G, dr, vec, stream);
-    else st = launch_route_dr<32>(X, w_in, B, cand, r, slots, Kc, G, dr, vec, stream);
+    st = route_dr_impl(X, w_in, B, cand, r, slots, Kc, G, dr, stream);
     if (st || !dX) return st;
     const int nE = slots * Kc;
-    const bool vx = vec && aligned16(dX);
+    const bool vx = (B % 4 == 0) && aligned16(G) && aligned16(dX);
     const long long per_block = vx ? 128 : 32;
     const long long gy = (B + per_block - 1) / per_block;
     if (gy > 65535) return BITLOGIC_ERR_SHAPE;
@@ -406,6 +516,21 @@ extern "C" int bitlogic_route_backward(const float* X, int32_t w_in, int64_t B, 
     else
         route_dx_kernel<false><<<grid, kRdxWarps * 32, 0, stream>>>(G, B, prob, Kc, csr_off, csr_edge, w_in, nE, dX);
     return launch_status();
+}
+
+extern "C" int bitlogic_route_backward_u8(const uint8_t* X, int32_t w_in, int64_t B, const int32_t* cand,
+                                          const float* r, int32_t slots, int32_t Kc, const float* G, float* dr,
+                                          cudaStream_t stream) {
+    int st = check_route(X, w_in, B, cand, r, slots, Kc);
+    if (st) return st;
+    if (!dr) return BITLOGIC_ERR_NULL;
+    if (B > 0 && !G) return BITLOGIC_ERR_NULL;
+    if (B == 0) {
+        if (cudaMemsetAsync(dr, 0, sizeof(float) * (size_t)slots * (size_t)Kc, stream) != cudaSuccess)
+            return BITLOGIC_ERR_CUDA;
+        return BITLOGIC_OK;
+    }
+    return route_dr_impl(X, w_in, B, cand, r, slots, Kc, G, dr, stream);
 }
 
 extern "C" int bitlogic_route_snap(const int32_t* cand, const float* r, int32_t slots, int32_t Kc, int32_t* conn,

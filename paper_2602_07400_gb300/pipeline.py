@@ -21,7 +21,8 @@ from . import (NODE_FORMS, bitlogic_adamw_update, bitlogic_binarize_tables, bitl
                bitlogic_csr_positions, bitlogic_csr_reduce, bitlogic_pixel_histogram, bitlogic_quantile_thresholds,
                bitlogic_encode_thermometer, bitlogic_hard_forward, bitlogic_head_loss_ex,
                bitlogic_head_loss_workspace, bitlogic_lut_backward_node, bitlogic_lut_forward_node,
-               bitlogic_pack_bits, bitlogic_route_backward, bitlogic_route_forward, bitlogic_route_snap)
+               bitlogic_pack_bits, bitlogic_route_backward, bitlogic_route_backward_u8, bitlogic_route_forward,
+               bitlogic_route_forward_u8, bitlogic_route_snap, bitlogic_encode_thermometer_u8)
 
 
 def _nomark(name: str) -> None:
@@ -311,7 +312,8 @@ class RoutedTrainStep:
     """One training step of a RoutedNetwork: encode, per layer the routing
     (slot inputs as the expected selection) and the LUT nodes over them,
     head, and the backward through nodes and routing (gradients of the
-    table and routing logits)."""
+    table and routing logits).  The encoder's wires are kept as bytes: the
+    layer-1 routing gathers them from a quarter of the memory."""
 
     def __init__(self, net: RoutedNetwork, B: int, d: int, thresholds: Sequence[int], C: int, tau: float,
                  node: str = "soft", device="cuda"):
@@ -325,7 +327,7 @@ class RoutedTrainStep:
         s1, s2 = net.w1 * net.k1, net.w2 * net.k2
         self.x = torch.zeros(B, d, dtype=torch.uint8, device=dev)
         self.labels = torch.zeros(B, dtype=torch.int32, device=dev)
-        self.bits = torch.empty(net.w_in, B, **f32)
+        self.bits = torch.empty(net.w_in, B, dtype=torch.uint8, device=dev)   # 0/1 wires
         self.xr1, self.xr2 = torch.empty(s1, B, **f32), torch.empty(s2, B, **f32)
         self.p1, self.p2 = torch.empty(s1, net.Kc, **f32), torch.empty(s2, net.Kc, **f32)
         self.y1 = torch.empty(net.w1, B, **f32)
@@ -345,9 +347,9 @@ class RoutedTrainStep:
 
     def forward(self, stream=None, mark=_nomark):
         n = self.net
-        bitlogic_encode_thermometer(self.x, self.thr, self.bits, stream)
+        bitlogic_encode_thermometer_u8(self.x, self.thr, self.bits, stream)
         mark("encode")
-        bitlogic_route_forward(self.bits, n.cand1, n.r1, self.xr1, self.p1, stream)
+        bitlogic_route_forward_u8(self.bits, n.cand1, n.r1, self.xr1, self.p1, stream)
         mark("route1")
         bitlogic_lut_forward_node(self.xr1, n.ident1, n.theta1, self.y1, self.node, stream)
         mark("forward1")
@@ -372,7 +374,7 @@ class RoutedTrainStep:
         bitlogic_lut_backward_node(self.xr1, n.ident1, n.theta1, self.dth1, self.node, dY=self.dy1,
                                    edge_terms=self.g1, stream=stream)
         mark("backward1")
-        bitlogic_route_backward(self.bits, n.cand1, n.r1, self.g1, self.dr1, stream=stream)
+        bitlogic_route_backward_u8(self.bits, n.cand1, n.r1, self.g1, self.dr1, stream)
         mark("route_bwd1")
 
     def run(self, stream=None, mark=_nomark):

@@ -154,6 +154,9 @@ def test_host_validation_returns_before_any_launch():
     assert rs(fake, fake, 10, 0, fake, None) == -3
     assert rs(fake, fake, 0, 4, fake, None) == -2
     assert rs(None, fake, 10, 4, fake, None) == -1
+    assert lib.bitlogic_route_forward_u8(fake, 64, 8, fake, fake, 10, 33, fake, None, None) == -3
+    assert lib.bitlogic_route_backward_u8(fake, 64, 8, fake, fake, 10, 4, fake, None, None) == -1
+    assert lib.bitlogic_encode_thermometer_u8(fake, 64, 4, thr, 0, fake, None) == -9
     # node form: only soft (0) and straight-through (1)
     fwd_node, bwd_node = lib.bitlogic_lut_forward_node, lib.bitlogic_lut_backward_node
     assert fwd_node(fake, 8, 64, fake, fake, 4, 2, 2, fake, None) == -12

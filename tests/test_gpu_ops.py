@@ -236,6 +236,48 @@ def test_route_forward_backward(slots, Kc, w_in, B):
     no_device_error()
 
 
+@pytest.mark.parametrize("slots,Kc,w_in,B,binary", [(96, 16, 2352, 1024, True), (33, 8, 300, 259, True),
+                                                     (40, 32, 64, 100, False), (7, 5, 9, 4, False)])
+def test_route_over_byte_rows(slots, Kc, w_in, B, binary):
+    # routing over a uint8 layer input (the encoder's 0/1 wires, or any bytes)
+    # against the oracle on the same values
+    rng = np.random.default_rng(slots + Kc)
+    X8 = (rng.integers(0, 2, size=(w_in, B)) if binary else rng.integers(0, 256, size=(w_in, B))).astype(np.uint8)
+    cand = synth.candidate_pools(slots, Kc, w_in, seed=Kc)
+    r = synth.table_logits(slots, Kc, seed=slots)
+    G = synth.uniform_gradients(slots, B, seed=B, scale=1e-3)
+    Xr = torch.full((slots, B), np.nan, device="cuda")
+    prob = torch.empty(slots, Kc, device="cuda")
+    bl.bitlogic_route_forward_u8(dev(X8), dev(cand), dev(r), Xr, prob)
+    wXr, wp = oracle.route_forward(X8.astype(np.float64), cand, r)
+    check_fwd(Xr, wXr, "Xr from bytes")
+    check_fwd(prob, wp, "prob")
+    dr = torch.full((slots, Kc), np.nan, device="cuda")
+    bl.bitlogic_route_backward_u8(dev(X8), dev(cand), dev(r), dev(G), dr)
+    wdr, _ = oracle.route_backward(X8.astype(np.float64), cand, r, G.astype(np.float64), want_dx=False)
+    check_grad(dr, wdr, "dr from bytes")
+    # equal to the fp32 calls on the same values bit for bit (the same
+    # products in the same order)
+    Xf = dev(X8.astype(np.float32))
+    Xr_f = torch.empty_like(Xr)
+    bl.bitlogic_route_forward(Xf, dev(cand), dev(r), Xr_f)
+    check_exact(Xr.cpu().numpy(), Xr_f.cpu().numpy(), "Xr bytes vs fp32")
+    dr_f = torch.empty_like(dr)
+    bl.bitlogic_route_backward(Xf, dev(cand), dev(r), dev(G), dr_f)
+    check_exact(dr.cpu().numpy(), dr_f.cpu().numpy(), "dr bytes vs fp32")
+    no_device_error()
+
+
+@pytest.mark.parametrize("B,d,b", [(1, 5, 3), (37, 784, 3), (256, 70, 7), (1024, 784, 4)])
+def test_encode_thermometer_bytes(B, d, b):
+    rng = np.random.default_rng(B + d)
+    x = rng.integers(0, 256, size=(B, d), dtype=np.uint8)
+    thr = sorted(rng.choice(256, size=b, replace=False).tolist())
+    bits = torch.full((d * b, B), 7, dtype=torch.uint8, device="cuda")
+    bl.bitlogic_encode_thermometer_u8(dev(x), thr, bits)
+    check_exact(bits.cpu().numpy().astype(np.float64), oracle.encode_thermometer(x, thr), "byte wires")
+
+
 def test_route_unaligned_and_tied_logits():
     # a view 4 bytes into an allocation takes the scalar paths; tied logits
     # snap to the first candidate
