@@ -71,15 +71,12 @@ __device__ __forceinline__ void mux_tree4_smem(const int2* __restrict__ sPQ, con
 }
 
 // Per-warp node set-up: lane m derives (p, q) of pair m from the table, the
-// warp shares them through shared memory (sPQ: 2 * 2^(k-1) ints per warp).
-#ifndef BITLOGIC_PQ_LAYOUT
-#define BITLOGIC_PQ_LAYOUT 0
-#endif
+// warp shares them through shared memory (sPQ: 2 * 2^(k-1) ints per warp)
+// and every lane reads all pairs into registers (two per 16-byte load).
 template <int k>
 __device__ __forceinline__ void node_pairs(uint64_t T, int lane, int2* sPQ,
                                            int (&p)[1 << (k - 1)], int (&q)[1 << (k - 1)]) {
     constexpr int H = 1 << (k - 1);
-#if BITLOGIC_PQ_LAYOUT == 0
     if (lane < H) {
         const int t0 = (int)((T >> (2 * lane)) & 1u), t1 = (int)((T >> (2 * lane + 1)) & 1u);
         sPQ[lane] = make_int2(t1 - t0, -t0);
@@ -95,45 +92,6 @@ __device__ __forceinline__ void node_pairs(uint64_t T, int lane, int2* sPQ,
             p[m] = v.x; q[m] = v.y;
         }
     }
-#elif BITLOGIC_PQ_LAYOUT == 1
-    if (lane < H) {
-        const int t0 = (int)((T >> (2 * lane)) & 1u), t1 = (int)((T >> (2 * lane + 1)) & 1u);
-        sPQ[lane] = make_int2(t1 - t0, -t0);
-    }
-    __syncwarp();
-#pragma unroll
-    for (int m = 0; m < H; ++m) {
-        const int2 v = sPQ[m];
-        p[m] = v.x; q[m] = v.y;
-    }
-#else
-    int* sP = reinterpret_cast<int*>(sPQ);
-    int* sQ = sP + H;
-    if (lane < H) {
-        const int t0 = (int)((T >> (2 * lane)) & 1u), t1 = (int)((T >> (2 * lane + 1)) & 1u);
-        sP[lane] = t1 - t0;
-        sQ[lane] = -t0;
-    }
-    __syncwarp();
-#if BITLOGIC_PQ_LAYOUT == 2
-    if constexpr (H >= 4) {
-#pragma unroll
-        for (int m = 0; m < H; m += 4) {
-            const int4 a = *reinterpret_cast<const int4*>(sP + m);
-            const int4 b = *reinterpret_cast<const int4*>(sQ + m);
-            p[m] = a.x; p[m + 1] = a.y; p[m + 2] = a.z; p[m + 3] = a.w;
-            q[m] = b.x; q[m + 1] = b.y; q[m + 2] = b.z; q[m + 3] = b.w;
-        }
-    } else
-#endif
-    {
-#pragma unroll
-        for (int m = 0; m < H; ++m) {
-            p[m] = sP[m];
-            q[m] = sQ[m];
-        }
-    }
-#endif
     __syncwarp();
 }
 
