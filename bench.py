@@ -235,8 +235,8 @@ TRAFFIC = {
         "sha256": "180fc79502da4e837de466268e4dd9af96f7da65e286f6b8dce737f118e99f43",
         "note": "ncu capture of this workload"},
     ("hard_cifar10", "hard1"): {
-        "bytes": 16 * (1.216602e9 + 2.055721e9), "source": "hard.cu",
-        "sha256": "d74b4bd59b0e0e01d38d71386c9777f1454a99b4b319ccc4118923c90ee96232",
+        "bytes": 16 * (1.214920e9 + 2.055323e9), "source": "hard.cu",
+        "sha256": "0b8bea4460672c58351ea8f7e4078919658f6173b9ed26297aa7e38de8426587",
         "note": "ncu capture at 2^18 samples, scaled x16 to 2^22 by the words processed"},
 }
 
