@@ -60,8 +60,8 @@ def capture_graph(fn) -> torch.cuda.CUDAGraph:
 
 
 def allreduce_gradients(grads, group=None) -> None:
-    """Data-parallel exchange of a training step (§8 of the build plan: the
-    batch is sharded over ranks, every rank holds the whole network): sum
+    """Data-parallel exchange of a training step (the batch is sharded over
+    ranks, every rank holds the whole network): sum
     the ranks' gradients and divide by the number of ranks, in place, one
     all-reduce per tensor in list order.  Each rank's loss is the mean over
     its own batch, so with equal batches the result is the gradient of the
