@@ -43,7 +43,7 @@ template <int L, int M, int H, int k>
 __device__ __forceinline__ uint32_t mux_tree(const int (&p)[H], const int (&q)[H],
                                              const uint32_t (&x)[k]) {
     if constexpr (L == 0) {
-        return (uint32_t)((int)x[0] * p[M] + q[M]);
+        return x[0] * (uint32_t)p[M] + (uint32_t)q[M];   // modulo 2^32
     } else {
         const uint32_t a = mux_tree<L - 1, 2 * M>(p, q, x);
         const uint32_t b = mux_tree<L - 1, 2 * M + 1>(p, q, x);
@@ -60,7 +60,7 @@ __device__ __forceinline__ void mux_tree4_smem(const int2* __restrict__ sPQ, con
     if constexpr (L == 0) {
         const int2 v = sPQ[M];
 #pragma unroll
-        for (int r = 0; r < 4; ++r) out[r] = (uint32_t)((int)x[r][0] * v.x + v.y);
+        for (int r = 0; r < 4; ++r) out[r] = x[r][0] * (uint32_t)v.x + (uint32_t)v.y;
     } else {
         uint32_t lo[4], hi[4];
         mux_tree4_smem<L - 1, 2 * M, k>(sPQ, x, lo);
