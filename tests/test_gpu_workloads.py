@@ -9,9 +9,12 @@ configuration the benchmark times (``pipeline.TrainStep`` / ``HardInfer``).
   nodes of both layers and the layer-1 output gradient of sampled nodes, each
   computed by the oracle on the sub-network that feeds them (every consumer
   of a sampled node is included, so the sums are the full sums).
-* hard_cifar10 (2^22 samples): every sample runs on the GPU; sampled samples
-  (first and last included) are recomputed by the oracle from the raw
-  samples, bit-exact for the packed input, both layers, counts and argmax.
+* mnist_k4_routed16 (routed, 8000 x 8000, k = 4, 16 candidates): every
+  output element, routing-logit gradients included.
+* hard_cifar10 and hard_mnist_w4000_4m (2^22 samples): every sample runs on
+  the GPU; sampled samples (first and last included) are recomputed by the
+  oracle from the raw samples, bit-exact for the packed input, both layers,
+  counts and argmax; hard_mnist_w4000 (batch 1024): every sample.
 """
 import os
 
@@ -248,6 +251,30 @@ def test_tiny_routed_step_all_outputs(k, Kc, node):
     assert bl_device_ok()
 
 
+@pytest.mark.slow
+def test_mnist_routed16_step_all_outputs():
+    # the routed MNIST-shaped step at its benchmark size (8000 x 8000, k = 4,
+    # 16 candidates per slot, batch 1024; layer 1 routed from byte wires),
+    # routing logits drawn away from uniform so every softmax weight differs:
+    # every output and gradient against the oracle
+    wl = synth.WORKLOADS["mnist_k4_routed16"]
+    net, st, (cand1, r1, th1, cand2, r2, th2) = _routed(wl, wl.Kc, seed=3)
+    x, labels = synth.blob_batch(wl.batch, wl.d, wl.classes, wl.sigma, seed=41)
+    st.load(x.cuda(), labels.cuda())
+    st.run()
+    torch.cuda.synchronize()
+    r = oracle.routed_train_step(x.numpy(), labels.numpy(), wl.thresholds, cand1, r1, th1, cand2, r2, th2,
+                                 wl.classes, wl.tau)
+    check_exact(st.bits.cpu().numpy().astype(np.float64), r["bits"], "bits")
+    for name in ("xr1", "y1", "xr2", "y2", "logits"):
+        check_fwd(getattr(st, name), r[name], name)
+    check_fwd(st.loss, np.array([r["loss"]]), "loss")
+    for name in ("dth2", "dr2", "dy1", "dth1", "dr1"):
+        check_grad(getattr(st, name), r[name], name)
+    check_grad(st.g2, r["dxr2"], "dXr2")
+    assert bl_device_ok()
+
+
 def bl_device_ok():
     import paper_2602_07400_gb300 as bl
     return bl.bitlogic_device_error() == 0
@@ -377,6 +404,19 @@ def _hard_run(wl, N, seed=0, samples=1536):
 @pytest.mark.slow
 def test_hard_cifar10_full_size_sampled():
     wl = synth.WORKLOADS["hard_cifar10"]
+    _hard_run(wl, wl.batch)
+
+
+def test_hard_mnist_w4000_every_sample():
+    # the deployed-MNIST shape (784 x 4 thresholds, 4000 x 4000, k = 4) at
+    # batch 1024: every sample bit-exact against the oracle
+    wl = synth.WORKLOADS["hard_mnist_w4000"]
+    _hard_run(wl, wl.batch, samples=wl.batch)
+
+
+@pytest.mark.slow
+def test_hard_mnist_w4000_4m_sampled():
+    wl = synth.WORKLOADS["hard_mnist_w4000_4m"]
     _hard_run(wl, wl.batch)
 
 
