@@ -528,6 +528,7 @@ def run_ours(args):
                                      "bytes_per_rank": int(sum(g.numel() * 4 for g in grads))}
     if not args.profile and rank == 0:
         result["fit"] = time_quantile_fit(wl, flush)
+        result["pipe_rates"] = measure_pipe_rates()
     if not args.profile and not args.no_e2e:
         e2e = run_e2e(args, st, hi, wl, B, use_graph)
         if result is not None:
@@ -568,6 +569,37 @@ def time_quantile_fit(wl, flush, iters: int = 20):
     return {"kernel": "pixel_histogram_kernel", "split": f"{n_samples} x {wl.d} uint8 (a training split of the "
             f"workload's shape)", "ms": t, "GB/s": gbs, "frac_hbm": gbs / hbm,
             "thresholds_b": [int(v) for v in thr]}
+
+
+def measure_pipe_rates(iters: int = 2048, reps: int = 5) -> dict:
+    """Sustained issue rates of the pipes the kernels run on, from the
+    library's throughput probe (independent chains of one instruction kind
+    over 4 blocks of 256 threads per SM): LOP3 (logic pipe, the hard mux
+    tree's upper levels), IMAD (FMA pipe, its level 0) and FFMA (FMA pipe,
+    the soft kernels).  Median of `reps` launches, CUDA events."""
+    import paper_2602_07400_gb300 as bl
+    n = bl.bitlogic_issue_probe_threads()
+    sms = n // (4 * 256)
+    sink = torch.empty(n, dtype=torch.int32, device="cuda")
+    ops = n * iters * bl.bitlogic_issue_probe_ops_per_iter()
+    _, sm_max, _ = peaks()
+    out = {"sms": sms, "clock_mhz_assumed": sm_max,
+           "probe": "independent dependency chains, 4 x 256 threads per SM, median of 5 launches"}
+    for kind in ("lop3", "imad", "ffma"):
+        bl.bitlogic_issue_probe(kind, iters, sink)
+        evs = []
+        for _ in range(reps):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            bl.bitlogic_issue_probe(kind, iters, sink)
+            e1.record()
+            evs.append((e0, e1))
+        torch.cuda.synchronize()
+        t = float(np.median([a.elapsed_time(b) for a, b in evs]))
+        rate = ops / (t * 1e-3)
+        out[kind] = {"T_lane_ops_s": round(rate / 1e12, 3),
+                     "lane_ops_per_sm_per_clk": round(rate / (sms * sm_max * 1e6), 1)}
+    return out
 
 
 def time_update(st, iters: int) -> float:

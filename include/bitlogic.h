@@ -385,6 +385,27 @@ int bitlogic_csr_positions(const int32_t* edge_host, int32_t n_edges, int32_t* p
  * range since the last call, or BITLOGIC_ERR_CUDA. */
 int bitlogic_device_error(cudaStream_t stream);
 
+/* Issue-throughput probe (measurement support, not part of the method): the
+ * roofline of the hard layer counts its mux operations against the issue
+ * rate of the two pipes they run on, IMAD (FMA pipe) and LOP3 (logic pipe);
+ * this launch measures what each sustains.  Every thread of a grid of
+ * bitlogic_issue_probe_threads() threads (4 blocks of 256 per SM) runs
+ * `iters` x bitlogic_issue_probe_ops_per_iter() instructions of one kind,
+ * in independent dependency chains; the caller times the launch on `stream`
+ * and divides.  sink: device, >= bitlogic_issue_probe_threads() uint32
+ * (one per thread, written so the work is kept).  Returns
+ * BITLOGIC_ERR_NULL, BITLOGIC_ERR_SHAPE (iters < 0, sink too short, unknown
+ * kind) or BITLOGIC_ERR_CUDA. */
+typedef enum {
+    BITLOGIC_PROBE_LOP3 = 0,
+    BITLOGIC_PROBE_IMAD = 1,
+    BITLOGIC_PROBE_FFMA = 2
+} bitlogic_probe_t;
+int64_t bitlogic_issue_probe_threads(void);
+int64_t bitlogic_issue_probe_ops_per_iter(void);
+int bitlogic_issue_probe(int32_t kind, int64_t iters, uint32_t seed, uint32_t* sink,
+                         int64_t sink_len, cudaStream_t stream);
+
 /* Static text for a status code. */
 const char* bitlogic_status_string(int code);
 

@@ -34,6 +34,7 @@ __all__ = [
     "bitlogic_route_forward_u8", "bitlogic_route_backward_u8", "bitlogic_encode_thermometer_u8",
     "bitlogic_pixel_histogram", "bitlogic_quantile_thresholds", "bitlogic_lut_forward_node", "bitlogic_lut_backward_node", "NODE_FORMS",
     "bitlogic_status_string", "bitlogic_version", "LIB_PATH",
+    "bitlogic_issue_probe", "bitlogic_issue_probe_threads", "bitlogic_issue_probe_ops_per_iter", "PROBE_KINDS",
 ]
 
 LIB_PATH = _build.LIB
@@ -41,6 +42,9 @@ LIB_PATH = _build.LIB
 # node forms (bitlogic_node_t): the soft LightLUT node and its
 # straight-through hard form
 NODE_FORMS = {"soft": 0, "st": 1}
+
+# instruction kinds of the issue-throughput probe (bitlogic_probe_t)
+PROBE_KINDS = {"lop3": 0, "imad": 1, "ffma": 2}
 
 
 def _node_code(node) -> int:
@@ -98,6 +102,9 @@ _SIGS = {
     "bitlogic_device_error": ([_P], ctypes.c_int),
     "bitlogic_status_string": ([ctypes.c_int], ctypes.c_char_p),
     "bitlogic_version": ([], ctypes.c_int),
+    "bitlogic_issue_probe_threads": ([], _I64),
+    "bitlogic_issue_probe_ops_per_iter": ([], _I64),
+    "bitlogic_issue_probe": ([_I32, _I64, ctypes.c_uint32, _P, _I64, _P], ctypes.c_int),
 }
 
 
@@ -159,6 +166,29 @@ def bitlogic_status_string(code: int) -> str:
 
 def bitlogic_version() -> int:
     return load().bitlogic_version()
+
+
+def bitlogic_issue_probe_threads() -> int:
+    return int(load().bitlogic_issue_probe_threads())
+
+
+def bitlogic_issue_probe_ops_per_iter() -> int:
+    return int(load().bitlogic_issue_probe_ops_per_iter())
+
+
+def bitlogic_issue_probe(kind, iters: int, sink: torch.Tensor, seed: int = 1, stream=None):
+    """One launch of the issue-throughput probe: bitlogic_issue_probe_threads()
+    threads x iters x bitlogic_issue_probe_ops_per_iter() instructions of
+    `kind` ("lop3", "imad" or "ffma"); time it with events on `stream`."""
+    if isinstance(kind, str):
+        if kind not in PROBE_KINDS:
+            raise ValueError(f"kind must be one of {sorted(PROBE_KINDS)}")
+        kind = PROBE_KINDS[kind]
+    if not isinstance(sink, torch.Tensor) or sink.dtype != torch.int32 or not sink.is_cuda \
+            or not sink.is_contiguous():
+        raise ValueError("sink must be a contiguous int32 CUDA tensor")
+    _check("bitlogic_issue_probe", load().bitlogic_issue_probe(
+        int(kind), int(iters), int(seed) & 0xffffffff, _ptr(sink), sink.numel(), _stream(stream)))
 
 
 def bitlogic_encode_thermometer(x: torch.Tensor, thresholds, bits: torch.Tensor, stream=None):

@@ -114,6 +114,13 @@ def test_host_validation_returns_before_any_launch():
                                      fake, fake, fake, 4, None) == -5
     assert lib.bitlogic_lut_backward(fake, 4, 8, fake, fake, 2, 2, fake, fake, fake,
                                      fake, fake, P(17), 1 << 20, None) == -4
+    # issue probe: NULL sink, short sink, negative iterations, unknown kind
+    n = lib.bitlogic_issue_probe_threads()
+    assert n > 0 and lib.bitlogic_issue_probe_ops_per_iter() > 0
+    assert lib.bitlogic_issue_probe(0, 1, 1, None, n, None) == -1
+    assert lib.bitlogic_issue_probe(0, 1, 1, fake, n - 1, None) == -2
+    assert lib.bitlogic_issue_probe(0, -1, 1, fake, n, None) == -2
+    assert lib.bitlogic_issue_probe(7, 1, 1, fake, n, None) == -2
     # head: w % C != 0, tau <= 0
     assert lib.bitlogic_head_loss(fake, 10, 8, 3, 1.0, fake, None, fake, None, fake, 1 << 20, None) == -2
     assert lib.bitlogic_head_loss(fake, 9, 8, 3, 0.0, fake, None, fake, None, fake, 1 << 20, None) == -2

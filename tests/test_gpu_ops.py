@@ -648,6 +648,22 @@ def test_binding_rejects_wrong_tensors():
         bl.bitlogic_lut_forward(X.cpu(), conn, theta, torch.empty(4, 8, device="cuda"))
 
 
+def test_issue_probe_runs_every_kind():
+    # the throughput probe behind the pipe rates the benchmark reports: every
+    # thread writes the combination of its chains
+    n = bl.bitlogic_issue_probe_threads()
+    sink = torch.zeros(n, dtype=torch.int32, device="cuda")
+    for kind in ("lop3", "imad", "ffma"):
+        sink.zero_()
+        bl.bitlogic_issue_probe(kind, 4, sink, seed=12345)
+        torch.cuda.synchronize()
+        assert int((sink != 0).sum()) > n // 2, kind
+    with pytest.raises(ValueError):
+        bl.bitlogic_issue_probe("lop4", 1, sink)
+    with pytest.raises(bl.BitLogicError):
+        bl.bitlogic_issue_probe(7, 1, sink)
+
+
 # ------------------------------------------------------------------ AdamW --
 
 @pytest.mark.parametrize("n,wd", [(4096, 0.0), (1000003, 0.0), (64000 * 64, 0.1), (7, 0.05)])
