@@ -394,8 +394,8 @@ int bitlogic_device_error(cudaStream_t stream);
  * in independent dependency chains; the caller times the launch on `stream`
  * and divides.  sink: device, >= bitlogic_issue_probe_threads() uint32
  * (one per thread, written so the work is kept).  Returns
- * BITLOGIC_ERR_NULL, BITLOGIC_ERR_SHAPE (iters < 0, sink too short, unknown
- * kind) or BITLOGIC_ERR_CUDA. */
+ * BITLOGIC_ERR_NULL, BITLOGIC_ERR_SHAPE (iters outside [0, 2^20], sink too
+ * short, unknown kind) or BITLOGIC_ERR_CUDA. */
 typedef enum {
     BITLOGIC_PROBE_LOP3 = 0,
     BITLOGIC_PROBE_IMAD = 1,

@@ -72,7 +72,8 @@ extern "C" int bitlogic_issue_probe(int32_t kind, int64_t iters, uint32_t seed, 
                                     int64_t sink_len, cudaStream_t stream) {
     using namespace bitlogic;
     if (!sink) return BITLOGIC_ERR_NULL;
-    if (iters < 0 || sink_len < bitlogic_issue_probe_threads()) return BITLOGIC_ERR_SHAPE;
+    // at most 2^20 iterations: about 1.6 s at the slowest rate measured
+    if (iters < 0 || iters > (1ll << 20) || sink_len < bitlogic_issue_probe_threads()) return BITLOGIC_ERR_SHAPE;
     const unsigned grid = (unsigned)(sm_count() * kProbeBlocksPerSM);
     switch (kind) {
         case BITLOGIC_PROBE_LOP3:

@@ -120,6 +120,7 @@ def test_host_validation_returns_before_any_launch():
     assert lib.bitlogic_issue_probe(0, 1, 1, None, n, None) == -1
     assert lib.bitlogic_issue_probe(0, 1, 1, fake, n - 1, None) == -2
     assert lib.bitlogic_issue_probe(0, -1, 1, fake, n, None) == -2
+    assert lib.bitlogic_issue_probe(0, (1 << 20) + 1, 1, fake, n, None) == -2
     assert lib.bitlogic_issue_probe(7, 1, 1, fake, n, None) == -2
     # head: w % C != 0, tau <= 0
     assert lib.bitlogic_head_loss(fake, 10, 8, 3, 1.0, fake, None, fake, None, fake, 1 << 20, None) == -2
