@@ -15,7 +15,7 @@ static __device__ unsigned int g_index_error;
 __device__ __forceinline__ void flag_index_error() { atomicOr(&g_index_error, 1u); }
 
 // Reads and clears this unit's flag (synchronizes the stream).
-static int read_and_clear_index_error(cudaStream_t stream) {
+static inline int read_and_clear_index_error(cudaStream_t stream) {
     unsigned int v = 0, zero = 0;
     if (cudaMemcpyFromSymbolAsync(&v, g_index_error, sizeof(v), 0,
                                   cudaMemcpyDeviceToHost, stream) != cudaSuccess)
