@@ -103,3 +103,33 @@ def test_traffic_record_digest_ignores_comments(tmp_path):
     c.write_text("int f(int x) { return x + 2; }\n")
     assert bench.code_digest(str(a)) == bench.code_digest(str(b))
     assert bench.code_digest(str(a)) != bench.code_digest(str(c))
+
+
+def test_algorithmic_work_of_the_roofline_calls():
+    # the per-call work the roofline divides by, restated from the counts:
+    # layer-2 backward with input-gradient terms, 4(2^k-1) + 2^k operations
+    # per (node, sample) and X + per-class dY rows + terms + 2 tables + conn;
+    # hard layer, 2^k - 1 mux operations per (node, 32-sample word) and the
+    # packed input and output words + conn + tables
+    import bench
+    from paper_2602_07400_gb300 import synth
+    wl = synth.WORKLOADS["mnist"]
+    work = bench.call_work(wl, 1024)
+    B, w, k, K, C = 1024, 8000, 6, 64, 10
+    assert work["backward2"][1] == 316 * w * B
+    assert work["backward2"][0] == 4 * (w * B + C * B + w * k * B + 2 * w * K + w * k)
+    assert work["forward2"][1] == 132 * w * B
+    hw = synth.WORKLOADS["hard_cifar10"]
+    N = 1 << 22
+    W = N // 32
+    hwork = bench.call_work(hw, N)
+    assert hwork["hard1"][1] == 63 * 64000 * W
+    assert hwork["hard1"][0] == 4 * (21504 * W + 64000 * W + 64000 * 6) + 8 * 64000
+
+
+def test_integer_pipe_ceiling_is_the_sum_of_both_pipes():
+    import bench
+    roof = {"achieved": 10.0}
+    rates = {"imad": {"T_lane_ops_s": 12.0}, "lop3": {"T_lane_ops_s": 8.0}}
+    got = bench.integer_pipe_fraction(roof, rates)
+    assert got["peak"] == 20.0 and abs(got["frac"] - 0.5) < 1e-12
