@@ -201,3 +201,32 @@ def test_workspace_queries():
     assert bl.bitlogic_lut_backward_workspace(100, 64, 10, 6, False) == 0
     assert bl.bitlogic_lut_backward_workspace(100, 64, 10, 6, True) == 10 * 6 * 64 * 4
     assert bl.bitlogic_head_loss_workspace(64, 10) >= 2 * 64 * 10 * 4 + 64 * 4
+
+
+def test_no_cpu_fallback_without_the_library(monkeypatch):
+    # with the shared library absent (and building switched off) the binding
+    # raises instead of computing anything another way
+    missing = os.path.join(ROOT, "no_such_dir", "libbitlogic.so")
+    monkeypatch.setattr(bl, "_lib", None)
+    monkeypatch.setattr(bl, "LIB_PATH", missing)
+    monkeypatch.setattr(bl._build, "LIB", missing)
+    with pytest.raises(RuntimeError):
+        bl.load(build_if_missing=False)
+
+
+def test_compute_calls_reject_host_tensors():
+    # every compute call takes device tensors only: host tensors are refused
+    # before any launch, so there is no CPU path to fall back on
+    import torch
+    x = torch.zeros(4, 8, dtype=torch.uint8)
+    X = torch.zeros(16, 4)
+    conn = torch.zeros(2, 2, dtype=torch.int32)
+    theta = torch.zeros(2, 4)
+    with pytest.raises(ValueError, match="CUDA"):
+        bl.bitlogic_encode_thermometer(x, [64, 128], torch.zeros(16, 4))
+    with pytest.raises(ValueError, match="CUDA"):
+        bl.bitlogic_lut_forward(X, conn, theta, torch.zeros(2, 4))
+    with pytest.raises(ValueError, match="CUDA"):
+        bl.bitlogic_pack_bits(x, [64, 128], torch.zeros(16, 1, dtype=torch.int32))
+    with pytest.raises(ValueError, match="CUDA"):
+        bl.bitlogic_issue_probe("lop3", 1, torch.zeros(8, dtype=torch.int32))
