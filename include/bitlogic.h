@@ -225,10 +225,10 @@ int bitlogic_lut_backward_node(const float* X, int32_t w_in, int64_t B,
                                float* dtheta, float* edge_terms, const int32_t* edge_pos,
                                float* dY_out, cudaStream_t stream);
 
-/* Learnable routing (§3 "Connectivity is the main per-layer design choice":
- * a per-slot candidate pool whose selection is differentiable in training
- * and snapped to a sparse mapping at discretization; App. A
- * "Initialization": pools drawn uniformly, logits zero).  Slot e = j*k + i of
+/* Learnable routing (§3, the paragraph on connectivity: a per-slot
+ * candidate pool whose selection is differentiable in training and snapped
+ * to a sparse mapping at discretization; App. A "Initialization": pools
+ * drawn uniformly, logits zero).  Slot e = j*k + i of
  * a layer of w nodes (slots = w*k) has candidates cand[e][m] and logits
  * r[e][m], m < Kc, 1 <= Kc <= 32:
  *   p_e = softmax(r_e),   Xr[e][s] = sum_m p_e[m] X[cand[e][m]][s].

@@ -234,8 +234,8 @@ void oracle_lut_backward(const double* X, int32_t w_in, int64_t B,
     free(tt);
 }
 
-/* Learnable routing (§3 "Connectivity is the main per-layer design choice":
- * a per-slot candidate pool, a selection that is differentiable in training
+/* Learnable routing (§3, the paragraph on connectivity: a per-slot
+ * candidate pool, a selection that is differentiable in training
  * and snapped to a sparse mapping at discretization; App. A
  * "Initialization": pools drawn uniformly, routing logits zero so the
  * expected selection is uniform).  Slot e (e = j*k + i, n_slots = w*k) has

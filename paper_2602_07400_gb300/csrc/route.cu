@@ -1,5 +1,5 @@
-// Learnable routing (paper §3 "Connectivity is the main per-layer design
-// choice": each node slot selects its input from a candidate pool through a
+// Learnable routing (paper §3, the paragraph on connectivity: each node
+// slot selects its input from a candidate pool through a
 // selection that is differentiable in training and snapped to a sparse
 // mapping at discretization; App. A "Initialization": pools drawn uniformly,
 // routing logits zero).
