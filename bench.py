@@ -1,24 +1,37 @@
 #!/usr/bin/env python3
 """Throughput of the LUT-network hot path on GB300 (one JSON line on rank 0).
 
-A step is one pass of the whole hot path over one batch of synthetic input:
-the soft training step (thermometer encode, two LUT forwards, group-sum head
-with cross-entropy, two LUT backwards with the CSR input-gradient
-reduction) followed by the hard evaluation of the same batch (table
-binarization, encode + pack, hard layer 1, hard layer 2 with the fused
-popcount head and argmax).  ``value`` is the training throughput (samples
-per second through the fwd+bwd part); the hard part is reported in the
-``hard`` object.  L2 is flushed between steps (a 512 MB write outside the
-timed events), so every step starts cold.  The timed loop replays the step as
-CUDA graphs captured once (no host work between launches); the per-call
-split comes from eager steps with an event after every call.
+Default run (no ``--workload``): the headline workloads.
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload mnist]
-  python bench.py --impl reference ...   # the CPU oracle on the same workload
+* ``value`` / ``ms_per_step`` / ``roofline`` / ``cpu_baseline`` / ``e2e``:
+  the CIFAR-100-shaped soft training step (B = 2048, 46080 thermometer bits,
+  two 128000-node layers, k = 6, 100 x 1280 group-sum head, tau = 100):
+  thermometer encode, two LUT forwards, group-sum head with cross-entropy,
+  layer-2 backward (table gradient + per-edge input-gradient terms), CSR
+  reduction of the terms into layer 1's output gradient, layer-1 table
+  gradient.
+* ``hard``: the bit-packed evaluation of the CIFAR-10-shaped network
+  (21504 bits, 64000 x 64000, k = 6, tables theta > 0) on 2^22 samples:
+  table binarization, encode + pack, hard layer 1, hard layer 2 with the fused
+  popcount head and argmax, with its own roofline, oracle baseline and
+  end-to-end figure.
+* ``extra``: the MNIST-shaped step at k = 6 and k = 2 and the
+  CIFAR-10-shaped step (value, per-call split, roofline).
+
+The two headline parts run one after the other, each over its own K timed
+steps; the buffers of one are freed before the next is allocated.  L2 is
+flushed between steps (a 512 MB write outside the timed events).  The timed
+loops replay CUDA graphs captured once (no host work between launches); the
+per-call split comes from eager steps with an event after every call.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W]          # headline
+  python bench.py --workload mnist ...      # one workload (train + hard on its batch)
+  python bench.py --impl reference ...      # the CPU oracle on the same workloads
 
 Multi-GPU (torchrun, one process per GPU): every rank trains its own batch
-(weak scaling, no data-path collective); the job's time is the max over
-ranks and ``value`` sums the samples of all ranks.
+and evaluates its own samples (weak scaling, no data-path collective); the
+job's time is the max over ranks and ``value`` sums the samples of all
+ranks.
 """
 from __future__ import annotations
 
@@ -43,6 +56,9 @@ if ROOT not in sys.path:
 from paper_2602_07400_gb300 import synth  # noqa: E402
 
 METRIC = "LUT train samples/s (fwd+bwd) and hard bit-packed MSamples/s; % of roofline"
+HEADLINE_TRAIN = "cifar100"
+HEADLINE_HARD = "hard_cifar10"
+EXTRAS = ("mnist", "mnist_k2", "cifar10")
 FP32_LANES_PER_SM = 128
 # the paper's own figures for a workload of the same shape, on its hardware
 # (context only, not a target: another machine and its own timing protocol)
@@ -57,13 +73,18 @@ SMI_FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.act
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
 
-def parse_args():
+def parse_args(argv=None):
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=400)
-    p.add_argument("--warmup", type=int, default=20)
+    p.add_argument("--steps", type=int, default=30)
+    p.add_argument("--warmup", type=int, default=5)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    p.add_argument("--workload", default="mnist", choices=sorted(synth.WORKLOADS))
+    p.add_argument("--workload", default=None, choices=sorted(synth.WORKLOADS),
+                   help="one workload (training step plus the hard pass on its batch); "
+                        "default: the headline workloads")
+    p.add_argument("--extras", default=",".join(EXTRAS),
+                   help="comma-separated training workloads reported under 'extra' in the headline run")
+    p.add_argument("--no-extras", action="store_true")
     p.add_argument("--node", default="soft", choices=["soft", "st"],
                    help="LightLUT node form of the training step: soft, or straight-through hard")
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -74,10 +95,11 @@ def parse_args():
                    help="plain timed loop only (for ncu launch lists)")
     p.add_argument("--batch", type=int, default=0,
                    help="override the workload's batch (smaller cases for ncu captures)")
-    return p.parse_args()
+    return p.parse_args(argv)
 
 
 def peaks():
+    """(HBM GB/s, SM max MHz, source) from the measured peaks file."""
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
         with open(path) as f:
@@ -86,55 +108,85 @@ def peaks():
     return 6800.0, 2070.0, "fallback"
 
 
+def device_sms(device=None) -> int:
+    """SM count of the device, read from the device."""
+    return int(torch.cuda.get_device_properties(device if device is not None
+                                                else torch.cuda.current_device()).multi_processor_count)
+
+
+def issue_peak(sms: int, mhz: float) -> float:
+    """Lane-operations per second at one warp instruction per clock and
+    scheduler (128 lanes per SM)."""
+    return sms * FP32_LANES_PER_SM * mhz * 1e6
+
+
 # ------------------------------------------------------------- clocks --
 
 class ClockSampler:
-    def __init__(self, index: int, period_ms: int = 100):
+    """nvidia-smi samples of one GPU, taken only while a segment is open
+    (start() .. stop()); summary() covers every segment so far."""
+
+    def __init__(self, index: int, period_ms: int = 50):
         self.index, self.period = index, period_ms
+        self.rows = []
+        self.available = True
         self.proc = None
-        self.path = None
 
     def start(self):
+        if not self.available:
+            return
         try:
             fd, self.path = tempfile.mkstemp(suffix=".csv")
             os.close(fd)
             self.out = open(self.path, "w")
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.index}", f"--query-gpu={SMI_FIELDS}",
-                 "--format=csv,noheader,nounits", f"-lms", str(self.period)],
+                 "--format=csv,noheader,nounits", "-lms", str(self.period)],
                 stdout=self.out, stderr=subprocess.DEVNULL)
         except (OSError, FileNotFoundError):
+            self.available = False
             self.proc = None
-        self.t0 = time.time()
+        time.sleep(0.1)   # let the first sample land inside the segment
 
-    def stop(self):
-        if self.proc is None:
+    def stop(self) -> dict:
+        seg = []
+        if self.proc is not None:
+            time.sleep(0.1)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.out.close()
+            with open(self.path) as f:
+                for line in f:
+                    parts = [p.strip() for p in line.split(",")]
+                    if len(parts) >= 9:
+                        seg.append(parts)
+            os.unlink(self.path)
+            self.proc = None
+        self.rows.extend(seg)
+        return self._summary(seg)
+
+    def summary(self) -> dict:
+        return self._summary(self.rows)
+
+    def _summary(self, rows) -> dict:
+        if not self.available:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0,
                     "note": "nvidia-smi unavailable"}
-        time.sleep(0.25)
-        self.proc.terminate()
-        try:
-            self.proc.wait(timeout=5)
-        except subprocess.TimeoutExpired:
-            self.proc.kill()
-        self.out.close()
         sm, mx, pw, reasons = [], [], [], set()
-        names = ["active", "hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        with open(self.path) as f:
-            for line in f:
-                parts = [p.strip() for p in line.split(",")]
-                if len(parts) < 9:
-                    continue
-                try:
-                    sm.append(float(parts[1]))
-                    mx.append(float(parts[2]))
-                    pw.append(float(parts[3]))
-                except ValueError:
-                    continue
-                for name, val in zip(names[1:], parts[5:9]):
-                    if val.lower().startswith("active"):
-                        reasons.add(name)
-        os.unlink(self.path)
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for parts in rows:
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+                pw.append(float(parts[3]))
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
         return {"sm_mhz": statistics.median(sm) if sm else None,
                 "sm_max_mhz": max(mx) if mx else None,
                 "power_w_max": max(pw) if pw else None,
@@ -158,77 +210,98 @@ def job_rate(world: int, samples_per_rank_step: int, steps: int, max_ms: float) 
     return world * samples_per_rank_step * steps / (max_ms * 1e-3)
 
 
+def barrier(world: int):
+    if world > 1:
+        torch.distributed.barrier()
+
+
 # ------------------------------------------------------ work per call --
 
 def call_work_routed(wl, B):
-    """Work of the calls of a routed training step: the routing calls count
-    their HBM bytes (each slot's Kc candidate rows are gathered from the
-    layer input, which stays in L2, so the gathered bytes are not HBM
-    traffic) and one FMA per (candidate, sample); the LUT calls read the
-    slot rows through the identity connectivity."""
+    """Work of the calls of a routed training step: (algorithmic bytes, ops,
+    bytes moved).  The routing calls count their HBM bytes (each slot's Kc
+    candidate rows are gathered from the layer input, which stays in L2, so
+    the gathered bytes are not HBM traffic) and one FMA per (candidate,
+    sample); the LUT calls read the slot rows through the identity
+    connectivity."""
     K, k, Kc = wl.K, wl.k, wl.Kc
     w1, w2 = wl.widths
     win, d, C = wl.w_in, wl.d, wl.classes
     s1, s2 = w1 * k, w2 * k
     f = 4
-    return {
+    W = (B + 31) // 32
+    work = {
         # the encoder's wires are bytes in the routed step (layer 1 gathers them)
         "encode": (B * d + win * B, 0),
         "route1": (win * B + f * (s1 * B + 2 * s1 * Kc), Kc * s1 * B),
         "forward1": (f * (s1 * B + w1 * B + w1 * K + w1 * k), (2 * (K - 1) + k) * w1 * B),
         "route2": (f * (w1 * B + s2 * B + 2 * s2 * Kc), Kc * s2 * B),
         "forward2": (f * (s2 * B + w2 * B + w2 * K + w2 * k), (2 * (K - 1) + k) * w2 * B),
-        "head": (f * (w2 * B + 4 * B * C), 0),
+        "head": (f * (w2 * B + 2 * B * C + B), 0),
         "backward2": (f * (s2 * B + C * B + s2 * B + 2 * w2 * K + w2 * k), (4 * (K - 1) + K) * w2 * B),
         "route_bwd2": (f * (w1 * B + 2 * s2 * B + w1 * B + 3 * s2 * Kc), 2 * Kc * s2 * B),
         "backward1": (f * (s1 * B + w1 * B + s1 * B + 2 * w1 * K + w1 * k), (4 * (K - 1) + K) * w1 * B),
         "route_bwd1": (win * B + f * (s1 * B + 2 * s1 * Kc), Kc * s1 * B),
         "binarize": (f * (w1 * K + w2 * K) + 8 * (w1 + w2), 0),
-        "pack": (B * d + f * win * ((B + 31) // 32), 0),
-        "hard1": (f * (win * ((B + 31) // 32) + w1 * ((B + 31) // 32) + w1 * k) + 8 * w1,
-                  (K - 1) * w1 * ((B + 31) // 32)),
-        "hard2": (f * (w1 * ((B + 31) // 32) + w2 * k + B * C * 2 + B) + 8 * w2, (K - 1) * w2 * ((B + 31) // 32)),
-    }
-
-
-def call_work(wl, B, fuse_dy1=False):
-    """Algorithmic work of each library call of one step on a batch of B:
-    (bytes, fp32 or logic ops).  Ops follow the lerp-tree counts: forward
-    2(2^k-1)+k per (node, sample); backward with input gradient
-    4(2^k-1)+2^k; backward without it 2(2^k-1)+2^k; hard layer 2^k-1 LOP3
-    per (node, 32-sample word)."""
-    K, k = wl.K, wl.k
-    w1, w2 = wl.widths
-    win, d, b, C = wl.w_in, wl.d, wl.b, wl.classes
-    W = (B + 31) // 32
-    f = 4
-    return {
-        "encode": (B * d + f * win * B, 0),
-        "forward1": (f * (win * B + w1 * B + w1 * K + w1 * k), (2 * (K - 1) + k) * w1 * B),
-        "forward2": (f * (w1 * B + w2 * B + w2 * K + w2 * k), (2 * (K - 1) + k) * w2 * B),
-        "head": (f * (w2 * B + 4 * B * C), 0),
-        # layer 2: reads Y1 and the per-class gradient rows, writes dtheta and
-        # the per-edge input-gradient terms
-        "backward2": (f * (w1 * B + C * B + w2 * k * B + 2 * w2 * K + w2 * k), (4 * (K - 1) + K) * w2 * B),
-        # layer 1 (fused form): reads the encoder bits and layer 2's per-edge
-        # terms (its output gradient, reduced through the CSR map in the
-        # kernel); unfused form: the CSR reduction of those terms into dY1
-        # ("csr2"), then the dtheta-only backward reading dY1
-        "backward1": (f * (win * B + w2 * k * B + 2 * w1 * K + w1 * k + w1 + w2 * k), (2 * (K - 1) + K) * w1 * B)
-        if fuse_dy1 else (f * (win * B + w1 * B + 2 * w1 * K + w1 * k), (2 * (K - 1) + K) * w1 * B),
-        "csr2": (f * (w2 * k * B + w1 * B + w1 + 1 + w2 * k), 0),
-        "binarize": (f * (w1 * K + w2 * K) + 8 * (w1 + w2), 0),
         "pack": (B * d + f * win * W, 0),
         "hard1": (f * (win * W + w1 * W + w1 * k) + 8 * w1, (K - 1) * w1 * W),
         "hard2": (f * (w1 * W + w2 * k + B * C * 2 + B) + 8 * w2, (K - 1) * w2 * W),
     }
+    return {n: (b, o, b) for n, (b, o) in work.items()}
 
 
-# DRAM traffic per launch of the roofline kernel, dram__bytes_read.sum +
-# dram__bytes_write.sum from one ncu capture, keyed by workload
-# and call.  Valid only for the kernel source it was taken on: the SHA-256 of
-# the source file's code (comments and blank space removed) is recorded, and
-# any later change of the code reports null.
+def call_work(wl, B, fuse_dy1=False):
+    """Algorithmic work of each library call of one step on a batch of B:
+    (algorithmic bytes, algorithmic ops, bytes the call moves).
+
+    Ops follow the lerp-tree counts per (node, sample): forward 2(2^k-1)+k;
+    backward with input gradient 4(2^k-1)+2^k; backward without it
+    2(2^k-1)+2^k; hard layer 2^k-1 mux operations per (node, 32-sample word).
+    Algorithmic bytes count each tensor the step must read or write once: the
+    layer input X, the output gradient dY, the input gradient dX, the tables
+    and their gradients, the connectivity and the CSR map.  The head's output
+    gradient is one row per class (every node of a class has the same
+    gradient), so dY is C x B, not w x B.  The per-edge input-gradient terms
+    that the layer-2 backward writes and the CSR reduction reads are not
+    algorithmic: they appear only in the bytes moved."""
+    K, k = wl.K, wl.k
+    w1, w2 = wl.widths
+    win, d, C = wl.w_in, wl.d, wl.classes
+    W = (B + 31) // 32
+    f = 4
+    terms = f * w2 * k * B
+    csr2 = f * (w1 + 1 + w2 * k)
+    work = {
+        "encode": (B * d + f * win * B, 0, B * d + f * win * B),
+        "forward1": (f * (win * B + w1 * B + w1 * K + w1 * k), (2 * (K - 1) + k) * w1 * B, None),
+        "forward2": (f * (w1 * B + w2 * B + w2 * K + w2 * k), (2 * (K - 1) + k) * w2 * B, None),
+        # reads Y2 and the labels; writes the logits and one gradient row per class
+        "head": (f * (w2 * B + 2 * B * C + B), 0, None),
+        # §8(a) a4 with dX for layer 2 is backward2 + csr2: X = Y1, dY rows,
+        # the table and its gradient, the connectivity (here), the CSR map and
+        # dX = dY1 (the reduction); both calls carry the per-edge terms
+        "backward2": (f * (w1 * B + C * B + 2 * w2 * K + w2 * k), (4 * (K - 1) + K) * w2 * B,
+                      f * (w1 * B + C * B + 2 * w2 * K + w2 * k) + terms),
+        "csr2": (f * w1 * B + csr2, 0, f * w1 * B + csr2 + terms),
+        "backward1": (f * (win * B + w1 * B + 2 * w1 * K + w1 * k), (2 * (K - 1) + K) * w1 * B, None),
+        "binarize": (f * (w1 * K + w2 * K) + 8 * (w1 + w2), 0, None),
+        "pack": (B * d + f * win * W, 0, None),
+        "hard1": (f * (win * W + w1 * W + w1 * k) + 8 * w1, (K - 1) * w1 * W, None),
+        "hard2": (f * (w1 * W + w2 * k + B * C * 2 + B) + 8 * w2, (K - 1) * w2 * W, None),
+    }
+    if fuse_dy1:
+        # layer 1 sums layer 2's per-edge terms through the CSR map itself
+        work["backward1"] = (f * (win * B + w1 * B + 2 * w1 * K + w1 * k) + csr2, (2 * (K - 1) + K) * w1 * B,
+                             f * (win * B + 2 * w1 * K + w1 * k) + csr2 + terms)
+        del work["csr2"]
+    return {n: (b, o, b if m is None else m) for n, (b, o, m) in work.items()}
+
+
+# DRAM traffic per launch of a roofline kernel, dram__bytes_read.sum +
+# dram__bytes_write.sum from one ncu capture, keyed by workload and call.
+# Valid only for the kernel source it was taken on: the SHA-256 of the
+# source file's code (comments and blank space removed) is recorded, and any
+# later change of the code reports null.
 TRAFFIC = {
     ("mnist", "backward2"): {
         "bytes": 59.670016e6 + 147.641856e6, "source": "lut_soft.cu",
@@ -277,6 +350,62 @@ KERNEL_OF_CALL = {
     "route1": "route_forward_vec_kernel<KC>", "route2": "route_forward_vec_kernel<KC>",
     "route_bwd2": "route_dr_kernel + route_dx_kernel", "route_bwd1": "route_dr_kernel<KC> (byte rows)",
 }
+# calls that launch more than one kernel: not a single-kernel roofline
+MULTI_KERNEL_CALLS = ("head", "binarize", "hard2", "route_bwd2")
+
+
+def roofline_of(call, work, per_call_ms, sms, clocks, workload, hbm, sm_max, peak_kind):
+    """Roofline object of one single-kernel call: the bound (HBM bytes or
+    issue-rate lane-operations, whichever takes longer at peak), achieved
+    rate, peak, fraction (also at the median SM clock sampled during the
+    timed region) and the ncu DRAM traffic per launch."""
+    byts, ops, moved = work[call]
+    t_s = per_call_ms[call] * 1e-3
+    alu_peak = issue_peak(sms, sm_max)
+    t_hbm, t_alu = byts / (hbm * 1e9), ops / alu_peak
+    if t_alu >= t_hbm:
+        unit = ("Tops/s (integer mux lane-ops against the issue rate)" if call.startswith("hard")
+                else "Tops/s (fp32 pipe lane-ops)")
+        roof = {"bound": "alu", "achieved": ops / t_s / 1e12, "peak": alu_peak / 1e12, "unit": unit}
+        med = clocks.get("sm_mhz")
+        if med:
+            roof["frac_at_sampled_clock"] = ops / t_s / issue_peak(sms, med)
+    else:
+        roof = {"bound": "hbm", "achieved": byts / t_s / 1e9, "peak": hbm, "unit": "GB/s"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    traffic, traffic_note = kernel_traffic(workload, call)
+    roof.update({"traffic": traffic, "traffic_source": traffic_note,
+                 "traffic_over_algorithmic": (traffic / byts) if traffic else None,
+                 "kernel": KERNEL_OF_CALL[call], "call": call,
+                 "ms_per_launch": per_call_ms[call], "algorithmic_bytes": byts, "bytes_moved": moved,
+                 "algorithmic_ops": ops,
+                 "peak_source": f"{peak_kind} HBM copy ({hbm:.1f} GB/s); {sms} SMs (read from the device) x "
+                                f"{FP32_LANES_PER_SM} lanes x {sm_max:.0f} MHz (alu: one issue per lane and clock)"})
+    return roof
+
+
+def calls_table(work, per_call_ms, hbm):
+    out = {}
+    for n, t in per_call_ms.items():
+        b_, o_, m_ = work[n]
+        e = {"ms": round(t, 5), "alg_GB/s": round(b_ / (t * 1e-3) / 1e9, 1),
+             "frac_hbm": round(b_ / (t * 1e-3) / 1e9 / hbm, 3),
+             "Tops/s": round(o_ / (t * 1e-3) / 1e12, 2) if o_ else None}
+        if m_ != b_:
+            e["moved_GB/s"] = round(m_ / (t * 1e-3) / 1e9, 1)
+        out[n] = e
+    return out
+
+
+def step_hbm_fraction(work, names, ms_step, hbm):
+    """Algorithmic bytes of the step's calls over the step time, against the HBM peak."""
+    byts = sum(work[n][0] for n in names if n in work)
+    moved = sum(work[n][2] for n in names if n in work)
+    gbs = byts / (ms_step * 1e-3) / 1e9
+    return {"algorithmic_bytes": byts, "bytes_moved": moved, "alg_GB/s": gbs, "frac_hbm": gbs / hbm,
+            "moved_over_algorithmic": moved / byts}
+
+
 
 
 # --------------------------------------------------------------- ours --
@@ -288,260 +417,484 @@ def dist_env():
     return world, rank, local
 
 
-def run_ours(args):
-    import paper_2602_07400_gb300 as bl
-    from paper_2602_07400_gb300.pipeline import HardInfer, Network, RoutedNetwork, RoutedTrainStep, TrainStep
+def with_batch(wl, batch):
+    if not batch:
+        return wl
+    return synth.Workload(wl.name, batch, wl.d, wl.classes, wl.sigma, wl.thresholds, wl.widths, wl.k, wl.tau,
+                          wl.Kc)
 
-    world, rank, local = dist_env()
-    torch.cuda.set_device(local)
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
-    bl.load()
-    wl = synth.WORKLOADS[args.workload]
-    if args.batch:
-        wl = synth.Workload(wl.name, args.batch, wl.d, wl.classes, wl.sigma, wl.thresholds,
-                            wl.widths, wl.k, wl.tau)
-    hard_only = wl.name.startswith("hard_")
-    B = wl.batch
-    if wl.Kc:
-        rnet = RoutedNetwork(*synth.routed_network(wl, seed=0), wl.w_in)
-        net = rnet.snap()                # the hard pass evaluates the discretized network
-    else:
-        conn1, th1, conn2, th2 = synth.network(wl, seed=0)
-        net = Network(conn1, th1, conn2, th2, wl.w_in)
-    x_gen, lab_gen = synth.blob_batch(B, wl.d, wl.classes, wl.sigma, seed=1000 + rank,
-                                      device="cuda" if hard_only else "cpu")
-    st = None
-    if not hard_only:
-        if wl.Kc:
-            st = RoutedTrainStep(rnet, B, wl.d, wl.thresholds, wl.classes, wl.tau, node=args.node)
-        else:
-            st = TrainStep(net, B, wl.d, wl.thresholds, wl.classes, wl.tau, node=args.node)
-        st.load(x_gen.cuda(), lab_gen.cuda())
-    hi = HardInfer(net, B, wl.d, wl.thresholds, wl.classes)
-    if st is not None:
-        hi.x = st.x                      # the hard pass evaluates the same batch
-    else:
-        hi.x.copy_(x_gen)
-    del x_gen
-    flush = torch.empty(512 << 20, dtype=torch.uint8, device="cuda")
-    stream = torch.cuda.current_stream()
 
-    def step(mark):
-        if st is not None:
-            st.run(mark=mark)
-            mark("train_end")
-        hi.binarize(mark=mark)
-        hi.run(mark=mark)
+class Timer:
+    """Timed loops and eager per-call splits over one step function, with L2
+    flushed before every step and CUDA events on the launching stream."""
 
-    for _ in range(args.warmup):
-        flush.fill_(1)
-        step(lambda n: None)
-    torch.cuda.synchronize()
+    def __init__(self, flush, stream, clock, world):
+        self.flush, self.stream, self.clock, self.world = flush, stream, clock, world
 
-    K = args.steps
-    use_graph = not (args.no_graph or args.profile)
+    def timed(self, replay, K):
+        """ms of each of K steps (events around each replay) and the clocks
+        sampled during the loop."""
+        barrier(self.world)
+        torch.cuda.synchronize()
+        self.clock.start()
+        wall0 = time.perf_counter()
+        evs = []
+        for _ in range(K):
+            self.flush.fill_(1)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(self.stream)
+            replay()
+            e1.record(self.stream)
+            evs.append((e0, e1))
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - wall0
+        barrier(self.world)
+        clocks = self.clock.stop()
+        return [a.elapsed_time(b) for a, b in evs], clocks, wall
 
-    def eager_steps(n):
-        """n eager steps with a CUDA event after every library call:
-        per-call durations and per-step (train, hard) sums."""
+    def eager_split(self, step, n):
+        """n eager steps with an event after every library call: mean ms per
+        call and per step."""
         marks = []
         for _ in range(n):
-            flush.fill_(1)
+            self.flush.fill_(1)
             lst = []
             marks.append(lst)
 
             def mark(name, lst=lst):
                 ev = torch.cuda.Event(enable_timing=True)
-                ev.record(stream)
+                ev.record(self.stream)
                 lst.append((name, ev))
             mark("start")
             step(mark)
         torch.cuda.synchronize()
-        calls, train_ms, hard_ms = {}, [], []
+        calls, totals = {}, []
         for lst in marks:
             prev = lst[0][1]
-            t_train = 0.0
-            t_total = 0.0
+            tot = 0.0
             for name, ev in lst[1:]:
                 dt = prev.elapsed_time(ev)
                 prev = ev
-                if name == "train_end":
-                    t_train = t_total
-                    continue
                 calls.setdefault(name, []).append(dt)
-                t_total += dt
-            train_ms.append(t_train)
-            hard_ms.append(t_total - t_train)
-        return calls, train_ms, hard_ms
+                tot += dt
+            totals.append(tot)
+        return {n: float(np.mean(v)) for n, v in calls.items()}, float(np.mean(totals))
 
-    if use_graph:
-        # the step as two CUDA graphs (training fwd+bwd; hard pass with its
-        # binarization), replayed in the timed loop
-        g_train = st.capture() if st is not None else None
-        g_hard = hi.capture(binarize=True)
-        for _ in range(3):
-            flush.fill_(1)
-            if g_train is not None:
-                g_train.replay()
-            g_hard.replay()
-        torch.cuda.synchronize()
 
-    clock = ClockSampler(local)
-    if world > 1:
-        torch.distributed.barrier()
-    torch.cuda.synchronize()
-    clock.start()
-    wall0 = time.perf_counter()
-    if use_graph:
-        evs = []
-        for _ in range(K):
-            flush.fill_(1)
-            e = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
-            e[0].record(stream)
-            if g_train is not None:
-                g_train.replay()
-            e[1].record(stream)
-            g_hard.replay()
-            e[2].record(stream)
-            evs.append(e)
-        torch.cuda.synchronize()
-        train_ms = [e[0].elapsed_time(e[1]) for e in evs]
-        hard_ms = [e[1].elapsed_time(e[2]) for e in evs]
+def build_train(wl, rank, node="soft"):
+    from paper_2602_07400_gb300.pipeline import Network, RoutedNetwork, RoutedTrainStep, TrainStep
+    B = wl.batch
+    if wl.Kc:
+        rnet = RoutedNetwork(*synth.routed_network(wl, seed=0), wl.w_in)
+        st = RoutedTrainStep(rnet, B, wl.d, wl.thresholds, wl.classes, wl.tau, node=node)
+        net = rnet
     else:
-        calls, train_ms, hard_ms = eager_steps(K)
-    wall = time.perf_counter() - wall0
-    if world > 1:
-        torch.distributed.barrier()
-    clocks = clock.stop()
-    assert bl.bitlogic_device_error() == 0
-    train_sum, hard_sum = max_over_ranks([sum(train_ms), sum(hard_ms)], "cuda")
-    eager_ms = None
+        conn1, th1, conn2, th2 = synth.network(wl, seed=0)
+        net = Network(conn1, th1, conn2, th2, wl.w_in)
+        st = TrainStep(net, B, wl.d, wl.thresholds, wl.classes, wl.tau, node=node)
+    x, lab = synth.blob_batch(B, wl.d, wl.classes, wl.sigma, seed=1000 + rank)
+    st.load(x.cuda(), lab.cuda())
+    return net, st
+
+
+def measure_train(wl, st, args, timer, hbm, sm_max, peak_kind, sms, world, detail=True):
+    """Timed training steps of ``st`` (graph replays unless --no-graph), the
+    per-call split and the roofline of the dominant single-kernel call."""
+    import paper_2602_07400_gb300 as bl
+    B, K = wl.batch, args.steps
+    for _ in range(args.warmup):
+        timer.flush.fill_(1)
+        st.run()
+    torch.cuda.synchronize()
+    use_graph = not (args.no_graph or args.profile)
     if use_graph:
-        # per-call split (and the roofline kernel's duration) from eager steps
-        # with an event after every call, outside the timed loop
-        calls, tr_e, hd_e = eager_steps(max(3, min(K, 100)))
-        eager_ms = {"train": float(np.mean(tr_e)), "hard": float(np.mean(hd_e))}
-
-    launches = K * (hi.kernels_per_binarize + hi.kernels_per_run)
-    if st is not None:
-        launches += K * st.kernels_per_run
-
-    result = None
-    if rank == 0:
-        hbm, sm_max, peak_kind = peaks()
-        work = call_work_routed(wl, B) if wl.Kc else call_work(wl, B, fuse_dy1=st.fuse_dy1 if st is not None else False)
-        per_call_ms = {n: float(np.mean(v)) for n, v in calls.items()}
-        ms_step_train = train_sum / K
-        ms_step_hard = hard_sum / K
-        # roofline of the dominant single-kernel call
-        single = {n: t for n, t in per_call_ms.items() if n not in ("head", "binarize", "hard2", "route_bwd2")}
-        dom = max(single, key=single.get)
-        byts, ops = work[dom]
-        t_s = per_call_ms[dom] * 1e-3
-        fp32_peak = 152 * FP32_LANES_PER_SM * sm_max * 1e6
-        t_hbm, t_alu = byts / (hbm * 1e9), ops / fp32_peak
-        if t_alu >= t_hbm:
-            unit = ("Tops/s (integer mux lane-ops against the issue rate)" if dom.startswith("hard")
-                    else "Tops/s (fp32 pipe lane-ops)")
-            roof = {"bound": "alu", "achieved": ops / t_s / 1e12, "peak": fp32_peak / 1e12, "unit": unit}
-        else:
-            roof = {"bound": "hbm", "achieved": byts / t_s / 1e9, "peak": hbm, "unit": "GB/s"}
-        roof["frac"] = roof["achieved"] / roof["peak"]
-        traffic, traffic_note = kernel_traffic(wl.name, dom)
-        roof.update({"traffic": traffic, "traffic_source": traffic_note, "kernel": KERNEL_OF_CALL[dom], "call": dom,
-                     "ms_per_launch": per_call_ms[dom], "algorithmic_bytes": byts,
-                     "algorithmic_ops": ops, "peak_source": f"{peak_kind} (HBM), "
-                     f"152 SMs x {FP32_LANES_PER_SM} lanes x {sm_max:.0f} MHz (alu: one issue per lane "
-                     f"and clock)"})
-        calls_out = {}
-        for n, t in per_call_ms.items():
-            b_, o_ = work[n]
-            calls_out[n] = {"ms": round(t, 5), "GB/s": round(b_ / (t * 1e-3) / 1e9, 1),
-                            "Tops/s": round(o_ / (t * 1e-3) / 1e12, 2) if o_ else None}
-        value = job_rate(world, B, K, train_sum if st is not None else hard_sum)
-        result = {
-            "metric": METRIC,
-            "value": value,
-            "unit": "samples/s",
-            "n_gpus": world,
-            "steps": K,
-            "warmup": args.warmup,
-            "ms_per_step": ms_step_train if st is not None else ms_step_hard,
-            "higher_is_better": True,
-            "scaling": "weak",
-            "vs_baseline": None,
-            "dtype": "f32",
-            "data": "synthetic (seeded class-conditional Gaussian blobs, MNIST/CIFAR shapes; random-init tables)",
-            "config": {"workload": wl.name, "batch_per_gpu": B, "d": wl.d, "thresholds": list(wl.thresholds),
-                       "widths": list(wl.widths), "k": wl.k, "classes": wl.classes, "tau": wl.tau,
-                       "routing": f"learnable, {wl.Kc} candidates per slot" if wl.Kc else "fixed (random-unique)",
-                       "node": "LightLUT " + ("soft" if args.node == "soft" else "straight-through hard"),
-                       "l2": "flushed between steps (512 MB write outside the timed events)",
-                       "parallelism": f"dp{world} (independent batches, no collective)"},
-            "hard": {"value": job_rate(world, B, K, hard_sum) / 1e6, "unit": "MSamples/s",
-                     "ms_per_batch": ms_step_hard, "batch": B,
-                     "includes": "binarize + encode/pack + 2 hard layers + popcount head + argmax"},
-            "ms_per_step_total": ms_step_train + ms_step_hard,
-            "timing": ("CUDA-graph replays of the step (training fwd+bwd graph, hard-pass graph), CUDA events "
-                       "around each replay; per-call split from eager steps with an event after every call"
-                       if use_graph else "eager launches, CUDA events after every library call"),
-            **({"eager_ms_per_step": eager_ms} if eager_ms else {}),
-            **({"context": PAPER_CONTEXT[wl.name]} if wl.name in PAPER_CONTEXT else {}),
-            "calls": calls_out,
-            "roofline": roof,
-            "gpu_launches": launches,
-            "clocks": clocks,
-            "wall_s_timed_loop": wall,
-        }
-    if st is not None and not args.profile:
-        # the AdamW update of both layers' logits (not part of `value`, which
-        # is the fwd+bwd step): timed on its own from the last gradients
-        upd = time_update(st, max(3, min(args.steps, 50)))
-        if result is not None:
-            n_par = int(st.net.theta1.numel() + st.net.theta2.numel())
-            if wl.Kc:
-                n_par += int(st.net.r1.numel() + st.net.r2.numel())
-            result["optimizer"] = {"ms_per_update": upd,
-                                   "kernel": f"adamw_vec_kernel (x{4 if wl.Kc else 2})",
-                                   "algorithmic_bytes": 28 * n_par,
-                                   "GB/s": 28 * n_par / (upd * 1e-3) / 1e9,
-                                   "settings": "AdamW beta (0.9, 0.999), eps 1e-8, lr 0.01, wd 0"}
-    if st is not None and world > 1 and not args.profile:
-        # the data-parallel exchange of a training step (all-reduce of the
-        # gradients before the update), timed on its own: the fwd+bwd step
-        # above has no collective
-        from paper_2602_07400_gb300.pipeline import allreduce_gradients
-        grads = st.gradients()
+        g = st.capture()
         for _ in range(3):
-            allreduce_gradients(grads)
+            timer.flush.fill_(1)
+            g.replay()
         torch.cuda.synchronize()
-        torch.distributed.barrier()
+        ms, clocks, wall = timer.timed(g.replay, K)
+    else:
+        ms, clocks, wall = timer.timed(st.run, K)
+    assert bl.bitlogic_device_error() == 0
+    tot = max_over_ranks([sum(ms)], "cuda")[0]
+    per_call, eager_step = timer.eager_split(lambda mark: st.run(mark=mark), max(3, min(K, 30)))
+    work = call_work_routed(wl, B) if wl.Kc else call_work(wl, B, fuse_dy1=st.fuse_dy1)
+    single = {n: t for n, t in per_call.items() if n not in MULTI_KERNEL_CALLS}
+    dom = max(single, key=single.get)
+    res = {
+        "value": job_rate(world, B, K, tot), "unit": "samples/s", "ms_per_step": tot / K,
+        "eager_ms_per_step": eager_step,
+        "roofline": roofline_of(dom, work, per_call, sms, clocks, wl.name, hbm, sm_max, peak_kind),
+        "calls": calls_table(work, per_call, hbm),
+        "step_hbm": step_hbm_fraction(work, per_call.keys(), tot / K, hbm),
+        "gpu_launches": K * st.kernels_per_run,
+        "clocks": clocks, "wall_s_timed_loop": wall,
+        "timing": ("CUDA-graph replays of the training step (fwd+bwd), CUDA events around each replay; "
+                   "per-call split from eager steps with an event after every call" if use_graph else
+                   "eager launches, CUDA events around each step"),
+    }
+    if detail:
+        res["roofline_by_call"] = {n: {k_: v for k_, v in roofline_of(n, work, per_call, sms, clocks, wl.name,
+                                                                      hbm, sm_max, peak_kind).items()
+                                       if k_ in ("bound", "frac", "frac_at_sampled_clock", "achieved", "unit")}
+                                   for n in single}
+    return res
+
+
+def build_hard(wl, net, rank, x_dev=None):
+    from paper_2602_07400_gb300.pipeline import HardInfer
+    hi = HardInfer(net, wl.batch, wl.d, wl.thresholds, wl.classes)
+    if x_dev is not None:
+        hi.x = x_dev                 # evaluate the training batch
+    else:
+        x, _ = synth.blob_batch(wl.batch, wl.d, wl.classes, wl.sigma, seed=1000 + rank, device="cuda")
+        hi.x.copy_(x)
+        del x
+    return hi
+
+
+def measure_hard(wl, hi, args, timer, hbm, sm_max, peak_kind, sms, world):
+    """Timed hard passes (binarize + pack + 2 layers + popcount head + argmax)."""
+    import paper_2602_07400_gb300 as bl
+    N, K = wl.batch, args.steps
+    for _ in range(max(1, args.warmup)):
+        timer.flush.fill_(1)
+        hi.binarize()
+        hi.run()
+    torch.cuda.synchronize()
+    use_graph = not (args.no_graph or args.profile)
+    if use_graph:
+        g = hi.capture(binarize=True)
+        for _ in range(2):
+            timer.flush.fill_(1)
+            g.replay()
+        torch.cuda.synchronize()
+        ms, clocks, wall = timer.timed(g.replay, K)
+    else:
+        ms, clocks, wall = timer.timed(lambda: (hi.binarize(), hi.run()), K)
+    assert bl.bitlogic_device_error() == 0
+    tot = max_over_ranks([sum(ms)], "cuda")[0]
+
+    def step(mark):
+        hi.binarize(mark=mark)
+        hi.run(mark=mark)
+    n_split = max(3, min(K, 100 if N <= (1 << 16) else 10))
+    per_call, eager_step = timer.eager_split(step, n_split)
+    work = call_work(wl, N)
+    per_call_w = {n: t for n, t in per_call.items()}
+    res = {
+        "value": job_rate(world, N, K, tot) / 1e6, "unit": "MSamples/s", "ms_per_batch": tot / K,
+        "batch": N, "eager_ms_per_batch": eager_step,
+        "includes": "binarize + encode/pack + 2 hard layers + popcount head + argmax",
+        "calls": calls_table(work, per_call_w, hbm),
+        "gpu_launches": K * (hi.kernels_per_binarize + hi.kernels_per_run),
+        "clocks": clocks, "wall_s_timed_loop": wall,
+    }
+    roof = roofline_of("hard1", work, per_call_w, sms, clocks, wl.name, hbm, sm_max, peak_kind)
+    res["roofline"] = roof
+    # layer 2 with the fused head: its mux tree against the same peak (the
+    # call also runs the argmax kernel, a few hundred microseconds at 2^22)
+    r2 = roofline_of("hard2", work, per_call_w, sms, clocks, wl.name, hbm, sm_max, peak_kind)
+    res["roofline_hard2"] = {k_: r2[k_] for k_ in ("bound", "achieved", "peak", "unit", "frac", "ms_per_launch")
+                             if k_ in r2}
+    return res
+
+
+def run_e2e_train(st, wl, K, world, rank, use_graph=True):
+    """The training metric end to end through the public API: every step
+    copies its batch (raw uint8 samples and labels) from pinned host memory
+    and reads the loss back.  With graphs, ``pipeline.Prefetcher`` overlaps
+    the copy of the next batch with the current step (two input buffers, a
+    copy stream); without, the copy, the step and the read-back run in
+    sequence."""
+    from paper_2602_07400_gb300.pipeline import Prefetcher
+    B = wl.batch
+    x_host, lab_host = synth.blob_batch(B, wl.d, wl.classes, wl.sigma, seed=2000 + rank)
+    x_host, lab_host = x_host.pin_memory(), lab_host.pin_memory()
+    loss_host = torch.empty(1, dtype=torch.float32).pin_memory()
+
+    def eager():
+        st.load(x_host, lab_host, non_blocking=True)
+        st.run()
+        loss_host.copy_(st.loss, non_blocking=True)
+    pf = Prefetcher(st, ("x", "labels"), "loss") if use_graph else None
+    ms = _e2e_loop(pf, {"x": x_host, "labels": lab_host}, loss_host, eager, K)
+    return {"value": job_rate(world, B, K, ms), "unit": "samples/s",
+            "h2d_bytes_per_step": x_host.numel() + 4 * lab_host.numel(),
+            "d2h_bytes_per_step": 4, "overlap": bool(use_graph)}
+
+
+def run_e2e_hard(hi, wl, K, world, rank, use_graph=True):
+    """The hard metric end to end: every batch of raw samples is copied from
+    pinned host memory and the predictions are read back.  For the large
+    batches the host copy of the samples is taken from the device-generated
+    batch (drawing 2^22 x 3072 pixels on the host would take minutes)."""
+    from paper_2602_07400_gb300.pipeline import Prefetcher
+    N = wl.batch
+    if N > (1 << 16):
+        x_host = torch.empty(N, wl.d, dtype=torch.uint8).pin_memory()
+        x_host.copy_(hi.x)
+    else:
+        x_host, _ = synth.blob_batch(N, wl.d, wl.classes, wl.sigma, seed=2000 + rank)
+        x_host = x_host.pin_memory()
+    pred_host = torch.empty(N, dtype=torch.int32).pin_memory()
+
+    def eager():
+        hi.x.copy_(x_host, non_blocking=True)
+        hi.binarize()
+        hi.run()
+        pred_host.copy_(hi.pred, non_blocking=True)
+    pf = Prefetcher(hi, ("x",), "pred", capture=lambda: hi.capture(binarize=True)) if use_graph else None
+    ms = _e2e_loop(pf, {"x": x_host}, pred_host, eager, K)
+    del pf
+    return {"value": job_rate(world, N, K, ms) / 1e6, "unit": "MSamples/s",
+            "h2d_bytes_per_step": x_host.numel(), "d2h_bytes_per_step": 4 * N, "overlap": bool(use_graph)}
+
+
+def _e2e_loop(pf, host, res, eager, K):
+    if pf is None:
+        for _ in range(3):
+            eager()
+        torch.cuda.synchronize()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record()
-        for _ in range(20):
-            allreduce_gradients(grads)
+        for _ in range(K):
+            eager()
         e1.record()
         torch.cuda.synchronize()
-        ms_x = max_over_ranks([e0.elapsed_time(e1) / 20], "cuda")[0]
-        if result is not None:
-            result["dp_exchange"] = {"ms": ms_x, "collective": "NCCL all-reduce (sum) of the gradients, then / N",
-                                     "bytes_per_rank": int(sum(g.numel() * 4 for g in grads))}
-    if not args.profile and rank == 0:
-        result["fit"] = time_quantile_fit(wl, flush)
-        result["pipe_rates"] = measure_pipe_rates()
-        if result["roofline"]["call"] in ("hard1", "hard2"):
-            result["roofline"]["integer_pipes"] = integer_pipe_fraction(result["roofline"], result["pipe_rates"])
-    if not args.profile and not args.no_e2e:
-        e2e = run_e2e(args, st, hi, wl, B, use_graph)
-        if result is not None:
-            result["e2e"] = e2e["train"] if st is not None else e2e["hard"]
-            result["hard"]["e2e"] = e2e["hard"]
-    if world > 1:
-        torch.distributed.barrier()
-        torch.distributed.destroy_process_group()
-    return result
+        return max_over_ranks([e0.elapsed_time(e1)], "cuda")[0]
+    for _ in range(3):
+        pf.prefetch(host)
+        pf.run(res)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    pf.start()
+    pf.prefetch(host)
+    for i in range(K):
+        if i + 1 < K:
+            pf.prefetch(host)   # batch i + 1 streams in while step i runs
+        pf.run(res)
+    e1.record()
+    torch.cuda.synchronize()
+    return max_over_ranks([e0.elapsed_time(e1)], "cuda")[0]
+
+
+def free_cuda():
+    import gc
+    gc.collect()
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+
+
+def config_of(wl, world, node="soft"):
+    return {"workload": wl.name, "batch_per_gpu": wl.batch, "d": wl.d, "thresholds": list(wl.thresholds),
+            "widths": list(wl.widths), "k": wl.k, "classes": wl.classes, "tau": wl.tau,
+            "routing": f"learnable, {wl.Kc} candidates per slot" if wl.Kc else "fixed (random-unique)",
+            "node": "LightLUT " + ("soft" if node == "soft" else "straight-through hard"),
+            "l2": "flushed between steps (512 MB write outside the timed events)",
+            "parallelism": f"dp{world} (independent batches, no collective)"}
+
+
+def base_line(world, K, W):
+    return {"metric": METRIC, "n_gpus": world, "steps": K, "warmup": W, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic (seeded class-conditional Gaussian blobs, MNIST/CIFAR shapes; random-init tables)"}
+
+
+def run_headline(args):
+    """The default run: CIFAR-100-shaped training (value), 2^22-sample hard
+    pass of the CIFAR-10-shaped network (hard), extra training workloads."""
+    import paper_2602_07400_gb300 as bl
+    world, rank, local = dist_env()
+    hbm, sm_max, peak_kind = peaks()
+    sms = device_sms(local)
+    flush = torch.empty(512 << 20, dtype=torch.uint8, device="cuda")
+    stream = torch.cuda.current_stream()
+    clock = ClockSampler(local)
+    timer = Timer(flush, stream, clock, world)
+    use_graph = not (args.no_graph or args.profile)
+    K = args.steps
+
+    # -- headline training workload
+    wl = with_batch(synth.WORKLOADS[HEADLINE_TRAIN], args.batch)
+    net, st = build_train(wl, rank, args.node)
+    train = measure_train(wl, st, args, timer, hbm, sm_max, peak_kind, sms, world)
+    upd = time_update(st, max(3, min(K, 20)))
+    n_par = int(net.theta1.numel() + net.theta2.numel())
+    optimizer = {"ms_per_update": upd, "kernel": "adamw_vec_kernel (x2)", "algorithmic_bytes": 28 * n_par,
+                 "GB/s": 28 * n_par / (upd * 1e-3) / 1e9,
+                 "settings": "AdamW beta (0.9, 0.999), eps 1e-8, lr 0.01, wd 0"}
+    dp = time_dp_exchange(st, world) if world > 1 else None
+    e2e = None if (args.no_e2e or args.profile) else run_e2e_train(st, wl, K, world, rank, use_graph)
+    del st, net
+    free_cuda()
+
+    # -- headline hard workload (its own network and 2^22 samples)
+    wh = synth.WORKLOADS[HEADLINE_HARD]
+    if args.batch:
+        wh = with_batch(wh, max(32, args.batch))
+    from paper_2602_07400_gb300.pipeline import Network
+    conn1, th1, conn2, th2 = synth.network(wh, seed=0)
+    hnet = Network(conn1, th1, conn2, th2, wh.w_in)
+    hi = build_hard(wh, hnet, rank)
+    hard = measure_hard(wh, hi, args, timer, hbm, sm_max, peak_kind, sms, world)
+    if not args.profile:
+        rates = measure_pipe_rates(sms)
+        hard["roofline"]["integer_pipes"] = integer_pipe_fraction(hard["roofline"], rates)
+    if not (args.no_e2e or args.profile):
+        hard["e2e"] = run_e2e_hard(hi, wh, K, world, rank, use_graph)
+    hard["config"] = config_of(wh, world)
+    del hi, hnet
+    free_cuda()
+
+    # -- extra training workloads: value, split and roofline each
+    extra = {}
+    names = [] if (args.no_extras or args.profile) else [n for n in args.extras.split(",") if n]
+    for name in names:
+        we = synth.WORKLOADS[name]
+        enet, est = build_train(we, rank, args.node)
+        r = measure_train(we, est, args, timer, hbm, sm_max, peak_kind, sms, world, detail=False)
+        r["config"] = {k_: v for k_, v in config_of(we, world, args.node).items()
+                       if k_ in ("workload", "batch_per_gpu", "widths", "k", "classes", "tau")}
+        extra[name] = r
+        del est, enet
+        free_cuda()
+
+    if rank != 0:
+        return None
+    out = base_line(world, K, args.warmup)
+    out.update({
+        "value": train["value"], "unit": "samples/s", "ms_per_step": train["ms_per_step"],
+        "config": config_of(wl, world, args.node),
+        "roofline": train["roofline"],
+        "gpu_launches": train["gpu_launches"],
+        "clocks": train["clocks"],
+        "timing": train["timing"],
+        "eager_ms_per_step": train["eager_ms_per_step"],
+        "calls": train["calls"],
+        "roofline_by_call": train["roofline_by_call"],
+        "step_hbm": train["step_hbm"],
+        "wall_s_timed_loop": train["wall_s_timed_loop"],
+        "optimizer": optimizer,
+        "hard": hard,
+        "extra": extra,
+        "clocks_all_timed_loops": clock.summary(),
+        "gpu_launches_all_timed_loops": train["gpu_launches"] + hard["gpu_launches"] +
+        sum(v["gpu_launches"] for v in extra.values()),
+    })
+    if dp:
+        out["dp_exchange"] = dp
+    if e2e:
+        out["e2e"] = e2e
+    if not args.profile:
+        out["fit"] = time_quantile_fit(wl, flush)
+        out["pipe_rates"] = rates
+    return out
+
+
+def run_single(args):
+    """One workload: its training step and the hard pass on the same batch
+    (or the hard pass alone for the hard workloads)."""
+    import paper_2602_07400_gb300 as bl
+    world, rank, local = dist_env()
+    hbm, sm_max, peak_kind = peaks()
+    sms = device_sms(local)
+    wl = with_batch(synth.WORKLOADS[args.workload], args.batch)
+    hard_only = wl.name.startswith("hard_")
+    flush = torch.empty(512 << 20, dtype=torch.uint8, device="cuda")
+    stream = torch.cuda.current_stream()
+    clock = ClockSampler(local)
+    timer = Timer(flush, stream, clock, world)
+    use_graph = not (args.no_graph or args.profile)
+    K = args.steps
+    train = None
+    if hard_only:
+        from paper_2602_07400_gb300.pipeline import Network
+        net = Network(*synth.network(wl, seed=0), wl.w_in)
+        hi = build_hard(wl, net, rank)
+    else:
+        rnet, st = build_train(wl, rank, args.node)
+        net = rnet.snap() if wl.Kc else rnet   # the hard pass evaluates the discretized network
+        train = measure_train(wl, st, args, timer, hbm, sm_max, peak_kind, sms, world)
+        hi = build_hard(wl, net, rank, x_dev=st.x)
+    hard = measure_hard(wl, hi, args, timer, hbm, sm_max, peak_kind, sms, world)
+    rates = None
+    if not args.profile:
+        rates = measure_pipe_rates(sms)
+        hard["roofline"]["integer_pipes"] = integer_pipe_fraction(hard["roofline"], rates)
+    e2e_train = e2e_hard = None
+    if not (args.no_e2e or args.profile):
+        if train is not None:
+            e2e_train = run_e2e_train(st, wl, K, world, rank, use_graph)
+        e2e_hard = run_e2e_hard(hi, wl, K, world, rank, use_graph)
+    optimizer = None
+    if train is not None and not args.profile:
+        upd = time_update(st, max(3, min(K, 50)))
+        n_par = int(st.net.theta1.numel() + st.net.theta2.numel())
+        if wl.Kc:
+            n_par += int(st.net.r1.numel() + st.net.r2.numel())
+        optimizer = {"ms_per_update": upd, "kernel": f"adamw_vec_kernel (x{4 if wl.Kc else 2})",
+                     "algorithmic_bytes": 28 * n_par, "GB/s": 28 * n_par / (upd * 1e-3) / 1e9,
+                     "settings": "AdamW beta (0.9, 0.999), eps 1e-8, lr 0.01, wd 0"}
+    dp = time_dp_exchange(st, world) if (train is not None and world > 1 and not args.profile) else None
+    if rank != 0:
+        return None
+    out = base_line(world, K, args.warmup)
+    main = train if train is not None else hard
+    out.update({
+        "value": train["value"] if train else hard["value"],
+        "unit": "samples/s" if train else "MSamples/s",
+        "ms_per_step": train["ms_per_step"] if train else hard["ms_per_batch"],
+        "config": config_of(wl, world, args.node),
+        "roofline": main["roofline"],
+        "gpu_launches": main["gpu_launches"],
+        "clocks": main["clocks"],
+        "calls": main["calls"],
+        "hard": hard,
+    })
+    if train:
+        out.update({"timing": train["timing"], "eager_ms_per_step": train["eager_ms_per_step"],
+                    "roofline_by_call": train["roofline_by_call"], "step_hbm": train["step_hbm"],
+                    "wall_s_timed_loop": train["wall_s_timed_loop"]})
+    if wl.name in PAPER_CONTEXT:
+        out["context"] = PAPER_CONTEXT[wl.name]
+    if optimizer:
+        out["optimizer"] = optimizer
+    if dp:
+        out["dp_exchange"] = dp
+    if e2e_train:
+        out["e2e"] = e2e_train
+    if e2e_hard:
+        hard["e2e"] = e2e_hard
+        if train is None:
+            out["e2e"] = e2e_hard
+    if not args.profile:
+        out["fit"] = time_quantile_fit(wl, flush)
+        out["pipe_rates"] = rates
+    return out
+
+
+def time_dp_exchange(st, world):
+    """The data-parallel exchange of a training step (all-reduce of the
+    gradients before the update), timed on its own: the fwd+bwd step has no
+    collective."""
+    from paper_2602_07400_gb300.pipeline import allreduce_gradients
+    grads = st.gradients()
+    for _ in range(3):
+        allreduce_gradients(grads)
+    torch.cuda.synchronize()
+    torch.distributed.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(20):
+        allreduce_gradients(grads)
+    e1.record()
+    torch.cuda.synchronize()
+    ms_x = max_over_ranks([e0.elapsed_time(e1) / 20], "cuda")[0]
+    return {"ms": ms_x, "collective": "NCCL all-reduce (sum) of the gradients, then / N",
+            "bytes_per_rank": int(sum(g.numel() * 4 for g in grads))}
 
 
 # training split sizes of the datasets the workloads stand in for
@@ -575,7 +928,7 @@ def time_quantile_fit(wl, flush, iters: int = 20):
             "thresholds_b": [int(v) for v in thr]}
 
 
-def measure_pipe_rates(iters: int = 2048, reps: int = 5) -> dict:
+def measure_pipe_rates(sms: int, iters: int = 2048, reps: int = 5) -> dict:
     """Sustained issue rates of the pipes the kernels run on, from the
     library's throughput probe (independent chains of one instruction kind
     over 4 blocks of 256 threads per SM): LOP3 (logic pipe, the hard mux
@@ -583,7 +936,6 @@ def measure_pipe_rates(iters: int = 2048, reps: int = 5) -> dict:
     the soft kernels).  Median of `reps` launches, CUDA events."""
     import paper_2602_07400_gb300 as bl
     n = bl.bitlogic_issue_probe_threads()
-    sms = n // (4 * 256)
     sink = torch.empty(n, dtype=torch.int32, device="cuda")
     ops = n * iters * bl.bitlogic_issue_probe_ops_per_iter()
     _, sm_max, _ = peaks()
@@ -630,73 +982,6 @@ def time_update(st, iters: int) -> float:
     return e0.elapsed_time(e1) / iters
 
 
-def run_e2e(args, st, hi, wl, B, use_graph=True):
-    """The same metric end to end through the public API: every step copies
-    its batch from pinned host memory and its result (loss, or predictions)
-    back.  With graphs, ``pipeline.Prefetcher`` overlaps the copy of the
-    next batch with the current step (two input buffers, a copy stream);
-    without, the copy, the step and the read-back run in sequence."""
-    from paper_2602_07400_gb300.pipeline import Prefetcher
-    world, rank, _ = dist_env()
-    x_host, lab_host = synth.blob_batch(B, wl.d, wl.classes, wl.sigma, seed=2000 + rank)
-    x_host = x_host.pin_memory()
-    lab_host = lab_host.pin_memory()
-    loss_host = torch.empty(1, dtype=torch.float32).pin_memory()
-    pred_host = torch.empty(B, dtype=torch.int32).pin_memory()
-    K = max(1, args.steps)
-    out = {}
-
-    def timed(pf, host, res, eager):
-        if pf is None:
-            for _ in range(3):
-                eager()
-            torch.cuda.synchronize()
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            e0.record()
-            for _ in range(K):
-                eager()
-            e1.record()
-            torch.cuda.synchronize()
-            return max_over_ranks([e0.elapsed_time(e1)], "cuda")[0]
-        for _ in range(3):
-            pf.prefetch(host)
-            pf.run(res)
-        torch.cuda.synchronize()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record()
-        pf.start()
-        pf.prefetch(host)
-        for i in range(K):
-            if i + 1 < K:
-                pf.prefetch(host)   # batch i + 1 streams in while step i runs
-            pf.run(res)
-        e1.record()
-        torch.cuda.synchronize()
-        return max_over_ranks([e0.elapsed_time(e1)], "cuda")[0]
-
-    if st is not None:
-        def eager_train():
-            st.load(x_host, lab_host, non_blocking=True)
-            st.run()
-            loss_host.copy_(st.loss, non_blocking=True)
-        pf = Prefetcher(st, ("x", "labels"), "loss") if use_graph else None
-        ms = timed(pf, {"x": x_host, "labels": lab_host}, loss_host, eager_train)
-        out["train"] = {"value": job_rate(world, B, K, ms), "unit": "samples/s",
-                        "h2d_bytes_per_step": x_host.numel() + 4 * lab_host.numel(),
-                        "d2h_bytes_per_step": 4, "overlap": bool(use_graph)}
-
-    def eager_hard():
-        hi.x.copy_(x_host, non_blocking=True)
-        hi.binarize()
-        hi.run()
-        pred_host.copy_(hi.pred, non_blocking=True)
-    pf = Prefetcher(hi, ("x",), "pred", capture=lambda: hi.capture(binarize=True)) if use_graph else None
-    ms = timed(pf, {"x": x_host}, pred_host, eager_hard)
-    out["hard"] = {"value": job_rate(world, B, K, ms) / 1e6, "unit": "MSamples/s",
-                   "h2d_bytes_per_step": x_host.numel(), "d2h_bytes_per_step": 4 * B, "overlap": bool(use_graph)}
-    return out
-
-
 # -------------------------------------------------- oracle (CPU) legs --
 
 _NETWORKS = {}
@@ -741,61 +1026,88 @@ def calibrated(rate_fn, wl, budget_s: float, lo: int, hi: int):
     return rate_fn(wl, n, seed=1), n
 
 
-def cpu_baseline(wl, budget_s=12.0, node="soft"):
+def cpu_baseline_train(wl, budget_s=12.0, node="soft"):
     import oracle
-    hard_only = wl.name.startswith("hard_")
     cores = oracle.max_threads()
-    out = {}
-    if not hard_only:
-        r, n = calibrated(lambda w_, n_, seed=0: oracle_train_rate(w_, n_, seed, node), wl, budget_s, 4, wl.batch)
-        out = {"value": r, "unit": "samples/s", "cores": cores, "kind": "oracle",
-               "sample": f"train step (fwd+bwd) on {n} of the {wl.batch} samples of a batch, "
-                         f"full network, fp64, OpenMP over independent outputs"}
-    rh, nh = calibrated(oracle_hard_rate, wl, budget_s / 2, 32, 1 << 16)
-    hard = {"value": rh / 1e6, "unit": "MSamples/s", "cores": cores, "kind": "oracle",
-            "sample": f"hard pass (encode+pack, 2 layers, popcount head) on {nh} samples"}
-    return out, hard
+    r, n = calibrated(lambda w_, n_, seed=0: oracle_train_rate(w_, n_, seed, node), wl, budget_s, 4, wl.batch)
+    return {"value": r, "unit": "samples/s", "cores": cores, "kind": "oracle",
+            "sample": f"train step (fwd+bwd) on {n} of the {wl.batch} samples of a batch, "
+                      f"full {wl.widths[0]} x {wl.widths[1]} network, fp64, OpenMP over independent outputs"}
+
+
+def cpu_baseline_hard(wl, budget_s=6.0):
+    import oracle
+    cores = oracle.max_threads()
+    rh, nh = calibrated(oracle_hard_rate, wl, budget_s, 32, 1 << 16)
+    return {"value": rh / 1e6, "unit": "MSamples/s", "cores": cores, "kind": "oracle",
+            "sample": f"hard pass (encode+pack, 2 layers, popcount head) on {nh} of the {wl.batch} samples"}
+
+
+def _reference_rate(fn, wl, lo, steps, warmup, per_step_s, calib_n):
+    """Oracle rate over `steps` bounded samples of the workload (each about
+    per_step_s of work) after `warmup` small ones."""
+    r0 = fn(wl, min(wl.batch, calib_n))
+    n = max(lo, int(r0 * per_step_s) // lo * lo)
+    n = min(n, wl.batch)
+    for i in range(warmup):
+        fn(wl, lo, seed=100 + i)
+    tot_s, tot_n = 0.0, 0
+    for i in range(steps):
+        r = fn(wl, n, seed=i)
+        tot_s += n / r
+        tot_n += n
+    return tot_n / tot_s, n, tot_s
 
 
 def run_reference(args):
+    """The oracle as it stands on the host cores, on the same workloads,
+    metric and unit as the GPU arm (each step a bounded sample)."""
     world, rank, _ = dist_env()
     if rank != 0:
         return None
     import oracle
+    cores = oracle.max_threads()
+    K, W = args.steps, args.warmup
+    train_fn = lambda w_, n_, seed=0: oracle_train_rate(w_, n_, seed, args.node)  # noqa: E731
+    out = {"impl": "reference"}
+    out.update(base_line(world, K, W))
+    out["dtype"] = "f64"
+    if args.workload is None:
+        # about 90 s of training-step oracle work and 30 s of hard-pass work
+        wl = synth.WORKLOADS[HEADLINE_TRAIN]
+        wh = synth.WORKLOADS[HEADLINE_HARD]
+        v, n, tot = _reference_rate(train_fn, wl, 2, K, W, min(3.0, 90.0 / max(1, K + W)), 8)
+        vh, nh, _ = _reference_rate(oracle_hard_rate, wh, 32, K, W, min(1.0, 30.0 / max(1, K + W)), 4096)
+        out.update({"value": v, "unit": "samples/s", "ms_per_step": 1e3 * tot / max(1, K),
+                    "config": {"workload": wl.name, "batch_per_gpu": wl.batch},
+                    "cpu_baseline": {"value": v, "unit": "samples/s", "cores": cores, "kind": "oracle",
+                                     "sample": f"{n} samples of the workload per step (the plain C oracle, "
+                                               f"train fwd+bwd)"},
+                    "e2e": {"value": v, "unit": "samples/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+                    "hard": {"value": vh / 1e6, "unit": "MSamples/s", "config": {"workload": wh.name,
+                                                                                "batch_per_gpu": wh.batch},
+                             "cpu_baseline": {"value": vh / 1e6, "unit": "MSamples/s", "cores": cores,
+                                              "kind": "oracle",
+                                              "sample": f"{nh} samples of the workload per step (hard pass)"}}})
+        return out
     wl = synth.WORKLOADS[args.workload]
     hard_only = wl.name.startswith("hard_")
-    fn = oracle_hard_rate if hard_only else (lambda w_, n_, seed=0: oracle_train_rate(w_, n_, seed, args.node))
+    fn = oracle_hard_rate if hard_only else train_fn
     lo = 32 if hard_only else 2
     # size one step so that the whole run (warm-up and timed steps) takes
-    # about two minutes of oracle work, at most 1.5 s per step; the rate is
-    # calibrated on a sample large enough to amortise the per-call set-up
-    per_step_s = min(1.5, 120.0 / max(1, args.steps + args.warmup))
-    r0 = fn(wl, min(wl.batch, 4096 if hard_only else 64))
-    n = max(lo, int(r0 * per_step_s) // lo * lo)
-    n = min(n, wl.batch)
-    for i in range(args.warmup):
-        fn(wl, lo, seed=100 + i)
-    tot_s, tot_n = 0.0, 0
-    for i in range(args.steps):
-        r = fn(wl, n, seed=i)
-        tot_s += n / r
-        tot_n += n
-    value = tot_n / tot_s
+    # about two minutes of oracle work, at most 1.5 s per step
+    v, n, tot = _reference_rate(fn, wl, lo, K, W, min(1.5, 120.0 / max(1, K + W)), 4096 if hard_only else 64)
     unit = "samples/s"
     if hard_only:
-        value /= 1e6
+        v /= 1e6
         unit = "MSamples/s"
-    cores = oracle.max_threads()
-    return {
-        "impl": "reference", "metric": METRIC, "value": value, "unit": unit, "n_gpus": world,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot_s / max(1, args.steps),
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic", "config": {"workload": wl.name, "batch_per_gpu": wl.batch},
-        "cpu_baseline": {"value": value, "unit": unit, "cores": cores, "kind": "oracle",
-                         "sample": f"{n} samples of the workload per step (the plain C oracle, "
-                                   f"{'hard pass' if hard_only else 'train fwd+bwd'})"},
-        "e2e": {"value": value, "unit": unit, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
-    }
+    out.update({"value": v, "unit": unit, "ms_per_step": 1e3 * tot / max(1, K),
+                "config": {"workload": wl.name, "batch_per_gpu": wl.batch},
+                "cpu_baseline": {"value": v, "unit": unit, "cores": cores, "kind": "oracle",
+                                 "sample": f"{n} samples of the workload per step (the plain C oracle, "
+                                           f"{'hard pass' if hard_only else 'train fwd+bwd'})"},
+                "e2e": {"value": v, "unit": unit, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}})
+    return out
 
 
 def main():
@@ -805,15 +1117,30 @@ def main():
         if res is not None:
             print(json.dumps(res), flush=True)
         return
-    res = run_ours(args)
+    world, rank, local = dist_env()
+    torch.cuda.set_device(local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    import paper_2602_07400_gb300 as bl
+    bl.load()
+    res = run_headline(args) if args.workload is None else run_single(args)
+    if world > 1:
+        torch.distributed.barrier()
+        torch.distributed.destroy_process_group()
     if res is None:
         return
     if not args.profile and not args.no_cpu_baseline:
-        wl = synth.WORKLOADS[args.workload]
-        cb, cb_hard = cpu_baseline(wl, node=args.node)
-        if cb:
-            res["cpu_baseline"] = cb
-        res["hard"]["cpu_baseline"] = cb_hard
+        if args.workload is None:
+            res["cpu_baseline"] = cpu_baseline_train(synth.WORKLOADS[HEADLINE_TRAIN], node=args.node)
+            res["hard"]["cpu_baseline"] = cpu_baseline_hard(synth.WORKLOADS[HEADLINE_HARD])
+        else:
+            wl = synth.WORKLOADS[args.workload]
+            if not wl.name.startswith("hard_"):
+                res["cpu_baseline"] = cpu_baseline_train(wl, node=args.node)
+            res["hard"]["cpu_baseline"] = cpu_baseline_hard(wl)
+            if wl.name.startswith("hard_"):
+                res["cpu_baseline"] = res["hard"]["cpu_baseline"]
     print(json.dumps(res), flush=True)
 
 

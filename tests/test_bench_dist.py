@@ -117,8 +117,19 @@ def test_algorithmic_work_of_the_roofline_calls():
     work = bench.call_work(wl, 1024)
     B, w, k, K, C = 1024, 8000, 6, 64, 10
     assert work["backward2"][1] == 316 * w * B
-    assert work["backward2"][0] == 4 * (w * B + C * B + w * k * B + 2 * w * K + w * k)
+    # algorithmic bytes leave out the per-edge terms (implementation
+    # overhead); the bytes moved carry them (written here, read by csr2)
+    assert work["backward2"][0] == 4 * (w * B + C * B + 2 * w * K + w * k)
+    assert work["backward2"][2] == work["backward2"][0] + 4 * w * k * B
+    # the layer-2 backward with input gradient (backward2 + csr2) moves
+    # X, the per-class dY rows, dX, the table and its gradient, the
+    # connectivity and the CSR map once each
+    w_in1 = 8000
+    assert work["backward2"][0] + work["csr2"][0] == 4 * (w * B + C * B + w_in1 * B + 2 * w * K + w * k +
+                                                          (w_in1 + 1) + w * k)
+    assert work["csr2"][2] == work["csr2"][0] + 4 * w * k * B
     assert work["forward2"][1] == 132 * w * B
+    assert work["forward2"][0] == work["forward2"][2] == 4 * (w * B + w * B + w * K + w * k)
     hw = synth.WORKLOADS["hard_cifar10"]
     N = 1 << 22
     W = N // 32
@@ -133,3 +144,40 @@ def test_integer_pipe_ceiling_is_the_sum_of_both_pipes():
     rates = {"imad": {"T_lane_ops_s": 12.0}, "lop3": {"T_lane_ops_s": 8.0}}
     got = bench.integer_pipe_fraction(roof, rates)
     assert got["peak"] == 20.0 and abs(got["frac"] - 0.5) < 1e-12
+
+
+def test_default_run_is_the_headline_workloads():
+    # no --workload: the CIFAR-100-shaped training step and the 2^22-sample
+    # hard pass of the CIFAR-10-shaped network, with the extras beside them
+    import bench
+    from paper_2602_07400_gb300 import synth
+    a = bench.parse_args([])
+    assert a.workload is None and a.gpus == 1
+    assert a.warmup >= 3
+    wl = synth.WORKLOADS[bench.HEADLINE_TRAIN]
+    assert (wl.batch, wl.widths, wl.k, wl.classes, wl.tau, wl.w_in) == (2048, (128000, 128000), 6, 100, 100.0, 46080)
+    wh = synth.WORKLOADS[bench.HEADLINE_HARD]
+    assert (wh.batch, wh.widths, wh.k, wh.classes, wh.w_in) == (1 << 22, (64000, 64000), 6, 10, 21504)
+    assert set(bench.EXTRAS) == {"mnist", "mnist_k2", "cifar10"}
+
+
+def test_roofline_object_picks_the_slower_bound():
+    import bench
+    from paper_2602_07400_gb300 import synth
+    wl = synth.WORKLOADS["mnist"]
+    work = bench.call_work(wl, 1024)
+    per_call = {"backward2": 0.1, "csr2": 0.04}
+    roof = bench.roofline_of("backward2", work, per_call, 152, {"sm_mhz": 1035.0}, "no-such-workload",
+                             6767.1, 2070.0, "measured")
+    assert roof["bound"] == "alu"
+    peak = 152 * 128 * 2070e6
+    assert abs(roof["achieved"] - 316 * 8000 * 1024 / 1e-4 / 1e12) < 1e-9
+    assert abs(roof["frac"] - 316 * 8000 * 1024 / 1e-4 / peak) < 1e-12
+    # at half the clock the same time is twice the fraction
+    assert abs(roof["frac_at_sampled_clock"] - 2 * roof["frac"]) < 1e-12
+    assert roof["traffic"] is None and roof["traffic_over_algorithmic"] is None
+    hroof = bench.roofline_of("csr2", work, per_call, 152, {}, "x", 6767.1, 2070.0, "measured")
+    assert hroof["bound"] == "hbm"
+    assert abs(hroof["achieved"] - work["csr2"][0] / 4e-5 / 1e9) < 1e-6
+    frac = bench.step_hbm_fraction(work, ["backward2", "csr2"], 0.2, 6767.1)
+    assert frac["moved_over_algorithmic"] > 1.0
