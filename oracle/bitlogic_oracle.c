@@ -327,54 +327,72 @@ void oracle_binarize_tables(const float* theta, int32_t w, int32_t k, uint64_t* 
 void oracle_pack_bits(const uint8_t* x, int64_t N, int32_t d,
                       const uint8_t* thr, int32_t b, uint32_t* xp) {
     const int64_t W = (N + 31) / 32;
-    memset(xp, 0, sizeof(uint32_t) * (size_t)d * (size_t)b * (size_t)W);
-    for (int64_t s = 0; s < N; ++s)
+    /* word q holds samples 32q .. 32q + 31: the words are independent outputs */
+#pragma omp parallel for schedule(static)
+    for (int64_t q = 0; q < W; ++q)
         for (int32_t j = 0; j < d; ++j)
-            for (int32_t i = 0; i < b; ++i)
-                if (x[s * d + j] > thr[i])
-                    xp[((int64_t)j * b + i) * W + s / 32] |= (uint32_t)1 << (s % 32);
+            for (int32_t i = 0; i < b; ++i) {
+                uint32_t word = 0;
+                for (int t = 0; t < 32 && 32 * q + t < N; ++t)   /* sample s = 32 q + t */
+                    if (x[(32 * q + t) * d + j] > thr[i]) word |= (uint32_t)1 << t;
+                xp[((int64_t)j * b + i) * W + q] = word;
+            }
 }
 
 /* Hard LUT layer on packed bits (App. C.1): for each sample, the node's
  * index a = sum_i bit(input M_j(i), s) << i selects table bit a.  Written
- * per sample as a plain lookup on unpacked bits. */
+ * per sample as a plain lookup on unpacked bits; the k input words that hold
+ * a sample's bits are read once for the 32 samples of the word. */
 void oracle_hard_forward(const uint32_t* xp, int32_t w_in, int64_t N,
                          const int32_t* conn, const uint64_t* table, int32_t w, int32_t k,
                          uint32_t* yp) {
     const int64_t W = (N + 31) / 32;
     (void)w_in;
-    memset(yp, 0, sizeof(uint32_t) * (size_t)w * (size_t)W);
 #pragma omp parallel for schedule(static)
     for (int32_t j = 0; j < w; ++j) {
-        for (int64_t s = 0; s < N; ++s) {
-            uint64_t a = 0;
-            for (int32_t i = 0; i < k; ++i) {
-                const uint32_t word = xp[(int64_t)conn[(int64_t)j * k + i] * W + s / 32];
-                a |= (uint64_t)((word >> (s % 32)) & 1u) << i;
+        const uint64_t T = table[j];
+        for (int64_t q = 0; q < W; ++q) {
+            uint32_t in[6];
+            for (int32_t i = 0; i < k; ++i) in[i] = xp[(int64_t)conn[(int64_t)j * k + i] * W + q];
+            uint32_t out = 0;
+            for (int t = 0; t < 32 && 32 * q + t < N; ++t) {   /* sample s = 32 q + t */
+                uint32_t a = 0;
+                for (int32_t i = 0; i < k; ++i) a |= ((in[i] >> t) & 1u) << i;
+                out |= (uint32_t)((T >> a) & 1u) << t;
             }
-            if ((table[j] >> a) & 1u) yp[(int64_t)j * W + s / 32] |= (uint32_t)1 << (s % 32);
+            yp[(int64_t)j * W + q] = out;
         }
     }
 }
 
 /* Popcount GroupSum head in hard mode (§3 "Encoders and heads"): the score
  * of class c is the number of ones among its contiguous group of g = w/C
- * nodes; the prediction is the first class with the largest score. */
+ * nodes; the prediction is the first class with the largest score.  The
+ * samples of one packed word are counted together (each word of a node is
+ * read once for its 32 samples; integer counts do not depend on the order
+ * of the additions). */
 void oracle_popcount_head(const uint32_t* yp, int32_t w, int64_t N, int32_t C,
                           int32_t* counts, int32_t* pred) {
     const int64_t W = (N + 31) / 32;
     const int32_t g = w / C;
 #pragma omp parallel for schedule(static)
-    for (int64_t s = 0; s < N; ++s) {
-        int32_t best = 0, bestc = 0;
+    for (int64_t q = 0; q < W; ++q) {
+        int32_t cnt[32];
+        int32_t best[32], bestc[32];
         for (int32_t c = 0; c < C; ++c) {
-            int32_t cnt = 0;
-            for (int32_t j = c * g; j < (c + 1) * g; ++j)
-                cnt += (int32_t)((yp[(int64_t)j * W + s / 32] >> (s % 32)) & 1u);
-            if (counts) counts[s * C + c] = cnt;
-            if (c == 0 || cnt > best) { best = cnt; bestc = c; }
+            for (int t = 0; t < 32; ++t) cnt[t] = 0;
+            for (int32_t j = c * g; j < (c + 1) * g; ++j) {
+                const uint32_t word = yp[(int64_t)j * W + q];
+                for (int t = 0; t < 32; ++t) cnt[t] += (int32_t)((word >> t) & 1u);
+            }
+            for (int64_t s = 32 * q; s < N && s < 32 * q + 32; ++s) {
+                const int t = (int)(s % 32);
+                if (counts) counts[s * C + c] = cnt[t];
+                if (c == 0 || cnt[t] > best[t]) { best[t] = cnt[t]; bestc[t] = c; }
+            }
         }
-        if (pred) pred[s] = bestc;
+        for (int64_t s = 32 * q; s < N && s < 32 * q + 32; ++s)
+            if (pred) pred[s] = bestc[s % 32];
     }
 }
 
