@@ -12,6 +12,9 @@
 // reduction runs in a fixed order.
 #include <cfloat>
 #include <mutex>
+#include <vector>
+
+#include <cuda.h>
 
 #include "common.cuh"
 
@@ -262,23 +265,68 @@ namespace {
 constexpr size_t kNoAllocScratchBytes = (size_t)8 << 20;   // 8 MiB
 static __device__ __align__(256) unsigned char g_head_scratch[kNoAllocScratchBytes];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_scratch_mutex;
-void* g_scratch_addr[kMaxDevices] = {};
+// The array is a global of the library's module, and a module is loaded once
+// per CUDA context, so its device address belongs to a context: a device
+// reset or a context other than the primary one loads the module again,
+// possibly at another address.  The address is therefore looked up once per
+// context (with the calling thread's context current) and cached under the
+// context's unique id.  The host-side name g_head_scratch is only a stand-in
+// and is never passed to a kernel.
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long*);
 
-// Device address of the scratch array on the current device.  The host-side
-// name g_head_scratch is only a stand-in, so the address is looked up once per
-// device (with that device current) and cached.
-int noalloc_scratch(void** out) {
-    int dev = -1;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return BITLOGIC_ERR_CUDA;
-    std::lock_guard<std::mutex> lock(g_scratch_mutex);
-    if (!g_scratch_addr[dev]) {
-        void* p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_head_scratch) != cudaSuccess || !p) return BITLOGIC_ERR_CUDA;
-        g_scratch_addr[dev] = p;
+struct ScratchAddr {
+    unsigned long long ctx_id;
+    void* addr;
+};
+
+std::mutex g_scratch_mutex;
+std::vector<ScratchAddr> g_scratch_addr;
+CtxGetCurrentFn g_ctx_get_current = nullptr;
+CtxGetIdFn g_ctx_get_id = nullptr;
+bool g_ctx_fns_looked_up = false;
+
+// Unique id of the calling thread's current context (0 if there is none, or
+// the driver entry points cannot be found: then nothing is cached).
+unsigned long long current_context_id() {
+    if (!g_ctx_fns_looked_up) {
+        g_ctx_fns_looked_up = true;
+        void* f1 = nullptr;
+        void* f2 = nullptr;
+        cudaDriverEntryPointQueryResult q1 = cudaDriverEntryPointSymbolNotFound, q2 = q1;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f1, 12000, cudaEnableDefault, &q1) ==
+                cudaSuccess && q1 == cudaDriverEntryPointSuccess &&
+            cudaGetDriverEntryPointByVersion("cuCtxGetId", &f2, 12000, cudaEnableDefault, &q2) ==
+                cudaSuccess && q2 == cudaDriverEntryPointSuccess) {
+            g_ctx_get_current = reinterpret_cast<CtxGetCurrentFn>(f1);
+            g_ctx_get_id = reinterpret_cast<CtxGetIdFn>(f2);
+        }
     }
-    *out = g_scratch_addr[dev];
+    if (!g_ctx_get_current || !g_ctx_get_id) return 0;
+    CUcontext ctx = nullptr;
+    unsigned long long id = 0;
+    if (g_ctx_get_current(&ctx) != CUDA_SUCCESS || !ctx) return 0;
+    if (g_ctx_get_id(ctx, &id) != CUDA_SUCCESS) return 0;
+    return id;
+}
+
+// Device address of the scratch array in the current context.
+int noalloc_scratch(void** out) {
+    std::lock_guard<std::mutex> lock(g_scratch_mutex);
+    unsigned long long id = current_context_id();
+    if (id) {
+        for (const ScratchAddr& e : g_scratch_addr)
+            if (e.ctx_id == id) {
+                *out = e.addr;
+                return BITLOGIC_OK;
+            }
+    }
+    // the lookup makes the device's primary context current if no context is
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_head_scratch) != cudaSuccess || !p) return BITLOGIC_ERR_CUDA;
+    if (!id) id = current_context_id();
+    if (id) g_scratch_addr.push_back({id, p});
+    *out = p;
     return BITLOGIC_OK;
 }
 

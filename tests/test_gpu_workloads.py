@@ -4,17 +4,16 @@ configuration the benchmark times (``pipeline.TrainStep`` / ``HardInfer``).
 * tiny (256 x 784, 1000 x 1000, k=6): every output element, including the
   input gradients of both layers.
 * mnist (1024 x 784, 8000 x 8000, k=6 and k=2): every output element.
-* cifar10 / cifar100 (64000- and 128000-wide layers): the forward, logits,
-  loss and head gradient over the full batch; table gradients of sampled
-  nodes of both layers and the layer-1 output gradient of sampled nodes, each
-  computed by the oracle on the sub-network that feeds them (every consumer
-  of a sampled node is included, so the sums are the full sums).
+* cifar10 / cifar100 (64000- and 128000-wide layers, B = 1024 / 2048): every
+  output element, the table gradients of both layers and layer 1's output
+  gradient included.
 * mnist_k4_routed16 (routed, 8000 x 8000, k = 4, 16 candidates): every
   output element, routing-logit gradients included.
-* hard_cifar10 and hard_mnist_w4000_4m (2^22 samples): every sample runs on
-  the GPU; sampled samples (first and last included) are recomputed by the
-  oracle from the raw samples, bit-exact for the packed input, both layers,
-  counts and argmax; hard_mnist_w4000 (batch 1024): every sample.
+* hard_cifar10 (2^22 samples): every sample recomputed by the oracle in
+  chunks, bit-exact for the packed input, every layer-1 output word, the
+  counts and the argmax.  hard_mnist_w4000_4m (2^22 samples): sampled
+  samples (first and last included) bit-exact, plus count/argmax properties
+  over all samples; hard_mnist_w4000 (batch 1024): every sample.
 """
 import os
 
@@ -23,6 +22,7 @@ import pytest
 import torch
 
 import oracle
+import paper_2602_07400_gb300 as bl
 from paper_2602_07400_gb300 import synth
 from paper_2602_07400_gb300.pipeline import HardInfer, Network, TrainStep, unpack_bits
 from parity_util import check_exact, check_fwd, check_grad
@@ -322,44 +322,21 @@ def test_routed_training_learns_and_snaps_to_a_deployable_network():
     check_exact(hi.pred.cpu().numpy(), ro["pred"], "pred of the snapped network")
 
 
-def _sampled_compare(wl, st, x, labels, params, n_nodes=96, seed=0):
-    conn1, th1, conn2, th2 = params
-    bits = oracle.encode_thermometer(x, wl.thresholds)
-    check_exact(st.bits.cpu().numpy().astype(np.float64), bits, "bits")
-    y1 = oracle.lut_forward(bits, conn1, th1)
-    check_fwd(st.y1, y1, "y1")
-    y2 = oracle.lut_forward(y1, conn2, th2)
-    check_fwd(st.y2, y2, "y2")
-    logits, loss, dy2 = oracle.head_loss(y2, labels, wl.classes, wl.tau)
-    check_fwd(st.logits, logits, "logits")
-    check_fwd(st.loss, np.array([loss]), "loss")
-    _check_grouped(st, dy2, wl)
-    rng = np.random.default_rng(seed)
-    w1, w2 = wl.widths
-    # layer-2 table gradients of sampled nodes
-    n2 = np.unique(np.concatenate([[0, w2 - 1], rng.integers(0, w2, n_nodes)]))
-    dth2, _ = oracle.lut_backward(y1, conn2[n2], th2[n2], dy2[n2], want_dx=False)
-    check_grad(st.dth2[torch.from_numpy(n2).cuda()], dth2, "dtheta2[sampled]")
-    # layer-1 output gradient of sampled layer-1 nodes: all their consumers
-    n1 = np.unique(np.concatenate([[0, w1 - 1], rng.integers(0, w1, n_nodes)]))
-    cons = np.unique(np.nonzero(np.isin(conn2, n1))[0])
-    _, dx_sub = oracle.lut_backward(y1, conn2[cons], th2[cons], dy2[cons], want_dx=True)
-    dy1_s = dx_sub[n1]
-    check_grad(st.dy1[torch.from_numpy(n1).cuda()], dy1_s, "dy1[sampled]")
-    dth1, _ = oracle.lut_backward(bits, conn1[n1], th1[n1], dy1_s, want_dx=False)
-    check_grad(st.dth1[torch.from_numpy(n1).cuda()], dth1, "dtheta1[sampled]")
-
-
 @pytest.mark.slow
-def test_cifar10_step_sampled():
+def test_cifar10_step_all_outputs():
+    # every element of every output and gradient of the CIFAR-10-shaped step
+    # (64000 x 64000, B = 1024), against the oracle's full step
     wl, st, x, labels, params = _step(synth.WORKLOADS["cifar10"], want_dx1=False)
-    _sampled_compare(wl, st, x, labels, params)
+    _full_compare(wl, st, x, labels, params, False)
 
 
 @pytest.mark.slow
-def test_cifar100_step_sampled():
+def test_cifar100_step_all_outputs():
+    # every element of every output and gradient of the CIFAR-100-shaped
+    # step (128000 x 128000, B = 2048, 100 classes): about a minute and a half
+    # of oracle time on 16 host cores
     wl, st, x, labels, params = _step(synth.WORKLOADS["cifar100"], want_dx1=False)
-    _sampled_compare(wl, st, x, labels, params, n_nodes=64)
+    _full_compare(wl, st, x, labels, params, False)
 
 
 def _hard_run(wl, N, seed=0, samples=1536):
@@ -401,10 +378,44 @@ def _hard_run(wl, N, seed=0, samples=1536):
     assert torch.equal(first.int(), hi.pred)
 
 
+def _hard_every_sample(wl, N, seed=0, chunk=1 << 16):
+    """The hard pass on N samples on the GPU, then every sample recomputed by
+    the oracle in chunks of `chunk` samples (a multiple of 32, so the chunks
+    are whole packed words): the packed input, every layer-1 output word, the
+    counts and the argmax of every sample, bit-exact."""
+    assert chunk % 32 == 0
+    conn1, th1, conn2, th2 = synth.network(wl, seed)
+    net = Network(conn1, th1, conn2, th2, wl.w_in)
+    hi = HardInfer(net, N, wl.d, wl.thresholds, wl.classes)
+    x, labels = synth.blob_batch(N, wl.d, wl.classes, wl.sigma, seed=seed + 11, device="cuda")
+    hi.x.copy_(x)
+    del x, labels
+    hi.binarize()
+    hi.run()
+    torch.cuda.synchronize()
+    assert bl.bitlogic_device_error() == 0
+    t1 = oracle.binarize_tables(th1)
+    t2 = oracle.binarize_tables(th2)
+    check_exact(hi.table1.cpu().numpy().view(np.uint64), t1, "table1")
+    check_exact(hi.table2.cpu().numpy().view(np.uint64), t2, "table2")
+    counts = hi.counts.cpu().numpy()
+    pred = hi.pred.cpu().numpy()
+    for s0 in range(0, N, chunk):
+        s1 = min(N, s0 + chunk)
+        w0, w1 = s0 // 32, (s1 + 31) // 32
+        r = oracle.hard_infer(hi.x[s0:s1].cpu().numpy(), wl.thresholds, conn1, t1, conn2, t2, wl.classes)
+        check_exact(hi.xp[:, w0:w1].cpu().numpy().view(np.uint32), r["xp"], f"xp words {w0}..{w1}")
+        check_exact(hi.yp1[:, w0:w1].cpu().numpy().view(np.uint32), r["yp1"], f"yp1 words {w0}..{w1}")
+        check_exact(counts[s0:s1], r["counts"], f"counts of samples {s0}..{s1}")
+        check_exact(pred[s0:s1], r["pred"], f"pred of samples {s0}..{s1}")
+
+
 @pytest.mark.slow
-def test_hard_cifar10_full_size_sampled():
+def test_hard_cifar10_every_sample():
+    # the 2^22-sample hard pass of the CIFAR-10-shaped network: every sample
+    # (packed input, layer-1 words, counts, argmax) against the oracle
     wl = synth.WORKLOADS["hard_cifar10"]
-    _hard_run(wl, wl.batch)
+    _hard_every_sample(wl, wl.batch)
 
 
 def test_hard_mnist_w4000_every_sample():
