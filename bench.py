@@ -87,6 +87,8 @@ def parse_args(argv=None):
     p.add_argument("--no-extras", action="store_true")
     p.add_argument("--node", default="soft", choices=["soft", "st"],
                    help="LightLUT node form of the training step: soft, or straight-through hard")
+    p.add_argument("--fuse-dy1", action="store_true",
+                   help="layer 1's backward sums layer 2's per-edge terms itself (no separate CSR reduction)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-graph", action="store_true",
@@ -397,15 +399,38 @@ def calls_table(work, per_call_ms, hbm):
     return out
 
 
-def step_hbm_fraction(work, names, ms_step, hbm):
-    """Algorithmic bytes of the step's calls over the step time, against the HBM peak."""
-    byts = sum(work[n][0] for n in names if n in work)
+def step_bytes(wl, B):
+    """Algorithmic bytes of one training step (thermometer encode, two LUT
+    forwards, head + cross-entropy, layer-2 backward with the input gradient,
+    layer-1 backward without it), each tensor moved once, whatever calls the
+    step is split into.  "survey": every node has its own output-gradient row
+    (the head writes dY as w x B and the layer-2 backward reads it);
+    "design": the head writes one gradient row per class (C x B), which every
+    node of the class reads."""
+    K, k = wl.K, wl.k
+    w1, w2 = wl.widths
+    win, d, C = wl.w_in, wl.d, wl.classes
+    f = 4
+    enc = B * d + f * win * B
+    fwd = f * (win * B + w1 * B + w1 * K + w1 * k) + f * (w1 * B + w2 * B + w2 * K + w2 * k)
+    csr2, csr1 = f * (w1 + 1 + w2 * k), f * (win + 1 + w1 * k)
+    bwd1 = f * (win * B + w1 * B + 2 * w1 * K) + csr1
+    survey = enc + fwd + f * (2 * w2 * B) + f * (w1 * B + w2 * B + w1 * B + 2 * w2 * K) + csr2 + bwd1
+    design = enc + fwd + f * (w2 * B + 2 * B * C + B) + f * (w1 * B + C * B + w1 * B + 2 * w2 * K) + csr2 + bwd1
+    return {"survey": survey, "design": design}
+
+
+def step_hbm_fraction(wl, B, work, names, ms_step, hbm):
+    """The step's algorithmic bytes over the step time, against the HBM
+    peak, with the bytes the calls actually move (per-edge terms included)."""
+    sb = step_bytes(wl, B)
     moved = sum(work[n][2] for n in names if n in work)
-    gbs = byts / (ms_step * 1e-3) / 1e9
-    return {"algorithmic_bytes": byts, "bytes_moved": moved, "alg_GB/s": gbs, "frac_hbm": gbs / hbm,
-            "moved_over_algorithmic": moved / byts}
-
-
+    t = ms_step * 1e-3
+    return {"algorithmic_bytes": sb["design"], "alg_GB/s": sb["design"] / t / 1e9,
+            "frac_hbm": sb["design"] / t / 1e9 / hbm,
+            "algorithmic_bytes_survey": sb["survey"], "frac_hbm_survey": sb["survey"] / t / 1e9 / hbm,
+            "bytes_moved": moved, "moved_over_algorithmic": moved / sb["design"],
+            "note": "design bytes: per-class output-gradient rows (C x B); survey bytes: one row per node (w x B)"}
 
 
 # --------------------------------------------------------------- ours --
@@ -481,7 +506,7 @@ class Timer:
         return {n: float(np.mean(v)) for n, v in calls.items()}, float(np.mean(totals))
 
 
-def build_train(wl, rank, node="soft"):
+def build_train(wl, rank, node="soft", fuse_dy1=False):
     from paper_2602_07400_gb300.pipeline import Network, RoutedNetwork, RoutedTrainStep, TrainStep
     B = wl.batch
     if wl.Kc:
@@ -491,7 +516,7 @@ def build_train(wl, rank, node="soft"):
     else:
         conn1, th1, conn2, th2 = synth.network(wl, seed=0)
         net = Network(conn1, th1, conn2, th2, wl.w_in)
-        st = TrainStep(net, B, wl.d, wl.thresholds, wl.classes, wl.tau, node=node)
+        st = TrainStep(net, B, wl.d, wl.thresholds, wl.classes, wl.tau, node=node, fuse_dy1=fuse_dy1)
     x, lab = synth.blob_batch(B, wl.d, wl.classes, wl.sigma, seed=1000 + rank)
     st.load(x.cuda(), lab.cuda())
     return net, st
@@ -527,7 +552,7 @@ def measure_train(wl, st, args, timer, hbm, sm_max, peak_kind, sms, world, detai
         "eager_ms_per_step": eager_step,
         "roofline": roofline_of(dom, work, per_call, sms, clocks, wl.name, hbm, sm_max, peak_kind),
         "calls": calls_table(work, per_call, hbm),
-        "step_hbm": step_hbm_fraction(work, per_call.keys(), tot / K, hbm),
+        "step_hbm": step_hbm_fraction(wl, B, work, per_call.keys(), tot / K, hbm) if not wl.Kc else None,
         "gpu_launches": K * st.kernels_per_run,
         "clocks": clocks, "wall_s_timed_loop": wall,
         "timing": ("CUDA-graph replays of the training step (fwd+bwd), CUDA events around each replay; "
@@ -719,7 +744,7 @@ def run_headline(args):
 
     # -- headline training workload
     wl = with_batch(synth.WORKLOADS[HEADLINE_TRAIN], args.batch)
-    net, st = build_train(wl, rank, args.node)
+    net, st = build_train(wl, rank, args.node, args.fuse_dy1)
     train = measure_train(wl, st, args, timer, hbm, sm_max, peak_kind, sms, world)
     upd = time_update(st, max(3, min(K, 20)))
     n_par = int(net.theta1.numel() + net.theta2.numel())
@@ -754,7 +779,7 @@ def run_headline(args):
     names = [] if (args.no_extras or args.profile) else [n for n in args.extras.split(",") if n]
     for name in names:
         we = synth.WORKLOADS[name]
-        enet, est = build_train(we, rank, args.node)
+        enet, est = build_train(we, rank, args.node, args.fuse_dy1)
         r = measure_train(we, est, args, timer, hbm, sm_max, peak_kind, sms, world, detail=False)
         r["config"] = {k_: v for k_, v in config_of(we, world, args.node).items()
                        if k_ in ("workload", "batch_per_gpu", "widths", "k", "classes", "tau")}
@@ -815,7 +840,7 @@ def run_single(args):
         net = Network(*synth.network(wl, seed=0), wl.w_in)
         hi = build_hard(wl, net, rank)
     else:
-        rnet, st = build_train(wl, rank, args.node)
+        rnet, st = build_train(wl, rank, args.node, args.fuse_dy1)
         net = rnet.snap() if wl.Kc else rnet   # the hard pass evaluates the discretized network
         train = measure_train(wl, st, args, timer, hbm, sm_max, peak_kind, sms, world)
         hi = build_hard(wl, net, rank, x_dev=st.x)

@@ -179,5 +179,28 @@ def test_roofline_object_picks_the_slower_bound():
     hroof = bench.roofline_of("csr2", work, per_call, 152, {}, "x", 6767.1, 2070.0, "measured")
     assert hroof["bound"] == "hbm"
     assert abs(hroof["achieved"] - work["csr2"][0] / 4e-5 / 1e9) < 1e-6
-    frac = bench.step_hbm_fraction(work, ["backward2", "csr2"], 0.2, 6767.1)
+    names = ["encode", "forward1", "forward2", "head", "backward2", "csr2", "backward1"]
+    frac = bench.step_hbm_fraction(wl, 1024, work, names, 0.2, 6767.1)
     assert frac["moved_over_algorithmic"] > 1.0
+    assert frac["frac_hbm_survey"] > frac["frac_hbm"]
+
+
+def test_step_bytes_follow_the_survey_formula():
+    # C3 (CIFAR-10-shaped, B = 1024): ~2.64 GB per step for the two layers
+    # and the head with one gradient row per node, plus the encoder (3.1 MB
+    # of pixels in, 88.1 MB of bits out); the per-class rows save the head's
+    # dY write and the layer-2 backward's dY read (2 x 262 MB) less the
+    # C x B rows
+    import bench
+    from paper_2602_07400_gb300 import synth
+    wl = synth.WORKLOADS["cifar10"]
+    sb = bench.step_bytes(wl, 1024)
+    enc = 1024 * 3072 + 4 * 21504 * 1024
+    assert abs((sb["survey"] - enc) / 1e9 - 2.64) < 0.005, sb
+    wB = 4 * 64000 * 1024
+    assert abs((sb["survey"] - sb["design"]) - (2 * wB - 4 * (3 * 1024 * 10 + 1024))) < 1
+    # the per-call algorithmic bytes of the unfused step add up to the
+    # design total
+    work = bench.call_work(wl, 1024)
+    names = ["encode", "forward1", "forward2", "head", "backward2", "csr2", "backward1"]
+    assert abs(sum(work[n][0] for n in names) / sb["design"] - 1) < 1e-3
