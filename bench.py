@@ -56,6 +56,7 @@ if ROOT not in sys.path:
 from paper_2602_07400_gb300 import synth  # noqa: E402
 
 METRIC = "LUT train samples/s (fwd+bwd) and hard bit-packed MSamples/s; % of roofline"
+FUSE = {"auto": None, "on": True, "off": False}
 HEADLINE_TRAIN = "cifar100"
 HEADLINE_HARD = "hard_cifar10"
 EXTRAS = ("mnist", "mnist_k2", "cifar10")
@@ -87,8 +88,12 @@ def parse_args(argv=None):
     p.add_argument("--no-extras", action="store_true")
     p.add_argument("--node", default="soft", choices=["soft", "st"],
                    help="LightLUT node form of the training step: soft, or straight-through hard")
-    p.add_argument("--fuse-dy1", action="store_true",
-                   help="layer 1's backward sums layer 2's per-edge terms itself (no separate CSR reduction)")
+    p.add_argument("--fuse-dy1", choices=["auto", "on", "off"], default="auto",
+                   help="layer 1's backward sums layer 2's per-edge terms itself (no separate CSR reduction); "
+                        "auto: when the terms are much larger than L2")
+    p.add_argument("--through", choices=["auto", "on", "off"], default="auto",
+                   help="layer 1 recomputes its output gradient through layer 2 (fan-in <= 3) instead of "
+                        "reading layer 2's per-edge terms; auto: whenever layer 2's fan-in allows it")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-graph", action="store_true",
@@ -252,7 +257,7 @@ def call_work_routed(wl, B):
     return {n: (b, o, b) for n, (b, o) in work.items()}
 
 
-def call_work(wl, B, fuse_dy1=False):
+def call_work(wl, B, fuse_dy1=False, through=False):
     """Algorithmic work of each library call of one step on a batch of B:
     (algorithmic bytes, algorithmic ops, bytes the call moves).
 
@@ -291,6 +296,17 @@ def call_work(wl, B, fuse_dy1=False):
         "hard1": (f * (win * W + w1 * W + w1 * k) + 8 * w1, (K - 1) * w1 * W, None),
         "hard2": (f * (w1 * W + w2 * k + B * C * 2 + B) + 8 * w2, (K - 1) * w2 * W, None),
     }
+    if through:
+        # layer 2: table gradient only; layer 1: its table gradient with its
+        # output gradient recomputed through layer 2 (the consumers' other
+        # inputs from Y1, the per-class rows, layer 2's tables, connectivity
+        # and CSR map), so the a4 row's input-gradient work for layer 2 moves
+        # to backward1 and nothing per edge is stored
+        work["backward2"] = (f * (w1 * B + C * B + 2 * w2 * K + w2 * k), (2 * (K - 1) + K) * w2 * B, None)
+        work["backward1"] = (f * (win * B + w1 * B + C * B + 2 * w1 * K + w1 * k + w2 * K + w2 * k) + csr2,
+                             (2 * (K - 1) + K) * w1 * B + 2 * (K - 1) * w2 * B, None)
+        del work["csr2"]
+        return {n: (b, o, b if m is None else m) for n, (b, o, m) in work.items()}
     if fuse_dy1:
         # layer 1 sums layer 2's per-edge terms through the CSR map itself
         work["backward1"] = (f * (win * B + w1 * B + 2 * w1 * K + w1 * k) + csr2, (2 * (K - 1) + K) * w1 * B,
@@ -309,6 +325,26 @@ TRAFFIC = {
         "bytes": 59.670016e6 + 147.641856e6, "source": "lut_soft.cu",
         "sha256": "180fc79502da4e837de466268e4dd9af96f7da65e286f6b8dce737f118e99f43",
         "note": "ncu capture of this workload"},
+    ("cifar10", "forward2"): {
+        "bytes": 1.163448e9 + 0.248158464e9, "source": "lut_soft.cu",
+        "sha256": "180fc79502da4e837de466268e4dd9af96f7da65e286f6b8dce737f118e99f43",
+        "note": "ncu capture of this workload"},
+    ("cifar10", "backward2"): {
+        "bytes": 1.344971e9 + 1.545406e9, "source": "lut_soft.cu",
+        "sha256": "180fc79502da4e837de466268e4dd9af96f7da65e286f6b8dce737f118e99f43",
+        "note": "ncu capture of this workload"},
+    ("cifar100", "forward1"): {
+        "bytes": 5106130432 + 1034886144, "source": "lut_soft.cu",
+        "sha256": "180fc79502da4e837de466268e4dd9af96f7da65e286f6b8dce737f118e99f43",
+        "note": "ncu capture of this workload (one-pass DRAM metrics)"},
+    ("cifar100", "forward2"): {
+        "bytes": 5877215232 + 1032726272, "source": "lut_soft.cu",
+        "sha256": "180fc79502da4e837de466268e4dd9af96f7da65e286f6b8dce737f118e99f43",
+        "note": "ncu capture of this workload (one-pass DRAM metrics)"},
+    ("cifar100", "backward2"): {
+        "bytes": 6069030400 + 6277533952, "source": "lut_soft.cu",
+        "sha256": "180fc79502da4e837de466268e4dd9af96f7da65e286f6b8dce737f118e99f43",
+        "note": "ncu capture of this workload (one-pass DRAM metrics)"},
     ("hard_cifar10", "hard1"): {
         "bytes": 16 * (1.209681e9 + 2.054784e9), "source": "hard.cu",
         "sha256": "f9bed6fc20215df71b5e12eebae1c94762286b3c7b941dea9a2ff948bfb9ed3c",
@@ -344,7 +380,7 @@ def kernel_traffic(workload: str, call: str):
 
 KERNEL_OF_CALL = {
     "encode": "encode_soft_kernel", "forward1": "lut_forward_staged_kernel<k>",
-    "forward2": "lut_forward_staged_kernel<k>", "head": "head_* (3 kernels)",
+    "forward2": "lut_forward_staged_kernel<k>", "head": "head_group_sum + head_softmax (2 kernels)",
     "backward2": "lut_backward_node_kernel<k, dx, dY rows>",
     "backward1": "lut_backward_theta_kernel<k>", "csr2": "csr_reduce_kernel",
     "binarize": "binarize_kernel (x2)", "pack": "pack_bits_kernel", "hard1": "hard_layer_staged_kernel<k>",
@@ -386,7 +422,7 @@ def roofline_of(call, work, per_call_ms, sms, clocks, workload, hbm, sm_max, pea
     return roof
 
 
-def calls_table(work, per_call_ms, hbm):
+def calls_table(work, per_call_ms, hbm, workload=None):
     out = {}
     for n, t in per_call_ms.items():
         b_, o_, m_ = work[n]
@@ -395,6 +431,12 @@ def calls_table(work, per_call_ms, hbm):
              "Tops/s": round(o_ / (t * 1e-3) / 1e12, 2) if o_ else None}
         if m_ != b_:
             e["moved_GB/s"] = round(m_ / (t * 1e-3) / 1e9, 1)
+        traffic, _ = kernel_traffic(workload, n) if workload else (None, None)
+        if traffic:
+            # DRAM bytes per launch from ncu against the algorithmic bytes,
+            # and the DRAM rate they imply at the event-timed duration
+            e["traffic_over_algorithmic"] = round(traffic / b_, 2)
+            e["dram_GB/s"] = round(traffic / (t * 1e-3) / 1e9, 1)
         out[n] = e
     return out
 
@@ -479,10 +521,14 @@ class Timer:
 
     def eager_split(self, step, n):
         """n eager steps with an event after every library call: mean ms per
-        call and per step."""
+        call and per step.  Each step is queued behind a short bounded sleep
+        kernel (about 1 ms), so the host has enqueued the whole step before
+        the GPU reaches it and the events time the kernels, not the host's
+        launch path."""
         marks = []
         for _ in range(n):
             self.flush.fill_(1)
+            torch.cuda._sleep(2_000_000)
             lst = []
             marks.append(lst)
 
@@ -506,7 +552,7 @@ class Timer:
         return {n: float(np.mean(v)) for n, v in calls.items()}, float(np.mean(totals))
 
 
-def build_train(wl, rank, node="soft", fuse_dy1=False):
+def build_train(wl, rank, node="soft", fuse_dy1=None, through=None):
     from paper_2602_07400_gb300.pipeline import Network, RoutedNetwork, RoutedTrainStep, TrainStep
     B = wl.batch
     if wl.Kc:
@@ -516,7 +562,8 @@ def build_train(wl, rank, node="soft", fuse_dy1=False):
     else:
         conn1, th1, conn2, th2 = synth.network(wl, seed=0)
         net = Network(conn1, th1, conn2, th2, wl.w_in)
-        st = TrainStep(net, B, wl.d, wl.thresholds, wl.classes, wl.tau, node=node, fuse_dy1=fuse_dy1)
+        st = TrainStep(net, B, wl.d, wl.thresholds, wl.classes, wl.tau, node=node, fuse_dy1=fuse_dy1,
+                       through=through)
     x, lab = synth.blob_batch(B, wl.d, wl.classes, wl.sigma, seed=1000 + rank)
     st.load(x.cuda(), lab.cuda())
     return net, st
@@ -544,20 +591,21 @@ def measure_train(wl, st, args, timer, hbm, sm_max, peak_kind, sms, world, detai
     assert bl.bitlogic_device_error() == 0
     tot = max_over_ranks([sum(ms)], "cuda")[0]
     per_call, eager_step = timer.eager_split(lambda mark: st.run(mark=mark), max(3, min(K, 30)))
-    work = call_work_routed(wl, B) if wl.Kc else call_work(wl, B, fuse_dy1=st.fuse_dy1)
+    work = call_work_routed(wl, B) if wl.Kc else call_work(wl, B, fuse_dy1=st.fuse_dy1,
+                                                              through=getattr(st, "through", False))
     single = {n: t for n, t in per_call.items() if n not in MULTI_KERNEL_CALLS}
     dom = max(single, key=single.get)
     res = {
         "value": job_rate(world, B, K, tot), "unit": "samples/s", "ms_per_step": tot / K,
         "eager_ms_per_step": eager_step,
         "roofline": roofline_of(dom, work, per_call, sms, clocks, wl.name, hbm, sm_max, peak_kind),
-        "calls": calls_table(work, per_call, hbm),
+        "calls": calls_table(work, per_call, hbm, wl.name),
         "step_hbm": step_hbm_fraction(wl, B, work, per_call.keys(), tot / K, hbm) if not wl.Kc else None,
         "gpu_launches": K * st.kernels_per_run,
         "clocks": clocks, "wall_s_timed_loop": wall,
         "timing": ("CUDA-graph replays of the training step (fwd+bwd), CUDA events around each replay; "
-                   "per-call split from eager steps with an event after every call" if use_graph else
-                   "eager launches, CUDA events around each step"),
+                   "per-call split from eager steps queued behind a 1 ms sleep, an event after every call"
+                   if use_graph else "eager launches, CUDA events around each step"),
     }
     if detail:
         res["roofline_by_call"] = {n: {k_: v for k_, v in roofline_of(n, work, per_call, sms, clocks, wl.name,
@@ -612,7 +660,7 @@ def measure_hard(wl, hi, args, timer, hbm, sm_max, peak_kind, sms, world):
         "value": job_rate(world, N, K, tot) / 1e6, "unit": "MSamples/s", "ms_per_batch": tot / K,
         "batch": N, "eager_ms_per_batch": eager_step,
         "includes": "binarize + encode/pack + 2 hard layers + popcount head + argmax",
-        "calls": calls_table(work, per_call_w, hbm),
+        "calls": calls_table(work, per_call_w, hbm, wl.name),
         "gpu_launches": K * (hi.kernels_per_binarize + hi.kernels_per_run),
         "clocks": clocks, "wall_s_timed_loop": wall,
     }
@@ -744,7 +792,7 @@ def run_headline(args):
 
     # -- headline training workload
     wl = with_batch(synth.WORKLOADS[HEADLINE_TRAIN], args.batch)
-    net, st = build_train(wl, rank, args.node, args.fuse_dy1)
+    net, st = build_train(wl, rank, args.node, FUSE[args.fuse_dy1], FUSE[args.through])
     train = measure_train(wl, st, args, timer, hbm, sm_max, peak_kind, sms, world)
     upd = time_update(st, max(3, min(K, 20)))
     n_par = int(net.theta1.numel() + net.theta2.numel())
@@ -767,7 +815,10 @@ def run_headline(args):
     hard = measure_hard(wh, hi, args, timer, hbm, sm_max, peak_kind, sms, world)
     if not args.profile:
         rates = measure_pipe_rates(sms)
-        hard["roofline"]["integer_pipes"] = integer_pipe_fraction(hard["roofline"], rates)
+        hard["roofline"] = hard_roofline(hard["roofline"], rates, sms, hard["clocks"])
+        r2 = hard_roofline(hard["roofline_hard2"], rates, sms, hard["clocks"])
+        hard["roofline_hard2"] = {k_: r2[k_] for k_ in ("bound", "achieved", "peak", "unit", "frac",
+                                                       "frac_issue_rate", "ms_per_launch")}
     if not (args.no_e2e or args.profile):
         hard["e2e"] = run_e2e_hard(hi, wh, K, world, rank, use_graph)
     hard["config"] = config_of(wh, world)
@@ -779,7 +830,7 @@ def run_headline(args):
     names = [] if (args.no_extras or args.profile) else [n for n in args.extras.split(",") if n]
     for name in names:
         we = synth.WORKLOADS[name]
-        enet, est = build_train(we, rank, args.node, args.fuse_dy1)
+        enet, est = build_train(we, rank, args.node, FUSE[args.fuse_dy1], FUSE[args.through])
         r = measure_train(we, est, args, timer, hbm, sm_max, peak_kind, sms, world, detail=False)
         r["config"] = {k_: v for k_, v in config_of(we, world, args.node).items()
                        if k_ in ("workload", "batch_per_gpu", "widths", "k", "classes", "tau")}
@@ -840,7 +891,7 @@ def run_single(args):
         net = Network(*synth.network(wl, seed=0), wl.w_in)
         hi = build_hard(wl, net, rank)
     else:
-        rnet, st = build_train(wl, rank, args.node, args.fuse_dy1)
+        rnet, st = build_train(wl, rank, args.node, FUSE[args.fuse_dy1], FUSE[args.through])
         net = rnet.snap() if wl.Kc else rnet   # the hard pass evaluates the discretized network
         train = measure_train(wl, st, args, timer, hbm, sm_max, peak_kind, sms, world)
         hi = build_hard(wl, net, rank, x_dev=st.x)
@@ -848,7 +899,10 @@ def run_single(args):
     rates = None
     if not args.profile:
         rates = measure_pipe_rates(sms)
-        hard["roofline"]["integer_pipes"] = integer_pipe_fraction(hard["roofline"], rates)
+        hard["roofline"] = hard_roofline(hard["roofline"], rates, sms, hard["clocks"])
+        r2 = hard_roofline(hard["roofline_hard2"], rates, sms, hard["clocks"])
+        hard["roofline_hard2"] = {k_: r2[k_] for k_ in ("bound", "achieved", "peak", "unit", "frac",
+                                                       "frac_issue_rate", "ms_per_launch")}
     e2e_train = e2e_hard = None
     if not (args.no_e2e or args.profile):
         if train is not None:
@@ -954,43 +1008,59 @@ def time_quantile_fit(wl, flush, iters: int = 20):
 
 
 def measure_pipe_rates(sms: int, iters: int = 2048, reps: int = 5) -> dict:
-    """Sustained issue rates of the pipes the kernels run on, from the
-    library's throughput probe (independent chains of one instruction kind
-    over 4 blocks of 256 threads per SM): LOP3 (logic pipe, the hard mux
-    tree's upper levels), IMAD (FMA pipe, its level 0) and FFMA (FMA pipe,
-    the soft kernels).  Median of `reps` launches, CUDA events."""
+    """Sustained issue rates of the instructions the kernels run, per SM and
+    clock, from the library's throughput probe (one block of 1024 threads
+    per SM, independent chains of one instruction kind, SM cycles read with
+    clock64): the LOP3 mux with three varying registers ("mux3", the hard
+    tree's upper levels), IMAD (its level 0), the two interleaved ("mix",
+    the tree's instruction mix), the LOP3 mux with an invariant operand
+    ("lop3") and FFMA (the soft kernels).  Median over blocks, then over
+    `reps` launches."""
     import paper_2602_07400_gb300 as bl
     n = bl.bitlogic_issue_probe_threads()
+    nb = bl.bitlogic_issue_probe_blocks()
     sink = torch.empty(n, dtype=torch.int32, device="cuda")
-    ops = n * iters * bl.bitlogic_issue_probe_ops_per_iter()
+    cyc = torch.empty(nb, dtype=torch.int64, device="cuda")
+    ops_per_block = (n // nb) * iters * bl.bitlogic_issue_probe_ops_per_iter()
     _, sm_max, _ = peaks()
-    out = {"sms": sms, "clock_mhz_assumed": sm_max,
-           "probe": "independent dependency chains, 4 x 256 threads per SM, median of 5 launches"}
-    for kind in ("lop3", "imad", "ffma"):
-        bl.bitlogic_issue_probe(kind, iters, sink)
-        evs = []
+    out = {"sms": sms, "probe": "independent dependency chains, one block of 1024 threads per SM, "
+                                "SM cycles from clock64; median over blocks and 5 launches"}
+    for kind in ("mux3", "imad", "mix", "lop3", "ffma"):
+        bl.bitlogic_issue_probe(kind, iters, sink, cyc)
+        per = []
         for _ in range(reps):
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            e0.record()
-            bl.bitlogic_issue_probe(kind, iters, sink)
-            e1.record()
-            evs.append((e0, e1))
-        torch.cuda.synchronize()
-        t = float(np.median([a.elapsed_time(b) for a, b in evs]))
-        rate = ops / (t * 1e-3)
-        out[kind] = {"T_lane_ops_s": round(rate / 1e12, 3),
-                     "lane_ops_per_sm_per_clk": round(rate / (sms * sm_max * 1e6), 1)}
+            bl.bitlogic_issue_probe(kind, iters, sink, cyc)
+            c = cyc.cpu().numpy().astype(np.float64)
+            per.append(float(np.median(ops_per_block / c)))
+        r = float(np.median(per))
+        out[kind] = {"lane_ops_per_sm_per_clk": round(r, 2),
+                     "T_lane_ops_s_at_max_clock": round(r * sms * sm_max * 1e6 / 1e12, 3)}
     return out
 
 
-def integer_pipe_fraction(roof: dict, rates: dict) -> dict:
-    """The hard layer's mux operations against the measured integer ceiling:
-    a mix of IMAD (FMA pipe) and LOP3 (logic pipe) can at best keep both
-    pipes busy, so the ceiling is the sum of their measured rates (below the
-    issue rate the main roofline uses)."""
-    peak = rates["imad"]["T_lane_ops_s"] + rates["lop3"]["T_lane_ops_s"]
-    return {"peak": round(peak, 3), "unit": "T lane-ops/s", "frac": roof["achieved"] / peak,
-            "source": "issue probe: IMAD + LOP3 (mux) rates measured in this run"}
+def hard_roofline(roof: dict, rates: dict, sms: int, clocks: dict) -> dict:
+    """The hard layer against the rate at which this GPU issues its
+    instruction mix.  The mux tree is integer work only (IMAD at level 0,
+    three-register LOP3 muxes above), and no integer instruction stream
+    issues at the FP32 lanes' rate: the measured rate of IMAD and the mux
+    interleaved one to one, per SM and clock, times the SMs and the median
+    SM clock sampled while the kernel ran, is the peak.  The fraction against
+    the issue rate of 128 lanes per SM and clock stays beside it."""
+    mhz = clocks.get("sm_mhz") or clocks.get("sm_max_mhz") or 2070.0
+    mix = rates["mix"]["lane_ops_per_sm_per_clk"]
+    out = dict(roof)
+    out["frac_issue_rate"] = roof["frac"]
+    out["peak_issue_rate"] = roof["peak"]
+    out["peak"] = mix * sms * mhz * 1e6 / 1e12
+    out["frac"] = roof["achieved"] / out["peak"]
+    out["achieved_per_sm_per_clk"] = roof["achieved"] * 1e12 / (sms * mhz * 1e6)
+    out["unit"] = "Tops/s (mux operations against the measured IMAD + LOP3 mux issue rate)"
+    out["peak_source"] = (f"issue probe in this run: IMAD and three-register LOP3 interleaved 1:1, "
+                          f"{mix:.1f} lane-ops per SM and clock x {sms} SMs x {mhz:.0f} MHz (median SM clock "
+                          f"sampled during the timed loop); issue-rate peak (128 lanes per SM and clock) in "
+                          f"peak_issue_rate")
+    out.pop("frac_at_sampled_clock", None)
+    return out
 
 
 def time_update(st, iters: int) -> float:

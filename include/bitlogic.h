@@ -225,6 +225,42 @@ int bitlogic_lut_backward_node(const float* X, int32_t w_in, int64_t B,
                                float* dtheta, float* edge_terms, const int32_t* edge_pos,
                                float* dY_out, cudaStream_t stream);
 
+/* Table gradient of a layer whose output gradient is recomputed through a
+ * next layer of small fan-in (chain rule on the node of §2, the
+ * multilinear form of the relaxed table): output row j of this layer is an
+ * input of the next layer, and its gradient
+ *   g[j][s] = sum over the CSR positions p in [up_off[j], up_off[j+1]) (in
+ *             increasing p) of up_dY[j2 / up_group][s] * d y_j2 / d x_slot (s),
+ *             edge up_edge[p] = j2 * up_k + slot,
+ * where the derivative of next-layer node j2 with respect to its input slot
+ * is a multilinear function of its other up_k - 1 inputs, read from Y.  So
+ * neither the next layer's per-edge terms nor g is stored (g goes to dY_out
+ * when that is given).  dtheta is then as in bitlogic_lut_backward_node
+ * with g as the output gradient (overwritten, not accumulated).  `node`
+ * applies to both layers (the next layer's table entries in the derivative;
+ * the slope of the sigmoid in this layer's dtheta).
+ *   X         device fp32 [w_in][B]: this layer's input
+ *   conn      device int32 [w][k];  theta device fp32 [w][2^k]
+ *   Y         device fp32 [w][B]: this layer's output (the next layer's input)
+ *   up_conn   device int32 [up_w][up_k], entries in [0, w); up_theta fp32 [up_w][2^up_k]
+ *   up_dY     device fp32 [up_w / up_group][B]: the next layer's output
+ *             gradient, one row per group of up_group nodes
+ *   up_off    device int32 [w + 1], up_edge device int32 [up_w * up_k] or
+ *             NULL (identity): the CSR map of up_conn (bitlogic_build_csr)
+ *   dtheta    device fp32 [w][2^k];  dY_out device fp32 [w][B] or NULL
+ * Needs 1 <= up_k <= 3 (BITLOGIC_ERR_FANIN otherwise), B % 4 == 0 and
+ * 16-byte aligned X, Y, up_dY and dY_out (BITLOGIC_ERR_ALIGN otherwise); B = 0
+ * zeroes dtheta.  Out-of-range CSR positions, edge ids or rows raise the
+ * device flag and contribute nothing.  Returns BITLOGIC_ERR_NULL,
+ * BITLOGIC_ERR_SHAPE (up_w % up_group != 0), BITLOGIC_ERR_NODE,
+ * BITLOGIC_ERR_CUDA. */
+int bitlogic_lut_backward_through(const float* X, int32_t w_in, int64_t B, const int32_t* conn,
+                                  const float* theta, int32_t w, int32_t k, int32_t node,
+                                  const float* Y, const int32_t* up_conn, const float* up_theta,
+                                  int32_t up_w, int32_t up_k, const float* up_dY, int32_t up_group,
+                                  const int32_t* up_off, const int32_t* up_edge, float* dtheta,
+                                  float* dY_out, cudaStream_t stream);
+
 /* Learnable routing (§3, the paragraph on connectivity: a per-slot
  * candidate pool whose selection is differentiable in training and snapped
  * to a sparse mapping at discretization; App. A "Initialization": pools
@@ -386,25 +422,35 @@ int bitlogic_csr_positions(const int32_t* edge_host, int32_t n_edges, int32_t* p
 int bitlogic_device_error(cudaStream_t stream);
 
 /* Issue-throughput probe (measurement support, not part of the method): the
- * roofline of the hard layer counts its mux operations against the issue
- * rate of the two pipes they run on, IMAD (FMA pipe) and LOP3 (logic pipe);
- * this launch measures what each sustains.  Every thread of a grid of
- * bitlogic_issue_probe_threads() threads (4 blocks of 256 per SM) runs
- * `iters` x bitlogic_issue_probe_ops_per_iter() instructions of one kind,
- * in independent dependency chains; the caller times the launch on `stream`
- * and divides.  sink: device, >= bitlogic_issue_probe_threads() uint32
- * (one per thread, written so the work is kept).  Returns
- * BITLOGIC_ERR_NULL, BITLOGIC_ERR_SHAPE (iters outside [0, 2^20], sink too
- * short, unknown kind) or BITLOGIC_ERR_CUDA. */
+ * roofline of the hard layer counts its mux operations against the rate at
+ * which this GPU issues the instructions the mux tree is made of; this launch
+ * measures those rates.  One block of 1024 threads per SM
+ * (bitlogic_issue_probe_blocks() blocks, bitlogic_issue_probe_threads()
+ * threads) runs `iters` x bitlogic_issue_probe_ops_per_iter() instructions
+ * of one kind per thread, in independent dependency chains.  Kinds: LOP3, a
+ * mux with one loop-invariant operand; IMAD; FFMA (FP32 reference); MUX3, a
+ * LOP3 mux of three varying registers (the tree's upper levels); MIX, IMAD
+ * and MUX3 interleaved one to one (the tree's mix).
+ *   sink:   device, >= bitlogic_issue_probe_threads() uint32 (one per
+ *           thread, written so the work is kept);
+ *   cycles: device, >= bitlogic_issue_probe_blocks() int64 or NULL: the SM
+ *           clock cycles each block ran (clock64), so that
+ *           threads per block x iters x ops per iter / cycles is the rate per
+ *           SM and clock.
+ * Returns BITLOGIC_ERR_NULL, BITLOGIC_ERR_SHAPE (iters outside [0, 2^20],
+ * sink too short, unknown kind) or BITLOGIC_ERR_CUDA. */
 typedef enum {
     BITLOGIC_PROBE_LOP3 = 0,
     BITLOGIC_PROBE_IMAD = 1,
-    BITLOGIC_PROBE_FFMA = 2
+    BITLOGIC_PROBE_FFMA = 2,
+    BITLOGIC_PROBE_MUX3 = 3,
+    BITLOGIC_PROBE_MIX = 4
 } bitlogic_probe_t;
+int64_t bitlogic_issue_probe_blocks(void);
 int64_t bitlogic_issue_probe_threads(void);
 int64_t bitlogic_issue_probe_ops_per_iter(void);
 int bitlogic_issue_probe(int32_t kind, int64_t iters, uint32_t seed, uint32_t* sink,
-                         int64_t sink_len, cudaStream_t stream);
+                         int64_t sink_len, int64_t* cycles, cudaStream_t stream);
 
 /* Static text for a status code. */
 const char* bitlogic_status_string(int code);

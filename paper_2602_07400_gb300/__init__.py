@@ -27,14 +27,14 @@ __all__ = [
     "BitLogicError", "load", "bitlogic_encode_thermometer", "bitlogic_lut_forward",
     "bitlogic_lut_backward_workspace", "bitlogic_lut_backward", "bitlogic_lut_backward_edges",
     "bitlogic_csr_reduce", "bitlogic_lut_backward_ex", "bitlogic_head_loss_ex",
-    "bitlogic_head_loss_workspace", "bitlogic_head_loss_noalloc",
+    "bitlogic_head_loss_workspace", "bitlogic_head_loss_noalloc", "bitlogic_lut_backward_through",
     "bitlogic_head_loss", "bitlogic_binarize_tables", "bitlogic_pack_bits",
     "bitlogic_hard_forward", "bitlogic_build_csr", "bitlogic_csr_positions", "bitlogic_device_error",
     "bitlogic_adamw_update", "bitlogic_route_forward", "bitlogic_route_backward", "bitlogic_route_snap",
     "bitlogic_route_forward_u8", "bitlogic_route_backward_u8", "bitlogic_encode_thermometer_u8",
     "bitlogic_pixel_histogram", "bitlogic_quantile_thresholds", "bitlogic_lut_forward_node", "bitlogic_lut_backward_node", "NODE_FORMS",
     "bitlogic_status_string", "bitlogic_version", "LIB_PATH",
-    "bitlogic_issue_probe", "bitlogic_issue_probe_threads", "bitlogic_issue_probe_ops_per_iter", "PROBE_KINDS",
+    "bitlogic_issue_probe", "bitlogic_issue_probe_blocks", "bitlogic_issue_probe_threads", "bitlogic_issue_probe_ops_per_iter", "PROBE_KINDS",
 ]
 
 LIB_PATH = _build.LIB
@@ -44,7 +44,7 @@ LIB_PATH = _build.LIB
 NODE_FORMS = {"soft": 0, "st": 1}
 
 # instruction kinds of the issue-throughput probe (bitlogic_probe_t)
-PROBE_KINDS = {"lop3": 0, "imad": 1, "ffma": 2}
+PROBE_KINDS = {"lop3": 0, "imad": 1, "ffma": 2, "mux3": 3, "mix": 4}
 
 
 def _node_code(node) -> int:
@@ -86,6 +86,8 @@ _SIGS = {
                                   _P, _P, _P, _P, _P], ctypes.c_int),
     "bitlogic_lut_backward_node": ([_P, _I32, _I64, _P, _P, _I32, _I32, _I32, _P, _I32, _P, _P, _P, _I32,
                                     _P, _P, _P, _P, _P], ctypes.c_int),
+    "bitlogic_lut_backward_through": ([_P, _I32, _I64, _P, _P, _I32, _I32, _I32, _P, _P, _P, _I32, _I32, _P, _I32,
+                                       _P, _P, _P, _P, _P], ctypes.c_int),
     "bitlogic_head_loss_ex": ([_P, _I32, _I64, _I32, _F32, _P, _P, _P, _P, _P, _P, _SZ, _P],
                               ctypes.c_int),
     "bitlogic_head_loss_workspace": ([_I64, _I32], _SZ),
@@ -102,9 +104,10 @@ _SIGS = {
     "bitlogic_device_error": ([_P], ctypes.c_int),
     "bitlogic_status_string": ([ctypes.c_int], ctypes.c_char_p),
     "bitlogic_version": ([], ctypes.c_int),
+    "bitlogic_issue_probe_blocks": ([], _I64),
     "bitlogic_issue_probe_threads": ([], _I64),
     "bitlogic_issue_probe_ops_per_iter": ([], _I64),
-    "bitlogic_issue_probe": ([_I32, _I64, ctypes.c_uint32, _P, _I64, _P], ctypes.c_int),
+    "bitlogic_issue_probe": ([_I32, _I64, ctypes.c_uint32, _P, _I64, _P, _P], ctypes.c_int),
 }
 
 
@@ -168,6 +171,10 @@ def bitlogic_version() -> int:
     return load().bitlogic_version()
 
 
+def bitlogic_issue_probe_blocks() -> int:
+    return int(load().bitlogic_issue_probe_blocks())
+
+
 def bitlogic_issue_probe_threads() -> int:
     return int(load().bitlogic_issue_probe_threads())
 
@@ -176,10 +183,13 @@ def bitlogic_issue_probe_ops_per_iter() -> int:
     return int(load().bitlogic_issue_probe_ops_per_iter())
 
 
-def bitlogic_issue_probe(kind, iters: int, sink: torch.Tensor, seed: int = 1, stream=None):
+def bitlogic_issue_probe(kind, iters: int, sink: torch.Tensor, cycles: Optional[torch.Tensor] = None,
+                         seed: int = 1, stream=None):
     """One launch of the issue-throughput probe: bitlogic_issue_probe_threads()
     threads x iters x bitlogic_issue_probe_ops_per_iter() instructions of
-    `kind` ("lop3", "imad" or "ffma"); time it with events on `stream`."""
+    `kind` ("lop3", "imad", "ffma", "mux3" or "mix"); `cycles` (int64 CUDA
+    tensor of bitlogic_issue_probe_blocks() entries, optional) receives the
+    SM clock cycles of each block."""
     if isinstance(kind, str):
         if kind not in PROBE_KINDS:
             raise ValueError(f"kind must be one of {sorted(PROBE_KINDS)}")
@@ -187,8 +197,10 @@ def bitlogic_issue_probe(kind, iters: int, sink: torch.Tensor, seed: int = 1, st
     if not isinstance(sink, torch.Tensor) or sink.dtype != torch.int32 or not sink.is_cuda \
             or not sink.is_contiguous():
         raise ValueError("sink must be a contiguous int32 CUDA tensor")
+    if cycles is not None:
+        _need(cycles, "cycles", torch.int64, (bitlogic_issue_probe_blocks(),))
     _check("bitlogic_issue_probe", load().bitlogic_issue_probe(
-        int(kind), int(iters), int(seed) & 0xffffffff, _ptr(sink), sink.numel(), _stream(stream)))
+        int(kind), int(iters), int(seed) & 0xffffffff, _ptr(sink), sink.numel(), _ptr(cycles), _stream(stream)))
 
 
 def bitlogic_encode_thermometer(x: torch.Tensor, thresholds, bits: torch.Tensor, stream=None):
@@ -450,6 +462,38 @@ def _backward_general(fn, node, X, conn, theta, dtheta, dY, dy_group, up_terms, 
     head = (_ptr(X), w_in, B, _ptr(conn), _ptr(theta), w, k)
     args = head + rest if node is None else head + (node,) + rest
     _check(fn, getattr(load(), fn)(*args))
+
+
+def bitlogic_lut_backward_through(X: torch.Tensor, conn: torch.Tensor, theta: torch.Tensor, dtheta: torch.Tensor,
+                                  Y: torch.Tensor, up_conn: torch.Tensor, up_theta: torch.Tensor,
+                                  up_dY: torch.Tensor, up_group: int, up_off: torch.Tensor,
+                                  up_edge: Optional[torch.Tensor] = None, node="soft",
+                                  dY_out: Optional[torch.Tensor] = None, stream=None):
+    """Table gradient of a layer from the next layer's output gradient,
+    recomputing this layer's output gradient through the next layer (fan-in
+    1..3) instead of reading stored per-edge terms."""
+    w_in, B = X.shape
+    w, k = conn.shape
+    up_w, up_k = up_conn.shape
+    _need(X, "X", torch.float32, (w_in, B))
+    _need(conn, "conn", torch.int32, (w, k))
+    _need(theta, "theta", torch.float32, (w, 1 << k))
+    _need(dtheta, "dtheta", torch.float32, (w, 1 << k))
+    _need(Y, "Y", torch.float32, (w, B))
+    _need(up_conn, "up_conn", torch.int32, (up_w, up_k))
+    _need(up_theta, "up_theta", torch.float32, (up_w, 1 << up_k))
+    if up_group < 1 or up_w % up_group != 0:
+        raise ValueError("up_group must divide the next layer's width")
+    _need(up_dY, "up_dY", torch.float32, (up_w // up_group, B))
+    _need(up_off, "up_off", torch.int32, (w + 1,))
+    if up_edge is not None:
+        _need(up_edge, "up_edge", torch.int32, (up_w * up_k,))
+    if dY_out is not None:
+        _need(dY_out, "dY_out", torch.float32, (w, B))
+    _check("bitlogic_lut_backward_through", load().bitlogic_lut_backward_through(
+        _ptr(X), w_in, B, _ptr(conn), _ptr(theta), w, k, _node_code(node), _ptr(Y), _ptr(up_conn),
+        _ptr(up_theta), up_w, up_k, _ptr(up_dY), int(up_group), _ptr(up_off), _ptr(up_edge), _ptr(dtheta),
+        _ptr(dY_out), _stream(stream)))
 
 
 def bitlogic_head_loss_ex(Y: torch.Tensor, labels: torch.Tensor, C: int, tau: float,

@@ -30,6 +30,7 @@ extern "C" int bitlogic_internal_index_error_encode(cudaStream_t);
 extern "C" int bitlogic_internal_index_error_hard(cudaStream_t);
 extern "C" int bitlogic_internal_index_error_optim(cudaStream_t);
 extern "C" int bitlogic_internal_index_error_route(cudaStream_t);
+extern "C" int bitlogic_internal_index_error_lut_through(cudaStream_t);
 
 extern "C" const char* bitlogic_status_string(int code) {
     switch (code) {
@@ -85,12 +86,13 @@ extern "C" int bitlogic_csr_positions(const int32_t* edge_host, int32_t n_edges,
 
 extern "C" int bitlogic_device_error(cudaStream_t stream) {
     int worst = BITLOGIC_OK;
-    const int r[6] = {bitlogic_internal_index_error_lut_soft(stream),
+    const int r[7] = {bitlogic_internal_index_error_lut_soft(stream),
                       bitlogic_internal_index_error_head(stream),
                       bitlogic_internal_index_error_encode(stream),
                       bitlogic_internal_index_error_hard(stream),
                       bitlogic_internal_index_error_optim(stream),
-                      bitlogic_internal_index_error_route(stream)};
+                      bitlogic_internal_index_error_route(stream),
+                      bitlogic_internal_index_error_lut_through(stream)};
     for (int v : r) {
         if (v == BITLOGIC_ERR_CUDA) return v;
         if (v != BITLOGIC_OK) worst = v;

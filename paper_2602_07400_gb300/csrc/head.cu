@@ -6,10 +6,11 @@
 //   loss         = mean_s (logsumexp(logits[s]) - logits[s][label_s])
 //   dY[j][s]     = ((softmax(logits[s])[c(j)] - [c(j) == label_s]) / B) / tau
 //
-// Four short kernels: group sums (lanes over samples, warps over the rows of
-// a group), per-sample softmax (one warp per sample), the broadcast of
-// dlogit/tau over each group's rows, and a single-block batch mean.  Every
-// reduction runs in a fixed order.
+// Two short kernels (three when the per-node dY is requested): group sums
+// (lanes over samples, warps over the rows of a group), per-sample softmax
+// (one warp per sample) whose last block to finish also takes the batch mean,
+// and the broadcast of dlogit/tau over each group's rows.  Every reduction
+// runs in a fixed order.
 #include <cfloat>
 #include <mutex>
 #include <vector>
@@ -25,9 +26,10 @@ constexpr int kSumWarps = 8;
 
 __global__ void __launch_bounds__(kSumWarps * 32)
 head_group_sum_kernel(const float* __restrict__ Y, long long B, int C, int g, float tau,
-                      float* __restrict__ logits) {
+                      float* __restrict__ logits, unsigned int* __restrict__ done) {
     __shared__ float part[kSumWarps][32];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) *done = 0u;   // the softmax's block count
     const int c = blockIdx.x;
     const long long s = (long long)blockIdx.y * 32 + lane;
     float acc = 0.f;
@@ -59,9 +61,10 @@ constexpr int kMaxRowSplits = 4;
 __global__ void __launch_bounds__(kSumVecWarps * 32)
 head_group_sum_vec_kernel(const float* __restrict__ Y, long long B, int C, int g, float tau,
                           float* __restrict__ logits, float* __restrict__ split_sums, int splits,
-                          int rows_per_split) {
+                          int rows_per_split, unsigned int* __restrict__ done) {
     __shared__ __align__(16) float part[kSumVecWarps][128];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) *done = 0u;   // the softmax's block count
     const int c = blockIdx.x / splits, rs = blockIdx.x - c * splits;
     const int r0 = rs * rows_per_split, r1 = min(g, r0 + rows_per_split);
     const long long s4 = (long long)blockIdx.y * 128 + 4 * lane;
@@ -105,42 +108,77 @@ __device__ __forceinline__ float warp_sum(float v) {
 
 constexpr int kSoftWarps = 8;
 
+// One warp per sample.  The block adds its samples' losses in warp order and
+// publishes the sum in block_sums; the last block to finish (a device-wide
+// count in `done`, zeroed by the group-sum kernel that runs before) adds the
+// blocks' sums in index order and writes the batch mean: one pass, no
+// separate reduction launch, and a fixed summation order.
 __global__ void __launch_bounds__(kSoftWarps * 32)
 head_softmax_kernel(float* __restrict__ logits, long long B, int C,
                     const int* __restrict__ labels, float* __restrict__ dlogit,
-                    float* __restrict__ per_sample, float tau, float* __restrict__ dYg,
-                    const float* __restrict__ split_sums, int splits) {
+                    float* __restrict__ block_sums, unsigned int* __restrict__ done, float* __restrict__ loss,
+                    float tau, float* __restrict__ dYg, const float* __restrict__ split_sums, int splits) {
+    __shared__ float part[kSoftWarps];
+    __shared__ bool last;
+    __shared__ float red[kSoftWarps * 32];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const long long s = (long long)blockIdx.x * kSoftWarps + warp;
-    if (s >= B) return;
-    if (split_sums) {   // logits from the row splits' sums, added in split order
-        for (int c = lane; c < C; c += 32) {
-            float t = 0.f;
-            for (int rs = 0; rs < splits; ++rs) t += __ldg(split_sums + ((long long)rs * B + s) * C + c);
-            logits[s * C + c] = t / tau;
+    float li = 0.f;
+    if (s < B) {
+        if (split_sums) {   // logits from the row splits' sums, added in split order
+            for (int c = lane; c < C; c += 32) {
+                float t = 0.f;
+                for (int rs = 0; rs < splits; ++rs) t += __ldg(split_sums + ((long long)rs * B + s) * C + c);
+                logits[s * C + c] = t / tau;
+            }
+            __syncwarp();
         }
-        __syncwarp();
+        const float* l = logits + s * C;
+        float m = -FLT_MAX;
+        for (int c = lane; c < C; c += 32) m = fmaxf(m, l[c]);
+        m = warp_max(m);
+        float z = 0.f;
+        for (int c = lane; c < C; c += 32) z += expf(l[c] - m);
+        z = warp_sum(z);
+        const float lse = m + logf(z);
+        int lab = __ldg(labels + s);
+        if (lab < 0 || lab >= C) {
+            if (lane == 0) flag_index_error();
+            lab = 0;
+        }
+        li = lse - l[lab];
+        const float invB = 1.0f / (float)B;
+        for (int c = lane; c < C; c += 32) {
+            const float p = expf(l[c] - lse);
+            const float dl = (p - (c == lab ? 1.0f : 0.0f)) * invB;
+            dlogit[s * C + c] = dl;
+            if (dYg) dYg[(long long)c * B + s] = dl / tau;   // the gradient of every node of class c
+        }
     }
-    const float* l = logits + s * C;
-    float m = -FLT_MAX;
-    for (int c = lane; c < C; c += 32) m = fmaxf(m, l[c]);
-    m = warp_max(m);
-    float z = 0.f;
-    for (int c = lane; c < C; c += 32) z += expf(l[c] - m);
-    z = warp_sum(z);
-    const float lse = m + logf(z);
-    int lab = __ldg(labels + s);
-    if (lab < 0 || lab >= C) {
-        if (lane == 0) flag_index_error();
-        lab = 0;
+    if (lane == 0) part[warp] = li;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        float t = 0.f;
+#pragma unroll
+        for (int q = 0; q < kSoftWarps; ++q) t += part[q];
+        block_sums[blockIdx.x] = t;
+        __threadfence();   // the sum is visible before the count says so
+        last = atomicAdd(done, 1u) == gridDim.x - 1;
     }
-    if (lane == 0) per_sample[s] = lse - l[lab];
-    const float invB = 1.0f / (float)B;
-    for (int c = lane; c < C; c += 32) {
-        const float p = expf(l[c] - lse);
-        const float dl = (p - (c == lab ? 1.0f : 0.0f)) * invB;
-        dlogit[s * C + c] = dl;
-        if (dYg) dYg[(long long)c * B + s] = dl / tau;   // the gradient of every node of class c
+    __syncthreads();
+    if (!last) return;
+    // last block: the batch mean from every block's sum (read past L1)
+    float acc = 0.f;
+    for (unsigned i = threadIdx.x; i < gridDim.x; i += kSoftWarps * 32) acc += __ldcg(block_sums + i);
+    red[threadIdx.x] = acc;
+    __syncthreads();
+    for (int o = kSoftWarps * 16; o > 0; o >>= 1) {
+        if (threadIdx.x < o) red[threadIdx.x] += red[threadIdx.x + o];
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) {
+        loss[0] = red[0] / (float)B;
+        *done = 0u;
     }
 }
 
@@ -169,22 +207,6 @@ head_dy_kernel(const float* __restrict__ dlogit, long long B, int C, int g, int 
     }
 }
 
-// loss = (sum_s per_sample[s]) / B in one block: strided per-thread sums in
-// index order, then a fixed shared-memory tree.
-__global__ void __launch_bounds__(256)
-head_mean_kernel(const float* __restrict__ per_sample, long long B, float* __restrict__ loss) {
-    __shared__ float red[256];
-    float acc = 0.f;
-    for (long long s = threadIdx.x; s < B; s += 256) acc += per_sample[s];
-    red[threadIdx.x] = acc;
-    __syncthreads();
-    for (int o = 128; o > 0; o >>= 1) {
-        if (threadIdx.x < o) red[threadIdx.x] += red[threadIdx.x + o];
-        __syncthreads();
-    }
-    if (threadIdx.x == 0) loss[0] = red[0] / (float)B;
-}
-
 size_t align_up(size_t v) { return (v + 255) & ~(size_t)255; }
 
 }  // namespace
@@ -197,9 +219,11 @@ BITLOGIC_ERROR_READER(head)
 extern "C" size_t bitlogic_head_loss_workspace(int64_t B, int32_t C) {
     if (B <= 0 || C <= 0) return 0;
     const size_t bc = (size_t)B * (size_t)C * sizeof(float);
-    // dlogit [B][C], per-sample loss [B], logits [B][C] (used when the
-    // caller passes no logits buffer), the row splits' sums [splits][B][C]
-    return align_up(bc) + align_up((size_t)B * sizeof(float)) + align_up(bc) + align_up(kMaxRowSplits * bc);
+    // dlogit [B][C], the softmax blocks' loss sums [<= B], logits [B][C]
+    // (used when the caller passes no logits buffer), the row splits' sums
+    // [splits][B][C], the softmax's block count
+    return align_up(bc) + align_up((size_t)B * sizeof(float)) + align_up(bc) + align_up(kMaxRowSplits * bc) +
+           align_up(sizeof(unsigned int));
 }
 
 extern "C" int bitlogic_head_loss_ex(const float* Y, int32_t w, int64_t B, int32_t C, float tau,
@@ -218,31 +242,34 @@ extern "C" int bitlogic_head_loss_ex(const float* Y, int32_t w, int64_t B, int32
     char* ws = static_cast<char*>(workspace);
     const size_t bc = (size_t)B * (size_t)C * sizeof(float);
     float* dlogit = reinterpret_cast<float*>(ws);
-    float* per = reinterpret_cast<float*>(ws + align_up(bc));
+    float* block_sums = reinterpret_cast<float*>(ws + align_up(bc));
     float* lg = logits ? logits : reinterpret_cast<float*>(ws + align_up(bc) + align_up((size_t)B * 4));
     float* split_sums = reinterpret_cast<float*>(ws + align_up(bc) + align_up((size_t)B * 4) + align_up(bc));
+    unsigned int* done = reinterpret_cast<unsigned int*>(ws + align_up(bc) + align_up((size_t)B * 4) + align_up(bc) +
+                                                         align_up(kMaxRowSplits * bc));
     int splits = 1;
 
     if (B % 4 == 0 && aligned16(Y)) {
         // split the rows of a class until about two blocks per SM pull from
-        // HBM, keeping at least 16 rows per warp
+        // HBM, keeping at least 4 rows per warp
         const long long nsb = (B + 127) / 128;
         const int sms = sm_count();
         while (splits < kMaxRowSplits && (long long)C * splits * nsb < 2ll * sms &&
-               g / (2 * splits) >= 16 * kSumVecWarps)
+               g / (2 * splits) >= 4 * kSumVecWarps)
             splits *= 2;
         const int rows_per_split = (g + splits - 1) / splits;
         if ((long long)C * splits > 0x7fffffffll || nsb > 65535) return BITLOGIC_ERR_SHAPE;
         head_group_sum_vec_kernel<<<dim3((unsigned)(C * splits), (unsigned)nsb), kSumVecWarps * 32, 0, stream>>>(
-            Y, B, C, g, tau, lg, split_sums, splits, rows_per_split);
+            Y, B, C, g, tau, lg, split_sums, splits, rows_per_split, done);
     } else
-        head_group_sum_kernel<<<dim3((unsigned)C, (unsigned)sb), kSumWarps * 32, 0, stream>>>(Y, B, C, g, tau, lg);
+        head_group_sum_kernel<<<dim3((unsigned)C, (unsigned)sb), kSumWarps * 32, 0, stream>>>(Y, B, C, g, tau, lg,
+                                                                                          done);
     head_softmax_kernel<<<(unsigned)((B + kSoftWarps - 1) / kSoftWarps), kSoftWarps * 32, 0, stream>>>(
-        lg, B, C, labels, dlogit, per, tau, dY_grouped, splits > 1 ? split_sums : nullptr, splits);
+        lg, B, C, labels, dlogit, block_sums, done, loss, tau, dY_grouped, splits > 1 ? split_sums : nullptr,
+        splits);
     if (dY)
         head_dy_kernel<<<dim3((unsigned)((w + kDyRows - 1) / kDyRows), (unsigned)gy), kDyThreads, 0, stream>>>(
             dlogit, B, C, g, w, tau, dY);
-    head_mean_kernel<<<1, 256, 0, stream>>>(per, B, loss);
     return launch_status();
 }
 

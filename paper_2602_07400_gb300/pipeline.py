@@ -20,7 +20,8 @@ import torch
 from . import (NODE_FORMS, bitlogic_adamw_update, bitlogic_binarize_tables, bitlogic_build_csr,
                bitlogic_csr_positions, bitlogic_csr_reduce, bitlogic_pixel_histogram, bitlogic_quantile_thresholds,
                bitlogic_encode_thermometer, bitlogic_hard_forward, bitlogic_head_loss_ex,
-               bitlogic_head_loss_workspace, bitlogic_lut_backward_node, bitlogic_lut_forward_node,
+               bitlogic_head_loss_workspace, bitlogic_lut_backward_node, bitlogic_lut_backward_through,
+               bitlogic_lut_forward_node,
                bitlogic_pack_bits, bitlogic_route_backward, bitlogic_route_backward_u8, bitlogic_route_forward,
                bitlogic_route_forward_u8, bitlogic_route_snap, bitlogic_encode_thermometer_u8)
 
@@ -147,19 +148,38 @@ class Network:
         self.pos2 = torch.from_numpy(bitlogic_csr_positions(edge2)).to(dev)
 
 
+# Per-edge input-gradient terms larger than this are summed by the layer-1
+# backward itself instead of a separate CSR reduction (measured faster on
+# GB300 for the CIFAR-shaped layers, 1.6 and 6.3 GB of terms, and slower for
+# the MNIST-shaped one, 0.2 GB).
+FUSE_DY1_TERM_BYTES = 512 << 20
+
+
 class TrainStep:
     """One soft training step.  The backward is fused across the call
     boundaries the ABI offers: the head emits one gradient row per class
-    (``dyg``) that the layer-2 backward reads for every node of the class, and
-    the layer-1 backward reduces layer 2's per-edge input-gradient terms on
-    the fly through the CSR map, so neither dY2 nor dY1 is stored (set
-    ``keep_dy1`` to also write dY1, e.g. to check it).  ``node`` picks the
+    (``dyg``) that the layer-2 backward reads for every node of the class.
+    Layer 1's output gradient (the input gradient of layer 2) takes one of
+    three routes:
+
+    * ``through`` (default when layer 2's fan-in is at most 3): the layer-1
+      backward recomputes it from layer 2's connectivity, tables and output
+      gradient rows (bitlogic_lut_backward_through), so layer 2 needs only
+      its table gradient and nothing per edge is stored;
+    * ``fuse_dy1`` (default when layer 2's per-edge terms exceed
+      FUSE_DY1_TERM_BYTES): layer 2 stores its per-edge terms and the layer-1
+      backward sums them through the CSR map on the fly;
+    * otherwise a CSR reduction of the terms into ``dy1``, which the
+      dtheta-only layer-1 backward reads.
+
+    Set ``keep_dy1`` to also write dY1 (e.g. to check it).  ``node`` picks the
     LightLUT form of both layers: "soft", or "st" (hard table samples in the
     forward, straight-through gradient to the logits)."""
 
     def __init__(self, net: Network, B: int, d: int, thresholds: Sequence[int], C: int,
                  tau: float, want_dx1: bool = False, keep_dy1: bool = False,
-                 fuse_dy1: bool = False, csr_order: bool = True, node: str = "soft", device="cuda"):
+                 fuse_dy1: Optional[bool] = None, csr_order: bool = True, node: str = "soft",
+                 through: Optional[bool] = None, device="cuda"):
         dev = torch.device(device)
         if node not in NODE_FORMS:
             raise ValueError(f"node must be one of {sorted(NODE_FORMS)}")
@@ -168,6 +188,13 @@ class TrainStep:
         self.thr = [int(t) for t in thresholds]
         assert d * len(self.thr) == net.w_in
         assert net.w2 % C == 0
+        if through is None:
+            through = net.k2 <= 3 and B % 4 == 0 and not want_dx1
+        if through and (net.k2 > 3 or B % 4 != 0 or want_dx1):
+            raise ValueError("the through route needs layer-2 fan-in <= 3, B % 4 == 0 and no layer-1 input gradient")
+        self.through = bool(through)
+        if fuse_dy1 is None:
+            fuse_dy1 = 4 * net.w2 * net.k2 * B > FUSE_DY1_TERM_BYTES
         f32 = dict(dtype=torch.float32, device=dev)
         self.x = torch.zeros(B, d, dtype=torch.uint8, device=dev)
         self.labels = torch.zeros(B, dtype=torch.int32, device=dev)
@@ -177,20 +204,17 @@ class TrainStep:
         self.logits = torch.empty(B, C, **f32)
         self.loss = torch.zeros(1, **f32)
         self.dyg = torch.empty(C, B, **f32)          # gradient row shared by each class's nodes
-        # layer 1's output gradient: summed from layer 2's terms inside the
-        # layer-1 backward (fuse_dy1), or by a CSR reduction into dy1 that the
-        # dtheta-only kernel then reads
-        self.fuse_dy1 = bool(fuse_dy1)
+        self.fuse_dy1 = bool(fuse_dy1) and not self.through
         # per-edge terms stored in CSR order (each input's terms contiguous,
         # read without the edge map) instead of edge order
         self.csr_order = bool(csr_order)
-        self.dy1 = torch.empty(net.w1, B, **f32) if (keep_dy1 or not fuse_dy1) else None
+        self.dy1 = torch.empty(net.w1, B, **f32) if (keep_dy1 or not (self.fuse_dy1 or self.through)) else None
         self.dth1 = torch.empty_like(net.theta1)
         self.dth2 = torch.empty_like(net.theta2)
         self.dbits = torch.empty(net.w_in, B, **f32) if want_dx1 else None
         # per-edge input-gradient terms of layer 2 (and of layer 1 when its
         # input gradient is wanted)
-        self.edges2 = torch.empty(net.w2 * net.k2, B, **f32)
+        self.edges2 = None if self.through else torch.empty(net.w2 * net.k2, B, **f32)
         self.edges1 = torch.empty(net.w1 * net.k1, B, **f32) if want_dx1 else None
         self.ws_head = torch.empty(bitlogic_head_loss_workspace(B, C), dtype=torch.uint8, device=dev)
 
@@ -214,8 +238,19 @@ class TrainStep:
         n = self.net
         co = self.csr_order
         nd = self.node
+        g = n.w2 // self.C
+        if self.through:
+            # layer 2: table gradient only; layer 1: its output gradient
+            # recomputed through layer 2 inside its table-gradient kernel
+            bitlogic_lut_backward_node(self.y1, n.conn2, n.theta2, self.dth2, nd, dY=self.dyg, dy_group=g,
+                                       stream=stream)
+            mark("backward2")
+            bitlogic_lut_backward_through(self.bits, n.conn1, n.theta1, self.dth1, self.y1, n.conn2, n.theta2,
+                                          self.dyg, g, n.off2, n.edge2, node=nd, dY_out=self.dy1, stream=stream)
+            mark("backward1")
+            return
         bitlogic_lut_backward_node(self.y1, n.conn2, n.theta2, self.dth2, nd, dY=self.dyg,
-                                   dy_group=n.w2 // self.C, edge_terms=self.edges2,
+                                   dy_group=g, edge_terms=self.edges2,
                                    edge_pos=n.pos2 if co else None, stream=stream)
         mark("backward2")
         pos1 = n.pos1 if (co and self.edges1 is not None) else None
@@ -264,12 +299,12 @@ class TrainStep:
                               weight_decay, stream)
         mark("update")
 
-    # kernels one run() launches: encode 1, forwards 2, head 3, backwards 2
-    # (+ the CSR reduction of layer 2's terms unless fused, + the layer-1 CSR
-    # reduction when the input gradient is wanted)
+    # kernels one run() launches: encode 1, forwards 2, head 2, backwards 2
+    # (+ the CSR reduction of layer 2's terms unless fused or recomputed, +
+    # the layer-1 CSR reduction when the input gradient is wanted)
     @property
     def kernels_per_run(self) -> int:
-        return 8 + (0 if self.fuse_dy1 else 1) + (1 if self.dbits is not None else 0)
+        return 7 + (0 if (self.fuse_dy1 or self.through) else 1) + (1 if self.dbits is not None else 0)
 
 
 class RoutedNetwork:
@@ -400,9 +435,9 @@ class RoutedTrainStep:
             bitlogic_adamw_update(p, m, v, g, self.opt_step, lr, betas, eps, weight_decay, stream)
         mark("update")
 
-    # encode 1, routing forwards 2, LUT forwards 2, head 3, LUT backwards 2,
+    # encode 1, routing forwards 2, LUT forwards 2, head 2, LUT backwards 2,
     # routing dr 2, routing dX 1
-    kernels_per_run = 13
+    kernels_per_run = 12
     fuse_dy1 = False
 
 

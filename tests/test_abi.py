@@ -117,11 +117,20 @@ def test_host_validation_returns_before_any_launch():
     # issue probe: NULL sink, short sink, negative iterations, unknown kind
     n = lib.bitlogic_issue_probe_threads()
     assert n > 0 and lib.bitlogic_issue_probe_ops_per_iter() > 0
-    assert lib.bitlogic_issue_probe(0, 1, 1, None, n, None) == -1
-    assert lib.bitlogic_issue_probe(0, 1, 1, fake, n - 1, None) == -2
-    assert lib.bitlogic_issue_probe(0, -1, 1, fake, n, None) == -2
-    assert lib.bitlogic_issue_probe(0, (1 << 20) + 1, 1, fake, n, None) == -2
-    assert lib.bitlogic_issue_probe(7, 1, 1, fake, n, None) == -2
+    assert lib.bitlogic_issue_probe_blocks() > 0 and n == 1024 * lib.bitlogic_issue_probe_blocks()
+    assert lib.bitlogic_issue_probe(0, 1, 1, None, n, None, None) == -1
+    assert lib.bitlogic_issue_probe(0, 1, 1, fake, n - 1, None, None) == -2
+    assert lib.bitlogic_issue_probe(0, -1, 1, fake, n, None, None) == -2
+    assert lib.bitlogic_issue_probe(0, (1 << 20) + 1, 1, fake, n, None, None) == -2
+    assert lib.bitlogic_issue_probe(7, 1, 1, fake, n, None, None) == -2
+    # through backward: next-layer fan-in above 3, B not a multiple of 4,
+    # group not dividing the next layer, missing inputs
+    th = lib.bitlogic_lut_backward_through
+    assert th(fake, 8, 8, fake, fake, 8, 2, 0, fake, fake, fake, 8, 4, fake, 1, fake, None, fake, None, None) == -3
+    assert th(fake, 8, 6, fake, fake, 8, 2, 0, fake, fake, fake, 8, 2, fake, 1, fake, None, fake, None, None) == -4
+    assert th(fake, 8, 8, fake, fake, 8, 2, 0, fake, fake, fake, 8, 2, fake, 3, fake, None, fake, None, None) == -2
+    assert th(fake, 8, 8, fake, fake, 8, 2, 0, fake, None, fake, 8, 2, fake, 1, fake, None, fake, None, None) == -1
+    assert th(fake, 8, 8, fake, fake, 8, 2, 5, fake, fake, fake, 8, 2, fake, 1, fake, None, fake, None, None) == -12
     # head: w % C != 0, tau <= 0
     assert lib.bitlogic_head_loss(fake, 10, 8, 3, 1.0, fake, None, fake, None, fake, 1 << 20, None) == -2
     assert lib.bitlogic_head_loss(fake, 9, 8, 3, 0.0, fake, None, fake, None, fake, 1 << 20, None) == -2

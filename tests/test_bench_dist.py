@@ -138,12 +138,18 @@ def test_algorithmic_work_of_the_roofline_calls():
     assert hwork["hard1"][0] == 4 * (21504 * W + 64000 * W + 64000 * 6) + 8 * 64000
 
 
-def test_integer_pipe_ceiling_is_the_sum_of_both_pipes():
+def test_hard_roofline_uses_the_measured_mix_rate():
+    # the hard layer's peak is the measured issue rate of its instruction mix
+    # (per SM and clock) at the sampled clock; the issue-rate fraction stays
     import bench
-    roof = {"achieved": 10.0}
-    rates = {"imad": {"T_lane_ops_s": 12.0}, "lop3": {"T_lane_ops_s": 8.0}}
-    got = bench.integer_pipe_fraction(roof, rates)
-    assert got["peak"] == 20.0 and abs(got["frac"] - 0.5) < 1e-12
+    roof = {"achieved": 10.0, "peak": 40.0, "frac": 0.25, "frac_at_sampled_clock": 0.3}
+    rates = {"mix": {"lane_ops_per_sm_per_clk": 80.0}}
+    got = bench.hard_roofline(roof, rates, 100, {"sm_mhz": 2000.0})
+    assert abs(got["peak"] - 80.0 * 100 * 2000e6 / 1e12) < 1e-12
+    assert abs(got["frac"] - 10.0 / 16.0) < 1e-12
+    assert got["frac_issue_rate"] == 0.25 and got["peak_issue_rate"] == 40.0
+    assert abs(got["achieved_per_sm_per_clk"] - 50.0) < 1e-9
+    assert "frac_at_sampled_clock" not in got
 
 
 def test_default_run_is_the_headline_workloads():

@@ -416,6 +416,98 @@ def test_backward_is_deterministic_and_handles_skewed_consumers():
     check_grad(outs[0][1], wdx, "dX")
 
 
+THROUGH = [  # (k, ku, w_in, w, up_w, up_group, B)
+    (2, 2, 50, 64, 80, 8, 128), (6, 2, 300, 200, 150, 1, 260), (3, 3, 40, 96, 120, 12, 4),
+    (2, 1, 30, 40, 60, 6, 1028), (4, 3, 100, 256, 512, 64, 132), (1, 2, 9, 12, 20, 20, 8),
+]
+
+
+def _through_oracle(X, conn, theta, Y, up_conn, up_theta, up_dY, up_group, node):
+    # the next layer's per-node output gradient rows, its input gradient by
+    # the oracle's scatter-add, then this layer's table gradient
+    dY2 = np.repeat(np.asarray(up_dY, np.float64), up_group, axis=0)
+    _, g = oracle.lut_backward(Y, up_conn, up_theta, dY2, want_dx=True, node=node)
+    dth, _ = oracle.lut_backward(X, conn, theta, g, want_dx=False, node=node)
+    return dth, g
+
+
+@pytest.mark.parametrize("node", ["soft", "st"])
+@pytest.mark.parametrize("k,ku,w_in,w,up_w,up_group,B", THROUGH)
+def test_lut_backward_through(k, ku, w_in, w, up_w, up_group, B, node):
+    # this layer's table gradient with its output gradient recomputed through
+    # the next layer, against the oracle's two-layer chain rule
+    X = synth.uniform_activations(w_in, B, seed=k + 10)
+    conn = synth.connectivity(w, k, w_in, seed=k + 11)
+    theta = synth.table_logits(w, 1 << k, seed=k + 12)
+    Y = synth.uniform_activations(w, B, seed=k + 13)
+    up_conn = synth.connectivity(up_w, ku, w, seed=ku + 14)
+    up_theta = synth.table_logits(up_w, 1 << ku, seed=ku + 15)
+    up_dY = synth.uniform_gradients(up_w // up_group, B, seed=16, scale=1e-3)
+    off, edge = bl.bitlogic_build_csr(up_conn, w)
+    dth = torch.full((w, 1 << k), np.nan, device="cuda")
+    g = torch.full((w, B), np.nan, device="cuda")
+    bl.bitlogic_lut_backward_through(dev(X), dev(conn), dev(theta), dth, dev(Y), dev(up_conn), dev(up_theta),
+                                     dev(up_dY), up_group, dev(off), dev(edge), node=node, dY_out=g)
+    wdth, wg = _through_oracle(X, conn, theta, Y, up_conn, up_theta, up_dY, up_group, node)
+    check_grad(g, wg, "dY (recomputed)")
+    check_grad(dth, wdth, "dtheta")
+    # without the optional output: the same table gradient bit for bit
+    dth2 = torch.empty_like(dth)
+    bl.bitlogic_lut_backward_through(dev(X), dev(conn), dev(theta), dth2, dev(Y), dev(up_conn), dev(up_theta),
+                                     dev(up_dY), up_group, dev(off), dev(edge), node=node)
+    check_exact(dth2.cpu().numpy(), dth.cpu().numpy(), "dtheta without dY_out")
+    no_device_error()
+
+
+def test_lut_backward_through_many_and_no_consumers():
+    # inputs with more than 32 consumers (the consumer list is taken in
+    # chunks of 32) and inputs nobody reads (zero output gradient)
+    k, ku, w_in, w, up_w, B = 2, 2, 20, 40, 300, 64
+    rng = np.random.default_rng(3)
+    up_conn = np.stack([rng.choice([0, 1, 2, 3, 5], size=2, replace=False) for _ in range(up_w)]).astype(np.int32)
+    X = synth.uniform_activations(w_in, B, seed=1)
+    conn = synth.connectivity(w, k, w_in, seed=2)
+    theta = synth.table_logits(w, 4, seed=3)
+    Y = synth.uniform_activations(w, B, seed=4)
+    up_theta = synth.table_logits(up_w, 4, seed=5)
+    up_dY = synth.uniform_gradients(up_w, B, seed=6)
+    off, edge = bl.bitlogic_build_csr(up_conn, w)
+    assert np.diff(off).max() > 64
+    dth = torch.empty(w, 4, device="cuda")
+    g = torch.full((w, B), np.nan, device="cuda")
+    bl.bitlogic_lut_backward_through(dev(X), dev(conn), dev(theta), dth, dev(Y), dev(up_conn), dev(up_theta),
+                                     dev(up_dY), 1, dev(off), dev(edge), dY_out=g)
+    wdth, wg = _through_oracle(X, conn, theta, Y, up_conn, up_theta, up_dY, 1, "soft")
+    check_grad(g, wg, "dY (recomputed)")
+    check_grad(dth, wdth, "dtheta")
+    unused = np.setdiff1d(np.arange(w), up_conn.reshape(-1))
+    assert unused.size > 0
+    assert torch.all(g[torch.from_numpy(unused).cuda()] == 0)
+    no_device_error()
+
+
+def test_lut_backward_through_identity_edge_map():
+    # up_edge = NULL: the next layer's edges already in CSR order (node j2
+    # reads inputs 2 j2 and 2 j2 + 1, so edge e feeds input e)
+    k, ku, w_in, w, B = 3, 2, 30, 64, 256
+    up_w = w // 2
+    up_conn = np.arange(w, dtype=np.int32).reshape(up_w, 2)
+    X = synth.uniform_activations(w_in, B, seed=1)
+    conn = synth.connectivity(w, k, w_in, seed=2)
+    theta = synth.table_logits(w, 8, seed=3)
+    Y = synth.uniform_activations(w, B, seed=4)
+    up_theta = synth.table_logits(up_w, 4, seed=5)
+    up_dY = synth.uniform_gradients(up_w, B, seed=6)
+    off, edge = bl.bitlogic_build_csr(up_conn, w)
+    assert np.array_equal(edge, np.arange(w))
+    dth = torch.empty(w, 8, device="cuda")
+    bl.bitlogic_lut_backward_through(dev(X), dev(conn), dev(theta), dth, dev(Y), dev(up_conn), dev(up_theta),
+                                     dev(up_dY), 1, dev(off), None)
+    wdth, _ = _through_oracle(X, conn, theta, Y, up_conn, up_theta, up_dY, 1, "soft")
+    check_grad(dth, wdth, "dtheta")
+    no_device_error()
+
+
 def test_backward_unused_inputs_get_zero():
     k, w_in, w, B = 3, 50, 4, 40     # at most 12 of 50 inputs are read
     X = synth.uniform_activations(w_in, B, seed=5)
@@ -650,14 +742,23 @@ def test_binding_rejects_wrong_tensors():
 
 def test_issue_probe_runs_every_kind():
     # the throughput probe behind the pipe rates the benchmark reports: every
-    # thread writes the combination of its chains
+    # thread writes the combination of its chains, every block (one per SM)
+    # its clock cycles, which grow with the iteration count
     n = bl.bitlogic_issue_probe_threads()
+    nb = bl.bitlogic_issue_probe_blocks()
+    assert n == 1024 * nb
     sink = torch.zeros(n, dtype=torch.int32, device="cuda")
-    for kind in ("lop3", "imad", "ffma"):
+    cyc = torch.zeros(nb, dtype=torch.int64, device="cuda")
+    for kind in ("lop3", "imad", "ffma", "mux3", "mix"):
         sink.zero_()
-        bl.bitlogic_issue_probe(kind, 4, sink, seed=12345)
+        bl.bitlogic_issue_probe(kind, 4, sink, cyc, seed=12345)
         torch.cuda.synchronize()
         assert int((sink != 0).sum()) > n // 2, kind
+        short = cyc.clone()
+        bl.bitlogic_issue_probe(kind, 64, sink, cyc, seed=12345)
+        torch.cuda.synchronize()
+        assert bool((short > 0).all()) and bool((cyc > short).all()), kind
+    bl.bitlogic_issue_probe("mix", 4, sink)   # cycles are optional
     with pytest.raises(ValueError):
         bl.bitlogic_issue_probe("lop4", 1, sink)
     with pytest.raises(bl.BitLogicError):

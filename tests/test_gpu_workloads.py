@@ -32,14 +32,14 @@ pytestmark = pytest.mark.gpu
 oracle.set_threads(os.cpu_count() or 1)
 
 
-def _step(wl, want_dx1, seed=0, k=None, keep_dy1=True, fuse_dy1=False, csr_order=True, node="soft"):
+def _step(wl, want_dx1, seed=0, k=None, keep_dy1=True, fuse_dy1=None, csr_order=True, node="soft", through=None):
     if k is not None:
         wl = synth.Workload(wl.name, wl.batch, wl.d, wl.classes, wl.sigma, wl.thresholds, wl.widths, k, wl.tau)
     conn1, th1, conn2, th2 = synth.network(wl, seed)
     x, labels = synth.blob_batch(wl.batch, wl.d, wl.classes, wl.sigma, seed=seed + 7)
     net = Network(conn1, th1, conn2, th2, wl.w_in)
     st = TrainStep(net, wl.batch, wl.d, wl.thresholds, wl.classes, wl.tau, want_dx1=want_dx1,
-                   keep_dy1=keep_dy1, fuse_dy1=fuse_dy1, csr_order=csr_order, node=node)
+                   keep_dy1=keep_dy1, fuse_dy1=fuse_dy1, csr_order=csr_order, node=node, through=through)
     st.load(x.cuda(), labels.cuda())
     st.run()
     torch.cuda.synchronize()
@@ -109,6 +109,21 @@ def test_st_forward_is_the_deployed_network(k):
     check_fwd(st.logits, counts / wl.tau, "logits vs popcounts / tau")
 
 
+@pytest.mark.parametrize("node", ["soft", "st"])
+def test_mnist_k2_step_without_the_through_route(node):
+    # k = 2 takes the through route by default (layer 1 recomputes its
+    # output gradient through layer 2); the per-edge-term route still holds
+    wl, st, x, labels, params = _step(synth.WORKLOADS["mnist"], want_dx1=False, k=2, node=node, through=False)
+    assert not st.through
+    _full_compare(wl, st, x, labels, params, False, node=node)
+
+
+def test_mnist_k2_step_st_through():
+    wl, st, x, labels, params = _step(synth.WORKLOADS["mnist"], want_dx1=False, k=2, node="st")
+    assert st.through
+    _full_compare(wl, st, x, labels, params, False, node="st")
+
+
 def test_mnist_step_fused_layer1_gradient():
     # layer 1's output gradient summed inside its backward from layer 2's
     # CSR-ordered terms, instead of a CSR reduction followed by the
@@ -128,11 +143,12 @@ def test_tiny_step_edge_ordered_terms():
     _full_compare(wl, st, x, labels, params, True)
 
 
-def test_mnist_bench_configuration_matches():
+@pytest.mark.parametrize("k", [6, 2])
+def test_mnist_bench_configuration_matches(k):
     # the benchmark runs without storing dY1; its outputs equal the checked
     # configuration's bit for bit
-    _, a, *_ = _step(synth.WORKLOADS["mnist"], want_dx1=False, keep_dy1=True)
-    _, b, *_ = _step(synth.WORKLOADS["mnist"], want_dx1=False, keep_dy1=False)
+    _, a, *_ = _step(synth.WORKLOADS["mnist"], want_dx1=False, keep_dy1=True, k=k)
+    _, b, *_ = _step(synth.WORKLOADS["mnist"], want_dx1=False, keep_dy1=False, k=k)
     for name in ("y2", "logits", "loss", "dyg", "dth2", "dth1"):
         check_exact(getattr(b, name).cpu().numpy(), getattr(a, name).cpu().numpy(), name)
 
