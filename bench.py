@@ -94,6 +94,8 @@ def parse_args(argv=None):
     p.add_argument("--through", choices=["auto", "on", "off"], default="auto",
                    help="layer 1 recomputes its output gradient through layer 2 (fan-in <= 3) instead of "
                         "reading layer 2's per-edge terms; auto: whenever layer 2's fan-in allows it")
+    p.add_argument("--bytes1", choices=["auto", "on", "off"], default="auto",
+                   help="layer-1 backward gathers the encoder's wires as bytes (fused and through routes)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-graph", action="store_true",
@@ -257,7 +259,7 @@ def call_work_routed(wl, B):
     return {n: (b, o, b) for n, (b, o) in work.items()}
 
 
-def call_work(wl, B, fuse_dy1=False, through=False):
+def call_work(wl, B, fuse_dy1=False, through=False, bytes1=False):
     """Algorithmic work of each library call of one step on a batch of B:
     (algorithmic bytes, algorithmic ops, bytes the call moves).
 
@@ -296,6 +298,11 @@ def call_work(wl, B, fuse_dy1=False, through=False):
         "hard1": (f * (win * W + w1 * W + w1 * k) + 8 * w1, (K - 1) * w1 * W, None),
         "hard2": (f * (w1 * W + w2 * k + B * C * 2 + B) + 8 * w2, (K - 1) * w2 * W, None),
     }
+    xb1 = 1 if bytes1 else f   # bytes per layer-1 input value read by the layer-1 backward
+    if bytes1:
+        # the encoder also writes the wires as bytes, which the layer-1
+        # backward gathers instead of the fp32 rows
+        work["encode"] = (B * d + f * win * B + win * B, 0, B * d + f * win * B + win * B)
     if through:
         # layer 2: table gradient only; layer 1: its table gradient with its
         # output gradient recomputed through layer 2 (the consumers' other
@@ -303,14 +310,14 @@ def call_work(wl, B, fuse_dy1=False, through=False):
         # and CSR map), so the a4 row's input-gradient work for layer 2 moves
         # to backward1 and nothing per edge is stored
         work["backward2"] = (f * (w1 * B + C * B + 2 * w2 * K + w2 * k), (2 * (K - 1) + K) * w2 * B, None)
-        work["backward1"] = (f * (win * B + w1 * B + C * B + 2 * w1 * K + w1 * k + w2 * K + w2 * k) + csr2,
+        work["backward1"] = (xb1 * win * B + f * (w1 * B + C * B + 2 * w1 * K + w1 * k + w2 * K + w2 * k) + csr2,
                              (2 * (K - 1) + K) * w1 * B + 2 * (K - 1) * w2 * B, None)
         del work["csr2"]
         return {n: (b, o, b if m is None else m) for n, (b, o, m) in work.items()}
     if fuse_dy1:
         # layer 1 sums layer 2's per-edge terms through the CSR map itself
-        work["backward1"] = (f * (win * B + w1 * B + 2 * w1 * K + w1 * k) + csr2, (2 * (K - 1) + K) * w1 * B,
-                             f * (win * B + 2 * w1 * K + w1 * k) + csr2 + terms)
+        work["backward1"] = (xb1 * win * B + f * (w1 * B + 2 * w1 * K + w1 * k) + csr2, (2 * (K - 1) + K) * w1 * B,
+                             xb1 * win * B + f * (2 * w1 * K + w1 * k) + csr2 + terms)
         del work["csr2"]
     return {n: (b, o, b if m is None else m) for n, (b, o, m) in work.items()}
 
@@ -552,7 +559,7 @@ class Timer:
         return {n: float(np.mean(v)) for n, v in calls.items()}, float(np.mean(totals))
 
 
-def build_train(wl, rank, node="soft", fuse_dy1=None, through=None):
+def build_train(wl, rank, node="soft", fuse_dy1=None, through=None, bytes1=None):
     from paper_2602_07400_gb300.pipeline import Network, RoutedNetwork, RoutedTrainStep, TrainStep
     B = wl.batch
     if wl.Kc:
@@ -563,7 +570,7 @@ def build_train(wl, rank, node="soft", fuse_dy1=None, through=None):
         conn1, th1, conn2, th2 = synth.network(wl, seed=0)
         net = Network(conn1, th1, conn2, th2, wl.w_in)
         st = TrainStep(net, B, wl.d, wl.thresholds, wl.classes, wl.tau, node=node, fuse_dy1=fuse_dy1,
-                       through=through)
+                       through=through, bytes1=bytes1)
     x, lab = synth.blob_batch(B, wl.d, wl.classes, wl.sigma, seed=1000 + rank)
     st.load(x.cuda(), lab.cuda())
     return net, st
@@ -592,7 +599,8 @@ def measure_train(wl, st, args, timer, hbm, sm_max, peak_kind, sms, world, detai
     tot = max_over_ranks([sum(ms)], "cuda")[0]
     per_call, eager_step = timer.eager_split(lambda mark: st.run(mark=mark), max(3, min(K, 30)))
     work = call_work_routed(wl, B) if wl.Kc else call_work(wl, B, fuse_dy1=st.fuse_dy1,
-                                                              through=getattr(st, "through", False))
+                                                              through=getattr(st, "through", False),
+                                                              bytes1=getattr(st, "bytes1", False))
     single = {n: t for n, t in per_call.items() if n not in MULTI_KERNEL_CALLS}
     dom = max(single, key=single.get)
     res = {
@@ -792,7 +800,7 @@ def run_headline(args):
 
     # -- headline training workload
     wl = with_batch(synth.WORKLOADS[HEADLINE_TRAIN], args.batch)
-    net, st = build_train(wl, rank, args.node, FUSE[args.fuse_dy1], FUSE[args.through])
+    net, st = build_train(wl, rank, args.node, FUSE[args.fuse_dy1], FUSE[args.through], FUSE[args.bytes1])
     train = measure_train(wl, st, args, timer, hbm, sm_max, peak_kind, sms, world)
     upd = time_update(st, max(3, min(K, 20)))
     n_par = int(net.theta1.numel() + net.theta2.numel())
@@ -830,7 +838,7 @@ def run_headline(args):
     names = [] if (args.no_extras or args.profile) else [n for n in args.extras.split(",") if n]
     for name in names:
         we = synth.WORKLOADS[name]
-        enet, est = build_train(we, rank, args.node, FUSE[args.fuse_dy1], FUSE[args.through])
+        enet, est = build_train(we, rank, args.node, FUSE[args.fuse_dy1], FUSE[args.through], FUSE[args.bytes1])
         r = measure_train(we, est, args, timer, hbm, sm_max, peak_kind, sms, world, detail=False)
         r["config"] = {k_: v for k_, v in config_of(we, world, args.node).items()
                        if k_ in ("workload", "batch_per_gpu", "widths", "k", "classes", "tau")}
@@ -891,7 +899,7 @@ def run_single(args):
         net = Network(*synth.network(wl, seed=0), wl.w_in)
         hi = build_hard(wl, net, rank)
     else:
-        rnet, st = build_train(wl, rank, args.node, FUSE[args.fuse_dy1], FUSE[args.through])
+        rnet, st = build_train(wl, rank, args.node, FUSE[args.fuse_dy1], FUSE[args.through], FUSE[args.bytes1])
         net = rnet.snap() if wl.Kc else rnet   # the hard pass evaluates the discretized network
         train = measure_train(wl, st, args, timer, hbm, sm_max, peak_kind, sms, world)
         hi = build_hard(wl, net, rank, x_dev=st.x)

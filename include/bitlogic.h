@@ -92,6 +92,13 @@ int bitlogic_encode_thermometer_u8(const uint8_t* x, int64_t B, int32_t d,
                                    const uint8_t* thr_host, int32_t b,
                                    uint8_t* bits, cudaStream_t stream);
 
+/* Both forms in one pass: bits device fp32 [d*b][B] and bits8 device uint8
+ * [d*b][B], the same wires (for a step whose forward reads fp32 rows and
+ * whose backward gathers bytes).  BITLOGIC_ERR_NULL when bits8 is NULL. */
+int bitlogic_encode_thermometer_both(const uint8_t* x, int64_t B, int32_t d,
+                                     const uint8_t* thr_host, int32_t b,
+                                     float* bits, uint8_t* bits8, cudaStream_t stream);
+
 /* Distributive (quantile) thermometer fit (§3 "Encoders and heads"; App. A
  * "Initialization": thresholds fit once from the empirical pixel quantiles
  * of the training split, over the globally flattened pixels, App. B).  Two
@@ -260,6 +267,41 @@ int bitlogic_lut_backward_through(const float* X, int32_t w_in, int64_t B, const
                                   int32_t up_w, int32_t up_k, const float* up_dY, int32_t up_group,
                                   const int32_t* up_off, const int32_t* up_edge, float* dtheta,
                                   float* dY_out, cudaStream_t stream);
+
+/* bitlogic_lut_backward_through with the layer input as byte rows (binary
+ * wires, each byte 0 or 1, e.g. from bitlogic_encode_thermometer_u8):
+ * X device uint8 [w_in][B]; every other argument as above.  The result
+ * equals the fp32-row call on the same wires bit for bit. */
+int bitlogic_lut_backward_through_u8(const uint8_t* X, int32_t w_in, int64_t B, const int32_t* conn,
+                                     const float* theta, int32_t w, int32_t k, int32_t node,
+                                     const float* Y, const int32_t* up_conn, const float* up_theta,
+                                     int32_t up_w, int32_t up_k, const float* up_dY, int32_t up_group,
+                                     const int32_t* up_off, const int32_t* up_edge, float* dtheta,
+                                     float* dY_out, cudaStream_t stream);
+
+/* Table gradient (no input gradient) of a layer whose input is byte rows
+ * (binary wires, each byte 0 or 1): gathering bytes moves a quarter of the
+ * data of fp32 rows, which is what bounds the first layer once its input is
+ * larger than L2.  The output gradient comes from exactly one of
+ *   dY rows:  node j reads row j / dy_group of dY ([w / dy_group][B]);
+ *   up terms: the next layer's per-edge terms up_terms [up_edges][B] summed
+ *             over p in [up_off[j], up_off[j+1]) in increasing p (row
+ *             up_edge[p], or p when up_edge is NULL): the same sum, bit for
+ *             bit, as bitlogic_csr_reduce.
+ *   X         device uint8 [w_in][B];  conn, theta, dtheta, node as in
+ *             bitlogic_lut_backward_node;  dY_out device fp32 [w][B] or NULL
+ *             (the gradient used).
+ * The result equals bitlogic_lut_backward_node without edge terms on the
+ * same wires as fp32 rows, bit for bit.  Needs B % 4 == 0 and 16-byte
+ * aligned X, the source and dY_out (BITLOGIC_ERR_ALIGN otherwise); B = 0
+ * zeroes dtheta.  Out-of-range indices raise the device flag and read as
+ * zero.  Returns BITLOGIC_ERR_NULL (no source or two), BITLOGIC_ERR_SHAPE,
+ * BITLOGIC_ERR_FANIN, BITLOGIC_ERR_NODE, BITLOGIC_ERR_CUDA. */
+int bitlogic_lut_backward_u8(const uint8_t* X, int32_t w_in, int64_t B, const int32_t* conn,
+                             const float* theta, int32_t w, int32_t k, int32_t node,
+                             const float* dY, int32_t dy_group, const float* up_terms,
+                             const int32_t* up_off, const int32_t* up_edge, int32_t up_edges,
+                             float* dtheta, float* dY_out, cudaStream_t stream);
 
 /* Learnable routing (§3, the paragraph on connectivity: a per-slot
  * candidate pool whose selection is differentiable in training and snapped

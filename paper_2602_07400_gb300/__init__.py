@@ -27,11 +27,13 @@ __all__ = [
     "BitLogicError", "load", "bitlogic_encode_thermometer", "bitlogic_lut_forward",
     "bitlogic_lut_backward_workspace", "bitlogic_lut_backward", "bitlogic_lut_backward_edges",
     "bitlogic_csr_reduce", "bitlogic_lut_backward_ex", "bitlogic_head_loss_ex",
-    "bitlogic_head_loss_workspace", "bitlogic_head_loss_noalloc", "bitlogic_lut_backward_through",
+    "bitlogic_head_loss_workspace", "bitlogic_head_loss_noalloc", "bitlogic_lut_backward_through", "bitlogic_lut_backward_through_u8",
+    "bitlogic_lut_backward_u8",
     "bitlogic_head_loss", "bitlogic_binarize_tables", "bitlogic_pack_bits",
     "bitlogic_hard_forward", "bitlogic_build_csr", "bitlogic_csr_positions", "bitlogic_device_error",
     "bitlogic_adamw_update", "bitlogic_route_forward", "bitlogic_route_backward", "bitlogic_route_snap",
     "bitlogic_route_forward_u8", "bitlogic_route_backward_u8", "bitlogic_encode_thermometer_u8",
+    "bitlogic_encode_thermometer_both",
     "bitlogic_pixel_histogram", "bitlogic_quantile_thresholds", "bitlogic_lut_forward_node", "bitlogic_lut_backward_node", "NODE_FORMS",
     "bitlogic_status_string", "bitlogic_version", "LIB_PATH",
     "bitlogic_issue_probe", "bitlogic_issue_probe_blocks", "bitlogic_issue_probe_threads", "bitlogic_issue_probe_ops_per_iter", "PROBE_KINDS",
@@ -74,6 +76,7 @@ _SIGS = {
     "bitlogic_route_forward_u8": ([_P, _I32, _I64, _P, _P, _I32, _I32, _P, _P, _P], ctypes.c_int),
     "bitlogic_route_backward_u8": ([_P, _I32, _I64, _P, _P, _I32, _I32, _P, _P, _P], ctypes.c_int),
     "bitlogic_encode_thermometer_u8": ([_P, _I64, _I32, _P, _I32, _P, _P], ctypes.c_int),
+    "bitlogic_encode_thermometer_both": ([_P, _I64, _I32, _P, _I32, _P, _P, _P], ctypes.c_int),
     "bitlogic_quantile_thresholds": ([_P, _I32, _P], ctypes.c_int),
     "bitlogic_lut_forward_node": ([_P, _I32, _I64, _P, _P, _I32, _I32, _I32, _P, _P], ctypes.c_int),
     "bitlogic_lut_backward_workspace": ([_I32, _I64, _I32, _I32, _I32], _SZ),
@@ -88,6 +91,10 @@ _SIGS = {
                                     _P, _P, _P, _P, _P], ctypes.c_int),
     "bitlogic_lut_backward_through": ([_P, _I32, _I64, _P, _P, _I32, _I32, _I32, _P, _P, _P, _I32, _I32, _P, _I32,
                                        _P, _P, _P, _P, _P], ctypes.c_int),
+    "bitlogic_lut_backward_through_u8": ([_P, _I32, _I64, _P, _P, _I32, _I32, _I32, _P, _P, _P, _I32, _I32, _P,
+                                          _I32, _P, _P, _P, _P, _P], ctypes.c_int),
+    "bitlogic_lut_backward_u8": ([_P, _I32, _I64, _P, _P, _I32, _I32, _I32, _P, _I32, _P, _P, _P, _I32, _P, _P, _P],
+                                 ctypes.c_int),
     "bitlogic_head_loss_ex": ([_P, _I32, _I64, _I32, _F32, _P, _P, _P, _P, _P, _P, _SZ, _P],
                               ctypes.c_int),
     "bitlogic_head_loss_workspace": ([_I64, _I32], _SZ),
@@ -219,6 +226,18 @@ def bitlogic_encode_thermometer_u8(x: torch.Tensor, thresholds, bits: torch.Tens
     _need(bits, "bits", torch.uint8, (d * b, B))
     _check("bitlogic_encode_thermometer_u8", load().bitlogic_encode_thermometer_u8(
         _ptr(x), B, d, buf, b, _ptr(bits), _stream(stream)))
+
+
+def bitlogic_encode_thermometer_both(x: torch.Tensor, thresholds, bits: torch.Tensor, bits8: torch.Tensor,
+                                     stream=None):
+    """The thermometer wires as fp32 rows and as byte rows, in one pass."""
+    B, d = x.shape
+    thr, b = _thr_buf(thresholds)
+    _need(x, "x", torch.uint8, (B, d))
+    _need(bits, "bits", torch.float32, (d * b, B))
+    _need(bits8, "bits8", torch.uint8, (d * b, B))
+    _check("bitlogic_encode_thermometer_both", load().bitlogic_encode_thermometer_both(
+        _ptr(x), B, d, thr, b, _ptr(bits), _ptr(bits8), _stream(stream)))
 
 
 def bitlogic_route_forward_u8(X: torch.Tensor, cand: torch.Tensor, r: torch.Tensor, Xr: torch.Tensor,
@@ -471,11 +490,17 @@ def bitlogic_lut_backward_through(X: torch.Tensor, conn: torch.Tensor, theta: to
                                   dY_out: Optional[torch.Tensor] = None, stream=None):
     """Table gradient of a layer from the next layer's output gradient,
     recomputing this layer's output gradient through the next layer (fan-in
-    1..3) instead of reading stored per-edge terms."""
+    1..3) instead of reading stored per-edge terms.  X: fp32 rows, or uint8
+    rows of binary wires."""
     w_in, B = X.shape
     w, k = conn.shape
     up_w, up_k = up_conn.shape
-    _need(X, "X", torch.float32, (w_in, B))
+    if X.dtype == torch.uint8:
+        _need(X, "X", torch.uint8, (w_in, B))
+        fn = "bitlogic_lut_backward_through_u8"
+    else:
+        _need(X, "X", torch.float32, (w_in, B))
+        fn = "bitlogic_lut_backward_through"
     _need(conn, "conn", torch.int32, (w, k))
     _need(theta, "theta", torch.float32, (w, 1 << k))
     _need(dtheta, "dtheta", torch.float32, (w, 1 << k))
@@ -490,10 +515,48 @@ def bitlogic_lut_backward_through(X: torch.Tensor, conn: torch.Tensor, theta: to
         _need(up_edge, "up_edge", torch.int32, (up_w * up_k,))
     if dY_out is not None:
         _need(dY_out, "dY_out", torch.float32, (w, B))
-    _check("bitlogic_lut_backward_through", load().bitlogic_lut_backward_through(
+    _check(fn, getattr(load(), fn)(
         _ptr(X), w_in, B, _ptr(conn), _ptr(theta), w, k, _node_code(node), _ptr(Y), _ptr(up_conn),
         _ptr(up_theta), up_w, up_k, _ptr(up_dY), int(up_group), _ptr(up_off), _ptr(up_edge), _ptr(dtheta),
         _ptr(dY_out), _stream(stream)))
+
+
+def bitlogic_lut_backward_through_u8(X: torch.Tensor, *args, **kwargs):
+    """bitlogic_lut_backward_through with X as uint8 rows of binary wires."""
+    if not isinstance(X, torch.Tensor) or X.dtype != torch.uint8:
+        raise TypeError("X must be a uint8 tensor")
+    bitlogic_lut_backward_through(X, *args, **kwargs)
+
+
+def bitlogic_lut_backward_u8(X: torch.Tensor, conn: torch.Tensor, theta: torch.Tensor, dtheta: torch.Tensor,
+                             node="soft", dY: Optional[torch.Tensor] = None, dy_group: int = 1,
+                             up_terms: Optional[torch.Tensor] = None, up_off: Optional[torch.Tensor] = None,
+                             up_edge: Optional[torch.Tensor] = None, dY_out: Optional[torch.Tensor] = None,
+                             stream=None):
+    """Table gradient of a layer whose input is byte rows (binary wires),
+    from dY rows or from the next layer's per-edge terms (no input gradient)."""
+    w_in, B = X.shape
+    w, k = conn.shape
+    _need(X, "X", torch.uint8, (w_in, B))
+    _need(conn, "conn", torch.int32, (w, k))
+    _need(theta, "theta", torch.float32, (w, 1 << k))
+    _need(dtheta, "dtheta", torch.float32, (w, 1 << k))
+    n_up = 0
+    if dY is not None:
+        if w % dy_group != 0:
+            raise ValueError("dy_group must divide w")
+        _need(dY, "dY", torch.float32, (w // dy_group, B))
+    if up_terms is not None:
+        n_up = up_terms.shape[0]
+        _need(up_terms, "up_terms", torch.float32, (n_up, B))
+        _need(up_off, "up_off", torch.int32, (w + 1,))
+        if up_edge is not None:
+            _need(up_edge, "up_edge", torch.int32, (n_up,))
+    if dY_out is not None:
+        _need(dY_out, "dY_out", torch.float32, (w, B))
+    _check("bitlogic_lut_backward_u8", load().bitlogic_lut_backward_u8(
+        _ptr(X), w_in, B, _ptr(conn), _ptr(theta), w, k, _node_code(node), _ptr(dY), int(dy_group),
+        _ptr(up_terms), _ptr(up_off), _ptr(up_edge), n_up, _ptr(dtheta), _ptr(dY_out), _stream(stream)))
 
 
 def bitlogic_head_loss_ex(Y: torch.Tensor, labels: torch.Tensor, C: int, tau: float,

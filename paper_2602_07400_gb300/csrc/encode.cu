@@ -34,7 +34,7 @@ __device__ __forceinline__ void put_bits4(uint8_t* p, bool a, bool b, bool c, bo
 template <typename OutT>
 __global__ void __launch_bounds__(256)
 encode_soft_kernel(const uint8_t* __restrict__ x, long long B, int d, Thresholds th,
-                   OutT* __restrict__ bits) {
+                   OutT* __restrict__ bits, uint8_t* __restrict__ bits8) {
     __shared__ uint8_t tile[kEncTF][kEncTS + 4];   // feature-major
     __shared__ uint32_t sT[32];
     if (threadIdx.x < th.b) sT[threadIdx.x] = threshold_at(th, threadIdx.x);
@@ -59,7 +59,10 @@ encode_soft_kernel(const uint8_t* __restrict__ x, long long B, int d, Thresholds
     if (s >= B) return;
     for (int r = tr; r < rows; r += 4) {
         const int f = r / th.b, i = r - f * th.b;
-        put_bit(bits + ((long long)(f0 + f) * th.b + i) * B + s, tile[f][tsl] > sT[i]);
+        const long long o = ((long long)(f0 + f) * th.b + i) * B + s;
+        const bool v = tile[f][tsl] > sT[i];
+        put_bit(bits + o, v);
+        if (bits8) put_bit(bits8 + o, v);   // the same wires as bytes
     }
 }
 
@@ -73,7 +76,7 @@ constexpr int kEncVS = 128;   // samples per tile (vector form)
 template <typename OutT>
 __global__ void __launch_bounds__(256)
 encode_soft_vec_kernel(const uint8_t* __restrict__ x, long long B, int d, Thresholds th,
-                       OutT* __restrict__ bits, bool vec16) {
+                       OutT* __restrict__ bits, uint8_t* __restrict__ bits8, bool vec16) {
     __shared__ __align__(16) uint8_t tile[kEncTF][kEncVS];   // feature-major
     __shared__ uint32_t sT[32];
     if (threadIdx.x < th.b) sT[threadIdx.x] = threshold_at(th, threadIdx.x);
@@ -107,8 +110,10 @@ encode_soft_vec_kernel(const uint8_t* __restrict__ x, long long B, int d, Thresh
         const int f = r / th.b, i = r - f * th.b;
         const uint32_t q = *reinterpret_cast<const uint32_t*>(&tile[f][4 * u]);
         const uint32_t T = sT[i];
-        put_bits4(bits + ((long long)(f0 + f) * th.b + i) * B + s, (q & 0xffu) > T, ((q >> 8) & 0xffu) > T,
-                  ((q >> 16) & 0xffu) > T, (q >> 24) > T);
+        const long long o = ((long long)(f0 + f) * th.b + i) * B + s;
+        const bool v0 = (q & 0xffu) > T, v1 = ((q >> 8) & 0xffu) > T, v2 = ((q >> 16) & 0xffu) > T, v3 = (q >> 24) > T;
+        put_bits4(bits + o, v0, v1, v2, v3);
+        if (bits8) put_bits4(bits8 + o, v0, v1, v2, v3);   // the same wires as bytes
     }
 }
 
@@ -248,25 +253,25 @@ BITLOGIC_ERROR_READER(encode)
 namespace {
 template <typename OutT>
 int encode_impl(const uint8_t* x, int64_t B, int32_t d, const uint8_t* thr_host, int32_t b, OutT* bits,
-                cudaStream_t stream) {
+                uint8_t* bits8, cudaStream_t stream) {
     Thresholds th;
     int st = make_thresholds(thr_host, b, &th);
     if (st) return st;
     if (B < 0 || d <= 0) return BITLOGIC_ERR_SHAPE;
     if (B == 0) return BITLOGIC_OK;   // an empty batch may come as NULL
     if (!x || !bits) return BITLOGIC_ERR_NULL;
-    if (B % 4 == 0 && aligned16(bits)) {
+    if (B % 4 == 0 && aligned16(bits) && (!bits8 || aligned16(bits8))) {
         const long long gy = (B + kEncVS - 1) / kEncVS;
         if (gy > 65535) return BITLOGIC_ERR_SHAPE;
         const bool vec16 = (d % 16 == 0) && aligned16(x);
         dim3 grid((unsigned)((d + kEncTF - 1) / kEncTF), (unsigned)gy);
-        encode_soft_vec_kernel<OutT><<<grid, 256, 0, stream>>>(x, B, d, th, bits, vec16);
+        encode_soft_vec_kernel<OutT><<<grid, 256, 0, stream>>>(x, B, d, th, bits, bits8, vec16);
         return launch_status();
     }
     const long long gy = (B + kEncTS - 1) / kEncTS;
     if (gy > 65535) return BITLOGIC_ERR_SHAPE;
     dim3 grid((unsigned)((d + kEncTF - 1) / kEncTF), (unsigned)gy);
-    encode_soft_kernel<OutT><<<grid, 256, 0, stream>>>(x, B, d, th, bits);
+    encode_soft_kernel<OutT><<<grid, 256, 0, stream>>>(x, B, d, th, bits, bits8);
     return launch_status();
 }
 }  // namespace
@@ -274,13 +279,20 @@ int encode_impl(const uint8_t* x, int64_t B, int32_t d, const uint8_t* thr_host,
 extern "C" int bitlogic_encode_thermometer(const uint8_t* x, int64_t B, int32_t d,
                                            const uint8_t* thr_host, int32_t b,
                                            float* bits, cudaStream_t stream) {
-    return encode_impl(x, B, d, thr_host, b, bits, stream);
+    return encode_impl(x, B, d, thr_host, b, bits, nullptr, stream);
 }
 
 extern "C" int bitlogic_encode_thermometer_u8(const uint8_t* x, int64_t B, int32_t d,
                                               const uint8_t* thr_host, int32_t b,
                                               uint8_t* bits, cudaStream_t stream) {
-    return encode_impl(x, B, d, thr_host, b, bits, stream);
+    return encode_impl(x, B, d, thr_host, b, bits, nullptr, stream);
+}
+
+extern "C" int bitlogic_encode_thermometer_both(const uint8_t* x, int64_t B, int32_t d,
+                                                const uint8_t* thr_host, int32_t b,
+                                                float* bits, uint8_t* bits8, cudaStream_t stream) {
+    if (B > 0 && !bits8) return BITLOGIC_ERR_NULL;
+    return encode_impl(x, B, d, thr_host, b, bits, bits8, stream);
 }
 
 extern "C" int bitlogic_pack_bits(const uint8_t* x, int64_t N, int32_t d,

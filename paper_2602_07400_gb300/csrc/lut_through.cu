@@ -1,11 +1,23 @@
-// Table gradient of a LUT layer whose output gradient is recomputed from the
-// next layer (chain rule through a next layer of small fan-in), so that
-// neither the next layer's per-edge input-gradient terms nor this layer's
-// output gradient are stored.
+// Table gradient of a LUT layer (the dtheta-only backward: no input
+// gradient), for the inputs and output-gradient sources the training step
+// uses on its first layer:
 //
-// For the node j of this layer, output row j is an input of the next layer;
-// its gradient (the next layer's input gradient, summed over the consumers)
-// is
+// * the layer input as fp32 rows or as byte rows (binary wires, e.g. the
+//   thermometer encoder's output written by bitlogic_encode_thermometer_u8):
+//   gathering bytes moves a quarter of the data, which matters when the input
+//   is larger than L2 and every node's k gathered rows come from DRAM;
+// * the output gradient from
+//   - rows: row j / group of dY (group = 1: one row per node);
+//   - terms: the next layer's per-edge input-gradient terms, summed over the
+//     node's consumers in increasing CSR position (the order of
+//     bitlogic_csr_reduce, so the sum is the same bit for bit);
+//   - through: recomputed from the next layer itself (chain rule through a
+//     next layer of small fan-in), so that neither the next layer's per-edge
+//     terms nor this layer's output gradient are stored.
+//
+// Through: for the node j of this layer, output row j is an input of the
+// next layer; its gradient (the next layer's input gradient, summed over
+// the consumers) is
 //   g_j[s] = sum over the consumer edges e = (j2, slot) of j, in increasing
 //            CSR position (node order), of dY2[j2][s] * d y_j2 / d x_slot (s),
 // and for a next-layer node of fan-in ku the derivative with respect to one
@@ -28,11 +40,12 @@
 // Layout and scheduling follow the dtheta-only kernel: persistent one-warp
 // blocks, a node over the whole batch, 4 consecutive samples per lane in each
 // 128-sample stage, the node's k input rows streamed through a lane-private
-// cp.async ring that runs across node boundaries, and a fixed butterfly of
-// shuffles for the batch reduction.  The consumers' rows are gathered for
-// several stages at a time (eight for k <= 3), so a warp has eight (ku = 1)
-// to twenty-four (ku = 3) independent loads in flight per consumer.  Needs B % 4 == 0 and 16-byte aligned
-// X, Y, the next layer's gradient rows and dY_out.
+// cp.async ring that runs across node boundaries (16 bytes per lane and row
+// for fp32 rows, 4 for byte rows), and a fixed butterfly of shuffles for the
+// batch reduction.  The output gradient is formed for several stages at a
+// time (a chunk), so the rows it reads (gradient rows, term rows, consumer
+// rows) have several independent loads in flight per row.  Needs B % 4 == 0
+// and 16-byte aligned X, the gradient rows, the terms, Y and dY_out.
 #include "common.cuh"
 
 namespace bitlogic {
@@ -40,11 +53,21 @@ namespace {
 
 constexpr int kTStageSamples = 128;   // one 16-byte chunk per lane and row
 constexpr int kTStages = 3;           // ring stages in flight per warp
-constexpr int kTMinBlocks = 16;       // one-warp blocks per SM
+#ifndef BITLOGIC_THROUGH_MIN_BLOCKS
+#define BITLOGIC_THROUGH_MIN_BLOCKS 16
+#endif
+#ifndef BITLOGIC_THROUGH_CHUNK
+#define BITLOGIC_THROUGH_CHUNK 8
+#endif
+constexpr int kTMinBlocks = BITLOGIC_THROUGH_MIN_BLOCKS;   // one-warp blocks per SM
+static_assert(kTMinBlocks >= 1 && kTMinBlocks <= 32, "one-warp blocks per SM");
+static_assert(BITLOGIC_THROUGH_CHUNK >= 1 && BITLOGIC_THROUGH_CHUNK <= 16, "stages gathered together");
 // stages whose consumer rows are gathered together: fewer for the wider
 // tables, whose 2^k accumulators already take most registers
 template <int k>
-__host__ __device__ constexpr int through_chunk() { return k <= 3 ? 8 : (k == 4 ? 4 : (k == 5 ? 2 : 1)); }
+__host__ __device__ constexpr int through_chunk() {
+    return k <= 3 ? BITLOGIC_THROUGH_CHUNK : (k == 4 ? 4 : (k == 5 ? 2 : 1));
+}
 
 __device__ __forceinline__ float4 ldg4t(const float* p) { return __ldg(reinterpret_cast<const float4*>(p)); }
 
@@ -182,29 +205,86 @@ __device__ __forceinline__ void add_consumer(float4& g, const Consumer<ku>& q, c
     }
 }
 
-template <int k>
-__host__ __device__ constexpr int through_floats_per_warp() {
-    return kTStages * k * kTStageSamples;
+// The output-gradient sources.
+constexpr int kSrcRows = 0, kSrcTerms = 1, kSrcThrough = 2;
+
+struct GradIn {
+    const float* dY;        // rows: [w / group][B]
+    int group;
+    const float* terms;     // terms: [n_terms][B]
+    int n_terms;
+    const int* off;         // terms, through: CSR positions of this layer's rows [w + 1]
+    const int* edge;        // terms, through: edge ids in CSR order (NULL: identity)
+    const float* Y;         // through: this layer's output [w][B]
+    const int* up_conn;     // through: the next layer [up_w][up_k]
+    const float* up_theta;
+    int up_w;
+    const float* up_dY;     // through: the next layer's gradient rows [up_w / up_group][B]
+    int up_group;
+};
+
+// Stages whose output gradient is formed together (registers: four float4
+// per stage of the chunk, besides the 2^k accumulators).
+#ifndef BITLOGIC_TERMS_CHUNK
+#define BITLOGIC_TERMS_CHUNK 2      // stages per chunk, k >= 5, rows and terms sources
+#endif
+#ifndef BITLOGIC_TERMS_ROWS
+#define BITLOGIC_TERMS_ROWS 2       // term rows whose loads are in flight together
+#endif
+#ifndef BITLOGIC_TERMS_BLOCKS
+#define BITLOGIC_TERMS_BLOCKS 12    // one-warp blocks per SM, k = 6, rows and terms sources
+#endif
+static_assert(BITLOGIC_TERMS_ROWS == 1 || BITLOGIC_TERMS_ROWS == 2 || BITLOGIC_TERMS_ROWS == 4, "rows in flight");
+template <int k, int SRC>
+__host__ __device__ constexpr int grad_chunk() {
+    if constexpr (SRC == kSrcThrough) return k <= 3 ? BITLOGIC_THROUGH_CHUNK : (k == 4 ? 4 : (k == 5 ? 2 : 1));
+    else return k <= 4 ? 4 : BITLOGIC_TERMS_CHUNK;
+}
+// one-warp blocks per SM: fewer for the widest tables (their accumulators
+// and the loads in flight take more registers)
+template <int k, int SRC>
+__host__ __device__ constexpr int grad_min_blocks() {
+    return (k >= 6 && SRC != kSrcThrough) ? BITLOGIC_TERMS_BLOCKS : kTMinBlocks;
 }
 
-template <int k, int ku>
-__global__ void __launch_bounds__(32, kTMinBlocks)
-lut_theta_through_kernel(const float* __restrict__ X, int w_in, long long B, const int* __restrict__ conn,
-                         const float* __restrict__ theta, int w, const float* __restrict__ Y,
-                         const int* __restrict__ up_conn, const float* __restrict__ up_theta, int up_w,
-                         const float* __restrict__ up_dY, int up_group, const int* __restrict__ up_off,
-                         const int* __restrict__ up_edge, int node, float* __restrict__ dtheta,
-                         float* __restrict__ dY_out) {
+template <typename TX>
+__host__ __device__ constexpr int ring_bytes_per_warp(int k) {
+    return kTStages * k * kTStageSamples * (int)sizeof(TX);
+}
+
+// The lane's 16 (fp32) or 4 (bytes) bytes of one row of one stage.
+__device__ __forceinline__ void copy_row_part(float* dst, const float* src) { cp_async16(dst, src); }
+__device__ __forceinline__ void copy_row_part(uint8_t* dst, const uint8_t* src) {
+    const unsigned sa = (unsigned)__cvta_generic_to_shared(dst);
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;\n" ::"r"(sa), "l"(src) : "memory");
+}
+// Its four samples as floats (a byte b becomes b exactly: 2^23 + b in the
+// mantissa, minus 2^23).
+__device__ __forceinline__ float4 read_row_part(const float* p) { return *reinterpret_cast<const float4*>(p); }
+__device__ __forceinline__ float4 read_row_part(const uint8_t* p) {
+    const uint32_t v = *reinterpret_cast<const uint32_t*>(p);
+    const float m = 8388608.0f;
+    return make_float4(__int_as_float(__byte_perm(v, 0x4B000000u, 0x7440)) - m,
+                       __int_as_float(__byte_perm(v, 0x4B000000u, 0x7441)) - m,
+                       __int_as_float(__byte_perm(v, 0x4B000000u, 0x7442)) - m,
+                       __int_as_float(__byte_perm(v, 0x4B000000u, 0x7443)) - m);
+}
+
+template <int k, int ku, typename TX, int SRC>
+__global__ void __launch_bounds__(32, (grad_min_blocks<k, SRC>()))
+lut_theta_src_kernel(const TX* __restrict__ X, int w_in, long long B, const int* __restrict__ conn,
+                     const float* __restrict__ theta, int w, GradIn gi, int node, float* __restrict__ dtheta,
+                     float* __restrict__ dY_out) {
     constexpr int K = 1 << k, KL = k / 2, NU = 1 << KL, NV = 1 << (k - KL);
     constexpr int CH = kTStageSamples;
-    constexpr int kTChunk = through_chunk<k>();
-    extern __shared__ __align__(16) float smem[];
+    constexpr int kTChunk = grad_chunk<k, SRC>();
+    extern __shared__ __align__(16) unsigned char smem_raw[];
     const int lane = threadIdx.x & 31;
-    float* ring = smem;
+    TX* ring = reinterpret_cast<TX*>(smem_raw);
     const int G = gridDim.x;
     const int jfirst = blockIdx.x;
     const int nst = (int)((B + CH - 1) / CH);
-    const int n_up = up_w * ku;
+    const int n_up = SRC == kSrcThrough ? gi.up_w * ku : gi.n_terms;   // CSR positions
 
     // issue stream: stage si of node ji, kTStages - 1 stages ahead of the
     // compute stream; rows of the warp's node after ji are loaded ahead
@@ -231,9 +311,9 @@ lut_theta_through_kernel(const float* __restrict__ X, int w_in, long long B, con
         if (ji < w) {
             const long long s4 = (long long)si * CH + 4 * lane;
             if (s4 < B) {
-                float* buf = ring + ib * (k * CH) + 4 * lane;
+                TX* buf = ring + ib * (k * CH) + 4 * lane;
 #pragma unroll
-                for (int r = 0; r < k; ++r) cp_async16(buf + r * CH, X + (long long)ri[r] * B + s4);
+                for (int r = 0; r < k; ++r) copy_row_part(buf + r * CH, X + (long long)ri[r] * B + s4);
             }
             if (++si == nst) {
                 si = 0;
@@ -252,52 +332,110 @@ lut_theta_through_kernel(const float* __restrict__ X, int w_in, long long B, con
     int rb = 0;
 #pragma unroll 1
     for (int j = jfirst; j < w; j += G) {
-        // the node's consumers in the next layer (CSR positions e0 .. e1 - 1)
-        int e0 = __ldg(up_off + j), e1 = __ldg(up_off + j + 1);
-        if (e0 < 0 || e1 < e0 || e1 > n_up) {
-            if (lane == 0) flag_index_error();
-            e0 = e1 = 0;
+        // the node's upstream edges (terms, through: CSR positions e0 .. e1 - 1)
+        int e0 = 0, deg = 0;
+        if constexpr (SRC != kSrcRows) {
+            int e1;
+            e0 = __ldg(gi.off + j);
+            e1 = __ldg(gi.off + j + 1);
+            if (e0 < 0 || e1 < e0 || e1 > n_up) {
+                if (lane == 0) flag_index_error();
+                e0 = e1 = 0;
+            }
+            deg = e1 - e0;
         }
-        const int deg = e1 - e0;
-        bool bad = false;
+        // per lane one upstream edge: a term row id (terms) or a consumer
+        // (through), for the positions e0 .. e0 + 31
+        int my_id = -1;
         Consumer<ku> mine;
         mine.grow = -1;
-        if (lane < deg)
-            mine = load_consumer<ku>(e0 + lane, up_edge, n_up, up_conn, up_theta, up_group, w, node, bad);
-        if (__any_sync(0xffffffffu, bad) && lane == 0) flag_index_error();
+        auto load_edges = [&](int c0) {
+            bool bad = false;
+            my_id = -1;
+            mine.grow = -1;
+            if (c0 + lane < deg) {
+                if constexpr (SRC == kSrcTerms) {
+                    const int p = e0 + c0 + lane;
+                    my_id = gi.edge ? __ldg(gi.edge + p) : p;
+                    if ((unsigned)my_id >= (unsigned)gi.n_terms) {
+                        bad = true;
+                        my_id = -1;
+                    }
+                } else if constexpr (SRC == kSrcThrough) {
+                    mine = load_consumer<ku>(e0 + c0 + lane, gi.edge, n_up, gi.up_conn, gi.up_theta,
+                                             gi.up_group, w, node, bad);
+                }
+            }
+            if (__any_sync(0xffffffffu, bad) && lane == 0) flag_index_error();
+        };
+        if constexpr (SRC != kSrcRows) load_edges(0);
 
         float acc[K];
 #pragma unroll
         for (int a = 0; a < K; ++a) acc[a] = 0.f;
 #pragma unroll 1
         for (int sc0 = 0; sc0 < nst; sc0 += kTChunk) {
-            // the node's output gradient over kTChunk stages, consumers in
-            // increasing CSR position: each consumer's rows are gathered for
-            // all the chunk's stages at once (kTChunk loads per row in flight)
+            // the node's output gradient over kTChunk stages
             float4 gv[kTChunk];
 #pragma unroll
             for (int t = 0; t < kTChunk; ++t) gv[t] = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 1
-            for (int c0 = 0; c0 < deg; c0 += 32) {
-                Consumer<ku> cur = mine;
-                if (c0 > 0) {   // more than 32 consumers: this chunk's edges
-                    bool bad2 = false;
-                    cur.grow = -1;
-                    if (c0 + lane < deg)
-                        cur = load_consumer<ku>(e0 + c0 + lane, up_edge, n_up, up_conn, up_theta, up_group, w,
-                                                node, bad2);
-                    if (__any_sync(0xffffffffu, bad2) && lane == 0) flag_index_error();
-                }
-                const int n = min(32, deg - c0);
-#pragma unroll 1
-                for (int e = 0; e < n; ++e) {
-                    const Consumer<ku> q = shfl_consumer<ku>(cur, e);
+            if constexpr (SRC == kSrcRows) {
+                const float* row = gi.dY + (long long)(j / gi.group) * B;
 #pragma unroll
-                    for (int t = 0; t < kTChunk; ++t) {
-                        const long long s4 = (long long)(sc0 + t) * CH + 4 * lane;
-                        if (s4 < B) add_consumer<ku>(gv[t], q, Y, up_dY, B, s4);
+                for (int t = 0; t < kTChunk; ++t) {
+                    const long long s4 = (long long)(sc0 + t) * CH + 4 * lane;
+                    if (s4 < B) gv[t] = ldg4t(row + s4);
+                }
+            } else {
+#pragma unroll 1
+                for (int c0 = 0; c0 < deg; c0 += 32) {
+                    if (c0 > 0) load_edges(c0);   // more than 32 upstream edges: this chunk's
+                    const int n = min(32, deg - c0);
+                    if constexpr (SRC == kSrcTerms) {
+                        // term rows in increasing CSR position, kRows rows' loads in flight
+                        constexpr int kRows = BITLOGIC_TERMS_ROWS;
+#pragma unroll 1
+                        for (int e = 0; e < n; e += kRows) {
+                            int id[kRows];
+#pragma unroll
+                            for (int u = 0; u < kRows; ++u) {
+                                id[u] = __shfl_sync(0xffffffffu, my_id, (e + u) & 31);
+                                if (e + u >= n) id[u] = -1;
+                            }
+                            float4 v[kRows][kTChunk];
+#pragma unroll
+                            for (int u = 0; u < kRows; ++u)
+#pragma unroll
+                                for (int t = 0; t < kTChunk; ++t) {
+                                    const long long s4 = (long long)(sc0 + t) * CH + 4 * lane;
+                                    v[u][t] = (s4 < B && id[u] >= 0) ? ldg4t(gi.terms + (long long)id[u] * B + s4)
+                                                                     : make_float4(0.f, 0.f, 0.f, 0.f);
+                                }
+#pragma unroll
+                            for (int u = 0; u < kRows; ++u)
+#pragma unroll
+                                for (int t = 0; t < kTChunk; ++t) {
+                                    if (e + u < n) {
+                                        gv[t].x += v[u][t].x; gv[t].y += v[u][t].y;
+                                        gv[t].z += v[u][t].z; gv[t].w += v[u][t].w;
+                                    }
+                                }
+                        }
+                    } else {
+                        // consumers in increasing CSR position: each consumer's rows
+                        // for all the chunk's stages at once
+#pragma unroll 1
+                        for (int e = 0; e < n; ++e) {
+                            const Consumer<ku> q = shfl_consumer<ku>(mine, e);
+#pragma unroll
+                            for (int t = 0; t < kTChunk; ++t) {
+                                const long long s4 = (long long)(sc0 + t) * CH + 4 * lane;
+                                if (s4 < B) add_consumer<ku>(gv[t], q, gi.Y, gi.up_dY, B, s4);
+                            }
+                        }
                     }
                 }
+                if (deg > 32) load_edges(0);   // the next chunk of stages starts again at position e0
             }
             // the chunk's stages: the table gradient from the node's inputs
 #pragma unroll
@@ -308,10 +446,10 @@ lut_theta_through_kernel(const float* __restrict__ X, int w_in, long long B, con
                     const long long s4 = (long long)(sc0 + t) * CH + 4 * lane;   // this lane's 4 samples
                     if (s4 < B) {   // B % 4 == 0: all four samples are in range
                         if (dY_out) *reinterpret_cast<float4*>(dY_out + (long long)j * B + s4) = gv[t];
-                        const float* buf = ring + rb * (k * CH) + 4 * lane;
+                        const TX* buf = ring + rb * (k * CH) + 4 * lane;
                         float4 xv[k];
 #pragma unroll
-                        for (int q = 0; q < k; ++q) xv[q] = *reinterpret_cast<const float4*>(buf + q * CH);
+                        for (int q = 0; q < k; ++q) xv[q] = read_row_part(buf + q * CH);
 #pragma unroll
                         for (int r = 0; r < 4; ++r) {
                             float x[k], omx[k];
@@ -366,40 +504,278 @@ lut_theta_through_kernel(const float* __restrict__ X, int w_in, long long B, con
     cp_async_wait<0>();
 }
 
-template <int k, int ku>
-int launch_through(const float* X, int w_in, long long B, const int* conn, const float* theta, int w,
-                   const float* Y, const int* up_conn, const float* up_theta, int up_w, const float* up_dY,
-                   int up_group, const int* up_off, const int* up_edge, int node, float* dtheta, float* dY_out,
-                   cudaStream_t st) {
-    constexpr size_t smem = (size_t)through_floats_per_warp<k>() * sizeof(float);
-    auto kern = lut_theta_through_kernel<k, ku>;
-    if (smem > 40 * 1024 &&
-        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+// Terms source with the term rows streamed through the cp.async ring: a
+// ring slot holds the node's k input rows of one stage (fp32 or bytes) and
+// the stage's segments of its first kRingTerms term rows (fp32, in CSR
+// order), copied kTStages - 1 stages ahead like the input rows, so the term
+// rows are in flight without holding registers; the term rows of a node
+// with more consumers than kRingTerms are read directly after those (in
+// CSR order: the sum keeps the order of bitlogic_csr_reduce).  The issue
+// stream keeps the term row ids of its node one per lane, and loads the ids
+// of the node after it ahead, like the input rows.
+#ifndef BITLOGIC_TERMS_RING_ROWS
+#define BITLOGIC_TERMS_RING_ROWS 10
+#endif
+constexpr int kRingTerms = BITLOGIC_TERMS_RING_ROWS;
+static_assert(kRingTerms >= 1 && kRingTerms <= 32, "term rows per ring slot");
+constexpr int kTermsRingBlocks = 12;   // one-warp blocks per SM (shared memory: ~17.7 KB per warp)
+
+template <int k, typename TX>
+__host__ __device__ constexpr int terms_slot_bytes() {
+    return k * kTStageSamples * (int)sizeof(TX) + kRingTerms * kTStageSamples * (int)sizeof(float);
+}
+
+template <int k, typename TX>
+__global__ void __launch_bounds__(32, kTermsRingBlocks)
+lut_theta_terms_ring_kernel(const TX* __restrict__ X, int w_in, long long B, const int* __restrict__ conn,
+                            const float* __restrict__ theta, int w, GradIn gi, float* __restrict__ dtheta,
+                            float* __restrict__ dY_out) {
+    constexpr int K = 1 << k, KL = k / 2, NU = 1 << KL, NV = 1 << (k - KL);
+    constexpr int CH = kTStageSamples;
+    constexpr int SLOT = terms_slot_bytes<k, TX>();
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    const int lane = threadIdx.x & 31;
+    const int G = gridDim.x;
+    const int jfirst = blockIdx.x;
+    const int nst = (int)((B + CH - 1) / CH);
+    const int n_terms = gi.n_terms;
+
+    // a node's input rows, CSR range and the ids of its first 32 term rows
+    struct NodeIn {
+        int r[k];
+        int e0, deg, id;
+    };
+    auto node_in = [&](int j, NodeIn& nd) {
+        bool bad = false;
+#pragma unroll
+        for (int i = 0; i < k; ++i) {
+            int c = __ldg(conn + (long long)j * k + i);
+            if ((unsigned)c >= (unsigned)w_in) {
+                bad = true;
+                c = 0;
+            }
+            nd.r[i] = c;
+        }
+        int e0 = __ldg(gi.off + j), e1 = __ldg(gi.off + j + 1);
+        if (e0 < 0 || e1 < e0 || e1 > n_terms) {
+            bad = true;
+            e0 = e1 = 0;
+        }
+        nd.e0 = e0;
+        nd.deg = e1 - e0;
+        nd.id = -1;
+        if (lane < nd.deg) {
+            const int p = e0 + lane;
+            nd.id = gi.edge ? __ldg(gi.edge + p) : p;
+            if ((unsigned)nd.id >= (unsigned)n_terms) {
+                bad = true;
+                nd.id = -1;
+            }
+        }
+        if (__any_sync(0xffffffffu, bad) && lane == 0) flag_index_error();
+    };
+
+    // issue stream: stage si of node ji, kTStages - 1 stages ahead of the
+    // compute stream
+    int ji = jfirst, si = 0, ib = 0;
+    NodeIn ni, nn;
+    if (ji < w) node_in(ji, ni);
+    if (ji + G < w) node_in(ji + G, nn);
+    auto issue = [&]() {
+        if (ji < w) {
+            const long long s4 = (long long)si * CH + 4 * lane;
+            const bool in = s4 < B;
+            unsigned char* slot = smem_raw + ib * SLOT;
+            TX* xb = reinterpret_cast<TX*>(slot) + 4 * lane;
+            if (in) {
+#pragma unroll
+                for (int r = 0; r < k; ++r) copy_row_part(xb + r * CH, X + (long long)ni.r[r] * B + s4);
+            }
+            float* tb = reinterpret_cast<float*>(slot + k * CH * sizeof(TX)) + 4 * lane;
+            const int nr = min(ni.deg, kRingTerms);
+            for (int t = 0; t < nr; ++t) {   // warp-uniform count; every lane takes the shuffle
+                const int id = __shfl_sync(0xffffffffu, ni.id, t);
+                if (in && id >= 0) cp_async16(tb + t * CH, gi.terms + (long long)id * B + s4);
+            }
+            if (++si == nst) {
+                si = 0;
+                ji += G;
+                ni = nn;
+                if (ji + G < w) node_in(ji + G, nn);
+            }
+        }
+        cp_async_commit();
+        ib = (ib + 1 == kTStages) ? 0 : ib + 1;
+    };
+#pragma unroll 1
+    for (int i = 0; i < kTStages - 1; ++i) issue();
+
+    int rb = 0;
+#pragma unroll 1
+    for (int j = jfirst; j < w; j += G) {
+        // the compute stream's own copy of the node's CSR range and ids (the
+        // issue stream has moved on by up to kTStages - 1 stages)
+        NodeIn nc;
+        node_in(j, nc);
+        float acc[K];
+#pragma unroll
+        for (int a = 0; a < K; ++a) acc[a] = 0.f;
+#pragma unroll 1
+        for (int sc = 0; sc < nst; ++sc) {
+            issue();
+            cp_async_wait<kTStages - 1>();
+            const long long s4 = (long long)sc * CH + 4 * lane;   // this lane's 4 samples
+            const bool in = s4 < B;   // B % 4 == 0: all four samples are in range
+            const unsigned char* slot = smem_raw + rb * SLOT;
+            const float* tb = reinterpret_cast<const float*>(slot + k * CH * sizeof(TX)) + 4 * lane;
+            // the output gradient: ring rows, then any further rows, in CSR
+            // order (warp-uniform loops: every lane takes the shuffles)
+            float4 g = make_float4(0.f, 0.f, 0.f, 0.f);
+            const int nr = min(nc.deg, kRingTerms);
+            for (int t = 0; t < nr; ++t) {
+                const int id = __shfl_sync(0xffffffffu, nc.id, t);
+                if (in && id >= 0) {
+                    const float4 v = *reinterpret_cast<const float4*>(tb + t * CH);
+                    g.x += v.x; g.y += v.y; g.z += v.z; g.w += v.w;
+                }
+            }
+            for (int t = kRingTerms; t < nc.deg; ++t) {
+                int id;
+                if (t < 32) {
+                    id = __shfl_sync(0xffffffffu, nc.id, t);
+                } else {
+                    const int p = nc.e0 + t;
+                    id = gi.edge ? __ldg(gi.edge + p) : p;
+                    if ((unsigned)id >= (unsigned)n_terms) {
+                        if (lane == 0) flag_index_error();
+                        id = -1;
+                    }
+                }
+                if (in && id >= 0) {
+                    const float4 v = ldg4t(gi.terms + (long long)id * B + s4);
+                    g.x += v.x; g.y += v.y; g.z += v.z; g.w += v.w;
+                }
+            }
+            if (in) {
+                if (dY_out) *reinterpret_cast<float4*>(dY_out + (long long)j * B + s4) = g;
+                const TX* xb = reinterpret_cast<const TX*>(slot) + 4 * lane;
+                float4 xv[k];
+#pragma unroll
+                for (int q = 0; q < k; ++q) xv[q] = read_row_part(xb + q * CH);
+#pragma unroll
+                for (int r = 0; r < 4; ++r) {
+                    float x[k], omx[k];
+#pragma unroll
+                    for (int q = 0; q < k; ++q) {
+                        x[q] = comp4(xv[q], r);
+                        omx[q] = 1.0f - x[q];
+                    }
+                    float U[NU], V[NV];
+                    U[0] = comp4(g, r);
+#pragma unroll
+                    for (int q = 0; q < KL; ++q) {   // slot q doubles U: index bit q
+#pragma unroll
+                        for (int m = 0; m < (1 << q); ++m) {
+                            U[m + (1 << q)] = U[m] * x[q];
+                            U[m] = U[m] * omx[q];
+                        }
+                    }
+                    V[0] = omx[KL];
+                    V[1] = x[KL];
+#pragma unroll
+                    for (int q = KL + 1; q < k; ++q) {   // slot q doubles V: index bit q - KL
+#pragma unroll
+                        for (int m = 0; m < (1 << (q - KL)); ++m) {
+                            V[m + (1 << (q - KL))] = V[m] * x[q];
+                            V[m] = V[m] * omx[q];
+                        }
+                    }
+#pragma unroll
+                    for (int b = 0; b < NV; ++b)
+#pragma unroll
+                        for (int a = 0; a < NU; ++a) acc[a + b * NU] = fmaf(U[a], V[b], acc[a + b * NU]);
+                }
+            }
+            rb = (rb + 1 == kTStages) ? 0 : rb + 1;
+        }
+        // the node's dtheta: butterfly over the lanes, then t (1 - t)
+        reduce_scatter<K, 16>(acc, lane);
+        constexpr int NF = K >= 32 ? K / 32 : 1;   // entries per lane
+        constexpr int SH = K >= 32 ? 0 : 5 - k;    // lanes sharing an entry (K < 32)
+        if ((lane & ((1 << SH) - 1)) == 0) {
+#pragma unroll
+            for (int i = 0; i < NF; ++i) {
+                const int a = K >= 32 ? lane * NF + i : lane >> SH;
+                const float t = sigmoidf(__ldg(theta + (long long)j * K + a));
+                dtheta[(long long)j * K + a] = t * (1.0f - t) * acc[i];
+            }
+        }
+    }
+    cp_async_wait<0>();
+}
+
+template <int k, typename TX>
+int launch_terms_ring(const TX* X, int w_in, long long B, const int* conn, const float* theta, int w,
+                      const GradIn& gi, float* dtheta, float* dY_out, cudaStream_t st) {
+    constexpr int smem = kTStages * terms_slot_bytes<k, TX>();
+    auto kern = lut_theta_terms_ring_kernel<k, TX>;
+    if (smem > 40 * 1024 && cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
         return BITLOGIC_ERR_CUDA;
-    // one wave of persistent one-warp blocks (nodes dealt round-robin)
-    const long long resident = (long long)sm_count() * kTMinBlocks;
+    const long long resident = (long long)sm_count() * kTermsRingBlocks;
     const long long blocks = w < resident ? w : resident;
-    kern<<<(unsigned)blocks, 32, smem, st>>>(X, w_in, B, conn, theta, w, Y, up_conn, up_theta, up_w, up_dY,
-                                             up_group, up_off, up_edge, node, dtheta, dY_out);
+    kern<<<(unsigned)blocks, 32, smem, st>>>(X, w_in, B, conn, theta, w, gi, dtheta, dY_out);
     return launch_status();
 }
 
-template <int k>
-int launch_through_k(int up_k, const float* X, int w_in, long long B, const int* conn, const float* theta, int w,
-                     const float* Y, const int* up_conn, const float* up_theta, int up_w, const float* up_dY,
-                     int up_group, const int* up_off, const int* up_edge, int node, float* dtheta,
-                     float* dY_out, cudaStream_t st) {
+template <int k, int ku, typename TX, int SRC>
+int launch_src(const TX* X, int w_in, long long B, const int* conn, const float* theta, int w, const GradIn& gi,
+               int node, float* dtheta, float* dY_out, cudaStream_t st) {
+    constexpr int smem = ring_bytes_per_warp<TX>(k);
+    auto kern = lut_theta_src_kernel<k, ku, TX, SRC>;
+    if (smem > 40 * 1024 && cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
+        return BITLOGIC_ERR_CUDA;
+    // one wave of persistent one-warp blocks (nodes dealt round-robin)
+    const long long resident = (long long)sm_count() * grad_min_blocks<k, SRC>();
+    const long long blocks = w < resident ? w : resident;
+    kern<<<(unsigned)blocks, 32, smem, st>>>(X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out);
+    return launch_status();
+}
+
+template <int k, typename TX>
+int launch_src_k(int src, int up_k, const TX* X, int w_in, long long B, const int* conn, const float* theta, int w,
+                 const GradIn& gi, int node, float* dtheta, float* dY_out, cudaStream_t st) {
+    if (src == kSrcRows) return launch_src<k, 1, TX, kSrcRows>(X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
+    if (src == kSrcTerms) return launch_terms_ring<k, TX>(X, w_in, B, conn, theta, w, gi, dtheta, dY_out, st);
     switch (up_k) {
-        case 1:
-            return launch_through<k, 1>(X, w_in, B, conn, theta, w, Y, up_conn, up_theta, up_w, up_dY, up_group,
-                                        up_off, up_edge, node, dtheta, dY_out, st);
-        case 2:
-            return launch_through<k, 2>(X, w_in, B, conn, theta, w, Y, up_conn, up_theta, up_w, up_dY, up_group,
-                                        up_off, up_edge, node, dtheta, dY_out, st);
-        default:
-            return launch_through<k, 3>(X, w_in, B, conn, theta, w, Y, up_conn, up_theta, up_w, up_dY, up_group,
-                                        up_off, up_edge, node, dtheta, dY_out, st);
+        case 1: return launch_src<k, 1, TX, kSrcThrough>(X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
+        case 2: return launch_src<k, 2, TX, kSrcThrough>(X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
+        default: return launch_src<k, 3, TX, kSrcThrough>(X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
     }
+}
+
+template <typename TX>
+int run_src(int src, int up_k, const TX* X, int w_in, long long B, const int* conn, const float* theta, int w,
+            int k, const GradIn& gi, int node, float* dtheta, float* dY_out, cudaStream_t st) {
+    switch (k) {
+        case 1: return launch_src_k<1, TX>(src, up_k, X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
+        case 2: return launch_src_k<2, TX>(src, up_k, X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
+        case 3: return launch_src_k<3, TX>(src, up_k, X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
+        case 4: return launch_src_k<4, TX>(src, up_k, X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
+        case 5: return launch_src_k<5, TX>(src, up_k, X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
+        default: return launch_src_k<6, TX>(src, up_k, X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
+    }
+}
+
+// Host checks shared by the entry points (before any CUDA call).
+int check_common(const void* X, int32_t w_in, int64_t B, const int32_t* conn, const float* theta, int32_t w,
+                 int32_t k, int32_t node, const float* dtheta) {
+    if (!conn || !theta || !dtheta) return BITLOGIC_ERR_NULL;
+    if (w_in <= 0 || w <= 0 || B < 0) return BITLOGIC_ERR_SHAPE;
+    if (k < 1 || k > 6 || k > w_in) return BITLOGIC_ERR_FANIN;
+    if ((int64_t)w * k > 0x7fffffffLL) return BITLOGIC_ERR_SHAPE;
+    if (node != BITLOGIC_NODE_SOFT && node != BITLOGIC_NODE_ST) return BITLOGIC_ERR_NODE;
+    if (B > 0 && !X) return BITLOGIC_ERR_NULL;
+    return BITLOGIC_OK;
 }
 
 }  // namespace
@@ -409,38 +785,89 @@ using namespace bitlogic;
 
 BITLOGIC_ERROR_READER(lut_through)
 
+// The through form for either input type.
+template <typename TX>
+static int backward_through(const TX* X, int32_t w_in, int64_t B, const int32_t* conn, const float* theta,
+                            int32_t w, int32_t k, int32_t node, const float* Y, const int32_t* up_conn,
+                            const float* up_theta, int32_t up_w, int32_t up_k, const float* up_dY, int32_t up_group,
+                            const int32_t* up_off, const int32_t* up_edge, float* dtheta, float* dY_out,
+                            cudaStream_t stream) {
+    int st = check_common(X, w_in, B, conn, theta, w, k, node, dtheta);
+    if (st) return st;
+    if (!up_conn || !up_theta || !up_off) return BITLOGIC_ERR_NULL;
+    if (up_w <= 0) return BITLOGIC_ERR_SHAPE;
+    if (up_k < 1 || up_k > 3 || up_k > w) return BITLOGIC_ERR_FANIN;
+    if ((int64_t)up_w * up_k > 0x7fffffffLL) return BITLOGIC_ERR_SHAPE;
+    if (up_group < 1 || up_group > up_w || up_w % up_group != 0) return BITLOGIC_ERR_SHAPE;
+    if (B == 0) {
+        if (cudaMemsetAsync(dtheta, 0, sizeof(float) * (size_t)w * ((size_t)1 << k), stream) != cudaSuccess)
+            return BITLOGIC_ERR_CUDA;
+        return BITLOGIC_OK;
+    }
+    if (!Y || !up_dY) return BITLOGIC_ERR_NULL;
+    if (B % 4 != 0 || !aligned16(X) || !aligned16(Y) || !aligned16(up_dY) || (dY_out && !aligned16(dY_out)))
+        return BITLOGIC_ERR_ALIGN;
+    GradIn gi{};
+    gi.off = up_off;
+    gi.edge = up_edge;
+    gi.Y = Y;
+    gi.up_conn = up_conn;
+    gi.up_theta = up_theta;
+    gi.up_w = up_w;
+    gi.up_dY = up_dY;
+    gi.up_group = up_group;
+    return run_src<TX>(kSrcThrough, up_k, X, w_in, B, conn, theta, w, k, gi, node, dtheta, dY_out, stream);
+}
+
 extern "C" int bitlogic_lut_backward_through(const float* X, int32_t w_in, int64_t B, const int32_t* conn,
                                              const float* theta, int32_t w, int32_t k, int32_t node,
                                              const float* Y, const int32_t* up_conn, const float* up_theta,
                                              int32_t up_w, int32_t up_k, const float* up_dY, int32_t up_group,
                                              const int32_t* up_off, const int32_t* up_edge, float* dtheta,
                                              float* dY_out, cudaStream_t stream) {
-    if (!conn || !theta || !up_conn || !up_theta || !up_off || !dtheta) return BITLOGIC_ERR_NULL;
-    if (w_in <= 0 || w <= 0 || B < 0 || up_w <= 0) return BITLOGIC_ERR_SHAPE;
-    if (k < 1 || k > 6 || k > w_in || up_k < 1 || up_k > 3 || up_k > w) return BITLOGIC_ERR_FANIN;
-    if ((int64_t)w * k > 0x7fffffffLL || (int64_t)up_w * up_k > 0x7fffffffLL) return BITLOGIC_ERR_SHAPE;
-    if (up_group < 1 || up_group > up_w || up_w % up_group != 0) return BITLOGIC_ERR_SHAPE;
-    if (node != BITLOGIC_NODE_SOFT && node != BITLOGIC_NODE_ST) return BITLOGIC_ERR_NODE;
+    return backward_through<float>(X, w_in, B, conn, theta, w, k, node, Y, up_conn, up_theta, up_w, up_k, up_dY,
+                                   up_group, up_off, up_edge, dtheta, dY_out, stream);
+}
+
+extern "C" int bitlogic_lut_backward_through_u8(const uint8_t* X, int32_t w_in, int64_t B, const int32_t* conn,
+                                                const float* theta, int32_t w, int32_t k, int32_t node,
+                                                const float* Y, const int32_t* up_conn, const float* up_theta,
+                                                int32_t up_w, int32_t up_k, const float* up_dY, int32_t up_group,
+                                                const int32_t* up_off, const int32_t* up_edge, float* dtheta,
+                                                float* dY_out, cudaStream_t stream) {
+    return backward_through<uint8_t>(X, w_in, B, conn, theta, w, k, node, Y, up_conn, up_theta, up_w, up_k, up_dY,
+                                     up_group, up_off, up_edge, dtheta, dY_out, stream);
+}
+
+extern "C" int bitlogic_lut_backward_u8(const uint8_t* X, int32_t w_in, int64_t B, const int32_t* conn,
+                                        const float* theta, int32_t w, int32_t k, int32_t node,
+                                        const float* dY, int32_t dy_group, const float* up_terms,
+                                        const int32_t* up_off, const int32_t* up_edge, int32_t up_edges,
+                                        float* dtheta, float* dY_out, cudaStream_t stream) {
+    int st = check_common(X, w_in, B, conn, theta, w, k, node, dtheta);
+    if (st) return st;
+    const bool terms = up_terms != nullptr;
+    if (B > 0 && terms == (dY != nullptr)) return BITLOGIC_ERR_NULL;   // exactly one source
+    if (terms) {
+        if (!up_off) return BITLOGIC_ERR_NULL;
+        if (up_edges < 0) return BITLOGIC_ERR_SHAPE;
+    } else if (dy_group < 1 || dy_group > w || w % dy_group != 0) {
+        return BITLOGIC_ERR_SHAPE;
+    }
     if (B == 0) {
         if (cudaMemsetAsync(dtheta, 0, sizeof(float) * (size_t)w * ((size_t)1 << k), stream) != cudaSuccess)
             return BITLOGIC_ERR_CUDA;
         return BITLOGIC_OK;
     }
-    if (!X || !Y || !up_dY) return BITLOGIC_ERR_NULL;
-    if (B % 4 != 0 || !aligned16(X) || !aligned16(Y) || !aligned16(up_dY) || (dY_out && !aligned16(dY_out)))
+    if (B % 4 != 0 || !aligned16(X) || !aligned16(terms ? up_terms : dY) || (dY_out && !aligned16(dY_out)))
         return BITLOGIC_ERR_ALIGN;
-    switch (k) {
-        case 1: return launch_through_k<1>(up_k, X, w_in, B, conn, theta, w, Y, up_conn, up_theta, up_w, up_dY,
-                                           up_group, up_off, up_edge, node, dtheta, dY_out, stream);
-        case 2: return launch_through_k<2>(up_k, X, w_in, B, conn, theta, w, Y, up_conn, up_theta, up_w, up_dY,
-                                           up_group, up_off, up_edge, node, dtheta, dY_out, stream);
-        case 3: return launch_through_k<3>(up_k, X, w_in, B, conn, theta, w, Y, up_conn, up_theta, up_w, up_dY,
-                                           up_group, up_off, up_edge, node, dtheta, dY_out, stream);
-        case 4: return launch_through_k<4>(up_k, X, w_in, B, conn, theta, w, Y, up_conn, up_theta, up_w, up_dY,
-                                           up_group, up_off, up_edge, node, dtheta, dY_out, stream);
-        case 5: return launch_through_k<5>(up_k, X, w_in, B, conn, theta, w, Y, up_conn, up_theta, up_w, up_dY,
-                                           up_group, up_off, up_edge, node, dtheta, dY_out, stream);
-        default: return launch_through_k<6>(up_k, X, w_in, B, conn, theta, w, Y, up_conn, up_theta, up_w, up_dY,
-                                            up_group, up_off, up_edge, node, dtheta, dY_out, stream);
-    }
+    GradIn gi{};
+    gi.dY = dY;
+    gi.group = dy_group;
+    gi.terms = up_terms;
+    gi.n_terms = up_edges;
+    gi.off = up_off;
+    gi.edge = up_edge;
+    return run_src<uint8_t>(terms ? kSrcTerms : kSrcRows, 1, X, w_in, B, conn, theta, w, k, gi, node, dtheta, dY_out,
+                            stream);
 }

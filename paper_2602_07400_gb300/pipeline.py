@@ -21,9 +21,10 @@ from . import (NODE_FORMS, bitlogic_adamw_update, bitlogic_binarize_tables, bitl
                bitlogic_csr_positions, bitlogic_csr_reduce, bitlogic_pixel_histogram, bitlogic_quantile_thresholds,
                bitlogic_encode_thermometer, bitlogic_hard_forward, bitlogic_head_loss_ex,
                bitlogic_head_loss_workspace, bitlogic_lut_backward_node, bitlogic_lut_backward_through,
-               bitlogic_lut_forward_node,
+               bitlogic_lut_backward_u8, bitlogic_lut_forward_node,
                bitlogic_pack_bits, bitlogic_route_backward, bitlogic_route_backward_u8, bitlogic_route_forward,
-               bitlogic_route_forward_u8, bitlogic_route_snap, bitlogic_encode_thermometer_u8)
+               bitlogic_route_forward_u8, bitlogic_route_snap, bitlogic_encode_thermometer_u8,
+               bitlogic_encode_thermometer_both)
 
 
 def _nomark(name: str) -> None:
@@ -172,14 +173,21 @@ class TrainStep:
     * otherwise a CSR reduction of the terms into ``dy1``, which the
       dtheta-only layer-1 backward reads.
 
-    Set ``keep_dy1`` to also write dY1 (e.g. to check it).  ``node`` picks the
+    On the first two routes the layer-1 backward can read the encoder's wires
+    as bytes (``bytes1``; the encoder then writes, in one pass, both the fp32
+    rows the forward reads and byte rows): the node gathers a quarter of the
+    data.  The results are the same bit for bit; at the CIFAR shapes on
+    GB300 the step was no faster (7.025 against 7.028 ms at the CIFAR-100
+    shape, 1.842 against 1.818 ms at the CIFAR-10 shape), so it is off by
+    default.  Set
+    ``keep_dy1`` to also write dY1 (e.g. to check it).  ``node`` picks the
     LightLUT form of both layers: "soft", or "st" (hard table samples in the
     forward, straight-through gradient to the logits)."""
 
     def __init__(self, net: Network, B: int, d: int, thresholds: Sequence[int], C: int,
                  tau: float, want_dx1: bool = False, keep_dy1: bool = False,
                  fuse_dy1: Optional[bool] = None, csr_order: bool = True, node: str = "soft",
-                 through: Optional[bool] = None, device="cuda"):
+                 through: Optional[bool] = None, bytes1: Optional[bool] = None, device="cuda"):
         dev = torch.device(device)
         if node not in NODE_FORMS:
             raise ValueError(f"node must be one of {sorted(NODE_FORMS)}")
@@ -205,6 +213,12 @@ class TrainStep:
         self.loss = torch.zeros(1, **f32)
         self.dyg = torch.empty(C, B, **f32)          # gradient row shared by each class's nodes
         self.fuse_dy1 = bool(fuse_dy1) and not self.through
+        if bytes1 is None:
+            bytes1 = False   # measured no faster on GB300 at the CIFAR shapes (see the class docstring)
+        if bytes1 and not (self.fuse_dy1 or self.through):
+            raise ValueError("byte wires for layer 1 need the fused or the through route")
+        self.bytes1 = bool(bytes1)
+        self.bits8 = torch.empty(net.w_in, B, dtype=torch.uint8, device=dev) if self.bytes1 else None
         # per-edge terms stored in CSR order (each input's terms contiguous,
         # read without the edge map) instead of edge order
         self.csr_order = bool(csr_order)
@@ -224,7 +238,10 @@ class TrainStep:
 
     def forward(self, stream=None, mark=_nomark):
         n = self.net
-        bitlogic_encode_thermometer(self.x, self.thr, self.bits, stream)
+        if self.bits8 is not None:
+            bitlogic_encode_thermometer_both(self.x, self.thr, self.bits, self.bits8, stream)
+        else:
+            bitlogic_encode_thermometer(self.x, self.thr, self.bits, stream)
         mark("encode")
         bitlogic_lut_forward_node(self.bits, n.conn1, n.theta1, self.y1, self.node, stream)
         mark("forward1")
@@ -245,8 +262,9 @@ class TrainStep:
             bitlogic_lut_backward_node(self.y1, n.conn2, n.theta2, self.dth2, nd, dY=self.dyg, dy_group=g,
                                        stream=stream)
             mark("backward2")
-            bitlogic_lut_backward_through(self.bits, n.conn1, n.theta1, self.dth1, self.y1, n.conn2, n.theta2,
-                                          self.dyg, g, n.off2, n.edge2, node=nd, dY_out=self.dy1, stream=stream)
+            bitlogic_lut_backward_through(self.bits8 if self.bytes1 else self.bits, n.conn1, n.theta1, self.dth1,
+                                          self.y1, n.conn2, n.theta2, self.dyg, g, n.off2, n.edge2, node=nd,
+                                          dY_out=self.dy1, stream=stream)
             mark("backward1")
             return
         bitlogic_lut_backward_node(self.y1, n.conn2, n.theta2, self.dth2, nd, dY=self.dyg,
@@ -255,7 +273,10 @@ class TrainStep:
         mark("backward2")
         pos1 = n.pos1 if (co and self.edges1 is not None) else None
         edge2 = None if co else n.edge2
-        if self.fuse_dy1:
+        if self.fuse_dy1 and self.bytes1:
+            bitlogic_lut_backward_u8(self.bits8, n.conn1, n.theta1, self.dth1, nd, up_terms=self.edges2,
+                                     up_off=n.off2, up_edge=edge2, dY_out=self.dy1, stream=stream)
+        elif self.fuse_dy1:
             bitlogic_lut_backward_node(self.bits, n.conn1, n.theta1, self.dth1, nd, up_terms=self.edges2,
                                        up_off=n.off2, up_edge=edge2, edge_terms=self.edges1,
                                        edge_pos=pos1, dY_out=self.dy1, stream=stream)

@@ -37,7 +37,14 @@ def test_encode_thermometer(B, d, b):
     thr = sorted(rng.choice(256, size=b, replace=False).tolist())
     bits = torch.full((d * b, B), -1.0, device="cuda")
     bl.bitlogic_encode_thermometer(dev(x), thr, bits)
-    check_exact(bits.cpu().numpy().astype(np.float64), oracle.encode_thermometer(x, thr), "bits")
+    want = oracle.encode_thermometer(x, thr)
+    check_exact(bits.cpu().numpy().astype(np.float64), want, "bits")
+    # both forms in one pass: the same wires as fp32 rows and as byte rows
+    bits2 = torch.full((d * b, B), -1.0, device="cuda")
+    bits8 = torch.full((d * b, B), 7, dtype=torch.uint8, device="cuda")
+    bl.bitlogic_encode_thermometer_both(dev(x), thr, bits2, bits8)
+    check_exact(bits2.cpu().numpy().astype(np.float64), want, "bits (both)")
+    check_exact(bits8.cpu().numpy().astype(np.float64), want, "bits8 (both)")
     no_device_error()
 
 
@@ -505,6 +512,68 @@ def test_lut_backward_through_identity_edge_map():
                                      dev(up_dY), 1, dev(off), None)
     wdth, _ = _through_oracle(X, conn, theta, Y, up_conn, up_theta, up_dY, 1, "soft")
     check_grad(dth, wdth, "dtheta")
+    no_device_error()
+
+
+BYTES = [(1, 10, 7, 4), (2, 50, 64, 128), (3, 40, 33, 260), (4, 100, 65, 1028), (5, 64, 40, 132),
+         (6, 300, 129, 1024), (6, 2000, 77, 516)]
+
+
+@pytest.mark.parametrize("node", ["soft", "st"])
+@pytest.mark.parametrize("k,w_in,w,B", BYTES)
+def test_lut_backward_u8_rows_and_terms(k, w_in, w, B, node):
+    # byte-row input (binary wires): dtheta from dY rows and from the next
+    # layer's per-edge terms, equal bit for bit to the fp32-row dtheta-only
+    # backward on the same wires (the terms summed by bitlogic_csr_reduce
+    # first), and within the parity tolerance of the oracle
+    Xb = synth.binary_activations(w_in, B, seed=k + 20)
+    X8 = dev(Xb.astype(np.uint8))
+    conn = synth.connectivity(w, k, w_in, seed=k + 21)
+    theta = synth.table_logits(w, 1 << k, seed=k + 22)
+    dY = synth.uniform_gradients(w, B, seed=k + 23, scale=1e-3)
+    ref = torch.empty(w, 1 << k, device="cuda")
+    bl.bitlogic_lut_backward_node(dev(Xb), dev(conn), dev(theta), ref, node, dY=dev(dY))
+    got = torch.full((w, 1 << k), np.nan, device="cuda")
+    out = torch.full((w, B), np.nan, device="cuda")
+    bl.bitlogic_lut_backward_u8(X8, dev(conn), dev(theta), got, node, dY=dev(dY), dY_out=out)
+    check_exact(got.cpu().numpy(), ref.cpu().numpy(), "dtheta (rows) vs fp32 rows")
+    check_exact(out.cpu().numpy(), dY, "dY_out (rows)")
+    wdth, _ = oracle.lut_backward(Xb, conn, theta, dY, want_dx=False, node=node)
+    check_grad(got, wdth, "dtheta (rows) vs oracle")
+    # per-edge terms of a next layer (fan-in 3 over these w rows), in CSR order
+    up_w = max(4, w // 2)
+    up_conn = synth.connectivity(up_w, 3, w, seed=k + 24)
+    off, edge = bl.bitlogic_build_csr(up_conn, w)
+    terms = synth.uniform_gradients(up_w * 3, B, seed=k + 25, scale=1e-3)
+    summed = torch.empty(w, B, device="cuda")
+    bl.bitlogic_csr_reduce(dev(terms), dev(off), dev(edge), summed)
+    ref2 = torch.empty(w, 1 << k, device="cuda")
+    bl.bitlogic_lut_backward_node(dev(Xb), dev(conn), dev(theta), ref2, node, dY=summed)
+    got2 = torch.full((w, 1 << k), np.nan, device="cuda")
+    out2 = torch.full((w, B), np.nan, device="cuda")
+    bl.bitlogic_lut_backward_u8(X8, dev(conn), dev(theta), got2, node, up_terms=dev(terms), up_off=dev(off),
+                                up_edge=dev(edge), dY_out=out2)
+    check_exact(out2.cpu().numpy(), summed.cpu().numpy(), "dY_out (terms) vs CSR reduction")
+    check_exact(got2.cpu().numpy(), ref2.cpu().numpy(), "dtheta (terms) vs fp32 rows")
+    no_device_error()
+
+
+def test_lut_backward_through_u8_equals_fp32():
+    k, ku, w_in, w, up_w, up_group, B = 6, 2, 300, 200, 150, 5, 260
+    Xb = synth.binary_activations(w_in, B, seed=1)
+    conn = synth.connectivity(w, k, w_in, seed=2)
+    theta = synth.table_logits(w, 1 << k, seed=3)
+    Y = synth.uniform_activations(w, B, seed=4)
+    up_conn = synth.connectivity(up_w, ku, w, seed=5)
+    up_theta = synth.table_logits(up_w, 1 << ku, seed=6)
+    up_dY = synth.uniform_gradients(up_w // up_group, B, seed=7, scale=1e-3)
+    off, edge = bl.bitlogic_build_csr(up_conn, w)
+    a = torch.empty(w, 1 << k, device="cuda")
+    b = torch.empty(w, 1 << k, device="cuda")
+    args = (dev(Y), dev(up_conn), dev(up_theta), dev(up_dY), up_group, dev(off), dev(edge))
+    bl.bitlogic_lut_backward_through(dev(Xb), dev(conn), dev(theta), a, *args)
+    bl.bitlogic_lut_backward_through_u8(dev(Xb.astype(np.uint8)), dev(conn), dev(theta), b, *args)
+    check_exact(b.cpu().numpy(), a.cpu().numpy(), "through dtheta, byte rows vs fp32 rows")
     no_device_error()
 
 

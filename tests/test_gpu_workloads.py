@@ -32,14 +32,16 @@ pytestmark = pytest.mark.gpu
 oracle.set_threads(os.cpu_count() or 1)
 
 
-def _step(wl, want_dx1, seed=0, k=None, keep_dy1=True, fuse_dy1=None, csr_order=True, node="soft", through=None):
+def _step(wl, want_dx1, seed=0, k=None, keep_dy1=True, fuse_dy1=None, csr_order=True, node="soft", through=None,
+          bytes1=None):
     if k is not None:
         wl = synth.Workload(wl.name, wl.batch, wl.d, wl.classes, wl.sigma, wl.thresholds, wl.widths, k, wl.tau)
     conn1, th1, conn2, th2 = synth.network(wl, seed)
     x, labels = synth.blob_batch(wl.batch, wl.d, wl.classes, wl.sigma, seed=seed + 7)
     net = Network(conn1, th1, conn2, th2, wl.w_in)
     st = TrainStep(net, wl.batch, wl.d, wl.thresholds, wl.classes, wl.tau, want_dx1=want_dx1,
-                   keep_dy1=keep_dy1, fuse_dy1=fuse_dy1, csr_order=csr_order, node=node, through=through)
+                   keep_dy1=keep_dy1, fuse_dy1=fuse_dy1, csr_order=csr_order, node=node, through=through,
+                   bytes1=bytes1)
     st.load(x.cuda(), labels.cuda())
     st.run()
     torch.cuda.synchronize()
@@ -122,6 +124,24 @@ def test_mnist_k2_step_st_through():
     wl, st, x, labels, params = _step(synth.WORKLOADS["mnist"], want_dx1=False, k=2, node="st")
     assert st.through
     _full_compare(wl, st, x, labels, params, False, node="st")
+
+
+@pytest.mark.parametrize("k", [6, 2])
+def test_byte_wires_for_layer1_match_fp32_wires(k):
+    # the layer-1 backward reading the encoder's wires as bytes (the default
+    # of the fused and through routes) gives the fp32-row result bit for bit:
+    # k = 6, the byte-row kernel summing layer 2's terms itself against the
+    # CSR reduction followed by the fp32 dtheta-only kernel; k = 2, the
+    # through route on byte rows against fp32 rows
+    if k == 6:
+        _, a, *_ = _step(synth.WORKLOADS["mnist"], want_dx1=False, k=k, fuse_dy1=True, bytes1=True)
+        _, b, *_ = _step(synth.WORKLOADS["mnist"], want_dx1=False, k=k, fuse_dy1=False)
+    else:
+        _, a, *_ = _step(synth.WORKLOADS["mnist"], want_dx1=False, k=k, bytes1=True)
+        _, b, *_ = _step(synth.WORKLOADS["mnist"], want_dx1=False, k=k, bytes1=False)
+    assert a.bytes1 and not b.bytes1
+    for name in ("dy1", "dth1", "dth2", "loss"):
+        check_exact(getattr(a, name).cpu().numpy(), getattr(b, name).cpu().numpy(), name)
 
 
 def test_mnist_step_fused_layer1_gradient():
