@@ -329,29 +329,41 @@ def call_work(wl, B, fuse_dy1=False, through=False, bytes1=False):
 # later change of the code reports null.
 TRAFFIC = {
     ("mnist", "backward2"): {
-        "bytes": 59.670016e6 + 147.641856e6, "source": "lut_soft.cu",
-        "sha256": "180fc79502da4e837de466268e4dd9af96f7da65e286f6b8dce737f118e99f43",
-        "note": "ncu capture of this workload"},
+        "bytes": 59560448 + 144350720, "source": "lut_soft.cu",
+        "sha256": "78edac247d6c64dc0042c15287b5174dfc03ecac6e7945ec4beb26e9e6cc6800",
+        "note": "ncu capture of this workload (one-pass DRAM metrics)"},
+    ("cifar10", "forward1"): {
+        "bytes": 511101952 + 243450624, "source": "lut_soft.cu",
+        "sha256": "78edac247d6c64dc0042c15287b5174dfc03ecac6e7945ec4beb26e9e6cc6800",
+        "note": "ncu capture of this workload (one-pass DRAM metrics)"},
     ("cifar10", "forward2"): {
-        "bytes": 1.163448e9 + 0.248158464e9, "source": "lut_soft.cu",
-        "sha256": "180fc79502da4e837de466268e4dd9af96f7da65e286f6b8dce737f118e99f43",
-        "note": "ncu capture of this workload"},
+        "bytes": 1162980096 + 245190144, "source": "lut_soft.cu",
+        "sha256": "78edac247d6c64dc0042c15287b5174dfc03ecac6e7945ec4beb26e9e6cc6800",
+        "note": "ncu capture of this workload (one-pass DRAM metrics)"},
     ("cifar10", "backward2"): {
-        "bytes": 1.344971e9 + 1.545406e9, "source": "lut_soft.cu",
-        "sha256": "180fc79502da4e837de466268e4dd9af96f7da65e286f6b8dce737f118e99f43",
-        "note": "ncu capture of this workload"},
+        "bytes": 1344603136 + 1542144768, "source": "lut_soft.cu",
+        "sha256": "78edac247d6c64dc0042c15287b5174dfc03ecac6e7945ec4beb26e9e6cc6800",
+        "note": "ncu capture of this workload (one-pass DRAM metrics)"},
+    ("cifar10", "backward1"): {
+        "bytes": 2504033536 + 15722496, "source": "lut_soft.cu",
+        "sha256": "78edac247d6c64dc0042c15287b5174dfc03ecac6e7945ec4beb26e9e6cc6800",
+        "note": "ncu capture of this workload (one-pass DRAM metrics; layer 1 summing layer 2's terms)"},
     ("cifar100", "forward1"): {
-        "bytes": 5106130432 + 1034886144, "source": "lut_soft.cu",
-        "sha256": "180fc79502da4e837de466268e4dd9af96f7da65e286f6b8dce737f118e99f43",
+        "bytes": 5106467072 + 1034765312, "source": "lut_soft.cu",
+        "sha256": "78edac247d6c64dc0042c15287b5174dfc03ecac6e7945ec4beb26e9e6cc6800",
         "note": "ncu capture of this workload (one-pass DRAM metrics)"},
     ("cifar100", "forward2"): {
-        "bytes": 5877215232 + 1032726272, "source": "lut_soft.cu",
-        "sha256": "180fc79502da4e837de466268e4dd9af96f7da65e286f6b8dce737f118e99f43",
+        "bytes": 5876089344 + 1032741376, "source": "lut_soft.cu",
+        "sha256": "78edac247d6c64dc0042c15287b5174dfc03ecac6e7945ec4beb26e9e6cc6800",
         "note": "ncu capture of this workload (one-pass DRAM metrics)"},
     ("cifar100", "backward2"): {
-        "bytes": 6069030400 + 6277533952, "source": "lut_soft.cu",
-        "sha256": "180fc79502da4e837de466268e4dd9af96f7da65e286f6b8dce737f118e99f43",
+        "bytes": 6068320768 + 6277417984, "source": "lut_soft.cu",
+        "sha256": "78edac247d6c64dc0042c15287b5174dfc03ecac6e7945ec4beb26e9e6cc6800",
         "note": "ncu capture of this workload (one-pass DRAM metrics)"},
+    ("cifar100", "backward1"): {
+        "bytes": 11884503296 + 32632576, "source": "lut_soft.cu",
+        "sha256": "78edac247d6c64dc0042c15287b5174dfc03ecac6e7945ec4beb26e9e6cc6800",
+        "note": "ncu capture of this workload (one-pass DRAM metrics; layer 1 summing layer 2's terms)"},
     ("hard_cifar10", "hard1"): {
         "bytes": 16 * (1.209681e9 + 2.054784e9), "source": "hard.cu",
         "sha256": "f9bed6fc20215df71b5e12eebae1c94762286b3c7b941dea9a2ff948bfb9ed3c",

@@ -28,7 +28,10 @@ namespace bitlogic {
 namespace {
 
 #ifndef BITLOGIC_BWD_MIN_BLOCKS
-#define BITLOGIC_BWD_MIN_BLOCKS 16  // dtheta-only kernel: blocks per SM
+#define BITLOGIC_BWD_MIN_BLOCKS 16  // dtheta-only kernel: blocks per SM (k >= 4)
+#endif
+#ifndef BITLOGIC_BWD_MIN_BLOCKS_SMALL
+#define BITLOGIC_BWD_MIN_BLOCKS_SMALL 24  // dtheta-only kernel: blocks per SM (k <= 3, fewer registers)
 #endif
 #ifndef BITLOGIC_NODE_MIN_BLOCKS
 #define BITLOGIC_NODE_MIN_BLOCKS 12  // backward with input gradient: blocks per SM
@@ -850,7 +853,12 @@ __device__ __forceinline__ void warp_reduce_scatter(float (&v)[M], int lane) {
 }
 
 template <int k>
-__global__ void __launch_bounds__(kThetaWarps * 32, BITLOGIC_BWD_MIN_BLOCKS)
+__host__ __device__ constexpr int theta_min_blocks() {
+    return k <= 3 ? BITLOGIC_BWD_MIN_BLOCKS_SMALL : BITLOGIC_BWD_MIN_BLOCKS;
+}
+
+template <int k>
+__global__ void __launch_bounds__(kThetaWarps * 32, theta_min_blocks<k>())
 lut_backward_theta_kernel(const float* __restrict__ X, int w_in, long long B,
                           const int* __restrict__ conn, const float* __restrict__ theta, int w,
                           const float* __restrict__ dY, int group, float* __restrict__ dtheta,
@@ -1112,7 +1120,7 @@ int launch_backward(const float* X, int w_in, long long B, const int* conn, cons
             return BITLOGIC_ERR_CUDA;
         // one wave of persistent warps filling every SM alike (nodes dealt
         // round-robin, so warps differ by at most one node)
-        const long long resident = (long long)sm_count() * BITLOGIC_BWD_MIN_BLOCKS * kThetaWarps;
+        const long long resident = (long long)sm_count() * theta_min_blocks<k>() * kThetaWarps;
         const long long warps = w < resident ? w : resident;
         kern<<<(unsigned)((warps + kThetaWarps - 1) / kThetaWarps), kThetaWarps * 32, smem, st>>>(
             X, w_in, B, conn, theta, w, gs.dY, gs.group, dtheta, dY_out);
