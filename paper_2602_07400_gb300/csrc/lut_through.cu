@@ -225,26 +225,22 @@ struct GradIn {
 
 // Stages whose output gradient is formed together (registers: four float4
 // per stage of the chunk, besides the 2^k accumulators).
-#ifndef BITLOGIC_TERMS_CHUNK
-#define BITLOGIC_TERMS_CHUNK 2      // stages per chunk, k >= 5, rows and terms sources
+#ifndef BITLOGIC_ROWS_CHUNK
+#define BITLOGIC_ROWS_CHUNK 2       // stages per chunk, k >= 5, rows source
 #endif
-#ifndef BITLOGIC_TERMS_ROWS
-#define BITLOGIC_TERMS_ROWS 2       // term rows whose loads are in flight together
+#ifndef BITLOGIC_ROWS_BLOCKS
+#define BITLOGIC_ROWS_BLOCKS 12     // one-warp blocks per SM, k = 6, rows source
 #endif
-#ifndef BITLOGIC_TERMS_BLOCKS
-#define BITLOGIC_TERMS_BLOCKS 12    // one-warp blocks per SM, k = 6, rows and terms sources
-#endif
-static_assert(BITLOGIC_TERMS_ROWS == 1 || BITLOGIC_TERMS_ROWS == 2 || BITLOGIC_TERMS_ROWS == 4, "rows in flight");
 template <int k, int SRC>
 __host__ __device__ constexpr int grad_chunk() {
     if constexpr (SRC == kSrcThrough) return k <= 3 ? BITLOGIC_THROUGH_CHUNK : (k == 4 ? 4 : (k == 5 ? 2 : 1));
-    else return k <= 4 ? 4 : BITLOGIC_TERMS_CHUNK;
+    else return k <= 4 ? 4 : BITLOGIC_ROWS_CHUNK;
 }
 // one-warp blocks per SM: fewer for the widest tables (their accumulators
 // and the loads in flight take more registers)
 template <int k, int SRC>
 __host__ __device__ constexpr int grad_min_blocks() {
-    return (k >= 6 && SRC != kSrcThrough) ? BITLOGIC_TERMS_BLOCKS : kTMinBlocks;
+    return (k >= 6 && SRC != kSrcThrough) ? BITLOGIC_ROWS_BLOCKS : kTMinBlocks;
 }
 
 template <typename TX>
@@ -284,7 +280,8 @@ lut_theta_src_kernel(const TX* __restrict__ X, int w_in, long long B, const int*
     const int G = gridDim.x;
     const int jfirst = blockIdx.x;
     const int nst = (int)((B + CH - 1) / CH);
-    const int n_up = SRC == kSrcThrough ? gi.up_w * ku : gi.n_terms;   // CSR positions
+    static_assert(SRC == kSrcRows || SRC == kSrcThrough, "the terms source has its own kernel");
+    const int n_up = SRC == kSrcThrough ? gi.up_w * ku : 0;   // CSR positions
 
     // issue stream: stage si of node ji, kTStages - 1 stages ahead of the
     // compute stream; rows of the warp's node after ji are loaded ahead
@@ -344,28 +341,15 @@ lut_theta_src_kernel(const TX* __restrict__ X, int w_in, long long B, const int*
             }
             deg = e1 - e0;
         }
-        // per lane one upstream edge: a term row id (terms) or a consumer
-        // (through), for the positions e0 .. e0 + 31
-        int my_id = -1;
+        // per lane one consumer (through), for the positions e0 .. e0 + 31
         Consumer<ku> mine;
         mine.grow = -1;
         auto load_edges = [&](int c0) {
             bool bad = false;
-            my_id = -1;
             mine.grow = -1;
-            if (c0 + lane < deg) {
-                if constexpr (SRC == kSrcTerms) {
-                    const int p = e0 + c0 + lane;
-                    my_id = gi.edge ? __ldg(gi.edge + p) : p;
-                    if ((unsigned)my_id >= (unsigned)gi.n_terms) {
-                        bad = true;
-                        my_id = -1;
-                    }
-                } else if constexpr (SRC == kSrcThrough) {
-                    mine = load_consumer<ku>(e0 + c0 + lane, gi.edge, n_up, gi.up_conn, gi.up_theta,
-                                             gi.up_group, w, node, bad);
-                }
-            }
+            if (c0 + lane < deg)
+                mine = load_consumer<ku>(e0 + c0 + lane, gi.edge, n_up, gi.up_conn, gi.up_theta, gi.up_group, w,
+                                         node, bad);
             if (__any_sync(0xffffffffu, bad) && lane == 0) flag_index_error();
         };
         if constexpr (SRC != kSrcRows) load_edges(0);
@@ -391,37 +375,7 @@ lut_theta_src_kernel(const TX* __restrict__ X, int w_in, long long B, const int*
                 for (int c0 = 0; c0 < deg; c0 += 32) {
                     if (c0 > 0) load_edges(c0);   // more than 32 upstream edges: this chunk's
                     const int n = min(32, deg - c0);
-                    if constexpr (SRC == kSrcTerms) {
-                        // term rows in increasing CSR position, kRows rows' loads in flight
-                        constexpr int kRows = BITLOGIC_TERMS_ROWS;
-#pragma unroll 1
-                        for (int e = 0; e < n; e += kRows) {
-                            int id[kRows];
-#pragma unroll
-                            for (int u = 0; u < kRows; ++u) {
-                                id[u] = __shfl_sync(0xffffffffu, my_id, (e + u) & 31);
-                                if (e + u >= n) id[u] = -1;
-                            }
-                            float4 v[kRows][kTChunk];
-#pragma unroll
-                            for (int u = 0; u < kRows; ++u)
-#pragma unroll
-                                for (int t = 0; t < kTChunk; ++t) {
-                                    const long long s4 = (long long)(sc0 + t) * CH + 4 * lane;
-                                    v[u][t] = (s4 < B && id[u] >= 0) ? ldg4t(gi.terms + (long long)id[u] * B + s4)
-                                                                     : make_float4(0.f, 0.f, 0.f, 0.f);
-                                }
-#pragma unroll
-                            for (int u = 0; u < kRows; ++u)
-#pragma unroll
-                                for (int t = 0; t < kTChunk; ++t) {
-                                    if (e + u < n) {
-                                        gv[t].x += v[u][t].x; gv[t].y += v[u][t].y;
-                                        gv[t].z += v[u][t].z; gv[t].w += v[u][t].w;
-                                    }
-                                }
-                        }
-                    } else {
+                    {
                         // consumers in increasing CSR position: each consumer's rows
                         // for all the chunk's stages at once
 #pragma unroll 1
@@ -745,6 +699,7 @@ template <int k, typename TX>
 int launch_src_k(int src, int up_k, const TX* X, int w_in, long long B, const int* conn, const float* theta, int w,
                  const GradIn& gi, int node, float* dtheta, float* dY_out, cudaStream_t st) {
     if (src == kSrcRows) return launch_src<k, 1, TX, kSrcRows>(X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
+    // the terms source streams its rows through the ring kernel
     if (src == kSrcTerms) return launch_terms_ring<k, TX>(X, w_in, B, conn, theta, w, gi, dtheta, dY_out, st);
     switch (up_k) {
         case 1: return launch_src<k, 1, TX, kSrcThrough>(X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);

@@ -558,6 +558,41 @@ def test_lut_backward_u8_rows_and_terms(k, w_in, w, B, node):
     no_device_error()
 
 
+@pytest.mark.parametrize("k", [2, 6])
+def test_lut_backward_u8_terms_with_many_and_no_consumers(k):
+    # the term rows of a node beyond the ones its ring slot holds (ten), and
+    # beyond 32 (read in chunks), and nodes with no consumers: the same sum
+    # as the CSR reduction, bit for bit, and the same dtheta as the fp32
+    # dtheta-only kernel on it
+    w_in, w, up_w, B = 50, 40, 300, 260
+    rng = np.random.default_rng(7)
+    up_conn = np.stack([rng.choice([0, 1, 2, 3, 5, 8, 13], size=2, replace=False)
+                        for _ in range(up_w)]).astype(np.int32)
+    up_conn[:12] = np.arange(14, 38, dtype=np.int32).reshape(12, 2)   # 24 rows with one consumer
+    up_conn[12:41] = [9, 10]                                            # two rows with 29
+    off, edge = bl.bitlogic_build_csr(up_conn, w)
+    deg = np.diff(off)
+    assert (deg > 32).any() and ((deg > 10) & (deg <= 32)).any() and (deg == 0).any() and (deg == 1).any()
+    Xb = synth.binary_activations(w_in, B, seed=k + 30)
+    conn = synth.connectivity(w, k, w_in, seed=k + 31)
+    theta = synth.table_logits(w, 1 << k, seed=k + 32)
+    terms = synth.uniform_gradients(up_w * 2, B, seed=k + 33, scale=1e-3)
+    summed = torch.empty(w, B, device="cuda")
+    bl.bitlogic_csr_reduce(dev(terms), dev(off), dev(edge), summed)
+    ref = torch.empty(w, 1 << k, device="cuda")
+    bl.bitlogic_lut_backward_node(dev(Xb), dev(conn), dev(theta), ref, dY=summed)
+    got = torch.full((w, 1 << k), np.nan, device="cuda")
+    out = torch.full((w, B), np.nan, device="cuda")
+    bl.bitlogic_lut_backward_u8(dev(Xb.astype(np.uint8)), dev(conn), dev(theta), got, up_terms=dev(terms),
+                                up_off=dev(off), up_edge=dev(edge), dY_out=out)
+    check_exact(out.cpu().numpy(), summed.cpu().numpy(), "dY_out vs CSR reduction")
+    check_exact(got.cpu().numpy(), ref.cpu().numpy(), "dtheta vs fp32 rows")
+    wdth, _ = oracle.lut_backward(Xb, conn, theta, summed.cpu().numpy().astype(np.float64), want_dx=False)
+    check_grad(got, wdth, "dtheta vs oracle")
+    assert torch.all(out[torch.from_numpy(np.nonzero(deg == 0)[0]).cuda()] == 0)
+    no_device_error()
+
+
 def test_lut_backward_through_u8_equals_fp32():
     k, ku, w_in, w, up_w, up_group, B = 6, 2, 300, 200, 150, 5, 260
     Xb = synth.binary_activations(w_in, B, seed=1)
