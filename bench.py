@@ -570,6 +570,21 @@ class Timer:
             totals.append(tot)
         return {n: float(np.mean(v)) for n, v in calls.items()}, float(np.mean(totals))
 
+    def event_floor(self, n=30):
+        """ms the eager split reports for a near-empty kernel (the issue
+        probe with one iteration: one block of 1024 threads per SM) placed
+        where a step's first call sits: the launch and event overhead that
+        every entry of the split carries."""
+        import paper_2602_07400_gb300 as bl
+        if not hasattr(self, "_floor_sink"):
+            self._floor_sink = torch.empty(bl.bitlogic_issue_probe_threads(), dtype=torch.int32, device="cuda")
+
+        def step(mark):
+            bl.bitlogic_issue_probe("ffma", 1, self._floor_sink)
+            mark("empty")
+        per_call, _ = self.eager_split(step, n)
+        return per_call["empty"]
+
 
 def build_train(wl, rank, node="soft", fuse_dy1=None, through=None, bytes1=None):
     from paper_2602_07400_gb300.pipeline import Network, RoutedNetwork, RoutedTrainStep, TrainStep
@@ -620,6 +635,7 @@ def measure_train(wl, st, args, timer, hbm, sm_max, peak_kind, sms, world, detai
         "eager_ms_per_step": eager_step,
         "roofline": roofline_of(dom, work, per_call, sms, clocks, wl.name, hbm, sm_max, peak_kind),
         "calls": calls_table(work, per_call, hbm, wl.name),
+        "calls_event_floor_ms": timer.event_floor(),
         "step_hbm": step_hbm_fraction(wl, B, work, per_call.keys(), tot / K, hbm) if not wl.Kc else None,
         "gpu_launches": K * st.kernels_per_run,
         "clocks": clocks, "wall_s_timed_loop": wall,
@@ -870,6 +886,7 @@ def run_headline(args):
         "timing": train["timing"],
         "eager_ms_per_step": train["eager_ms_per_step"],
         "calls": train["calls"],
+        "calls_event_floor_ms": train["calls_event_floor_ms"],
         "roofline_by_call": train["roofline_by_call"],
         "step_hbm": train["step_hbm"],
         "wall_s_timed_loop": train["wall_s_timed_loop"],
@@ -955,6 +972,7 @@ def run_single(args):
     })
     if train:
         out.update({"timing": train["timing"], "eager_ms_per_step": train["eager_ms_per_step"],
+                    "calls_event_floor_ms": train["calls_event_floor_ms"],
                     "roofline_by_call": train["roofline_by_call"], "step_hbm": train["step_hbm"],
                     "wall_s_timed_loop": train["wall_s_timed_loop"]})
     if wl.name in PAPER_CONTEXT:

@@ -76,6 +76,44 @@ __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commi
 template <int N>
 __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
 
+// Programmatic dependent launch (sm_90 and later).  A kernel launched with
+// launch_dependent() may start while the kernel before it on the stream is
+// still finishing: it runs grid_dependency_wait() before its first access to
+// memory that the earlier work writes or reads, and the wait returns once that
+// work has completed with its writes visible.  The earlier kernel lets its
+// dependent start early with allow_dependent_launch() (else the dependent
+// starts as its blocks exit).  When the previous operation on the stream is
+// not a kernel, the launch is an ordinary one and the wait returns at once.
+__device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;\n" ::: "memory"); }
+__device__ __forceinline__ void allow_dependent_launch() {
+    asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+}
+
+// First statement of every kernel launched with launch_dependent(): wait for
+// the work before it on the stream, then let the next kernel be scheduled.
+// Waiting before triggering makes the chain transitive: once a kernel's wait
+// returns, everything before its predecessor has completed too.
+__device__ __forceinline__ void dependent_kernel_start() {
+    grid_dependency_wait();
+    allow_dependent_launch();
+}
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_dependent(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                                    cudaStream_t stream, Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
 }  // namespace bitlogic
 
 #define BITLOGIC_ERROR_READER(name)                                            \

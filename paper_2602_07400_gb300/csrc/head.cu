@@ -9,8 +9,9 @@
 // Two short kernels (three when the per-node dY is requested): group sums
 // (lanes over samples, warps over the rows of a group), per-sample softmax
 // (one warp per sample) whose last block to finish also takes the batch mean,
-// and the broadcast of dlogit/tau over each group's rows.  Every reduction
-// runs in a fixed order.
+// and the broadcast of dlogit/tau over each group's rows.  Each kernel after
+// the first is a programmatic dependent launch, so it is scheduled while the
+// one before it drains.  Every reduction runs in a fixed order.
 #include <cfloat>
 #include <mutex>
 #include <vector>
@@ -29,6 +30,7 @@ head_group_sum_kernel(const float* __restrict__ Y, long long B, int C, int g, fl
                       float* __restrict__ logits, unsigned int* __restrict__ done) {
     __shared__ float part[kSumWarps][32];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    dependent_kernel_start();
     if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) *done = 0u;   // the softmax's block count
     const int c = blockIdx.x;
     const long long s = (long long)blockIdx.y * 32 + lane;
@@ -55,7 +57,10 @@ head_group_sum_kernel(const float* __restrict__ Y, long long B, int C, int g, fl
 // 32 warps' partial sums of sample t in order.  With one split the block
 // writes the logits; with several (so that enough blocks pull from HBM) it
 // writes the split's sum, and the softmax kernel adds the splits in order.
-constexpr int kSumVecWarps = 32;
+#ifndef BITLOGIC_SUM_VEC_WARPS
+#define BITLOGIC_SUM_VEC_WARPS 16
+#endif
+constexpr int kSumVecWarps = BITLOGIC_SUM_VEC_WARPS;
 constexpr int kMaxRowSplits = 4;
 
 __global__ void __launch_bounds__(kSumVecWarps * 32)
@@ -64,6 +69,7 @@ head_group_sum_vec_kernel(const float* __restrict__ Y, long long B, int C, int g
                           int rows_per_split, unsigned int* __restrict__ done) {
     __shared__ __align__(16) float part[kSumVecWarps][128];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    dependent_kernel_start();
     if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) *done = 0u;   // the softmax's block count
     const int c = blockIdx.x / splits, rs = blockIdx.x - c * splits;
     const int r0 = rs * rows_per_split, r1 = min(g, r0 + rows_per_split);
@@ -107,12 +113,15 @@ __device__ __forceinline__ float warp_sum(float v) {
 }
 
 constexpr int kSoftWarps = 8;
+constexpr int kSoftRegs = 4;   // classes per lane held in registers (C <= 128)
 
 // One warp per sample.  The block adds its samples' losses in warp order and
 // publishes the sum in block_sums; the last block to finish (a device-wide
 // count in `done`, zeroed by the group-sum kernel that runs before) adds the
 // blocks' sums in index order and writes the batch mean: one pass, no
-// separate reduction launch, and a fixed summation order.
+// separate reduction launch, and a fixed summation order.  Up to 128 classes
+// a lane keeps its classes' logits (c = lane + 32 j) in registers; wider heads
+// read them back from memory.  Data of the group-sum kernel is read past L1.
 __global__ void __launch_bounds__(kSoftWarps * 32)
 head_softmax_kernel(float* __restrict__ logits, long long B, int C,
                     const int* __restrict__ labels, float* __restrict__ dlogit,
@@ -123,36 +132,82 @@ head_softmax_kernel(float* __restrict__ logits, long long B, int C,
     __shared__ float red[kSoftWarps * 32];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const long long s = (long long)blockIdx.x * kSoftWarps + warp;
+    dependent_kernel_start();
     float li = 0.f;
     if (s < B) {
-        if (split_sums) {   // logits from the row splits' sums, added in split order
-            for (int c = lane; c < C; c += 32) {
-                float t = 0.f;
-                for (int rs = 0; rs < splits; ++rs) t += __ldg(split_sums + ((long long)rs * B + s) * C + c);
-                logits[s * C + c] = t / tau;
-            }
-            __syncwarp();
-        }
-        const float* l = logits + s * C;
-        float m = -FLT_MAX;
-        for (int c = lane; c < C; c += 32) m = fmaxf(m, l[c]);
-        m = warp_max(m);
-        float z = 0.f;
-        for (int c = lane; c < C; c += 32) z += expf(l[c] - m);
-        z = warp_sum(z);
-        const float lse = m + logf(z);
         int lab = __ldg(labels + s);
         if (lab < 0 || lab >= C) {
             if (lane == 0) flag_index_error();
             lab = 0;
         }
-        li = lse - l[lab];
         const float invB = 1.0f / (float)B;
-        for (int c = lane; c < C; c += 32) {
-            const float p = expf(l[c] - lse);
-            const float dl = (p - (c == lab ? 1.0f : 0.0f)) * invB;
-            dlogit[s * C + c] = dl;
-            if (dYg) dYg[(long long)c * B + s] = dl / tau;   // the gradient of every node of class c
+        float* l = logits + s * C;
+        if (C <= 32 * kSoftRegs) {
+            float v[kSoftRegs];
+#pragma unroll
+            for (int q = 0; q < kSoftRegs; ++q) {
+                const int c = lane + 32 * q;
+                v[q] = -FLT_MAX;
+                if (c < C) {
+                    if (split_sums) {   // logits from the row splits' sums, added in split order
+                        float t = 0.f;
+                        for (int rs = 0; rs < splits; ++rs) t += __ldcg(split_sums + ((long long)rs * B + s) * C + c);
+                        v[q] = t / tau;
+                        l[c] = v[q];
+                    } else {
+                        v[q] = __ldcg(l + c);
+                    }
+                }
+            }
+            float m = -FLT_MAX;
+#pragma unroll
+            for (int q = 0; q < kSoftRegs; ++q)
+                if (lane + 32 * q < C) m = fmaxf(m, v[q]);
+            m = warp_max(m);
+            float z = 0.f;
+#pragma unroll
+            for (int q = 0; q < kSoftRegs; ++q)
+                if (lane + 32 * q < C) z += expf(v[q] - m);
+            z = warp_sum(z);
+            const float lse = m + logf(z);
+            float vl = 0.f;
+#pragma unroll
+            for (int q = 0; q < kSoftRegs; ++q)
+                if (q == (lab >> 5)) vl = v[q];
+            li = lse - __shfl_sync(0xffffffffu, vl, lab & 31);
+#pragma unroll
+            for (int q = 0; q < kSoftRegs; ++q) {
+                const int c = lane + 32 * q;
+                if (c < C) {
+                    const float p = expf(v[q] - lse);
+                    const float dl = (p - (c == lab ? 1.0f : 0.0f)) * invB;
+                    dlogit[s * C + c] = dl;
+                    if (dYg) dYg[(long long)c * B + s] = dl / tau;   // the gradient of every node of class c
+                }
+            }
+        } else {
+            if (split_sums) {
+                for (int c = lane; c < C; c += 32) {
+                    float t = 0.f;
+                    for (int rs = 0; rs < splits; ++rs) t += __ldcg(split_sums + ((long long)rs * B + s) * C + c);
+                    l[c] = t / tau;
+                }
+                __syncwarp();
+            }
+            float m = -FLT_MAX;
+            for (int c = lane; c < C; c += 32) m = fmaxf(m, __ldcg(l + c));
+            m = warp_max(m);
+            float z = 0.f;
+            for (int c = lane; c < C; c += 32) z += expf(__ldcg(l + c) - m);
+            z = warp_sum(z);
+            const float lse = m + logf(z);
+            li = lse - __ldcg(l + lab);
+            for (int c = lane; c < C; c += 32) {
+                const float p = expf(__ldcg(l + c) - lse);
+                const float dl = (p - (c == lab ? 1.0f : 0.0f)) * invB;
+                dlogit[s * C + c] = dl;
+                if (dYg) dYg[(long long)c * B + s] = dl / tau;
+            }
         }
     }
     if (lane == 0) part[warp] = li;
@@ -190,6 +245,7 @@ constexpr int kDyRows = 32;
 __global__ void __launch_bounds__(kDyThreads)
 head_dy_kernel(const float* __restrict__ dlogit, long long B, int C, int g, int w, float tau,
                float* __restrict__ dY) {
+    dependent_kernel_start();
     const long long s = (long long)blockIdx.y * kDyThreads + threadIdx.x;
     if (s >= B) return;
     const int j0 = blockIdx.x * kDyRows;
@@ -250,26 +306,29 @@ extern "C" int bitlogic_head_loss_ex(const float* Y, int32_t w, int64_t B, int32
     int splits = 1;
 
     if (B % 4 == 0 && aligned16(Y)) {
-        // split the rows of a class until about two blocks per SM pull from
-        // HBM, keeping at least 4 rows per warp
+        // split the rows of a class while the doubled grid still fits one
+        // wave of resident blocks, keeping at least 4 rows per warp
         const long long nsb = (B + 127) / 128;
-        const int sms = sm_count();
-        while (splits < kMaxRowSplits && (long long)C * splits * nsb < 2ll * sms &&
+        const long long resident = (long long)(2048 / (kSumVecWarps * 32)) * sm_count();
+        while (splits < kMaxRowSplits && (long long)C * (2 * splits) * nsb <= resident &&
                g / (2 * splits) >= 4 * kSumVecWarps)
             splits *= 2;
         const int rows_per_split = (g + splits - 1) / splits;
         if ((long long)C * splits > 0x7fffffffll || nsb > 65535) return BITLOGIC_ERR_SHAPE;
-        head_group_sum_vec_kernel<<<dim3((unsigned)(C * splits), (unsigned)nsb), kSumVecWarps * 32, 0, stream>>>(
-            Y, B, C, g, tau, lg, split_sums, splits, rows_per_split, done);
+        (void)launch_dependent(head_group_sum_vec_kernel, dim3((unsigned)(C * splits), (unsigned)nsb),
+                               kSumVecWarps * 32, 0, stream, Y, B, C, g, tau, lg, split_sums, splits,
+                               rows_per_split, done);
     } else
-        head_group_sum_kernel<<<dim3((unsigned)C, (unsigned)sb), kSumWarps * 32, 0, stream>>>(Y, B, C, g, tau, lg,
-                                                                                          done);
-    head_softmax_kernel<<<(unsigned)((B + kSoftWarps - 1) / kSoftWarps), kSoftWarps * 32, 0, stream>>>(
-        lg, B, C, labels, dlogit, block_sums, done, loss, tau, dY_grouped, splits > 1 ? split_sums : nullptr,
-        splits);
-    if (dY)
-        head_dy_kernel<<<dim3((unsigned)((w + kDyRows - 1) / kDyRows), (unsigned)gy), kDyThreads, 0, stream>>>(
-            dlogit, B, C, g, w, tau, dY);
+        (void)launch_dependent(head_group_sum_kernel, dim3((unsigned)C, (unsigned)sb), kSumWarps * 32, 0, stream, Y,
+                               B, C, g, tau, lg, done);
+    if (launch_status()) return BITLOGIC_ERR_CUDA;
+    if (launch_dependent(head_softmax_kernel, (unsigned)((B + kSoftWarps - 1) / kSoftWarps), kSoftWarps * 32, 0,
+                         stream, lg, B, C, labels, dlogit, block_sums, done, loss, tau,
+                         dY_grouped, splits > 1 ? split_sums : nullptr, splits) != cudaSuccess)
+        return BITLOGIC_ERR_CUDA;
+    if (dY && launch_dependent(head_dy_kernel, dim3((unsigned)((w + kDyRows - 1) / kDyRows), (unsigned)gy),
+                               kDyThreads, 0, stream, dlogit, B, C, g, w, tau, dY) != cudaSuccess)
+        return BITLOGIC_ERR_CUDA;
     return launch_status();
 }
 

@@ -122,9 +122,11 @@ def test_noalloc_head_matches_workspace_head_and_oracle_twice():
 def test_noalloc_head_at_its_size_limits():
     lib = bl.load()
     stream = P(torch.cuda.current_stream().cuda_stream)
-    # four row splits of the group sum (every split slot of the workspace is
-    # written and read): 10 classes of 2048 rows over 1024 samples
+    # row splits of the group sum: 10 classes of 2048 rows over 1024 samples
+    # (split while the grid fits one wave), and over 256 samples (four
+    # splits: every split slot of the workspace is written and read)
     _noalloc_matches(lib, stream, 10, 2048, 1024, 50.0, 3)
+    _noalloc_matches(lib, stream, 10, 2048, 256, 50.0, 6)
     # the largest batch of 10 classes whose workspace fits the 8 MiB array,
     # rounded down to a multiple of 4 (the vector group sum)
     B = _largest_batch(10) // 4 * 4
