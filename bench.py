@@ -95,7 +95,8 @@ def parse_args(argv=None):
                    help="layer 1 recomputes its output gradient through layer 2 (fan-in <= 3) instead of "
                         "reading layer 2's per-edge terms; auto: whenever layer 2's fan-in allows it")
     p.add_argument("--bytes1", choices=["auto", "on", "off"], default="auto",
-                   help="layer-1 backward gathers the encoder's wires as bytes (fused and through routes)")
+                   help="layer 1 reads the encoder's wires as bytes: lookup forward and one-hot table "
+                        "gradient (auto: whenever B % 4 == 0)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-graph", action="store_true",
@@ -272,7 +273,13 @@ def call_work(wl, B, fuse_dy1=False, through=False, bytes1=False):
     gradient is one row per class (every node of a class has the same
     gradient), so dY is C x B, not w x B.  The per-edge input-gradient terms
     that the layer-2 backward writes and the CSR reduction reads are not
-    algorithmic: they appear only in the bytes moved."""
+    algorithmic: they appear only in the bytes moved.
+
+    With byte wires for layer 1 (``bytes1``) the encoder writes one byte per
+    wire and layer 1's inputs are binary, so its corner weights are one-hot:
+    the forward is a lookup (no arithmetic beyond the k-byte gather and one
+    table read) and the table gradient one add per (node, sample); both
+    calls are then bounded by their bytes."""
     K, k = wl.K, wl.k
     w1, w2 = wl.widths
     win, d, C = wl.w_in, wl.d, wl.classes
@@ -298,11 +305,14 @@ def call_work(wl, B, fuse_dy1=False, through=False, bytes1=False):
         "hard1": (f * (win * W + w1 * W + w1 * k) + 8 * w1, (K - 1) * w1 * W, None),
         "hard2": (f * (w1 * W + w2 * k + B * C * 2 + B) + 8 * w2, (K - 1) * w2 * W, None),
     }
-    xb1 = 1 if bytes1 else f   # bytes per layer-1 input value read by the layer-1 backward
+    xb1 = 1 if bytes1 else f   # bytes per layer-1 input value
+    dth1_ops = w1 * B if bytes1 else (2 * (K - 1) + K) * w1 * B   # layer-1 table gradient
     if bytes1:
-        # the encoder also writes the wires as bytes, which the layer-1
-        # backward gathers instead of the fp32 rows
-        work["encode"] = (B * d + f * win * B + win * B, 0, B * d + f * win * B + win * B)
+        # byte rows: the encoder writes one byte per wire, the layer-1
+        # forward gathers bytes and reads one table entry per output
+        work["encode"] = (B * d + win * B, 0, B * d + win * B)
+        work["forward1"] = (win * B + f * (w1 * B + w1 * K + w1 * k), 0, None)
+        work["backward1"] = (win * B + f * (w1 * B + 2 * w1 * K + w1 * k), dth1_ops, None)
     if through:
         # layer 2: table gradient only; layer 1: its table gradient with its
         # output gradient recomputed through layer 2 (the consumers' other
@@ -311,12 +321,12 @@ def call_work(wl, B, fuse_dy1=False, through=False, bytes1=False):
         # to backward1 and nothing per edge is stored
         work["backward2"] = (f * (w1 * B + C * B + 2 * w2 * K + w2 * k), (2 * (K - 1) + K) * w2 * B, None)
         work["backward1"] = (xb1 * win * B + f * (w1 * B + C * B + 2 * w1 * K + w1 * k + w2 * K + w2 * k) + csr2,
-                             (2 * (K - 1) + K) * w1 * B + 2 * (K - 1) * w2 * B, None)
+                             dth1_ops + 2 * (K - 1) * w2 * B, None)
         del work["csr2"]
         return {n: (b, o, b if m is None else m) for n, (b, o, m) in work.items()}
     if fuse_dy1:
         # layer 1 sums layer 2's per-edge terms through the CSR map itself
-        work["backward1"] = (xb1 * win * B + f * (w1 * B + 2 * w1 * K + w1 * k) + csr2, (2 * (K - 1) + K) * w1 * B,
+        work["backward1"] = (xb1 * win * B + f * (w1 * B + 2 * w1 * K + w1 * k) + csr2, dth1_ops,
                              xb1 * win * B + f * (2 * w1 * K + w1 * k) + csr2 + terms)
         del work["csr2"]
     return {n: (b, o, b if m is None else m) for n, (b, o, m) in work.items()}
@@ -332,24 +342,12 @@ TRAFFIC = {
         "bytes": 59560448 + 144350720, "source": "lut_soft.cu",
         "sha256": "78edac247d6c64dc0042c15287b5174dfc03ecac6e7945ec4beb26e9e6cc6800",
         "note": "ncu capture of this workload (one-pass DRAM metrics)"},
-    ("cifar10", "forward1"): {
-        "bytes": 511101952 + 243450624, "source": "lut_soft.cu",
-        "sha256": "78edac247d6c64dc0042c15287b5174dfc03ecac6e7945ec4beb26e9e6cc6800",
-        "note": "ncu capture of this workload (one-pass DRAM metrics)"},
     ("cifar10", "forward2"): {
         "bytes": 1162980096 + 245190144, "source": "lut_soft.cu",
         "sha256": "78edac247d6c64dc0042c15287b5174dfc03ecac6e7945ec4beb26e9e6cc6800",
         "note": "ncu capture of this workload (one-pass DRAM metrics)"},
     ("cifar10", "backward2"): {
         "bytes": 1344603136 + 1542144768, "source": "lut_soft.cu",
-        "sha256": "78edac247d6c64dc0042c15287b5174dfc03ecac6e7945ec4beb26e9e6cc6800",
-        "note": "ncu capture of this workload (one-pass DRAM metrics)"},
-    ("cifar10", "backward1"): {
-        "bytes": 2504033536 + 15722496, "source": "lut_soft.cu",
-        "sha256": "78edac247d6c64dc0042c15287b5174dfc03ecac6e7945ec4beb26e9e6cc6800",
-        "note": "ncu capture of this workload (one-pass DRAM metrics; layer 1 summing layer 2's terms)"},
-    ("cifar100", "forward1"): {
-        "bytes": 5106467072 + 1034765312, "source": "lut_soft.cu",
         "sha256": "78edac247d6c64dc0042c15287b5174dfc03ecac6e7945ec4beb26e9e6cc6800",
         "note": "ncu capture of this workload (one-pass DRAM metrics)"},
     ("cifar100", "forward2"): {
@@ -360,10 +358,6 @@ TRAFFIC = {
         "bytes": 6068320768 + 6277417984, "source": "lut_soft.cu",
         "sha256": "78edac247d6c64dc0042c15287b5174dfc03ecac6e7945ec4beb26e9e6cc6800",
         "note": "ncu capture of this workload (one-pass DRAM metrics)"},
-    ("cifar100", "backward1"): {
-        "bytes": 11884503296 + 32632576, "source": "lut_soft.cu",
-        "sha256": "78edac247d6c64dc0042c15287b5174dfc03ecac6e7945ec4beb26e9e6cc6800",
-        "note": "ncu capture of this workload (one-pass DRAM metrics; layer 1 summing layer 2's terms)"},
     ("hard_cifar10", "hard1"): {
         "bytes": 16 * (1.209681e9 + 2.054784e9), "source": "hard.cu",
         "sha256": "f9bed6fc20215df71b5e12eebae1c94762286b3c7b941dea9a2ff948bfb9ed3c",

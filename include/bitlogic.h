@@ -190,6 +190,24 @@ int bitlogic_csr_reduce(const float* edge_terms, int64_t B, const int32_t* csr_o
                         const int32_t* csr_edge, int32_t w_in, int32_t n_edges,
                         float* dX, cudaStream_t stream);
 
+/* bitlogic_lut_forward_node on byte rows (binary wires, each byte 0 or 1,
+ * e.g. from bitlogic_encode_thermometer_u8; a byte is read by its lowest
+ * bit).  On binary inputs the corner weights prod_i x_i^{a_i}(1-x_i)^{1-a_i}
+ * are 1 for a = sum_i x_i 2^i and 0 for every other corner (§2: a soft node
+ * on binary inputs returns its table entry), so
+ *   Y[j][s] = t_a,  a = sum_i X[conn[j][i]][s] 2^i,
+ * with t_a = sigmoid(theta_j[a]) (BITLOGIC_NODE_SOFT) or [theta_j[a] > 0]
+ * (BITLOGIC_NODE_ST): a gather of k bytes and one table read per output.
+ *   X     device uint8 [w_in][B];  conn, theta, Y, k, node as in
+ *         bitlogic_lut_forward_node.
+ * Any B and alignment (B % 4 == 0 with 4-byte aligned X and 16-byte aligned
+ * Y takes the vector form).  Out-of-range connectivity raises the device
+ * flag and reads row 0.  Returns BITLOGIC_ERR_NULL, BITLOGIC_ERR_SHAPE,
+ * BITLOGIC_ERR_FANIN, BITLOGIC_ERR_NODE, BITLOGIC_ERR_CUDA. */
+int bitlogic_lut_forward_u8(const uint8_t* X, int32_t w_in, int64_t B, const int32_t* conn,
+                            const float* theta, int32_t w, int32_t k, int32_t node, float* Y,
+                            cudaStream_t stream);
+
 /* General form of the layer backward, with the output gradient taken from
  * one of two sources (exactly one of dY and up_terms is non-NULL):
  *   dY rows:  node j reads row j / dy_group of dY ([w / dy_group][B]);
@@ -269,9 +287,12 @@ int bitlogic_lut_backward_through(const float* X, int32_t w_in, int64_t B, const
                                   float* dY_out, cudaStream_t stream);
 
 /* bitlogic_lut_backward_through with the layer input as byte rows (binary
- * wires, each byte 0 or 1, e.g. from bitlogic_encode_thermometer_u8):
- * X device uint8 [w_in][B]; every other argument as above.  The result
- * equals the fp32-row call on the same wires bit for bit. */
+ * wires, each byte 0 or 1, e.g. from bitlogic_encode_thermometer_u8; a byte
+ * is read by its lowest bit): X device uint8 [w_in][B]; every other argument
+ * as above.  On binary wires the corner weights are one-hot (§2), so each
+ * sample adds its gradient to the one table entry its input bits select, in
+ * the sample order of the fp32 form: the result equals the fp32-row call on
+ * the same wires bit for bit. */
 int bitlogic_lut_backward_through_u8(const uint8_t* X, int32_t w_in, int64_t B, const int32_t* conn,
                                      const float* theta, int32_t w, int32_t k, int32_t node,
                                      const float* Y, const int32_t* up_conn, const float* up_theta,
@@ -280,9 +301,11 @@ int bitlogic_lut_backward_through_u8(const uint8_t* X, int32_t w_in, int64_t B, 
                                      float* dY_out, cudaStream_t stream);
 
 /* Table gradient (no input gradient) of a layer whose input is byte rows
- * (binary wires, each byte 0 or 1): gathering bytes moves a quarter of the
- * data of fp32 rows, which is what bounds the first layer once its input is
- * larger than L2.  The output gradient comes from exactly one of
+ * (binary wires, each byte 0 or 1; a byte is read by its lowest bit):
+ * gathering bytes moves a quarter of the data of fp32 rows, and on binary
+ * wires the corner weights are one-hot (§2), so each sample adds its
+ * gradient to the one table entry its input bits select instead of 2^k
+ * multiply-adds.  The output gradient comes from exactly one of
  *   dY rows:  node j reads row j / dy_group of dY ([w / dy_group][B]);
  *   up terms: the next layer's per-edge terms up_terms [up_edges][B] summed
  *             over p in [up_off[j], up_off[j+1]) in increasing p (row

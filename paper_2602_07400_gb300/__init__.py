@@ -28,7 +28,7 @@ __all__ = [
     "bitlogic_lut_backward_workspace", "bitlogic_lut_backward", "bitlogic_lut_backward_edges",
     "bitlogic_csr_reduce", "bitlogic_lut_backward_ex", "bitlogic_head_loss_ex",
     "bitlogic_head_loss_workspace", "bitlogic_head_loss_noalloc", "bitlogic_lut_backward_through", "bitlogic_lut_backward_through_u8",
-    "bitlogic_lut_backward_u8",
+    "bitlogic_lut_backward_u8", "bitlogic_lut_forward_u8",
     "bitlogic_head_loss", "bitlogic_binarize_tables", "bitlogic_pack_bits",
     "bitlogic_hard_forward", "bitlogic_build_csr", "bitlogic_csr_positions", "bitlogic_device_error",
     "bitlogic_adamw_update", "bitlogic_route_forward", "bitlogic_route_backward", "bitlogic_route_snap",
@@ -79,6 +79,7 @@ _SIGS = {
     "bitlogic_encode_thermometer_both": ([_P, _I64, _I32, _P, _I32, _P, _P, _P], ctypes.c_int),
     "bitlogic_quantile_thresholds": ([_P, _I32, _P], ctypes.c_int),
     "bitlogic_lut_forward_node": ([_P, _I32, _I64, _P, _P, _I32, _I32, _I32, _P, _P], ctypes.c_int),
+    "bitlogic_lut_forward_u8": ([_P, _I32, _I64, _P, _P, _I32, _I32, _I32, _P, _P], ctypes.c_int),
     "bitlogic_lut_backward_workspace": ([_I32, _I64, _I32, _I32, _I32], _SZ),
     "bitlogic_lut_backward": ([_P, _I32, _I64, _P, _P, _I32, _I32, _P, _P, _P, _P, _P,
                                _P, _SZ, _P], ctypes.c_int),
@@ -360,6 +361,21 @@ def bitlogic_lut_forward_node(X: torch.Tensor, conn: torch.Tensor, theta: torch.
     _need(theta, "theta", torch.float32, (w, 1 << k))
     _need(Y, "Y", torch.float32, (w, B))
     _check("bitlogic_lut_forward_node", load().bitlogic_lut_forward_node(
+        _ptr(X), w_in, B, _ptr(conn), _ptr(theta), w, k, code, _ptr(Y), _stream(stream)))
+
+
+def bitlogic_lut_forward_u8(X: torch.Tensor, conn: torch.Tensor, theta: torch.Tensor,
+                            Y: torch.Tensor, node="soft", stream=None):
+    """Layer forward on byte rows (binary wires): Y[j][s] = the table entry
+    the inputs' bits select."""
+    code = _node_code(node)
+    w_in, B = X.shape
+    w, k = conn.shape
+    _need(X, "X", torch.uint8, (w_in, B))
+    _need(conn, "conn", torch.int32, (w, k))
+    _need(theta, "theta", torch.float32, (w, 1 << k))
+    _need(Y, "Y", torch.float32, (w, B))
+    _check("bitlogic_lut_forward_u8", load().bitlogic_lut_forward_u8(
         _ptr(X), w_in, B, _ptr(conn), _ptr(theta), w, k, code, _ptr(Y), _stream(stream)))
 
 

@@ -18,7 +18,7 @@ CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libbitlogic.so")
 INCLUDE = os.path.join(ROOT, "include")
-SOURCES = ["abi.cu", "encode.cu", "fit.cu", "lut_soft.cu", "lut_through.cu", "route.cu", "head.cu", "hard.cu", "optim.cu", "peaks.cu"]
+SOURCES = ["abi.cu", "encode.cu", "fit.cu", "lut_soft.cu", "lut_through.cu", "lut_bytes.cu", "route.cu", "head.cu", "hard.cu", "optim.cu", "peaks.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
          f"-I{INCLUDE}", f"-I{CSRC}"]

@@ -31,6 +31,7 @@ extern "C" int bitlogic_internal_index_error_hard(cudaStream_t);
 extern "C" int bitlogic_internal_index_error_optim(cudaStream_t);
 extern "C" int bitlogic_internal_index_error_route(cudaStream_t);
 extern "C" int bitlogic_internal_index_error_lut_through(cudaStream_t);
+extern "C" int bitlogic_internal_index_error_lut_bytes(cudaStream_t);
 
 extern "C" const char* bitlogic_status_string(int code) {
     switch (code) {
@@ -86,13 +87,14 @@ extern "C" int bitlogic_csr_positions(const int32_t* edge_host, int32_t n_edges,
 
 extern "C" int bitlogic_device_error(cudaStream_t stream) {
     int worst = BITLOGIC_OK;
-    const int r[7] = {bitlogic_internal_index_error_lut_soft(stream),
+    const int r[8] = {bitlogic_internal_index_error_lut_soft(stream),
                       bitlogic_internal_index_error_head(stream),
                       bitlogic_internal_index_error_encode(stream),
                       bitlogic_internal_index_error_hard(stream),
                       bitlogic_internal_index_error_optim(stream),
                       bitlogic_internal_index_error_route(stream),
-                      bitlogic_internal_index_error_lut_through(stream)};
+                      bitlogic_internal_index_error_lut_through(stream),
+                      bitlogic_internal_index_error_lut_bytes(stream)};
     for (int v : r) {
         if (v == BITLOGIC_ERR_CUDA) return v;
         if (v != BITLOGIC_OK) worst = v;

@@ -1,0 +1,177 @@
+// Soft forward of a LUT layer whose input is byte rows (binary wires, each
+// byte 0 or 1: the thermometer encoder's output, §3 "Encoders and heads").
+//
+// The relaxed table of §2, y = sum_a t_a prod_i x_i^{a_i} (1 - x_i)^{1 - a_i},
+// has one-hot corner weights on binary inputs: the product is 1 for the
+// corner a = sum_i x_i 2^i the inputs sit on and 0 for every other corner, so
+// y is the table entry t_a itself.  On byte rows the layer is therefore a
+// gather of k bytes and one table read per (node, sample); the first layer of
+// the training step sees only such inputs.  Table entries follow the node
+// form (the sigmoid of the logit, or [theta > 0] for the straight-through
+// node), the same entries the fp32 forward interpolates.
+//
+// Layout: a warp per node over a batch slice; lanes over 4 consecutive
+// samples (one 32-bit load per input row gives the 4 samples' bytes of that
+// input); the corner indices of the 4 samples are built byte-wise in one
+// register (shift and OR, no carry crosses a byte for k <= 7); the node's
+// table (2^k <= 64 entries) sits in two registers per lane and each lookup is
+// a shuffle from the lane holding the entry.  Rows are gathered with several
+// 128-sample groups in flight per lane.  A scalar form (one sample per lane)
+// serves ragged batches and unaligned rows.
+#include "common.cuh"
+
+namespace bitlogic {
+namespace {
+
+#ifndef BITLOGIC_BYTES_FWD_GROUPS
+#define BITLOGIC_BYTES_FWD_GROUPS 8
+#endif
+#ifndef BITLOGIC_BYTES_FWD_STREAM
+#define BITLOGIC_BYTES_FWD_STREAM 1
+#endif
+constexpr int kBytesFwdWarps = 8;    // warps (nodes) per block
+constexpr int kBytesFwdGroups = BITLOGIC_BYTES_FWD_GROUPS;   // 128-sample groups in flight per lane
+
+__device__ __forceinline__ float node_entry(float th, int node) {
+    return node == BITLOGIC_NODE_ST ? (th > 0.f ? 1.f : 0.f) : sigmoidf(th);
+}
+
+// Entry a (< 2^k) of the node's table, held as entry lane in `lo` and entry
+// 32 + lane in `hi`.  Every lane of the warp takes part.
+template <int K>
+__device__ __forceinline__ float table_at(float lo, float hi, uint32_t a) {
+    const float vlo = __shfl_sync(0xffffffffu, lo, (int)(a & 31u));
+    if constexpr (K > 32) {
+        const float vhi = __shfl_sync(0xffffffffu, hi, (int)(a & 31u));
+        return (a & 32u) ? vhi : vlo;
+    } else {
+        (void)hi;
+        return vlo;
+    }
+}
+
+template <int k, bool VEC>
+__global__ void __launch_bounds__(kBytesFwdWarps * 32)
+lut_forward_u8_kernel(const uint8_t* __restrict__ X, int w_in, long long B, const int* __restrict__ conn,
+                      const float* __restrict__ theta, int w, int node, float* __restrict__ Y, long long chunk) {
+    constexpr int K = 1 << k;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int j = blockIdx.x * kBytesFwdWarps + warp;
+    if (j >= w) return;   // warp-uniform
+    const uint8_t* xr[k];
+    bool bad = false;
+#pragma unroll
+    for (int i = 0; i < k; ++i) {
+        int c = __ldg(conn + (long long)j * k + i);
+        if ((unsigned)c >= (unsigned)w_in) {
+            bad = true;
+            c = 0;
+        }
+        xr[i] = X + (long long)c * B;
+    }
+    if (bad && lane == 0) flag_index_error();
+    const float lo = lane < K ? node_entry(__ldg(theta + (long long)j * K + lane), node) : 0.f;
+    const float hi = K > 32 ? node_entry(__ldg(theta + (long long)j * K + 32 + (lane & 31)), node) : 0.f;
+    const long long s0 = (long long)blockIdx.y * chunk;
+    const long long s1 = min(B, s0 + chunk);
+    float* yr = Y + (long long)j * B;
+    if constexpr (VEC) {
+        // lane: samples base + 128 u + 4 lane .. + 3 (B % 4 == 0: all four in range)
+        for (long long base = s0; base < s1; base += 128 * kBytesFwdGroups) {
+            uint32_t v[kBytesFwdGroups];
+#pragma unroll
+            for (int u = 0; u < kBytesFwdGroups; ++u) {
+                const long long s4 = base + 128 * u + 4 * lane;
+                v[u] = 0u;
+                if (s4 < s1) {
+                    v[u] = __ldg(reinterpret_cast<const uint32_t*>(xr[k - 1] + s4)) & 0x01010101u;
+#pragma unroll
+                    for (int i = k - 2; i >= 0; --i)
+                        v[u] = (v[u] << 1) | (__ldg(reinterpret_cast<const uint32_t*>(xr[i] + s4)) & 0x01010101u);
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < kBytesFwdGroups; ++u) {
+                const long long s4 = base + 128 * u + 4 * lane;
+                float4 y;
+                y.x = table_at<K>(lo, hi, v[u] & 0xffu);
+                y.y = table_at<K>(lo, hi, (v[u] >> 8) & 0xffu);
+                y.z = table_at<K>(lo, hi, (v[u] >> 16) & 0xffu);
+                y.w = table_at<K>(lo, hi, v[u] >> 24);
+                if (s4 < s1) {
+#if BITLOGIC_BYTES_FWD_STREAM
+                    __stcs(reinterpret_cast<float4*>(yr + s4), y);
+#else
+                    *reinterpret_cast<float4*>(yr + s4) = y;
+#endif
+                }
+            }
+        }
+    } else {
+        for (long long base = s0; base < s1; base += 32) {
+            const long long s = base + lane;
+            uint32_t a = 0u;
+            if (s < s1) {
+#pragma unroll
+                for (int i = 0; i < k; ++i) a |= (uint32_t)(__ldg(xr[i] + s) & 1u) << i;
+            }
+            const float y = table_at<K>(lo, hi, a);
+            if (s < s1) yr[s] = y;
+        }
+    }
+}
+
+// Samples per warp: the whole batch unless that leaves fewer than about two
+// waves of warps (then slices of at least 512 samples, a multiple of 128).
+long long forward_u8_chunk(int w, long long B) {
+    const long long wanted = 2ll * sm_count() * 64;
+    long long c = (long long)w * B / wanted;
+    c = (c / 128) * 128;
+    if (c < 512) c = 512;
+    return c < B ? c : B;
+}
+
+template <int k>
+int launch_forward_u8(const uint8_t* X, int w_in, long long B, const int* conn, const float* theta, int w,
+                      int node, float* Y, cudaStream_t st) {
+    const bool vec = (B % 4 == 0) && ((reinterpret_cast<uintptr_t>(X) & 3u) == 0) && aligned16(Y);
+    long long chunk = forward_u8_chunk(w, B);
+    if (vec) chunk = (chunk + 3) / 4 * 4;
+    const long long ny = (B + chunk - 1) / chunk;
+    if (ny > 65535) return BITLOGIC_ERR_SHAPE;
+    dim3 grid((unsigned)((w + kBytesFwdWarps - 1) / kBytesFwdWarps), (unsigned)ny);
+    if (vec)
+        lut_forward_u8_kernel<k, true><<<grid, kBytesFwdWarps * 32, 0, st>>>(X, w_in, B, conn, theta, w, node, Y,
+                                                                            chunk);
+    else
+        lut_forward_u8_kernel<k, false><<<grid, kBytesFwdWarps * 32, 0, st>>>(X, w_in, B, conn, theta, w, node, Y,
+                                                                             chunk);
+    return launch_status();
+}
+
+}  // namespace
+}  // namespace bitlogic
+
+using namespace bitlogic;
+
+BITLOGIC_ERROR_READER(lut_bytes)
+
+extern "C" int bitlogic_lut_forward_u8(const uint8_t* X, int32_t w_in, int64_t B, const int32_t* conn,
+                                       const float* theta, int32_t w, int32_t k, int32_t node, float* Y,
+                                       cudaStream_t stream) {
+    if (!conn || !theta) return BITLOGIC_ERR_NULL;
+    if (B > 0 && (!X || !Y)) return BITLOGIC_ERR_NULL;   // an empty batch may come as NULL
+    if (w_in <= 0 || w <= 0 || B < 0) return BITLOGIC_ERR_SHAPE;
+    if (k < 1 || k > 6 || k > w_in) return BITLOGIC_ERR_FANIN;
+    if ((int64_t)w * k > 0x7fffffffLL) return BITLOGIC_ERR_SHAPE;
+    if (node != BITLOGIC_NODE_SOFT && node != BITLOGIC_NODE_ST) return BITLOGIC_ERR_NODE;
+    if (B == 0) return BITLOGIC_OK;
+    switch (k) {
+        case 1: return launch_forward_u8<1>(X, w_in, B, conn, theta, w, node, Y, stream);
+        case 2: return launch_forward_u8<2>(X, w_in, B, conn, theta, w, node, Y, stream);
+        case 3: return launch_forward_u8<3>(X, w_in, B, conn, theta, w, node, Y, stream);
+        case 4: return launch_forward_u8<4>(X, w_in, B, conn, theta, w, node, Y, stream);
+        case 5: return launch_forward_u8<5>(X, w_in, B, conn, theta, w, node, Y, stream);
+        default: return launch_forward_u8<6>(X, w_in, B, conn, theta, w, node, Y, stream);
+    }
+}

@@ -3,17 +3,15 @@
 // uses on its first layer:
 //
 // * the layer input as fp32 rows or as byte rows (binary wires, e.g. the
-//   thermometer encoder's output written by bitlogic_encode_thermometer_u8):
-//   gathering bytes moves a quarter of the data, which matters when the input
-//   is larger than L2 and every node's k gathered rows come from DRAM;
-// * the output gradient from
-//   - rows: row j / group of dY (group = 1: one row per node);
-//   - terms: the next layer's per-edge input-gradient terms, summed over the
-//     node's consumers in increasing CSR position (the order of
-//     bitlogic_csr_reduce, so the sum is the same bit for bit);
-//   - through: recomputed from the next layer itself (chain rule through a
+//   thermometer encoder's output written by bitlogic_encode_thermometer_u8);
+// * the output gradient
+//   - recomputed from the next layer itself (through: chain rule through a
 //     next layer of small fan-in), so that neither the next layer's per-edge
-//     terms nor this layer's output gradient are stored.
+//     terms nor this layer's output gradient are stored (fp32 or byte rows);
+//   - from rows: row j / group of dY (byte rows);
+//   - from terms: the next layer's per-edge input-gradient terms, summed over
+//     the node's consumers in increasing CSR position (the order of
+//     bitlogic_csr_reduce, so the sum is the same bit for bit; byte rows).
 //
 // Through: for the node j of this layer, output row j is an input of the
 // next layer; its gradient (the next layer's input gradient, summed over
@@ -35,17 +33,27 @@
 // The table gradient itself is the dtheta-only form of the soft backward:
 //   dtheta_a = t_a (1 - t_a) sum_s g_s w_a(x_s),
 // with the corner weights w_a built per sample as the outer product of the
-// low-half and high-half corner weights of the node's own k inputs.
+// low-half and high-half corner weights of the node's own k inputs.  On byte
+// rows (binary wires) the corner weights of a sample are one-hot: w_a is 1
+// for the corner a = sum_i x_i 2^i the inputs sit on and 0 elsewhere (the
+// identity behind "a soft node on binary inputs returns its table entry",
+// §2), so the sum adds g_s to one entry per sample.  Each lane keeps its
+// 2^k partial sums in its own column of a shared [2^k][32] array (no bank
+// conflicts) and adds each sample's g to the entry its index selects, in the
+// sample order of the register form; since g * 1 and g * 0 are exact, the
+// partial sums, and after the same butterfly dtheta, are the fp32 form's bit
+// for bit, for a few instructions per sample instead of ~2^k multiply-adds.
 //
-// Layout and scheduling follow the dtheta-only kernel: persistent one-warp
-// blocks, a node over the whole batch, 4 consecutive samples per lane in each
-// 128-sample stage, the node's k input rows streamed through a lane-private
-// cp.async ring that runs across node boundaries (16 bytes per lane and row
-// for fp32 rows, 4 for byte rows), and a fixed butterfly of shuffles for the
-// batch reduction.  The output gradient is formed for several stages at a
-// time (a chunk), so the rows it reads (gradient rows, term rows, consumer
-// rows) have several independent loads in flight per row.  Needs B % 4 == 0
-// and 16-byte aligned X, the gradient rows, the terms, Y and dY_out.
+// The through kernel follows the dtheta-only kernel's layout: persistent
+// one-warp blocks, a node over the whole batch, 4 consecutive samples per
+// lane in each 128-sample stage, the node's k input rows streamed through a
+// lane-private cp.async ring that runs across node boundaries (16 bytes per
+// lane and row for fp32 rows, 4 for byte rows), and a fixed butterfly of
+// shuffles for the batch reduction; the output gradient is formed for
+// several stages at a time (a chunk), so the consumer rows it reads have
+// several independent loads in flight.  The rows and terms sources on byte
+// rows have a streaming kernel of their own (below).  Needs B % 4 == 0 and
+// 16-byte aligned X, the gradient rows, the terms, Y and dY_out.
 #include "common.cuh"
 
 namespace bitlogic {
@@ -73,6 +81,47 @@ __device__ __forceinline__ float4 ldg4t(const float* p) { return __ldg(reinterpr
 
 __device__ __forceinline__ float comp4(const float4& v, int c) {
     return c == 0 ? v.x : c == 1 ? v.y : c == 2 ? v.z : v.w;
+}
+
+// Binary wires: the corner index of the lane's 4 samples of a stage, one
+// per byte (byte r = sum_i bit(x_i[s + r]) 2^i); `xb` points at the lane's 4
+// bytes of row 0 in a ring slot whose rows are `stride` bytes apart.  A byte
+// is read by its lowest bit.
+template <int k>
+__device__ __forceinline__ uint32_t corner_index4(const uint8_t* xb, int stride) {
+    uint32_t v = *reinterpret_cast<const uint32_t*>(xb + (k - 1) * stride) & 0x01010101u;
+#pragma unroll
+    for (int q = k - 2; q >= 0; --q) v = (v << 1) | (*reinterpret_cast<const uint32_t*>(xb + q * stride) & 0x01010101u);
+    return v;
+}
+
+// Adds the 4 samples' gradients to the entries their indices select in the
+// lane's column (`col` = the [2^k][32] array + lane), in sample order.
+__device__ __forceinline__ void corner_add4(float* col, uint32_t v, const float4& g) {
+    col[(v & 0xffu) * 32] += g.x;
+    col[((v >> 8) & 0xffu) * 32] += g.y;
+    col[((v >> 16) & 0xffu) * 32] += g.z;
+    col[(v >> 24) * 32] += g.w;
+}
+
+// Moves the lane's column into registers (for the butterfly) and clears it
+// for the next node.
+template <int K>
+__device__ __forceinline__ void corner_take(float* col, float (&acc)[K]) {
+#pragma unroll
+    for (int a = 0; a < K; ++a) {
+        acc[a] = col[a * 32];
+        col[a * 32] = 0.f;
+    }
+}
+
+template <typename TX>
+__host__ __device__ constexpr bool byte_rows() { return sizeof(TX) == 1; }
+
+// Shared bytes of the per-lane corner sums (byte rows only).
+template <typename TX>
+__host__ __device__ constexpr int corner_bytes(int k) {
+    return byte_rows<TX>() ? (1 << k) * 32 * (int)sizeof(float) : 0;
 }
 
 // Table entry of a node form: the sigmoid of the logit (soft LightLUT), or
@@ -205,9 +254,6 @@ __device__ __forceinline__ void add_consumer(float4& g, const Consumer<ku>& q, c
     }
 }
 
-// The output-gradient sources.
-constexpr int kSrcRows = 0, kSrcTerms = 1, kSrcThrough = 2;
-
 struct GradIn {
     const float* dY;        // rows: [w / group][B]
     int group;
@@ -223,26 +269,6 @@ struct GradIn {
     int up_group;
 };
 
-// Stages whose output gradient is formed together (registers: four float4
-// per stage of the chunk, besides the 2^k accumulators).
-#ifndef BITLOGIC_ROWS_CHUNK
-#define BITLOGIC_ROWS_CHUNK 2       // stages per chunk, k >= 5, rows source
-#endif
-#ifndef BITLOGIC_ROWS_BLOCKS
-#define BITLOGIC_ROWS_BLOCKS 12     // one-warp blocks per SM, k = 6, rows source
-#endif
-template <int k, int SRC>
-__host__ __device__ constexpr int grad_chunk() {
-    if constexpr (SRC == kSrcThrough) return k <= 3 ? BITLOGIC_THROUGH_CHUNK : (k == 4 ? 4 : (k == 5 ? 2 : 1));
-    else return k <= 4 ? 4 : BITLOGIC_ROWS_CHUNK;
-}
-// one-warp blocks per SM: fewer for the widest tables (their accumulators
-// and the loads in flight take more registers)
-template <int k, int SRC>
-__host__ __device__ constexpr int grad_min_blocks() {
-    return (k >= 6 && SRC != kSrcThrough) ? BITLOGIC_ROWS_BLOCKS : kTMinBlocks;
-}
-
 template <typename TX>
 __host__ __device__ constexpr int ring_bytes_per_warp(int k) {
     return kTStages * k * kTStageSamples * (int)sizeof(TX);
@@ -254,34 +280,30 @@ __device__ __forceinline__ void copy_row_part(uint8_t* dst, const uint8_t* src) 
     const unsigned sa = (unsigned)__cvta_generic_to_shared(dst);
     asm volatile("cp.async.ca.shared.global [%0], [%1], 4;\n" ::"r"(sa), "l"(src) : "memory");
 }
-// Its four samples as floats (a byte b becomes b exactly: 2^23 + b in the
-// mantissa, minus 2^23).
+// Its four samples (fp32 rows; byte rows take the one-hot form).
 __device__ __forceinline__ float4 read_row_part(const float* p) { return *reinterpret_cast<const float4*>(p); }
-__device__ __forceinline__ float4 read_row_part(const uint8_t* p) {
-    const uint32_t v = *reinterpret_cast<const uint32_t*>(p);
-    const float m = 8388608.0f;
-    return make_float4(__int_as_float(__byte_perm(v, 0x4B000000u, 0x7440)) - m,
-                       __int_as_float(__byte_perm(v, 0x4B000000u, 0x7441)) - m,
-                       __int_as_float(__byte_perm(v, 0x4B000000u, 0x7442)) - m,
-                       __int_as_float(__byte_perm(v, 0x4B000000u, 0x7443)) - m);
-}
 
-template <int k, int ku, typename TX, int SRC>
-__global__ void __launch_bounds__(32, (grad_min_blocks<k, SRC>()))
-lut_theta_src_kernel(const TX* __restrict__ X, int w_in, long long B, const int* __restrict__ conn,
-                     const float* __restrict__ theta, int w, GradIn gi, int node, float* __restrict__ dtheta,
-                     float* __restrict__ dY_out) {
+template <int k, int ku, typename TX>
+__global__ void __launch_bounds__(32, kTMinBlocks)
+lut_theta_through_kernel(const TX* __restrict__ X, int w_in, long long B, const int* __restrict__ conn,
+                         const float* __restrict__ theta, int w, GradIn gi, int node, float* __restrict__ dtheta,
+                         float* __restrict__ dY_out) {
     constexpr int K = 1 << k, KL = k / 2, NU = 1 << KL, NV = 1 << (k - KL);
     constexpr int CH = kTStageSamples;
-    constexpr int kTChunk = grad_chunk<k, SRC>();
+    constexpr int kTChunk = through_chunk<k>();
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const int lane = threadIdx.x & 31;
     TX* ring = reinterpret_cast<TX*>(smem_raw);
+    constexpr bool BIN = byte_rows<TX>();   // one-hot corner weights
+    float* corners = reinterpret_cast<float*>(smem_raw + ring_bytes_per_warp<TX>(k)) + lane;
+    if constexpr (BIN) {
+#pragma unroll
+        for (int a = 0; a < K; ++a) corners[a * 32] = 0.f;
+    }
     const int G = gridDim.x;
     const int jfirst = blockIdx.x;
     const int nst = (int)((B + CH - 1) / CH);
-    static_assert(SRC == kSrcRows || SRC == kSrcThrough, "the terms source has its own kernel");
-    const int n_up = SRC == kSrcThrough ? gi.up_w * ku : 0;   // CSR positions
+    const int n_up = gi.up_w * ku;   // CSR positions
 
     // issue stream: stage si of node ji, kTStages - 1 stages ahead of the
     // compute stream; rows of the warp's node after ji are loaded ahead
@@ -330,17 +352,12 @@ lut_theta_src_kernel(const TX* __restrict__ X, int w_in, long long B, const int*
 #pragma unroll 1
     for (int j = jfirst; j < w; j += G) {
         // the node's upstream edges (terms, through: CSR positions e0 .. e1 - 1)
-        int e0 = 0, deg = 0;
-        if constexpr (SRC != kSrcRows) {
-            int e1;
-            e0 = __ldg(gi.off + j);
-            e1 = __ldg(gi.off + j + 1);
-            if (e0 < 0 || e1 < e0 || e1 > n_up) {
-                if (lane == 0) flag_index_error();
-                e0 = e1 = 0;
-            }
-            deg = e1 - e0;
+        int e0 = __ldg(gi.off + j), e1 = __ldg(gi.off + j + 1);
+        if (e0 < 0 || e1 < e0 || e1 > n_up) {
+            if (lane == 0) flag_index_error();
+            e0 = e1 = 0;
         }
+        const int deg = e1 - e0;
         // per lane one consumer (through), for the positions e0 .. e0 + 31
         Consumer<ku> mine;
         mine.grow = -1;
@@ -352,7 +369,7 @@ lut_theta_src_kernel(const TX* __restrict__ X, int w_in, long long B, const int*
                                          node, bad);
             if (__any_sync(0xffffffffu, bad) && lane == 0) flag_index_error();
         };
-        if constexpr (SRC != kSrcRows) load_edges(0);
+        load_edges(0);
 
         float acc[K];
 #pragma unroll
@@ -363,34 +380,25 @@ lut_theta_src_kernel(const TX* __restrict__ X, int w_in, long long B, const int*
             float4 gv[kTChunk];
 #pragma unroll
             for (int t = 0; t < kTChunk; ++t) gv[t] = make_float4(0.f, 0.f, 0.f, 0.f);
-            if constexpr (SRC == kSrcRows) {
-                const float* row = gi.dY + (long long)(j / gi.group) * B;
-#pragma unroll
-                for (int t = 0; t < kTChunk; ++t) {
-                    const long long s4 = (long long)(sc0 + t) * CH + 4 * lane;
-                    if (s4 < B) gv[t] = ldg4t(row + s4);
-                }
-            } else {
 #pragma unroll 1
-                for (int c0 = 0; c0 < deg; c0 += 32) {
-                    if (c0 > 0) load_edges(c0);   // more than 32 upstream edges: this chunk's
-                    const int n = min(32, deg - c0);
-                    {
-                        // consumers in increasing CSR position: each consumer's rows
-                        // for all the chunk's stages at once
+            for (int c0 = 0; c0 < deg; c0 += 32) {
+                if (c0 > 0) load_edges(c0);   // more than 32 upstream edges: this chunk's
+                const int n = min(32, deg - c0);
+                {
+                    // consumers in increasing CSR position: each consumer's rows
+                    // for all the chunk's stages at once
 #pragma unroll 1
-                        for (int e = 0; e < n; ++e) {
-                            const Consumer<ku> q = shfl_consumer<ku>(mine, e);
+                    for (int e = 0; e < n; ++e) {
+                        const Consumer<ku> q = shfl_consumer<ku>(mine, e);
 #pragma unroll
-                            for (int t = 0; t < kTChunk; ++t) {
-                                const long long s4 = (long long)(sc0 + t) * CH + 4 * lane;
-                                if (s4 < B) add_consumer<ku>(gv[t], q, gi.Y, gi.up_dY, B, s4);
-                            }
+                        for (int t = 0; t < kTChunk; ++t) {
+                            const long long s4 = (long long)(sc0 + t) * CH + 4 * lane;
+                            if (s4 < B) add_consumer<ku>(gv[t], q, gi.Y, gi.up_dY, B, s4);
                         }
                     }
                 }
-                if (deg > 32) load_edges(0);   // the next chunk of stages starts again at position e0
             }
+            if (deg > 32) load_edges(0);   // the next chunk of stages starts again at position e0
             // the chunk's stages: the table gradient from the node's inputs
 #pragma unroll
             for (int t = 0; t < kTChunk; ++t) {
@@ -401,41 +409,45 @@ lut_theta_src_kernel(const TX* __restrict__ X, int w_in, long long B, const int*
                     if (s4 < B) {   // B % 4 == 0: all four samples are in range
                         if (dY_out) *reinterpret_cast<float4*>(dY_out + (long long)j * B + s4) = gv[t];
                         const TX* buf = ring + rb * (k * CH) + 4 * lane;
-                        float4 xv[k];
+                        if constexpr (BIN) {
+                            corner_add4(corners, corner_index4<k>(reinterpret_cast<const uint8_t*>(buf), CH), gv[t]);
+                        } else {
+                            float4 xv[k];
 #pragma unroll
-                        for (int q = 0; q < k; ++q) xv[q] = read_row_part(buf + q * CH);
+                            for (int q = 0; q < k; ++q) xv[q] = read_row_part(buf + q * CH);
 #pragma unroll
-                        for (int r = 0; r < 4; ++r) {
-                            float x[k], omx[k];
+                            for (int r = 0; r < 4; ++r) {
+                                float x[k], omx[k];
 #pragma unroll
-                            for (int q = 0; q < k; ++q) {
-                                x[q] = comp4(xv[q], r);
-                                omx[q] = 1.0f - x[q];
-                            }
-                            float U[NU], V[NV];
-                            U[0] = comp4(gv[t], r);
-#pragma unroll
-                            for (int q = 0; q < KL; ++q) {   // slot q doubles U: index bit q
-#pragma unroll
-                                for (int m = 0; m < (1 << q); ++m) {
-                                    U[m + (1 << q)] = U[m] * x[q];
-                                    U[m] = U[m] * omx[q];
+                                for (int q = 0; q < k; ++q) {
+                                    x[q] = comp4(xv[q], r);
+                                    omx[q] = 1.0f - x[q];
                                 }
-                            }
-                            V[0] = omx[KL];
-                            V[1] = x[KL];
+                                float U[NU], V[NV];
+                                U[0] = comp4(gv[t], r);
 #pragma unroll
-                            for (int q = KL + 1; q < k; ++q) {   // slot q doubles V: index bit q - KL
+                                for (int q = 0; q < KL; ++q) {   // slot q doubles U: index bit q
 #pragma unroll
-                                for (int m = 0; m < (1 << (q - KL)); ++m) {
-                                    V[m + (1 << (q - KL))] = V[m] * x[q];
-                                    V[m] = V[m] * omx[q];
+                                    for (int m = 0; m < (1 << q); ++m) {
+                                        U[m + (1 << q)] = U[m] * x[q];
+                                        U[m] = U[m] * omx[q];
+                                    }
                                 }
+                                V[0] = omx[KL];
+                                V[1] = x[KL];
+#pragma unroll
+                                for (int q = KL + 1; q < k; ++q) {   // slot q doubles V: index bit q - KL
+#pragma unroll
+                                    for (int m = 0; m < (1 << (q - KL)); ++m) {
+                                        V[m + (1 << (q - KL))] = V[m] * x[q];
+                                        V[m] = V[m] * omx[q];
+                                    }
+                                }
+#pragma unroll
+                                for (int b = 0; b < NV; ++b)
+#pragma unroll
+                                    for (int a = 0; a < NU; ++a) acc[a + b * NU] = fmaf(U[a], V[b], acc[a + b * NU]);
                             }
-#pragma unroll
-                            for (int b = 0; b < NV; ++b)
-#pragma unroll
-                                for (int a = 0; a < NU; ++a) acc[a + b * NU] = fmaf(U[a], V[b], acc[a + b * NU]);
                         }
                     }
                     rb = (rb + 1 == kTStages) ? 0 : rb + 1;
@@ -443,6 +455,7 @@ lut_theta_src_kernel(const TX* __restrict__ X, int w_in, long long B, const int*
             }
         }
         // the node's dtheta: butterfly over the lanes, then t (1 - t)
+        if constexpr (BIN) corner_take<K>(corners, acc);
         reduce_scatter<K, 16>(acc, lane);
         constexpr int NF = K >= 32 ? K / 32 : 1;   // entries per lane
         constexpr int SH = K >= 32 ? 0 : 5 - k;    // lanes sharing an entry (K < 32)
@@ -458,266 +471,212 @@ lut_theta_src_kernel(const TX* __restrict__ X, int w_in, long long B, const int*
     cp_async_wait<0>();
 }
 
-// Terms source with the term rows streamed through the cp.async ring: a
-// ring slot holds the node's k input rows of one stage (fp32 or bytes) and
-// the stage's segments of its first kRingTerms term rows (fp32, in CSR
-// order), copied kTStages - 1 stages ahead like the input rows, so the term
-// rows are in flight without holding registers; the term rows of a node
-// with more consumers than kRingTerms are read directly after those (in
-// CSR order: the sum keeps the order of bitlogic_csr_reduce).  The issue
-// stream keeps the term row ids of its node one per lane, and loads the ids
-// of the node after it ahead, like the input rows.
-#ifndef BITLOGIC_TERMS_RING_ROWS
-#define BITLOGIC_TERMS_RING_ROWS 10
+// Byte rows (binary wires) with the output gradient from dY rows or from
+// the next layer's per-edge terms: the one-hot table gradient, streaming
+// form.  The arithmetic per sample is one add, so the kernel moves data: a
+// warp per node over the whole batch in chunks of kBytesChunk stages (128
+// samples each, 4 per lane); per chunk each lane loads its output-gradient
+// segments (a dY row, or the node's consumer term rows summed in increasing
+// CSR position, the order of bitlogic_csr_reduce) and its k input words per
+// stage straight into registers, so a warp has a few KB of independent loads
+// in flight and no ring to wait on, and then adds each sample's gradient to
+// the entry its bits select in the lane's column of a shared [2^k][32] array.
+// The lane visits its samples in the order of the fp32 kernels and the lanes
+// are combined by the same butterfly, so dtheta is theirs bit for bit.
+#ifndef BITLOGIC_BYTES_WARPS
+#define BITLOGIC_BYTES_WARPS 2
 #endif
-constexpr int kRingTerms = BITLOGIC_TERMS_RING_ROWS;
-static_assert(kRingTerms >= 1 && kRingTerms <= 32, "term rows per ring slot");
-constexpr int kTermsRingBlocks = 12;   // one-warp blocks per SM (shared memory: ~17.7 KB per warp)
+#ifndef BITLOGIC_BYTES_CHUNK
+#define BITLOGIC_BYTES_CHUNK 4
+#endif
+#ifndef BITLOGIC_BYTES_STREAM
+#define BITLOGIC_BYTES_STREAM 1
+#endif
+#ifndef BITLOGIC_BYTES_UNROLL
+#define BITLOGIC_BYTES_UNROLL 4
+#endif
+constexpr int kBytesWarps = BITLOGIC_BYTES_WARPS;   // warps (nodes) per block
+constexpr int kBytesChunk = BITLOGIC_BYTES_CHUNK;   // stages per chunk
+constexpr int kBytesUnroll = BITLOGIC_BYTES_UNROLL;   // term rows whose loads are issued together
 
-template <int k, typename TX>
-__host__ __device__ constexpr int terms_slot_bytes() {
-    return k * kTStageSamples * (int)sizeof(TX) + kRingTerms * kTStageSamples * (int)sizeof(float);
-}
-
-template <int k, typename TX>
-__global__ void __launch_bounds__(32, kTermsRingBlocks)
-lut_theta_terms_ring_kernel(const TX* __restrict__ X, int w_in, long long B, const int* __restrict__ conn,
-                            const float* __restrict__ theta, int w, GradIn gi, float* __restrict__ dtheta,
-                            float* __restrict__ dY_out) {
-    constexpr int K = 1 << k, KL = k / 2, NU = 1 << KL, NV = 1 << (k - KL);
-    constexpr int CH = kTStageSamples;
-    constexpr int SLOT = terms_slot_bytes<k, TX>();
+template <int k, bool TERMS>
+__global__ void __launch_bounds__(kBytesWarps * 32)
+lut_theta_bytes_kernel(const uint8_t* __restrict__ X, int w_in, long long B, const int* __restrict__ conn,
+                       const float* __restrict__ theta, int w, GradIn gi, float* __restrict__ dtheta,
+                       float* __restrict__ dY_out) {
+    constexpr int K = 1 << k, CH = kTStageSamples;
     extern __shared__ __align__(16) unsigned char smem_raw[];
-    const int lane = threadIdx.x & 31;
-    const int G = gridDim.x;
-    const int jfirst = blockIdx.x;
-    const int nst = (int)((B + CH - 1) / CH);
-    const int n_terms = gi.n_terms;
-
-    // a node's input rows, CSR range and the ids of its first 32 term rows
-    struct NodeIn {
-        int r[k];
-        int e0, deg, id;
-    };
-    auto node_in = [&](int j, NodeIn& nd) {
-        bool bad = false;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int j = blockIdx.x * kBytesWarps + warp;
+    if (j >= w) return;   // warp-uniform; the block has no barrier
+    float* col = reinterpret_cast<float*>(smem_raw) + warp * K * 32 + lane;
 #pragma unroll
-        for (int i = 0; i < k; ++i) {
-            int c = __ldg(conn + (long long)j * k + i);
-            if ((unsigned)c >= (unsigned)w_in) {
-                bad = true;
-                c = 0;
-            }
-            nd.r[i] = c;
+    for (int a = 0; a < K; ++a) col[a * 32] = 0.f;
+    bool bad = false;
+    const uint8_t* xr[k];
+#pragma unroll
+    for (int i = 0; i < k; ++i) {
+        int c = __ldg(conn + (long long)j * k + i);
+        if ((unsigned)c >= (unsigned)w_in) {
+            bad = true;
+            c = 0;
         }
-        int e0 = __ldg(gi.off + j), e1 = __ldg(gi.off + j + 1);
-        if (e0 < 0 || e1 < e0 || e1 > n_terms) {
+        xr[i] = X + (long long)c * B + 4 * lane;
+    }
+    // the node's term rows: CSR positions e0 .. e0 + deg - 1, ids of the
+    // first 32 one per lane
+    int e0 = 0, deg = 0, my_id = -1;
+    if constexpr (TERMS) {
+        int e1;
+        e0 = __ldg(gi.off + j);
+        e1 = __ldg(gi.off + j + 1);
+        if (e0 < 0 || e1 < e0 || e1 > gi.n_terms) {
             bad = true;
             e0 = e1 = 0;
         }
-        nd.e0 = e0;
-        nd.deg = e1 - e0;
-        nd.id = -1;
-        if (lane < nd.deg) {
-            const int p = e0 + lane;
-            nd.id = gi.edge ? __ldg(gi.edge + p) : p;
-            if ((unsigned)nd.id >= (unsigned)n_terms) {
+        deg = e1 - e0;
+        if (lane < deg) {
+            my_id = gi.edge ? __ldg(gi.edge + e0 + lane) : e0 + lane;
+            if ((unsigned)my_id >= (unsigned)gi.n_terms) {
                 bad = true;
-                nd.id = -1;
+                my_id = -1;
             }
         }
-        if (__any_sync(0xffffffffu, bad) && lane == 0) flag_index_error();
-    };
-
-    // issue stream: stage si of node ji, kTStages - 1 stages ahead of the
-    // compute stream
-    int ji = jfirst, si = 0, ib = 0;
-    NodeIn ni, nn;
-    if (ji < w) node_in(ji, ni);
-    if (ji + G < w) node_in(ji + G, nn);
-    auto issue = [&]() {
-        if (ji < w) {
-            const long long s4 = (long long)si * CH + 4 * lane;
-            const bool in = s4 < B;
-            unsigned char* slot = smem_raw + ib * SLOT;
-            TX* xb = reinterpret_cast<TX*>(slot) + 4 * lane;
-            if (in) {
+    }
+    if (__any_sync(0xffffffffu, bad) && lane == 0) flag_index_error();
+    const float* grow = TERMS ? nullptr : gi.dY + (long long)(j / gi.group) * B + 4 * lane;
+    const int nst = (int)((B + CH - 1) / CH);
+#pragma unroll 1
+    for (int c0 = 0; c0 < nst; c0 += kBytesChunk) {
+        // stage c0 + c of this lane: samples (c0 + c) * CH + 4 lane .. + 3,
+        // all in range when the first is (B % 4 == 0)
+        bool in[kBytesChunk];
 #pragma unroll
-                for (int r = 0; r < k; ++r) copy_row_part(xb + r * CH, X + (long long)ni.r[r] * B + s4);
-            }
-            float* tb = reinterpret_cast<float*>(slot + k * CH * sizeof(TX)) + 4 * lane;
-            const int nr = min(ni.deg, kRingTerms);
-            for (int t = 0; t < nr; ++t) {   // warp-uniform count; every lane takes the shuffle
-                const int id = __shfl_sync(0xffffffffu, ni.id, t);
-                if (in && id >= 0) cp_async16(tb + t * CH, gi.terms + (long long)id * B + s4);
-            }
-            if (++si == nst) {
-                si = 0;
-                ji += G;
-                ni = nn;
-                if (ji + G < w) node_in(ji + G, nn);
-            }
-        }
-        cp_async_commit();
-        ib = (ib + 1 == kTStages) ? 0 : ib + 1;
-    };
-#pragma unroll 1
-    for (int i = 0; i < kTStages - 1; ++i) issue();
-
-    int rb = 0;
-#pragma unroll 1
-    for (int j = jfirst; j < w; j += G) {
-        // the compute stream's own copy of the node's CSR range and ids (the
-        // issue stream has moved on by up to kTStages - 1 stages)
-        NodeIn nc;
-        node_in(j, nc);
-        float acc[K];
+        for (int c = 0; c < kBytesChunk; ++c) in[c] = c0 + c < nst && (long long)(c0 + c) * CH + 4 * lane < B;
+        uint32_t xw[kBytesChunk][k];
 #pragma unroll
-        for (int a = 0; a < K; ++a) acc[a] = 0.f;
-#pragma unroll 1
-        for (int sc = 0; sc < nst; ++sc) {
-            issue();
-            cp_async_wait<kTStages - 1>();
-            const long long s4 = (long long)sc * CH + 4 * lane;   // this lane's 4 samples
-            const bool in = s4 < B;   // B % 4 == 0: all four samples are in range
-            const unsigned char* slot = smem_raw + rb * SLOT;
-            const float* tb = reinterpret_cast<const float*>(slot + k * CH * sizeof(TX)) + 4 * lane;
-            // the output gradient: ring rows, then any further rows, in CSR
-            // order (warp-uniform loops: every lane takes the shuffles)
-            float4 g = make_float4(0.f, 0.f, 0.f, 0.f);
-            const int nr = min(nc.deg, kRingTerms);
-            for (int t = 0; t < nr; ++t) {
-                const int id = __shfl_sync(0xffffffffu, nc.id, t);
-                if (in && id >= 0) {
-                    const float4 v = *reinterpret_cast<const float4*>(tb + t * CH);
-                    g.x += v.x; g.y += v.y; g.z += v.z; g.w += v.w;
-                }
-            }
-            for (int t = kRingTerms; t < nc.deg; ++t) {
+        for (int c = 0; c < kBytesChunk; ++c)
+#pragma unroll
+            for (int i = 0; i < k; ++i)
+                xw[c][i] = in[c] ? __ldg(reinterpret_cast<const uint32_t*>(xr[i] + (long long)(c0 + c) * CH)) : 0u;
+        float4 g[kBytesChunk];
+#pragma unroll
+        for (int c = 0; c < kBytesChunk; ++c) g[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if constexpr (TERMS) {
+#pragma unroll kBytesUnroll
+            for (int e = 0; e < deg; ++e) {   // warp-uniform count; every lane takes the shuffle
                 int id;
-                if (t < 32) {
-                    id = __shfl_sync(0xffffffffu, nc.id, t);
+                if (e < 32) {
+                    id = __shfl_sync(0xffffffffu, my_id, e);
                 } else {
-                    const int p = nc.e0 + t;
-                    id = gi.edge ? __ldg(gi.edge + p) : p;
-                    if ((unsigned)id >= (unsigned)n_terms) {
+                    id = gi.edge ? __ldg(gi.edge + e0 + e) : e0 + e;
+                    if ((unsigned)id >= (unsigned)gi.n_terms) {
                         if (lane == 0) flag_index_error();
                         id = -1;
                     }
                 }
-                if (in && id >= 0) {
-                    const float4 v = ldg4t(gi.terms + (long long)id * B + s4);
-                    g.x += v.x; g.y += v.y; g.z += v.z; g.w += v.w;
-                }
-            }
-            if (in) {
-                if (dY_out) *reinterpret_cast<float4*>(dY_out + (long long)j * B + s4) = g;
-                const TX* xb = reinterpret_cast<const TX*>(slot) + 4 * lane;
-                float4 xv[k];
+                if (id >= 0) {
+                    const float* row = gi.terms + (long long)id * B + 4 * lane;
 #pragma unroll
-                for (int q = 0; q < k; ++q) xv[q] = read_row_part(xb + q * CH);
-#pragma unroll
-                for (int r = 0; r < 4; ++r) {
-                    float x[k], omx[k];
-#pragma unroll
-                    for (int q = 0; q < k; ++q) {
-                        x[q] = comp4(xv[q], r);
-                        omx[q] = 1.0f - x[q];
-                    }
-                    float U[NU], V[NV];
-                    U[0] = comp4(g, r);
-#pragma unroll
-                    for (int q = 0; q < KL; ++q) {   // slot q doubles U: index bit q
-#pragma unroll
-                        for (int m = 0; m < (1 << q); ++m) {
-                            U[m + (1 << q)] = U[m] * x[q];
-                            U[m] = U[m] * omx[q];
+                    for (int c = 0; c < kBytesChunk; ++c) {
+                        if (in[c]) {
+#if BITLOGIC_BYTES_STREAM
+                            const float4 v = __ldcs(reinterpret_cast<const float4*>(row + (long long)(c0 + c) * CH));
+#else
+                            const float4 v = ldg4t(row + (long long)(c0 + c) * CH);
+#endif
+                            g[c].x += v.x; g[c].y += v.y; g[c].z += v.z; g[c].w += v.w;
                         }
                     }
-                    V[0] = omx[KL];
-                    V[1] = x[KL];
-#pragma unroll
-                    for (int q = KL + 1; q < k; ++q) {   // slot q doubles V: index bit q - KL
-#pragma unroll
-                        for (int m = 0; m < (1 << (q - KL)); ++m) {
-                            V[m + (1 << (q - KL))] = V[m] * x[q];
-                            V[m] = V[m] * omx[q];
-                        }
-                    }
-#pragma unroll
-                    for (int b = 0; b < NV; ++b)
-#pragma unroll
-                        for (int a = 0; a < NU; ++a) acc[a + b * NU] = fmaf(U[a], V[b], acc[a + b * NU]);
                 }
             }
-            rb = (rb + 1 == kTStages) ? 0 : rb + 1;
+        } else {
+#pragma unroll
+            for (int c = 0; c < kBytesChunk; ++c)
+                if (in[c]) g[c] = ldg4t(grow + (long long)(c0 + c) * CH);
         }
-        // the node's dtheta: butterfly over the lanes, then t (1 - t)
-        reduce_scatter<K, 16>(acc, lane);
-        constexpr int NF = K >= 32 ? K / 32 : 1;   // entries per lane
-        constexpr int SH = K >= 32 ? 0 : 5 - k;    // lanes sharing an entry (K < 32)
-        if ((lane & ((1 << SH) - 1)) == 0) {
 #pragma unroll
-            for (int i = 0; i < NF; ++i) {
-                const int a = K >= 32 ? lane * NF + i : lane >> SH;
-                const float t = sigmoidf(__ldg(theta + (long long)j * K + a));
-                dtheta[(long long)j * K + a] = t * (1.0f - t) * acc[i];
+        for (int c = 0; c < kBytesChunk; ++c) {
+            if (in[c]) {
+                if (dY_out) *reinterpret_cast<float4*>(dY_out + (long long)j * B + (long long)(c0 + c) * CH + 4 * lane) = g[c];
+                uint32_t v = xw[c][k - 1] & 0x01010101u;
+#pragma unroll
+                for (int i = k - 2; i >= 0; --i) v = (v << 1) | (xw[c][i] & 0x01010101u);
+                corner_add4(col, v, g[c]);
             }
         }
     }
-    cp_async_wait<0>();
+    // the node's dtheta: butterfly over the lanes, then t (1 - t)
+    float acc[K];
+    corner_take<K>(col, acc);
+    reduce_scatter<K, 16>(acc, lane);
+    constexpr int NF = K >= 32 ? K / 32 : 1;   // entries per lane
+    constexpr int SH = K >= 32 ? 0 : 5 - k;    // lanes sharing an entry (K < 32)
+    if ((lane & ((1 << SH) - 1)) == 0) {
+#pragma unroll
+        for (int i = 0; i < NF; ++i) {
+            const int a = K >= 32 ? lane * NF + i : lane >> SH;
+            const float t = sigmoidf(__ldg(theta + (long long)j * K + a));
+            dtheta[(long long)j * K + a] = t * (1.0f - t) * acc[i];
+        }
+    }
 }
 
-template <int k, typename TX>
-int launch_terms_ring(const TX* X, int w_in, long long B, const int* conn, const float* theta, int w,
-                      const GradIn& gi, float* dtheta, float* dY_out, cudaStream_t st) {
-    constexpr int smem = kTStages * terms_slot_bytes<k, TX>();
-    auto kern = lut_theta_terms_ring_kernel<k, TX>;
-    if (smem > 40 * 1024 && cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
-        return BITLOGIC_ERR_CUDA;
-    const long long resident = (long long)sm_count() * kTermsRingBlocks;
-    const long long blocks = w < resident ? w : resident;
-    kern<<<(unsigned)blocks, 32, smem, st>>>(X, w_in, B, conn, theta, w, gi, dtheta, dY_out);
+template <int k>
+int launch_bytes(bool terms, const uint8_t* X, int w_in, long long B, const int* conn, const float* theta, int w,
+                 const GradIn& gi, float* dtheta, float* dY_out, cudaStream_t st) {
+    constexpr int smem = kBytesWarps * (1 << k) * 32 * (int)sizeof(float);
+    const unsigned blocks = (unsigned)((w + kBytesWarps - 1) / kBytesWarps);
+    if (smem > 40 * 1024) {
+        auto kt = lut_theta_bytes_kernel<k, true>;
+        auto kr = lut_theta_bytes_kernel<k, false>;
+        if (cudaFuncSetAttribute(kt, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess ||
+            cudaFuncSetAttribute(kr, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
+            return BITLOGIC_ERR_CUDA;
+    }
+    if (terms)
+        lut_theta_bytes_kernel<k, true><<<blocks, kBytesWarps * 32, smem, st>>>(X, w_in, B, conn, theta, w, gi,
+                                                                              dtheta, dY_out);
+    else
+        lut_theta_bytes_kernel<k, false><<<blocks, kBytesWarps * 32, smem, st>>>(X, w_in, B, conn, theta, w, gi,
+                                                                               dtheta, dY_out);
     return launch_status();
 }
 
-template <int k, int ku, typename TX, int SRC>
-int launch_src(const TX* X, int w_in, long long B, const int* conn, const float* theta, int w, const GradIn& gi,
-               int node, float* dtheta, float* dY_out, cudaStream_t st) {
-    constexpr int smem = ring_bytes_per_warp<TX>(k);
-    auto kern = lut_theta_src_kernel<k, ku, TX, SRC>;
+template <int k, int ku, typename TX>
+int launch_through(const TX* X, int w_in, long long B, const int* conn, const float* theta, int w,
+                   const GradIn& gi, int node, float* dtheta, float* dY_out, cudaStream_t st) {
+    constexpr int smem = ring_bytes_per_warp<TX>(k) + corner_bytes<TX>(k);
+    auto kern = lut_theta_through_kernel<k, ku, TX>;
     if (smem > 40 * 1024 && cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
         return BITLOGIC_ERR_CUDA;
     // one wave of persistent one-warp blocks (nodes dealt round-robin)
-    const long long resident = (long long)sm_count() * grad_min_blocks<k, SRC>();
+    const long long resident = (long long)sm_count() * kTMinBlocks;
     const long long blocks = w < resident ? w : resident;
     kern<<<(unsigned)blocks, 32, smem, st>>>(X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out);
     return launch_status();
 }
 
 template <int k, typename TX>
-int launch_src_k(int src, int up_k, const TX* X, int w_in, long long B, const int* conn, const float* theta, int w,
-                 const GradIn& gi, int node, float* dtheta, float* dY_out, cudaStream_t st) {
-    if (src == kSrcRows) return launch_src<k, 1, TX, kSrcRows>(X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
-    // the terms source streams its rows through the ring kernel
-    if (src == kSrcTerms) return launch_terms_ring<k, TX>(X, w_in, B, conn, theta, w, gi, dtheta, dY_out, st);
+int launch_through_k(int up_k, const TX* X, int w_in, long long B, const int* conn, const float* theta, int w,
+                     const GradIn& gi, int node, float* dtheta, float* dY_out, cudaStream_t st) {
     switch (up_k) {
-        case 1: return launch_src<k, 1, TX, kSrcThrough>(X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
-        case 2: return launch_src<k, 2, TX, kSrcThrough>(X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
-        default: return launch_src<k, 3, TX, kSrcThrough>(X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
+        case 1: return launch_through<k, 1, TX>(X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
+        case 2: return launch_through<k, 2, TX>(X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
+        default: return launch_through<k, 3, TX>(X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
     }
 }
 
 template <typename TX>
-int run_src(int src, int up_k, const TX* X, int w_in, long long B, const int* conn, const float* theta, int w,
-            int k, const GradIn& gi, int node, float* dtheta, float* dY_out, cudaStream_t st) {
+int run_through(int up_k, const TX* X, int w_in, long long B, const int* conn, const float* theta, int w, int k,
+                const GradIn& gi, int node, float* dtheta, float* dY_out, cudaStream_t st) {
     switch (k) {
-        case 1: return launch_src_k<1, TX>(src, up_k, X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
-        case 2: return launch_src_k<2, TX>(src, up_k, X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
-        case 3: return launch_src_k<3, TX>(src, up_k, X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
-        case 4: return launch_src_k<4, TX>(src, up_k, X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
-        case 5: return launch_src_k<5, TX>(src, up_k, X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
-        default: return launch_src_k<6, TX>(src, up_k, X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
+        case 1: return launch_through_k<1, TX>(up_k, X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
+        case 2: return launch_through_k<2, TX>(up_k, X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
+        case 3: return launch_through_k<3, TX>(up_k, X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
+        case 4: return launch_through_k<4, TX>(up_k, X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
+        case 5: return launch_through_k<5, TX>(up_k, X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
+        default: return launch_through_k<6, TX>(up_k, X, w_in, B, conn, theta, w, gi, node, dtheta, dY_out, st);
     }
 }
 
@@ -771,7 +730,7 @@ static int backward_through(const TX* X, int32_t w_in, int64_t B, const int32_t*
     gi.up_w = up_w;
     gi.up_dY = up_dY;
     gi.up_group = up_group;
-    return run_src<TX>(kSrcThrough, up_k, X, w_in, B, conn, theta, w, k, gi, node, dtheta, dY_out, stream);
+    return run_through<TX>(up_k, X, w_in, B, conn, theta, w, k, gi, node, dtheta, dY_out, stream);
 }
 
 extern "C" int bitlogic_lut_backward_through(const float* X, int32_t w_in, int64_t B, const int32_t* conn,
@@ -823,6 +782,12 @@ extern "C" int bitlogic_lut_backward_u8(const uint8_t* X, int32_t w_in, int64_t 
     gi.n_terms = up_edges;
     gi.off = up_off;
     gi.edge = up_edge;
-    return run_src<uint8_t>(terms ? kSrcTerms : kSrcRows, 1, X, w_in, B, conn, theta, w, k, gi, node, dtheta, dY_out,
-                            stream);
+    switch (k) {
+        case 1: return launch_bytes<1>(terms, X, w_in, B, conn, theta, w, gi, dtheta, dY_out, stream);
+        case 2: return launch_bytes<2>(terms, X, w_in, B, conn, theta, w, gi, dtheta, dY_out, stream);
+        case 3: return launch_bytes<3>(terms, X, w_in, B, conn, theta, w, gi, dtheta, dY_out, stream);
+        case 4: return launch_bytes<4>(terms, X, w_in, B, conn, theta, w, gi, dtheta, dY_out, stream);
+        case 5: return launch_bytes<5>(terms, X, w_in, B, conn, theta, w, gi, dtheta, dY_out, stream);
+        default: return launch_bytes<6>(terms, X, w_in, B, conn, theta, w, gi, dtheta, dY_out, stream);
+    }
 }

@@ -24,7 +24,7 @@ from . import (NODE_FORMS, bitlogic_adamw_update, bitlogic_binarize_tables, bitl
                bitlogic_lut_backward_u8, bitlogic_lut_forward_node,
                bitlogic_pack_bits, bitlogic_route_backward, bitlogic_route_backward_u8, bitlogic_route_forward,
                bitlogic_route_forward_u8, bitlogic_route_snap, bitlogic_encode_thermometer_u8,
-               bitlogic_encode_thermometer_both)
+               bitlogic_lut_forward_u8)
 
 
 def _nomark(name: str) -> None:
@@ -173,13 +173,15 @@ class TrainStep:
     * otherwise a CSR reduction of the terms into ``dy1``, which the
       dtheta-only layer-1 backward reads.
 
-    On the first two routes the layer-1 backward can read the encoder's wires
-    as bytes (``bytes1``; the encoder then writes, in one pass, both the fp32
-    rows the forward reads and byte rows): the node gathers a quarter of the
-    data.  The results are the same bit for bit; at the CIFAR shapes on
-    GB300 the step was no faster (7.025 against 7.028 ms at the CIFAR-100
-    shape, 1.842 against 1.818 ms at the CIFAR-10 shape), so it is off by
-    default.  Set
+    Layer 1 reads the encoder's wires as bytes (``bytes1``, the default when
+    B % 4 == 0 and no layer-1 input gradient is wanted): its inputs are
+    binary, so every corner weight of the relaxed table is 0 or 1 and the
+    layer-1 forward is a table lookup (bitlogic_lut_forward_u8) and its table
+    gradient adds each sample's gradient to the one entry the sample selects
+    (bitlogic_lut_backward_u8 / _through on byte rows); the encoder then
+    writes byte rows only, and ``bits`` is that uint8 tensor.  The table
+    gradient equals the fp32-row form bit for bit; the forward returns the
+    table entry itself, which the fp32 lerp tree reaches up to rounding.  Set
     ``keep_dy1`` to also write dY1 (e.g. to check it).  ``node`` picks the
     LightLUT form of both layers: "soft", or "st" (hard table samples in the
     forward, straight-through gradient to the logits)."""
@@ -206,7 +208,6 @@ class TrainStep:
         f32 = dict(dtype=torch.float32, device=dev)
         self.x = torch.zeros(B, d, dtype=torch.uint8, device=dev)
         self.labels = torch.zeros(B, dtype=torch.int32, device=dev)
-        self.bits = torch.empty(net.w_in, B, **f32)
         self.y1 = torch.empty(net.w1, B, **f32)
         self.y2 = torch.empty(net.w2, B, **f32)
         self.logits = torch.empty(B, C, **f32)
@@ -214,11 +215,12 @@ class TrainStep:
         self.dyg = torch.empty(C, B, **f32)          # gradient row shared by each class's nodes
         self.fuse_dy1 = bool(fuse_dy1) and not self.through
         if bytes1 is None:
-            bytes1 = False   # measured no faster on GB300 at the CIFAR shapes (see the class docstring)
-        if bytes1 and not (self.fuse_dy1 or self.through):
-            raise ValueError("byte wires for layer 1 need the fused or the through route")
+            bytes1 = B % 4 == 0 and not want_dx1
+        if bytes1 and (B % 4 != 0 or want_dx1):
+            raise ValueError("byte wires for layer 1 need B % 4 == 0 and no layer-1 input gradient")
         self.bytes1 = bool(bytes1)
-        self.bits8 = torch.empty(net.w_in, B, dtype=torch.uint8, device=dev) if self.bytes1 else None
+        # the encoder's output: byte rows (bytes1) or fp32 rows
+        self.bits = torch.empty(net.w_in, B, dtype=torch.uint8 if self.bytes1 else torch.float32, device=dev)
         # per-edge terms stored in CSR order (each input's terms contiguous,
         # read without the edge map) instead of edge order
         self.csr_order = bool(csr_order)
@@ -238,12 +240,14 @@ class TrainStep:
 
     def forward(self, stream=None, mark=_nomark):
         n = self.net
-        if self.bits8 is not None:
-            bitlogic_encode_thermometer_both(self.x, self.thr, self.bits, self.bits8, stream)
+        if self.bytes1:
+            bitlogic_encode_thermometer_u8(self.x, self.thr, self.bits, stream)
+            mark("encode")
+            bitlogic_lut_forward_u8(self.bits, n.conn1, n.theta1, self.y1, self.node, stream)
         else:
             bitlogic_encode_thermometer(self.x, self.thr, self.bits, stream)
-        mark("encode")
-        bitlogic_lut_forward_node(self.bits, n.conn1, n.theta1, self.y1, self.node, stream)
+            mark("encode")
+            bitlogic_lut_forward_node(self.bits, n.conn1, n.theta1, self.y1, self.node, stream)
         mark("forward1")
         bitlogic_lut_forward_node(self.y1, n.conn2, n.theta2, self.y2, self.node, stream)
         mark("forward2")
@@ -262,7 +266,7 @@ class TrainStep:
             bitlogic_lut_backward_node(self.y1, n.conn2, n.theta2, self.dth2, nd, dY=self.dyg, dy_group=g,
                                        stream=stream)
             mark("backward2")
-            bitlogic_lut_backward_through(self.bits8 if self.bytes1 else self.bits, n.conn1, n.theta1, self.dth1,
+            bitlogic_lut_backward_through(self.bits, n.conn1, n.theta1, self.dth1,
                                           self.y1, n.conn2, n.theta2, self.dyg, g, n.off2, n.edge2, node=nd,
                                           dY_out=self.dy1, stream=stream)
             mark("backward1")
@@ -274,7 +278,7 @@ class TrainStep:
         pos1 = n.pos1 if (co and self.edges1 is not None) else None
         edge2 = None if co else n.edge2
         if self.fuse_dy1 and self.bytes1:
-            bitlogic_lut_backward_u8(self.bits8, n.conn1, n.theta1, self.dth1, nd, up_terms=self.edges2,
+            bitlogic_lut_backward_u8(self.bits, n.conn1, n.theta1, self.dth1, nd, up_terms=self.edges2,
                                      up_off=n.off2, up_edge=edge2, dY_out=self.dy1, stream=stream)
         elif self.fuse_dy1:
             bitlogic_lut_backward_node(self.bits, n.conn1, n.theta1, self.dth1, nd, up_terms=self.edges2,
@@ -283,8 +287,11 @@ class TrainStep:
         else:
             bitlogic_csr_reduce(self.edges2, n.off2, edge2, self.dy1, stream)
             mark("csr2")
-            bitlogic_lut_backward_node(self.bits, n.conn1, n.theta1, self.dth1, nd, dY=self.dy1,
-                                       edge_terms=self.edges1, edge_pos=pos1, stream=stream)
+            if self.bytes1:
+                bitlogic_lut_backward_u8(self.bits, n.conn1, n.theta1, self.dth1, nd, dY=self.dy1, stream=stream)
+            else:
+                bitlogic_lut_backward_node(self.bits, n.conn1, n.theta1, self.dth1, nd, dY=self.dy1,
+                                           edge_terms=self.edges1, edge_pos=pos1, stream=stream)
         mark("backward1")
         if self.dbits is not None:
             bitlogic_csr_reduce(self.edges1, n.off1, None if co else n.edge1, self.dbits, stream)

@@ -183,6 +183,17 @@ def test_host_validation_returns_before_any_launch():
                     None, None) == -12
     with pytest.raises(ValueError):
         bl.bitlogic_lut_forward_node(None, None, None, None, node="hard")
+    # forward on byte rows: node form, fan-in, shapes, NULLs (B = 0 is a no-op)
+    fwd_u8 = lib.bitlogic_lut_forward_u8
+    assert fwd_u8(fake, 8, 64, fake, fake, 4, 2, 2, fake, None) == -12
+    assert fwd_u8(fake, 8, 64, fake, fake, 4, 7, 0, fake, None) == -3
+    assert fwd_u8(fake, 8, 64, fake, fake, 4, 9, 0, fake, None) == -3   # k > w_in
+    assert fwd_u8(fake, 0, 64, fake, fake, 4, 2, 0, fake, None) == -2
+    assert fwd_u8(fake, 8, -1, fake, fake, 4, 2, 0, fake, None) == -2
+    assert fwd_u8(None, 8, 64, fake, fake, 4, 2, 0, fake, None) == -1
+    assert fwd_u8(fake, 8, 64, fake, fake, 4, 2, 0, None, None) == -1
+    assert fwd_u8(fake, 8, 64, None, fake, 4, 2, 0, fake, None) == -1
+    assert fwd_u8(None, 8, 0, fake, fake, 4, 2, 0, None, None) == 0
 
 
 @pytest.mark.parametrize("n,b,seed", [(1, 1, 0), (5, 4, 1), (1000, 8, 2), (65537, 32, 3), (300, 15, 4)])

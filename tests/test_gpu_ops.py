@@ -126,6 +126,75 @@ def test_lut_forward_unaligned_scalar_path():
     check_fwd(Y, oracle.lut_forward(X.astype(np.float64), conn, theta), "Y")
 
 
+# ------------------------------------------- soft forward on byte rows --
+#
+# Binary wires as bytes: on binary inputs the corner weights are one-hot, so
+# the layer returns the table entry each sample's input bits select (the
+# oracle's multilinear form reaches it exactly on binary inputs).
+
+@pytest.mark.parametrize("k,w_in,w,B", SHAPES)
+@pytest.mark.parametrize("node", ["soft", "st"])
+def test_lut_forward_u8(k, w_in, w, B, node):
+    Xb = synth.binary_activations(w_in, B, seed=k + 3 * B)
+    conn = synth.connectivity(w, k, w_in, seed=w + 7)
+    theta = synth.table_logits(w, 1 << k, seed=k + 11)
+    theta[0, :] = 0.0                    # ties sample 0 (st: [0 > 0] = 0)
+    Y = torch.full((w, B), np.nan, device="cuda")
+    bl.bitlogic_lut_forward_u8(dev(Xb.astype(np.uint8)), dev(conn), dev(theta), Y, node=node)
+    want = oracle.lut_forward(Xb.astype(np.float64), conn, theta, node)
+    if node == "st":
+        check_exact(Y.cpu().numpy().astype(np.float64), want, "Y")
+    else:
+        check_fwd(Y, want, "Y")
+    # the table entry itself: the sigmoid the fp32 kernels take, bit for bit
+    idx = np.zeros((w, B), dtype=np.int64)
+    for i in range(k):
+        idx += Xb[conn[:, i]].astype(np.int64) << i
+    tab = torch.sigmoid(dev(theta)).cpu().numpy() if node == "soft" else (theta > 0).astype(np.float32)
+    entries = np.take_along_axis(tab, idx, axis=1)
+    if node == "soft":
+        check_fwd(Y, entries.astype(np.float64), "Y vs the selected entries")
+    else:
+        check_exact(Y.cpu().numpy(), entries, "Y vs the selected entries")
+    no_device_error()
+
+
+def test_lut_forward_u8_scalar_path_and_lowest_bit():
+    # a view one byte into an allocation (and B % 4 != 0) takes the scalar
+    # form; bytes other than 0 and 1 are read by their lowest bit
+    k, w_in, w, B = 6, 50, 20, 67
+    rng = np.random.default_rng(5)
+    X = rng.integers(0, 256, size=(w_in, B), dtype=np.uint8)
+    conn = synth.connectivity(w, k, w_in, seed=6)
+    theta = synth.table_logits(w, 64, seed=7)
+    big = torch.zeros(w_in * B + 1, dtype=torch.uint8, device="cuda")
+    big[1:] = dev(X).reshape(-1)
+    Y = torch.empty(w, B, device="cuda")
+    bl.bitlogic_lut_forward_u8(big[1:].view(w_in, B), dev(conn), dev(theta), Y)
+    check_fwd(Y, oracle.lut_forward((X & 1).astype(np.float64), conn, theta), "Y")
+    for B2 in (64, 1024):   # the vector form with the same bytes
+        X2 = rng.integers(0, 256, size=(w_in, B2), dtype=np.uint8)
+        Y2 = torch.empty(w, B2, device="cuda")
+        bl.bitlogic_lut_forward_u8(dev(X2), dev(conn), dev(theta), Y2)
+        check_fwd(Y2, oracle.lut_forward((X2 & 1).astype(np.float64), conn, theta), "Y (vector)")
+    no_device_error()
+
+
+def test_lut_forward_u8_out_of_range_row_is_flagged():
+    k, w_in, w, B = 3, 16, 8, 128
+    Xb = synth.binary_activations(w_in, B, seed=9)
+    conn = synth.connectivity(w, k, w_in, seed=10)
+    conn[3, 1] = w_in + 5
+    theta = synth.table_logits(w, 8, seed=11)
+    assert bl.bitlogic_device_error() == 0
+    Y = torch.empty(w, B, device="cuda")
+    bl.bitlogic_lut_forward_u8(dev(Xb.astype(np.uint8)), dev(conn), dev(theta), Y)
+    assert bl.bitlogic_device_error() == -8
+    clamped = conn.copy()
+    clamped[3, 1] = 0
+    check_fwd(Y, oracle.lut_forward(Xb.astype(np.float64), clamped, theta), "Y (clamped)")
+
+
 # ---------------------------------------------------------- soft backward --
 
 @pytest.mark.parametrize("k,w_in,w,B", SHAPES)

@@ -126,22 +126,32 @@ def test_mnist_k2_step_st_through():
     _full_compare(wl, st, x, labels, params, False, node="st")
 
 
-@pytest.mark.parametrize("k", [6, 2])
-def test_byte_wires_for_layer1_match_fp32_wires(k):
-    # the layer-1 backward reading the encoder's wires as bytes (the default
-    # of the fused and through routes) gives the fp32-row result bit for bit:
-    # k = 6, the byte-row kernel summing layer 2's terms itself against the
-    # CSR reduction followed by the fp32 dtheta-only kernel; k = 2, the
-    # through route on byte rows against fp32 rows
-    if k == 6:
-        _, a, *_ = _step(synth.WORKLOADS["mnist"], want_dx1=False, k=k, fuse_dy1=True, bytes1=True)
-        _, b, *_ = _step(synth.WORKLOADS["mnist"], want_dx1=False, k=k, fuse_dy1=False)
+@pytest.mark.parametrize("k,route", [(6, "fused"), (6, "csr"), (2, "through")])
+def test_byte_wires_for_layer1_match_fp32_wires(k, route):
+    # layer 1 on the encoder's wires as bytes (the step's default): the
+    # forward is the table entry each sample selects, which the fp32 lerp tree
+    # on the same wires reaches within the forward tolerance, and the table
+    # gradient equals the fp32-row kernels' bit for bit given the same output
+    # gradient: the dtheta-only kernel on dY1 (fused: layer 2's terms summed
+    # inside the byte-row kernel; csr: the CSR reduction first), and the
+    # through kernel on fp32 rows (k = 2)
+    kw = {"fused": dict(fuse_dy1=True), "csr": dict(fuse_dy1=False), "through": {}}[route]
+    wl, a, *_ = _step(synth.WORKLOADS["mnist"], want_dx1=False, k=k, **kw)
+    assert a.bytes1 and a.bits.dtype == torch.uint8 and a.through == (route == "through")
+    n = a.net
+    bits32 = a.bits.float()
+    y1 = torch.empty_like(a.y1)
+    bl.bitlogic_lut_forward_node(bits32, n.conn1, n.theta1, y1)
+    check_fwd(a.y1, y1.cpu().numpy().astype(np.float64), "y1 (lookup vs lerp tree)")
+    ref = torch.empty_like(a.dth1)
+    if route == "through":
+        g = n.w2 // wl.classes
+        bl.bitlogic_lut_backward_through(bits32, n.conn1, n.theta1, ref, a.y1, n.conn2, n.theta2, a.dyg, g,
+                                         n.off2, n.edge2)
     else:
-        _, a, *_ = _step(synth.WORKLOADS["mnist"], want_dx1=False, k=k, bytes1=True)
-        _, b, *_ = _step(synth.WORKLOADS["mnist"], want_dx1=False, k=k, bytes1=False)
-    assert a.bytes1 and not b.bytes1
-    for name in ("dy1", "dth1", "dth2", "loss"):
-        check_exact(getattr(a, name).cpu().numpy(), getattr(b, name).cpu().numpy(), name)
+        bl.bitlogic_lut_backward_node(bits32, n.conn1, n.theta1, ref, "soft", dY=a.dy1)
+    check_exact(a.dth1.cpu().numpy(), ref.cpu().numpy(), "dtheta1 (byte rows vs fp32 rows)")
+    assert bl.bitlogic_device_error() == 0
 
 
 def test_mnist_step_fused_layer1_gradient():
