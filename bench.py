@@ -358,6 +358,22 @@ TRAFFIC = {
         "bytes": 6068320768 + 6277417984, "source": "lut_soft.cu",
         "sha256": "78edac247d6c64dc0042c15287b5174dfc03ecac6e7945ec4beb26e9e6cc6800",
         "note": "ncu capture of this workload (one-pass DRAM metrics)"},
+    ("cifar10", "forward1"): {
+        "bytes": 42786816 + 199091456, "source": "lut_bytes.cu",
+        "sha256": "e65fff6a177a4f30744daa6ea751b933665c0db5387208a8689380c7f9d81ef8",
+        "note": "ncu capture of this workload (one-pass DRAM metrics)"},
+    ("cifar10", "backward1"): {
+        "bytes": 1613265664 + 3451136, "source": "lut_through.cu",
+        "sha256": "1ccfe000d8131c42950c67c661f1be21f83f53ac829efb4a363e9e33a38e73a4",
+        "note": "ncu capture of this workload (one-pass DRAM metrics)"},
+    ("cifar100", "forward1"): {
+        "bytes": 825120000 + 993534976, "source": "lut_bytes.cu",
+        "sha256": "e65fff6a177a4f30744daa6ea751b933665c0db5387208a8689380c7f9d81ef8",
+        "note": "ncu capture of this workload (one-pass DRAM metrics)"},
+    ("cifar100", "backward1"): {
+        "bytes": 6813448448 + 30162688, "source": "lut_through.cu",
+        "sha256": "1ccfe000d8131c42950c67c661f1be21f83f53ac829efb4a363e9e33a38e73a4",
+        "note": "ncu capture of this workload (one-pass DRAM metrics)"},
     ("hard_cifar10", "hard1"): {
         "bytes": 16 * (1.209681e9 + 2.054784e9), "source": "hard.cu",
         "sha256": "f9bed6fc20215df71b5e12eebae1c94762286b3c7b941dea9a2ff948bfb9ed3c",
@@ -405,7 +421,27 @@ KERNEL_OF_CALL = {
 MULTI_KERNEL_CALLS = ("head", "binarize", "hard2", "route_bwd2")
 
 
-def roofline_of(call, work, per_call_ms, sms, clocks, workload, hbm, sm_max, peak_kind):
+def kernels_of_step(st) -> dict:
+    """The kernel behind each call of a training step, by its route: byte
+    wires for layer 1 or fp32, the fused, through or CSR route for layer 1's
+    output gradient."""
+    names = dict(KERNEL_OF_CALL)
+    if getattr(st, "bytes1", False):
+        names["encode"] = "encode_soft_vec_kernel<uint8_t>"
+        names["forward1"] = "lut_forward_u8_kernel<k> (lookup)"
+    through, fused = getattr(st, "through", False), getattr(st, "fuse_dy1", False)
+    if through:
+        names["backward2"] = "lut_backward_theta_kernel<k> (dtheta only, class rows)"
+        names["backward1"] = "lut_theta_through_kernel<k, ku, " + ("uint8_t>" if st.bytes1 else "float>")
+    elif getattr(st, "bytes1", False):
+        names["backward1"] = ("lut_theta_bytes_kernel<k, terms> (one-hot)" if fused
+                              else "lut_theta_bytes_kernel<k, dY rows> (one-hot)")
+    elif fused:
+        names["backward1"] = "lut_backward_node_kernel<k, 0, terms>"
+    return names
+
+
+def roofline_of(call, work, per_call_ms, sms, clocks, workload, hbm, sm_max, peak_kind, kernels=None):
     """Roofline object of one single-kernel call: the bound (HBM bytes or
     issue-rate lane-operations, whichever takes longer at peak), achieved
     rate, peak, fraction (also at the median SM clock sampled during the
@@ -427,7 +463,7 @@ def roofline_of(call, work, per_call_ms, sms, clocks, workload, hbm, sm_max, pea
     traffic, traffic_note = kernel_traffic(workload, call)
     roof.update({"traffic": traffic, "traffic_source": traffic_note,
                  "traffic_over_algorithmic": (traffic / byts) if traffic else None,
-                 "kernel": KERNEL_OF_CALL[call], "call": call,
+                 "kernel": (kernels or KERNEL_OF_CALL)[call], "call": call,
                  "ms_per_launch": per_call_ms[call], "algorithmic_bytes": byts, "bytes_moved": moved,
                  "algorithmic_ops": ops,
                  "peak_source": f"{peak_kind} HBM copy ({hbm:.1f} GB/s); {sms} SMs (read from the device) x "
@@ -435,7 +471,7 @@ def roofline_of(call, work, per_call_ms, sms, clocks, workload, hbm, sm_max, pea
     return roof
 
 
-def calls_table(work, per_call_ms, hbm, workload=None):
+def calls_table(work, per_call_ms, hbm, workload=None, kernels=None):
     out = {}
     for n, t in per_call_ms.items():
         b_, o_, m_ = work[n]
@@ -450,6 +486,8 @@ def calls_table(work, per_call_ms, hbm, workload=None):
             # and the DRAM rate they imply at the event-timed duration
             e["traffic_over_algorithmic"] = round(traffic / b_, 2)
             e["dram_GB/s"] = round(traffic / (t * 1e-3) / 1e9, 1)
+        if kernels and n in kernels:
+            e["kernel"] = kernels[n]
         out[n] = e
     return out
 
@@ -627,8 +665,9 @@ def measure_train(wl, st, args, timer, hbm, sm_max, peak_kind, sms, world, detai
     res = {
         "value": job_rate(world, B, K, tot), "unit": "samples/s", "ms_per_step": tot / K,
         "eager_ms_per_step": eager_step,
-        "roofline": roofline_of(dom, work, per_call, sms, clocks, wl.name, hbm, sm_max, peak_kind),
-        "calls": calls_table(work, per_call, hbm, wl.name),
+        "roofline": roofline_of(dom, work, per_call, sms, clocks, wl.name, hbm, sm_max, peak_kind,
+                                kernels=None if wl.Kc else kernels_of_step(st)),
+        "calls": calls_table(work, per_call, hbm, wl.name, kernels=None if wl.Kc else kernels_of_step(st)),
         "calls_event_floor_ms": timer.event_floor(),
         "step_hbm": step_hbm_fraction(wl, B, work, per_call.keys(), tot / K, hbm) if not wl.Kc else None,
         "gpu_launches": K * st.kernels_per_run,

@@ -24,11 +24,30 @@ constexpr int kEncTF = 32;   // features per tile
 // consumers such as the routing gathers).
 __device__ __forceinline__ void put_bit(float* p, bool v) { *p = v ? 1.0f : 0.0f; }
 __device__ __forceinline__ void put_bit(uint8_t* p, bool v) { *p = v ? 1u : 0u; }
-__device__ __forceinline__ void put_bits4(float* p, bool a, bool b, bool c, bool d) {
-    *reinterpret_cast<float4*>(p) = make_float4(a ? 1.0f : 0.0f, b ? 1.0f : 0.0f, c ? 1.0f : 0.0f, d ? 1.0f : 0.0f);
+// The 4 comparisons of a SWAR test (bit 7 of byte r set: sample r's wire is 1).
+__device__ __forceinline__ void put_high_bits4(float* p, uint32_t hb) {
+    *reinterpret_cast<float4*>(p) = make_float4((hb & 0x80u) ? 1.0f : 0.0f, (hb & 0x8000u) ? 1.0f : 0.0f,
+                                                (hb & 0x800000u) ? 1.0f : 0.0f, (hb & 0x80000000u) ? 1.0f : 0.0f);
 }
-__device__ __forceinline__ void put_bits4(uint8_t* p, bool a, bool b, bool c, bool d) {
-    *reinterpret_cast<uint32_t*>(p) = (uint32_t)a | ((uint32_t)b << 8) | ((uint32_t)c << 16) | ((uint32_t)d << 24);
+__device__ __forceinline__ void put_high_bits4(uint8_t* p, uint32_t hb) {
+    *reinterpret_cast<uint32_t*>(p) = hb >> 7;
+}
+
+// Byte-wise test v > T on 4 bytes at once (no carry crosses a byte):
+//   T < 127:  v > T  <=>  v >= 128 or (v & 127) + (127 - T) >= 128
+//   T >= 127: v > T  <=>  v >= 128 and (v & 127) + (255 - T) >= 128
+// with C = the byte constant times 0x01010101 and `orf` the first form;
+// returns the high bits 0x80 of the bytes whose test holds.
+struct ThresholdSwar {
+    uint32_t C;
+    bool orf;
+};
+__device__ __forceinline__ ThresholdSwar threshold_swar(uint32_t T) {
+    // T == 255: nothing exceeds it (C = 0, AND form: the sum never reaches 128)
+    return ThresholdSwar{(T < 127u ? 127u - T : 255u - T) * 0x01010101u, T < 127u};
+}
+__device__ __forceinline__ uint32_t swar_greater(uint32_t q, uint32_t lo7, const ThresholdSwar& t) {
+    return (t.orf ? (q | (lo7 + t.C)) : (q & (lo7 + t.C))) & 0x80808080u;
 }
 
 template <typename OutT>
@@ -78,8 +97,8 @@ __global__ void __launch_bounds__(256)
 encode_soft_vec_kernel(const uint8_t* __restrict__ x, long long B, int d, Thresholds th,
                        OutT* __restrict__ bits, uint8_t* __restrict__ bits8, bool vec16) {
     __shared__ __align__(16) uint8_t tile[kEncTF][kEncVS];   // feature-major
-    __shared__ uint32_t sT[32];
-    if (threadIdx.x < th.b) sT[threadIdx.x] = threshold_at(th, threadIdx.x);
+    __shared__ ThresholdSwar sT[32];
+    if (threadIdx.x < th.b) sT[threadIdx.x] = threshold_swar(threshold_at(th, threadIdx.x));
     const long long s0 = (long long)blockIdx.y * kEncVS;
     const int f0 = blockIdx.x * kEncTF;
     const int nf = min(kEncTF, d - f0);
@@ -102,18 +121,22 @@ encode_soft_vec_kernel(const uint8_t* __restrict__ x, long long B, int d, Thresh
         for (int f = 0; f < 16; ++f) tile[16 * half + f][sl] = (uint8_t)(v[f >> 2] >> (8 * (f & 3)));
     }
     __syncthreads();
-    const int u = threadIdx.x & 31, rg = threadIdx.x >> 5;   // 8 rows per pass
+    // warp w: features w, w + 8, ...; per feature one shared load of the
+    // lane's 4 samples and, per threshold, a byte-wise test of all four
+    const int u = threadIdx.x & 31, rg = threadIdx.x >> 5;
     const long long s = s0 + 4 * u;
     if (s >= B) return;   // B % 4 == 0: the thread's four samples are in range
-    const int rows = nf * th.b;
-    for (int r = rg; r < rows; r += 8) {
-        const int f = r / th.b, i = r - f * th.b;
+    for (int f = rg; f < nf; f += 8) {
         const uint32_t q = *reinterpret_cast<const uint32_t*>(&tile[f][4 * u]);
-        const uint32_t T = sT[i];
-        const long long o = ((long long)(f0 + f) * th.b + i) * B + s;
-        const bool v0 = (q & 0xffu) > T, v1 = ((q >> 8) & 0xffu) > T, v2 = ((q >> 16) & 0xffu) > T, v3 = (q >> 24) > T;
-        put_bits4(bits + o, v0, v1, v2, v3);
-        if (bits8) put_bits4(bits8 + o, v0, v1, v2, v3);   // the same wires as bytes
+        const uint32_t lo7 = q & 0x7f7f7f7fu;
+        const long long o = (long long)(f0 + f) * th.b * B + s;
+        OutT* out = bits + o;
+        uint8_t* out8 = bits8 ? bits8 + o : nullptr;
+        for (int i = 0; i < th.b; ++i) {
+            const uint32_t hb = swar_greater(q, lo7, sT[i]);
+            put_high_bits4(out + (long long)i * B, hb);
+            if (out8) put_high_bits4(out8 + (long long)i * B, hb);   // the same wires as bytes
+        }
     }
 }
 

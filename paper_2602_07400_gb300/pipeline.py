@@ -149,10 +149,11 @@ class Network:
         self.pos2 = torch.from_numpy(bitlogic_csr_positions(edge2)).to(dev)
 
 
-# Per-edge input-gradient terms larger than this are summed by the layer-1
-# backward itself instead of a separate CSR reduction (measured faster on
-# GB300 for the CIFAR-shaped layers, 1.6 and 6.3 GB of terms, and slower for
-# the MNIST-shaped one, 0.2 GB).
+# On fp32 wires, per-edge input-gradient terms larger than this are summed by
+# the layer-1 backward itself instead of a separate CSR reduction (measured
+# faster on GB300 for the CIFAR-shaped layers, 1.6 and 6.3 GB of terms, and
+# slower for the MNIST-shaped one, 0.2 GB).  On byte wires the layer-1
+# backward always sums them (MNIST shape: 0.216 against 0.2235 ms per step).
 FUSE_DY1_TERM_BYTES = 512 << 20
 
 
@@ -167,9 +168,9 @@ class TrainStep:
       backward recomputes it from layer 2's connectivity, tables and output
       gradient rows (bitlogic_lut_backward_through), so layer 2 needs only
       its table gradient and nothing per edge is stored;
-    * ``fuse_dy1`` (default when layer 2's per-edge terms exceed
-      FUSE_DY1_TERM_BYTES): layer 2 stores its per-edge terms and the layer-1
-      backward sums them through the CSR map on the fly;
+    * ``fuse_dy1`` (default on byte wires, and on fp32 wires when layer 2's
+      per-edge terms exceed FUSE_DY1_TERM_BYTES): layer 2 stores its per-edge
+      terms and the layer-1 backward sums them through the CSR map on the fly;
     * otherwise a CSR reduction of the terms into ``dy1``, which the
       dtheta-only layer-1 backward reads.
 
@@ -203,8 +204,13 @@ class TrainStep:
         if through and (net.k2 > 3 or B % 4 != 0 or want_dx1):
             raise ValueError("the through route needs layer-2 fan-in <= 3, B % 4 == 0 and no layer-1 input gradient")
         self.through = bool(through)
+        if bytes1 is None:
+            bytes1 = B % 4 == 0 and not want_dx1
         if fuse_dy1 is None:
-            fuse_dy1 = 4 * net.w2 * net.k2 * B > FUSE_DY1_TERM_BYTES
+            # on byte wires the layer-1 backward streams the terms itself
+            # (faster than the CSR reduction at every measured shape); on fp32
+            # wires the separate reduction wins below FUSE_DY1_TERM_BYTES
+            fuse_dy1 = bool(bytes1) or 4 * net.w2 * net.k2 * B > FUSE_DY1_TERM_BYTES
         f32 = dict(dtype=torch.float32, device=dev)
         self.x = torch.zeros(B, d, dtype=torch.uint8, device=dev)
         self.labels = torch.zeros(B, dtype=torch.int32, device=dev)
@@ -214,8 +220,6 @@ class TrainStep:
         self.loss = torch.zeros(1, **f32)
         self.dyg = torch.empty(C, B, **f32)          # gradient row shared by each class's nodes
         self.fuse_dy1 = bool(fuse_dy1) and not self.through
-        if bytes1 is None:
-            bytes1 = B % 4 == 0 and not want_dx1
         if bytes1 and (B % 4 != 0 or want_dx1):
             raise ValueError("byte wires for layer 1 need B % 4 == 0 and no layer-1 input gradient")
         self.bytes1 = bool(bytes1)
