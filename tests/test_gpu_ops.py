@@ -48,6 +48,24 @@ def test_encode_thermometer(B, d, b):
     no_device_error()
 
 
+@pytest.mark.parametrize("B", [256, 255])
+def test_encode_thermometer_edge_thresholds(B):
+    # every byte value against the thresholds where the byte-wise test
+    # changes form (T < 127: OR form, T >= 127: AND form, T = 255: nothing
+    # exceeds it), on the vector (B % 4 == 0) and the scalar path
+    d = 16
+    x = ((np.arange(B * d, dtype=np.int64) * 37) % 256).astype(np.uint8).reshape(B, d)
+    thr = [0, 1, 126, 127, 128, 254, 255]
+    want = oracle.encode_thermometer(x, thr)
+    bits = torch.full((d * len(thr), B), -1.0, device="cuda")
+    bl.bitlogic_encode_thermometer(dev(x), thr, bits)
+    check_exact(bits.cpu().numpy().astype(np.float64), want, "bits")
+    bits8 = torch.full((d * len(thr), B), 7, dtype=torch.uint8, device="cuda")
+    bl.bitlogic_encode_thermometer_u8(dev(x), thr, bits8)
+    check_exact(bits8.cpu().numpy().astype(np.float64), want, "byte wires")
+    no_device_error()
+
+
 # ------------------------------------------------ quantile thermometer fit --
 
 @pytest.mark.parametrize("n,offset,skew", [(1, 0, False), (15, 3, False), (16, 0, True), (17, 1, True),
