@@ -138,6 +138,36 @@ def test_algorithmic_work_of_the_roofline_calls():
     assert hwork["hard1"][0] == 4 * (21504 * W + 64000 * W + 64000 * 6) + 8 * 64000
 
 
+def test_byte_wire_layer1_work_and_kernel_names():
+    # layer 1 on byte wires: the encoder writes one byte per wire, the
+    # lookup forward has no arithmetic (HBM-bound), the one-hot table
+    # gradient one add per (node, sample); the call table names the route's
+    # kernels
+    import types
+    import bench
+    from paper_2602_07400_gb300 import synth
+    wl = synth.WORKLOADS["cifar100"]
+    B, d, w_in, w1, K, k = 2048, 3072, 46080, 128000, 64, 6
+    f32 = bench.call_work(wl, B, fuse_dy1=True)
+    u8 = bench.call_work(wl, B, fuse_dy1=True, bytes1=True)
+    assert u8["encode"][0] == B * d + w_in * B < f32["encode"][0]
+    assert u8["forward1"][1] == 0 and f32["forward1"][1] == 132 * w1 * B
+    assert u8["forward1"][0] == w_in * B + 4 * (w1 * B + w1 * K + w1 * k)
+    assert u8["backward1"][1] == w1 * B
+    # the fused route moves the per-edge terms in place of dY1
+    assert u8["backward1"][2] - u8["backward1"][0] == 4 * w1 * k * B - 4 * w1 * B
+    roof = bench.roofline_of("forward1", u8, {"forward1": 0.3}, 152, {}, "none", 6767.1, 2070.0, "measured")
+    assert roof["bound"] == "hbm"
+    st = types.SimpleNamespace(bytes1=True, through=False, fuse_dy1=True)
+    names = bench.kernels_of_step(st)
+    assert names["forward1"].startswith("lut_forward_u8_kernel")
+    assert names["backward1"].startswith("lut_theta_bytes_kernel")
+    st = types.SimpleNamespace(bytes1=True, through=True, fuse_dy1=False)
+    assert bench.kernels_of_step(st)["backward1"] == "lut_theta_through_kernel<k, ku, uint8_t>"
+    st = types.SimpleNamespace(bytes1=False, through=False, fuse_dy1=False)
+    assert bench.kernels_of_step(st)["backward1"] == bench.KERNEL_OF_CALL["backward1"]
+
+
 def test_hard_roofline_uses_the_measured_mix_rate():
     # the hard layer's peak is the measured issue rate of its instruction mix
     # (per SM and clock) at the sampled clock; the issue-rate fraction stays
