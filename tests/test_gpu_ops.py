@@ -645,6 +645,26 @@ def test_lut_backward_u8_rows_and_terms(k, w_in, w, B, node):
     no_device_error()
 
 
+@pytest.mark.parametrize("k,group", [(6, 4), (3, 13), (2, 52)])
+def test_lut_backward_u8_grouped_rows(k, group):
+    # dY rows shared by groups of nodes (the head's per-class rows): the
+    # byte-row kernel equals the fp32-row dtheta-only kernel bit for bit
+    w_in, w, B = 90, 52, 516
+    Xb = synth.binary_activations(w_in, B, seed=k + 60)
+    conn = synth.connectivity(w, k, w_in, seed=k + 61)
+    theta = synth.table_logits(w, 1 << k, seed=k + 62)
+    dY = synth.uniform_gradients(w // group, B, seed=k + 63, scale=1e-3)
+    ref = torch.empty(w, 1 << k, device="cuda")
+    bl.bitlogic_lut_backward_node(dev(Xb), dev(conn), dev(theta), ref, "soft", dY=dev(dY), dy_group=group)
+    got = torch.full((w, 1 << k), np.nan, device="cuda")
+    bl.bitlogic_lut_backward_u8(dev(Xb.astype(np.uint8)), dev(conn), dev(theta), got, dY=dev(dY), dy_group=group)
+    check_exact(got.cpu().numpy(), ref.cpu().numpy(), "dtheta (grouped rows)")
+    dYfull = np.repeat(dY, group, axis=0)
+    wdth, _ = oracle.lut_backward(Xb, conn, theta, dYfull, want_dx=False)
+    check_grad(got, wdth, "dtheta (grouped rows) vs oracle")
+    no_device_error()
+
+
 @pytest.mark.parametrize("k", [2, 6])
 def test_lut_backward_u8_terms_with_many_and_no_consumers(k):
     # the term rows of a node beyond the ones its ring slot holds (ten), and
