@@ -421,6 +421,20 @@ KERNEL_OF_CALL = {
 MULTI_KERNEL_CALLS = ("head", "binarize", "hard2", "route_bwd2")
 
 
+def route_of_step(st) -> dict:
+    """How the step runs layer 1: its input wires and where its output
+    gradient comes from."""
+    if getattr(st, "through", False):
+        grad = "recomputed through layer 2 (fan-in <= 3)"
+    elif getattr(st, "fuse_dy1", False):
+        grad = "layer 2's per-edge terms summed in the layer-1 kernel"
+    else:
+        grad = "CSR reduction of layer 2's per-edge terms"
+    wires = ("bytes: lookup forward, one-hot table gradient" if getattr(st, "bytes1", False)
+             else "fp32: lerp-tree forward, multilinear table gradient")
+    return {"layer1_wires": wires, "layer1_output_gradient": grad}
+
+
 def kernels_of_step(st) -> dict:
     """The kernel behind each call of a training step, by its route: byte
     wires for layer 1 or fp32, the fused, through or CSR route for layer 1's
@@ -669,6 +683,7 @@ def measure_train(wl, st, args, timer, hbm, sm_max, peak_kind, sms, world, detai
                                 kernels=None if wl.Kc else kernels_of_step(st)),
         "calls": calls_table(work, per_call, hbm, wl.name, kernels=None if wl.Kc else kernels_of_step(st)),
         "calls_event_floor_ms": timer.event_floor(),
+        "route": None if wl.Kc else route_of_step(st),
         "step_hbm": step_hbm_fraction(wl, B, work, per_call.keys(), tot / K, hbm) if not wl.Kc else None,
         "gpu_launches": K * st.kernels_per_run,
         "clocks": clocks, "wall_s_timed_loop": wall,
@@ -920,6 +935,7 @@ def run_headline(args):
         "eager_ms_per_step": train["eager_ms_per_step"],
         "calls": train["calls"],
         "calls_event_floor_ms": train["calls_event_floor_ms"],
+        "route": train["route"],
         "roofline_by_call": train["roofline_by_call"],
         "step_hbm": train["step_hbm"],
         "wall_s_timed_loop": train["wall_s_timed_loop"],
