@@ -97,6 +97,9 @@ def parse_args(argv=None):
     p.add_argument("--bytes1", choices=["auto", "on", "off"], default="auto",
                    help="layer 1 reads the encoder's wires as bytes: lookup forward and one-hot table "
                         "gradient (auto: whenever B % 4 == 0)")
+    p.add_argument("--bits1", choices=["auto", "on", "off"], default="auto",
+                   help="layer 1's binary wires kept at one bit per sample (wire bit rows) instead of a byte "
+                        "(auto: on byte wires off the through route)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-graph", action="store_true",
@@ -260,7 +263,7 @@ def call_work_routed(wl, B):
     return {n: (b, o, b) for n, (b, o) in work.items()}
 
 
-def call_work(wl, B, fuse_dy1=False, through=False, bytes1=False):
+def call_work(wl, B, fuse_dy1=False, through=False, bytes1=False, bits1=False):
     """Algorithmic work of each library call of one step on a batch of B:
     (algorithmic bytes, algorithmic ops, bytes the call moves).
 
@@ -279,7 +282,9 @@ def call_work(wl, B, fuse_dy1=False, through=False, bytes1=False):
     wire and layer 1's inputs are binary, so its corner weights are one-hot:
     the forward is a lookup (no arithmetic beyond the k-byte gather and one
     table read) and the table gradient one add per (node, sample); both
-    calls are then bounded by their bytes."""
+    calls are then bounded by their bytes.  With wire bit rows (``bits1``)
+    each wire takes one bit per sample (32-bit words, 32 per 1024-sample
+    block), written by the encoder and read by both layer-1 calls."""
     K, k = wl.K, wl.k
     w1, w2 = wl.widths
     win, d, C = wl.w_in, wl.d, wl.classes
@@ -313,6 +318,11 @@ def call_work(wl, B, fuse_dy1=False, through=False, bytes1=False):
         work["encode"] = (B * d + win * B, 0, B * d + win * B)
         work["forward1"] = (win * B + f * (w1 * B + w1 * K + w1 * k), 0, None)
         work["backward1"] = (win * B + f * (w1 * B + 2 * w1 * K + w1 * k), dth1_ops, None)
+    if bits1:
+        xw1 = 4 * win * (32 * ((B + 1023) // 1024))   # the wire bit rows
+        work["encode"] = (B * d + xw1, 0, B * d + xw1)
+        work["forward1"] = (xw1 + f * (w1 * B + w1 * K + w1 * k), 0, None)
+        work["backward1"] = (xw1 + f * (w1 * B + 2 * w1 * K + w1 * k), dth1_ops, None)
     if through:
         # layer 2: table gradient only; layer 1: its table gradient with its
         # output gradient recomputed through layer 2 (the consumers' other
@@ -326,8 +336,9 @@ def call_work(wl, B, fuse_dy1=False, through=False, bytes1=False):
         return {n: (b, o, b if m is None else m) for n, (b, o, m) in work.items()}
     if fuse_dy1:
         # layer 1 sums layer 2's per-edge terms through the CSR map itself
-        work["backward1"] = (xb1 * win * B + f * (w1 * B + 2 * w1 * K + w1 * k) + csr2, dth1_ops,
-                             xb1 * win * B + f * (2 * w1 * K + w1 * k) + csr2 + terms)
+        xin = xw1 if bits1 else xb1 * win * B
+        work["backward1"] = (xin + f * (w1 * B + 2 * w1 * K + w1 * k) + csr2, dth1_ops,
+                             xin + f * (2 * w1 * K + w1 * k) + csr2 + terms)
         del work["csr2"]
     return {n: (b, o, b if m is None else m) for n, (b, o, m) in work.items()}
 
@@ -432,6 +443,8 @@ def route_of_step(st) -> dict:
         grad = "CSR reduction of layer 2's per-edge terms"
     wires = ("bytes: lookup forward, one-hot table gradient" if getattr(st, "bytes1", False)
              else "fp32: lerp-tree forward, multilinear table gradient")
+    if getattr(st, "bits1", False):
+        wires = "bits (one per sample): lookup forward, one-hot table gradient"
     return {"layer1_wires": wires, "layer1_output_gradient": grad}
 
 
@@ -440,7 +453,10 @@ def kernels_of_step(st) -> dict:
     wires for layer 1 or fp32, the fused, through or CSR route for layer 1's
     output gradient."""
     names = dict(KERNEL_OF_CALL)
-    if getattr(st, "bytes1", False):
+    if getattr(st, "bits1", False):
+        names["encode"] = "encode_bitrows_kernel"
+        names["forward1"] = "lut_forward_bits_kernel<k> (lookup)"
+    elif getattr(st, "bytes1", False):
         names["encode"] = "encode_soft_vec_kernel<uint8_t>"
         names["forward1"] = "lut_forward_u8_kernel<k> (lookup)"
     through, fused = getattr(st, "through", False), getattr(st, "fuse_dy1", False)
@@ -448,8 +464,9 @@ def kernels_of_step(st) -> dict:
         names["backward2"] = "lut_backward_theta_kernel<k> (dtheta only, class rows)"
         names["backward1"] = "lut_theta_through_kernel<k, ku, " + ("uint8_t>" if st.bytes1 else "float>")
     elif getattr(st, "bytes1", False):
-        names["backward1"] = ("lut_theta_bytes_kernel<k, terms> (one-hot)" if fused
-                              else "lut_theta_bytes_kernel<k, dY rows> (one-hot)")
+        src = "bit rows" if getattr(st, "bits1", False) else "byte rows"
+        names["backward1"] = (f"lut_theta_bytes_kernel<k, terms, {src}> (one-hot)" if fused
+                              else f"lut_theta_bytes_kernel<k, dY rows, {src}> (one-hot)")
     elif fused:
         names["backward1"] = "lut_backward_node_kernel<k, 0, terms>"
     return names
@@ -632,7 +649,7 @@ class Timer:
         return per_call["empty"]
 
 
-def build_train(wl, rank, node="soft", fuse_dy1=None, through=None, bytes1=None):
+def build_train(wl, rank, node="soft", fuse_dy1=None, through=None, bytes1=None, bits1=None):
     from paper_2602_07400_gb300.pipeline import Network, RoutedNetwork, RoutedTrainStep, TrainStep
     B = wl.batch
     if wl.Kc:
@@ -643,7 +660,7 @@ def build_train(wl, rank, node="soft", fuse_dy1=None, through=None, bytes1=None)
         conn1, th1, conn2, th2 = synth.network(wl, seed=0)
         net = Network(conn1, th1, conn2, th2, wl.w_in)
         st = TrainStep(net, B, wl.d, wl.thresholds, wl.classes, wl.tau, node=node, fuse_dy1=fuse_dy1,
-                       through=through, bytes1=bytes1)
+                       through=through, bytes1=bytes1, bits1=bits1)
     x, lab = synth.blob_batch(B, wl.d, wl.classes, wl.sigma, seed=1000 + rank)
     st.load(x.cuda(), lab.cuda())
     return net, st
@@ -673,7 +690,8 @@ def measure_train(wl, st, args, timer, hbm, sm_max, peak_kind, sms, world, detai
     per_call, eager_step = timer.eager_split(lambda mark: st.run(mark=mark), max(3, min(K, 30)))
     work = call_work_routed(wl, B) if wl.Kc else call_work(wl, B, fuse_dy1=st.fuse_dy1,
                                                               through=getattr(st, "through", False),
-                                                              bytes1=getattr(st, "bytes1", False))
+                                                              bytes1=getattr(st, "bytes1", False),
+                                                              bits1=getattr(st, "bits1", False))
     single = {n: t for n, t in per_call.items() if n not in MULTI_KERNEL_CALLS}
     dom = max(single, key=single.get)
     res = {
@@ -876,7 +894,7 @@ def run_headline(args):
 
     # -- headline training workload
     wl = with_batch(synth.WORKLOADS[HEADLINE_TRAIN], args.batch)
-    net, st = build_train(wl, rank, args.node, FUSE[args.fuse_dy1], FUSE[args.through], FUSE[args.bytes1])
+    net, st = build_train(wl, rank, args.node, FUSE[args.fuse_dy1], FUSE[args.through], FUSE[args.bytes1], FUSE[args.bits1])
     train = measure_train(wl, st, args, timer, hbm, sm_max, peak_kind, sms, world)
     upd = time_update(st, max(3, min(K, 20)))
     n_par = int(net.theta1.numel() + net.theta2.numel())
@@ -914,7 +932,7 @@ def run_headline(args):
     names = [] if (args.no_extras or args.profile) else [n for n in args.extras.split(",") if n]
     for name in names:
         we = synth.WORKLOADS[name]
-        enet, est = build_train(we, rank, args.node, FUSE[args.fuse_dy1], FUSE[args.through], FUSE[args.bytes1])
+        enet, est = build_train(we, rank, args.node, FUSE[args.fuse_dy1], FUSE[args.through], FUSE[args.bytes1], FUSE[args.bits1])
         r = measure_train(we, est, args, timer, hbm, sm_max, peak_kind, sms, world, detail=False)
         r["config"] = {k_: v for k_, v in config_of(we, world, args.node).items()
                        if k_ in ("workload", "batch_per_gpu", "widths", "k", "classes", "tau")}
@@ -977,7 +995,7 @@ def run_single(args):
         net = Network(*synth.network(wl, seed=0), wl.w_in)
         hi = build_hard(wl, net, rank)
     else:
-        rnet, st = build_train(wl, rank, args.node, FUSE[args.fuse_dy1], FUSE[args.through], FUSE[args.bytes1])
+        rnet, st = build_train(wl, rank, args.node, FUSE[args.fuse_dy1], FUSE[args.through], FUSE[args.bytes1], FUSE[args.bits1])
         net = rnet.snap() if wl.Kc else rnet   # the hard pass evaluates the discretized network
         train = measure_train(wl, st, args, timer, hbm, sm_max, peak_kind, sms, world)
         hi = build_hard(wl, net, rank, x_dev=st.x)

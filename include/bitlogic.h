@@ -99,6 +99,21 @@ int bitlogic_encode_thermometer_both(const uint8_t* x, int64_t B, int32_t d,
                                      const uint8_t* thr_host, int32_t b,
                                      float* bits, uint8_t* bits8, cudaStream_t stream);
 
+/* The same wires at one bit per sample ("wire bit rows"), for the soft
+ * layer-1 kernels on binary wires (bitlogic_lut_forward_bitrows,
+ * bitlogic_lut_backward_bitrows): an eighth of the bytes of byte rows.  The
+ * batch is cut into blocks of 1024 samples; each wire row holds 32 words
+ * per block, W = 32 * ceil(B / 1024) words in all, and bit 8m + r of word L
+ * of block q is the wire of sample 1024q + 128r + 4L + m (r < 8, m < 4), the
+ * order in which those kernels' lanes visit the samples.  Samples past B
+ * read 0.
+ *   bits  device uint32 [d*b][W]
+ * Any B and alignment of x; B == 0 is a no-op.  Returns BITLOGIC_ERR_NULL,
+ * BITLOGIC_ERR_SHAPE, BITLOGIC_ERR_THRESH, BITLOGIC_ERR_CUDA. */
+int bitlogic_encode_thermometer_bitrows(const uint8_t* x, int64_t B, int32_t d,
+                                        const uint8_t* thr_host, int32_t b,
+                                        uint32_t* bits, cudaStream_t stream);
+
 /* Distributive (quantile) thermometer fit (§3 "Encoders and heads"; App. A
  * "Initialization": thresholds fit once from the empirical pixel quantiles
  * of the training split, over the globally flattened pixels, App. B).  Two
@@ -207,6 +222,16 @@ int bitlogic_csr_reduce(const float* edge_terms, int64_t B, const int32_t* csr_o
 int bitlogic_lut_forward_u8(const uint8_t* X, int32_t w_in, int64_t B, const int32_t* conn,
                             const float* theta, int32_t w, int32_t k, int32_t node, float* Y,
                             cudaStream_t stream);
+
+/* bitlogic_lut_forward_u8 on wire bit rows (the layout of
+ * bitlogic_encode_thermometer_bitrows): X device uint32 [w_in][W], W = 32 *
+ * ceil(B / 1024), 4-byte aligned (BITLOGIC_ERR_ALIGN otherwise).  Every
+ * other argument, the result and the errors as bitlogic_lut_forward_u8: the
+ * same wires give the same Y bit for bit.  B % 4 == 0 with 16-byte aligned
+ * Y takes vector stores. */
+int bitlogic_lut_forward_bitrows(const uint32_t* X, int32_t w_in, int64_t B, const int32_t* conn,
+                                 const float* theta, int32_t w, int32_t k, int32_t node, float* Y,
+                                 cudaStream_t stream);
 
 /* General form of the layer backward, with the output gradient taken from
  * one of two sources (exactly one of dY and up_terms is non-NULL):
@@ -325,6 +350,17 @@ int bitlogic_lut_backward_u8(const uint8_t* X, int32_t w_in, int64_t B, const in
                              const float* dY, int32_t dy_group, const float* up_terms,
                              const int32_t* up_off, const int32_t* up_edge, int32_t up_edges,
                              float* dtheta, float* dY_out, cudaStream_t stream);
+
+/* bitlogic_lut_backward_u8 on wire bit rows: X device uint32 [w_in][W]
+ * (the layout of bitlogic_encode_thermometer_bitrows), 16-byte aligned.
+ * Every other argument, the result and the errors as
+ * bitlogic_lut_backward_u8: the same wires give the same dtheta and dY_out
+ * bit for bit (the samples are visited in the same order). */
+int bitlogic_lut_backward_bitrows(const uint32_t* X, int32_t w_in, int64_t B, const int32_t* conn,
+                                  const float* theta, int32_t w, int32_t k, int32_t node,
+                                  const float* dY, int32_t dy_group, const float* up_terms,
+                                  const int32_t* up_off, const int32_t* up_edge, int32_t up_edges,
+                                  float* dtheta, float* dY_out, cudaStream_t stream);
 
 /* Learnable routing (§3, the paragraph on connectivity: a per-slot
  * candidate pool whose selection is differentiable in training and snapped

@@ -28,7 +28,8 @@ __all__ = [
     "bitlogic_lut_backward_workspace", "bitlogic_lut_backward", "bitlogic_lut_backward_edges",
     "bitlogic_csr_reduce", "bitlogic_lut_backward_ex", "bitlogic_head_loss_ex",
     "bitlogic_head_loss_workspace", "bitlogic_head_loss_noalloc", "bitlogic_lut_backward_through", "bitlogic_lut_backward_through_u8",
-    "bitlogic_lut_backward_u8", "bitlogic_lut_forward_u8",
+    "bitlogic_lut_backward_u8", "bitlogic_lut_forward_u8", "bitlogic_encode_thermometer_bitrows",
+    "bitlogic_lut_forward_bitrows", "bitlogic_lut_backward_bitrows", "bitrow_words",
     "bitlogic_head_loss", "bitlogic_binarize_tables", "bitlogic_pack_bits",
     "bitlogic_hard_forward", "bitlogic_build_csr", "bitlogic_csr_positions", "bitlogic_device_error",
     "bitlogic_adamw_update", "bitlogic_route_forward", "bitlogic_route_backward", "bitlogic_route_snap",
@@ -80,6 +81,10 @@ _SIGS = {
     "bitlogic_quantile_thresholds": ([_P, _I32, _P], ctypes.c_int),
     "bitlogic_lut_forward_node": ([_P, _I32, _I64, _P, _P, _I32, _I32, _I32, _P, _P], ctypes.c_int),
     "bitlogic_lut_forward_u8": ([_P, _I32, _I64, _P, _P, _I32, _I32, _I32, _P, _P], ctypes.c_int),
+    "bitlogic_encode_thermometer_bitrows": ([_P, _I64, _I32, _P, _I32, _P, _P], ctypes.c_int),
+    "bitlogic_lut_forward_bitrows": ([_P, _I32, _I64, _P, _P, _I32, _I32, _I32, _P, _P], ctypes.c_int),
+    "bitlogic_lut_backward_bitrows": ([_P, _I32, _I64, _P, _P, _I32, _I32, _I32, _P, _I32, _P, _P, _P, _I32, _P,
+                                       _P, _P], ctypes.c_int),
     "bitlogic_lut_backward_workspace": ([_I32, _I64, _I32, _I32, _I32], _SZ),
     "bitlogic_lut_backward": ([_P, _I32, _I64, _P, _P, _I32, _I32, _P, _P, _P, _P, _P,
                                _P, _SZ, _P], ctypes.c_int),
@@ -226,6 +231,21 @@ def bitlogic_encode_thermometer_u8(x: torch.Tensor, thresholds, bits: torch.Tens
     _need(x, "x", torch.uint8, (B, d))
     _need(bits, "bits", torch.uint8, (d * b, B))
     _check("bitlogic_encode_thermometer_u8", load().bitlogic_encode_thermometer_u8(
+        _ptr(x), B, d, buf, b, _ptr(bits), _stream(stream)))
+
+
+def bitrow_words(B: int) -> int:
+    """32-bit words per wire bit row of a batch of B (32 per 1024-sample block)."""
+    return 32 * ((int(B) + 1023) // 1024)
+
+
+def bitlogic_encode_thermometer_bitrows(x: torch.Tensor, thresholds, bits: torch.Tensor, stream=None):
+    """The thermometer wires at one bit per sample, [d*b, bitrow_words(B)] int32."""
+    B, d = x.shape
+    buf, b = _thr_buf(thresholds)
+    _need(x, "x", torch.uint8, (B, d))
+    _need(bits, "bits", torch.int32, (d * b, bitrow_words(B)))
+    _check("bitlogic_encode_thermometer_bitrows", load().bitlogic_encode_thermometer_bitrows(
         _ptr(x), B, d, buf, b, _ptr(bits), _stream(stream)))
 
 
@@ -376,6 +396,21 @@ def bitlogic_lut_forward_u8(X: torch.Tensor, conn: torch.Tensor, theta: torch.Te
     _need(theta, "theta", torch.float32, (w, 1 << k))
     _need(Y, "Y", torch.float32, (w, B))
     _check("bitlogic_lut_forward_u8", load().bitlogic_lut_forward_u8(
+        _ptr(X), w_in, B, _ptr(conn), _ptr(theta), w, k, code, _ptr(Y), _stream(stream)))
+
+
+def bitlogic_lut_forward_bitrows(X: torch.Tensor, B: int, conn: torch.Tensor, theta: torch.Tensor,
+                                 Y: torch.Tensor, node="soft", stream=None):
+    """Layer forward on wire bit rows X [w_in, bitrow_words(B)] int32 (binary
+    wires at one bit per sample): the table entry the inputs' bits select."""
+    code = _node_code(node)
+    w_in = X.shape[0]
+    w, k = conn.shape
+    _need(X, "X", torch.int32, (w_in, bitrow_words(B)))
+    _need(conn, "conn", torch.int32, (w, k))
+    _need(theta, "theta", torch.float32, (w, 1 << k))
+    _need(Y, "Y", torch.float32, (w, B))
+    _check("bitlogic_lut_forward_bitrows", load().bitlogic_lut_forward_bitrows(
         _ptr(X), w_in, B, _ptr(conn), _ptr(theta), w, k, code, _ptr(Y), _stream(stream)))
 
 
@@ -571,6 +606,36 @@ def bitlogic_lut_backward_u8(X: torch.Tensor, conn: torch.Tensor, theta: torch.T
     if dY_out is not None:
         _need(dY_out, "dY_out", torch.float32, (w, B))
     _check("bitlogic_lut_backward_u8", load().bitlogic_lut_backward_u8(
+        _ptr(X), w_in, B, _ptr(conn), _ptr(theta), w, k, _node_code(node), _ptr(dY), int(dy_group),
+        _ptr(up_terms), _ptr(up_off), _ptr(up_edge), n_up, _ptr(dtheta), _ptr(dY_out), _stream(stream)))
+
+
+def bitlogic_lut_backward_bitrows(X: torch.Tensor, B: int, conn: torch.Tensor, theta: torch.Tensor,
+                                  dtheta: torch.Tensor, node="soft", dY: Optional[torch.Tensor] = None,
+                                  dy_group: int = 1, up_terms: Optional[torch.Tensor] = None,
+                                  up_off: Optional[torch.Tensor] = None, up_edge: Optional[torch.Tensor] = None,
+                                  dY_out: Optional[torch.Tensor] = None, stream=None):
+    """bitlogic_lut_backward_u8 on wire bit rows X [w_in, bitrow_words(B)] int32."""
+    w_in = X.shape[0]
+    _need(X, "X", torch.int32, (w_in, bitrow_words(B)))
+    w, k = conn.shape
+    _need(conn, "conn", torch.int32, (w, k))
+    _need(theta, "theta", torch.float32, (w, 1 << k))
+    _need(dtheta, "dtheta", torch.float32, (w, 1 << k))
+    n_up = 0
+    if dY is not None:
+        if w % dy_group != 0:
+            raise ValueError("dy_group must divide w")
+        _need(dY, "dY", torch.float32, (w // dy_group, B))
+    if up_terms is not None:
+        n_up = up_terms.shape[0]
+        _need(up_terms, "up_terms", torch.float32, (n_up, B))
+        _need(up_off, "up_off", torch.int32, (w + 1,))
+        if up_edge is not None:
+            _need(up_edge, "up_edge", torch.int32, (n_up,))
+    if dY_out is not None:
+        _need(dY_out, "dY_out", torch.float32, (w, B))
+    _check("bitlogic_lut_backward_bitrows", load().bitlogic_lut_backward_bitrows(
         _ptr(X), w_in, B, _ptr(conn), _ptr(theta), w, k, _node_code(node), _ptr(dY), int(dy_group),
         _ptr(up_terms), _ptr(up_off), _ptr(up_edge), n_up, _ptr(dtheta), _ptr(dY_out), _stream(stream)))
 

@@ -37,6 +37,11 @@ inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 
 // cached; 152 if the query fails).  Defined in abi.cu.
 int sm_count();
 
+// Wire bit rows (the layer-1 input at one bit per sample): samples per word
+// block; a row holds 32 words per block, bit 8 m + r of word L being the
+// block's sample 128 r + 4 L + m.
+constexpr int kBitBlock = 1024;
+
 // Thresholds travel by value in the kernel parameters: no constant-memory
 // state is shared between calls or streams.
 struct Thresholds {

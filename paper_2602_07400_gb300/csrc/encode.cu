@@ -140,6 +140,72 @@ encode_soft_vec_kernel(const uint8_t* __restrict__ x, long long B, int d, Thresh
     }
 }
 
+// ------------------------------------------------------------- bit rows --
+//
+// Layer-1 wires at one bit per sample for the soft layer-1 kernels (a
+// thirty-second of fp32 rows, an eighth of byte rows), in the order of those
+// kernels' lanes: the batch is cut into 1024-sample blocks of 32 words per
+// wire, and bit 8 m + r of word L of a block is the wire of the block's sample
+// 128 r + 4 L + m (r < 8, m < 4).  Lane L of a layer-1 kernel, taking samples
+// 128 r + 4 L .. + 3 of the block (stage r), finds their four wires as bytes
+// 0 .. 3 of (word >> r) & 0x01010101.  Samples past B have wire 0.
+//
+// A block encodes 8 features (one per warp) over one 1024-sample block: the
+// raw bytes go to a feature-major shared tile, then lane L reads its 8
+// stages' 4 pixels (one 32-bit word each) and per threshold assembles its
+// word from the byte-wise comparisons.
+constexpr int kBitsTF = 8;   // features per block (one per warp)
+
+__global__ void __launch_bounds__(256)
+encode_bitrows_kernel(const uint8_t* __restrict__ x, long long B, int d, Thresholds th,
+                      uint32_t* __restrict__ bits, long long words, bool vec8) {
+    __shared__ __align__(16) uint8_t tile[kBitsTF][kBitBlock];   // feature-major
+    __shared__ ThresholdSwar sT[32];
+    if (threadIdx.x < th.b) sT[threadIdx.x] = threshold_swar(threshold_at(th, threadIdx.x));
+    const long long s0 = (long long)blockIdx.y * kBitBlock;
+    const int f0 = blockIdx.x * kBitsTF;
+    const int nf = min(kBitsTF, d - f0);
+#pragma unroll
+    for (int q = 0; q < kBitBlock / 256; ++q) {   // thread t: samples t, t + 256, ...
+        const int sl = threadIdx.x + 256 * q;
+        const long long s = s0 + sl;
+        uint32_t lo = 0u, hi = 0u;   // the sample's 8 feature bytes
+        if (s < B) {
+            const uint8_t* p = x + s * d + f0;
+            if (vec8 && nf == kBitsTF) {
+                const uint2 v = __ldg(reinterpret_cast<const uint2*>(p));
+                lo = v.x;
+                hi = v.y;
+            } else {
+                for (int f = 0; f < nf; ++f) {
+                    const uint32_t v = __ldg(p + f);
+                    if (f < 4) lo |= v << (8 * f);
+                    else hi |= v << (8 * (f - 4));
+                }
+            }
+        }
+#pragma unroll
+        for (int f = 0; f < kBitsTF; ++f) tile[f][sl] = (uint8_t)((f < 4 ? lo : hi) >> (8 * (f & 3)));
+    }
+    __syncthreads();
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (warp >= nf) return;
+    uint32_t q[8], lo7[8];
+#pragma unroll
+    for (int r = 0; r < 8; ++r) {
+        q[r] = *reinterpret_cast<const uint32_t*>(&tile[warp][128 * r + 4 * lane]);
+        lo7[r] = q[r] & 0x7f7f7f7fu;
+    }
+    uint32_t* out = bits + (long long)(f0 + warp) * th.b * words + (long long)blockIdx.y * 32 + lane;
+    for (int i = 0; i < th.b; ++i) {
+        const ThresholdSwar t = sT[i];
+        uint32_t word = 0u;
+#pragma unroll
+        for (int r = 0; r < 8; ++r) word |= (swar_greater(q[r], lo7[r], t) >> 7) << r;
+        out[(long long)i * words] = word;
+    }
+}
+
 // --------------------------------------------------------------- packed --
 //
 // One lane per output word (32 samples), so every store is a coalesced
@@ -316,6 +382,23 @@ extern "C" int bitlogic_encode_thermometer_both(const uint8_t* x, int64_t B, int
                                                 float* bits, uint8_t* bits8, cudaStream_t stream) {
     if (B > 0 && !bits8) return BITLOGIC_ERR_NULL;
     return encode_impl(x, B, d, thr_host, b, bits, bits8, stream);
+}
+
+extern "C" int bitlogic_encode_thermometer_bitrows(const uint8_t* x, int64_t B, int32_t d,
+                                                   const uint8_t* thr_host, int32_t b,
+                                                   uint32_t* bits, cudaStream_t stream) {
+    Thresholds th;
+    int st = make_thresholds(thr_host, b, &th);
+    if (st) return st;
+    if (B < 0 || d <= 0) return BITLOGIC_ERR_SHAPE;
+    if (B == 0) return BITLOGIC_OK;   // an empty batch may come as NULL
+    if (!x || !bits) return BITLOGIC_ERR_NULL;
+    const long long nblk = (B + kBitBlock - 1) / kBitBlock;
+    if (nblk > 65535) return BITLOGIC_ERR_SHAPE;
+    const bool vec8 = (d % 8 == 0) && (reinterpret_cast<uintptr_t>(x) & 7u) == 0;
+    dim3 grid((unsigned)((d + kBitsTF - 1) / kBitsTF), (unsigned)nblk);
+    encode_bitrows_kernel<<<grid, 256, 0, stream>>>(x, B, d, th, bits, nblk * 32, vec8);
+    return launch_status();
 }
 
 extern "C" int bitlogic_pack_bits(const uint8_t* x, int64_t N, int32_t d,

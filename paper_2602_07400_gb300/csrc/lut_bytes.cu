@@ -121,6 +121,67 @@ lut_forward_u8_kernel(const uint8_t* __restrict__ X, int w_in, long long B, cons
     }
 }
 
+// The same forward on wire bit rows (one bit per sample; see kBitBlock): per
+// 1024-sample block each lane loads one 32-bit word per input row and finds
+// stage r's 4 samples' wires as bytes of (word >> r) & 0x01010101, so the
+// layer input is an eighth of the byte rows (12 MB at the CIFAR-100 shape,
+// resident in L2) and one load serves 32 samples.  Lanes, samples and
+// outputs are those of the byte-row form.  VEC: B % 4 == 0 and 16-byte
+// aligned Y (float4 stores), else per-sample stores.
+template <int k, bool VEC>
+__global__ void __launch_bounds__(kBytesFwdWarps * 32)
+lut_forward_bits_kernel(const uint32_t* __restrict__ X, int w_in, long long B, long long words,
+                        const int* __restrict__ conn, const float* __restrict__ theta, int w, int node,
+                        float* __restrict__ Y, long long chunk_blocks) {
+    constexpr int K = 1 << k;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int j = blockIdx.x * kBytesFwdWarps + warp;
+    if (j >= w) return;   // warp-uniform
+    const uint32_t* xr[k];
+    bool bad = false;
+#pragma unroll
+    for (int i = 0; i < k; ++i) {
+        int c = __ldg(conn + (long long)j * k + i);
+        if ((unsigned)c >= (unsigned)w_in) {
+            bad = true;
+            c = 0;
+        }
+        xr[i] = X + (long long)c * words + lane;
+    }
+    if (bad && lane == 0) flag_index_error();
+    const float lo = lane < K ? node_entry(__ldg(theta + (long long)j * K + lane), node) : 0.f;
+    const float hi = K > 32 ? node_entry(__ldg(theta + (long long)j * K + 32 + (lane & 31)), node) : 0.f;
+    const long long nblk = words / 32;
+    const long long b0 = (long long)blockIdx.y * chunk_blocks;
+    const long long b1 = min(nblk, b0 + chunk_blocks);
+    float* yr = Y + (long long)j * B;
+    for (long long blk = b0; blk < b1; ++blk) {
+        uint32_t wv[k];
+#pragma unroll
+        for (int i = 0; i < k; ++i) wv[i] = __ldg(xr[i] + blk * 32);
+#pragma unroll
+        for (int r = 0; r < 8; ++r) {
+            const long long s4 = blk * kBitBlock + 128 * r + 4 * lane;
+            uint32_t v = (wv[k - 1] >> r) & 0x01010101u;
+#pragma unroll
+            for (int i = k - 2; i >= 0; --i) v = (v << 1) | ((wv[i] >> r) & 0x01010101u);
+            float4 y;
+            y.x = table_at<K>(lo, hi, v & 0xffu);
+            y.y = table_at<K>(lo, hi, (v >> 8) & 0xffu);
+            y.z = table_at<K>(lo, hi, (v >> 16) & 0xffu);
+            y.w = table_at<K>(lo, hi, v >> 24);
+            if constexpr (VEC) {
+                if (s4 < B) __stcs(reinterpret_cast<float4*>(yr + s4), y);
+            } else {
+                if (s4 < B) yr[s4] = y.x;
+                if (s4 + 1 < B) yr[s4 + 1] = y.y;
+                if (s4 + 2 < B) yr[s4 + 2] = y.z;
+                if (s4 + 3 < B) yr[s4 + 3] = y.w;
+            }
+        }
+    }
+}
+
 // Samples per warp: the whole batch unless that leaves fewer than about two
 // waves of warps (then slices of at least 512 samples, a multiple of 128).
 // Slicing the batch so that a slice of the layer input stays in L2 was
@@ -153,6 +214,24 @@ int launch_forward_u8(const uint8_t* X, int w_in, long long B, const int* conn, 
     return launch_status();
 }
 
+template <int k>
+int launch_forward_bits(const uint32_t* X, int w_in, long long B, const int* conn, const float* theta, int w,
+                        int node, float* Y, cudaStream_t st) {
+    const long long nblk = (B + kBitBlock - 1) / kBitBlock;
+    long long chunk = (forward_u8_chunk(w, B) + kBitBlock - 1) / kBitBlock;   // in blocks
+    if (chunk < 1) chunk = 1;
+    const long long ny = (nblk + chunk - 1) / chunk;
+    if (ny > 65535) return BITLOGIC_ERR_SHAPE;
+    dim3 grid((unsigned)((w + kBytesFwdWarps - 1) / kBytesFwdWarps), (unsigned)ny);
+    if (B % 4 == 0 && aligned16(Y))
+        lut_forward_bits_kernel<k, true><<<grid, kBytesFwdWarps * 32, 0, st>>>(X, w_in, B, nblk * 32, conn, theta,
+                                                                               w, node, Y, chunk);
+    else
+        lut_forward_bits_kernel<k, false><<<grid, kBytesFwdWarps * 32, 0, st>>>(X, w_in, B, nblk * 32, conn, theta,
+                                                                                w, node, Y, chunk);
+    return launch_status();
+}
+
 }  // namespace
 }  // namespace bitlogic
 
@@ -177,5 +256,26 @@ extern "C" int bitlogic_lut_forward_u8(const uint8_t* X, int32_t w_in, int64_t B
         case 4: return launch_forward_u8<4>(X, w_in, B, conn, theta, w, node, Y, stream);
         case 5: return launch_forward_u8<5>(X, w_in, B, conn, theta, w, node, Y, stream);
         default: return launch_forward_u8<6>(X, w_in, B, conn, theta, w, node, Y, stream);
+    }
+}
+
+extern "C" int bitlogic_lut_forward_bitrows(const uint32_t* X, int32_t w_in, int64_t B, const int32_t* conn,
+                                            const float* theta, int32_t w, int32_t k, int32_t node, float* Y,
+                                            cudaStream_t stream) {
+    if (!conn || !theta) return BITLOGIC_ERR_NULL;
+    if (B > 0 && (!X || !Y)) return BITLOGIC_ERR_NULL;   // an empty batch may come as NULL
+    if (w_in <= 0 || w <= 0 || B < 0) return BITLOGIC_ERR_SHAPE;
+    if (k < 1 || k > 6 || k > w_in) return BITLOGIC_ERR_FANIN;
+    if ((int64_t)w * k > 0x7fffffffLL) return BITLOGIC_ERR_SHAPE;
+    if (node != BITLOGIC_NODE_SOFT && node != BITLOGIC_NODE_ST) return BITLOGIC_ERR_NODE;
+    if (B == 0) return BITLOGIC_OK;
+    if ((reinterpret_cast<uintptr_t>(X) & 3u) != 0) return BITLOGIC_ERR_ALIGN;
+    switch (k) {
+        case 1: return launch_forward_bits<1>(X, w_in, B, conn, theta, w, node, Y, stream);
+        case 2: return launch_forward_bits<2>(X, w_in, B, conn, theta, w, node, Y, stream);
+        case 3: return launch_forward_bits<3>(X, w_in, B, conn, theta, w, node, Y, stream);
+        case 4: return launch_forward_bits<4>(X, w_in, B, conn, theta, w, node, Y, stream);
+        case 5: return launch_forward_bits<5>(X, w_in, B, conn, theta, w, node, Y, stream);
+        default: return launch_forward_bits<6>(X, w_in, B, conn, theta, w, node, Y, stream);
     }
 }

@@ -499,11 +499,17 @@ constexpr int kBytesWarps = BITLOGIC_BYTES_WARPS;   // warps (nodes) per block
 constexpr int kBytesChunk = BITLOGIC_BYTES_CHUNK;   // stages per chunk
 constexpr int kBytesUnroll = BITLOGIC_BYTES_UNROLL;   // term rows whose loads are issued together
 
-template <int k, bool TERMS>
+// BITS: the input is wire bit rows (one bit per sample, `words` 32-bit words
+// per row; see kBitBlock) instead of byte rows: a chunk's 4 stages lie in one
+// 1024-sample block, so each lane loads one word per input row per chunk and
+// finds stage r's 4 wires as bytes of (word >> r) & 0x01010101.
+static_assert((kBitBlock / kTStageSamples) % kBytesChunk == 0, "a chunk's stages lie in one bit-row block");
+
+template <int k, bool TERMS, bool BITS>
 __global__ void __launch_bounds__(kBytesWarps * 32)
-lut_theta_bytes_kernel(const uint8_t* __restrict__ X, int w_in, long long B, const int* __restrict__ conn,
-                       const float* __restrict__ theta, int w, GradIn gi, float* __restrict__ dtheta,
-                       float* __restrict__ dY_out) {
+lut_theta_bytes_kernel(const void* __restrict__ Xv, int w_in, long long B, long long words,
+                       const int* __restrict__ conn, const float* __restrict__ theta, int w, GradIn gi,
+                       float* __restrict__ dtheta, float* __restrict__ dY_out) {
     constexpr int K = 1 << k, CH = kTStageSamples;
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -513,7 +519,8 @@ lut_theta_bytes_kernel(const uint8_t* __restrict__ X, int w_in, long long B, con
 #pragma unroll
     for (int a = 0; a < K; ++a) col[a * 32] = 0.f;
     bool bad = false;
-    const uint8_t* xr[k];
+    const uint8_t* xr[k];                 // byte rows: the lane's first 4 bytes
+    const uint32_t* xb[k];                // bit rows: the lane's word of block 0
 #pragma unroll
     for (int i = 0; i < k; ++i) {
         int c = __ldg(conn + (long long)j * k + i);
@@ -521,7 +528,8 @@ lut_theta_bytes_kernel(const uint8_t* __restrict__ X, int w_in, long long B, con
             bad = true;
             c = 0;
         }
-        xr[i] = X + (long long)c * B + 4 * lane;
+        if constexpr (BITS) xb[i] = static_cast<const uint32_t*>(Xv) + (long long)c * words + lane;
+        else xr[i] = static_cast<const uint8_t*>(Xv) + (long long)c * B + 4 * lane;
     }
     // the node's term rows: CSR positions e0 .. e0 + deg - 1, ids of the
     // first 32 one per lane
@@ -553,12 +561,17 @@ lut_theta_bytes_kernel(const uint8_t* __restrict__ X, int w_in, long long B, con
         bool in[kBytesChunk];
 #pragma unroll
         for (int c = 0; c < kBytesChunk; ++c) in[c] = c0 + c < nst && (long long)(c0 + c) * CH + 4 * lane < B;
-        uint32_t xw[kBytesChunk][k];
+        uint32_t xw[BITS ? 1 : kBytesChunk][k];
+        if constexpr (BITS) {
 #pragma unroll
-        for (int c = 0; c < kBytesChunk; ++c)
+            for (int i = 0; i < k; ++i) xw[0][i] = __ldg(xb[i] + (long long)(c0 / 8) * 32);
+        } else {
 #pragma unroll
-            for (int i = 0; i < k; ++i)
-                xw[c][i] = in[c] ? __ldg(reinterpret_cast<const uint32_t*>(xr[i] + (long long)(c0 + c) * CH)) : 0u;
+            for (int c = 0; c < kBytesChunk; ++c)
+#pragma unroll
+                for (int i = 0; i < k; ++i)
+                    xw[c][i] = in[c] ? __ldg(reinterpret_cast<const uint32_t*>(xr[i] + (long long)(c0 + c) * CH)) : 0u;
+        }
         float4 g[kBytesChunk];
 #pragma unroll
         for (int c = 0; c < kBytesChunk; ++c) g[c] = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -599,9 +612,14 @@ lut_theta_bytes_kernel(const uint8_t* __restrict__ X, int w_in, long long B, con
         for (int c = 0; c < kBytesChunk; ++c) {
             if (in[c]) {
                 if (dY_out) *reinterpret_cast<float4*>(dY_out + (long long)j * B + (long long)(c0 + c) * CH + 4 * lane) = g[c];
-                uint32_t v = xw[c][k - 1] & 0x01010101u;
+                // the 4 samples' wires of input i, as bytes 0 / 1
+                auto wire4 = [&](int i) {
+                    if constexpr (BITS) return (xw[0][i] >> ((c0 & 7) + c)) & 0x01010101u;
+                    else return xw[c][i] & 0x01010101u;
+                };
+                uint32_t v = wire4(k - 1);
 #pragma unroll
-                for (int i = k - 2; i >= 0; --i) v = (v << 1) | (xw[c][i] & 0x01010101u);
+                for (int i = k - 2; i >= 0; --i) v = (v << 1) | wire4(i);
                 corner_add4(col, v, g[c]);
             }
         }
@@ -622,24 +640,16 @@ lut_theta_bytes_kernel(const uint8_t* __restrict__ X, int w_in, long long B, con
     }
 }
 
-template <int k>
-int launch_bytes(bool terms, const uint8_t* X, int w_in, long long B, const int* conn, const float* theta, int w,
+template <int k, bool BITS>
+int launch_bytes(bool terms, const void* X, int w_in, long long B, const int* conn, const float* theta, int w,
                  const GradIn& gi, float* dtheta, float* dY_out, cudaStream_t st) {
     constexpr int smem = kBytesWarps * (1 << k) * 32 * (int)sizeof(float);
     const unsigned blocks = (unsigned)((w + kBytesWarps - 1) / kBytesWarps);
-    if (smem > 40 * 1024) {
-        auto kt = lut_theta_bytes_kernel<k, true>;
-        auto kr = lut_theta_bytes_kernel<k, false>;
-        if (cudaFuncSetAttribute(kt, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess ||
-            cudaFuncSetAttribute(kr, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
-            return BITLOGIC_ERR_CUDA;
-    }
-    if (terms)
-        lut_theta_bytes_kernel<k, true><<<blocks, kBytesWarps * 32, smem, st>>>(X, w_in, B, conn, theta, w, gi,
-                                                                              dtheta, dY_out);
-    else
-        lut_theta_bytes_kernel<k, false><<<blocks, kBytesWarps * 32, smem, st>>>(X, w_in, B, conn, theta, w, gi,
-                                                                               dtheta, dY_out);
+    const long long words = (B + kBitBlock - 1) / kBitBlock * 32;
+    auto kern = terms ? lut_theta_bytes_kernel<k, true, BITS> : lut_theta_bytes_kernel<k, false, BITS>;
+    if (smem > 40 * 1024 && cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
+        return BITLOGIC_ERR_CUDA;
+    kern<<<blocks, kBytesWarps * 32, smem, st>>>(X, w_in, B, words, conn, theta, w, gi, dtheta, dY_out);
     return launch_status();
 }
 
@@ -753,11 +763,11 @@ extern "C" int bitlogic_lut_backward_through_u8(const uint8_t* X, int32_t w_in, 
                                      up_group, up_off, up_edge, dtheta, dY_out, stream);
 }
 
-extern "C" int bitlogic_lut_backward_u8(const uint8_t* X, int32_t w_in, int64_t B, const int32_t* conn,
-                                        const float* theta, int32_t w, int32_t k, int32_t node,
-                                        const float* dY, int32_t dy_group, const float* up_terms,
-                                        const int32_t* up_off, const int32_t* up_edge, int32_t up_edges,
-                                        float* dtheta, float* dY_out, cudaStream_t stream) {
+namespace {
+int backward_bytes(const void* X, int32_t w_in, int64_t B, const int32_t* conn, const float* theta, int32_t w,
+                   int32_t k, int32_t node, const float* dY, int32_t dy_group, const float* up_terms,
+                   const int32_t* up_off, const int32_t* up_edge, int32_t up_edges, float* dtheta, float* dY_out,
+                   bool bits, cudaStream_t stream) {
     int st = check_common(X, w_in, B, conn, theta, w, k, node, dtheta);
     if (st) return st;
     const bool terms = up_terms != nullptr;
@@ -782,12 +792,35 @@ extern "C" int bitlogic_lut_backward_u8(const uint8_t* X, int32_t w_in, int64_t 
     gi.n_terms = up_edges;
     gi.off = up_off;
     gi.edge = up_edge;
+#define BITLOGIC_BYTES_K(K)                                                                           \
+    return bits ? launch_bytes<K, true>(terms, X, w_in, B, conn, theta, w, gi, dtheta, dY_out, stream) \
+                : launch_bytes<K, false>(terms, X, w_in, B, conn, theta, w, gi, dtheta, dY_out, stream)
     switch (k) {
-        case 1: return launch_bytes<1>(terms, X, w_in, B, conn, theta, w, gi, dtheta, dY_out, stream);
-        case 2: return launch_bytes<2>(terms, X, w_in, B, conn, theta, w, gi, dtheta, dY_out, stream);
-        case 3: return launch_bytes<3>(terms, X, w_in, B, conn, theta, w, gi, dtheta, dY_out, stream);
-        case 4: return launch_bytes<4>(terms, X, w_in, B, conn, theta, w, gi, dtheta, dY_out, stream);
-        case 5: return launch_bytes<5>(terms, X, w_in, B, conn, theta, w, gi, dtheta, dY_out, stream);
-        default: return launch_bytes<6>(terms, X, w_in, B, conn, theta, w, gi, dtheta, dY_out, stream);
+        case 1: BITLOGIC_BYTES_K(1);
+        case 2: BITLOGIC_BYTES_K(2);
+        case 3: BITLOGIC_BYTES_K(3);
+        case 4: BITLOGIC_BYTES_K(4);
+        case 5: BITLOGIC_BYTES_K(5);
+        default: BITLOGIC_BYTES_K(6);
     }
+#undef BITLOGIC_BYTES_K
+}
+}  // namespace
+
+extern "C" int bitlogic_lut_backward_u8(const uint8_t* X, int32_t w_in, int64_t B, const int32_t* conn,
+                                        const float* theta, int32_t w, int32_t k, int32_t node,
+                                        const float* dY, int32_t dy_group, const float* up_terms,
+                                        const int32_t* up_off, const int32_t* up_edge, int32_t up_edges,
+                                        float* dtheta, float* dY_out, cudaStream_t stream) {
+    return backward_bytes(X, w_in, B, conn, theta, w, k, node, dY, dy_group, up_terms, up_off, up_edge, up_edges,
+                          dtheta, dY_out, false, stream);
+}
+
+extern "C" int bitlogic_lut_backward_bitrows(const uint32_t* X, int32_t w_in, int64_t B, const int32_t* conn,
+                                             const float* theta, int32_t w, int32_t k, int32_t node,
+                                             const float* dY, int32_t dy_group, const float* up_terms,
+                                             const int32_t* up_off, const int32_t* up_edge, int32_t up_edges,
+                                             float* dtheta, float* dY_out, cudaStream_t stream) {
+    return backward_bytes(X, w_in, B, conn, theta, w, k, node, dY, dy_group, up_terms, up_off, up_edge, up_edges,
+                          dtheta, dY_out, true, stream);
 }

@@ -24,7 +24,8 @@ from . import (NODE_FORMS, bitlogic_adamw_update, bitlogic_binarize_tables, bitl
                bitlogic_lut_backward_u8, bitlogic_lut_forward_node,
                bitlogic_pack_bits, bitlogic_route_backward, bitlogic_route_backward_u8, bitlogic_route_forward,
                bitlogic_route_forward_u8, bitlogic_route_snap, bitlogic_encode_thermometer_u8,
-               bitlogic_lut_forward_u8)
+               bitlogic_lut_forward_u8, bitlogic_encode_thermometer_bitrows, bitlogic_lut_forward_bitrows,
+               bitlogic_lut_backward_bitrows, bitrow_words)
 
 
 def _nomark(name: str) -> None:
@@ -182,7 +183,14 @@ class TrainStep:
     (bitlogic_lut_backward_u8 / _through on byte rows); the encoder then
     writes byte rows only, and ``bits`` is that uint8 tensor.  The table
     gradient equals the fp32-row form bit for bit; the forward returns the
-    table entry itself, which the fp32 lerp tree reaches up to rounding.  Set
+    table entry itself, which the fp32 lerp tree reaches up to rounding.
+    With ``bits1`` (the default on byte wires off the through route) the
+    wires are kept at one bit per sample instead, an eighth of the bytes (the
+    CIFAR-100-shaped layer input then stays in L2):
+    bitlogic_encode_thermometer_bitrows writes them and the layer-1 kernels
+    read those words (bitlogic_lut_forward_bitrows / _backward_bitrows) with
+    the same results bit for bit; ``bits`` is then the int32 tensor of words
+    and ``wires()`` writes the wires out as bytes on demand.  Set
     ``keep_dy1`` to also write dY1 (e.g. to check it).  ``node`` picks the
     LightLUT form of both layers: "soft", or "st" (hard table samples in the
     forward, straight-through gradient to the logits)."""
@@ -190,7 +198,8 @@ class TrainStep:
     def __init__(self, net: Network, B: int, d: int, thresholds: Sequence[int], C: int,
                  tau: float, want_dx1: bool = False, keep_dy1: bool = False,
                  fuse_dy1: Optional[bool] = None, csr_order: bool = True, node: str = "soft",
-                 through: Optional[bool] = None, bytes1: Optional[bool] = None, device="cuda"):
+                 through: Optional[bool] = None, bytes1: Optional[bool] = None,
+                 bits1: Optional[bool] = None, device="cuda"):
         dev = torch.device(device)
         if node not in NODE_FORMS:
             raise ValueError(f"node must be one of {sorted(NODE_FORMS)}")
@@ -223,8 +232,17 @@ class TrainStep:
         if bytes1 and (B % 4 != 0 or want_dx1):
             raise ValueError("byte wires for layer 1 need B % 4 == 0 and no layer-1 input gradient")
         self.bytes1 = bool(bytes1)
-        # the encoder's output: byte rows (bytes1) or fp32 rows
-        self.bits = torch.empty(net.w_in, B, dtype=torch.uint8 if self.bytes1 else torch.float32, device=dev)
+        if bits1 is None:
+            bits1 = self.bytes1 and not self.through
+        if bits1 and not (self.bytes1 and not self.through):
+            raise ValueError("wire bit rows need byte wires for layer 1 and a route other than through")
+        self.bits1 = bool(bits1)
+        # the encoder's output: wire bit rows (bits1), byte rows (bytes1) or
+        # fp32 rows
+        if self.bits1:
+            self.bits = torch.empty(net.w_in, bitrow_words(B), dtype=torch.int32, device=dev)
+        else:
+            self.bits = torch.empty(net.w_in, B, dtype=torch.uint8 if self.bytes1 else torch.float32, device=dev)
         # per-edge terms stored in CSR order (each input's terms contiguous,
         # read without the edge map) instead of edge order
         self.csr_order = bool(csr_order)
@@ -244,7 +262,11 @@ class TrainStep:
 
     def forward(self, stream=None, mark=_nomark):
         n = self.net
-        if self.bytes1:
+        if self.bits1:
+            bitlogic_encode_thermometer_bitrows(self.x, self.thr, self.bits, stream)
+            mark("encode")
+            bitlogic_lut_forward_bitrows(self.bits, self.B, n.conn1, n.theta1, self.y1, self.node, stream)
+        elif self.bytes1:
             bitlogic_encode_thermometer_u8(self.x, self.thr, self.bits, stream)
             mark("encode")
             bitlogic_lut_forward_u8(self.bits, n.conn1, n.theta1, self.y1, self.node, stream)
@@ -281,7 +303,10 @@ class TrainStep:
         mark("backward2")
         pos1 = n.pos1 if (co and self.edges1 is not None) else None
         edge2 = None if co else n.edge2
-        if self.fuse_dy1 and self.bytes1:
+        if self.fuse_dy1 and self.bits1:
+            bitlogic_lut_backward_bitrows(self.bits, self.B, n.conn1, n.theta1, self.dth1, nd, up_terms=self.edges2,
+                                          up_off=n.off2, up_edge=edge2, dY_out=self.dy1, stream=stream)
+        elif self.fuse_dy1 and self.bytes1:
             bitlogic_lut_backward_u8(self.bits, n.conn1, n.theta1, self.dth1, nd, up_terms=self.edges2,
                                      up_off=n.off2, up_edge=edge2, dY_out=self.dy1, stream=stream)
         elif self.fuse_dy1:
@@ -291,7 +316,10 @@ class TrainStep:
         else:
             bitlogic_csr_reduce(self.edges2, n.off2, edge2, self.dy1, stream)
             mark("csr2")
-            if self.bytes1:
+            if self.bits1:
+                bitlogic_lut_backward_bitrows(self.bits, self.B, n.conn1, n.theta1, self.dth1, nd, dY=self.dy1,
+                                              stream=stream)
+            elif self.bytes1:
                 bitlogic_lut_backward_u8(self.bits, n.conn1, n.theta1, self.dth1, nd, dY=self.dy1, stream=stream)
             else:
                 bitlogic_lut_backward_node(self.bits, n.conn1, n.theta1, self.dth1, nd, dY=self.dy1,
@@ -304,6 +332,16 @@ class TrainStep:
     def run(self, stream=None, mark=_nomark):
         self.forward(stream, mark)
         self.backward(stream, mark)
+
+    def wires(self, stream=None) -> torch.Tensor:
+        """Layer 1's input wires [w_in, B]: ``bits``, or under ``bits1`` the
+        thermometer of the loaded samples written out as bytes into a new
+        tensor."""
+        if not self.bits1:
+            return self.bits
+        out = torch.empty(self.net.w_in, self.B, dtype=torch.uint8, device=self.bits.device)
+        bitlogic_encode_thermometer_u8(self.x, self.thr, out, stream)
+        return out
 
     def capture(self) -> torch.cuda.CUDAGraph:
         """One run() (forward + backward) as a CUDA graph: a replay launches

@@ -194,6 +194,26 @@ def test_host_validation_returns_before_any_launch():
     assert fwd_u8(fake, 8, 64, fake, fake, 4, 2, 0, None, None) == -1
     assert fwd_u8(fake, 8, 64, None, fake, 4, 2, 0, fake, None) == -1
     assert fwd_u8(None, 8, 0, fake, fake, 4, 2, 0, None, None) == 0
+    # wire bit rows: encoder thresholds and shapes, forward and backward
+    # checks as on byte rows, 4-byte aligned words, B % 4 == 0 for the
+    # backward (B = 0 is a no-op)
+    enc_b, fwd_b, bwd_b = (lib.bitlogic_encode_thermometer_bitrows, lib.bitlogic_lut_forward_bitrows,
+                           lib.bitlogic_lut_backward_bitrows)
+    assert enc_b(fake, 64, 4, thr, 0, fake, None) == -9
+    assert enc_b(fake, 64, 0, thr, 3, fake, None) == -2
+    assert enc_b(None, 64, 4, thr, 3, fake, None) == -1
+    assert enc_b(None, 0, 4, thr, 3, None, None) == 0
+    assert fwd_b(fake, 8, 64, fake, fake, 4, 2, 2, fake, None) == -12
+    assert fwd_b(fake, 8, 64, fake, fake, 4, 7, 0, fake, None) == -3
+    assert fwd_b(fake, 0, 64, fake, fake, 4, 2, 0, fake, None) == -2
+    assert fwd_b(None, 8, 64, fake, fake, 4, 2, 0, fake, None) == -1
+    assert fwd_b(P(18), 8, 64, fake, fake, 4, 2, 0, fake, None) == -4
+    assert fwd_b(None, 8, 0, fake, fake, 4, 2, 0, None, None) == 0
+    assert bwd_b(fake, 8, 64, fake, fake, 4, 2, 0, None, 1, None, None, None, 0, fake, None, None) == -1
+    assert bwd_b(fake, 8, 64, fake, fake, 4, 2, 0, fake, 1, fake, fake, None, 4, fake, None, None) == -1
+    assert bwd_b(fake, 8, 64, fake, fake, 4, 2, 0, fake, 3, None, None, None, 0, fake, None, None) == -2
+    assert bwd_b(fake, 8, 66, fake, fake, 4, 2, 0, fake, 1, None, None, None, 0, fake, None, None) == -4
+    assert bwd_b(fake, 8, 64, fake, fake, 4, 2, 2, fake, 1, None, None, None, 0, fake, None, None) == -12
 
 
 @pytest.mark.parametrize("n,b,seed", [(1, 1, 0), (5, 4, 1), (1000, 8, 2), (65537, 32, 3), (300, 15, 4)])

@@ -166,6 +166,21 @@ def test_byte_wire_layer1_work_and_kernel_names():
     assert bench.kernels_of_step(st)["backward1"] == "lut_theta_through_kernel<k, ku, uint8_t>"
     st = types.SimpleNamespace(bytes1=False, through=False, fuse_dy1=False)
     assert bench.kernels_of_step(st)["backward1"] == bench.KERNEL_OF_CALL["backward1"]
+    # wire bit rows: one bit per wire and sample (32 words per 1024-sample
+    # block), written by the encoder and read by both layer-1 calls
+    bw = bench.call_work(wl, B, fuse_dy1=True, bytes1=True, bits1=True)
+    xw1 = 4 * w_in * 64            # B = 2048: two blocks of 32 words per row
+    assert xw1 * 8 == w_in * B
+    assert bw["encode"][0] == B * d + xw1
+    assert bw["forward1"][0] == xw1 + 4 * (w1 * B + w1 * K + w1 * k)
+    assert bw["backward1"][0] == u8["backward1"][0] - w_in * B + xw1
+    assert bw["backward1"][2] - bw["backward1"][0] == u8["backward1"][2] - u8["backward1"][0]
+    assert bw["forward2"] == u8["forward2"] and bw["backward1"][1] == w1 * B
+    st = types.SimpleNamespace(bytes1=True, bits1=True, through=False, fuse_dy1=True)
+    names = bench.kernels_of_step(st)
+    assert names["encode"] == "encode_bitrows_kernel" and names["forward1"].startswith("lut_forward_bits_kernel")
+    assert "bit rows" in names["backward1"]
+    assert bench.route_of_step(st)["layer1_wires"].startswith("bits")
 
 
 def test_hard_roofline_uses_the_measured_mix_rate():

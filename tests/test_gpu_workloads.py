@@ -33,7 +33,7 @@ oracle.set_threads(os.cpu_count() or 1)
 
 
 def _step(wl, want_dx1, seed=0, k=None, keep_dy1=True, fuse_dy1=None, csr_order=True, node="soft", through=None,
-          bytes1=None):
+          bytes1=None, bits1=None):
     if k is not None:
         wl = synth.Workload(wl.name, wl.batch, wl.d, wl.classes, wl.sigma, wl.thresholds, wl.widths, k, wl.tau)
     conn1, th1, conn2, th2 = synth.network(wl, seed)
@@ -41,7 +41,7 @@ def _step(wl, want_dx1, seed=0, k=None, keep_dy1=True, fuse_dy1=None, csr_order=
     net = Network(conn1, th1, conn2, th2, wl.w_in)
     st = TrainStep(net, wl.batch, wl.d, wl.thresholds, wl.classes, wl.tau, want_dx1=want_dx1,
                    keep_dy1=keep_dy1, fuse_dy1=fuse_dy1, csr_order=csr_order, node=node, through=through,
-                   bytes1=bytes1)
+                   bytes1=bytes1, bits1=bits1)
     st.load(x.cuda(), labels.cuda())
     st.run()
     torch.cuda.synchronize()
@@ -60,7 +60,7 @@ def _full_compare(wl, st, x, labels, params, want_dx1, node="soft"):
     conn1, th1, conn2, th2 = params
     r = oracle.train_step(x, labels, wl.thresholds, conn1, th1, conn2, th2, wl.classes, wl.tau,
                           want_dx1=want_dx1, node=node)
-    check_exact(st.bits.cpu().numpy().astype(np.float64), r["bits"], "bits")
+    check_exact(st.wires().cpu().numpy().astype(np.float64), r["bits"], "bits")
     if node == "st":   # hard tables on binary inputs: every activation is a table entry
         check_exact(st.y1.cpu().numpy().astype(np.float64), r["y1"], "y1")
         check_exact(st.y2.cpu().numpy().astype(np.float64), r["y2"], "y2")
@@ -136,7 +136,7 @@ def test_byte_wires_for_layer1_match_fp32_wires(k, route):
     # inside the byte-row kernel; csr: the CSR reduction first), and the
     # through kernel on fp32 rows (k = 2)
     kw = {"fused": dict(fuse_dy1=True), "csr": dict(fuse_dy1=False), "through": {}}[route]
-    wl, a, *_ = _step(synth.WORKLOADS["mnist"], want_dx1=False, k=k, **kw)
+    wl, a, *_ = _step(synth.WORKLOADS["mnist"], want_dx1=False, k=k, bits1=False, **kw)
     assert a.bytes1 and a.bits.dtype == torch.uint8 and a.through == (route == "through")
     n = a.net
     bits32 = a.bits.float()
@@ -151,6 +151,23 @@ def test_byte_wires_for_layer1_match_fp32_wires(k, route):
     else:
         bl.bitlogic_lut_backward_node(bits32, n.conn1, n.theta1, ref, "soft", dY=a.dy1)
     check_exact(a.dth1.cpu().numpy(), ref.cpu().numpy(), "dtheta1 (byte rows vs fp32 rows)")
+    assert bl.bitlogic_device_error() == 0
+
+
+@pytest.mark.parametrize("route", ["fused", "csr"])
+def test_wire_bit_rows_equal_byte_wires(route):
+    # the step's default off the through route: layer 1's wires at one bit
+    # per sample; the lookup forward and the one-hot table gradient read the
+    # same wires in the same order as the byte-row kernels, so every output
+    # equals theirs bit for bit
+    kw = dict(fuse_dy1=route == "fused")
+    wl, a, *_ = _step(synth.WORKLOADS["mnist"], want_dx1=False, k=6, **kw)
+    assert a.bits1 and a.bits.dtype == torch.int32 and a.bits.shape == (wl.w_in, bl.bitrow_words(wl.batch))
+    _, b, *_ = _step(synth.WORKLOADS["mnist"], want_dx1=False, k=6, bits1=False, **kw)
+    assert not b.bits1 and b.bits.dtype == torch.uint8
+    check_exact(a.wires().cpu().numpy(), b.bits.cpu().numpy(), "wires")
+    for name in ("y1", "y2", "logits", "loss", "dyg", "dy1", "dth1", "dth2"):
+        check_exact(getattr(a, name).cpu().numpy(), getattr(b, name).cpu().numpy(), name)
     assert bl.bitlogic_device_error() == 0
 
 
