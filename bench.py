@@ -370,20 +370,28 @@ TRAFFIC = {
         "sha256": "78edac247d6c64dc0042c15287b5174dfc03ecac6e7945ec4beb26e9e6cc6800",
         "note": "ncu capture of this workload (one-pass DRAM metrics)"},
     ("cifar10", "forward1"): {
-        "bytes": 42786816 + 199091456, "source": "lut_bytes.cu",
-        "sha256": "e65fff6a177a4f30744daa6ea751b933665c0db5387208a8689380c7f9d81ef8",
+        "bytes": 20694272 + 196729088, "source": "lut_bytes.cu",
+        "sha256": "88cd7e78b309d49ee5835ba21aeb26fbdf1a8e144188cac4f9338e562f6c3f57",
         "note": "ncu capture of this workload (one-pass DRAM metrics)"},
     ("cifar10", "backward1"): {
-        "bytes": 1613265664 + 3451136, "source": "lut_through.cu",
-        "sha256": "1ccfe000d8131c42950c67c661f1be21f83f53ac829efb4a363e9e33a38e73a4",
+        "bytes": 1593852672 + 3620608, "source": "lut_through.cu",
+        "sha256": "7c8274d9e0ac03637e86af0d7b0c6716a0d8e84b412c07fc0a513d0cc3e3485b",
         "note": "ncu capture of this workload (one-pass DRAM metrics)"},
     ("cifar100", "forward1"): {
-        "bytes": 825120000 + 993534976, "source": "lut_bytes.cu",
-        "sha256": "e65fff6a177a4f30744daa6ea751b933665c0db5387208a8689380c7f9d81ef8",
+        "bytes": 50327040 + 984133120, "source": "lut_bytes.cu",
+        "sha256": "88cd7e78b309d49ee5835ba21aeb26fbdf1a8e144188cac4f9338e562f6c3f57",
         "note": "ncu capture of this workload (one-pass DRAM metrics)"},
     ("cifar100", "backward1"): {
-        "bytes": 6813448448 + 30162688, "source": "lut_through.cu",
-        "sha256": "1ccfe000d8131c42950c67c661f1be21f83f53ac829efb4a363e9e33a38e73a4",
+        "bytes": 6339823104 + 5000960, "source": "lut_through.cu",
+        "sha256": "7c8274d9e0ac03637e86af0d7b0c6716a0d8e84b412c07fc0a513d0cc3e3485b",
+        "note": "ncu capture of this workload (one-pass DRAM metrics)"},
+    ("cifar10", "encode"): {
+        "bytes": 3160576 + 0, "source": "encode.cu",
+        "sha256": "e6c29181c8e57f1b0f92ecd6dfdad87e8d79378c78599c3d42e80904a0b689a6",
+        "note": "ncu capture of this workload (one-pass DRAM metrics)"},
+    ("cifar100", "encode"): {
+        "bytes": 6312448 + 0, "source": "encode.cu",
+        "sha256": "e6c29181c8e57f1b0f92ecd6dfdad87e8d79378c78599c3d42e80904a0b689a6",
         "note": "ncu capture of this workload (one-pass DRAM metrics)"},
     ("hard_cifar10", "hard1"): {
         "bytes": 16 * (1.209681e9 + 2.054784e9), "source": "hard.cu",

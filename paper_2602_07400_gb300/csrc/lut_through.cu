@@ -104,14 +104,14 @@ __device__ __forceinline__ void corner_add4(float* col, uint32_t v, const float4
     col[(v >> 24) * 32] += g.w;
 }
 
-// Moves the lane's column into registers (for the butterfly) and clears it
-// for the next node.
-template <int K>
+// Moves the lane's column into registers (for the butterfly) and, with
+// CLEAR, clears it for the warp's next node.
+template <int K, bool CLEAR = true>
 __device__ __forceinline__ void corner_take(float* col, float (&acc)[K]) {
 #pragma unroll
     for (int a = 0; a < K; ++a) {
         acc[a] = col[a * 32];
-        col[a * 32] = 0.f;
+        if constexpr (CLEAR) col[a * 32] = 0.f;
     }
 }
 
@@ -626,7 +626,7 @@ lut_theta_bytes_kernel(const void* __restrict__ Xv, int w_in, long long B, long 
     }
     // the node's dtheta: butterfly over the lanes, then t (1 - t)
     float acc[K];
-    corner_take<K>(col, acc);
+    corner_take<K, false>(col, acc);   // the warp's only node
     reduce_scatter<K, 16>(acc, lane);
     constexpr int NF = K >= 32 ? K / 32 : 1;   // entries per lane
     constexpr int SH = K >= 32 ? 0 : 5 - k;    // lanes sharing an entry (K < 32)
