@@ -353,6 +353,13 @@ int bitlogic_lut_backward_u8(const uint8_t* X, int32_t w_in, int64_t B, const in
 
 /* bitlogic_lut_backward_u8 on wire bit rows: X device uint32 [w_in][W]
  * (the layout of bitlogic_encode_thermometer_bitrows), 16-byte aligned.
+ *   order  device int32 [w] or NULL: the order in which the kernel's warps
+ *          take the nodes (a permutation of 0 .. w-1; bitlogic_degree_order
+ *          over up_off puts the nodes with the most term rows first, which
+ *          shortens the launch's tail); NULL takes them in index order.  An
+ *          entry outside [0, w) raises the device flag and is skipped; a
+ *          repeated entry leaves another node's dtheta unwritten.  The
+ *          order does not change any result.
  * Every other argument, the result and the errors as
  * bitlogic_lut_backward_u8: the same wires give the same dtheta and dY_out
  * bit for bit (the samples are visited in the same order). */
@@ -360,7 +367,8 @@ int bitlogic_lut_backward_bitrows(const uint32_t* X, int32_t w_in, int64_t B, co
                                   const float* theta, int32_t w, int32_t k, int32_t node,
                                   const float* dY, int32_t dy_group, const float* up_terms,
                                   const int32_t* up_off, const int32_t* up_edge, int32_t up_edges,
-                                  float* dtheta, float* dY_out, cudaStream_t stream);
+                                  const int32_t* order, float* dtheta, float* dY_out,
+                                  cudaStream_t stream);
 
 /* Learnable routing (§3, the paragraph on connectivity: a per-slot
  * candidate pool whose selection is differentiable in training and snapped
@@ -516,6 +524,15 @@ int bitlogic_build_csr(const int32_t* conn_host, int32_t w, int32_t k, int32_t w
  * edge_host: pos_host[edge_host[p]] = p for p < n_edges.  Returns
  * BITLOGIC_ERR_INDEX unless edge_host is a permutation of [0, n_edges). */
 int bitlogic_csr_positions(const int32_t* edge_host, int32_t n_edges, int32_t* pos_host);
+
+/* Host: the nodes 0 .. n-1 by decreasing CSR degree off_host[i+1] -
+ * off_host[i] (ties in increasing i), the order in which
+ * bitlogic_lut_backward_bitrows can take the nodes of a layer whose output
+ * gradient it sums from the next layer's terms, so that the nodes with the
+ * most term rows start first and the launch ends on short ones.
+ * off_host [n+1] (off_host[0] == 0, non-decreasing: BITLOGIC_ERR_INDEX
+ * otherwise), order_host [n]. */
+int bitlogic_degree_order(const int32_t* off_host, int32_t n, int32_t* order_host);
 
 /* Synchronizes `stream`, then reports (and clears) the device-side index
  * flag: BITLOGIC_OK, or BITLOGIC_ERR_DEVICE when a kernel met an index out of

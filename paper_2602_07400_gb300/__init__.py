@@ -31,7 +31,8 @@ __all__ = [
     "bitlogic_lut_backward_u8", "bitlogic_lut_forward_u8", "bitlogic_encode_thermometer_bitrows",
     "bitlogic_lut_forward_bitrows", "bitlogic_lut_backward_bitrows", "bitrow_words",
     "bitlogic_head_loss", "bitlogic_binarize_tables", "bitlogic_pack_bits",
-    "bitlogic_hard_forward", "bitlogic_build_csr", "bitlogic_csr_positions", "bitlogic_device_error",
+    "bitlogic_hard_forward", "bitlogic_build_csr", "bitlogic_csr_positions", "bitlogic_degree_order",
+    "bitlogic_device_error",
     "bitlogic_adamw_update", "bitlogic_route_forward", "bitlogic_route_backward", "bitlogic_route_snap",
     "bitlogic_route_forward_u8", "bitlogic_route_backward_u8", "bitlogic_encode_thermometer_u8",
     "bitlogic_encode_thermometer_both",
@@ -84,7 +85,8 @@ _SIGS = {
     "bitlogic_encode_thermometer_bitrows": ([_P, _I64, _I32, _P, _I32, _P, _P], ctypes.c_int),
     "bitlogic_lut_forward_bitrows": ([_P, _I32, _I64, _P, _P, _I32, _I32, _I32, _P, _P], ctypes.c_int),
     "bitlogic_lut_backward_bitrows": ([_P, _I32, _I64, _P, _P, _I32, _I32, _I32, _P, _I32, _P, _P, _P, _I32, _P,
-                                       _P, _P], ctypes.c_int),
+                                       _P, _P, _P], ctypes.c_int),
+    "bitlogic_degree_order": ([_P, _I32, _P], ctypes.c_int),
     "bitlogic_lut_backward_workspace": ([_I32, _I64, _I32, _I32, _I32], _SZ),
     "bitlogic_lut_backward": ([_P, _I32, _I64, _P, _P, _I32, _I32, _P, _P, _P, _P, _P,
                                _P, _SZ, _P], ctypes.c_int),
@@ -614,8 +616,11 @@ def bitlogic_lut_backward_bitrows(X: torch.Tensor, B: int, conn: torch.Tensor, t
                                   dtheta: torch.Tensor, node="soft", dY: Optional[torch.Tensor] = None,
                                   dy_group: int = 1, up_terms: Optional[torch.Tensor] = None,
                                   up_off: Optional[torch.Tensor] = None, up_edge: Optional[torch.Tensor] = None,
-                                  dY_out: Optional[torch.Tensor] = None, stream=None):
-    """bitlogic_lut_backward_u8 on wire bit rows X [w_in, bitrow_words(B)] int32."""
+                                  dY_out: Optional[torch.Tensor] = None, order: Optional[torch.Tensor] = None,
+                                  stream=None):
+    """bitlogic_lut_backward_u8 on wire bit rows X [w_in, bitrow_words(B)] int32;
+    ``order`` (int32 [w], e.g. bitlogic_degree_order(up_off)) is the order
+    in which the nodes are taken (no effect on the results)."""
     w_in = X.shape[0]
     _need(X, "X", torch.int32, (w_in, bitrow_words(B)))
     w, k = conn.shape
@@ -635,9 +640,12 @@ def bitlogic_lut_backward_bitrows(X: torch.Tensor, B: int, conn: torch.Tensor, t
             _need(up_edge, "up_edge", torch.int32, (n_up,))
     if dY_out is not None:
         _need(dY_out, "dY_out", torch.float32, (w, B))
+    if order is not None:
+        _need(order, "order", torch.int32, (w,))
     _check("bitlogic_lut_backward_bitrows", load().bitlogic_lut_backward_bitrows(
         _ptr(X), w_in, B, _ptr(conn), _ptr(theta), w, k, _node_code(node), _ptr(dY), int(dy_group),
-        _ptr(up_terms), _ptr(up_off), _ptr(up_edge), n_up, _ptr(dtheta), _ptr(dY_out), _stream(stream)))
+        _ptr(up_terms), _ptr(up_off), _ptr(up_edge), n_up, _ptr(order), _ptr(dtheta), _ptr(dY_out),
+        _stream(stream)))
 
 
 def bitlogic_head_loss_ex(Y: torch.Tensor, labels: torch.Tensor, C: int, tau: float,
@@ -764,6 +772,16 @@ def bitlogic_adamw_update(theta: torch.Tensor, m: torch.Tensor, v: torch.Tensor,
     _check("bitlogic_adamw_update", load().bitlogic_adamw_update(
         _ptr(theta), _ptr(m), _ptr(v), _ptr(grad), theta.numel(), int(step), float(lr),
         float(betas[0]), float(betas[1]), float(eps), float(weight_decay), _stream(stream)))
+
+
+def bitlogic_degree_order(csr_off: np.ndarray) -> np.ndarray:
+    """Host call: the nodes by decreasing CSR degree (ties by index)."""
+    off = np.ascontiguousarray(csr_off, dtype=np.int32)
+    n = off.shape[0] - 1
+    order = np.zeros(max(n, 0), np.int32)
+    _check("bitlogic_degree_order", load().bitlogic_degree_order(
+        off.ctypes.data_as(_P), n, order.ctypes.data_as(_P)))
+    return order
 
 
 def bitlogic_csr_positions(csr_edge: np.ndarray) -> np.ndarray:

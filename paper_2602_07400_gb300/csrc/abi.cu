@@ -85,6 +85,24 @@ extern "C" int bitlogic_csr_positions(const int32_t* edge_host, int32_t n_edges,
     return BITLOGIC_OK;
 }
 
+extern "C" int bitlogic_degree_order(const int32_t* off_host, int32_t n, int32_t* order_host) {
+    if (!off_host || !order_host) return BITLOGIC_ERR_NULL;
+    if (n <= 0) return BITLOGIC_ERR_SHAPE;
+    if (off_host[0] != 0) return BITLOGIC_ERR_INDEX;
+    int32_t dmax = 0;
+    for (int32_t i = 0; i < n; ++i) {
+        const int32_t d = off_host[i + 1] - off_host[i];
+        if (d < 0) return BITLOGIC_ERR_INDEX;
+        dmax = d > dmax ? d : dmax;
+    }
+    // counting sort by decreasing degree, increasing index within a degree
+    std::vector<int32_t> start((size_t)dmax + 2, 0);
+    for (int32_t i = 0; i < n; ++i) ++start[(size_t)(dmax - (off_host[i + 1] - off_host[i])) + 1];
+    for (int32_t d = 0; d <= dmax; ++d) start[(size_t)d + 1] += start[(size_t)d];
+    for (int32_t i = 0; i < n; ++i) order_host[start[(size_t)(dmax - (off_host[i + 1] - off_host[i]))]++] = i;
+    return BITLOGIC_OK;
+}
+
 extern "C" int bitlogic_device_error(cudaStream_t stream) {
     int worst = BITLOGIC_OK;
     const int r[8] = {bitlogic_internal_index_error_lut_soft(stream),

@@ -505,16 +505,24 @@ constexpr int kBytesUnroll = BITLOGIC_BYTES_UNROLL;   // term rows whose loads a
 // finds stage r's 4 wires as bytes of (word >> r) & 0x01010101.
 static_assert((kBitBlock / kTStageSamples) % kBytesChunk == 0, "a chunk's stages lie in one bit-row block");
 
+// order (or NULL): the warp at position p takes node order[p] (a permutation
+// of the nodes, e.g. by decreasing term count so that the longest nodes start
+// first); only the schedule changes.
 template <int k, bool TERMS, bool BITS>
 __global__ void __launch_bounds__(kBytesWarps * 32)
 lut_theta_bytes_kernel(const void* __restrict__ Xv, int w_in, long long B, long long words,
                        const int* __restrict__ conn, const float* __restrict__ theta, int w, GradIn gi,
-                       float* __restrict__ dtheta, float* __restrict__ dY_out) {
+                       float* __restrict__ dtheta, float* __restrict__ dY_out, const int* __restrict__ order) {
     constexpr int K = 1 << k, CH = kTStageSamples;
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int j = blockIdx.x * kBytesWarps + warp;
-    if (j >= w) return;   // warp-uniform; the block has no barrier
+    const int p = blockIdx.x * kBytesWarps + warp;
+    if (p >= w) return;   // warp-uniform; the block has no barrier
+    const int j = order ? __ldg(order + p) : p;
+    if ((unsigned)j >= (unsigned)w) {   // not a node: flagged, nothing written
+        if (lane == 0) flag_index_error();
+        return;
+    }
     float* col = reinterpret_cast<float*>(smem_raw) + warp * K * 32 + lane;
 #pragma unroll
     for (int a = 0; a < K; ++a) col[a * 32] = 0.f;
@@ -642,14 +650,14 @@ lut_theta_bytes_kernel(const void* __restrict__ Xv, int w_in, long long B, long 
 
 template <int k, bool BITS>
 int launch_bytes(bool terms, const void* X, int w_in, long long B, const int* conn, const float* theta, int w,
-                 const GradIn& gi, float* dtheta, float* dY_out, cudaStream_t st) {
+                 const GradIn& gi, float* dtheta, float* dY_out, const int* order, cudaStream_t st) {
     constexpr int smem = kBytesWarps * (1 << k) * 32 * (int)sizeof(float);
     const unsigned blocks = (unsigned)((w + kBytesWarps - 1) / kBytesWarps);
     const long long words = (B + kBitBlock - 1) / kBitBlock * 32;
     auto kern = terms ? lut_theta_bytes_kernel<k, true, BITS> : lut_theta_bytes_kernel<k, false, BITS>;
     if (smem > 40 * 1024 && cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
         return BITLOGIC_ERR_CUDA;
-    kern<<<blocks, kBytesWarps * 32, smem, st>>>(X, w_in, B, words, conn, theta, w, gi, dtheta, dY_out);
+    kern<<<blocks, kBytesWarps * 32, smem, st>>>(X, w_in, B, words, conn, theta, w, gi, dtheta, dY_out, order);
     return launch_status();
 }
 
@@ -767,7 +775,7 @@ namespace {
 int backward_bytes(const void* X, int32_t w_in, int64_t B, const int32_t* conn, const float* theta, int32_t w,
                    int32_t k, int32_t node, const float* dY, int32_t dy_group, const float* up_terms,
                    const int32_t* up_off, const int32_t* up_edge, int32_t up_edges, float* dtheta, float* dY_out,
-                   bool bits, cudaStream_t stream) {
+                   bool bits, const int32_t* order, cudaStream_t stream) {
     int st = check_common(X, w_in, B, conn, theta, w, k, node, dtheta);
     if (st) return st;
     const bool terms = up_terms != nullptr;
@@ -793,8 +801,8 @@ int backward_bytes(const void* X, int32_t w_in, int64_t B, const int32_t* conn, 
     gi.off = up_off;
     gi.edge = up_edge;
 #define BITLOGIC_BYTES_K(K)                                                                           \
-    return bits ? launch_bytes<K, true>(terms, X, w_in, B, conn, theta, w, gi, dtheta, dY_out, stream) \
-                : launch_bytes<K, false>(terms, X, w_in, B, conn, theta, w, gi, dtheta, dY_out, stream)
+    return bits ? launch_bytes<K, true>(terms, X, w_in, B, conn, theta, w, gi, dtheta, dY_out, order, stream) \
+                : launch_bytes<K, false>(terms, X, w_in, B, conn, theta, w, gi, dtheta, dY_out, order, stream)
     switch (k) {
         case 1: BITLOGIC_BYTES_K(1);
         case 2: BITLOGIC_BYTES_K(2);
@@ -813,14 +821,15 @@ extern "C" int bitlogic_lut_backward_u8(const uint8_t* X, int32_t w_in, int64_t 
                                         const int32_t* up_off, const int32_t* up_edge, int32_t up_edges,
                                         float* dtheta, float* dY_out, cudaStream_t stream) {
     return backward_bytes(X, w_in, B, conn, theta, w, k, node, dY, dy_group, up_terms, up_off, up_edge, up_edges,
-                          dtheta, dY_out, false, stream);
+                          dtheta, dY_out, false, nullptr, stream);
 }
 
 extern "C" int bitlogic_lut_backward_bitrows(const uint32_t* X, int32_t w_in, int64_t B, const int32_t* conn,
                                              const float* theta, int32_t w, int32_t k, int32_t node,
                                              const float* dY, int32_t dy_group, const float* up_terms,
                                              const int32_t* up_off, const int32_t* up_edge, int32_t up_edges,
-                                             float* dtheta, float* dY_out, cudaStream_t stream) {
+                                             const int32_t* order, float* dtheta, float* dY_out,
+                                             cudaStream_t stream) {
     return backward_bytes(X, w_in, B, conn, theta, w, k, node, dY, dy_group, up_terms, up_off, up_edge, up_edges,
-                          dtheta, dY_out, true, stream);
+                          dtheta, dY_out, true, order, stream);
 }

@@ -25,7 +25,7 @@ from . import (NODE_FORMS, bitlogic_adamw_update, bitlogic_binarize_tables, bitl
                bitlogic_pack_bits, bitlogic_route_backward, bitlogic_route_backward_u8, bitlogic_route_forward,
                bitlogic_route_forward_u8, bitlogic_route_snap, bitlogic_encode_thermometer_u8,
                bitlogic_lut_forward_u8, bitlogic_encode_thermometer_bitrows, bitlogic_lut_forward_bitrows,
-               bitlogic_lut_backward_bitrows, bitrow_words)
+               bitlogic_lut_backward_bitrows, bitrow_words, bitlogic_degree_order)
 
 
 def _nomark(name: str) -> None:
@@ -148,6 +148,9 @@ class Network:
         # in CSR order, so each input's terms are one contiguous block
         self.pos1 = torch.from_numpy(bitlogic_csr_positions(edge1)).to(dev)
         self.pos2 = torch.from_numpy(bitlogic_csr_positions(edge2)).to(dev)
+        # layer-1 nodes by decreasing consumer count: the order in which the
+        # layer-1 backward on wire bit rows takes them (the longest first)
+        self.order1 = torch.from_numpy(bitlogic_degree_order(off2)).to(dev)
 
 
 # On fp32 wires, per-edge input-gradient terms larger than this are summed by
@@ -305,7 +308,8 @@ class TrainStep:
         edge2 = None if co else n.edge2
         if self.fuse_dy1 and self.bits1:
             bitlogic_lut_backward_bitrows(self.bits, self.B, n.conn1, n.theta1, self.dth1, nd, up_terms=self.edges2,
-                                          up_off=n.off2, up_edge=edge2, dY_out=self.dy1, stream=stream)
+                                          up_off=n.off2, up_edge=edge2, dY_out=self.dy1, order=n.order1,
+                                          stream=stream)
         elif self.fuse_dy1 and self.bytes1:
             bitlogic_lut_backward_u8(self.bits, n.conn1, n.theta1, self.dth1, nd, up_terms=self.edges2,
                                      up_off=n.off2, up_edge=edge2, dY_out=self.dy1, stream=stream)

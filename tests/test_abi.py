@@ -209,11 +209,11 @@ def test_host_validation_returns_before_any_launch():
     assert fwd_b(None, 8, 64, fake, fake, 4, 2, 0, fake, None) == -1
     assert fwd_b(P(18), 8, 64, fake, fake, 4, 2, 0, fake, None) == -4
     assert fwd_b(None, 8, 0, fake, fake, 4, 2, 0, None, None) == 0
-    assert bwd_b(fake, 8, 64, fake, fake, 4, 2, 0, None, 1, None, None, None, 0, fake, None, None) == -1
-    assert bwd_b(fake, 8, 64, fake, fake, 4, 2, 0, fake, 1, fake, fake, None, 4, fake, None, None) == -1
-    assert bwd_b(fake, 8, 64, fake, fake, 4, 2, 0, fake, 3, None, None, None, 0, fake, None, None) == -2
-    assert bwd_b(fake, 8, 66, fake, fake, 4, 2, 0, fake, 1, None, None, None, 0, fake, None, None) == -4
-    assert bwd_b(fake, 8, 64, fake, fake, 4, 2, 2, fake, 1, None, None, None, 0, fake, None, None) == -12
+    assert bwd_b(fake, 8, 64, fake, fake, 4, 2, 0, None, 1, None, None, None, 0, None, fake, None, None) == -1
+    assert bwd_b(fake, 8, 64, fake, fake, 4, 2, 0, fake, 1, fake, fake, None, 4, None, fake, None, None) == -1
+    assert bwd_b(fake, 8, 64, fake, fake, 4, 2, 0, fake, 3, None, None, None, 0, None, fake, None, None) == -2
+    assert bwd_b(fake, 8, 66, fake, fake, 4, 2, 0, fake, 1, None, None, None, 0, None, fake, None, None) == -4
+    assert bwd_b(fake, 8, 64, fake, fake, 4, 2, 2, fake, 1, None, None, None, 0, None, fake, None, None) == -12
 
 
 @pytest.mark.parametrize("n,b,seed", [(1, 1, 0), (5, 4, 1), (1000, 8, 2), (65537, 32, 3), (300, 15, 4)])
@@ -226,6 +226,27 @@ def test_quantile_thresholds_from_a_histogram_match_the_oracle(n, b, seed):
         x[rng.random(n) < 0.8] = 0               # a point mass, as in digit images
     hist = np.bincount(x, minlength=256).astype(np.uint64)
     np.testing.assert_array_equal(bl.bitlogic_quantile_thresholds(hist, b), oracle.quantile_thresholds(x, b))
+
+
+def test_degree_order_is_a_stable_sort_by_decreasing_degree():
+    # host helper: nodes by decreasing CSR degree, ties in increasing index
+    rng = np.random.default_rng(3)
+    for w, w_in, k in ((50, 40, 3), (300, 1000, 6), (7, 7, 1)):
+        conn = rng.integers(0, w_in, size=(w, k)).astype(np.int32)
+        off, _ = bl.bitlogic_build_csr(conn, w_in)
+        deg = np.diff(off)
+        order = bl.bitlogic_degree_order(off)
+        np.testing.assert_array_equal(order, np.argsort(-deg, kind="stable"))
+        assert sorted(order.tolist()) == list(range(w_in))
+    lib = bl.load()
+    P = ctypes.c_void_p
+    off = np.array([0, 2, 1], np.int32)               # decreasing: not a CSR map
+    out = np.zeros(2, np.int32)
+    assert lib.bitlogic_degree_order(off.ctypes.data_as(P), 2, out.ctypes.data_as(P)) == -7
+    off = np.array([1, 2, 3], np.int32)               # does not start at 0
+    assert lib.bitlogic_degree_order(off.ctypes.data_as(P), 2, out.ctypes.data_as(P)) == -7
+    assert lib.bitlogic_degree_order(off.ctypes.data_as(P), 0, out.ctypes.data_as(P)) == -2
+    assert lib.bitlogic_degree_order(None, 2, out.ctypes.data_as(P)) == -1
 
 
 def test_quantile_thresholds_rejects_bad_input():

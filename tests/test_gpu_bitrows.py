@@ -164,6 +164,40 @@ def test_lut_backward_bitrows_rows_and_terms(k, w_in, w, B, node):
     assert bl.bitlogic_device_error() == 0
 
 
+@pytest.mark.parametrize("k", [2, 6])
+def test_lut_backward_bitrows_node_order(k):
+    # the order in which the warps take the nodes changes no result; an
+    # entry outside the nodes is flagged and skipped
+    w_in, w, up_w, B = 80, 70, 90, 1028
+    Xb = synth.binary_activations(w_in, B, seed=k + 70)
+    XW = dev(pack_rows(Xb))
+    conn = dev(synth.connectivity(w, k, w_in, seed=k + 71))
+    theta = dev(synth.table_logits(w, 1 << k, seed=k + 72))
+    up_conn = synth.connectivity(up_w, 4, w, seed=k + 73)
+    off, edge = bl.bitlogic_build_csr(up_conn, w)
+    terms = dev(synth.uniform_gradients(up_w * 4, B, seed=k + 74, scale=1e-3))
+    kw = dict(up_terms=terms, up_off=dev(off), up_edge=dev(edge))
+    ref = torch.empty(w, 1 << k, device="cuda")
+    out_ref = torch.empty(w, B, device="cuda")
+    bl.bitlogic_lut_backward_bitrows(XW, B, conn, theta, ref, dY_out=out_ref, **kw)
+    for order in (bl.bitlogic_degree_order(off), np.random.default_rng(k).permutation(w).astype(np.int32)):
+        got = torch.full((w, 1 << k), np.nan, device="cuda")
+        out = torch.full((w, B), np.nan, device="cuda")
+        bl.bitlogic_lut_backward_bitrows(XW, B, conn, theta, got, dY_out=out, order=dev(order), **kw)
+        check_exact(got.cpu().numpy(), ref.cpu().numpy(), "dtheta (ordered)")
+        check_exact(out.cpu().numpy(), out_ref.cpu().numpy(), "dY_out (ordered)")
+    assert bl.bitlogic_device_error() == 0
+    bad = np.arange(w, dtype=np.int32)
+    bad[5] = w                                   # one entry past the last node
+    got = torch.full((w, 1 << k), np.nan, device="cuda")
+    bl.bitlogic_lut_backward_bitrows(XW, B, conn, theta, got, order=dev(bad), **kw)
+    assert bl.bitlogic_device_error() == -8
+    g = got.cpu().numpy()
+    assert np.isnan(g[5]).all()                  # node 5 was never taken
+    keep = np.arange(w) != 5
+    check_exact(g[keep], ref.cpu().numpy()[keep], "dtheta (other nodes)")
+
+
 @pytest.mark.parametrize("k,group", [(6, 4), (2, 13)])
 def test_lut_backward_bitrows_grouped_rows(k, group):
     w_in, w, B = 90, 52, 2052
