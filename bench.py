@@ -374,16 +374,16 @@ TRAFFIC = {
         "sha256": "88cd7e78b309d49ee5835ba21aeb26fbdf1a8e144188cac4f9338e562f6c3f57",
         "note": "ncu capture of this workload (one-pass DRAM metrics)"},
     ("cifar10", "backward1"): {
-        "bytes": 1593852672 + 3620608, "source": "lut_through.cu",
-        "sha256": "7c8274d9e0ac03637e86af0d7b0c6716a0d8e84b412c07fc0a513d0cc3e3485b",
+        "bytes": 1594115840 + 5145600, "source": "lut_through.cu",
+        "sha256": "490278457365ad944f8a52c158573b408a956203bc3f2c848618cd16f764cefd",
         "note": "ncu capture of this workload (one-pass DRAM metrics)"},
     ("cifar100", "forward1"): {
         "bytes": 50327040 + 984133120, "source": "lut_bytes.cu",
         "sha256": "88cd7e78b309d49ee5835ba21aeb26fbdf1a8e144188cac4f9338e562f6c3f57",
         "note": "ncu capture of this workload (one-pass DRAM metrics)"},
     ("cifar100", "backward1"): {
-        "bytes": 6339823104 + 5000960, "source": "lut_through.cu",
-        "sha256": "7c8274d9e0ac03637e86af0d7b0c6716a0d8e84b412c07fc0a513d0cc3e3485b",
+        "bytes": 6340807168 + 7737344, "source": "lut_through.cu",
+        "sha256": "490278457365ad944f8a52c158573b408a956203bc3f2c848618cd16f764cefd",
         "note": "ncu capture of this workload (one-pass DRAM metrics)"},
     ("cifar10", "encode"): {
         "bytes": 3160576 + 0, "source": "encode.cu",
