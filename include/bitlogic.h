@@ -355,11 +355,15 @@ int bitlogic_lut_backward_u8(const uint8_t* X, int32_t w_in, int64_t B, const in
  * (the layout of bitlogic_encode_thermometer_bitrows), 16-byte aligned.
  *   order  device int32 [w] or NULL: the order in which the kernel's warps
  *          take the nodes (a permutation of 0 .. w-1; bitlogic_degree_order
- *          over up_off puts the nodes with the most term rows first, which
- *          shortens the launch's tail); NULL takes them in index order.  An
- *          entry outside [0, w) raises the device flag and is skipped; a
- *          repeated entry leaves another node's dtheta unwritten.  The
- *          order does not change any result.
+ *          over the CSR offsets puts the nodes with the most term rows
+ *          first, which shortens the launch's tail); NULL takes them in
+ *          index order.  With an order, up_off and up_edge are the CSR map
+ *          in the order's sequence: the rows of node order[p] are the CSR
+ *          positions up_off[p] .. up_off[p+1] - 1 (bitlogic_build_csr over
+ *          the next layer's connectivity with node i renamed to its
+ *          position in the order).  An entry outside [0, w) raises the
+ *          device flag and is skipped; a repeated entry leaves another
+ *          node's dtheta unwritten.  The order changes no result.
  * Every other argument, the result and the errors as
  * bitlogic_lut_backward_u8: the same wires give the same dtheta and dY_out
  * bit for bit (the samples are visited in the same order). */

@@ -507,7 +507,9 @@ static_assert((kBitBlock / kTStageSamples) % kBytesChunk == 0, "a chunk's stages
 
 // order (or NULL): the warp at position p takes node order[p] (a permutation
 // of the nodes, e.g. by decreasing term count so that the longest nodes start
-// first); only the schedule changes.
+// first); only the schedule changes.  With an order the terms' CSR map is
+// the one in the order's sequence (position p's rows at off[p] ..
+// off[p+1] - 1), so a node's range does not wait for its index.
 template <int k, bool TERMS, bool BITS>
 __global__ void __launch_bounds__(kBytesWarps * 32)
 lut_theta_bytes_kernel(const void* __restrict__ Xv, int w_in, long long B, long long words,
@@ -544,8 +546,9 @@ lut_theta_bytes_kernel(const void* __restrict__ Xv, int w_in, long long B, long 
     int e0 = 0, deg = 0, my_id = -1;
     if constexpr (TERMS) {
         int e1;
-        e0 = __ldg(gi.off + j);
-        e1 = __ldg(gi.off + j + 1);
+        const int r = order ? p : j;   // the node's entry in the CSR map
+        e0 = __ldg(gi.off + r);
+        e1 = __ldg(gi.off + r + 1);
         if (e0 < 0 || e1 < e0 || e1 > gi.n_terms) {
             bad = true;
             e0 = e1 = 0;

@@ -149,8 +149,17 @@ class Network:
         self.pos1 = torch.from_numpy(bitlogic_csr_positions(edge1)).to(dev)
         self.pos2 = torch.from_numpy(bitlogic_csr_positions(edge2)).to(dev)
         # layer-1 nodes by decreasing consumer count: the order in which the
-        # layer-1 backward on wire bit rows takes them (the longest first)
-        self.order1 = torch.from_numpy(bitlogic_degree_order(off2)).to(dev)
+        # layer-1 backward on wire bit rows takes them (the longest first),
+        # with layer 2's CSR map in that order's sequence (node order1[p]'s
+        # edges at positions off2o[p] .. off2o[p+1] - 1; layer 2 stores its
+        # terms at those positions for that backward)
+        order1 = bitlogic_degree_order(off2)
+        rank = np.empty_like(order1)
+        rank[order1] = np.arange(self.w1, dtype=np.int32)
+        off2o, edge2o = bitlogic_build_csr(rank[np.ascontiguousarray(conn2, np.int32)], self.w1)
+        self.order1 = torch.from_numpy(order1).to(dev)
+        self.off2o, self.edge2o = torch.from_numpy(off2o).to(dev), torch.from_numpy(edge2o).to(dev)
+        self.pos2o = torch.from_numpy(bitlogic_csr_positions(edge2o)).to(dev)
 
 
 # On fp32 wires, per-edge input-gradient terms larger than this are summed by
@@ -300,16 +309,19 @@ class TrainStep:
                                           dY_out=self.dy1, stream=stream)
             mark("backward1")
             return
+        # the bit-row layer-1 backward reads the terms through the CSR map in
+        # its node order; every other consumer through the map in node order
+        ordered = self.fuse_dy1 and self.bits1
         bitlogic_lut_backward_node(self.y1, n.conn2, n.theta2, self.dth2, nd, dY=self.dyg,
                                    dy_group=g, edge_terms=self.edges2,
-                                   edge_pos=n.pos2 if co else None, stream=stream)
+                                   edge_pos=(n.pos2o if ordered else n.pos2) if co else None, stream=stream)
         mark("backward2")
         pos1 = n.pos1 if (co and self.edges1 is not None) else None
         edge2 = None if co else n.edge2
-        if self.fuse_dy1 and self.bits1:
+        if ordered:
             bitlogic_lut_backward_bitrows(self.bits, self.B, n.conn1, n.theta1, self.dth1, nd, up_terms=self.edges2,
-                                          up_off=n.off2, up_edge=edge2, dY_out=self.dy1, order=n.order1,
-                                          stream=stream)
+                                          up_off=n.off2o, up_edge=None if co else n.edge2o, dY_out=self.dy1,
+                                          order=n.order1, stream=stream)
         elif self.fuse_dy1 and self.bytes1:
             bitlogic_lut_backward_u8(self.bits, n.conn1, n.theta1, self.dth1, nd, up_terms=self.edges2,
                                      up_off=n.off2, up_edge=edge2, dY_out=self.dy1, stream=stream)

@@ -181,11 +181,25 @@ def test_lut_backward_bitrows_node_order(k):
     out_ref = torch.empty(w, B, device="cuda")
     bl.bitlogic_lut_backward_bitrows(XW, B, conn, theta, ref, dY_out=out_ref, **kw)
     for order in (bl.bitlogic_degree_order(off), np.random.default_rng(k).permutation(w).astype(np.int32)):
+        # the next layer's CSR map in the order's sequence: node order[p]'s
+        # edges (the same ones, in the same increasing order) at position p
+        rank = np.empty_like(order)
+        rank[order] = np.arange(w, dtype=np.int32)
+        off_o, edge_o = bl.bitlogic_build_csr(rank[up_conn], w)
+        np.testing.assert_array_equal(np.diff(off_o), np.diff(off)[order])
         got = torch.full((w, 1 << k), np.nan, device="cuda")
         out = torch.full((w, B), np.nan, device="cuda")
-        bl.bitlogic_lut_backward_bitrows(XW, B, conn, theta, got, dY_out=out, order=dev(order), **kw)
+        bl.bitlogic_lut_backward_bitrows(XW, B, conn, theta, got, dY_out=out, order=dev(order), up_terms=terms,
+                                         up_off=dev(off_o), up_edge=dev(edge_o))
         check_exact(got.cpu().numpy(), ref.cpu().numpy(), "dtheta (ordered)")
         check_exact(out.cpu().numpy(), out_ref.cpu().numpy(), "dY_out (ordered)")
+        # dY rows: the order changes the schedule only
+        dY = dev(synth.uniform_gradients(w, B, seed=k + 75, scale=1e-3))
+        ref_r = torch.empty(w, 1 << k, device="cuda")
+        bl.bitlogic_lut_backward_bitrows(XW, B, conn, theta, ref_r, dY=dY)
+        got_r = torch.full((w, 1 << k), np.nan, device="cuda")
+        bl.bitlogic_lut_backward_bitrows(XW, B, conn, theta, got_r, dY=dY, order=dev(order))
+        check_exact(got_r.cpu().numpy(), ref_r.cpu().numpy(), "dtheta (ordered, dY rows)")
     assert bl.bitlogic_device_error() == 0
     bad = np.arange(w, dtype=np.int32)
     bad[5] = w                                   # one entry past the last node
