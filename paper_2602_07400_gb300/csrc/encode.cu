@@ -2,13 +2,16 @@
 // emits b+1 levels on b wires; wire j*b + i of feature j is x_j > T_i, with
 // the strict comparison of App. B's "(pixel > 0)").
 //
-// Two forms:
-//   * soft:   fp32 {0,1} rows [d*b][B] feeding the first soft LUT layer;
-//   * packed: 32 samples per uint32 along the batch (App. C.1 "Bit-packed
+// Three forms:
+//   * soft:     fp32 {0,1} rows [d*b][B] (or bytes 0/1) feeding the first
+//     soft LUT layer;
+//   * bit rows: the soft layer-1 input at one bit per sample, in the order
+//     of the layer-1 kernels' lanes (below);
+//   * packed:   32 samples per uint32 along the batch (App. C.1 "Bit-packed
 //     inference" packs samples along the batch into machine words), fused
 //     with the comparison so the fp32 form is never materialised.
 //
-// Both stage a tile of raw samples (sample-major uint8) in shared memory and
+// All stage a tile of raw samples (sample-major uint8) in shared memory and
 // write feature-major rows, so global reads and writes are coalesced.
 #include "common.cuh"
 

@@ -1,5 +1,6 @@
-// Soft forward of a LUT layer whose input is byte rows (binary wires, each
-// byte 0 or 1: the thermometer encoder's output, §3 "Encoders and heads").
+// Soft forward of a LUT layer whose input is binary wires (the thermometer
+// encoder's output, §3 "Encoders and heads"), as byte rows (each byte 0 or
+// 1) or as wire bit rows (one bit per sample, the training step's form).
 //
 // The relaxed table of §2, y = sum_a t_a prod_i x_i^{a_i} (1 - x_i)^{1 - a_i},
 // has one-hot corner weights on binary inputs: the product is 1 for the
@@ -17,7 +18,9 @@
 // table (2^k <= 64 entries) sits in two registers per lane and each lookup is
 // a shuffle from the lane holding the entry.  Rows are gathered with several
 // 128-sample groups in flight per lane.  A scalar form (one sample per lane)
-// serves ragged batches and unaligned rows.
+// serves ragged batches and unaligned rows.  The bit-row form takes the
+// same lanes and samples with one 32-bit word per input row and 1024-sample
+// block in place of the byte loads.
 #include "common.cuh"
 
 namespace bitlogic {
