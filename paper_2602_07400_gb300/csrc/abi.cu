@@ -1,5 +1,6 @@
 // Host-side parts of the C ABI that launch no kernels: status strings, the
 // inverse-connectivity (CSR) builder, and the device-side index flag reader.
+#include <algorithm>
 #include <atomic>
 #include <vector>
 
@@ -89,17 +90,13 @@ extern "C" int bitlogic_degree_order(const int32_t* off_host, int32_t n, int32_t
     if (!off_host || !order_host) return BITLOGIC_ERR_NULL;
     if (n <= 0) return BITLOGIC_ERR_SHAPE;
     if (off_host[0] != 0) return BITLOGIC_ERR_INDEX;
-    int32_t dmax = 0;
-    for (int32_t i = 0; i < n; ++i) {
-        const int32_t d = off_host[i + 1] - off_host[i];
-        if (d < 0) return BITLOGIC_ERR_INDEX;
-        dmax = d > dmax ? d : dmax;
-    }
-    // counting sort by decreasing degree, increasing index within a degree
-    std::vector<int32_t> start((size_t)dmax + 2, 0);
-    for (int32_t i = 0; i < n; ++i) ++start[(size_t)(dmax - (off_host[i + 1] - off_host[i])) + 1];
-    for (int32_t d = 0; d <= dmax; ++d) start[(size_t)d + 1] += start[(size_t)d];
-    for (int32_t i = 0; i < n; ++i) order_host[start[(size_t)(dmax - (off_host[i + 1] - off_host[i]))]++] = i;
+    for (int32_t i = 0; i < n; ++i)
+        if (off_host[i + 1] < off_host[i]) return BITLOGIC_ERR_INDEX;
+    // stable sort by decreasing degree: ties keep increasing index
+    for (int32_t i = 0; i < n; ++i) order_host[i] = i;
+    std::stable_sort(order_host, order_host + n, [off_host](int32_t a, int32_t b) {
+        return off_host[a + 1] - off_host[a] > off_host[b + 1] - off_host[b];
+    });
     return BITLOGIC_OK;
 }
 
